@@ -1,0 +1,186 @@
+/*
+ * catq.h — C ABI of the CAT-Q soft-ternary calibration hot path on GB300 (sm_103a).
+ *
+ * CAT-Q ternarizes a linear layer W [N out, K in] as W ~ alpha * T, T in {-1, 0, +1},
+ * per non-overlapping group of g consecutive elements of row-major W (App. B.2).
+ * Each group carries frozen statistics (mu0, alpha0, Delta0) and three learnable
+ * factors (d_mu, d_alpha, d_delta) (Eq. 3, §2.2):
+ *
+ *   mu = mu0 + d_mu * alpha0,  alpha = d_alpha * alpha0,  Delta = d_delta * Delta0,
+ *   What = (W - mu) / alpha                                  (Eq. 3)
+ *   T    = W                       (teacher, t = 0)          (Eq. 6)
+ *        = f(What; s, Delta)       (soft stage, 0 < t <= gamma)
+ *        = Q(What; Delta)          (hard stage, gamma < t <= 1)
+ *   f(x; s, D) = [tanh(s(x-D)) + tanh(s(x+D))] / (2 tanh s)  (Eq. 5)
+ *   Q(x; D)    = +1 if x > D, 0 if |x| <= D, -1 if x < -D   (Eq. 2)
+ *   Wq   = alpha * T  (no mu in the reconstruction, §2.2 and App. B.2); Wq = W for the teacher.
+ *
+ * A calibration step for one linear computes Y = X Wq^T, the reconstruction loss
+ * against the teacher output (Eq. 7, one linear), and the gradients into X and into the
+ * three factors.  The GEMMs never write Wq to HBM: the modulation, the transition
+ * function and alpha are applied while the weight tile sits in shared memory.
+ *
+ * Conventions for every call:
+ *   - All tensors are caller-owned.  No call allocates device or host memory.
+ *   - Pointers named "device" must be CUDA device pointers of the current device.
+ *   - Every call is asynchronous on `stream` (NULL = legacy default stream).
+ *   - Argument errors return a non-zero catq_status before anything is launched.
+ *   - Conditions detected on the device (a bounded wait that expired) are latched in a
+ *     per-device status word; read and clear it with catq_device_status().
+ *   - Shapes: g divides K.  bf16 weights need g % 64 == 0 and N % 8 == 0; fp32 weights
+ *     need g % 64 == 0 or g in {4, 8, 16, 32}.  The weight and activation dtypes must
+ *     match: both CATQ_F32 (CUDA-core path) or both CATQ_BF16 (tensor-core path,
+ *     fp32 accumulation).  bf16 buffers must be 16-byte aligned.
+ *   - A group whose alpha is exactly 0 (constant weights, or d_alpha == 0) has Wq = 0,
+ *     hard code 0 and zero factor gradients.
+ */
+#ifndef CATQ_H
+#define CATQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; NULL selects the legacy default stream. */
+typedef struct CUstream_st* catq_stream;
+
+typedef enum {
+  CATQ_OK = 0,
+  CATQ_ERR_INVALID_ARG = 1, /* null pointer, bad enum, non-finite or non-positive s */
+  CATQ_ERR_SHAPE = 2,       /* g does not divide K, unsupported g, M < 0, N/K < 1 */
+  CATQ_ERR_DTYPE = 3,       /* unknown dtype or mixed weight/activation dtypes */
+  CATQ_ERR_ALIGN = 4,       /* bf16 buffer not 16-byte aligned */
+  CATQ_ERR_CUDA = 5,        /* a CUDA runtime call failed (launch, attribute, tensor map) */
+  CATQ_ERR_TIMEOUT = 6,     /* a bounded device-side wait expired (latched) */
+  CATQ_ERR_NONFINITE = 7,   /* reserved: non-finite data detected (latched) */
+  CATQ_ERR_UNSUPPORTED = 8, /* valid request this build does not implement (e.g. no sm_100-class GPU) */
+  CATQ_ERR_WORKSPACE = 9    /* workspace missing or smaller than the *_workspace_bytes() result */
+} catq_status;
+
+typedef enum { CATQ_F32 = 0, CATQ_BF16 = 1 } catq_dtype;
+
+/* Eq. 6: which branch of the softened ternarization produces T. */
+typedef enum {
+  CATQ_PHASE_TEACHER = 0, /* t = 0: T = W, Wq = W (the full-precision teacher) */
+  CATQ_PHASE_SOFT = 1,    /* 0 < t <= gamma: T = f(What; s, Delta) */
+  CATQ_PHASE_HARD = 2     /* gamma < t <= 1: T = Q(What; Delta) */
+} catq_phase;
+
+/* Initial threshold Delta0 in What units (§2.2). */
+typedef enum {
+  CATQ_THR_HALF = 0,  /* Delta0 = 0.5, the paper's default (§2.2, App. B.1) */
+  CATQ_THR_TWN07 = 1  /* Delta0 = 0.7 * mean|W_group| / alpha0: TWN's 0.7 mean|W| rule (§2.2)
+                         expressed in What units, so alpha*Delta equals it at identity factors */
+} catq_thr_init;
+
+typedef enum { CATQ_REDUCE_MEAN = 0, CATQ_REDUCE_SUM = 1 } catq_reduction;
+
+/* Eq. 6 schedule point.  SOFT: s = (t / gamma) * s0 > 0.  HARD: s is the sharpness of the
+ * surrogate f used for the backward pass (§2.3, last stage-1 sharpness = s0).  TEACHER:
+ * s is ignored. */
+typedef struct {
+  int32_t phase; /* catq_phase */
+  float s;
+} catq_schedule;
+
+/* One linear layer.  All pointers are device pointers owned by the caller.
+ * G = N*K/g groups; group j holds elements [j*g, (j+1)*g) of row-major W. */
+typedef struct {
+  int64_t N;       /* out_features (rows of W) */
+  int64_t K;       /* in_features (columns of W) */
+  int32_t g;       /* group size; g == K is channel-wise */
+  int32_t w_dtype; /* catq_dtype of W */
+  const void* W;   /* [N, K] row-major, read-only */
+  float* mu0;      /* [G] written by catq_group_stats, read by every other call */
+  float* alpha0;   /* [G] */
+  float* delta0;   /* [G] */
+  const float* d_mu;    /* [G] learnable factor d_mu    (Eq. 3), -1 < d_mu < 1 */
+  const float* d_alpha; /* [G] learnable factor d_alpha (Eq. 3), > 0 */
+  const float* d_delta; /* [G] learnable factor d_delta (§2.2), > 0 */
+} catq_layer;
+
+/* ABI version of this header; bumped on any incompatible change. */
+#define CATQ_ABI_VERSION 1
+int32_t catq_abi_version(void);
+
+/* Human-readable name of a status code (static storage, never NULL). */
+const char* catq_status_string(int32_t status);
+
+/* Group statistics (Eq. 3; TWN 0.7 rule of §2.2 for CATQ_THR_TWN07):
+ *   mu0[j] = mean of group j;  alpha0[j] = mean |W - mu0[j]| over group j;
+ *   delta0[j] = 0.5, or 0.7 * mean|W| / alpha0[j] (0.5 if alpha0[j] == 0).
+ * Sums run in fp64 on the device; results are stored as fp32.  Reads W once. */
+catq_status catq_group_stats(const catq_layer* layer, int32_t thr_init, catq_stream stream);
+
+/* Materialises the Eq. 6 weight for inspection (not used inside the GEMMs, which fuse it).
+ *   Wq_out   [N, K], dtype w_dtype, nullable: alpha * T for the schedule's phase (W for
+ *            TEACHER), computed exactly as the fused GEMM operand producer computes it.
+ *   T_out    [N, K] int8, nullable: hard codes Q(What; Delta) in {-1, 0, 1} (Eq. 4).
+ *   alpha_out [G] fp32, nullable: alpha = d_alpha * alpha0.                              */
+catq_status catq_modulate_ternarize(const catq_layer* layer, catq_schedule sched, void* Wq_out,
+                                    int8_t* T_out, float* alpha_out, catq_stream stream);
+
+/* Forward Y = X Wq^T (Eq. 6 weight, Eq. 7 window output for one linear).
+ *   X [M, K] row-major, Y [M, N] row-major, both of dtype x_dtype (== w_dtype); fp32
+ *   accumulation.  M == 0 is a no-op.                                                    */
+catq_status catq_soft_ternary_linear_fwd(const catq_layer* layer, catq_schedule sched,
+                                         const void* X, int64_t M, int32_t x_dtype, void* Y,
+                                         catq_stream stream);
+
+/* Workspace bytes catq_soft_ternary_linear_bwd needs for this layer and M (partial
+ * per-group sums); 0 is never returned for M > 0. */
+size_t catq_bwd_workspace_bytes(const catq_layer* layer, int64_t M);
+
+/* Backward of Y = X Wq^T given dY = dL/dY [M, N] (dtype x_dtype):
+ *   dX [M, K] = dY Wq            (nullable: skipped when NULL)
+ *   with G = dY^T X [N, K] (never written to memory), per group j:
+ *   g_dmu[j]    = -alpha0 * sum_j G * f'(What)
+ *   g_dalpha[j] =  alpha0 * sum_j G * (T - What * f'(What))
+ *   g_ddelta[j] =  Delta0 * alpha * sum_j G * df/dDelta(What)
+ * f' and df/dDelta are the derivatives of Eq. 5 at the schedule's s.  In the HARD phase T
+ * is the forward value Q(What; Delta) and the derivatives are those of f at s (the
+ * surrogate reading of §2.3's stage-2 rule).  In the TEACHER phase Wq = W does not depend
+ * on the factors: the three gradients are written as zeros.  Gradients are overwritten,
+ * not accumulated.  workspace: device, >= catq_bwd_workspace_bytes(layer, M) bytes,
+ * 256-byte aligned, contents scratch.                                                    */
+catq_status catq_soft_ternary_linear_bwd(const catq_layer* layer, catq_schedule sched,
+                                         const void* X, const void* dY, int64_t M,
+                                         int32_t x_dtype, void* dX, float* g_dmu,
+                                         float* g_dalpha, float* g_ddelta, void* workspace,
+                                         size_t ws_bytes, catq_stream stream);
+
+/* Workspace bytes catq_recon_loss needs for `count` elements (block partial sums). */
+size_t catq_recon_loss_workspace_bytes(int64_t count);
+
+/* Reconstruction loss of Eq. 7 for one linear output, and its gradient:
+ *   loss_out[0] = sum (Y - Y_ref)^2 / count   (CATQ_REDUCE_MEAN)  or the plain sum (SUM)
+ *   dY          = 2 (Y - Y_ref) / count       (MEAN)              or 2 (Y - Y_ref) (SUM)
+ * Y, Y_ref, dY: device, `count` elements of `dtype`; dY nullable.  loss_out: device fp32
+ * scalar.  The sum runs in fp64 with a fixed reduction order (deterministic).
+ * workspace: device, >= catq_recon_loss_workspace_bytes(count) bytes, 256-byte aligned. */
+catq_status catq_recon_loss(const void* Y, const void* Y_ref, int64_t count, int32_t dtype,
+                            int32_t reduction, float* loss_out, void* dY, void* workspace,
+                            size_t ws_bytes, catq_stream stream);
+
+/* Final hard ternarization and 2-bit packing (Eq. 2 / Eq. 4 at the end of calibration,
+ * deployment keeps only T and the group scale alpha, App. B.2):
+ *   codes [N*K/4] uint8: element e of row-major W stores Q(What_e; Delta) + 1 in bits
+ *         [2*(e%4), 2*(e%4)+1] of byte e/4 (values 0, 1, 2; 3 never occurs).
+ *   alpha [G] fp32: d_alpha * alpha0.  Requires N*K % 4 == 0.  The encoding is this
+ *   library's; the paper fixes none.                                                     */
+catq_status catq_hard_ternarize_pack(const catq_layer* layer, uint8_t* codes, float* alpha,
+                                     catq_stream stream);
+
+/* Synchronises `stream`, then returns in *out the status latched on the current device
+ * since the last call (CATQ_OK if none) and clears it.  The return value reports whether
+ * the query itself succeeded. */
+catq_status catq_device_status(catq_stream stream, int32_t* out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CATQ_H */

@@ -1,0 +1,228 @@
+"""Plain fp64 CPU oracle of the CAT-Q soft-ternary calibration hot path.
+
+TEST INFRASTRUCTURE ONLY.  This module is imported by ``tests/``, by
+``__graft_entry__.smoke()`` and by ``bench.py``'s CPU-baseline leg, and by nothing
+else.  It shares no code with the CUDA path and never reads anything the CUDA path
+produced.  Every function is the paper's definition written out in fp64 numpy, in the
+paper's order and notation; matrix products use numpy's matmul as a library step.
+
+Notation (CAT-Q, §2): W [N, K] is a linear layer's weight (row-major, out x in), X [M, K]
+its calibration input, Y = X Wq^T its output.  W is flattened row-major and split into
+G = N*K/g consecutive groups of g elements (App. B.2); every statistic and factor is per
+group.
+
+Pins (tests/test_oracle_pins.py) tie each function to something other than itself:
+brute force, closed forms, limits and finite differences.  One part is
+"parity unpinned": the HARD-phase factor gradients (see ``linear_bwd``), which rest on
+this library's reading of §2.3's stage-2 rule and have no independent reference.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+PHASE_TEACHER, PHASE_SOFT, PHASE_HARD = 0, 1, 2
+THR_HALF, THR_TWN07 = 0, 1
+
+
+def _groups(W: np.ndarray, g: int) -> np.ndarray:
+    """Row-major flatten and split into [G, g] (App. B.2: flattened, non-overlapping
+    groups of size g)."""
+    W = np.asarray(W, dtype=np.float64)
+    assert W.size % g == 0
+    return W.reshape(-1, g)
+
+
+def group_stats(W: np.ndarray, g: int, thr_init: int = THR_HALF):
+    """Eq. 3's frozen statistics per group and the initial threshold of §2.2.
+
+    mu0 = mean of the group; alpha0 = mean |W - mu0|.  Delta0 = 0.5 in What units
+    (§2.2 default) or, for the TWN rule of §2.2, the threshold 0.7 * mean|W| expressed
+    in What units at identity factors: 0.7 * mean|W| / alpha0.
+    """
+    Wg = _groups(W, g)
+    mu0 = Wg.mean(axis=1)
+    alpha0 = np.abs(Wg - mu0[:, None]).mean(axis=1)
+    if thr_init == THR_HALF:
+        delta0 = np.full_like(mu0, 0.5)
+    elif thr_init == THR_TWN07:
+        mean_abs = np.abs(Wg).mean(axis=1)
+        with np.errstate(divide="ignore", invalid="ignore"):
+            delta0 = np.where(alpha0 > 0, 0.7 * mean_abs / np.where(alpha0 > 0, alpha0, 1.0), 0.5)
+    else:
+        raise ValueError("thr_init")
+    return mu0, alpha0, delta0
+
+
+def modulation(mu0, alpha0, delta0, d_mu, d_alpha, d_delta):
+    """Eq. 3 and the threshold rule of §2.2:
+    mu = mu0 + d_mu * alpha0, alpha = d_alpha * alpha0, Delta = d_delta * Delta0."""
+    mu0, alpha0, delta0 = (np.asarray(a, np.float64) for a in (mu0, alpha0, delta0))
+    d_mu, d_alpha, d_delta = (np.asarray(a, np.float64) for a in (d_mu, d_alpha, d_delta))
+    mu = mu0 + d_mu * alpha0
+    alpha = d_alpha * alpha0
+    Delta = d_delta * delta0
+    return mu, alpha, Delta
+
+
+def transformed_weight(W, g, mu, alpha):
+    """Eq. 3: What = (W - mu) / alpha, per group, returned as [G, g].
+    A group with alpha == 0 is degenerate; its What is set to 0 (library reading)."""
+    Wg = _groups(W, g)
+    safe = np.where(alpha != 0, alpha, 1.0)
+    What = (Wg - mu[:, None]) / safe[:, None]
+    return np.where((alpha != 0)[:, None], What, 0.0)
+
+
+def transition_f(x, s, Delta):
+    """Eq. 5: f(x; s, Delta) = [tanh(s(x - Delta)) + tanh(s(x + Delta))] / (2 tanh s)."""
+    x = np.asarray(x, np.float64)
+    return (np.tanh(s * (x - Delta)) + np.tanh(s * (x + Delta))) / (2.0 * np.tanh(s))
+
+
+def transition_f_grads(x, s, Delta):
+    """Partial derivatives of Eq. 5 with respect to its input x and to Delta:
+    with a = tanh(s(x-Delta)), b = tanh(s(x+Delta)) and c = 2 tanh s,
+    df/dx = s [(1 - a^2) + (1 - b^2)] / c,  df/dDelta = s [(1 - b^2) - (1 - a^2)] / c."""
+    x = np.asarray(x, np.float64)
+    a = np.tanh(s * (x - Delta))
+    b = np.tanh(s * (x + Delta))
+    c = 2.0 * np.tanh(s)
+    dfdx = s * ((1.0 - a * a) + (1.0 - b * b)) / c
+    dfdD = s * ((1.0 - b * b) - (1.0 - a * a)) / c
+    return dfdx, dfdD
+
+
+def hard_q(x, Delta):
+    """Eq. 2: Q(x; Delta) = 1 if x > Delta, 0 if |x| <= Delta, -1 if x < -Delta."""
+    x = np.asarray(x, np.float64)
+    return np.where(x > Delta, 1.0, np.where(x < -Delta, -1.0, 0.0))
+
+
+def _per_elem(v, g):
+    return np.repeat(np.asarray(v, np.float64), g)
+
+
+def ternary_weight(W, g, stats, factors, phase, s):
+    """Eq. 6 and the reconstruction W ~ alpha T without mu (§2.2, App. B.2).
+
+    Returns (Wq [N, K], T [N, K], What [N, K], alpha [G], Delta [G]).
+    TEACHER (t = 0): T = W and Wq = W.  SOFT: T = f(What; s, Delta).  HARD: T = Q(What; Delta).
+    """
+    W = np.asarray(W, np.float64)
+    N, K = W.shape
+    mu, alpha, Delta = modulation(*stats, *factors)
+    What = transformed_weight(W, g, mu, alpha)
+    if phase == PHASE_TEACHER:
+        return W.copy(), W.copy(), What.reshape(N, K), alpha, Delta
+    if phase == PHASE_SOFT:
+        T = transition_f(What, s, Delta[:, None])
+    elif phase == PHASE_HARD:
+        T = hard_q(What, Delta[:, None])
+    else:
+        raise ValueError("phase")
+    T = np.where((alpha != 0)[:, None], T, 0.0)
+    Wq = alpha[:, None] * T
+    return Wq.reshape(N, K), T.reshape(N, K), What.reshape(N, K), alpha, Delta
+
+
+def linear_fwd(X, Wq):
+    """The contraction of one linear: Y = X Wq^T (Y [M, N], X [M, K], Wq [N, K])."""
+    return np.asarray(X, np.float64) @ np.asarray(Wq, np.float64).T
+
+
+def recon_loss(Y, Y_ref, reduction: int = 0):
+    """Eq. 7 for one linear: the squared L2 distance between the quantized output and the
+    full-precision (teacher) output, averaged over elements (reduction 0, the library
+    default) or summed (1).  Returns (loss, dL/dY)."""
+    d = np.asarray(Y, np.float64) - np.asarray(Y_ref, np.float64)
+    if reduction == 0:
+        n = d.size
+        return float((d * d).sum() / n), 2.0 * d / n
+    return float((d * d).sum()), 2.0 * d
+
+
+def factor_grads_from_G(Gw, W, g, stats, factors, phase, s):
+    """Chain rule of Eq. 3 and Eq. 5/6 from G = dL/dWq [N, K] into the three factors.
+
+    Wq = alpha * T(What), What = (W - mu)/alpha, mu = mu0 + d_mu*alpha0,
+    alpha = d_alpha*alpha0, Delta = d_delta*Delta0 give per element
+      dWq/dmu = -f'(What),  dWq/dalpha = T - What f'(What),  dWq/dDelta = alpha df/dDelta,
+    and the factor gradients are the group sums times alpha0, alpha0 and Delta0.
+    SOFT: T = f.  HARD (reading of §2.3's stage-2 rule): T = Q(What; Delta) as in the
+    forward, with f's derivatives at the given s — parity unpinned.  TEACHER: zeros.
+    """
+    mu0, alpha0, delta0 = (np.asarray(a, np.float64) for a in stats)
+    G = mu0.shape[0]
+    if phase == PHASE_TEACHER:
+        z = np.zeros(G)
+        return z, z.copy(), z.copy()
+    mu, alpha, Delta = modulation(*stats, *factors)
+    What = transformed_weight(W, g, mu, alpha)
+    Gg = np.asarray(Gw, np.float64).reshape(-1, g)
+    dfdx, dfdD = transition_f_grads(What, s, Delta[:, None])
+    if phase == PHASE_SOFT:
+        T = transition_f(What, s, Delta[:, None])
+    elif phase == PHASE_HARD:
+        T = hard_q(What, Delta[:, None])
+    else:
+        raise ValueError("phase")
+    live = alpha != 0
+    g_dmu = np.where(live, -alpha0 * (Gg * dfdx).sum(axis=1), 0.0)
+    g_dalpha = np.where(live, alpha0 * (Gg * (T - What * dfdx)).sum(axis=1), 0.0)
+    g_ddelta = np.where(live, delta0 * alpha * (Gg * dfdD).sum(axis=1), 0.0)
+    return g_dmu, g_dalpha, g_ddelta
+
+
+def linear_bwd(X, dY, W, g, stats, factors, phase, s):
+    """Backward of Y = X Wq^T: dX = dY Wq, G = dY^T X (= dL/dWq), then the factor
+    gradients of ``factor_grads_from_G``.  Returns (dX, g_dmu, g_dalpha, g_ddelta)."""
+    X = np.asarray(X, np.float64)
+    dY = np.asarray(dY, np.float64)
+    Wq = ternary_weight(W, g, stats, factors, phase, s)[0]
+    dX = dY @ Wq
+    Gw = dY.T @ X
+    return (dX,) + factor_grads_from_G(Gw, W, g, stats, factors, phase, s)
+
+
+def calibration_step(X, W, g, stats, factors, phase, s, reduction=0):
+    """One soft-ternary calibration step for one linear (Eq. 6, Eq. 7): teacher output,
+    quantized output, loss, and every gradient.  Returns a dict."""
+    Y_ref = linear_fwd(X, W)
+    Wq = ternary_weight(W, g, stats, factors, phase, s)[0]
+    Y = linear_fwd(X, Wq)
+    loss, dY = recon_loss(Y, Y_ref, reduction)
+    dX, g_dmu, g_dalpha, g_ddelta = linear_bwd(X, dY, W, g, stats, factors, phase, s)
+    return dict(Y_ref=Y_ref, Y=Y, loss=loss, dY=dY, dX=dX, g_dmu=g_dmu, g_dalpha=g_dalpha,
+                g_ddelta=g_ddelta, Wq=Wq)
+
+
+def hard_codes(W, g, stats, factors):
+    """Eq. 4: T = Q(What; d_delta * Delta0) as int8, plus alpha per group and the fp64
+    distance of every |What| from its threshold (for the near-threshold listing)."""
+    mu, alpha, Delta = modulation(*stats, *factors)
+    What = transformed_weight(W, g, mu, alpha)
+    T = hard_q(What, Delta[:, None])
+    T = np.where((alpha != 0)[:, None], T, 0.0).astype(np.int8)
+    gap = np.abs(np.abs(What) - Delta[:, None])
+    rel_gap = gap / np.where(Delta != 0, np.abs(Delta), 1.0)[:, None]
+    return T.reshape(-1), alpha, rel_gap.reshape(-1)
+
+
+def pack_codes(T):
+    """2-bit packing of ternary codes (this library's encoding; the paper fixes none):
+    element e stores T_e + 1 in bits [2*(e % 4), 2*(e % 4) + 1] of byte e // 4."""
+    T = np.asarray(T).reshape(-1).astype(np.int64)
+    assert T.size % 4 == 0
+    out = np.zeros(T.size // 4, dtype=np.int64)
+    for i in range(4):
+        out |= (T[i::4] + 1) << (2 * i)
+    return out.astype(np.uint8)
+
+
+def unpack_codes(codes, n):
+    """Inverse of ``pack_codes`` (used only by tests)."""
+    codes = np.asarray(codes, np.uint8).astype(np.int64)
+    T = np.zeros(codes.size * 4, dtype=np.int64)
+    for i in range(4):
+        T[i::4] = ((codes >> (2 * i)) & 3) - 1
+    return T[:n].astype(np.int8)

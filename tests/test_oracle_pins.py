@@ -1,0 +1,406 @@
+"""Pins of the fp64 oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle against something other than itself: exhaustive
+enumeration, closed forms, limits stated in §2.3, special cases that reduce to a
+textbook rule, and central finite differences.  A plausible slip in the oracle (a
+dropped term, a flipped sign, a transposed operand, a wrong group index) fails at least
+one of them.  No GPU is used.
+"""
+import itertools
+import os
+
+import numpy as np
+import pytest
+
+from oracle import catq_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+# ----------------------------------------------------------------- Eq. 1 / Eq. 2 (brute force)
+
+def _half_enum():
+    """All 3^8 ternary vectors of length 8."""
+    return np.array(list(itertools.product([-1, 0, 1], repeat=8)), dtype=np.float64)
+
+
+@pytest.mark.parametrize("delta", [0.5, 0.3, 0.8])
+def test_q_is_the_exhaustive_minimiser_4x4(delta):
+    """For a fixed scale, Q(x; Delta) (Eq. 2) is the unique minimiser over all 3^16 ternary
+    4x4 matrices of sum (x - T)^2 + (2 Delta - 1) ||T||_0: choosing +-1 over 0 costs
+    (|x| - 1)^2 - x^2 + (2 Delta - 1) = 2 (Delta - |x|), negative iff |x| > Delta.  At
+    Delta = 1/2 this is nearest-ternary rounding, i.e. argmin_T ||What - T||^2 with the
+    paper's Delta0 = 0.5 in What units (§2.2)."""
+    r = np.random.default_rng(7)
+    half = _half_enum()
+    for trial in range(3):
+        x = r.uniform(-1.6, 1.6, 16)
+        x[np.abs(np.abs(x) - delta) < 1e-3] += 0.01  # keep clear of exact ties
+        pen = 2 * delta - 1
+        a, b = x[:8], x[8:]
+        cost_a = ((a[None, :] - half) ** 2).sum(1) + pen * (half != 0).sum(1)
+        cost_b = ((b[None, :] - half) ** 2).sum(1) + pen * (half != 0).sum(1)
+        best, arg = np.inf, None
+        for i in range(half.shape[0]):  # exhaustive over all 3^16 pairs
+            tot = cost_a[i] + cost_b
+            j = int(np.argmin(tot))
+            if tot[j] < best:
+                best, arg = tot[j], (i, j)
+        T_brute = np.concatenate([half[arg[0]], half[arg[1]]])
+        np.testing.assert_array_equal(O.hard_q(x, delta), T_brute)
+
+
+def test_twn_objective_brute_force_is_a_threshold_ternarization():
+    """Eq. 1 solved by enumerating all 3^16 T for a 4x4 W (best alpha > 0 per T): the
+    minimiser keeps the largest |W| with their signs, i.e. it is Q(W; Delta) (Eq. 2) for a
+    threshold between the kept and the dropped magnitudes, and alpha is the mean |W| over
+    the kept set (TWN's alpha, §2.2)."""
+    r = np.random.default_rng(11)
+    half = _half_enum()
+    nnz_h = (half != 0).sum(1).astype(np.float64)
+    for trial in range(3):
+        W = r.standard_normal(16)
+        a, b = W[:8], W[8:]
+        dot_a, dot_b = half @ a, half @ b
+        best, arg = np.inf, None
+        for i in range(half.shape[0]):
+            nnz = nnz_h[i] + nnz_h
+            dot = dot_a[i] + dot_b
+            with np.errstate(divide="ignore", invalid="ignore"):
+                red = np.where((nnz > 0) & (dot > 0), dot * dot / np.where(nnz > 0, nnz, 1), 0.0)
+            obj = (W * W).sum() - red  # min over alpha > 0 of ||W - alpha T||^2
+            j = int(np.argmin(obj))
+            if obj[j] < best:
+                best, arg = obj[j], (i, j)
+        T = np.concatenate([half[arg[0]], half[arg[1]]])
+        kept = np.abs(W[T != 0])
+        dropped = np.abs(W[T == 0])
+        assert kept.size > 0
+        lo = dropped.max() if dropped.size else 0.0
+        delta = 0.5 * (lo + kept.min())
+        np.testing.assert_array_equal(O.hard_q(W, delta), T)
+        alpha = (W * T).sum() / (T != 0).sum()
+        np.testing.assert_allclose(alpha, kept.mean(), rtol=1e-12)
+
+
+def test_q_tie_goes_to_zero():
+    """Eq. 2 uses |x| <= Delta for the zero state."""
+    np.testing.assert_array_equal(O.hard_q(np.array([0.5, -0.5, 0.5000001, -0.5000001]), 0.5),
+                                  [0, 0, 1, -1])
+
+
+# ----------------------------------------------------------------- Eq. 5 (closed forms, limits)
+
+@pytest.mark.parametrize("s", [1e-3, 0.625, 4.95, 30.0, 300.0])
+def test_f_at_threshold_half_is_half(s):
+    """f(1/2; s, 1/2) = [tanh 0 + tanh s] / (2 tanh s) = 1/2 for every s."""
+    assert abs(O.transition_f(0.5, s, 0.5) - 0.5) < 1e-15
+
+
+@pytest.mark.parametrize("s,D", [(0.625, 0.5), (15.0, 0.4), (30.0, 0.6)])
+def test_f_is_odd(s, D):
+    """Property (1) of §2.3: the curve is symmetric about the origin."""
+    x = np.linspace(-3, 3, 601)
+    np.testing.assert_allclose(O.transition_f(-x, s, D), -O.transition_f(x, s, D), atol=1e-15)
+
+
+@pytest.mark.parametrize("D", [0.3, 0.5, 1.2])
+def test_f_small_s_series(D):
+    """Property (2) of §2.3 (s -> 0 gives the identity), to second order: expanding tanh
+    gives f(x) = x - s^2 x (x^2 + 3 Delta^2 - 1) / 3 + O(s^4)."""
+    s = 1e-4
+    x = np.linspace(-2, 2, 41)
+    corr = -(s * s) * x * (x * x + 3 * D * D - 1) / 3  # ~1e-8; the O(s^4) rest is ~1e-16
+    np.testing.assert_allclose(O.transition_f(x, s, D) - x, corr, atol=2e-13)
+    np.testing.assert_allclose(O.transition_f(x, 1e-6, D), x, atol=1e-11)
+
+
+@pytest.mark.parametrize("D", [0.3, 0.5, 0.9])
+def test_f_hard_limit_is_q(D):
+    """Property (4) of §2.3: s -> infinity gives Q (Eq. 2) away from |x| = Delta; scaled by
+    alpha the outputs lie in {-alpha, 0, alpha}; at |x| = Delta the limit is +-1/2."""
+    s = 1e5
+    x = np.linspace(-3, 3, 6001)
+    x = x[np.abs(np.abs(x) - D) > 1e-3]
+    f = O.transition_f(x, s, D)
+    np.testing.assert_allclose(f, O.hard_q(x, D), atol=1e-12)
+    alpha = 0.037
+    vals = np.unique(np.round(alpha * f / alpha * 1e9) / 1e9)
+    assert set(vals.tolist()) <= {-1.0, 0.0, 1.0}
+    np.testing.assert_allclose(O.transition_f(np.array([D, -D]), s, D), [0.5, -0.5], atol=1e-12)
+
+
+def test_f_sharpens_monotonically():
+    """Property (3) of §2.3: with growing s the distance to Q shrinks (away from the
+    threshold)."""
+    x = np.linspace(-2, 2, 401)
+    D = 0.5
+    x = x[np.abs(np.abs(x) - D) > 0.05]
+    errs = [np.abs(O.transition_f(x, s, D) - O.hard_q(x, D)).max() for s in (5, 10, 20, 40, 80)]
+    assert all(a > b for a, b in zip(errs, errs[1:]))
+
+
+@pytest.mark.parametrize("s,D", [(0.625, 0.5), (15.0, 0.45), (30.0, 0.55)])
+def test_f_derivatives_match_finite_differences(s, D):
+    x = np.linspace(-2, 2, 81)
+    h = 1e-6
+    dfdx, dfdD = O.transition_f_grads(x, s, D)
+    fd_x = (O.transition_f(x + h, s, D) - O.transition_f(x - h, s, D)) / (2 * h)
+    fd_D = (O.transition_f(x, s, D + h) - O.transition_f(x, s, D - h)) / (2 * h)
+    scale = max(1.0, np.abs(fd_x).max())
+    np.testing.assert_allclose(dfdx, fd_x, atol=1e-6 * scale)
+    np.testing.assert_allclose(dfdD, fd_D, atol=1e-6 * scale)
+
+
+# ----------------------------------------------------------------- Eq. 3 statistics
+
+def test_group_stats_closed_form():
+    """Two-valued groups [a]*h + [b]*h: mu0 = (a + b)/2, alpha0 = |a - b|/2, and the TWN
+    rule's Delta0 = 0.7 * (|a| + |b|)/2 / alpha0.  Groups are consecutive runs of g in the
+    row-major flattening (App. B.2), so a 2 x 8 matrix with g = 4 has 4 groups."""
+    W = np.array([[1, 1, 3, 3, -2, -2, -2, -2],
+                  [0.5, 0.5, -1.5, -1.5, 4, 4, 8, 8]], dtype=np.float64)
+    mu0, alpha0, delta0 = O.group_stats(W, 4, O.THR_TWN07)
+    np.testing.assert_allclose(mu0, [2, -2, -0.5, 6])
+    np.testing.assert_allclose(alpha0, [1, 0, 1, 2])
+    np.testing.assert_allclose(delta0, [0.7 * 2 / 1, 0.5, 0.7 * 1 / 1, 0.7 * 6 / 2])
+    _, _, d_half = O.group_stats(W, 4, O.THR_HALF)
+    np.testing.assert_allclose(d_half, 0.5)
+
+
+def test_group_stats_equivariance():
+    r = np.random.default_rng(3)
+    W = r.standard_normal((6, 64))
+    mu0, alpha0, _ = O.group_stats(W, 16)
+    mu1, alpha1, _ = O.group_stats(3.0 * W + 0.25, 16)
+    np.testing.assert_allclose(mu1, 3.0 * mu0 + 0.25, rtol=1e-13, atol=1e-14)
+    np.testing.assert_allclose(alpha1, 3.0 * alpha0, rtol=1e-13)
+
+
+# ----------------------------------------------------------------- LM reduces to plain ternarization
+
+def _zero_mean_weight(rows, K, g, seed):
+    """Groups of the form [v, -v] with v on a 1/64 grid: the group mean is exactly 0."""
+    r = np.random.default_rng(seed)
+    v = r.integers(-40, 41, size=(rows * K // g, g // 2)) / 64.0
+    return np.concatenate([v, -v], axis=1).reshape(rows, K)
+
+
+def test_identity_modulation_is_unmodulated_ternarization():
+    """At identity factors (d_mu, d_alpha, d_delta) = (0, 1, 1) and mu0 = 0, Eq. 3-4 give
+    alpha T = alpha0 Q(W; Delta0 alpha0): LM ternarization of What equals plain threshold
+    ternarization of W scaled by alpha0."""
+    g = 8
+    W = _zero_mean_weight(4, 16, g, 1)
+    stats = O.group_stats(W, g, O.THR_HALF)
+    assert np.all(stats[0] == 0)
+    G = W.size // g
+    ident = (np.zeros(G), np.ones(G), np.ones(G))
+    Wq, T, _, alpha, _ = O.ternary_weight(W, g, stats, ident, O.PHASE_HARD, 30.0)
+    alpha0 = np.repeat(stats[1], g).reshape(W.shape)
+    thr = 0.5 * alpha0
+    plain = np.where(W > thr, 1.0, np.where(W < -thr, -1.0, 0.0))
+    np.testing.assert_array_equal(T, plain)
+    np.testing.assert_allclose(Wq, alpha0 * plain, rtol=0, atol=0)
+
+
+def test_twn_rule_at_identity_factors():
+    """With Delta0 from TWN's rule (§2.2) and identity factors the hard codes are TWN's
+    Q(W; 0.7 mean|W|) for zero-mean groups (channel-wise groups, one per row)."""
+    K = 32
+    W = _zero_mean_weight(5, K, K, 2)
+    stats = O.group_stats(W, K, O.THR_TWN07)
+    G = W.shape[0]
+    ident = (np.zeros(G), np.ones(G), np.ones(G))
+    _, T, _, _, _ = O.ternary_weight(W, K, stats, ident, O.PHASE_HARD, 30.0)
+    thr = 0.7 * np.abs(W).mean(axis=1, keepdims=True)
+    twn = np.where(W > thr, 1.0, np.where(W < -thr, -1.0, 0.0))
+    np.testing.assert_array_equal(T, twn)
+
+
+def test_modulation_shifts_and_scales():
+    """d_mu shifts the centre by d_mu * alpha0 and d_alpha rescales: for a group with
+    mu0 = 0, alpha0 = 1, the element W = mu + alpha * x maps to What = x (Eq. 3)."""
+    g = 4
+    W = np.array([[1.0, -1.0, 1.0, -1.0]])
+    stats = O.group_stats(W, g)
+    assert stats[0][0] == 0 and stats[1][0] == 1
+    d_mu, d_alpha = 0.25, 2.0
+    mu, alpha, Delta = O.modulation(*stats, [d_mu], [d_alpha], [1.5])
+    assert mu[0] == 0.25 and alpha[0] == 2.0 and Delta[0] == 0.75
+    x = np.array([0.1, -0.3, 1.2, -2.0])
+    W2 = (0.25 + 2.0 * x)[None, :]
+    What = O.transformed_weight(W2, g, mu, alpha)
+    np.testing.assert_allclose(What.reshape(-1), x, rtol=1e-15)
+
+
+# ----------------------------------------------------------------- forward / loss special cases
+
+def test_teacher_forward_identity_input():
+    """Eq. 6 at t = 0 leaves W untouched; with X = I the output is W^T."""
+    r = np.random.default_rng(5)
+    W = r.standard_normal((6, 8))
+    stats = O.group_stats(W, 4)
+    G = W.size // 4
+    fac = (np.zeros(G), np.ones(G), np.ones(G))
+    Wq = O.ternary_weight(W, 4, stats, fac, O.PHASE_TEACHER, 0.0)[0]
+    Y = O.linear_fwd(np.eye(8), Wq)
+    np.testing.assert_array_equal(Y, W.T)
+
+
+def test_hard_forward_is_integer_code_gemm_scaled_per_group():
+    """With T in {-1,0,1} and integer X, Y = X (alpha T)^T equals, per group of g input
+    columns, alpha times the exact integer product X_block T_block^T."""
+    r = np.random.default_rng(9)
+    N, K, g, M = 6, 16, 4, 5
+    W = r.standard_normal((N, K))
+    stats = O.group_stats(W, g)
+    G = N * K // g
+    fac = (r.uniform(-0.1, 0.1, G), r.uniform(0.8, 1.2, G), r.uniform(0.8, 1.2, G))
+    Wq, T, _, alpha, _ = O.ternary_weight(W, g, stats, fac, O.PHASE_HARD, 30.0)
+    X = r.integers(-5, 6, size=(M, K))
+    Ti = T.astype(np.int64)
+    a = alpha.reshape(N, K // g)
+    Y = np.zeros((M, N))
+    for blk in range(K // g):
+        cols = slice(blk * g, (blk + 1) * g)
+        Y += (X[:, cols] @ Ti[:, cols].T) * a[:, blk][None, :]
+    np.testing.assert_allclose(O.linear_fwd(X, Wq), Y, rtol=1e-13, atol=1e-13)
+
+
+def test_recon_loss_constant_offset():
+    Y_ref = np.random.default_rng(1).standard_normal((3, 4))
+    loss, dY = O.recon_loss(Y_ref + 0.5, Y_ref, 0)
+    assert abs(loss - 0.25) < 1e-15
+    np.testing.assert_allclose(dY, np.full((3, 4), 2 * 0.5 / 12))
+    loss_s, dY_s = O.recon_loss(Y_ref + 0.5, Y_ref, 1)
+    assert abs(loss_s - 0.25 * 12) < 1e-13
+    np.testing.assert_allclose(dY_s, 1.0)
+
+
+# ----------------------------------------------------------------- gradients (finite differences)
+
+def _tiny(seed=0, N=4, K=8, g=4, M=3):
+    r = np.random.default_rng(seed)
+    W = r.standard_normal((N, K)) * 0.05
+    X = r.standard_normal((M, K))
+    stats = O.group_stats(W, g)
+    G = N * K // g
+    fac = [r.uniform(-0.1, 0.1, G), r.uniform(0.8, 1.2, G), r.uniform(0.8, 1.2, G)]
+    return W, X, g, stats, fac
+
+
+def _loss(W, X, g, stats, fac, s, Y_ref):
+    Wq = O.ternary_weight(W, g, stats, fac, O.PHASE_SOFT, s)[0]
+    return O.recon_loss(O.linear_fwd(X, Wq), Y_ref)[0]
+
+
+@pytest.mark.parametrize("s", [0.625, 15.0, 30.0])
+def test_soft_gradients_match_central_differences(s):
+    """Analytic dX and factor gradients of the SOFT step against central differences of
+    the oracle's loss (teacher output held fixed), h = 1e-6, relative agreement 1e-6."""
+    W, X, g, stats, fac = _tiny()
+    Y_ref = O.linear_fwd(X, W)
+    Wq = O.ternary_weight(W, g, stats, fac, O.PHASE_SOFT, s)[0]
+    _, dY = O.recon_loss(O.linear_fwd(X, Wq), Y_ref)
+    dX, gmu, galpha, gdelta = O.linear_bwd(X, dY, W, g, stats, fac, O.PHASE_SOFT, s)
+    h = 1e-6
+    for which, analytic in ((0, gmu), (1, galpha), (2, gdelta)):
+        fd = np.zeros_like(analytic)
+        for j in range(analytic.size):
+            fp = [a.copy() for a in fac]
+            fm = [a.copy() for a in fac]
+            fp[which][j] += h
+            fm[which][j] -= h
+            fd[j] = (_loss(W, X, g, stats, fp, s, Y_ref) - _loss(W, X, g, stats, fm, s, Y_ref)) / (2 * h)
+        scale = np.abs(fd).max()
+        np.testing.assert_allclose(analytic, fd, atol=1e-6 * scale + 1e-12)
+    fdX = np.zeros_like(X)
+    for idx in np.ndindex(*X.shape):
+        Xp, Xm = X.copy(), X.copy()
+        Xp[idx] += h
+        Xm[idx] -= h
+        lp = O.recon_loss(O.linear_fwd(Xp, Wq), Y_ref)[0]
+        lm = O.recon_loss(O.linear_fwd(Xm, Wq), Y_ref)[0]
+        fdX[idx] = (lp - lm) / (2 * h)
+    np.testing.assert_allclose(dX, fdX, atol=1e-6 * np.abs(fdX).max())
+
+
+def test_bwd_uses_transposes_correctly_non_square():
+    """Shapes of dX [M, K] and G = dY^T X [N, K] on a non-square layer (M != N != K)."""
+    W, X, g, stats, fac = _tiny(seed=4, N=6, K=12, g=4, M=5)
+    Y_ref = O.linear_fwd(X, W)
+    step = O.calibration_step(X, W, g, stats, fac, O.PHASE_SOFT, 15.0)
+    assert step["dX"].shape == X.shape and step["Y"].shape == (5, 6)
+    assert step["g_dmu"].shape == (6 * 12 // 4,)
+    np.testing.assert_allclose(step["Y_ref"], Y_ref)
+
+
+def test_hard_gradients_reading_self_consistency():
+    """HARD-phase factor gradients (parity unpinned: §2.3's stage-2 rule read as a
+    surrogate) coincide with the SOFT ones at the same large s when no element sits
+    near its threshold, where f and Q agree."""
+    r = np.random.default_rng(12)
+    g = 4
+    N, K, M = 4, 8, 6
+    x = r.choice([-1.3, -0.9, -0.2, 0.1, 0.8, 1.4], size=(N, K))
+    W = x * 0.05
+    stats = O.group_stats(W, g)
+    G = N * K // g
+    fac = [np.zeros(G), np.ones(G), np.ones(G)]
+    X = r.standard_normal((M, K))
+    dY = r.standard_normal((M, N))
+    s = 400.0
+    soft = O.linear_bwd(X, dY, W, g, stats, fac, O.PHASE_SOFT, s)
+    hard = O.linear_bwd(X, dY, W, g, stats, fac, O.PHASE_HARD, s)
+    What = O.transformed_weight(W, g, *O.modulation(*stats, *fac)[:2])
+    assert np.abs(np.abs(What) - 0.5).min() > 0.05
+    for a, b in zip(soft, hard):
+        np.testing.assert_allclose(a, b, rtol=1e-9, atol=1e-12)
+
+
+def test_teacher_bwd_has_zero_factor_grads():
+    W, X, g, stats, fac = _tiny()
+    dY = np.ones((X.shape[0], W.shape[0]))
+    dX, a, b, c = O.linear_bwd(X, dY, W, g, stats, fac, O.PHASE_TEACHER, 0.0)
+    np.testing.assert_allclose(dX, dY @ W)
+    assert not a.any() and not b.any() and not c.any()
+
+
+def test_degenerate_group_is_zero():
+    """A constant group has alpha0 = 0: its Wq, hard codes and gradients are 0."""
+    W = np.array([[0.3, 0.3, 0.3, 0.3, 1.0, -1.0, 0.5, -0.5]])
+    stats = O.group_stats(W, 4)
+    assert stats[1][0] == 0
+    fac = (np.zeros(2), np.ones(2), np.ones(2))
+    Wq, T, _, _, _ = O.ternary_weight(W, 4, stats, fac, O.PHASE_SOFT, 30.0)
+    assert not Wq[0, :4].any()
+    codes, _, _ = O.hard_codes(W, 4, stats, fac)
+    assert not codes[:4].any()
+    X = np.ones((2, 8))
+    dY = np.ones((2, 1))
+    _, gm, ga, gd = O.linear_bwd(X, dY, W, 4, stats, fac, O.PHASE_SOFT, 30.0)
+    assert gm[0] == 0 and ga[0] == 0 and gd[0] == 0
+
+
+# ----------------------------------------------------------------- packing
+
+def _golden_pack():
+    codes = bytes_ = None
+    with open(os.path.join(GOLDEN, "pack_example.txt")) as fh:
+        for line in fh:
+            if line.startswith("codes:"):
+                codes = [int(v) for v in line.split(":")[1].split()]
+            elif line.startswith("bytes:"):
+                bytes_ = [int(v) for v in line.split(":")[1].split()]
+    return np.array(codes), np.array(bytes_, dtype=np.uint8)
+
+
+def test_pack_hand_example():
+    codes, expect = _golden_pack()
+    np.testing.assert_array_equal(O.pack_codes(codes), expect)
+
+
+def test_pack_round_trip():
+    T = np.random.default_rng(2).integers(-1, 2, 4096)
+    np.testing.assert_array_equal(O.unpack_codes(O.pack_codes(T), T.size), T)
