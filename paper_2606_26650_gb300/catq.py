@@ -1,0 +1,223 @@
+"""Python binding of libcatq (include/catq.h): argument marshalling only.
+
+Every function here has the C name of the call it wraps, takes torch tensors that live on
+the current CUDA device, passes their data pointers and the current torch stream to the
+library, and raises CatqError on a non-zero status.  All arithmetic runs in the library's
+CUDA kernels; there is no fallback.  PyTorch provides device memory and streams.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+import re
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "libcatq.so")
+HEADER = os.path.join(os.path.dirname(PKG), "include", "catq.h")
+
+F32, BF16 = 0, 1
+PHASE_TEACHER, PHASE_SOFT, PHASE_HARD = 0, 1, 2
+THR_HALF, THR_TWN07 = 0, 1
+REDUCE_MEAN, REDUCE_SUM = 0, 1
+
+STATUS = {
+    0: "CATQ_OK", 1: "CATQ_ERR_INVALID_ARG", 2: "CATQ_ERR_SHAPE", 3: "CATQ_ERR_DTYPE",
+    4: "CATQ_ERR_ALIGN", 5: "CATQ_ERR_CUDA", 6: "CATQ_ERR_TIMEOUT", 7: "CATQ_ERR_NONFINITE",
+    8: "CATQ_ERR_UNSUPPORTED", 9: "CATQ_ERR_WORKSPACE",
+}
+
+
+class CatqError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {STATUS.get(status, status)}")
+
+
+class catq_layer(ctypes.Structure):
+    _fields_ = [
+        ("N", ctypes.c_int64), ("K", ctypes.c_int64), ("g", ctypes.c_int32), ("w_dtype", ctypes.c_int32),
+        ("W", ctypes.c_void_p),
+        ("mu0", ctypes.c_void_p), ("alpha0", ctypes.c_void_p), ("delta0", ctypes.c_void_p),
+        ("d_mu", ctypes.c_void_p), ("d_alpha", ctypes.c_void_p), ("d_delta", ctypes.c_void_p),
+    ]
+
+
+class catq_schedule(ctypes.Structure):
+    _fields_ = [("phase", ctypes.c_int32), ("s", ctypes.c_float)]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded library; raises if it has not been built (there is no fallback)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with __graft_entry__.build()")
+    L = ctypes.CDLL(LIB_PATH)
+    P, I64, I32, F, S = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_float, ctypes.c_size_t
+    LP = ctypes.POINTER(catq_layer)
+    sig = {
+        "catq_abi_version": (I32, []),
+        "catq_status_string": (ctypes.c_char_p, [I32]),
+        "catq_group_stats": (I32, [LP, I32, P]),
+        "catq_modulate_ternarize": (I32, [LP, catq_schedule, P, P, P, P]),
+        "catq_soft_ternary_linear_fwd": (I32, [LP, catq_schedule, P, I64, I32, P, P]),
+        "catq_bwd_workspace_bytes": (S, [LP, I64]),
+        "catq_soft_ternary_linear_bwd": (I32, [LP, catq_schedule, P, P, I64, I32, P, P, P, P, P, S, P]),
+        "catq_recon_loss_workspace_bytes": (S, [I64]),
+        "catq_recon_loss": (I32, [P, P, I64, I32, I32, P, P, P, S, P]),
+        "catq_hard_ternarize_pack": (I32, [LP, P, P, P]),
+        "catq_device_status": (I32, [P, ctypes.POINTER(I32)]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(L, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = L
+    return L
+
+
+def header_functions(path: str = HEADER):
+    """Names of the functions include/catq.h declares."""
+    text = open(path).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(catq_[a-z0-9_]+)\s*\(", text)))
+
+
+# ------------------------------------------------------------------ marshalling helpers
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _dtype_code(t) -> int:
+    import torch
+    if t.dtype == torch.bfloat16:
+        return BF16
+    if t.dtype == torch.float32:
+        return F32
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _check(status: int, where: str):
+    if status != 0:
+        raise CatqError(status, where)
+
+
+@dataclasses.dataclass
+class Layer:
+    """One linear layer's device state: W [N, K] and the per-group arrays ([G] fp32)."""
+    W: object
+    g: int
+    mu0: object
+    alpha0: object
+    delta0: object
+    d_mu: object
+    d_alpha: object
+    d_delta: object
+
+    @classmethod
+    def create(cls, W, g, d_mu=None, d_alpha=None, d_delta=None):
+        """Allocates the statistics and (identity, unless given) factor tensors."""
+        import torch
+        N, K = W.shape
+        G = N * K // g
+        kw = dict(device=W.device, dtype=torch.float32)
+        return cls(W, g, torch.empty(G, **kw), torch.empty(G, **kw), torch.empty(G, **kw),
+                   d_mu if d_mu is not None else torch.zeros(G, **kw),
+                   d_alpha if d_alpha is not None else torch.ones(G, **kw),
+                   d_delta if d_delta is not None else torch.ones(G, **kw))
+
+    @property
+    def N(self):
+        return self.W.shape[0]
+
+    @property
+    def K(self):
+        return self.W.shape[1]
+
+    @property
+    def G(self):
+        return self.N * self.K // self.g
+
+    def struct(self) -> catq_layer:
+        return catq_layer(self.N, self.K, self.g, _dtype_code(self.W), self.W.data_ptr(),
+                          self.mu0.data_ptr(), self.alpha0.data_ptr(), self.delta0.data_ptr(),
+                          self.d_mu.data_ptr(), self.d_alpha.data_ptr(), self.d_delta.data_ptr())
+
+
+def schedule(phase: int, s: float = 0.0) -> catq_schedule:
+    return catq_schedule(int(phase), float(s))
+
+
+# ------------------------------------------------------------------ the C calls
+
+def catq_group_stats(layer: Layer, thr_init: int = THR_HALF, stream=None):
+    st = layer.struct()
+    _check(lib().catq_group_stats(ctypes.byref(st), int(thr_init), _stream(stream)), "catq_group_stats")
+
+
+def catq_modulate_ternarize(layer: Layer, sched: catq_schedule, Wq_out=None, T_out=None, alpha_out=None,
+                            stream=None):
+    st = layer.struct()
+    _check(lib().catq_modulate_ternarize(ctypes.byref(st), sched, _ptr(Wq_out), _ptr(T_out), _ptr(alpha_out),
+                                         _stream(stream)), "catq_modulate_ternarize")
+
+
+def catq_soft_ternary_linear_fwd(layer: Layer, sched: catq_schedule, X, Y, stream=None):
+    st = layer.struct()
+    _check(lib().catq_soft_ternary_linear_fwd(ctypes.byref(st), sched, _ptr(X), X.shape[0], _dtype_code(X),
+                                              _ptr(Y), _stream(stream)), "catq_soft_ternary_linear_fwd")
+
+
+def catq_bwd_workspace_bytes(layer: Layer, M: int) -> int:
+    st = layer.struct()
+    return int(lib().catq_bwd_workspace_bytes(ctypes.byref(st), int(M)))
+
+
+def catq_soft_ternary_linear_bwd(layer: Layer, sched: catq_schedule, X, dY, dX, g_dmu, g_dalpha, g_ddelta,
+                                 workspace, stream=None):
+    st = layer.struct()
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib().catq_soft_ternary_linear_bwd(ctypes.byref(st), sched, _ptr(X), _ptr(dY), X.shape[0],
+                                              _dtype_code(X), _ptr(dX), _ptr(g_dmu), _ptr(g_dalpha),
+                                              _ptr(g_ddelta), _ptr(workspace), ws_bytes, _stream(stream)),
+           "catq_soft_ternary_linear_bwd")
+
+
+def catq_recon_loss_workspace_bytes(count: int) -> int:
+    return int(lib().catq_recon_loss_workspace_bytes(int(count)))
+
+
+def catq_recon_loss(Y, Y_ref, loss_out, dY=None, workspace=None, reduction: int = REDUCE_MEAN, stream=None):
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib().catq_recon_loss(_ptr(Y), _ptr(Y_ref), Y.numel(), _dtype_code(Y), int(reduction), _ptr(loss_out),
+                                 _ptr(dY), _ptr(workspace), ws_bytes, _stream(stream)), "catq_recon_loss")
+
+
+def catq_hard_ternarize_pack(layer: Layer, codes, alpha=None, stream=None):
+    st = layer.struct()
+    _check(lib().catq_hard_ternarize_pack(ctypes.byref(st), _ptr(codes), _ptr(alpha), _stream(stream)),
+           "catq_hard_ternarize_pack")
+
+
+def catq_device_status(stream=None) -> int:
+    out = ctypes.c_int32(0)
+    _check(lib().catq_device_status(_stream(stream), ctypes.byref(out)), "catq_device_status")
+    return int(out.value)
+
+
+def workspace(nbytes: int, device):
+    """A byte tensor of at least nbytes (256-byte aligned by the caching allocator)."""
+    import torch
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)

@@ -1,0 +1,253 @@
+// api.cu — the extern "C" boundary (include/catq.h): argument validation, dtype routing
+// (bf16 -> tensor-core kernels, fp32 -> CUDA-core kernels) and workspace sizing.  Nothing
+// here allocates memory; every launch goes to the caller's stream.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+
+#include "catq.h"
+#include "launch.h"
+
+using namespace catq;
+
+namespace {
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool aligned256(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 255u) == 0; }
+
+size_t round256(size_t b) { return (b + 255) & ~static_cast<size_t>(255); }
+
+catq_status cuda_status(cudaError_t e) { return e == cudaSuccess ? CATQ_OK : CATQ_ERR_CUDA; }
+
+// Shape / dtype / pointer checks common to every layer call.  `need_factors` also requires
+// the statistics and learnable-factor arrays.
+catq_status check_layer(const catq_layer* L, bool need_factors) {
+  if (!L || !L->W) return CATQ_ERR_INVALID_ARG;
+  if (L->w_dtype != CATQ_F32 && L->w_dtype != CATQ_BF16) return CATQ_ERR_DTYPE;
+  if (L->N < 1 || L->K < 1 || L->g < 1) return CATQ_ERR_SHAPE;
+  if (L->K % L->g != 0) return CATQ_ERR_SHAPE;
+  if (L->w_dtype == CATQ_BF16) {
+    if (L->g % 64 != 0 || L->N % 8 != 0) return CATQ_ERR_SHAPE;
+  } else {
+    if (!(L->g % 64 == 0 || L->g == 4 || L->g == 8 || L->g == 16 || L->g == 32)) return CATQ_ERR_SHAPE;
+  }
+  if (!aligned16(L->W)) return CATQ_ERR_ALIGN;
+  if (!L->mu0 || !L->alpha0 || !L->delta0) return CATQ_ERR_INVALID_ARG;
+  if (need_factors && (!L->d_mu || !L->d_alpha || !L->d_delta)) return CATQ_ERR_INVALID_ARG;
+  return CATQ_OK;
+}
+
+catq_status check_schedule(catq_schedule sc, bool need_s) {
+  if (sc.phase != CATQ_PHASE_TEACHER && sc.phase != CATQ_PHASE_SOFT && sc.phase != CATQ_PHASE_HARD)
+    return CATQ_ERR_INVALID_ARG;
+  if (need_s && !(std::isfinite(sc.s) && sc.s > 0.0f)) return CATQ_ERR_INVALID_ARG;
+  return CATQ_OK;
+}
+
+LayerDev to_dev(const catq_layer* L) {
+  LayerDev d;
+  d.W = L->W;
+  d.N = L->N;
+  d.K = L->K;
+  d.g = L->g;
+  d.groups_per_row = static_cast<int32_t>(L->K / L->g);
+  d.mu0 = L->mu0;
+  d.alpha0 = L->alpha0;
+  d.delta0 = L->delta0;
+  d.d_mu = L->d_mu;
+  d.d_alpha = L->d_alpha;
+  d.d_delta = L->d_delta;
+  return d;
+}
+
+StepScalars scalars(catq_schedule sc) {
+  StepScalars s;
+  s.phase = sc.phase;
+  s.s = sc.s;
+  const double t = (sc.s > 0.0f && std::isfinite(sc.s)) ? std::tanh(static_cast<double>(sc.s)) : 0.0;
+  s.inv_2tanh_s = t > 0.0 ? static_cast<float>(1.0 / (2.0 * t)) : 0.0f;
+  return s;
+}
+
+// The bf16 path needs an sm_100-class GPU (tcgen05, TMA) and the driver's tensor-map encoder.
+catq_status check_tensor_core_device() {
+  int dev = 0, major = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return CATQ_ERR_CUDA;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess) return CATQ_ERR_CUDA;
+  if (major != 10) return CATQ_ERR_UNSUPPORTED;
+  if (!tensor_map_encoder_available()) return CATQ_ERR_UNSUPPORTED;
+  return CATQ_OK;
+}
+
+int current_sm_count() {
+  int dev = 0, n = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  return n > 0 ? n : 1;
+}
+
+size_t bwd_partials_bytes(const catq_layer* L, int64_t M, TcPlan* plan_out, int32_t* P_out, int32_t* splits_out) {
+  if (L->w_dtype == CATQ_BF16) {
+    const TcPlan p = tc_plan_bwd(to_dev(L), M, current_sm_count());
+    if (plan_out) *plan_out = p;
+    if (P_out) *P_out = p.dw_P;
+    if (splits_out) *splits_out = p.dw_splits;
+    return static_cast<size_t>(p.dw_splits) * 3 * static_cast<size_t>(L->N) * static_cast<size_t>(L->K / p.dw_P) *
+           sizeof(float);
+  }
+  const int32_t P = L->g < kSimtTile ? L->g : kSimtTile;
+  if (P_out) *P_out = P;
+  if (splits_out) *splits_out = 1;
+  return 3 * static_cast<size_t>(L->N) * static_cast<size_t>(L->K / P) * sizeof(float);
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t catq_abi_version(void) { return CATQ_ABI_VERSION; }
+
+const char* catq_status_string(int32_t s) {
+  switch (s) {
+    case CATQ_OK: return "CATQ_OK";
+    case CATQ_ERR_INVALID_ARG: return "CATQ_ERR_INVALID_ARG";
+    case CATQ_ERR_SHAPE: return "CATQ_ERR_SHAPE";
+    case CATQ_ERR_DTYPE: return "CATQ_ERR_DTYPE";
+    case CATQ_ERR_ALIGN: return "CATQ_ERR_ALIGN";
+    case CATQ_ERR_CUDA: return "CATQ_ERR_CUDA";
+    case CATQ_ERR_TIMEOUT: return "CATQ_ERR_TIMEOUT";
+    case CATQ_ERR_NONFINITE: return "CATQ_ERR_NONFINITE";
+    case CATQ_ERR_UNSUPPORTED: return "CATQ_ERR_UNSUPPORTED";
+    case CATQ_ERR_WORKSPACE: return "CATQ_ERR_WORKSPACE";
+    default: return "CATQ_ERR_UNKNOWN";
+  }
+}
+
+catq_status catq_group_stats(const catq_layer* layer, int32_t thr_init, catq_stream stream) {
+  catq_status st = check_layer(layer, false);
+  if (st != CATQ_OK) return st;
+  if (thr_init != CATQ_THR_HALF && thr_init != CATQ_THR_TWN07) return CATQ_ERR_INVALID_ARG;
+  const LayerDev L = to_dev(layer);
+  return cuda_status(launch_group_stats(L, layer->w_dtype, thr_init, layer->mu0, layer->alpha0, layer->delta0,
+                                        reinterpret_cast<cudaStream_t>(stream)));
+}
+
+catq_status catq_modulate_ternarize(const catq_layer* layer, catq_schedule sched, void* Wq_out, int8_t* T_out,
+                                    float* alpha_out, catq_stream stream) {
+  catq_status st = check_layer(layer, true);
+  if (st != CATQ_OK) return st;
+  if ((st = check_schedule(sched, sched.phase == CATQ_PHASE_SOFT)) != CATQ_OK) return st;
+  if (Wq_out && !aligned16(Wq_out)) return CATQ_ERR_ALIGN;
+  if (T_out && !aligned16(T_out)) return CATQ_ERR_ALIGN;
+  if (!Wq_out && !T_out && !alpha_out) return CATQ_OK;
+  return cuda_status(launch_modulate_ternarize(to_dev(layer), layer->w_dtype, scalars(sched), Wq_out, T_out,
+                                               alpha_out, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+catq_status catq_soft_ternary_linear_fwd(const catq_layer* layer, catq_schedule sched, const void* X, int64_t M,
+                                         int32_t x_dtype, void* Y, catq_stream stream) {
+  catq_status st = check_layer(layer, sched.phase != CATQ_PHASE_TEACHER);
+  if (st != CATQ_OK) return st;
+  if ((st = check_schedule(sched, sched.phase == CATQ_PHASE_SOFT)) != CATQ_OK) return st;
+  if (x_dtype != layer->w_dtype) return CATQ_ERR_DTYPE;
+  if (M < 0) return CATQ_ERR_SHAPE;
+  if (M == 0) return CATQ_OK;
+  if (!X || !Y) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(X) || !aligned16(Y)) return CATQ_ERR_ALIGN;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const LayerDev L = to_dev(layer);
+  if (layer->w_dtype == CATQ_F32)
+    return cuda_status(launch_simt_fwd(L, scalars(sched), static_cast<const float*>(X), M, static_cast<float*>(Y), s));
+  if ((st = check_tensor_core_device()) != CATQ_OK) return st;
+  return cuda_status(launch_tc_fwd(L, scalars(sched), X, M, Y, s));
+}
+
+size_t catq_bwd_workspace_bytes(const catq_layer* layer, int64_t M) {
+  if (!layer || layer->g < 1 || layer->K % layer->g != 0 || layer->N < 1) return 0;
+  if (M < 1) M = 1;
+  return round256(bwd_partials_bytes(layer, M, nullptr, nullptr, nullptr));
+}
+
+catq_status catq_soft_ternary_linear_bwd(const catq_layer* layer, catq_schedule sched, const void* X, const void* dY,
+                                         int64_t M, int32_t x_dtype, void* dX, float* g_dmu, float* g_dalpha,
+                                         float* g_ddelta, void* workspace, size_t ws_bytes, catq_stream stream) {
+  catq_status st = check_layer(layer, sched.phase != CATQ_PHASE_TEACHER);
+  if (st != CATQ_OK) return st;
+  if ((st = check_schedule(sched, sched.phase != CATQ_PHASE_TEACHER)) != CATQ_OK) return st;
+  if (x_dtype != layer->w_dtype) return CATQ_ERR_DTYPE;
+  if (M < 0) return CATQ_ERR_SHAPE;
+  if (!g_dmu || !g_dalpha || !g_ddelta) return CATQ_ERR_INVALID_ARG;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const LayerDev L = to_dev(layer);
+  const int64_t G = layer->N * layer->K / layer->g;
+  const bool need_dw = sched.phase != CATQ_PHASE_TEACHER && M > 0;
+  if (M > 0) {
+    if (!X || !dY) return CATQ_ERR_INVALID_ARG;
+    if (!aligned16(X) || !aligned16(dY) || (dX && !aligned16(dX))) return CATQ_ERR_ALIGN;
+  }
+  TcPlan plan{};
+  int32_t P = 0, splits = 0;
+  if (need_dw) {
+    const size_t need = bwd_partials_bytes(layer, M, &plan, &P, &splits);
+    if (!workspace || ws_bytes < need) return CATQ_ERR_WORKSPACE;
+    if (!aligned256(workspace)) return CATQ_ERR_ALIGN;
+  }
+  if (layer->w_dtype == CATQ_BF16 && M > 0 && (st = check_tensor_core_device()) != CATQ_OK) return st;
+  const StepScalars sc = scalars(sched);
+  cudaError_t e = cudaSuccess;
+  if (dX && M > 0) {
+    e = layer->w_dtype == CATQ_F32
+            ? launch_simt_dx(L, sc, static_cast<const float*>(dY), M, static_cast<float*>(dX), s)
+            : launch_tc_dx(L, sc, dY, M, dX, s);
+    if (e != cudaSuccess) return CATQ_ERR_CUDA;
+  }
+  if (!need_dw) {
+    const size_t b = static_cast<size_t>(G) * sizeof(float);
+    if (cudaMemsetAsync(g_dmu, 0, b, s) != cudaSuccess || cudaMemsetAsync(g_dalpha, 0, b, s) != cudaSuccess ||
+        cudaMemsetAsync(g_ddelta, 0, b, s) != cudaSuccess)
+      return CATQ_ERR_CUDA;
+    return CATQ_OK;
+  }
+  float* part = static_cast<float*>(workspace);
+  e = layer->w_dtype == CATQ_F32
+          ? launch_simt_dw(L, sc, static_cast<const float*>(X), static_cast<const float*>(dY), M, part, s)
+          : launch_tc_dw(L, sc, X, dY, M, plan, part, s);
+  if (e != cudaSuccess) return CATQ_ERR_CUDA;
+  return cuda_status(launch_grad_reduce(L, sc, part, splits, P, g_dmu, g_dalpha, g_ddelta, s));
+}
+
+size_t catq_recon_loss_workspace_bytes(int64_t count) {
+  return round256(static_cast<size_t>(recon_loss_blocks(count < 1 ? 1 : count)) * sizeof(double));
+}
+
+catq_status catq_recon_loss(const void* Y, const void* Y_ref, int64_t count, int32_t dtype, int32_t reduction,
+                            float* loss_out, void* dY, void* workspace, size_t ws_bytes, catq_stream stream) {
+  if (dtype != CATQ_F32 && dtype != CATQ_BF16) return CATQ_ERR_DTYPE;
+  if (reduction != CATQ_REDUCE_MEAN && reduction != CATQ_REDUCE_SUM) return CATQ_ERR_INVALID_ARG;
+  if (count < 1) return CATQ_ERR_SHAPE;
+  if (!Y || !Y_ref || !loss_out) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(Y) || !aligned16(Y_ref) || (dY && !aligned16(dY))) return CATQ_ERR_ALIGN;
+  if (!workspace || ws_bytes < catq_recon_loss_workspace_bytes(count)) return CATQ_ERR_WORKSPACE;
+  if (!aligned256(workspace)) return CATQ_ERR_ALIGN;
+  return cuda_status(launch_recon_loss(Y, Y_ref, count, dtype, reduction, loss_out, dY,
+                                       static_cast<double*>(workspace), reinterpret_cast<cudaStream_t>(stream)));
+}
+
+catq_status catq_hard_ternarize_pack(const catq_layer* layer, uint8_t* codes, float* alpha, catq_stream stream) {
+  catq_status st = check_layer(layer, true);
+  if (st != CATQ_OK) return st;
+  if (!codes) return CATQ_ERR_INVALID_ARG;
+  if ((layer->N * layer->K) % 4 != 0) return CATQ_ERR_SHAPE;
+  if (layer->g % 16 == 0 && !aligned16(codes)) return CATQ_ERR_ALIGN;
+  return cuda_status(launch_hard_pack(to_dev(layer), layer->w_dtype, codes, alpha,
+                                      reinterpret_cast<cudaStream_t>(stream)));
+}
+
+catq_status catq_device_status(catq_stream stream, int32_t* out) {
+  if (!out) return CATQ_ERR_INVALID_ARG;
+  if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return CATQ_ERR_CUDA;
+  return cuda_status(read_and_clear_device_status(out));
+}
+
+}  // extern "C"

@@ -1,0 +1,377 @@
+// elementwise.cu — the HBM-bound kernels of the path: group statistics (Eq. 3), the
+// materialised Eq. 6 weight (inspection only), the reconstruction loss of Eq. 7 with its
+// gradient, the final hard ternarization + 2-bit pack, and the reduction of the dW
+// epilogue's partial sums into the three factor gradients.
+#include <cuda_bf16.h>
+
+#include "launch.h"
+
+namespace catq {
+namespace {
+
+constexpr int kThreads = 256;
+
+__device__ __forceinline__ double warp_sum(double v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+template <typename T>
+struct Vec16;  // 16-byte vector of T, unpacked to floats
+template <>
+struct Vec16<float> {
+  static constexpr int n = 4;
+  __device__ static void load(const float* p, float (&v)[4]) {
+    const float4 q = __ldg(reinterpret_cast<const float4*>(p));
+    v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+  }
+};
+template <>
+struct Vec16<__nv_bfloat16> {
+  static constexpr int n = 8;
+  __device__ static void load(const __nv_bfloat16* p, float (&v)[8]) {
+    const uint4 q = __ldg(reinterpret_cast<const uint4*>(p));
+    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      v[2 * i] = bf16lo_to_f32(w[i]);
+      v[2 * i + 1] = bf16hi_to_f32(w[i]);
+    }
+  }
+};
+
+// ---------------------------------------------------------------- Eq. 3 statistics
+// One warp per group; fp64 sums; two passes over the group (mean, then deviations).
+template <typename T>
+__global__ void __launch_bounds__(kThreads) group_stats_kernel(const T* __restrict__ W, int64_t G, int32_t g,
+                                                               int32_t thr_init, float* __restrict__ mu0,
+                                                               float* __restrict__ alpha0,
+                                                               float* __restrict__ delta0) {
+  constexpr int V = Vec16<T>::n;
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
+  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
+  for (int64_t j = warp; j < G; j += nwarps) {
+    const T* base = W + j * g;
+    double sum = 0.0;
+    for (int i = lane * V; i < g; i += 32 * V) {
+      float v[V];
+      Vec16<T>::load(base + i, v);
+#pragma unroll
+      for (int q = 0; q < V; ++q) sum += static_cast<double>(v[q]);
+    }
+    const double mu = warp_sum(sum) / static_cast<double>(g);
+    double dev = 0.0, mag = 0.0;
+    for (int i = lane * V; i < g; i += 32 * V) {
+      float v[V];
+      Vec16<T>::load(base + i, v);
+#pragma unroll
+      for (int q = 0; q < V; ++q) {
+        dev += fabs(static_cast<double>(v[q]) - mu);
+        mag += fabs(static_cast<double>(v[q]));
+      }
+    }
+    const double a0 = warp_sum(dev) / static_cast<double>(g);
+    const double m = warp_sum(mag) / static_cast<double>(g);
+    if (lane == 0) {
+      mu0[j] = static_cast<float>(mu);
+      alpha0[j] = static_cast<float>(a0);
+      delta0[j] = (thr_init == 1 && a0 > 0.0) ? static_cast<float>(0.7 * m / a0) : 0.5f;
+    }
+  }
+}
+
+// ---------------------------------------------------------------- materialised Eq. 6 weight
+// One thread per 8 consecutive elements (g % 8 == 0 on the bf16 path keeps them in one
+// group and one row); the bf16 arithmetic is the fused producer's.
+__global__ void __launch_bounds__(kThreads) modulate_bf16_kernel(LayerDev L, StepScalars sc, uint16_t* __restrict__ Wq,
+                                                                 int8_t* __restrict__ Tout, float* __restrict__ alpha) {
+  const int64_t nchunks = L.N * L.K / 8;
+  const int64_t G = L.N * L.K / L.g;
+  const uint16_t* W = static_cast<const uint16_t*>(L.W);
+  for (int64_t c = blockIdx.x * (int64_t)kThreads + threadIdx.x; c < nchunks; c += (int64_t)gridDim.x * kThreads) {
+    const int64_t e = c * 8;
+    const int64_t j = e / L.g;
+    const GroupConst gc = group_const(L, j);
+    const uint4 v = __ldg(reinterpret_cast<const uint4*>(W + e));
+    if (Wq) {
+      const ProducerConst pc = producer_const(gc, sc.s, sc.inv_2tanh_s, sc.phase);
+      *reinterpret_cast<uint4*>(Wq + e) = transform_chunk_bf16(v, pc, sc.phase);
+    }
+    if (Tout) {
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      uint32_t packed[2] = {0u, 0u};
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float x = (i & 1) ? bf16hi_to_f32(w[i >> 1]) : bf16lo_to_f32(w[i >> 1]);
+        const int t = (gc.alpha != 0.0f) ? static_cast<int>(hard_q(what(x, gc), gc.delta)) : 0;
+        packed[i >> 2] |= (static_cast<uint32_t>(static_cast<uint8_t>(static_cast<int8_t>(t)))) << (8 * (i & 3));
+      }
+      *reinterpret_cast<uint2*>(Tout + e) = make_uint2(packed[0], packed[1]);
+    }
+  }
+  if (alpha)
+    for (int64_t j = blockIdx.x * (int64_t)kThreads + threadIdx.x; j < G; j += (int64_t)gridDim.x * kThreads)
+      alpha[j] = __ldg(L.d_alpha + j) * __ldg(L.alpha0 + j);
+}
+
+__global__ void __launch_bounds__(kThreads) modulate_f32_kernel(LayerDev L, StepScalars sc, float* __restrict__ Wq,
+                                                                int8_t* __restrict__ Tout, float* __restrict__ alpha) {
+  const int64_t n = L.N * L.K;
+  const int64_t G = n / L.g;
+  const float* W = static_cast<const float*>(L.W);
+  for (int64_t e = blockIdx.x * (int64_t)kThreads + threadIdx.x; e < n; e += (int64_t)gridDim.x * kThreads) {
+    const GroupConst gc = group_const(L, e / L.g);
+    const float w = W[e];
+    if (Wq) Wq[e] = ternary_weight_f32(w, gc, sc.s, sc.inv_2tanh_s, sc.phase);
+    if (Tout) Tout[e] = (gc.alpha != 0.0f) ? static_cast<int8_t>(hard_q(what(w, gc), gc.delta)) : int8_t(0);
+  }
+  if (alpha)
+    for (int64_t j = blockIdx.x * (int64_t)kThreads + threadIdx.x; j < G; j += (int64_t)gridDim.x * kThreads)
+      alpha[j] = __ldg(L.d_alpha + j) * __ldg(L.alpha0 + j);
+}
+
+// ---------------------------------------------------------------- hard ternarize + pack
+// EPT consecutive elements per thread (EPT divides g, so one group), EPT/4 output bytes.
+template <typename T, int EPT>
+__global__ void __launch_bounds__(kThreads) hard_pack_kernel(LayerDev L, uint8_t* __restrict__ codes,
+                                                             float* __restrict__ alpha) {
+  const int64_t n = L.N * L.K;
+  const int64_t G = n / L.g;
+  const T* W = static_cast<const T*>(L.W);
+  for (int64_t t = blockIdx.x * (int64_t)kThreads + threadIdx.x; t * EPT < n; t += (int64_t)gridDim.x * kThreads) {
+    const int64_t e0 = t * EPT;
+    const GroupConst gc = group_const(L, e0 / L.g);
+    float v[EPT];
+    constexpr int V = Vec16<T>::n;
+    if constexpr (EPT % V == 0) {
+#pragma unroll
+      for (int i = 0; i < EPT; i += V) {
+        float q[V];
+        Vec16<T>::load(W + e0 + i, q);
+#pragma unroll
+        for (int k = 0; k < V; ++k) v[i + k] = q[k];
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < EPT; ++i) {
+        if constexpr (sizeof(T) == 4)
+          v[i] = W[e0 + i];
+        else
+          v[i] = bf16lo_to_f32(static_cast<uint32_t>(reinterpret_cast<const uint16_t*>(W)[e0 + i]));
+      }
+    }
+    uint32_t word = 0;
+#pragma unroll
+    for (int i = 0; i < EPT; ++i) {
+      const int q = (gc.alpha != 0.0f) ? static_cast<int>(hard_q(what(v[i], gc), gc.delta)) : 0;
+      word |= static_cast<uint32_t>(q + 1) << (2 * (i & 15));
+      if ((i & 15) == 15 || i == EPT - 1) {
+        if constexpr (EPT >= 16)
+          reinterpret_cast<uint32_t*>(codes)[(e0 + i) / 16] = word;
+        else
+          codes[e0 / 4] = static_cast<uint8_t>(word);
+        word = 0;
+      }
+    }
+  }
+  if (alpha)
+    for (int64_t j = blockIdx.x * (int64_t)kThreads + threadIdx.x; j < G; j += (int64_t)gridDim.x * kThreads)
+      alpha[j] = __ldg(L.d_alpha + j) * __ldg(L.alpha0 + j);
+}
+
+// ---------------------------------------------------------------- Eq. 7 loss and dY
+constexpr int kLossMaxBlocks = 1216;
+
+template <typename T>
+__device__ __forceinline__ void store_scaled(T* p, const float (&d)[Vec16<T>::n], float scale);
+template <>
+__device__ __forceinline__ void store_scaled<float>(float* p, const float (&d)[4], float scale) {
+  *reinterpret_cast<float4*>(p) = make_float4(d[0] * scale, d[1] * scale, d[2] * scale, d[3] * scale);
+}
+template <>
+__device__ __forceinline__ void store_scaled<__nv_bfloat16>(__nv_bfloat16* p, const float (&d)[8], float scale) {
+  uint4 q;
+  q.x = pack_bf16x2(d[0] * scale, d[1] * scale);
+  q.y = pack_bf16x2(d[2] * scale, d[3] * scale);
+  q.z = pack_bf16x2(d[4] * scale, d[5] * scale);
+  q.w = pack_bf16x2(d[6] * scale, d[7] * scale);
+  *reinterpret_cast<uint4*>(p) = q;
+}
+
+__device__ __forceinline__ float load_scalar(const float* p) { return *p; }
+__device__ __forceinline__ float load_scalar(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+__device__ __forceinline__ void store_scalar(float* p, float v) { *p = v; }
+__device__ __forceinline__ void store_scalar(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads) recon_loss_partial_kernel(const T* __restrict__ Y, const T* __restrict__ Yr,
+                                                                      int64_t count, float scale, T* __restrict__ dY,
+                                                                      double* __restrict__ partials) {
+  constexpr int V = Vec16<T>::n;
+  const int64_t nvec = count / V;
+  double acc = 0.0;
+  for (int64_t i = blockIdx.x * (int64_t)kThreads + threadIdx.x; i < nvec; i += (int64_t)gridDim.x * kThreads) {
+    float a[V], b[V], d[V];
+    Vec16<T>::load(Y + i * V, a);
+    Vec16<T>::load(Yr + i * V, b);
+#pragma unroll
+    for (int q = 0; q < V; ++q) {
+      d[q] = a[q] - b[q];
+      acc += static_cast<double>(d[q]) * static_cast<double>(d[q]);
+    }
+    if (dY) store_scaled<T>(dY + i * V, d, scale);
+  }
+  if (blockIdx.x == 0)
+    for (int64_t i = nvec * V + threadIdx.x; i < count; i += kThreads) {
+      const float d = load_scalar(Y + i) - load_scalar(Yr + i);
+      acc += static_cast<double>(d) * static_cast<double>(d);
+      if (dY) store_scalar(dY + i, d * scale);
+    }
+  __shared__ double red[kThreads / 32];
+  acc = warp_sum(acc);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    double v = threadIdx.x < kThreads / 32 ? red[threadIdx.x] : 0.0;
+    v = warp_sum(v);
+    if (threadIdx.x == 0) partials[blockIdx.x] = v;
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) recon_loss_final_kernel(const double* __restrict__ partials, int nblocks,
+                                                                    double out_scale, float* __restrict__ loss) {
+  double acc = 0.0;
+  for (int i = threadIdx.x; i < nblocks; i += kThreads) acc += partials[i];
+  __shared__ double red[kThreads / 32];
+  acc = warp_sum(acc);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    double v = threadIdx.x < kThreads / 32 ? red[threadIdx.x] : 0.0;
+    v = warp_sum(v);
+    if (threadIdx.x == 0) loss[0] = static_cast<float>(v * out_scale);
+  }
+}
+
+// ---------------------------------------------------------------- factor-gradient reduction
+// One thread per group: sums the dW epilogue's partial sums over contraction splits and
+// over the g/P column chunks of the group in a fixed order, then applies
+//   d_mu = -alpha0 k S_mu,  d_alpha = alpha0 S_alpha,  d_delta = Delta0 alpha k S_delta,
+// k = s / (2 tanh s).
+__global__ void __launch_bounds__(kThreads) grad_reduce_kernel(LayerDev L, StepScalars sc,
+                                                               const float* __restrict__ part, int32_t splits,
+                                                               int32_t P, float* __restrict__ g_dmu,
+                                                               float* __restrict__ g_dalpha,
+                                                               float* __restrict__ g_ddelta) {
+  const int64_t G = L.N * L.K / L.g;
+  const int64_t cpr = L.K / P;  // partial chunks per row
+  const int32_t cpg = L.g / P;  // partial chunks per group
+  const int64_t plane = L.N * cpr;
+  for (int64_t j = blockIdx.x * (int64_t)kThreads + threadIdx.x; j < G; j += (int64_t)gridDim.x * kThreads) {
+    const int64_t n = j / L.groups_per_row;
+    const int64_t c0 = (j % L.groups_per_row) * cpg;
+    float s3[3] = {0.f, 0.f, 0.f};
+    for (int32_t sp = 0; sp < splits; ++sp)
+#pragma unroll
+      for (int q = 0; q < 3; ++q) {
+        const float* p = part + (static_cast<int64_t>(sp) * 3 + q) * plane + n * cpr + c0;
+        for (int32_t c = 0; c < cpg; ++c) s3[q] += p[c];
+      }
+    const GroupConst gc = group_const(L, j);
+    const float k = sc.s * sc.inv_2tanh_s;
+    const bool live = gc.alpha != 0.0f;
+    g_dmu[j] = live ? -gc.alpha0 * k * s3[0] : 0.0f;
+    g_dalpha[j] = live ? gc.alpha0 * s3[1] : 0.0f;
+    g_ddelta[j] = live ? gc.delta0 * gc.alpha * k * s3[2] : 0.0f;
+  }
+}
+
+int grid_for(int64_t work, int64_t per_block) {
+  int64_t b = (work + per_block - 1) / per_block;
+  if (b < 1) b = 1;
+  if (b > 152 * 16) b = 152 * 16;
+  return static_cast<int>(b);
+}
+
+}  // namespace
+
+cudaError_t launch_group_stats(const LayerDev& L, int32_t w_dtype, int32_t thr_init, float* mu0, float* alpha0,
+                               float* delta0, cudaStream_t st) {
+  const int64_t G = L.N * L.K / L.g;
+  const int grid = grid_for(G, kThreads / 32);
+  if (w_dtype == 1)
+    group_stats_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(static_cast<const __nv_bfloat16*>(L.W), G, L.g,
+                                                                   thr_init, mu0, alpha0, delta0);
+  else
+    group_stats_kernel<float><<<grid, kThreads, 0, st>>>(static_cast<const float*>(L.W), G, L.g, thr_init, mu0,
+                                                         alpha0, delta0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_modulate_ternarize(const LayerDev& L, int32_t w_dtype, StepScalars sc, void* Wq, int8_t* T,
+                                      float* alpha, cudaStream_t st) {
+  if (w_dtype == 1) {
+    const int grid = grid_for(L.N * L.K / 8, kThreads);
+    modulate_bf16_kernel<<<grid, kThreads, 0, st>>>(L, sc, static_cast<uint16_t*>(Wq), T, alpha);
+  } else {
+    const int grid = grid_for(L.N * L.K, kThreads);
+    modulate_f32_kernel<<<grid, kThreads, 0, st>>>(L, sc, static_cast<float*>(Wq), T, alpha);
+  }
+  return cudaGetLastError();
+}
+
+int recon_loss_blocks(int64_t count) {
+  int64_t b = (count + 8LL * kThreads * 4 - 1) / (8LL * kThreads * 4);
+  if (b < 1) b = 1;
+  if (b > kLossMaxBlocks) b = kLossMaxBlocks;
+  return static_cast<int>(b);
+}
+
+cudaError_t launch_recon_loss(const void* Y, const void* Yr, int64_t count, int32_t dtype, int32_t reduction,
+                              float* loss_out, void* dY, double* partials, cudaStream_t st) {
+  const int nb = recon_loss_blocks(count);
+  const double inv = reduction == 0 ? 1.0 / static_cast<double>(count) : 1.0;
+  const float scale = static_cast<float>(2.0 * inv);
+  if (dtype == 1)
+    recon_loss_partial_kernel<__nv_bfloat16><<<nb, kThreads, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(Y), static_cast<const __nv_bfloat16*>(Yr), count, scale,
+        static_cast<__nv_bfloat16*>(dY), partials);
+  else
+    recon_loss_partial_kernel<float><<<nb, kThreads, 0, st>>>(static_cast<const float*>(Y),
+                                                              static_cast<const float*>(Yr), count, scale,
+                                                              static_cast<float*>(dY), partials);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  recon_loss_final_kernel<<<1, kThreads, 0, st>>>(partials, nb, inv, loss_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_hard_pack(const LayerDev& L, int32_t w_dtype, uint8_t* codes, float* alpha, cudaStream_t st) {
+  const int64_t n = L.N * L.K;
+  if (L.g % 16 == 0) {
+    const int grid = grid_for(n / 16, kThreads);
+    if (w_dtype == 1)
+      hard_pack_kernel<__nv_bfloat16, 16><<<grid, kThreads, 0, st>>>(L, codes, alpha);
+    else
+      hard_pack_kernel<float, 16><<<grid, kThreads, 0, st>>>(L, codes, alpha);
+  } else {
+    const int grid = grid_for(n / 4, kThreads);
+    if (w_dtype == 1)
+      hard_pack_kernel<__nv_bfloat16, 4><<<grid, kThreads, 0, st>>>(L, codes, alpha);
+    else
+      hard_pack_kernel<float, 4><<<grid, kThreads, 0, st>>>(L, codes, alpha);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_grad_reduce(const LayerDev& L, StepScalars sc, const float* partials, int32_t splits, int32_t P,
+                               float* g_dmu, float* g_dalpha, float* g_ddelta, cudaStream_t st) {
+  const int64_t G = L.N * L.K / L.g;
+  grad_reduce_kernel<<<grid_for(G, kThreads), kThreads, 0, st>>>(L, sc, partials, splits, P, g_dmu, g_dalpha,
+                                                                 g_ddelta);
+  return cudaGetLastError();
+}
+
+}  // namespace catq

@@ -1,0 +1,55 @@
+// launch.h — host-side launchers shared between the C-ABI layer (api.cu) and the kernel
+// translation units.  Arguments are validated by api.cu before any of these is called.
+#pragma once
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+#include "catq_math.cuh"
+
+namespace catq {
+
+struct StepScalars {
+  int32_t phase;
+  float s;
+  float inv_2tanh_s;  // 1 / (2 tanh s); 0 when unused
+};
+
+// elementwise.cu
+cudaError_t launch_group_stats(const LayerDev& L, int32_t w_dtype, int32_t thr_init, float* mu0, float* alpha0,
+                               float* delta0, cudaStream_t st);
+cudaError_t launch_modulate_ternarize(const LayerDev& L, int32_t w_dtype, StepScalars sc, void* Wq, int8_t* T,
+                                      float* alpha, cudaStream_t st);
+int recon_loss_blocks(int64_t count);
+cudaError_t launch_recon_loss(const void* Y, const void* Yr, int64_t count, int32_t dtype, int32_t reduction,
+                              float* loss_out, void* dY, double* partials, cudaStream_t st);
+cudaError_t launch_hard_pack(const LayerDev& L, int32_t w_dtype, uint8_t* codes, float* alpha, cudaStream_t st);
+// Sums the partial group sums of the dW epilogue ([splits][3][N][K/P]) into the factor
+// gradients and applies the per-group scales.
+cudaError_t launch_grad_reduce(const LayerDev& L, StepScalars sc, const float* partials, int32_t splits, int32_t P,
+                               float* g_dmu, float* g_dalpha, float* g_ddelta, cudaStream_t st);
+
+// simt_f32.cu (fp32 CUDA-core path)
+cudaError_t launch_simt_fwd(const LayerDev& L, StepScalars sc, const float* X, int64_t M, float* Y, cudaStream_t st);
+cudaError_t launch_simt_dx(const LayerDev& L, StepScalars sc, const float* dY, int64_t M, float* dX, cudaStream_t st);
+cudaError_t launch_simt_dw(const LayerDev& L, StepScalars sc, const float* X, const float* dY, int64_t M,
+                           float* partials, cudaStream_t st);
+constexpr int32_t kSimtTile = 64;
+
+// tc_gemm.cu (bf16 tensor-core path)
+struct TcPlan {
+  int32_t dw_cg;      // CTA group of the dW kernel (1 or 2)
+  int32_t dw_splits;  // contraction splits of the dW kernel
+  int32_t dw_P;       // partial-sum chunk width (columns)
+};
+TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count);
+cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st);
+cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int64_t M, void* dX, cudaStream_t st);
+cudaError_t launch_tc_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M,
+                         const TcPlan& plan, float* partials, cudaStream_t st);
+// Status word latched by device-side bounded waits (0 = none); read-and-clear.
+cudaError_t read_and_clear_device_status(int32_t* out);
+bool tensor_map_encoder_available();
+
+}  // namespace catq

@@ -1,0 +1,708 @@
+// tc_gemm.cu — bf16 tensor-core contractions of the soft-ternary linear on sm_100-class
+// GPUs (tcgen05 MMA with TMEM accumulators, TMA-fed, warp-specialised, persistent).
+//
+// fused_gemm_kernel  C[M, ncols] = A[M, depth] * Wq-operand, with the Eq. 3/5/6 weight
+//                    (modulation, transition function, scale alpha) computed by producer
+//                    warps on the raw W tile while it sits in shared memory, in place, in
+//                    the 128-byte-swizzled layout the MMA reads.  Wq never reaches HBM.
+//                      forward:  A = X  [M, K],  operand = Wq   (K-major), C = Y  [M, N]
+//                      dX:       A = dY [M, N],  operand = Wq   (MN-major), C = dX [M, K]
+//                    Two M-tiles share each produced operand tile (two accumulators).
+// dw_kernel          G = dY^T X accumulated in TMEM (both operands MN-major, straight from
+//                    TMA); the epilogue applies the chain rule of Eq. 3/5/6 per element
+//                    and reduces each row's columns into per-group partial sums.  G is never
+//                    written to memory.
+//
+// CG = 1: one CTA per tile (MMA M = 128).  CG = 2: a CTA pair (cluster of 2) computes one
+// tile with tcgen05 cta_group::2 (MMA M = 256), each CTA holding half of the operand
+// columns; only the even CTA issues MMAs.
+//
+// Every mbarrier wait is bounded (ptx_sm100.cuh); on expiry the launch latches
+// CATQ_ERR_TIMEOUT, every role leaves its loop, in-flight copies and MMAs are drained
+// with bounded waits, and TMEM is freed before the kernel returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <atomic>
+#include <mutex>
+#include <numeric>
+
+#include "launch.h"
+#include "ptx_sm100.cuh"
+
+namespace catq {
+
+__device__ uint32_t g_abort_word;
+__device__ int32_t g_status_word;
+
+namespace {
+
+constexpr int BK = 64;    // contraction elements per pipeline stage (one 128-byte row)
+constexpr int BN = 256;   // MMA N
+constexpr int NACC = 2;   // accumulators sharing one produced operand tile (fused kernel)
+constexpr uint32_t kTmemCols = 512;
+constexpr uint64_t kWaitTimeoutNs = 4000000000ull;
+constexpr uint64_t kDrainTimeoutNs = 200000000ull;
+
+template <int CG>
+struct FusedCfg {
+  static constexpr int kRowsPerAcc = 128 * CG;          // MMA M
+  static constexpr int kTileRows = kRowsPerAcc * NACC;  // rows of C per tile
+  static constexpr int kBRows = BN / CG;                // 128-byte operand rows per CTA per stage
+  static constexpr int kABytes = NACC * 128 * BK * 2;   // this CTA's A rows
+  static constexpr int kBBytes = kBRows * BK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStages = CG == 1 ? 3 : 4;
+  static constexpr int kEpiWarps = 4;
+  static constexpr int kProdWarps = 8;
+  static constexpr int kThreads = 32 * (kEpiWarps + 2 + kProdWarps);
+  static constexpr int kBarBytes = 8 * (3 * kStages + 3) + 16;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + kBarBytes;
+};
+
+template <int CG>
+struct DwCfg {
+  static constexpr int kRowsPerCta = 128;    // G rows (n) per CTA
+  static constexpr int kTileRows = 128 * CG; // MMA M
+  static constexpr int kBCols = BN / CG;     // G columns (k) whose X slice this CTA loads
+  static constexpr int kABytes = 128 * BK * 2;
+  static constexpr int kBBytes = kBCols * BK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStages = CG == 1 ? 4 : 6;
+  static constexpr int kEpiWarps = 8;        // two warps per TMEM lane quarter (column halves)
+  static constexpr int kThreads = 32 * (kEpiWarps + 2);
+  static constexpr int kBarBytes = 8 * (2 * kStages + 5) + 16;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + kBarBytes;
+};
+
+struct FusedArgs {
+  LayerDev L;
+  StepScalars sc;
+  uint16_t* C;      // bf16 [M, ncols]
+  int64_t M;        // rows of A and C
+  int64_t ncols;    // columns of C
+  int32_t num_m_tiles, num_n_tiles, num_k_blocks;
+  WaitCtl wc;
+};
+
+struct DwArgs {
+  LayerDev L;
+  StepScalars sc;
+  float* part;      // [splits][3][N][K/P]
+  int64_t M;
+  int32_t splits, P, kb_per_split, kb_total;
+  int32_t num_n_tiles, num_k_tiles;
+  WaitCtl wc;
+};
+
+// Wait that ignores the abort flag (used to drain work already issued).
+__device__ __forceinline__ bool mbar_wait_drain(uint32_t bar, uint32_t parity) {
+  const uint64_t t0 = globaltimer_ns();
+  while (!mbar_try_wait(bar, parity))
+    if (globaltimer_ns() - t0 > kDrainTimeoutNs) return false;
+  return true;
+}
+
+__device__ __forceinline__ void store_bf16x32(uint16_t* dst, const uint32_t (&r)[32], int64_t cols_left) {
+#pragma unroll
+  for (int p = 0; p < 4; ++p) {
+    if (8 * p >= cols_left) break;
+    uint4 v;
+    v.x = pack_bf16x2(__uint_as_float(r[8 * p + 0]), __uint_as_float(r[8 * p + 1]));
+    v.y = pack_bf16x2(__uint_as_float(r[8 * p + 2]), __uint_as_float(r[8 * p + 3]));
+    v.z = pack_bf16x2(__uint_as_float(r[8 * p + 4]), __uint_as_float(r[8 * p + 5]));
+    v.w = pack_bf16x2(__uint_as_float(r[8 * p + 6]), __uint_as_float(r[8 * p + 7]));
+    *reinterpret_cast<uint4*>(dst + 8 * p) = v;
+  }
+}
+
+// ============================================================================ fused kernel
+
+template <int CG, bool B_MN>
+__global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
+    fused_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                      const FusedArgs args) {
+  using Cfg = FusedCfg<CG>;
+  constexpr int S = Cfg::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_addr = smem_u32(smem_raw);
+  const uint32_t base = (raw_addr + 1023u) & ~1023u;
+  uint8_t* base_ptr = smem_raw + (base - raw_addr);
+  const uint32_t bars = base + S * Cfg::kStageBytes;
+  const uint32_t tmem_full_bar = bars + 8 * (3 * S);
+  const uint32_t tmem_empty_bar = tmem_full_bar + 8;
+  const uint32_t final_bar = tmem_full_bar + 16;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base_ptr + (bars - base) + 8 * (3 * S + 3));
+  auto full_raw = [&](int s) { return bars + 8u * s; };
+  auto full = [&](int s) { return bars + 8u * (S + s); };
+  auto empty = [&](int s) { return bars + 8u * (2 * S + s); };
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t cta = CG == 2 ? cluster_ctarank() : 0u;
+  const uint32_t cluster = CG == 2 ? cluster_id_x() : blockIdx.x;
+  const uint32_t nclusters = CG == 2 ? num_clusters_x() : gridDim.x;
+  const WaitCtl& wc = args.wc;
+  const int num_tiles = args.num_m_tiles * args.num_n_tiles;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(full_raw(s), 1);
+      mbar_init(full(s), Cfg::kProdWarps * CG);
+      mbar_init(empty(s), 1);
+    }
+    mbar_init(tmem_full_bar, 1);
+    mbar_init(tmem_empty_bar, Cfg::kEpiWarps * CG);
+    mbar_init(final_bar, 1);
+    fence_mbar_init_cluster();
+  }
+  if (warp == Cfg::kEpiWarps + 1) tmem_alloc<CG>(smem_u32(tmem_slot), kTmemCols);
+  if (warp == Cfg::kEpiWarps && lane == 0) {
+    prefetch_tmap(&tmA);
+    prefetch_tmap(&tmB);
+  }
+  tc_fence_before();
+  if constexpr (CG == 2) cluster_sync_all(); else __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  // Barriers the whole pair signals live in the even CTA.
+  const uint32_t leader_full0 = CG == 2 ? mapa_shared(full(0), 0) : full(0);
+  const uint32_t leader_tmem_empty = CG == 2 ? mapa_shared(tmem_empty_bar, 0) : tmem_empty_bar;
+
+  if (warp == Cfg::kEpiWarps) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      uint32_t stage = 0, phase = 0;
+      uint32_t issued_mask = 0, issued_phase = 0;
+      bool ok = true;
+      for (int t = cluster; ok && t < num_tiles; t += nclusters) {
+        const int m_blk = t % args.num_m_tiles, n_blk = t / args.num_m_tiles;
+        const int32_t m0 = m_blk * Cfg::kTileRows, n0 = n_blk * BN;
+        for (int kb = 0; kb < args.num_k_blocks; ++kb) {
+          if (!mbar_wait(empty(stage), phase ^ 1u, wc)) { ok = false; break; }
+          const uint32_t sa = base + stage * Cfg::kStageBytes;
+          mbar_arrive_expect_tx(full_raw(stage), Cfg::kStageBytes);
+#pragma unroll
+          for (int acc = 0; acc < NACC; ++acc)
+            tma_load_2d(sa + acc * (128 * BK * 2), &tmA, full_raw(stage), kb * BK,
+                        m0 + acc * Cfg::kRowsPerAcc + cta * 128);
+          const uint32_t sb = sa + Cfg::kABytes;
+          if constexpr (!B_MN) {
+            tma_load_2d(sb, &tmB, full_raw(stage), kb * BK, n0 + cta * Cfg::kBRows);
+          } else {
+#pragma unroll
+            for (int b = 0; b < Cfg::kBRows / 64; ++b)
+              tma_load_2d(sb + b * 8192, &tmB, full_raw(stage), n0 + cta * Cfg::kBRows + 64 * b, kb * BK);
+          }
+          issued_mask |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == S) { stage = 0; phase ^= 1u; }
+        }
+      }
+      // Drain: every issued copy must land before the CTA may exit.
+      for (int s = 0; s < S; ++s)
+        if (issued_mask & (1u << s)) mbar_wait_drain(full_raw(s), (issued_phase >> s) & 1u);
+    }
+  } else if (warp == Cfg::kEpiWarps + 1) {
+    // ------------------------------------------------------------ MMA issuer (even CTA)
+    if (cta == 0 && lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(Cfg::kRowsPerAcc, BN, false, B_MN);
+      uint32_t stage = 0, phase = 0, it = 0;
+      bool ok = true;
+      for (int t = cluster; ok && t < num_tiles; t += nclusters, ++it) {
+        if (!mbar_wait(tmem_empty_bar, (it & 1u) ^ 1u, wc)) break;
+        tc_fence_after();
+        for (int kb = 0; kb < args.num_k_blocks; ++kb) {
+          if (!mbar_wait(full(stage), phase, wc)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t sa = base + stage * Cfg::kStageBytes;
+          const uint32_t sb = sa + Cfg::kABytes;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            const uint64_t bdesc = B_MN ? smem_desc_sw128(sb + kk * 2048, 8192, 1024)
+                                        : smem_desc_sw128(sb + kk * 32, 16, 1024);
+#pragma unroll
+            for (int acc = 0; acc < NACC; ++acc) {
+              const uint64_t adesc = smem_desc_sw128(sa + acc * (128 * BK * 2) + kk * 32, 16, 1024);
+              umma_bf16<CG>(tmem_base + acc * BN, adesc, bdesc, idesc, (kb | kk) != 0 ? 1u : 0u);
+            }
+          }
+          umma_commit<CG>(empty(stage));
+          if (++stage == S) { stage = 0; phase ^= 1u; }
+        }
+        if (ok) umma_commit<CG>(tmem_full_bar);
+      }
+      umma_commit<CG>(final_bar);
+      mbar_wait_drain(final_bar, 0);
+    }
+  } else if (warp < Cfg::kEpiWarps) {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp;  // TMEM lane quarter
+    uint32_t it = 0;
+    for (int t = cluster; t < num_tiles; t += nclusters, ++it) {
+      const int m_blk = t % args.num_m_tiles, n_blk = t / args.num_m_tiles;
+      if (!mbar_wait(tmem_full_bar, it & 1u, wc)) break;
+      tc_fence_after();
+#pragma unroll 1
+      for (int acc = 0; acc < NACC; ++acc) {
+        const int64_t row = (int64_t)m_blk * Cfg::kTileRows + acc * Cfg::kRowsPerAcc + cta * 128 + q * 32 + lane;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN + c * 32, r);
+          tmem_ld_wait();
+          const int64_t col = (int64_t)n_blk * BN + c * 32;
+          if (row < args.M && col < args.ncols) store_bf16x32(args.C + row * args.ncols + col, r, args.ncols - col);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(leader_tmem_empty);
+    }
+  } else {
+    // ------------------------------------------------------------ operand producers
+    const int tt = threadIdx.x - 32 * (Cfg::kEpiWarps + 2);
+    const int row = tt / CG;                 // 128-byte smem row of the operand tile
+    const int c_begin = (tt % CG) * (8 / CG);
+    const LayerDev& L = args.L;
+    const int32_t phase_t = args.sc.phase;
+    int64_t cached_j = -1;
+    ProducerConst pc{};
+    uint32_t stage = 0, phase = 0;
+    bool ok = true;
+    for (int t = cluster; ok && t < num_tiles; t += nclusters) {
+      const int n_blk = t / args.num_m_tiles;
+      for (int kb = 0; kb < args.num_k_blocks; ++kb) {
+        int64_t n, kc;
+        if constexpr (!B_MN) {
+          n = (int64_t)n_blk * BN + cta * Cfg::kBRows + row;
+          kc = (int64_t)kb * BK;
+        } else {
+          n = (int64_t)kb * BK + (row & 63);
+          kc = (int64_t)n_blk * BN + cta * Cfg::kBRows + 64 * (row >> 6);
+        }
+        const bool live = phase_t != PHASE_TEACHER && n < L.N && kc < L.K;
+        if (live) {
+          const int64_t j = n * L.groups_per_row + kc / L.g;
+          if (j != cached_j) {
+            pc = producer_const(group_const(L, j), args.sc.s, args.sc.inv_2tanh_s, phase_t);
+            cached_j = j;
+          }
+        }
+        if (!mbar_wait(full_raw(stage), phase, wc)) { ok = false; break; }
+        if (live) {
+          uint8_t* rowp = base_ptr + stage * Cfg::kStageBytes + Cfg::kABytes + row * 128;
+#pragma unroll
+          for (int i = 0; i < 8 / CG; ++i) {
+            const int phys = (c_begin + i) ^ (row & 7);
+            uint4* p = reinterpret_cast<uint4*>(rowp + phys * 16);
+            *p = transform_chunk_bf16(*p, pc, phase_t);
+          }
+          fence_proxy_async_smem();
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(leader_full0 + 8u * stage);
+        if (++stage == S) { stage = 0; phase ^= 1u; }
+      }
+    }
+  }
+
+  tc_fence_before();
+  if constexpr (CG == 2) cluster_sync_all(); else __syncthreads();
+  if (warp == Cfg::kEpiWarps + 1) {
+    tc_fence_after();
+    tmem_dealloc<CG>(tmem_base, kTmemCols);
+  }
+}
+
+// ============================================================================ dW kernel
+
+template <int CG>
+__global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
+    dw_kernel(const __grid_constant__ CUtensorMap tmDY, const __grid_constant__ CUtensorMap tmX, const DwArgs args) {
+  using Cfg = DwCfg<CG>;
+  constexpr int S = Cfg::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_addr = smem_u32(smem_raw);
+  const uint32_t base = (raw_addr + 1023u) & ~1023u;
+  uint8_t* base_ptr = smem_raw + (base - raw_addr);
+  const uint32_t bars = base + S * Cfg::kStageBytes;
+  auto full = [&](int s) { return bars + 8u * s; };
+  auto empty = [&](int s) { return bars + 8u * (S + s); };
+  const uint32_t tmem_full0 = bars + 8u * (2 * S);      // [2]
+  const uint32_t tmem_empty0 = tmem_full0 + 16;         // [2]
+  const uint32_t final_bar = tmem_full0 + 32;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base_ptr + (bars - base) + 8 * (2 * S + 5));
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t cta = CG == 2 ? cluster_ctarank() : 0u;
+  const uint32_t cluster = CG == 2 ? cluster_id_x() : blockIdx.x;
+  const uint32_t nclusters = CG == 2 ? num_clusters_x() : gridDim.x;
+  const WaitCtl& wc = args.wc;
+  const int tiles_per_split = args.num_n_tiles * args.num_k_tiles;
+  const int num_tiles = tiles_per_split * args.splits;
+  constexpr int kTma = Cfg::kEpiWarps, kMma = Cfg::kEpiWarps + 1;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(full(s), 1);
+      mbar_init(empty(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(tmem_full0 + 8u * b, 1);
+      mbar_init(tmem_empty0 + 8u * b, Cfg::kEpiWarps * CG);
+    }
+    mbar_init(final_bar, 1);
+    fence_mbar_init_cluster();
+  }
+  if (warp == kMma) tmem_alloc<CG>(smem_u32(tmem_slot), kTmemCols);
+  if (warp == kTma && lane == 0) {
+    prefetch_tmap(&tmDY);
+    prefetch_tmap(&tmX);
+  }
+  tc_fence_before();
+  if constexpr (CG == 2) cluster_sync_all(); else __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const uint32_t leader_full0 = CG == 2 ? mapa_shared(full(0), 0) : full(0);
+  const uint32_t leader_tmem_empty0 = CG == 2 ? mapa_shared(tmem_empty0, 0) : tmem_empty0;
+
+  if (warp == kTma) {
+    if (lane == 0) {
+      uint32_t stage = 0, phase = 0, issued_mask = 0, issued_phase = 0;
+      bool ok = true;
+      for (int t = cluster; ok && t < num_tiles; t += nclusters) {
+        const int split = t / tiles_per_split, r = t % tiles_per_split;
+        const int k_blk = r % args.num_k_tiles, n_blk = r / args.num_k_tiles;
+        const int kb0 = split * args.kb_per_split;
+        const int kb1 = min(kb0 + args.kb_per_split, args.kb_total);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(empty(stage), phase ^ 1u, wc)) { ok = false; break; }
+          const uint32_t sa = base + stage * Cfg::kStageBytes, sb = sa + Cfg::kABytes;
+          const int32_t m = kb * BK;
+          if (cta == 0) mbar_arrive_expect_tx(full(stage), Cfg::kStageBytes * CG);
+          const uint32_t fb = leader_full0 + 8u * stage;
+#pragma unroll
+          for (int b = 0; b < 2; ++b) {
+            const int32_t n = n_blk * Cfg::kTileRows + cta * 128 + 64 * b;
+            if constexpr (CG == 1) tma_load_2d(sa + b * 8192, &tmDY, fb, n, m);
+            else tma_load_2d_pair(sa + b * 8192, &tmDY, fb, n, m);
+          }
+#pragma unroll
+          for (int b = 0; b < Cfg::kBCols / 64; ++b) {
+            const int32_t k = k_blk * BN + cta * Cfg::kBCols + 64 * b;
+            if constexpr (CG == 1) tma_load_2d(sb + b * 8192, &tmX, fb, k, m);
+            else tma_load_2d_pair(sb + b * 8192, &tmX, fb, k, m);
+          }
+          issued_mask |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == S) { stage = 0; phase ^= 1u; }
+        }
+      }
+      // Drain (the even CTA's barriers observe both CTAs' copies).
+      if (cta == 0)
+        for (int s = 0; s < S; ++s)
+          if (issued_mask & (1u << s)) mbar_wait_drain(full(s), (issued_phase >> s) & 1u);
+    }
+  } else if (warp == kMma) {
+    if (cta == 0 && lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(Cfg::kTileRows, BN, true, true);
+      uint32_t stage = 0, phase = 0, it = 0;
+      bool ok = true;
+      for (int t = cluster; ok && t < num_tiles; t += nclusters, ++it) {
+        const int split = t / tiles_per_split;
+        const int kb0 = split * args.kb_per_split;
+        const int kb1 = min(kb0 + args.kb_per_split, args.kb_total);
+        const uint32_t buf = it & 1u;
+        if (!mbar_wait(tmem_empty0 + 8u * buf, ((it >> 1) & 1u) ^ 1u, wc)) break;
+        tc_fence_after();
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(full(stage), phase, wc)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t sa = base + stage * Cfg::kStageBytes, sb = sa + Cfg::kABytes;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            const uint64_t adesc = smem_desc_sw128(sa + kk * 2048, 8192, 1024);
+            const uint64_t bdesc = smem_desc_sw128(sb + kk * 2048, 8192, 1024);
+            umma_bf16<CG>(tmem_base + buf * BN, adesc, bdesc, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+          }
+          umma_commit<CG>(empty(stage));
+          if (++stage == S) { stage = 0; phase ^= 1u; }
+        }
+        if (ok) umma_commit<CG>(tmem_full0 + 8u * buf);
+      }
+      umma_commit<CG>(final_bar);
+      mbar_wait_drain(final_bar, 0);
+    }
+  } else {
+    // ------------------------------------------------------------ factor-gradient epilogue
+    const int q = warp & 3;        // TMEM lane quarter
+    const int half = warp >> 2;    // column half of the tile
+    const LayerDev& L = args.L;
+    const int64_t cpr = L.K / args.P;
+    const int64_t plane = L.N * cpr;
+    const uint16_t* W = static_cast<const uint16_t*>(L.W);
+    uint32_t it = 0;
+    for (int t = cluster; t < num_tiles; t += nclusters, ++it) {
+      const int split = t / tiles_per_split, r = t % tiles_per_split;
+      const int k_blk = r % args.num_k_tiles, n_blk = r / args.num_k_tiles;
+      const uint32_t buf = it & 1u;
+      if (!mbar_wait(tmem_full0 + 8u * buf, (it >> 1) & 1u, wc)) break;
+      tc_fence_after();
+      const int64_t n = (int64_t)n_blk * Cfg::kTileRows + cta * 128 + q * 32 + lane;
+      const bool row_ok = n < L.N;
+      float* out = args.part + (int64_t)split * 3 * plane;
+      int64_t cur_j = -1;
+      GroupConst gc{};
+      GradSums acc{0.f, 0.f, 0.f};
+#pragma unroll 1
+      for (int c = 0; c < (BN / 2) / 32; ++c) {
+        const int col = half * (BN / 2) + c * 32;
+        uint32_t rg[32];
+        tmem_ld32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + buf * BN + col, rg);
+        tmem_ld_wait();
+        const int64_t k = (int64_t)k_blk * BN + col;
+        if (row_ok && k < L.K) {
+          const int64_t j = n * L.groups_per_row + k / L.g;
+          if (j != cur_j) {
+            gc = group_const(L, j);
+            cur_j = j;
+          }
+          const uint4* wp = reinterpret_cast<const uint4*>(W + n * L.K + k);
+          if (gc.alpha != 0.0f) {
+#pragma unroll
+            for (int v = 0; v < 4; ++v) {
+              const uint4 wv = __ldg(wp + v);
+              const uint32_t w4[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                grad_element(__uint_as_float(rg[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), gc, args.sc.s,
+                             args.sc.inv_2tanh_s, args.sc.phase, acc);
+                grad_element(__uint_as_float(rg[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), gc, args.sc.s,
+                             args.sc.inv_2tanh_s, args.sc.phase, acc);
+              }
+            }
+          }
+          if (((k + 32) % args.P) == 0 || k + 32 >= L.K) {
+            const int64_t idx = n * cpr + k / args.P;
+            out[idx] = acc.smu;
+            out[plane + idx] = acc.salpha;
+            out[2 * plane + idx] = acc.sdelta;
+            acc = GradSums{0.f, 0.f, 0.f};
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(leader_tmem_empty0 + 8u * buf);
+    }
+  }
+
+  tc_fence_before();
+  if constexpr (CG == 2) cluster_sync_all(); else __syncthreads();
+  if (warp == kMma) {
+    tc_fence_after();
+    tmem_dealloc<CG>(tmem_base, kTmemCols);
+  }
+}
+
+// ============================================================================ host side
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+std::atomic<uint32_t> g_epoch{1};
+
+void init_encoder() {
+  std::call_once(g_encode_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+}
+
+// bf16 row-major [outer, inner] tensor, 128-byte swizzled boxes of box_inner x box_outer.
+bool make_tmap(CUtensorMap* m, const void* ptr, uint64_t inner, uint64_t outer, uint32_t box_inner,
+               uint32_t box_outer) {
+  init_encoder();
+  if (!g_encode) return false;
+  const cuuint64_t dims[2] = {inner, outer};
+  const cuuint64_t strides[1] = {inner * 2};
+  const cuuint32_t box[2] = {box_inner, box_outer};
+  const cuuint32_t estr[2] = {1, 1};
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+struct DeviceInfo {
+  int sm_count = 0;
+  uint32_t* abort_word = nullptr;
+  int32_t* status_word = nullptr;
+  bool ok = false;
+};
+
+DeviceInfo& device_info() {
+  static std::mutex mu;
+  static DeviceInfo infos[64];
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::lock_guard<std::mutex> lock(mu);
+  DeviceInfo& d = infos[dev & 63];
+  if (!d.ok) {
+    cudaDeviceGetAttribute(&d.sm_count, cudaDevAttrMultiProcessorCount, dev);
+    void* a = nullptr;
+    void* s = nullptr;
+    if (cudaGetSymbolAddress(&a, g_abort_word) == cudaSuccess &&
+        cudaGetSymbolAddress(&s, g_status_word) == cudaSuccess) {
+      d.abort_word = static_cast<uint32_t*>(a);
+      d.status_word = static_cast<int32_t*>(s);
+      d.ok = true;
+    }
+  }
+  return d;
+}
+
+WaitCtl make_wait_ctl(const DeviceInfo& d) {
+  WaitCtl w;
+  w.abort_word = d.abort_word;
+  w.status_word = d.status_word;
+  uint32_t e = g_epoch.fetch_add(1);
+  if (e == 0) e = g_epoch.fetch_add(1);
+  w.epoch = e;
+  w.timeout_ns = kWaitTimeoutNs;
+  return w;
+}
+
+template <typename Kern>
+cudaError_t launch_persistent(Kern kern, int cg, int grid_ctas, int threads, int smem, cudaStream_t st,
+                              const CUtensorMap& a, const CUtensorMap& b, const void* args_ptr) {
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(grid_ctas);
+  cfg.blockDim = dim3(threads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cg;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  void* params[3] = {const_cast<CUtensorMap*>(&a), const_cast<CUtensorMap*>(&b), const_cast<void*>(args_ptr)};
+  return cudaLaunchKernelExC(&cfg, reinterpret_cast<const void*>(kern), params);
+}
+
+int fused_cg_for(int64_t M) {
+  // Two-CTA tiles (512 rows) pay off once M fills them.
+  return M >= 512 ? 2 : 1;
+}
+
+template <int CG, bool B_MN>
+cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t M, int64_t depth, void* C,
+                      int64_t ncols, cudaStream_t st) {
+  using Cfg = FusedCfg<CG>;
+  DeviceInfo& d = device_info();
+  if (!d.ok) return cudaErrorInvalidDevice;
+  CUtensorMap ta, tb;
+  if (!make_tmap(&ta, A, depth, M, BK, 128)) return cudaErrorInvalidValue;
+  if constexpr (!B_MN) {
+    if (!make_tmap(&tb, L.W, L.K, L.N, BK, Cfg::kBRows)) return cudaErrorInvalidValue;
+  } else {
+    if (!make_tmap(&tb, L.W, L.K, L.N, 64, BK)) return cudaErrorInvalidValue;
+  }
+  FusedArgs args;
+  args.L = L;
+  args.sc = sc;
+  args.C = static_cast<uint16_t*>(C);
+  args.M = M;
+  args.ncols = ncols;
+  args.num_m_tiles = static_cast<int32_t>((M + Cfg::kTileRows - 1) / Cfg::kTileRows);
+  args.num_n_tiles = static_cast<int32_t>((ncols + BN - 1) / BN);
+  args.num_k_blocks = static_cast<int32_t>((depth + BK - 1) / BK);
+  args.wc = make_wait_ctl(d);
+  const int tiles = args.num_m_tiles * args.num_n_tiles;
+  const int clusters = std::min(tiles, d.sm_count / CG);
+  return launch_persistent(fused_gemm_kernel<CG, B_MN>, CG, clusters * CG, Cfg::kThreads, Cfg::kSmemBytes, st, ta,
+                           tb, &args);
+}
+
+template <int CG>
+cudaError_t run_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M, const TcPlan& plan,
+                   float* part, cudaStream_t st) {
+  using Cfg = DwCfg<CG>;
+  DeviceInfo& d = device_info();
+  if (!d.ok) return cudaErrorInvalidDevice;
+  CUtensorMap tdy, tx;
+  if (!make_tmap(&tdy, dY, L.N, M, 64, BK)) return cudaErrorInvalidValue;
+  if (!make_tmap(&tx, X, L.K, M, 64, BK)) return cudaErrorInvalidValue;
+  DwArgs args;
+  args.L = L;
+  args.sc = sc;
+  args.part = part;
+  args.M = M;
+  args.splits = plan.dw_splits;
+  args.P = plan.dw_P;
+  args.kb_total = static_cast<int32_t>((M + BK - 1) / BK);
+  args.kb_per_split = (args.kb_total + plan.dw_splits - 1) / plan.dw_splits;
+  args.num_n_tiles = static_cast<int32_t>((L.N + Cfg::kTileRows - 1) / Cfg::kTileRows);
+  args.num_k_tiles = static_cast<int32_t>((L.K + BN - 1) / BN);
+  args.wc = make_wait_ctl(d);
+  const int tiles = args.num_n_tiles * args.num_k_tiles * args.splits;
+  const int clusters = std::min(tiles, d.sm_count / CG);
+  return launch_persistent(dw_kernel<CG>, CG, clusters * CG, Cfg::kThreads, Cfg::kSmemBytes, st, tdy, tx, &args);
+}
+
+}  // namespace
+
+bool tensor_map_encoder_available() {
+  init_encoder();
+  return g_encode != nullptr;
+}
+
+TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count) {
+  TcPlan p;
+  p.dw_cg = L.N >= 256 ? 2 : 1;
+  const int64_t rows = 128 * p.dw_cg;
+  const int64_t tiles = ((L.N + rows - 1) / rows) * ((L.K + BN - 1) / BN);
+  const int64_t clusters = std::max(1, sm_count / p.dw_cg);
+  const int64_t kb_total = std::max<int64_t>(1, (M + BK - 1) / BK);
+  int64_t splits = 1;
+  if (tiles < clusters) splits = std::min<int64_t>(clusters / tiles, std::max<int64_t>(1, kb_total / 8));
+  const int64_t per = (kb_total + splits - 1) / splits;
+  splits = (kb_total + per - 1) / per;
+  p.dw_splits = static_cast<int32_t>(std::max<int64_t>(1, splits));
+  p.dw_P = std::gcd(L.g, 128);
+  return p;
+}
+
+cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st) {
+  if (fused_cg_for(M) == 2) return run_fused<2, false>(L, sc, X, M, L.K, Y, L.N, st);
+  return run_fused<1, false>(L, sc, X, M, L.K, Y, L.N, st);
+}
+
+cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int64_t M, void* dX, cudaStream_t st) {
+  if (fused_cg_for(M) == 2) return run_fused<2, true>(L, sc, dY, M, L.N, dX, L.K, st);
+  return run_fused<1, true>(L, sc, dY, M, L.N, dX, L.K, st);
+}
+
+cudaError_t launch_tc_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M,
+                         const TcPlan& plan, float* partials, cudaStream_t st) {
+  if (plan.dw_cg == 2) return run_dw<2>(L, sc, X, dY, M, plan, partials, st);
+  return run_dw<1>(L, sc, X, dY, M, plan, partials, st);
+}
+
+cudaError_t read_and_clear_device_status(int32_t* out) {
+  int32_t v = 0;
+  cudaError_t e = cudaMemcpyFromSymbol(&v, g_status_word, sizeof(v));
+  if (e != cudaSuccess) return e;
+  const int32_t zero = 0;
+  e = cudaMemcpyToSymbol(g_status_word, &zero, sizeof(zero));
+  *out = v;
+  return e;
+}
+
+}  // namespace catq

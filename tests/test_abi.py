@@ -1,0 +1,86 @@
+"""The C-ABI library without a GPU: it loads, exports every function include/catq.h
+declares, and rejects bad arguments on the host before anything reaches a device."""
+import ctypes
+import os
+
+import pytest
+
+from paper_2606_26650_gb300 import catq as C
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(C.LIB_PATH):
+        import __graft_entry__
+        __graft_entry__.build()
+    return C.lib()
+
+
+def test_exports_every_declared_symbol(lib):
+    names = C.header_functions()
+    assert len(names) >= 11
+    missing = [n for n in names if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_status_strings_and_version(lib):
+    assert lib.catq_abi_version() == 1
+    for code, name in C.STATUS.items():
+        assert lib.catq_status_string(code).decode() == name
+    assert lib.catq_status_string(99).decode() == "CATQ_ERR_UNKNOWN"
+
+
+def _layer(N=64, K=256, g=128, dtype=C.BF16, W=16, stats=32):
+    """A layer struct with fake (never dereferenced) device addresses."""
+    return C.catq_layer(N, K, g, dtype, W, stats, stats + 1024, stats + 2048, stats + 4096, stats + 8192,
+                        stats + 16384)
+
+
+def _stats(lib, layer, thr=0):
+    return lib.catq_group_stats(ctypes.byref(layer), thr, None)
+
+
+def test_layer_validation(lib):
+    assert lib.catq_group_stats(None, 0, None) == 1
+    assert _stats(lib, _layer(W=0)) == 1                     # null W
+    assert _stats(lib, _layer(K=250)) == 2                   # g does not divide K
+    assert _stats(lib, _layer(g=32)) == 2                    # bf16 needs g % 64 == 0
+    assert _stats(lib, _layer(N=60)) == 2                    # bf16 needs N % 8 == 0
+    assert _stats(lib, _layer(g=48, K=96, dtype=C.F32)) == 2  # fp32 g not supported
+    assert _stats(lib, _layer(dtype=7)) == 3                 # unknown dtype
+    assert _stats(lib, _layer(W=24)) == 4                    # misaligned W
+    assert _stats(lib, _layer(), thr=5) == 1                 # bad threshold rule
+    assert _stats(lib, _layer(N=0)) == 2
+
+
+def test_call_validation(lib):
+    L = _layer()
+    soft = C.schedule(C.PHASE_SOFT, 30.0)
+    fwd = lib.catq_soft_ternary_linear_fwd
+    assert fwd(ctypes.byref(L), C.schedule(9, 1.0), 16, 4, C.BF16, 16, None) == 1      # bad phase
+    assert fwd(ctypes.byref(L), C.schedule(C.PHASE_SOFT, 0.0), 16, 4, C.BF16, 16, None) == 1  # s must be > 0
+    assert fwd(ctypes.byref(L), C.schedule(C.PHASE_SOFT, float("nan")), 16, 4, C.BF16, 16, None) == 1
+    assert fwd(ctypes.byref(L), soft, 16, 4, C.F32, 16, None) == 3                   # mixed dtypes
+    assert fwd(ctypes.byref(L), soft, 16, -1, C.BF16, 16, None) == 2                 # M < 0
+    assert fwd(ctypes.byref(L), soft, 16, 0, C.BF16, 16, None) == 0                  # M == 0: no-op
+    assert fwd(ctypes.byref(L), soft, 0, 4, C.BF16, 16, None) == 1                   # null X
+    assert fwd(ctypes.byref(L), soft, 24, 4, C.BF16, 16, None) == 4                  # misaligned X
+    bwd = lib.catq_soft_ternary_linear_bwd
+    assert bwd(ctypes.byref(L), soft, 16, 16, 4, C.BF16, None, 0, 32, 32, 256, 1 << 30, None) == 1
+    F = _layer(dtype=C.F32)
+    need = lib.catq_bwd_workspace_bytes(ctypes.byref(F), 4)
+    assert need == 3 * 64 * (256 // 64) * 4
+    assert bwd(ctypes.byref(F), soft, 16, 16, 4, C.F32, None, 32, 32, 32, 256, need - 1, None) == 9
+    assert bwd(ctypes.byref(F), soft, 16, 16, 4, C.F32, None, 32, 32, 32, 0, need, None) == 9
+    assert bwd(ctypes.byref(F), soft, 16, 16, 4, C.F32, None, 32, 32, 32, 128, need, None) == 4
+    loss = lib.catq_recon_loss
+    ws = lib.catq_recon_loss_workspace_bytes(1000)
+    assert ws >= 8 and ws % 256 == 0
+    assert loss(16, 16, 1000, 5, 0, 16, None, 256, ws, None) == 3
+    assert loss(16, 16, 1000, C.BF16, 2, 16, None, 256, ws, None) == 1
+    assert loss(16, 16, 0, C.BF16, 0, 16, None, 256, ws, None) == 2
+    assert loss(16, 16, 1000, C.BF16, 0, 16, None, 256, ws - 256, None) == 9
+    assert loss(16, 24, 1000, C.BF16, 0, 16, None, 256, ws, None) == 4
+    pack = lib.catq_hard_ternarize_pack
+    assert pack(ctypes.byref(L), None, None, None) == 1
+    assert lib.catq_device_status(None, None) == 1
