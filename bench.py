@@ -1,0 +1,422 @@
+#!/usr/bin/env python
+"""Throughput of the CAT-Q soft-ternary calibration step on GB300.
+
+One step = one pass of the whole hot path over one calibration batch for every linear of
+a decoder block (default: the Llama-3-8B-shaped block, 4 x 2048 tokens):
+  group statistics (Eq. 3) -> fused soft-ternary forward Y = X Wq^T (Eq. 5/6, s = 30)
+  -> reconstruction loss and dY against the cached teacher output (Eq. 7)
+  -> dX = dY Wq -> factor gradients from dY^T X (chain rule of Eq. 3/5/6)
+  -> hard ternarization + 2-bit pack (Eq. 2/4).
+The metric is the algorithmic 6 M N K flops per linear (fwd + dX + dW) per second.
+
+Prints ONE JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle instead (the
+only other place this file runs the oracle besides the cpu_baseline leg).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from paper_2606_26650_gb300 import synthetic as syn  # noqa: E402
+
+METRIC = "soft-ternary linear fwd+bwd TFLOP/s per calibration step; % of GB300 BF16 peak"
+UNIT = "TFLOP/s"
+DEFAULT_WORKLOAD = "c3_llama3_8b_block"
+CPU_SAMPLE_LINEARS = ("q_proj", "k_proj", "down_proj")  # cpu_baseline leg of our arm
+CPU_SAMPLE_ROWS = 256
+REF_STEP_LINEARS = ("k_proj",)  # one step of the reference arm (runs K + W times)
+
+# DRAM traffic per launch of the dominant kernel from an ncu capture, keyed by the hash of
+# the sources it was taken at; reported only while those sources are unchanged.
+TRAFFIC = {}
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=60)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(syn.WORKLOADS))
+    p.add_argument("--s", type=float, default=30.0)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    return p.parse_args()
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
+            int(os.environ.get("WORLD_SIZE", 1)))
+
+
+def kernel_sources_sha() -> str:
+    h = hashlib.sha256()
+    for f in ("tc_gemm.cu", "catq_math.cuh", "ptx_sm100.cuh"):
+        with open(os.path.join(ROOT, "paper_2606_26650_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            d = json.load(fh)
+        return dict(bf16=float(d["bf16_tflops"]), bf16_sus=float(d["bf16_tflops_sustained"]),
+                    hbm=float(d["hbm_gbs"]), source="measured")
+    except Exception:
+        return dict(bf16=1900.0, bf16_sus=1700.0, hbm=6800.0, source="fallback")
+
+
+# ------------------------------------------------------------------ CPU oracle (baseline)
+
+def oracle_sample(wl, s, rows=CPU_SAMPLE_ROWS, linears=CPU_SAMPLE_LINEARS):
+    """Times the fp64 oracle on a bounded sample of the workload: the named linears at
+    `rows` tokens, every hot-path row (stats, fwd, loss, dX, factor gradients, pack).
+    Returns (seconds, algorithmic flops)."""
+    from oracle import catq_oracle as O
+    total_t, flops = 0.0, 0.0
+    for name in linears:
+        lin = wl.linear(name)
+        W = syn.weight(wl, lin).astype(np.float64)
+        X = syn.activations(wl, lin.x, rows, lin.K).astype(np.float64)
+        G = lin.N * lin.K // wl.g
+        fac = syn.factors(G, 0, f"bench/{name}", perturbed=True)
+        Y_ref = O.linear_fwd(X, W)  # cached teacher, not timed
+        t0 = time.perf_counter()
+        stats = O.group_stats(W, wl.g, wl.thr_init)
+        Wq = O.ternary_weight(W, wl.g, stats, fac, O.PHASE_SOFT, s)[0]
+        Y = O.linear_fwd(X, Wq)
+        _, dY = O.recon_loss(Y, Y_ref)
+        O.linear_bwd(X, dY, W, wl.g, stats, fac, O.PHASE_SOFT, s)
+        T, _, _ = O.hard_codes(W, wl.g, stats, fac)
+        O.pack_codes(T)
+        total_t += time.perf_counter() - t0
+        flops += 6.0 * rows * lin.N * lin.K
+    return total_t, flops
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def sample_text(wl, rows=CPU_SAMPLE_ROWS, linears=CPU_SAMPLE_LINEARS):
+    return (f"{'+'.join(linears)} of {wl.name} at {rows} of {wl.M} tokens, fp64 numpy oracle, all hot-path rows "
+            f"(stats, fwd, loss, dX, factor grads, pack); matmuls on multi-threaded BLAS, elementwise "
+            f"single-threaded; per-layer modulation cost is paid once per sample, as in the full step")
+
+
+def run_reference(args):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return
+    wl = syn.WORKLOADS[args.workload]
+    for _ in range(args.warmup):
+        oracle_sample(wl, args.s, linears=REF_STEP_LINEARS)
+    times, flops = [], 0.0
+    for _ in range(args.steps):
+        t, flops = oracle_sample(wl, args.s, linears=REF_STEP_LINEARS)
+        times.append(t)
+    tot = sum(times)
+    value = flops * len(times) / tot / 1e12
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / len(times),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": workload_config(wl, args),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                         "sample": sample_text(wl, linears=REF_STEP_LINEARS) + "; one sample per step"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def workload_config(wl, args):
+    return {"workload": wl.name, "tokens": wl.M, "group_size": wl.g, "phase": "soft", "s": args.s,
+            "linears": {lin.name: [lin.K, lin.N] for lin in wl.linears},
+            "flops_per_step": wl.flops_per_step,
+            "l2": "inputs larger than L2 (per-step working set of weights and activations > 129 MB)"}
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in (self.out or "").splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ GPU arm
+
+def run_ours(args):
+    import torch
+
+    from paper_2606_26650_gb300 import catq as C
+
+    rank, local, world = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    wl = syn.WORKLOADS[args.workload]
+    if wl.experts:
+        raise SystemExit("MoE workloads are parity cases, not bench lines")
+    M = wl.M
+    bf = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    sched = C.schedule(C.PHASE_SOFT, args.s)
+
+    def upload(a):
+        if wl.dtype == "bf16":
+            return torch.from_numpy(syn.bf16_bits(a).view(np.int16)).to(dev).view(torch.bfloat16)
+        return torch.from_numpy(a).to(dev)
+
+    Xs = {}
+    for lin in wl.linears:
+        if (lin.x, lin.K) not in Xs:
+            Xs[(lin.x, lin.K)] = upload(syn.activations(wl, lin.x, M, lin.K, seed=rank))
+    st = []
+    ws_bwd = ws_loss = 0
+    for lin in wl.linears:
+        G = lin.N * lin.K // wl.g
+        fac = [torch.from_numpy(f).to(dev) for f in syn.factors(G, rank, f"bench/{lin.name}", perturbed=True)]
+        layer = C.Layer.create(upload(syn.weight(wl, lin, seed=rank)), wl.g, *fac)
+        C.catq_group_stats(layer, wl.thr_init)
+        d = dict(lin=lin, layer=layer, X=Xs[(lin.x, lin.K)],
+                 Yt=torch.empty(M, lin.N, dtype=bf, device=dev), Y=torch.empty(M, lin.N, dtype=bf, device=dev),
+                 dY=torch.empty(M, lin.N, dtype=bf, device=dev), dX=torch.empty(M, lin.K, dtype=bf, device=dev),
+                 grads=[torch.empty(G, device=dev) for _ in range(3)],
+                 codes=torch.empty(lin.N * lin.K // 4, dtype=torch.uint8, device=dev),
+                 alpha=torch.empty(G, device=dev), loss=torch.empty(1, device=dev))
+        C.catq_soft_ternary_linear_fwd(layer, C.schedule(C.PHASE_TEACHER), d["X"], d["Yt"])
+        ws_bwd = max(ws_bwd, C.catq_bwd_workspace_bytes(layer, M))
+        ws_loss = max(ws_loss, C.catq_recon_loss_workspace_bytes(M * lin.N))
+        st.append(d)
+    wsb = C.workspace(ws_bwd, dev)
+    wsl = C.workspace(ws_loss, dev)
+    torch.cuda.synchronize()
+
+    kinds = ("fwd", "dx", "dw")
+
+    def step(ev=None):
+        for i, d in enumerate(st):
+            L = d["layer"]
+            C.catq_group_stats(L, wl.thr_init)
+            if ev is not None:
+                ev[i]["fwd"][0].record()
+            C.catq_soft_ternary_linear_fwd(L, sched, d["X"], d["Y"])
+            if ev is not None:
+                ev[i]["fwd"][1].record()
+            C.catq_recon_loss(d["Y"], d["Yt"], d["loss"], d["dY"], wsl)
+            if ev is not None:
+                ev[i]["dx"][0].record()
+            C.catq_soft_ternary_linear_bwd(L, sched, d["X"], d["dY"], dX=d["dX"])
+            if ev is not None:
+                ev[i]["dx"][1].record()
+                ev[i]["dw"][0].record()
+            C.catq_soft_ternary_linear_bwd(L, sched, d["X"], d["dY"], None, *d["grads"], workspace=wsb)
+            if ev is not None:
+                ev[i]["dw"][1].record()
+            C.catq_hard_ternarize_pack(L, d["codes"], d["alpha"])
+
+    launches_per_step = len(st) * (1 + 1 + 2 + 1 + 2 + 1)
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+            torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        step()
+    barrier()
+    if C.catq_device_status() != 0:
+        raise SystemExit("device status set during warm-up")
+
+    E = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    evs = [[{k: (E(), E()) for k in kinds} for _ in st] for _ in range(args.steps)]
+    t_start, t_end = E(), E()
+    with ClockSampler(local) as clk:
+        barrier()
+        t_start.record()
+        for k in range(args.steps):
+            step(evs[k])
+        t_end.record()
+        barrier()
+    status = C.catq_device_status()
+    if status != 0:
+        raise SystemExit(f"device status {C.STATUS.get(status, status)} in the timed region")
+    ms = t_start.elapsed_time(t_end) / args.steps
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    flops_step = wl.flops_per_step
+    value = world * flops_step / (ms * 1e-3) / 1e12
+
+    # per-kernel live timing (CUDA events on the launching stream)
+    per = {k: 0.0 for k in kinds}
+    for k in range(args.steps):
+        for i in range(len(st)):
+            for kind in kinds:
+                a, b = evs[k][i][kind]
+                per[kind] += a.elapsed_time(b)
+    flops_kind = sum(2.0 * M * d["lin"].N * d["lin"].K for d in st) * args.steps
+    dom = max(kinds, key=lambda k: per[k])
+    peaks = measured_peaks()
+    achieved = flops_kind / (per[dom] * 1e-3) / 1e12
+    kernel_name = {"fwd": "fused_gemm_kernel (forward, K-major Wq operand)",
+                   "dx": "fused_gemm_kernel (dX, MN-major Wq operand)",
+                   "dw": "dw_kernel + grad_reduce_kernel (dW factor-gradient epilogue)"}[dom]
+    sha = kernel_sources_sha()
+    traffic = TRAFFIC.get(dom) if TRAFFIC.get("sha") == sha else None
+    roofline = {"bound": "tensor", "kernel": kernel_name, "achieved": achieved, "peak": peaks["bf16_sus"],
+                "unit": UNIT, "frac": achieved / peaks["bf16_sus"], "traffic": traffic,
+                "peak_kind": f"bf16 dense sustained ({peaks['source']})",
+                "frac_of_burst": achieved / peaks["bf16"],
+                "per_kernel_ms_per_step": {k: per[k] / args.steps for k in kinds},
+                "per_kernel_tflops": {k: flops_kind / (per[k] * 1e-3) / 1e12 for k in kinds}}
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = measure_e2e(args, C, torch, st, step, barrier, flops_step, world, dev)
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        t, fl = oracle_sample(wl, args.s)
+        cpu = {"value": fl / t / 1e12, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+               "sample": sample_text(wl), "seconds": t}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
+            "config": workload_config(wl, args),
+            "frac_of_bf16_peak": {"sustained": value / world / peaks["bf16_sus"],
+                                  "burst": value / world / peaks["bf16"], "source": peaks["source"]},
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": launches_per_step * args.steps, "clocks": clk.summary(),
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def measure_e2e(args, C, torch, st, step, barrier, flops_step, world, dev):
+    """Same step through the public API with the calibration batch (activations) and the
+    teacher outputs copied from pinned host memory each step, and the losses and factor
+    gradients read back."""
+    xs = {}
+    for d in st:
+        key = d["X"].data_ptr()
+        if key not in xs:
+            xs[key] = (d["X"], torch.empty(d["X"].shape, dtype=d["X"].dtype, pin_memory=True))
+            xs[key][1].copy_(d["X"])
+    yts = [(d["Yt"], torch.empty(d["Yt"].shape, dtype=d["Yt"].dtype, pin_memory=True)) for d in st]
+    for dv, h in yts:
+        h.copy_(dv)
+    outs = [(t, torch.empty(t.shape, dtype=t.dtype, pin_memory=True)) for d in st for t in [d["loss"]] + d["grads"]]
+    h2d = sum(h.numel() * h.element_size() for _, h in xs.values()) + sum(h.numel() * h.element_size() for _, h in yts)
+    d2h = sum(h.numel() * h.element_size() for _, h in outs)
+
+    def e2e_step():
+        for dv, h in xs.values():
+            dv.copy_(h, non_blocking=True)
+        for dv, h in yts:
+            dv.copy_(h, non_blocking=True)
+        step()
+        for dv, h in outs:
+            h.copy_(dv, non_blocking=True)
+
+    steps = max(3, args.steps // 2)
+    for _ in range(2):
+        e2e_step()
+    barrier()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(steps):
+        e2e_step()
+    b.record()
+    barrier()
+    ms = a.elapsed_time(b) / steps
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return {"value": world * flops_step / (ms * 1e-3) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": steps}
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

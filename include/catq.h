@@ -30,7 +30,7 @@
  *   - Shapes: g divides K.  bf16 weights need g % 64 == 0 and N % 8 == 0; fp32 weights
  *     need g % 64 == 0 or g in {4, 8, 16, 32}.  The weight and activation dtypes must
  *     match: both CATQ_F32 (CUDA-core path) or both CATQ_BF16 (tensor-core path,
- *     fp32 accumulation).  bf16 buffers must be 16-byte aligned.
+ *     fp32 accumulation).  W, X, Y, dY, dX and Wq buffers must be 16-byte aligned.
  *   - A group whose alpha is exactly 0 (constant weights, or d_alpha == 0) has Wq = 0,
  *     hard code 0 and zero factor gradients.
  */
@@ -52,7 +52,7 @@ typedef enum {
   CATQ_ERR_INVALID_ARG = 1, /* null pointer, bad enum, non-finite or non-positive s */
   CATQ_ERR_SHAPE = 2,       /* g does not divide K, unsupported g, M < 0, N/K < 1 */
   CATQ_ERR_DTYPE = 3,       /* unknown dtype or mixed weight/activation dtypes */
-  CATQ_ERR_ALIGN = 4,       /* bf16 buffer not 16-byte aligned */
+  CATQ_ERR_ALIGN = 4,       /* buffer not 16-byte aligned (workspace: 256-byte) */
   CATQ_ERR_CUDA = 5,        /* a CUDA runtime call failed (launch, attribute, tensor map) */
   CATQ_ERR_TIMEOUT = 6,     /* a bounded device-side wait expired (latched) */
   CATQ_ERR_NONFINITE = 7,   /* reserved: non-finite data detected (latched) */
@@ -144,8 +144,10 @@ size_t catq_bwd_workspace_bytes(const catq_layer* layer, int64_t M);
  * is the forward value Q(What; Delta) and the derivatives are those of f at s (the
  * surrogate reading of §2.3's stage-2 rule).  In the TEACHER phase Wq = W does not depend
  * on the factors: the three gradients are written as zeros.  Gradients are overwritten,
- * not accumulated.  workspace: device, >= catq_bwd_workspace_bytes(layer, M) bytes,
- * 256-byte aligned, contents scratch.                                                    */
+ * not accumulated.  g_dmu, g_dalpha, g_ddelta: device fp32 [G], all three or none (NULL
+ * skips the factor gradients, e.g. a dX-only backward through frozen layers).
+ * workspace: device, >= catq_bwd_workspace_bytes(layer, M) bytes, 256-byte aligned,
+ * contents scratch; may be NULL when no factor gradients are computed.                  */
 catq_status catq_soft_ternary_linear_bwd(const catq_layer* layer, catq_schedule sched,
                                          const void* X, const void* dY, int64_t M,
                                          int32_t x_dtype, void* dX, float* g_dmu,

@@ -185,8 +185,8 @@ def catq_bwd_workspace_bytes(layer: Layer, M: int) -> int:
     return int(lib().catq_bwd_workspace_bytes(ctypes.byref(st), int(M)))
 
 
-def catq_soft_ternary_linear_bwd(layer: Layer, sched: catq_schedule, X, dY, dX, g_dmu, g_dalpha, g_ddelta,
-                                 workspace, stream=None):
+def catq_soft_ternary_linear_bwd(layer: Layer, sched: catq_schedule, X, dY, dX=None, g_dmu=None, g_dalpha=None,
+                                 g_ddelta=None, workspace=None, stream=None):
     st = layer.struct()
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     _check(lib().catq_soft_ternary_linear_bwd(ctypes.byref(st), sched, _ptr(X), _ptr(dY), X.shape[0],

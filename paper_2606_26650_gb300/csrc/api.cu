@@ -177,11 +177,12 @@ catq_status catq_soft_ternary_linear_bwd(const catq_layer* layer, catq_schedule 
   if ((st = check_schedule(sched, sched.phase != CATQ_PHASE_TEACHER)) != CATQ_OK) return st;
   if (x_dtype != layer->w_dtype) return CATQ_ERR_DTYPE;
   if (M < 0) return CATQ_ERR_SHAPE;
-  if (!g_dmu || !g_dalpha || !g_ddelta) return CATQ_ERR_INVALID_ARG;
+  const bool want_grads = g_dmu || g_dalpha || g_ddelta;
+  if (want_grads && !(g_dmu && g_dalpha && g_ddelta)) return CATQ_ERR_INVALID_ARG;
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const LayerDev L = to_dev(layer);
   const int64_t G = layer->N * layer->K / layer->g;
-  const bool need_dw = sched.phase != CATQ_PHASE_TEACHER && M > 0;
+  const bool need_dw = want_grads && sched.phase != CATQ_PHASE_TEACHER && M > 0;
   if (M > 0) {
     if (!X || !dY) return CATQ_ERR_INVALID_ARG;
     if (!aligned16(X) || !aligned16(dY) || (dX && !aligned16(dX))) return CATQ_ERR_ALIGN;
@@ -202,6 +203,7 @@ catq_status catq_soft_ternary_linear_bwd(const catq_layer* layer, catq_schedule 
             : launch_tc_dx(L, sc, dY, M, dX, s);
     if (e != cudaSuccess) return CATQ_ERR_CUDA;
   }
+  if (!want_grads) return CATQ_OK;
   if (!need_dw) {
     const size_t b = static_cast<size_t>(G) * sizeof(float);
     if (cudaMemsetAsync(g_dmu, 0, b, s) != cudaSuccess || cudaMemsetAsync(g_dalpha, 0, b, s) != cudaSuccess ||

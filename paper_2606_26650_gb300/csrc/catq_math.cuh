@@ -30,23 +30,39 @@ struct GroupConst {
   float r, b, alpha, delta, alpha0, delta0;
 };
 
-__device__ __forceinline__ GroupConst group_const(const LayerDev& L, int64_t j) {
-  const float a0 = __ldg(L.alpha0 + j);
-  const float m0 = __ldg(L.mu0 + j);
-  const float D0 = __ldg(L.delta0 + j);
-  const float mu = fmaf(__ldg(L.d_mu + j), a0, m0);
-  const float alpha = __ldg(L.d_alpha + j) * a0;
-  const float delta = __ldg(L.d_delta + j) * D0;
-  const float r = (alpha != 0.0f) ? 1.0f / alpha : 0.0f;
+// The six per-group inputs, loaded separately from the arithmetic so callers can issue the
+// loads a pipeline stage before they need the constants.
+struct GroupRaw {
+  float a0, m0, D0, dmu, dal, ddl;
+};
+
+__device__ __forceinline__ GroupRaw group_raw(const LayerDev& L, int64_t j) {
+  GroupRaw g;
+  g.a0 = __ldg(L.alpha0 + j);
+  g.m0 = __ldg(L.mu0 + j);
+  g.D0 = __ldg(L.delta0 + j);
+  g.dmu = __ldg(L.d_mu + j);
+  g.dal = __ldg(L.d_alpha + j);
+  g.ddl = __ldg(L.d_delta + j);
+  return g;
+}
+
+__device__ __forceinline__ GroupConst group_const(const GroupRaw& g) {
+  const float mu = fmaf(g.dmu, g.a0, g.m0);
+  const float alpha = g.dal * g.a0;
+  const float delta = g.ddl * g.D0;
+  const float r = (alpha != 0.0f) ? __frcp_rn(alpha) : 0.0f;  // correctly rounded 1 / alpha
   GroupConst c;
   c.r = r;
   c.b = -mu * r;
   c.alpha = alpha;
   c.delta = delta;
-  c.alpha0 = a0;
-  c.delta0 = D0;
+  c.alpha0 = g.a0;
+  c.delta0 = g.D0;
   return c;
 }
+
+__device__ __forceinline__ GroupConst group_const(const LayerDev& L, int64_t j) { return group_const(group_raw(L, j)); }
 
 __device__ __forceinline__ float what(float w, const GroupConst& c) { return fmaf(w, c.r, c.b); }
 
@@ -67,29 +83,16 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return d;
 }
 
-__device__ __forceinline__ uint32_t tanh_bf16x2(uint32_t x) {
-  uint32_t d;
-  asm("tanh.approx.bf16x2 %0, %1;" : "=r"(d) : "r"(x));
-  return d;
-}
-
-__device__ __forceinline__ uint32_t add_bf16x2(uint32_t a, uint32_t b) {
-  uint32_t d;
-  asm("add.rn.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-  return d;
-}
-
-__device__ __forceinline__ uint32_t mul_bf16x2(uint32_t a, uint32_t b) {
-  uint32_t d;
-  asm("mul.rn.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-  return d;
-}
-
-// Per-row constants of the bf16 operand producer for one group (see soft_pair_bf16).
+// Per-row constants of the bf16 operand producer for one group.
+//   SOFT: u = s What = fma(w, A, B), D = s Delta, C = alpha / (2 tanh s);
+//         `one_tanh` when D >= 6: for u >= 0 the term tanh(u + D) >= tanh 6 = 1 - 1.2e-5 is
+//         1 to well below bf16 resolution (and symmetrically for u < 0), so
+//         alpha f = sign(u) C (1 + tanh(|u| - D)) needs one tanh instead of two.
+//   HARD: What = fma(w, r, b), threshold Delta, C = alpha.
 struct ProducerConst {
-  float A, B, D;   // SOFT: u = s * What = fma(w, A, B); D = s * Delta
-  uint32_t C2;     // SOFT: alpha / (2 tanh s) as bf16x2; HARD: alpha as bf16x2
-  float r, b, delta;  // HARD: What = fma(w, r, b), threshold Delta
+  float A, B, D, C;
+  float r, b, delta;
+  bool one_tanh;
 };
 
 __device__ __forceinline__ ProducerConst producer_const(const GroupConst& c, float s, float inv_2tanh_s,
@@ -98,34 +101,44 @@ __device__ __forceinline__ ProducerConst producer_const(const GroupConst& c, flo
   p.A = s * c.r;
   p.B = s * c.b;
   p.D = s * c.delta;
-  const float C = (phase == PHASE_SOFT) ? c.alpha * inv_2tanh_s : c.alpha;
-  p.C2 = pack_bf16x2(C, C);
+  p.C = (phase == PHASE_SOFT) ? c.alpha * inv_2tanh_s : c.alpha;
   p.r = c.r;
   p.b = c.b;
   p.delta = c.delta;
+  p.one_tanh = p.D >= 6.0f;
   return p;
 }
 
-// Eq. 5/6 SOFT weight for two bf16 weights: alpha f(What; s, Delta) =
-//   [alpha / (2 tanh s)] * [tanh(u - s Delta) + tanh(u + s Delta)],  u = s What,
-// with u computed in fp32, both tanh arguments rounded to bf16 and evaluated together by
-// one packed tanh, and the sum and scale in bf16 (the operand's precision).
+__device__ __forceinline__ float tanh_fast(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Eq. 5/6 SOFT weight alpha f(What; s, Delta) for two bf16 weights, fp32 arithmetic with
+// the hardware tanh, rounded once to bf16.
 __device__ __forceinline__ uint32_t soft_pair_bf16(uint32_t w2, const ProducerConst& p) {
   const float u0 = fmaf(bf16lo_to_f32(w2), p.A, p.B);
   const float u1 = fmaf(bf16hi_to_f32(w2), p.A, p.B);
-  const uint32_t tm = tanh_bf16x2(pack_bf16x2(u0 - p.D, u1 - p.D));
-  const uint32_t tp = tanh_bf16x2(pack_bf16x2(u0 + p.D, u1 + p.D));
-  return mul_bf16x2(add_bf16x2(tm, tp), p.C2);
+  float y0, y1;
+  if (p.one_tanh) {
+    const float c0 = copysignf(p.C, u0), c1 = copysignf(p.C, u1);
+    y0 = fmaf(tanh_fast(fabsf(u0) - p.D), c0, c0);
+    y1 = fmaf(tanh_fast(fabsf(u1) - p.D), c1, c1);
+  } else {
+    y0 = p.C * (tanh_fast(u0 - p.D) + tanh_fast(u0 + p.D));
+    y1 = p.C * (tanh_fast(u1 - p.D) + tanh_fast(u1 + p.D));
+  }
+  return pack_bf16x2(y0, y1);
 }
 
-// Eq. 2/6 HARD weight for two bf16 weights: alpha Q(What; Delta).
+// Eq. 2/6 HARD weight alpha Q(What; Delta) for two bf16 weights.
 __device__ __forceinline__ uint32_t hard_pair_bf16(uint32_t w2, const ProducerConst& p) {
   const float x0 = fmaf(bf16lo_to_f32(w2), p.r, p.b);
   const float x1 = fmaf(bf16hi_to_f32(w2), p.r, p.b);
-  const uint32_t a = p.C2 & 0xFFFFu;
-  const uint32_t lo = x0 > p.delta ? a : (x0 < -p.delta ? (a | 0x8000u) : 0u);
-  const uint32_t hi = x1 > p.delta ? a : (x1 < -p.delta ? (a | 0x8000u) : 0u);
-  return lo | (hi << 16);
+  const float y0 = x0 > p.delta ? p.C : (x0 < -p.delta ? -p.C : 0.0f);
+  const float y1 = x1 > p.delta ? p.C : (x1 < -p.delta ? -p.C : 0.0f);
+  return pack_bf16x2(y0, y1);
 }
 
 __device__ __forceinline__ uint4 transform_chunk_bf16(uint4 v, const ProducerConst& p, int32_t phase) {

@@ -17,6 +17,7 @@ __device__ __forceinline__ double warp_sum(double v) {
   return v;
 }
 
+
 template <typename T>
 struct Vec16;  // 16-byte vector of T, unpacked to floats
 template <>
@@ -41,43 +42,131 @@ struct Vec16<__nv_bfloat16> {
   }
 };
 
+// ---------------------------------------------------------------- compensated fp32 sums
+// fp64 arithmetic is slow on this GPU, so sums use an fp32 value plus an fp32 error term
+// (Knuth's two-sum), which carries about twice fp32's precision.
+struct Sum2 {
+  float hi, lo;
+};
+
+__device__ __forceinline__ void sum2_add(Sum2& a, float x) {
+  const float s = a.hi + x;
+  const float bp = s - a.hi;
+  const float err = (a.hi - (s - bp)) + (x - bp);
+  a.hi = s;
+  a.lo += err;
+}
+
+__device__ __forceinline__ Sum2 sum2_merge(Sum2 a, Sum2 b) {
+  const float s = a.hi + b.hi;
+  const float bp = s - a.hi;
+  const float err = (a.hi - (s - bp)) + (b.hi - bp);
+  return Sum2{s, a.lo + b.lo + err};
+}
+
+// Butterfly reduction over aligned teams of `team` lanes (team a power of two <= 32).
+__device__ __forceinline__ Sum2 sum2_team(Sum2 v, int team) {
+  for (int o = team >> 1; o > 0; o >>= 1) {
+    Sum2 w;
+    w.hi = __shfl_xor_sync(0xffffffffu, v.hi, o);
+    w.lo = __shfl_xor_sync(0xffffffffu, v.lo, o);
+    v = sum2_merge(v, w);
+  }
+  return v;
+}
+
+__device__ __forceinline__ double sum2_value(Sum2 v) { return static_cast<double>(v.hi) + static_cast<double>(v.lo); }
+
 // ---------------------------------------------------------------- Eq. 3 statistics
-// One warp per group; fp64 sums; two passes over the group (mean, then deviations).
+// Register variant: a team of `team` lanes owns one group and keeps its R x 16-byte
+// vectors in registers (mean, then deviations, without re-reading W).
+template <typename T, int R>
+__global__ void __launch_bounds__(kThreads) group_stats_reg_kernel(const T* __restrict__ W, int64_t G, int32_t g,
+                                                                   int32_t team, int32_t thr_init,
+                                                                   float* __restrict__ mu0,
+                                                                   float* __restrict__ alpha0,
+                                                                   float* __restrict__ delta0) {
+  constexpr int V = Vec16<T>::n;
+  const int lane = threadIdx.x & 31;
+  const int sub = lane % team;
+  const int per_warp = 32 / team;
+  const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
+  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
+  for (int64_t wbase = warp * per_warp; wbase < G; wbase += nwarps * per_warp) {
+    const int64_t j = wbase + lane / team;
+    const bool live = j < G;
+    float v[R][V];
+    Sum2 sum{0.f, 0.f};
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      if (live) {
+        Vec16<T>::load(W + j * g + static_cast<int64_t>(sub + r * team) * V, v[r]);
+      } else {
+#pragma unroll
+        for (int q = 0; q < V; ++q) v[r][q] = 0.f;
+      }
+#pragma unroll
+      for (int q = 0; q < V; ++q) sum2_add(sum, v[r][q]);
+    }
+    sum = sum2_team(sum, team);
+    const float mu = static_cast<float>(sum2_value(sum) / g);
+    Sum2 dev{0.f, 0.f}, mag{0.f, 0.f};
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+#pragma unroll
+      for (int q = 0; q < V; ++q) {
+        sum2_add(dev, fabsf(v[r][q] - mu));
+        sum2_add(mag, fabsf(v[r][q]));
+      }
+    dev = sum2_team(dev, team);
+    mag = sum2_team(mag, team);
+    if (live && sub == 0) {
+      const double a0 = sum2_value(dev) / g;
+      mu0[j] = mu;
+      alpha0[j] = static_cast<float>(a0);
+      delta0[j] = (thr_init == 1 && a0 > 0.0) ? static_cast<float>(0.7 * (sum2_value(mag) / g) / a0) : 0.5f;
+    }
+  }
+}
+
+// Streaming variant for any g (one warp per group, second pass re-reads the group).
 template <typename T>
-__global__ void __launch_bounds__(kThreads) group_stats_kernel(const T* __restrict__ W, int64_t G, int32_t g,
-                                                               int32_t thr_init, float* __restrict__ mu0,
-                                                               float* __restrict__ alpha0,
-                                                               float* __restrict__ delta0) {
+__global__ void __launch_bounds__(kThreads) group_stats_stream_kernel(const T* __restrict__ W, int64_t G, int32_t g,
+                                                                      int32_t thr_init, float* __restrict__ mu0,
+                                                                      float* __restrict__ alpha0,
+                                                                      float* __restrict__ delta0) {
   constexpr int V = Vec16<T>::n;
   const int lane = threadIdx.x & 31;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
   const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
   for (int64_t j = warp; j < G; j += nwarps) {
     const T* base = W + j * g;
-    double sum = 0.0;
+    Sum2 sum{0.f, 0.f};
     for (int i = lane * V; i < g; i += 32 * V) {
       float v[V];
       Vec16<T>::load(base + i, v);
 #pragma unroll
-      for (int q = 0; q < V; ++q) sum += static_cast<double>(v[q]);
+      for (int q = 0; q < V; ++q) sum2_add(sum, v[q]);
     }
-    const double mu = warp_sum(sum) / static_cast<double>(g);
-    double dev = 0.0, mag = 0.0;
+    sum = sum2_team(sum, 32);
+    const float mu = static_cast<float>(sum2_value(sum) / g);
+    Sum2 dev{0.f, 0.f}, mag{0.f, 0.f};
     for (int i = lane * V; i < g; i += 32 * V) {
       float v[V];
       Vec16<T>::load(base + i, v);
 #pragma unroll
       for (int q = 0; q < V; ++q) {
-        dev += fabs(static_cast<double>(v[q]) - mu);
-        mag += fabs(static_cast<double>(v[q]));
+        sum2_add(dev, fabsf(v[q] - mu));
+        sum2_add(mag, fabsf(v[q]));
       }
     }
-    const double a0 = warp_sum(dev) / static_cast<double>(g);
-    const double m = warp_sum(mag) / static_cast<double>(g);
+    dev = sum2_team(dev, 32);
+    mag = sum2_team(mag, 32);
     if (lane == 0) {
-      mu0[j] = static_cast<float>(mu);
+      const double a0 = sum2_value(dev) / g;
+      mu0[j] = mu;
       alpha0[j] = static_cast<float>(a0);
-      delta0[j] = (thr_init == 1 && a0 > 0.0) ? static_cast<float>(0.7 * m / a0) : 0.5f;
+      delta0[j] = (thr_init == 1 && a0 > 0.0) ? static_cast<float>(0.7 * (sum2_value(mag) / g) / a0) : 0.5f;
     }
   }
 }
@@ -211,32 +300,34 @@ __global__ void __launch_bounds__(kThreads) recon_loss_partial_kernel(const T* _
                                                                       double* __restrict__ partials) {
   constexpr int V = Vec16<T>::n;
   const int64_t nvec = count / V;
-  double acc = 0.0;
+  Sum2 acc{0.f, 0.f};
   for (int64_t i = blockIdx.x * (int64_t)kThreads + threadIdx.x; i < nvec; i += (int64_t)gridDim.x * kThreads) {
     float a[V], b[V], d[V];
     Vec16<T>::load(Y + i * V, a);
     Vec16<T>::load(Yr + i * V, b);
+    Sum2 local{0.f, 0.f};
 #pragma unroll
     for (int q = 0; q < V; ++q) {
       d[q] = a[q] - b[q];
-      acc += static_cast<double>(d[q]) * static_cast<double>(d[q]);
+      sum2_add(local, d[q] * d[q]);
     }
+    acc = sum2_merge(acc, local);
     if (dY) store_scaled<T>(dY + i * V, d, scale);
   }
   if (blockIdx.x == 0)
     for (int64_t i = nvec * V + threadIdx.x; i < count; i += kThreads) {
       const float d = load_scalar(Y + i) - load_scalar(Yr + i);
-      acc += static_cast<double>(d) * static_cast<double>(d);
+      sum2_add(acc, d * d);
       if (dY) store_scalar(dY + i, d * scale);
     }
-  __shared__ double red[kThreads / 32];
-  acc = warp_sum(acc);
+  __shared__ Sum2 red[kThreads / 32];
+  acc = sum2_team(acc, 32);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
   __syncthreads();
   if (threadIdx.x < 32) {
-    double v = threadIdx.x < kThreads / 32 ? red[threadIdx.x] : 0.0;
-    v = warp_sum(v);
-    if (threadIdx.x == 0) partials[blockIdx.x] = v;
+    Sum2 v = threadIdx.x < kThreads / 32 ? red[threadIdx.x] : Sum2{0.f, 0.f};
+    v = sum2_team(v, 32);
+    if (threadIdx.x == 0) partials[blockIdx.x] = sum2_value(v);
   }
 }
 
@@ -300,13 +391,34 @@ int grid_for(int64_t work, int64_t per_block) {
 cudaError_t launch_group_stats(const LayerDev& L, int32_t w_dtype, int32_t thr_init, float* mu0, float* alpha0,
                                float* delta0, cudaStream_t st) {
   const int64_t G = L.N * L.K / L.g;
+  const int V = w_dtype == 1 ? 8 : 4;  // elements per 16-byte vector
+  const int nvec = L.g / V;            // vectors per group
+  if (L.g % V == 0 && nvec <= 128 && (nvec & (nvec - 1)) == 0) {
+    const int team = nvec < 32 ? nvec : 32;
+    const int R = nvec / team;
+    const int grid = grid_for((G + 32 / team - 1) / (32 / team), kThreads / 32);
+#define CATQ_STATS_REG(TT, RR)                                                                                  \
+  group_stats_reg_kernel<TT, RR><<<grid, kThreads, 0, st>>>(static_cast<const TT*>(L.W), G, L.g, team, thr_init, \
+                                                            mu0, alpha0, delta0)
+    if (w_dtype == 1) {
+      if (R == 1) CATQ_STATS_REG(__nv_bfloat16, 1);
+      else if (R == 2) CATQ_STATS_REG(__nv_bfloat16, 2);
+      else CATQ_STATS_REG(__nv_bfloat16, 4);
+    } else {
+      if (R == 1) CATQ_STATS_REG(float, 1);
+      else if (R == 2) CATQ_STATS_REG(float, 2);
+      else CATQ_STATS_REG(float, 4);
+    }
+#undef CATQ_STATS_REG
+    return cudaGetLastError();
+  }
   const int grid = grid_for(G, kThreads / 32);
   if (w_dtype == 1)
-    group_stats_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(static_cast<const __nv_bfloat16*>(L.W), G, L.g,
-                                                                   thr_init, mu0, alpha0, delta0);
+    group_stats_stream_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(static_cast<const __nv_bfloat16*>(L.W), G,
+                                                                          L.g, thr_init, mu0, alpha0, delta0);
   else
-    group_stats_kernel<float><<<grid, kThreads, 0, st>>>(static_cast<const float*>(L.W), G, L.g, thr_init, mu0,
-                                                         alpha0, delta0);
+    group_stats_stream_kernel<float><<<grid, kThreads, 0, st>>>(static_cast<const float*>(L.W), G, L.g, thr_init,
+                                                                mu0, alpha0, delta0);
   return cudaGetLastError();
 }
 

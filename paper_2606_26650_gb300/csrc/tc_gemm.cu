@@ -3,8 +3,9 @@
 //
 // fused_gemm_kernel  C[M, ncols] = A[M, depth] * Wq-operand, with the Eq. 3/5/6 weight
 //                    (modulation, transition function, scale alpha) computed by producer
-//                    warps on the raw W tile while it sits in shared memory, in place, in
+//                    warps on raw W tiles that TMA lands in their own ring, in place, in
 //                    the 128-byte-swizzled layout the MMA reads.  Wq never reaches HBM.
+//                    A tiles flow TMA -> MMA in a separate ring, off the producers' path.
 //                      forward:  A = X  [M, K],  operand = Wq   (K-major), C = Y  [M, N]
 //                      dX:       A = dY [M, N],  operand = Wq   (MN-major), C = dX [M, K]
 //                    Two M-tiles share each produced operand tile (two accumulators).
@@ -49,15 +50,22 @@ struct FusedCfg {
   static constexpr int kRowsPerAcc = 128 * CG;          // MMA M
   static constexpr int kTileRows = kRowsPerAcc * NACC;  // rows of C per tile
   static constexpr int kBRows = BN / CG;                // 128-byte operand rows per CTA per stage
-  static constexpr int kABytes = NACC * 128 * BK * 2;   // this CTA's A rows
-  static constexpr int kBBytes = kBRows * BK * 2;
-  static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kStages = CG == 1 ? 3 : 4;
+  static constexpr int kABytes = NACC * 128 * BK * 2;   // this CTA's A rows per stage
+  static constexpr int kWBytes = kBRows * BK * 2;       // this CTA's operand rows per stage
+  static constexpr int kStagesA = CG == 1 ? 3 : 4;      // A ring: TMA -> MMA
+  static constexpr int kStagesW = CG == 1 ? 3 : 5;      // W ring: TMA -> producers (in place) -> MMA
   static constexpr int kEpiWarps = 4;
-  static constexpr int kProdWarps = 8;
+  // Two groups of 8 producer warps take alternate stages, so each group has two stage
+  // periods per operand tile and the groups' MUFU work interleaves.
+  static constexpr int kProdGroups = 2;
+  static constexpr int kGroupWarps = 8;
+  static constexpr int kProdWarps = kProdGroups * kGroupWarps;
+  static constexpr int kGroupThreads = 32 * kGroupWarps;
+  static constexpr int kThreadsPerRow = kGroupThreads / kBRows;  // 1 (CG 1) or 2 (CG 2)
+  static constexpr int kChunksPerThread = 8 / kThreadsPerRow;    // 16-byte chunks of a 128-byte row
   static constexpr int kThreads = 32 * (kEpiWarps + 2 + kProdWarps);
-  static constexpr int kBarBytes = 8 * (3 * kStages + 3) + 16;
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + kBarBytes;
+  static constexpr int kBarBytes = 8 * (2 * kStagesA + 3 * kStagesW + 3) + 16;
+  static constexpr int kSmemBytes = kStagesA * kABytes + kStagesW * kWBytes + 1024 + kBarBytes;
 };
 
 template <int CG>
@@ -118,24 +126,52 @@ __device__ __forceinline__ void store_bf16x32(uint16_t* dst, const uint32_t (&r)
 
 // ============================================================================ fused kernel
 
+// Producer-side view of one 128-byte operand row for one pipeline stage: which W row and
+// which 64-element K chunk it holds, and its group.
+struct RowRef {
+  int64_t n, kc, j;
+  bool valid;
+};
+
+template <int CG, bool B_MN>
+__device__ __forceinline__ RowRef operand_row(const FusedArgs& a, uint32_t cta, int row, int t, int kb) {
+  using Cfg = FusedCfg<CG>;
+  const int n_blk = t / a.num_m_tiles;
+  RowRef r;
+  if constexpr (!B_MN) {  // forward: rows are output features n, the stage is a K chunk
+    r.n = (int64_t)n_blk * BN + cta * Cfg::kBRows + row;
+    r.kc = (int64_t)kb * BK;
+  } else {  // dX: rows are the contraction index n, 64-column blocks of output features k
+    r.n = (int64_t)kb * BK + (row & 63);
+    r.kc = (int64_t)n_blk * BN + cta * Cfg::kBRows + 64 * (row >> 6);
+  }
+  r.valid = r.n < a.L.N && r.kc < a.L.K;
+  r.j = r.n * a.L.groups_per_row + r.kc / a.L.g;
+  return r;
+}
+
 template <int CG, bool B_MN>
 __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
-    fused_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+    fused_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
                       const FusedArgs args) {
   using Cfg = FusedCfg<CG>;
-  constexpr int S = Cfg::kStages;
+  constexpr int SA = Cfg::kStagesA, SW = Cfg::kStagesW;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = smem_u32(smem_raw);
   const uint32_t base = (raw_addr + 1023u) & ~1023u;
   uint8_t* base_ptr = smem_raw + (base - raw_addr);
-  const uint32_t bars = base + S * Cfg::kStageBytes;
-  const uint32_t tmem_full_bar = bars + 8 * (3 * S);
+  const uint32_t a_base = base;                                // [SA][kABytes]
+  const uint32_t w_base = base + SA * Cfg::kABytes;            // [SW][kWBytes]
+  const uint32_t bars = w_base + SW * Cfg::kWBytes;
+  auto full_a = [&](int s) { return bars + 8u * s; };                   // A landed (pair: even CTA)
+  auto empty_a = [&](int s) { return bars + 8u * (SA + s); };           // A consumed by the MMA
+  auto raw_w = [&](int s) { return bars + 8u * (2 * SA + s); };         // raw W landed (local)
+  auto full_w = [&](int s) { return bars + 8u * (2 * SA + SW + s); };   // operand produced (pair: even CTA)
+  auto empty_w = [&](int s) { return bars + 8u * (2 * SA + 2 * SW + s); };
+  const uint32_t tmem_full_bar = bars + 8u * (2 * SA + 3 * SW);
   const uint32_t tmem_empty_bar = tmem_full_bar + 8;
   const uint32_t final_bar = tmem_full_bar + 16;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base_ptr + (bars - base) + 8 * (3 * S + 3));
-  auto full_raw = [&](int s) { return bars + 8u * s; };
-  auto full = [&](int s) { return bars + 8u * (S + s); };
-  auto empty = [&](int s) { return bars + 8u * (2 * S + s); };
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base_ptr + (bars - base) + 8 * (2 * SA + 3 * SW + 3));
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t cta = CG == 2 ? cluster_ctarank() : 0u;
@@ -143,91 +179,112 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
   const uint32_t nclusters = CG == 2 ? num_clusters_x() : gridDim.x;
   const WaitCtl& wc = args.wc;
   const int num_tiles = args.num_m_tiles * args.num_n_tiles;
+  constexpr int kTmaWarp = Cfg::kEpiWarps, kMmaWarp = Cfg::kEpiWarps + 1;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < S; ++s) {
-      mbar_init(full_raw(s), 1);
-      mbar_init(full(s), Cfg::kProdWarps * CG);
-      mbar_init(empty(s), 1);
+    for (int s = 0; s < SA; ++s) {
+      mbar_init(full_a(s), 1);
+      mbar_init(empty_a(s), 1);
+    }
+    for (int s = 0; s < SW; ++s) {
+      mbar_init(raw_w(s), 1);
+      mbar_init(full_w(s), Cfg::kGroupWarps * CG);  // one arrival per warp of the stage's group
+      mbar_init(empty_w(s), 1);
     }
     mbar_init(tmem_full_bar, 1);
     mbar_init(tmem_empty_bar, Cfg::kEpiWarps * CG);
     mbar_init(final_bar, 1);
     fence_mbar_init_cluster();
   }
-  if (warp == Cfg::kEpiWarps + 1) tmem_alloc<CG>(smem_u32(tmem_slot), kTmemCols);
-  if (warp == Cfg::kEpiWarps && lane == 0) {
+  if (warp == kMmaWarp) tmem_alloc<CG>(smem_u32(tmem_slot), kTmemCols);
+  if (warp == kTmaWarp && lane == 0) {
     prefetch_tmap(&tmA);
-    prefetch_tmap(&tmB);
+    prefetch_tmap(&tmW);
   }
   tc_fence_before();
   if constexpr (CG == 2) cluster_sync_all(); else __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   // Barriers the whole pair signals live in the even CTA.
-  const uint32_t leader_full0 = CG == 2 ? mapa_shared(full(0), 0) : full(0);
+  const uint32_t leader_full_a0 = CG == 2 ? mapa_shared(full_a(0), 0) : full_a(0);
+  const uint32_t leader_full_w0 = CG == 2 ? mapa_shared(full_w(0), 0) : full_w(0);
   const uint32_t leader_tmem_empty = CG == 2 ? mapa_shared(tmem_empty_bar, 0) : tmem_empty_bar;
 
-  if (warp == Cfg::kEpiWarps) {
-    // ------------------------------------------------------------ TMA producer
+  if (warp == kTmaWarp) {
     if (lane == 0) {
-      uint32_t stage = 0, phase = 0;
-      uint32_t issued_mask = 0, issued_phase = 0;
+      // ---------------------------------------------------------- TMA: A tiles (to the MMA)
+      uint32_t q = 0, issued_mask = 0, issued_phase = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
-        const int m_blk = t % args.num_m_tiles, n_blk = t / args.num_m_tiles;
-        const int32_t m0 = m_blk * Cfg::kTileRows, n0 = n_blk * BN;
-        for (int kb = 0; kb < args.num_k_blocks; ++kb) {
-          if (!mbar_wait(empty(stage), phase ^ 1u, wc)) { ok = false; break; }
-          const uint32_t sa = base + stage * Cfg::kStageBytes;
-          mbar_arrive_expect_tx(full_raw(stage), Cfg::kStageBytes);
+        const int32_t m0 = (t % args.num_m_tiles) * Cfg::kTileRows;
+        for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
+          const uint32_t s = q % SA, ph = (q / SA) & 1u;
+          if (!mbar_wait(empty_a(s), ph ^ 1u, wc)) { ok = false; break; }
+          if (cta == 0) mbar_arrive_expect_tx(full_a(s), Cfg::kABytes * CG);
+          const uint32_t dst = a_base + s * Cfg::kABytes, fb = leader_full_a0 + 8u * s;
 #pragma unroll
-          for (int acc = 0; acc < NACC; ++acc)
-            tma_load_2d(sa + acc * (128 * BK * 2), &tmA, full_raw(stage), kb * BK,
-                        m0 + acc * Cfg::kRowsPerAcc + cta * 128);
-          const uint32_t sb = sa + Cfg::kABytes;
-          if constexpr (!B_MN) {
-            tma_load_2d(sb, &tmB, full_raw(stage), kb * BK, n0 + cta * Cfg::kBRows);
-          } else {
-#pragma unroll
-            for (int b = 0; b < Cfg::kBRows / 64; ++b)
-              tma_load_2d(sb + b * 8192, &tmB, full_raw(stage), n0 + cta * Cfg::kBRows + 64 * b, kb * BK);
+          for (int acc = 0; acc < NACC; ++acc) {
+            const int32_t row = m0 + acc * Cfg::kRowsPerAcc + cta * 128;
+            if constexpr (CG == 1) tma_load_2d(dst + acc * (128 * BK * 2), &tmA, fb, kb * BK, row);
+            else tma_load_2d_pair(dst + acc * (128 * BK * 2), &tmA, fb, kb * BK, row);
           }
-          issued_mask |= 1u << stage;
-          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-          if (++stage == S) { stage = 0; phase ^= 1u; }
+          issued_mask |= 1u << s;
+          issued_phase = (issued_phase & ~(1u << s)) | (ph << s);
         }
       }
-      // Drain: every issued copy must land before the CTA may exit.
-      for (int s = 0; s < S; ++s)
-        if (issued_mask & (1u << s)) mbar_wait_drain(full_raw(s), (issued_phase >> s) & 1u);
+      if (cta == 0)
+        for (int s = 0; s < SA; ++s)
+          if (issued_mask & (1u << s)) mbar_wait_drain(full_a(s), (issued_phase >> s) & 1u);
+    } else if (lane == 1) {
+      // ---------------------------------------------------------- TMA: raw W tiles (to the producers)
+      uint32_t q = 0, issued_mask = 0, issued_phase = 0;
+      bool ok = true;
+      for (int t = cluster; ok && t < num_tiles; t += nclusters) {
+        const int32_t n0 = (t / args.num_m_tiles) * BN + cta * Cfg::kBRows;
+        for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
+          const uint32_t s = q % SW, ph = (q / SW) & 1u;
+          if (!mbar_wait(empty_w(s), ph ^ 1u, wc)) { ok = false; break; }
+          mbar_arrive_expect_tx(raw_w(s), Cfg::kWBytes);
+          const uint32_t dst = w_base + s * Cfg::kWBytes;
+          if constexpr (!B_MN) {
+            tma_load_2d(dst, &tmW, raw_w(s), kb * BK, n0);
+          } else {
+#pragma unroll
+            for (int b = 0; b < Cfg::kBRows / 64; ++b) tma_load_2d(dst + b * 8192, &tmW, raw_w(s), n0 + 64 * b, kb * BK);
+          }
+          issued_mask |= 1u << s;
+          issued_phase = (issued_phase & ~(1u << s)) | (ph << s);
+        }
+      }
+      for (int s = 0; s < SW; ++s)
+        if (issued_mask & (1u << s)) mbar_wait_drain(raw_w(s), (issued_phase >> s) & 1u);
     }
-  } else if (warp == Cfg::kEpiWarps + 1) {
+  } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer (even CTA)
     if (cta == 0 && lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(Cfg::kRowsPerAcc, BN, false, B_MN);
-      uint32_t stage = 0, phase = 0, it = 0;
+      uint32_t q = 0, it = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters, ++it) {
         if (!mbar_wait(tmem_empty_bar, (it & 1u) ^ 1u, wc)) break;
         tc_fence_after();
-        for (int kb = 0; kb < args.num_k_blocks; ++kb) {
-          if (!mbar_wait(full(stage), phase, wc)) { ok = false; break; }
+        for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
+          const uint32_t sa = q % SA, pa = (q / SA) & 1u, sw = q % SW, pw = (q / SW) & 1u;
+          if (!mbar_wait(full_a(sa), pa, wc) || !mbar_wait(full_w(sw), pw, wc)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t sa = base + stage * Cfg::kStageBytes;
-          const uint32_t sb = sa + Cfg::kABytes;
+          const uint32_t aa = a_base + sa * Cfg::kABytes, ww = w_base + sw * Cfg::kWBytes;
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t bdesc = B_MN ? smem_desc_sw128(sb + kk * 2048, 8192, 1024)
-                                        : smem_desc_sw128(sb + kk * 32, 16, 1024);
+            const uint64_t bdesc = B_MN ? smem_desc_sw128(ww + kk * 2048, 8192, 1024)
+                                        : smem_desc_sw128(ww + kk * 32, 16, 1024);
 #pragma unroll
             for (int acc = 0; acc < NACC; ++acc) {
-              const uint64_t adesc = smem_desc_sw128(sa + acc * (128 * BK * 2) + kk * 32, 16, 1024);
+              const uint64_t adesc = smem_desc_sw128(aa + acc * (128 * BK * 2) + kk * 32, 16, 1024);
               umma_bf16<CG>(tmem_base + acc * BN, adesc, bdesc, idesc, (kb | kk) != 0 ? 1u : 0u);
             }
           }
-          umma_commit<CG>(empty(stage));
-          if (++stage == S) { stage = 0; phase ^= 1u; }
+          umma_commit<CG>(empty_a(sa));
+          umma_commit<CG>(empty_w(sw));
         }
         if (ok) umma_commit<CG>(tmem_full_bar);
       }
@@ -236,7 +293,7 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
     }
   } else if (warp < Cfg::kEpiWarps) {
     // ------------------------------------------------------------ epilogue
-    const int q = warp;  // TMEM lane quarter
+    const int qd = warp;  // TMEM lane quarter
     uint32_t it = 0;
     for (int t = cluster; t < num_tiles; t += nclusters, ++it) {
       const int m_blk = t % args.num_m_tiles, n_blk = t / args.num_m_tiles;
@@ -244,11 +301,11 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
       tc_fence_after();
 #pragma unroll 1
       for (int acc = 0; acc < NACC; ++acc) {
-        const int64_t row = (int64_t)m_blk * Cfg::kTileRows + acc * Cfg::kRowsPerAcc + cta * 128 + q * 32 + lane;
+        const int64_t row = (int64_t)m_blk * Cfg::kTileRows + acc * Cfg::kRowsPerAcc + cta * 128 + qd * 32 + lane;
 #pragma unroll 1
         for (int c = 0; c < BN / 32; ++c) {
           uint32_t r[32];
-          tmem_ld32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN + c * 32, r);
+          tmem_ld32(tmem_base + (static_cast<uint32_t>(qd * 32) << 16) + acc * BN + c * 32, r);
           tmem_ld_wait();
           const int64_t col = (int64_t)n_blk * BN + c * 32;
           if (row < args.M && col < args.ncols) store_bf16x32(args.C + row * args.ncols + col, r, args.ncols - col);
@@ -260,55 +317,78 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ operand producers
-    const int tt = threadIdx.x - 32 * (Cfg::kEpiWarps + 2);
-    const int row = tt / CG;                 // 128-byte smem row of the operand tile
-    const int c_begin = (tt % CG) * (8 / CG);
+    // Within its group, each thread owns one row (CG 1) or half a row (CG 2) of the stage's
+    // raw W tile and rewrites it in place as the Eq. 6 weight.  A row holds 64 consecutive K
+    // elements of one W row, so it lies in one group.  Rows outside W were zero-filled by
+    // the copy and stay 0.
+    constexpr int CPT = Cfg::kChunksPerThread;
+    const int pw = warp - (Cfg::kEpiWarps + 2);  // producer warp index
+    const int grp = pw / Cfg::kGroupWarps;       // this warp's group: stages grp, grp + 2, ...
+    const int tt = threadIdx.x - 32 * (Cfg::kEpiWarps + 2) - grp * Cfg::kGroupThreads;
+    const int row = tt / Cfg::kThreadsPerRow;
+    const int c_begin = (tt % Cfg::kThreadsPerRow) * CPT;
     const LayerDev& L = args.L;
     const int32_t phase_t = args.sc.phase;
-    int64_t cached_j = -1;
+    const bool transform = phase_t != PHASE_TEACHER;
+    // stage q of this CTA's sequence is k block q % num_k_blocks of its (q / num_k_blocks)-th tile
+    auto advance = [&](int& t, int& kb, int steps) {
+      kb += steps;
+      while (kb >= args.num_k_blocks) {
+        kb -= args.num_k_blocks;
+        t += nclusters;
+      }
+    };
+    int t = cluster, kb = 0;
+    advance(t, kb, grp);
+    uint32_t q = grp;
+    RowRef cur{};
+    GroupRaw raw{};
+    int64_t j_raw = -1, j_have = -1;
     ProducerConst pc{};
-    uint32_t stage = 0, phase = 0;
-    bool ok = true;
-    for (int t = cluster; ok && t < num_tiles; t += nclusters) {
-      const int n_blk = t / args.num_m_tiles;
-      for (int kb = 0; kb < args.num_k_blocks; ++kb) {
-        int64_t n, kc;
-        if constexpr (!B_MN) {
-          n = (int64_t)n_blk * BN + cta * Cfg::kBRows + row;
-          kc = (int64_t)kb * BK;
-        } else {
-          n = (int64_t)kb * BK + (row & 63);
-          kc = (int64_t)n_blk * BN + cta * Cfg::kBRows + 64 * (row >> 6);
-        }
-        const bool live = phase_t != PHASE_TEACHER && n < L.N && kc < L.K;
-        if (live) {
-          const int64_t j = n * L.groups_per_row + kc / L.g;
-          if (j != cached_j) {
-            pc = producer_const(group_const(L, j), args.sc.s, args.sc.inv_2tanh_s, phase_t);
-            cached_j = j;
-          }
-        }
-        if (!mbar_wait(full_raw(stage), phase, wc)) { ok = false; break; }
-        if (live) {
-          uint8_t* rowp = base_ptr + stage * Cfg::kStageBytes + Cfg::kABytes + row * 128;
+    if (t < num_tiles) {
+      cur = operand_row<CG, B_MN>(args, cta, row, t, kb);
+      if (transform && cur.valid) {
+        raw = group_raw(L, cur.j);
+        j_raw = cur.j;
+      }
+    }
+    while (t < num_tiles) {
+      const uint32_t s = q % SW, ph = (q / SW) & 1u;
+      const bool live = transform && cur.valid;
+      if (live && cur.j != j_have) {
+        pc = producer_const(group_const(raw), args.sc.s, args.sc.inv_2tanh_s, phase_t);
+        j_have = cur.j;
+      }
+      if (!mbar_wait(raw_w(s), ph, wc)) break;
+      if (live) {
+        uint8_t* rowp = base_ptr + (w_base - base) + s * Cfg::kWBytes + row * 128;
+        uint4 v[CPT];
 #pragma unroll
-          for (int i = 0; i < 8 / CG; ++i) {
-            const int phys = (c_begin + i) ^ (row & 7);
-            uint4* p = reinterpret_cast<uint4*>(rowp + phys * 16);
-            *p = transform_chunk_bf16(*p, pc, phase_t);
-          }
-          fence_proxy_async_smem();
+        for (int i = 0; i < CPT; ++i) v[i] = *reinterpret_cast<const uint4*>(rowp + (((c_begin + i) ^ (row & 7)) * 16));
+#pragma unroll
+        for (int i = 0; i < CPT; ++i)
+          *reinterpret_cast<uint4*>(rowp + (((c_begin + i) ^ (row & 7)) * 16)) = transform_chunk_bf16(v[i], pc, phase_t);
+        fence_proxy_async_smem();
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(leader_full_w0 + 8u * s);
+      // This group's next stage; its group inputs are requested now, after this stage's
+      // proxy fence (which would otherwise wait for them), and land during the next wait.
+      q += Cfg::kProdGroups;
+      advance(t, kb, Cfg::kProdGroups);
+      if (t < num_tiles) {
+        cur = operand_row<CG, B_MN>(args, cta, row, t, kb);
+        if (transform && cur.valid && cur.j != j_raw) {
+          raw = group_raw(L, cur.j);
+          j_raw = cur.j;
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive_cluster(leader_full0 + 8u * stage);
-        if (++stage == S) { stage = 0; phase ^= 1u; }
       }
     }
   }
 
   tc_fence_before();
   if constexpr (CG == 2) cluster_sync_all(); else __syncthreads();
-  if (warp == Cfg::kEpiWarps + 1) {
+  if (warp == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc<CG>(tmem_base, kTmemCols);
   }
@@ -577,7 +657,7 @@ WaitCtl make_wait_ctl(const DeviceInfo& d) {
 
 template <typename Kern>
 cudaError_t launch_persistent(Kern kern, int cg, int grid_ctas, int threads, int smem, cudaStream_t st,
-                              const CUtensorMap& a, const CUtensorMap& b, const void* args_ptr) {
+                              void** params) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg{};
@@ -592,7 +672,6 @@ cudaError_t launch_persistent(Kern kern, int cg, int grid_ctas, int threads, int
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  void* params[3] = {const_cast<CUtensorMap*>(&a), const_cast<CUtensorMap*>(&b), const_cast<void*>(args_ptr)};
   return cudaLaunchKernelExC(&cfg, reinterpret_cast<const void*>(kern), params);
 }
 
@@ -607,12 +686,12 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
   using Cfg = FusedCfg<CG>;
   DeviceInfo& d = device_info();
   if (!d.ok) return cudaErrorInvalidDevice;
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tw;
   if (!make_tmap(&ta, A, depth, M, BK, 128)) return cudaErrorInvalidValue;
   if constexpr (!B_MN) {
-    if (!make_tmap(&tb, L.W, L.K, L.N, BK, Cfg::kBRows)) return cudaErrorInvalidValue;
+    if (!make_tmap(&tw, L.W, L.K, L.N, BK, Cfg::kBRows)) return cudaErrorInvalidValue;
   } else {
-    if (!make_tmap(&tb, L.W, L.K, L.N, 64, BK)) return cudaErrorInvalidValue;
+    if (!make_tmap(&tw, L.W, L.K, L.N, 64, BK)) return cudaErrorInvalidValue;
   }
   FusedArgs args;
   args.L = L;
@@ -626,8 +705,9 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
   args.wc = make_wait_ctl(d);
   const int tiles = args.num_m_tiles * args.num_n_tiles;
   const int clusters = std::min(tiles, d.sm_count / CG);
-  return launch_persistent(fused_gemm_kernel<CG, B_MN>, CG, clusters * CG, Cfg::kThreads, Cfg::kSmemBytes, st, ta,
-                           tb, &args);
+  void* params[3] = {&ta, &tw, &args};
+  return launch_persistent(fused_gemm_kernel<CG, B_MN>, CG, clusters * CG, Cfg::kThreads, Cfg::kSmemBytes, st,
+                           params);
 }
 
 template <int CG>
@@ -653,7 +733,8 @@ cudaError_t run_dw(const LayerDev& L, StepScalars sc, const void* X, const void*
   args.wc = make_wait_ctl(d);
   const int tiles = args.num_n_tiles * args.num_k_tiles * args.splits;
   const int clusters = std::min(tiles, d.sm_count / CG);
-  return launch_persistent(dw_kernel<CG>, CG, clusters * CG, Cfg::kThreads, Cfg::kSmemBytes, st, tdy, tx, &args);
+  void* params[3] = {&tdy, &tx, &args};
+  return launch_persistent(dw_kernel<CG>, CG, clusters * CG, Cfg::kThreads, Cfg::kSmemBytes, st, params);
 }
 
 }  // namespace
