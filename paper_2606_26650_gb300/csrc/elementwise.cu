@@ -77,6 +77,19 @@ __device__ __forceinline__ Sum2 sum2_team(Sum2 v, int team) {
 
 __device__ __forceinline__ double sum2_value(Sum2 v) { return static_cast<double>(v.hi) + static_cast<double>(v.lo); }
 
+// Rounded once to fp32 (all a stored fp32 statistic needs; avoids fp64 arithmetic).
+__device__ __forceinline__ float sum2_float(Sum2 v) { return v.hi + v.lo; }
+
+// mu0, alpha0, Delta0 of one group from its compensated sums (Eq. 3; TWN rule of §2.2).
+__device__ __forceinline__ void store_group_stats(int64_t j, int32_t g, int32_t thr_init, float mu, Sum2 dev,
+                                                  Sum2 mag, float* mu0, float* alpha0, float* delta0) {
+  const float inv_g = 1.0f / static_cast<float>(g);
+  const float a0 = sum2_float(dev) * inv_g;
+  mu0[j] = mu;
+  alpha0[j] = a0;
+  delta0[j] = (thr_init == 1 && a0 > 0.0f) ? 0.7f * (sum2_float(mag) * inv_g) / a0 : 0.5f;
+}
+
 // ---------------------------------------------------------------- Eq. 3 statistics
 // Register variant: a team of `team` lanes owns one group and keeps its R x 16-byte
 // vectors in registers (mean, then deviations, without re-reading W).
@@ -109,7 +122,7 @@ __global__ void __launch_bounds__(kThreads) group_stats_reg_kernel(const T* __re
       for (int q = 0; q < V; ++q) sum2_add(sum, v[r][q]);
     }
     sum = sum2_team(sum, team);
-    const float mu = static_cast<float>(sum2_value(sum) / g);
+    const float mu = sum2_float(sum) / static_cast<float>(g);
     Sum2 dev{0.f, 0.f}, mag{0.f, 0.f};
 #pragma unroll
     for (int r = 0; r < R; ++r)
@@ -120,12 +133,7 @@ __global__ void __launch_bounds__(kThreads) group_stats_reg_kernel(const T* __re
       }
     dev = sum2_team(dev, team);
     mag = sum2_team(mag, team);
-    if (live && sub == 0) {
-      const double a0 = sum2_value(dev) / g;
-      mu0[j] = mu;
-      alpha0[j] = static_cast<float>(a0);
-      delta0[j] = (thr_init == 1 && a0 > 0.0) ? static_cast<float>(0.7 * (sum2_value(mag) / g) / a0) : 0.5f;
-    }
+    if (live && sub == 0) store_group_stats(j, g, thr_init, mu, dev, mag, mu0, alpha0, delta0);
   }
 }
 
@@ -149,7 +157,7 @@ __global__ void __launch_bounds__(kThreads) group_stats_stream_kernel(const T* _
       for (int q = 0; q < V; ++q) sum2_add(sum, v[q]);
     }
     sum = sum2_team(sum, 32);
-    const float mu = static_cast<float>(sum2_value(sum) / g);
+    const float mu = sum2_float(sum) / static_cast<float>(g);
     Sum2 dev{0.f, 0.f}, mag{0.f, 0.f};
     for (int i = lane * V; i < g; i += 32 * V) {
       float v[V];
@@ -162,12 +170,7 @@ __global__ void __launch_bounds__(kThreads) group_stats_stream_kernel(const T* _
     }
     dev = sum2_team(dev, 32);
     mag = sum2_team(mag, 32);
-    if (lane == 0) {
-      const double a0 = sum2_value(dev) / g;
-      mu0[j] = mu;
-      alpha0[j] = static_cast<float>(a0);
-      delta0[j] = (thr_init == 1 && a0 > 0.0) ? static_cast<float>(0.7 * (sum2_value(mag) / g) / a0) : 0.5f;
-    }
+    if (lane == 0) store_group_stats(j, g, thr_init, mu, dev, mag, mu0, alpha0, delta0);
   }
 }
 

@@ -72,14 +72,18 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_bar) {
   asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar) : "memory");
 }
 
+// One bounded poll: the thread may be suspended until the phase completes or `kSuspendNs`
+// passes, so waiting warps do not spin on issue slots and shared-memory bandwidth.
+constexpr uint32_t kSuspendNs = 200000;
+
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(bar), "r"(parity)
+      : "r"(bar), "r"(parity), "r"(kSuspendNs)
       : "memory");
   return ok != 0;
 }
@@ -106,14 +110,12 @@ __device__ __noinline__ void signal_timeout(const WaitCtl& w) {
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const WaitCtl& w) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
-  for (uint32_t it = 1;; ++it) {
+  for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 255u) == 0u) {
-      if (aborted(w)) return false;
-      if (globaltimer_ns() - t0 > w.timeout_ns) {
-        signal_timeout(w);
-        return false;
-      }
+    if (aborted(w)) return false;
+    if (globaltimer_ns() - t0 > w.timeout_ns) {
+      signal_timeout(w);
+      return false;
     }
   }
 }

@@ -126,29 +126,69 @@ __device__ __forceinline__ void store_bf16x32(uint16_t* dst, const uint32_t (&r)
 
 // ============================================================================ fused kernel
 
-// Producer-side view of one 128-byte operand row for one pipeline stage: which W row and
-// which 64-element K chunk it holds, and its group.
-struct RowRef {
-  int64_t n, kc, j;
-  bool valid;
-};
-
+// Walks the pipeline stages one producer thread handles (every kProdGroups-th stage of its
+// CTA's tile sequence) and tracks which W row, K chunk and group its 128-byte operand row
+// holds.  Divisions happen once per tile; each stage step is a few integer adds.
 template <int CG, bool B_MN>
-__device__ __forceinline__ RowRef operand_row(const FusedArgs& a, uint32_t cta, int row, int t, int kb) {
+struct OperandRowIter {
   using Cfg = FusedCfg<CG>;
-  const int n_blk = t / a.num_m_tiles;
-  RowRef r;
-  if constexpr (!B_MN) {  // forward: rows are output features n, the stage is a K chunk
-    r.n = (int64_t)n_blk * BN + cta * Cfg::kBRows + row;
-    r.kc = (int64_t)kb * BK;
-  } else {  // dX: rows are the contraction index n, 64-column blocks of output features k
-    r.n = (int64_t)kb * BK + (row & 63);
-    r.kc = (int64_t)n_blk * BN + cta * Cfg::kBRows + 64 * (row >> 6);
+  int t, kb;      // tile index, k block
+  int64_t n, kc;  // W row, first K column of the 64-element chunk
+  int64_t j;      // group index of (n, kc)
+  int kin;        // forward: k blocks into the current group (kc / 64 mod g / 64)
+  bool tile_ok;   // forward: n < N; dX: kc < K
+
+  __device__ __forceinline__ void init(const FusedArgs& a, uint32_t cta, int row, int t_, int kb_) {
+    t = t_;
+    kb = kb_;
+    const int n_blk = t / a.num_m_tiles;
+    const int gk = a.L.g / BK;  // k blocks per group
+    if constexpr (!B_MN) {
+      n = (int64_t)n_blk * BN + cta * Cfg::kBRows + row;
+      kc = (int64_t)kb * BK;
+      tile_ok = n < a.L.N;
+      j = n * a.L.groups_per_row + kb / gk;
+      kin = kb % gk;
+    } else {
+      n = (int64_t)kb * BK + (row & 63);
+      kc = (int64_t)n_blk * BN + cta * Cfg::kBRows + 64 * (row >> 6);
+      tile_ok = kc < a.L.K;
+      j = n * a.L.groups_per_row + kc / a.L.g;
+      kin = 0;
+    }
   }
-  r.valid = r.n < a.L.N && r.kc < a.L.K;
-  r.j = r.n * a.L.groups_per_row + r.kc / a.L.g;
-  return r;
-}
+
+  __device__ __forceinline__ bool live(const FusedArgs& a, int num_tiles) const { return t < num_tiles; }
+  __device__ __forceinline__ bool valid(const FusedArgs& a) const {
+    if constexpr (!B_MN) return tile_ok;
+    else return tile_ok && n < a.L.N;
+  }
+
+  __device__ __forceinline__ void step(const FusedArgs& a, uint32_t cta, int row, uint32_t nclusters, int steps) {
+    kb += steps;
+    if (kb >= a.num_k_blocks) {
+      int t2 = t, kb2 = kb;
+      while (kb2 >= a.num_k_blocks) {
+        kb2 -= a.num_k_blocks;
+        t2 += nclusters;
+      }
+      init(a, cta, row, t2, kb2);
+      return;
+    }
+    if constexpr (!B_MN) {
+      kc += (int64_t)steps * BK;
+      kin += steps;
+      const int gk = a.L.g / BK;
+      while (kin >= gk) {
+        kin -= gk;
+        ++j;
+      }
+    } else {
+      n += (int64_t)steps * BK;
+      j += (int64_t)steps * BK * a.L.groups_per_row;
+    }
+  }
+};
 
 template <int CG, bool B_MN>
 __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
@@ -319,47 +359,54 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
     // ------------------------------------------------------------ operand producers
     // Within its group, each thread owns one row (CG 1) or half a row (CG 2) of the stage's
     // raw W tile and rewrites it in place as the Eq. 6 weight.  A row holds 64 consecutive K
-    // elements of one W row, so it lies in one group.  Rows outside W were zero-filled by
-    // the copy and stay 0.
+    // elements of one W row, so it lies in one group (g is a multiple of 64).  Rows outside
+    // W were zero-filled by the copy and stay 0.
     constexpr int CPT = Cfg::kChunksPerThread;
+    constexpr int PG = Cfg::kProdGroups;
     const int pw = warp - (Cfg::kEpiWarps + 2);  // producer warp index
-    const int grp = pw / Cfg::kGroupWarps;       // this warp's group: stages grp, grp + 2, ...
+    const int grp = pw / Cfg::kGroupWarps;       // this warp's group: stages grp, grp + PG, ...
     const int tt = threadIdx.x - 32 * (Cfg::kEpiWarps + 2) - grp * Cfg::kGroupThreads;
     const int row = tt / Cfg::kThreadsPerRow;
     const int c_begin = (tt % Cfg::kThreadsPerRow) * CPT;
     const LayerDev& L = args.L;
     const int32_t phase_t = args.sc.phase;
     const bool transform = phase_t != PHASE_TEACHER;
-    // stage q of this CTA's sequence is k block q % num_k_blocks of its (q / num_k_blocks)-th tile
-    auto advance = [&](int& t, int& kb, int steps) {
-      kb += steps;
-      while (kb >= args.num_k_blocks) {
-        kb -= args.num_k_blocks;
-        t += nclusters;
+    // `cur` is the stage being produced; `ahead` runs two of this thread's stages ahead and
+    // requests that stage's group inputs, so an L2 round trip is hidden behind two stages.
+    OperandRowIter<CG, B_MN> cur, ahead;
+    cur.init(args, cta, row, cluster, 0);
+    cur.step(args, cta, row, nclusters, grp);
+    ahead = cur;
+    GroupRaw raw0{}, raw1{};
+    int64_t j0 = -1, j1 = -1;
+    auto request = [&](const OperandRowIter<CG, B_MN>& it, GroupRaw& dst, int64_t& jd, const GroupRaw& other,
+                       int64_t jo) {
+      if (transform && it.live(args, num_tiles) && it.valid(args)) {
+        if (jo == it.j) dst = other;
+        else dst = group_raw(L, it.j);
+        jd = it.j;
       }
     };
-    int t = cluster, kb = 0;
-    advance(t, kb, grp);
-    uint32_t q = grp;
-    RowRef cur{};
-    GroupRaw raw{};
-    int64_t j_raw = -1, j_have = -1;
+    request(ahead, raw0, j0, raw1, j1);
+    ahead.step(args, cta, row, nclusters, PG);
+    request(ahead, raw1, j1, raw0, j0);
+    ahead.step(args, cta, row, nclusters, PG);
+    int64_t j_have = -1;
     ProducerConst pc{};
-    if (t < num_tiles) {
-      cur = operand_row<CG, B_MN>(args, cta, row, t, kb);
-      if (transform && cur.valid) {
-        raw = group_raw(L, cur.j);
-        j_raw = cur.j;
-      }
-    }
-    while (t < num_tiles) {
+    uint32_t q = grp;
+    bool ok = true;
+    // One stage: consume `mine` (requested two stages ago), then refill it two stages ahead.
+    auto produce = [&](GroupRaw& mine, int64_t& jm, const GroupRaw& other, int64_t jo) {
       const uint32_t s = q % SW, ph = (q / SW) & 1u;
-      const bool live = transform && cur.valid;
+      const bool live = transform && cur.valid(args);
       if (live && cur.j != j_have) {
-        pc = producer_const(group_const(raw), args.sc.s, args.sc.inv_2tanh_s, phase_t);
+        pc = producer_const(group_const(mine), args.sc.s, args.sc.inv_2tanh_s, phase_t);
         j_have = cur.j;
       }
-      if (!mbar_wait(raw_w(s), ph, wc)) break;
+      if (!mbar_wait(raw_w(s), ph, wc)) {
+        ok = false;
+        return;
+      }
       if (live) {
         uint8_t* rowp = base_ptr + (w_base - base) + s * Cfg::kWBytes + row * 128;
         uint4 v[CPT];
@@ -372,17 +419,16 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
       }
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(leader_full_w0 + 8u * s);
-      // This group's next stage; its group inputs are requested now, after this stage's
-      // proxy fence (which would otherwise wait for them), and land during the next wait.
-      q += Cfg::kProdGroups;
-      advance(t, kb, Cfg::kProdGroups);
-      if (t < num_tiles) {
-        cur = operand_row<CG, B_MN>(args, cta, row, t, kb);
-        if (transform && cur.valid && cur.j != j_raw) {
-          raw = group_raw(L, cur.j);
-          j_raw = cur.j;
-        }
-      }
+      // Issued after the proxy fence, which would otherwise wait for these loads.
+      request(ahead, mine, jm, other, jo);
+      ahead.step(args, cta, row, nclusters, PG);
+      q += PG;
+      cur.step(args, cta, row, nclusters, PG);
+    };
+    while (ok && cur.live(args, num_tiles)) {
+      produce(raw0, j0, raw1, j1);
+      if (!ok || !cur.live(args, num_tiles)) break;
+      produce(raw1, j1, raw0, j0);
     }
   }
 
