@@ -154,6 +154,28 @@ catq_status catq_soft_ternary_linear_bwd(const catq_layer* layer, catq_schedule 
                                          float* g_dalpha, float* g_ddelta, void* workspace,
                                          size_t ws_bytes, catq_stream stream);
 
+/* Allocation-free backward (this library's addition; the paper has no counterpart).
+ * For callers that cannot allocate device memory themselves, e.g. a host runtime without
+ * access to a device allocator, or a service whose device memory is fixed when it starts:
+ * identical to catq_soft_ternary_linear_bwd except that the partial group sums live in a
+ * scratch array inside the library (catq_bwd_noalloc_max_scratch_bytes() = 16 MiB, held
+ * by every GPU that loads the library until the process exits) instead of a workspace.
+ *   - Calls needing more scratch than that (catq_bwd_workspace_bytes(layer, M) > 16 MiB)
+ *     return CATQ_ERR_WORKSPACE before launching anything.
+ *   - The first call on a device looks up the array's device address on that device (make
+ *     it before any stream capture); this call allocates nothing, neither does any other.
+ *   - All calls share the one array: calls whose kernels overlap on the GPU (e.g. on two
+ *     streams) race and give wrong gradients.  Calls in order on one stream are safe; the
+ *     array keeps the last call's contents, which every call overwrites before reading. */
+catq_status catq_soft_ternary_linear_bwd_noalloc(const catq_layer* layer, catq_schedule sched,
+                                                 const void* X, const void* dY, int64_t M,
+                                                 int32_t x_dtype, void* dX, float* g_dmu,
+                                                 float* g_dalpha, float* g_ddelta,
+                                                 catq_stream stream);
+
+/* Size in bytes of the scratch array catq_soft_ternary_linear_bwd_noalloc uses. */
+size_t catq_bwd_noalloc_max_scratch_bytes(void);
+
 /* Workspace bytes catq_recon_loss needs for `count` elements (block partial sums). */
 size_t catq_recon_loss_workspace_bytes(int64_t count);
 

@@ -72,6 +72,8 @@ def lib() -> ctypes.CDLL:
         "catq_recon_loss": (I32, [P, P, I64, I32, I32, P, P, P, S, P]),
         "catq_hard_ternarize_pack": (I32, [LP, P, P, P]),
         "catq_device_status": (I32, [P, ctypes.POINTER(I32)]),
+        "catq_soft_ternary_linear_bwd_noalloc": (I32, [LP, catq_schedule, P, P, I64, I32, P, P, P, P, P]),
+        "catq_bwd_noalloc_max_scratch_bytes": (S, []),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -193,6 +195,19 @@ def catq_soft_ternary_linear_bwd(layer: Layer, sched: catq_schedule, X, dY, dX=N
                                               _dtype_code(X), _ptr(dX), _ptr(g_dmu), _ptr(g_dalpha),
                                               _ptr(g_ddelta), _ptr(workspace), ws_bytes, _stream(stream)),
            "catq_soft_ternary_linear_bwd")
+
+
+def catq_soft_ternary_linear_bwd_noalloc(layer: Layer, sched: catq_schedule, X, dY, dX=None, g_dmu=None,
+                                         g_dalpha=None, g_ddelta=None, stream=None):
+    st = layer.struct()
+    _check(lib().catq_soft_ternary_linear_bwd_noalloc(ctypes.byref(st), sched, _ptr(X), _ptr(dY), X.shape[0],
+                                                      _dtype_code(X), _ptr(dX), _ptr(g_dmu), _ptr(g_dalpha),
+                                                      _ptr(g_ddelta), _stream(stream)),
+           "catq_soft_ternary_linear_bwd_noalloc")
+
+
+def catq_bwd_noalloc_max_scratch_bytes() -> int:
+    return int(lib().catq_bwd_noalloc_max_scratch_bytes())
 
 
 def catq_recon_loss_workspace_bytes(count: int) -> int:

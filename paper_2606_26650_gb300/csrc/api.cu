@@ -5,6 +5,7 @@
 
 #include <cmath>
 #include <cstdint>
+#include <mutex>
 
 #include "catq.h"
 #include "launch.h"
@@ -100,6 +101,28 @@ size_t bwd_partials_bytes(const catq_layer* L, int64_t M, TcPlan* plan_out, int3
   if (P_out) *P_out = P;
   if (splits_out) *splits_out = 1;
   return 3 * static_cast<size_t>(L->N) * static_cast<size_t>(L->K / P) * sizeof(float);
+}
+
+// Scratch of catq_soft_ternary_linear_bwd_noalloc: the dW epilogue's partial group sums.
+// Every GPU that loads the library holds this array until the process exits.
+constexpr size_t kNoAllocScratchBytes = size_t(16) << 20;
+static __device__ __align__(256) unsigned char g_bwd_scratch[kNoAllocScratchBytes];
+
+// Device address of g_bwd_scratch on the current device, looked up once per device with
+// that device current (host code cannot use the array's name as a device address).
+catq_status noalloc_scratch(void** out) {
+  static std::mutex mu;
+  static void* addr[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return CATQ_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_bwd_scratch) != cudaSuccess || !p) return CATQ_ERR_CUDA;
+    addr[dev] = p;
+  }
+  *out = addr[dev];
+  return CATQ_OK;
 }
 
 }  // namespace
@@ -218,6 +241,26 @@ catq_status catq_soft_ternary_linear_bwd(const catq_layer* layer, catq_schedule 
   if (e != cudaSuccess) return CATQ_ERR_CUDA;
   return cuda_status(launch_grad_reduce(L, sc, part, splits, P, g_dmu, g_dalpha, g_ddelta, s));
 }
+
+catq_status catq_soft_ternary_linear_bwd_noalloc(const catq_layer* layer, catq_schedule sched, const void* X,
+                                                 const void* dY, int64_t M, int32_t x_dtype, void* dX,
+                                                 float* g_dmu, float* g_dalpha, float* g_ddelta,
+                                                 catq_stream stream) {
+  // Same validation and kernels as catq_soft_ternary_linear_bwd; only the scratch differs.
+  catq_status st = check_layer(layer, sched.phase != CATQ_PHASE_TEACHER);
+  if (st != CATQ_OK) return st;
+  const bool want_grads = g_dmu || g_dalpha || g_ddelta;
+  if (!want_grads || sched.phase == CATQ_PHASE_TEACHER || M <= 0)
+    return catq_soft_ternary_linear_bwd(layer, sched, X, dY, M, x_dtype, dX, g_dmu, g_dalpha, g_ddelta, nullptr,
+                                        0, stream);
+  if (bwd_partials_bytes(layer, M, nullptr, nullptr, nullptr) > kNoAllocScratchBytes) return CATQ_ERR_WORKSPACE;
+  void* scratch = nullptr;
+  if ((st = noalloc_scratch(&scratch)) != CATQ_OK) return st;
+  return catq_soft_ternary_linear_bwd(layer, sched, X, dY, M, x_dtype, dX, g_dmu, g_dalpha, g_ddelta, scratch,
+                                      kNoAllocScratchBytes, stream);
+}
+
+size_t catq_bwd_noalloc_max_scratch_bytes(void) { return kNoAllocScratchBytes; }
 
 size_t catq_recon_loss_workspace_bytes(int64_t count) {
   return round256(static_cast<size_t>(recon_loss_blocks(count < 1 ? 1 : count)) * sizeof(double));
