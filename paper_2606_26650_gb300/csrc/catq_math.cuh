@@ -116,12 +116,14 @@ __device__ __forceinline__ float tanh_fast(float x) {
 }
 
 // Eq. 5/6 SOFT weight alpha f(What; s, Delta) for two bf16 weights, fp32 arithmetic with
-// the hardware tanh, rounded once to bf16.
+// the hardware tanh, rounded once to bf16.  ONE_TANH selects the one-tanh form (valid when
+// p.one_tanh); the choice is made once per row, outside the element loop.
+template <bool ONE_TANH>
 __device__ __forceinline__ uint32_t soft_pair_bf16(uint32_t w2, const ProducerConst& p) {
   const float u0 = fmaf(bf16lo_to_f32(w2), p.A, p.B);
   const float u1 = fmaf(bf16hi_to_f32(w2), p.A, p.B);
   float y0, y1;
-  if (p.one_tanh) {
+  if constexpr (ONE_TANH) {
     const float c0 = copysignf(p.C, u0), c1 = copysignf(p.C, u1);
     y0 = fmaf(tanh_fast(fabsf(u0) - p.D), c0, c0);
     y1 = fmaf(tanh_fast(fabsf(u1) - p.D), c1, c1);
@@ -141,19 +143,43 @@ __device__ __forceinline__ uint32_t hard_pair_bf16(uint32_t w2, const ProducerCo
   return pack_bf16x2(y0, y1);
 }
 
-__device__ __forceinline__ uint4 transform_chunk_bf16(uint4 v, const ProducerConst& p, int32_t phase) {
-  if (phase == PHASE_SOFT) {
-    v.x = soft_pair_bf16(v.x, p);
-    v.y = soft_pair_bf16(v.y, p);
-    v.z = soft_pair_bf16(v.z, p);
-    v.w = soft_pair_bf16(v.w, p);
-  } else if (phase == PHASE_HARD) {
+enum : int32_t { XF_COPY = 0, XF_SOFT1 = 1, XF_SOFT2 = 2, XF_HARD = 3 };
+
+// Which element transform a row uses in `phase`.
+__device__ __forceinline__ int32_t transform_kind(const ProducerConst& p, int32_t phase) {
+  if (phase == PHASE_SOFT) return p.one_tanh ? XF_SOFT1 : XF_SOFT2;
+  return phase == PHASE_HARD ? XF_HARD : XF_COPY;
+}
+
+template <int KIND>
+__device__ __forceinline__ uint4 transform_chunk(uint4 v, const ProducerConst& p) {
+  if constexpr (KIND == XF_SOFT1) {
+    v.x = soft_pair_bf16<true>(v.x, p);
+    v.y = soft_pair_bf16<true>(v.y, p);
+    v.z = soft_pair_bf16<true>(v.z, p);
+    v.w = soft_pair_bf16<true>(v.w, p);
+  } else if constexpr (KIND == XF_SOFT2) {
+    v.x = soft_pair_bf16<false>(v.x, p);
+    v.y = soft_pair_bf16<false>(v.y, p);
+    v.z = soft_pair_bf16<false>(v.z, p);
+    v.w = soft_pair_bf16<false>(v.w, p);
+  } else if constexpr (KIND == XF_HARD) {
     v.x = hard_pair_bf16(v.x, p);
     v.y = hard_pair_bf16(v.y, p);
     v.z = hard_pair_bf16(v.z, p);
     v.w = hard_pair_bf16(v.w, p);
   }
   return v;
+}
+
+// The Eq. 6 operand for one 16-byte chunk of a row (8 bf16 weights of one group).
+__device__ __forceinline__ uint4 transform_chunk_bf16(uint4 v, const ProducerConst& p, int32_t phase) {
+  switch (transform_kind(p, phase)) {
+    case XF_SOFT1: return transform_chunk<XF_SOFT1>(v, p);
+    case XF_SOFT2: return transform_chunk<XF_SOFT2>(v, p);
+    case XF_HARD: return transform_chunk<XF_HARD>(v, p);
+    default: return v;
+  }
 }
 
 // ---------------------------------------------------------------- fp32 path

@@ -27,6 +27,7 @@
 #include <atomic>
 #include <mutex>
 #include <numeric>
+#include <type_traits>
 
 #include "launch.h"
 #include "ptx_sm100.cuh"
@@ -409,12 +410,22 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
       }
       if (live) {
         uint8_t* rowp = base_ptr + (w_base - base) + s * Cfg::kWBytes + row * 128;
-        uint4 v[CPT];
+        // One straight-line transform per row: the kind is uniform over the row's chunks.
+        auto run = [&](auto kind_tag) {
+          constexpr int KIND = decltype(kind_tag)::value;
+          uint4 v[CPT];
 #pragma unroll
-        for (int i = 0; i < CPT; ++i) v[i] = *reinterpret_cast<const uint4*>(rowp + (((c_begin + i) ^ (row & 7)) * 16));
+          for (int i = 0; i < CPT; ++i) v[i] = *reinterpret_cast<const uint4*>(rowp + (((c_begin + i) ^ (row & 7)) * 16));
 #pragma unroll
-        for (int i = 0; i < CPT; ++i)
-          *reinterpret_cast<uint4*>(rowp + (((c_begin + i) ^ (row & 7)) * 16)) = transform_chunk_bf16(v[i], pc, phase_t);
+          for (int i = 0; i < CPT; ++i)
+            *reinterpret_cast<uint4*>(rowp + (((c_begin + i) ^ (row & 7)) * 16)) = transform_chunk<KIND>(v[i], pc);
+        };
+        switch (transform_kind(pc, phase_t)) {
+          case XF_SOFT1: run(std::integral_constant<int, XF_SOFT1>{}); break;
+          case XF_SOFT2: run(std::integral_constant<int, XF_SOFT2>{}); break;
+          case XF_HARD: run(std::integral_constant<int, XF_HARD>{}); break;
+          default: break;
+        }
         fence_proxy_async_smem();
       }
       __syncwarp();
