@@ -198,6 +198,47 @@ catq_status catq_recon_loss(const void* Y, const void* Y_ref, int64_t count, int
 catq_status catq_hard_ternarize_pack(const catq_layer* layer, uint8_t* codes, float* alpha,
                                      catq_stream stream);
 
+/* ------------------------------------------------------------------ grouped (MoE) layers
+ * A mixture-of-experts layer quantizes every expert's linear like a dense one (App. B.2:
+ * experts are quantized, routers are not).  E experts of identical shape are stacked:
+ * W [E, N, K] and the per-group arrays [E, G] (expert e's groups follow expert e-1's), so
+ * catq_group_stats / catq_modulate_ternarize / catq_hard_ternarize_pack apply unchanged to
+ * the stacked layer seen as a dense [E*N, K] layer.  Tokens routed to experts are given
+ * expert-sorted: rows row_offsets[e] .. row_offsets[e+1]-1 of X [R, K] / Y [R, N] belong to
+ * expert e; row_offsets is a HOST array of E+1 non-decreasing int64 values, row_offsets[0]
+ * == 0, row_offsets[E] == R.  Experts with no rows get zero factor gradients. */
+typedef struct {
+  int32_t E;       /* number of experts */
+  int32_t g;       /* group size */
+  int64_t N, K;    /* one expert's out_features, in_features */
+  int32_t w_dtype; /* catq_dtype */
+  int32_t reserved;
+  const void* W;   /* [E, N, K] */
+  float* mu0;      /* [E, G] */
+  float* alpha0;
+  float* delta0;
+  const float* d_mu;
+  const float* d_alpha;
+  const float* d_delta;
+} catq_grouped_layer;
+
+/* Forward of every expert: Y[rows of e] = X[rows of e] Wq_e^T (Eq. 6 weight per expert). */
+catq_status catq_grouped_soft_ternary_linear_fwd(const catq_grouped_layer* layer, catq_schedule sched,
+                                                 const void* X, const int64_t* row_offsets,
+                                                 int32_t x_dtype, void* Y, catq_stream stream);
+
+/* Workspace bytes catq_grouped_soft_ternary_linear_bwd needs (the largest expert's). */
+size_t catq_grouped_bwd_workspace_bytes(const catq_grouped_layer* layer, const int64_t* row_offsets);
+
+/* Backward of every expert (see catq_soft_ternary_linear_bwd): dX [R, K] (nullable) and the
+ * factor gradients [E, G] (all three or none). */
+catq_status catq_grouped_soft_ternary_linear_bwd(const catq_grouped_layer* layer, catq_schedule sched,
+                                                 const void* X, const void* dY,
+                                                 const int64_t* row_offsets, int32_t x_dtype,
+                                                 void* dX, float* g_dmu, float* g_dalpha,
+                                                 float* g_ddelta, void* workspace, size_t ws_bytes,
+                                                 catq_stream stream);
+
 /* Synchronises `stream`, then returns in *out the status latched on the current device
  * since the last call (CATQ_OK if none) and clears it.  The return value reports whether
  * the query itself succeeded. */

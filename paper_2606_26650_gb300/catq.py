@@ -43,6 +43,15 @@ class catq_layer(ctypes.Structure):
     ]
 
 
+class catq_grouped_layer(ctypes.Structure):
+    _fields_ = [
+        ("E", ctypes.c_int32), ("g", ctypes.c_int32), ("N", ctypes.c_int64), ("K", ctypes.c_int64),
+        ("w_dtype", ctypes.c_int32), ("reserved", ctypes.c_int32), ("W", ctypes.c_void_p),
+        ("mu0", ctypes.c_void_p), ("alpha0", ctypes.c_void_p), ("delta0", ctypes.c_void_p),
+        ("d_mu", ctypes.c_void_p), ("d_alpha", ctypes.c_void_p), ("d_delta", ctypes.c_void_p),
+    ]
+
+
 class catq_schedule(ctypes.Structure):
     _fields_ = [("phase", ctypes.c_int32), ("s", ctypes.c_float)]
 
@@ -74,6 +83,11 @@ def lib() -> ctypes.CDLL:
         "catq_device_status": (I32, [P, ctypes.POINTER(I32)]),
         "catq_soft_ternary_linear_bwd_noalloc": (I32, [LP, catq_schedule, P, P, I64, I32, P, P, P, P, P]),
         "catq_bwd_noalloc_max_scratch_bytes": (S, []),
+        "catq_grouped_soft_ternary_linear_fwd": (I32, [ctypes.POINTER(catq_grouped_layer), catq_schedule, P, P, I32, P,
+                                                       P]),
+        "catq_grouped_bwd_workspace_bytes": (S, [ctypes.POINTER(catq_grouped_layer), P]),
+        "catq_grouped_soft_ternary_linear_bwd": (I32, [ctypes.POINTER(catq_grouped_layer), catq_schedule, P, P, P, I32,
+                                                       P, P, P, P, P, S, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -236,3 +250,57 @@ def workspace(nbytes: int, device):
     """A byte tensor of at least nbytes (256-byte aligned by the caching allocator)."""
     import torch
     return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+# ------------------------------------------------------------------ grouped (MoE) layers
+
+@dataclasses.dataclass
+class GroupedLayer:
+    """E experts stacked: W [E, N, K], per-group arrays [E * G] (expert-major).  `dense`
+    views the stack as one [E * N, K] layer for catq_group_stats / pack."""
+    W: object
+    g: int
+    dense: Layer
+
+    @classmethod
+    def create(cls, W, g, d_mu=None, d_alpha=None, d_delta=None):
+        E, N, K = W.shape
+        return cls(W, g, Layer.create(W.reshape(E * N, K), g, d_mu, d_alpha, d_delta))
+
+    @property
+    def E(self):
+        return self.W.shape[0]
+
+    def struct(self) -> catq_grouped_layer:
+        E, N, K = self.W.shape
+        d = self.dense
+        return catq_grouped_layer(E, self.g, N, K, _dtype_code(self.W), 0, self.W.data_ptr(), d.mu0.data_ptr(),
+                                  d.alpha0.data_ptr(), d.delta0.data_ptr(), d.d_mu.data_ptr(), d.d_alpha.data_ptr(),
+                                  d.d_delta.data_ptr())
+
+
+def _offsets(row_offsets):
+    arr = (ctypes.c_int64 * len(row_offsets))(*[int(v) for v in row_offsets])
+    return arr
+
+
+def catq_grouped_soft_ternary_linear_fwd(layer: GroupedLayer, sched: catq_schedule, X, row_offsets, Y, stream=None):
+    st = layer.struct()
+    off = _offsets(row_offsets)
+    _check(lib().catq_grouped_soft_ternary_linear_fwd(ctypes.byref(st), sched, _ptr(X), off, _dtype_code(X), _ptr(Y),
+                                                      _stream(stream)), "catq_grouped_soft_ternary_linear_fwd")
+
+
+def catq_grouped_bwd_workspace_bytes(layer: GroupedLayer, row_offsets) -> int:
+    st = layer.struct()
+    return int(lib().catq_grouped_bwd_workspace_bytes(ctypes.byref(st), _offsets(row_offsets)))
+
+
+def catq_grouped_soft_ternary_linear_bwd(layer: GroupedLayer, sched: catq_schedule, X, dY, row_offsets, dX=None,
+                                         g_dmu=None, g_dalpha=None, g_ddelta=None, workspace=None, stream=None):
+    st = layer.struct()
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib().catq_grouped_soft_ternary_linear_bwd(ctypes.byref(st), sched, _ptr(X), _ptr(dY),
+                                                      _offsets(row_offsets), _dtype_code(X), _ptr(dX), _ptr(g_dmu),
+                                                      _ptr(g_dalpha), _ptr(g_ddelta), _ptr(workspace), ws_bytes,
+                                                      _stream(stream)), "catq_grouped_soft_ternary_linear_bwd")

@@ -289,6 +289,87 @@ catq_status catq_hard_ternarize_pack(const catq_layer* layer, uint8_t* codes, fl
                                       reinterpret_cast<cudaStream_t>(stream)));
 }
 
+// ------------------------------------------------------------------ grouped (MoE) layers
+
+namespace {
+
+// Expert e of a stacked layer as a dense layer (pointer offsets only).
+catq_layer expert_layer(const catq_grouped_layer* G, int32_t e) {
+  const int64_t groups = G->N * G->K / G->g;
+  const size_t esize = G->w_dtype == CATQ_BF16 ? 2 : 4;
+  catq_layer L;
+  L.N = G->N;
+  L.K = G->K;
+  L.g = G->g;
+  L.w_dtype = G->w_dtype;
+  L.W = static_cast<const char*>(G->W) + static_cast<size_t>(e) * G->N * G->K * esize;
+  L.mu0 = G->mu0 ? G->mu0 + e * groups : nullptr;
+  L.alpha0 = G->alpha0 ? G->alpha0 + e * groups : nullptr;
+  L.delta0 = G->delta0 ? G->delta0 + e * groups : nullptr;
+  L.d_mu = G->d_mu ? G->d_mu + e * groups : nullptr;
+  L.d_alpha = G->d_alpha ? G->d_alpha + e * groups : nullptr;
+  L.d_delta = G->d_delta ? G->d_delta + e * groups : nullptr;
+  return L;
+}
+
+catq_status check_grouped(const catq_grouped_layer* G, const int64_t* off) {
+  if (!G || !off || G->E < 1) return CATQ_ERR_INVALID_ARG;
+  if (off[0] != 0) return CATQ_ERR_SHAPE;
+  for (int32_t e = 0; e < G->E; ++e)
+    if (off[e + 1] < off[e]) return CATQ_ERR_SHAPE;
+  return CATQ_OK;
+}
+
+}  // namespace
+
+catq_status catq_grouped_soft_ternary_linear_fwd(const catq_grouped_layer* G, catq_schedule sched, const void* X,
+                                                 const int64_t* off, int32_t x_dtype, void* Y, catq_stream stream) {
+  catq_status st = check_grouped(G, off);
+  if (st != CATQ_OK) return st;
+  const size_t esize = x_dtype == CATQ_BF16 ? 2 : 4;
+  for (int32_t e = 0; e < G->E; ++e) {
+    const catq_layer L = expert_layer(G, e);
+    const int64_t m = off[e + 1] - off[e];
+    st = catq_soft_ternary_linear_fwd(&L, sched, static_cast<const char*>(X) + off[e] * G->K * esize, m, x_dtype,
+                                      static_cast<char*>(Y) + off[e] * G->N * esize, stream);
+    if (st != CATQ_OK) return st;
+  }
+  return CATQ_OK;
+}
+
+size_t catq_grouped_bwd_workspace_bytes(const catq_grouped_layer* G, const int64_t* off) {
+  if (check_grouped(G, off) != CATQ_OK) return 0;
+  size_t best = 0;
+  for (int32_t e = 0; e < G->E; ++e) {
+    const catq_layer L = expert_layer(G, e);
+    const size_t b = catq_bwd_workspace_bytes(&L, off[e + 1] - off[e]);
+    if (b > best) best = b;
+  }
+  return best;
+}
+
+catq_status catq_grouped_soft_ternary_linear_bwd(const catq_grouped_layer* G, catq_schedule sched, const void* X,
+                                                 const void* dY, const int64_t* off, int32_t x_dtype, void* dX,
+                                                 float* g_dmu, float* g_dalpha, float* g_ddelta, void* workspace,
+                                                 size_t ws_bytes, catq_stream stream) {
+  catq_status st = check_grouped(G, off);
+  if (st != CATQ_OK) return st;
+  const size_t esize = x_dtype == CATQ_BF16 ? 2 : 4;
+  const int64_t groups = G->N * G->K / G->g;
+  for (int32_t e = 0; e < G->E; ++e) {
+    const catq_layer L = expert_layer(G, e);
+    const int64_t m = off[e + 1] - off[e];
+    st = catq_soft_ternary_linear_bwd(
+        &L, sched, static_cast<const char*>(X) + off[e] * G->K * esize,
+        static_cast<const char*>(dY) + off[e] * G->N * esize, m, x_dtype,
+        dX ? static_cast<char*>(dX) + off[e] * G->K * esize : nullptr, g_dmu ? g_dmu + e * groups : nullptr,
+        g_dalpha ? g_dalpha + e * groups : nullptr, g_ddelta ? g_ddelta + e * groups : nullptr, workspace, ws_bytes,
+        stream);
+    if (st != CATQ_OK) return st;
+  }
+  return CATQ_OK;
+}
+
 catq_status catq_device_status(catq_stream stream, int32_t* out) {
   if (!out) return CATQ_ERR_INVALID_ARG;
   if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return CATQ_ERR_CUDA;

@@ -138,8 +138,8 @@ __device__ __forceinline__ uint32_t soft_pair_bf16(uint32_t w2, const ProducerCo
 __device__ __forceinline__ uint32_t hard_pair_bf16(uint32_t w2, const ProducerConst& p) {
   const float x0 = fmaf(bf16lo_to_f32(w2), p.r, p.b);
   const float x1 = fmaf(bf16hi_to_f32(w2), p.r, p.b);
-  const float y0 = x0 > p.delta ? p.C : (x0 < -p.delta ? -p.C : 0.0f);
-  const float y1 = x1 > p.delta ? p.C : (x1 < -p.delta ? -p.C : 0.0f);
+  const float y0 = fabsf(x0) > p.delta ? copysignf(p.C, x0) : 0.0f;  // Q(x) = sign(x) [|x| > Delta]
+  const float y1 = fabsf(x1) > p.delta ? copysignf(p.C, x1) : 0.0f;
   return pack_bf16x2(y0, y1);
 }
 
