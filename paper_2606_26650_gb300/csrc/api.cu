@@ -28,6 +28,8 @@ catq_status check_layer(const catq_layer* L, bool need_factors) {
   if (L->w_dtype != CATQ_F32 && L->w_dtype != CATQ_BF16) return CATQ_ERR_DTYPE;
   if (L->N < 1 || L->K < 1 || L->g < 1) return CATQ_ERR_SHAPE;
   if (L->K % L->g != 0) return CATQ_ERR_SHAPE;
+  if (L->N * L->K / L->g >= (int64_t(1) << 31) || L->N >= (int64_t(1) << 31) || L->K >= (int64_t(1) << 31))
+    return CATQ_ERR_SHAPE;  // group and row indices are 32-bit inside the kernels
   if (L->w_dtype == CATQ_BF16) {
     if (L->g % 64 != 0 || L->N % 8 != 0) return CATQ_ERR_SHAPE;
   } else {
