@@ -92,7 +92,27 @@ __device__ __forceinline__ void store_group_stats(int64_t j, int32_t g, int32_t 
 
 // ---------------------------------------------------------------- Eq. 3 statistics
 // Register variant: a team of `team` lanes owns one group and keeps its R x 16-byte
-// vectors in registers (mean, then deviations, without re-reading W).
+// vectors in registers (mean, then deviations, without re-reading W); each warp works on
+// two rounds of groups at once so two loads per lane are in flight.  The signed sum (mean)
+// is compensated; the all-positive deviation and magnitude sums are pairwise fp32, whose
+// relative error stays below ~10 ulp for these group sizes.
+template <int V>
+__device__ __forceinline__ float pairwise_abs_sum(const float (&x)[V], float shift) {
+  float t[V];
+#pragma unroll
+  for (int q = 0; q < V; ++q) t[q] = fabsf(x[q] - shift);
+#pragma unroll
+  for (int w = 1; w < V; w <<= 1)
+#pragma unroll
+    for (int q = 0; q + w < V; q += 2 * w) t[q] += t[q + w];
+  return t[0];
+}
+
+__device__ __forceinline__ float team_sum(float v, int team) {
+  for (int o = team >> 1; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
 template <typename T, int R>
 __global__ void __launch_bounds__(kThreads) group_stats_reg_kernel(const T* __restrict__ W, int64_t G, int32_t g,
                                                                    int32_t team, int32_t thr_init,
@@ -100,40 +120,53 @@ __global__ void __launch_bounds__(kThreads) group_stats_reg_kernel(const T* __re
                                                                    float* __restrict__ alpha0,
                                                                    float* __restrict__ delta0) {
   constexpr int V = Vec16<T>::n;
+  constexpr int ROUNDS = 2;
   const int lane = threadIdx.x & 31;
   const int sub = lane % team;
   const int per_warp = 32 / team;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
   const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
-  for (int64_t wbase = warp * per_warp; wbase < G; wbase += nwarps * per_warp) {
-    const int64_t j = wbase + lane / team;
-    const bool live = j < G;
-    float v[R][V];
-    Sum2 sum{0.f, 0.f};
+  const float inv_g = 1.0f / static_cast<float>(g);
+  for (int64_t wbase = warp * per_warp * ROUNDS; wbase < G; wbase += nwarps * per_warp * ROUNDS) {
+    float v[ROUNDS][R][V];
+    int64_t jr[ROUNDS];
 #pragma unroll
-    for (int r = 0; r < R; ++r) {
-      if (live) {
-        Vec16<T>::load(W + j * g + static_cast<int64_t>(sub + r * team) * V, v[r]);
-      } else {
+    for (int u = 0; u < ROUNDS; ++u) {
+      jr[u] = wbase + u * per_warp + lane / team;
 #pragma unroll
-        for (int q = 0; q < V; ++q) v[r][q] = 0.f;
+      for (int r = 0; r < R; ++r) {
+        if (jr[u] < G) {
+          Vec16<T>::load(W + jr[u] * g + static_cast<int64_t>(sub + r * team) * V, v[u][r]);
+        } else {
+#pragma unroll
+          for (int q = 0; q < V; ++q) v[u][r][q] = 0.f;
+        }
       }
-#pragma unroll
-      for (int q = 0; q < V; ++q) sum2_add(sum, v[r][q]);
     }
-    sum = sum2_team(sum, team);
-    const float mu = sum2_float(sum) / static_cast<float>(g);
-    Sum2 dev{0.f, 0.f}, mag{0.f, 0.f};
 #pragma unroll
-    for (int r = 0; r < R; ++r)
+    for (int u = 0; u < ROUNDS; ++u) {
+      Sum2 sum{0.f, 0.f};
 #pragma unroll
-      for (int q = 0; q < V; ++q) {
-        sum2_add(dev, fabsf(v[r][q] - mu));
-        sum2_add(mag, fabsf(v[r][q]));
+      for (int r = 0; r < R; ++r)
+#pragma unroll
+        for (int q = 0; q < V; ++q) sum2_add(sum, v[u][r][q]);
+      sum = sum2_team(sum, team);
+      const float mu = sum2_float(sum) * inv_g;
+      float dev = 0.f, mag = 0.f;
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        dev += pairwise_abs_sum<V>(v[u][r], mu);
+        mag += pairwise_abs_sum<V>(v[u][r], 0.0f);
       }
-    dev = sum2_team(dev, team);
-    mag = sum2_team(mag, team);
-    if (live && sub == 0) store_group_stats(j, g, thr_init, mu, dev, mag, mu0, alpha0, delta0);
+      dev = team_sum(dev, team);
+      mag = team_sum(mag, team);
+      if (jr[u] < G && sub == 0) {
+        const float a0 = dev * inv_g;
+        mu0[jr[u]] = mu;
+        alpha0[jr[u]] = a0;
+        delta0[jr[u]] = (thr_init == 1 && a0 > 0.0f) ? 0.7f * (mag * inv_g) / a0 : 0.5f;
+      }
+    }
   }
 }
 
@@ -254,19 +287,18 @@ __global__ void __launch_bounds__(kThreads) hard_pack_kernel(LayerDev L, uint8_t
           v[i] = bf16lo_to_f32(static_cast<uint32_t>(reinterpret_cast<const uint16_t*>(W)[e0 + i]));
       }
     }
-    uint32_t word = 0;
+    uint32_t words[(EPT + 15) / 16] = {};
 #pragma unroll
     for (int i = 0; i < EPT; ++i) {
       const int q = (gc.alpha != 0.0f) ? static_cast<int>(hard_q(what(v[i], gc), gc.delta)) : 0;
-      word |= static_cast<uint32_t>(q + 1) << (2 * (i & 15));
-      if ((i & 15) == 15 || i == EPT - 1) {
-        if constexpr (EPT >= 16)
-          reinterpret_cast<uint32_t*>(codes)[(e0 + i) / 16] = word;
-        else
-          codes[e0 / 4] = static_cast<uint8_t>(word);
-        word = 0;
-      }
+      words[i / 16] |= static_cast<uint32_t>(q + 1) << (2 * (i & 15));
     }
+    if constexpr (EPT == 64)
+      *reinterpret_cast<uint4*>(codes + e0 / 4) = make_uint4(words[0], words[1], words[2], words[3]);
+    else if constexpr (EPT == 16)
+      reinterpret_cast<uint32_t*>(codes)[e0 / 16] = words[0];
+    else
+      codes[e0 / 4] = static_cast<uint8_t>(words[0]);
   }
   if (alpha)
     for (int64_t j = blockIdx.x * (int64_t)kThreads + threadIdx.x; j < G; j += (int64_t)gridDim.x * kThreads)
@@ -399,7 +431,7 @@ cudaError_t launch_group_stats(const LayerDev& L, int32_t w_dtype, int32_t thr_i
   if (L.g % V == 0 && nvec <= 128 && (nvec & (nvec - 1)) == 0) {
     const int team = nvec < 32 ? nvec : 32;
     const int R = nvec / team;
-    const int grid = grid_for((G + 32 / team - 1) / (32 / team), kThreads / 32);
+    const int grid = grid_for((G + 2 * (32 / team) - 1) / (2 * (32 / team)), kThreads / 32);
 #define CATQ_STATS_REG(TT, RR)                                                                                  \
   group_stats_reg_kernel<TT, RR><<<grid, kThreads, 0, st>>>(static_cast<const TT*>(L.W), G, L.g, team, thr_init, \
                                                             mu0, alpha0, delta0)
@@ -465,7 +497,13 @@ cudaError_t launch_recon_loss(const void* Y, const void* Yr, int64_t count, int3
 
 cudaError_t launch_hard_pack(const LayerDev& L, int32_t w_dtype, uint8_t* codes, float* alpha, cudaStream_t st) {
   const int64_t n = L.N * L.K;
-  if (L.g % 16 == 0) {
+  if (L.g % 64 == 0) {
+    const int grid = grid_for(n / 64, kThreads);
+    if (w_dtype == 1)
+      hard_pack_kernel<__nv_bfloat16, 64><<<grid, kThreads, 0, st>>>(L, codes, alpha);
+    else
+      hard_pack_kernel<float, 64><<<grid, kThreads, 0, st>>>(L, codes, alpha);
+  } else if (L.g % 16 == 0) {
     const int grid = grid_for(n / 16, kThreads);
     if (w_dtype == 1)
       hard_pack_kernel<__nv_bfloat16, 16><<<grid, kThreads, 0, st>>>(L, codes, alpha);
