@@ -46,18 +46,26 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitTimeoutNs = 4000000000ull;
 constexpr uint64_t kDrainTimeoutNs = 200000000ull;
 
-template <int CG>
+// PAIRS == 2 runs clusters of four CTAs: two CTA pairs compute adjacent 512-row M tiles
+// against the same produced operand tiles; each pair produces every other stage and sends
+// its transformed half-tiles to the other pair's CTAs through distributed shared memory,
+// which halves the per-SM transform work.
+template <int CG, int PAIRS = 1>
 struct FusedCfg {
+  static_assert(PAIRS == 1 || CG == 2, "pairs of pairs need CTA pairs");
+  static constexpr int kClusterCtas = CG * PAIRS;
   static constexpr int kRowsPerAcc = 128 * CG;          // MMA M
-  static constexpr int kTileRows = kRowsPerAcc * NACC;  // rows of C per tile
+  static constexpr int kTileRows = kRowsPerAcc * NACC;  // rows of C per pair per tile
   static constexpr int kBRows = BN / CG;                // 128-byte operand rows per CTA per stage
   static constexpr int kABytes = NACC * 128 * BK * 2;   // this CTA's A rows per stage
   static constexpr int kWBytes = kBRows * BK * 2;       // this CTA's operand rows per stage
   static constexpr int kStagesA = CG == 1 ? 3 : 4;      // A ring: TMA -> MMA
-  static constexpr int kStagesW = CG == 1 ? 3 : 5;      // W ring: TMA -> producers (in place) -> MMA
+  // W ring: TMA -> producers (in place) -> MMA.  Even with two pairs, so every slot is always
+  // produced by the same pair (and received by the other).
+  static constexpr int kStagesW = PAIRS == 2 ? 6 : (CG == 1 ? 3 : 5);
   static constexpr int kEpiWarps = 4;
-  // Two groups of 8 producer warps take alternate stages, so each group has two stage
-  // periods per operand tile and the groups' MUFU work interleaves.
+  // Two groups of 8 producer warps take alternate stages (of the ones this CTA produces), so
+  // each group has two stage periods per operand tile and the groups' MUFU work interleaves.
   static constexpr int kProdGroups = 2;
   static constexpr int kGroupWarps = 8;
   static constexpr int kProdWarps = kProdGroups * kGroupWarps;
@@ -65,7 +73,7 @@ struct FusedCfg {
   static constexpr int kThreadsPerRow = kGroupThreads / kBRows;  // 1 (CG 1) or 2 (CG 2)
   static constexpr int kChunksPerThread = 8 / kThreadsPerRow;    // 16-byte chunks of a 128-byte row
   static constexpr int kThreads = 32 * (kEpiWarps + 2 + kProdWarps);
-  static constexpr int kBarBytes = 8 * (2 * kStagesA + 3 * kStagesW + 3) + 16;
+  static constexpr int kBarBytes = 8 * (2 * kStagesA + 5 * kStagesW + 3) + 16;
   static constexpr int kSmemBytes = kStagesA * kABytes + kStagesW * kWBytes + 1024 + kBarBytes;
 };
 
@@ -191,11 +199,11 @@ struct OperandRowIter {
   }
 };
 
-template <int CG, bool B_MN>
-__global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
+template <int CG, bool B_MN, int PAIRS>
+__global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     fused_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
                       const FusedArgs args) {
-  using Cfg = FusedCfg<CG>;
+  using Cfg = FusedCfg<CG, PAIRS>;
   constexpr int SA = Cfg::kStagesA, SW = Cfg::kStagesW;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = smem_u32(smem_raw);
@@ -207,20 +215,27 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
   auto full_a = [&](int s) { return bars + 8u * s; };                   // A landed (pair: even CTA)
   auto empty_a = [&](int s) { return bars + 8u * (SA + s); };           // A consumed by the MMA
   auto raw_w = [&](int s) { return bars + 8u * (2 * SA + s); };         // raw W landed (local)
-  auto full_w = [&](int s) { return bars + 8u * (2 * SA + SW + s); };   // operand produced (pair: even CTA)
+  auto full_w = [&](int s) { return bars + 8u * (2 * SA + SW + s); };   // operand ready (pair: even CTA)
   auto empty_w = [&](int s) { return bars + 8u * (2 * SA + 2 * SW + s); };
-  const uint32_t tmem_full_bar = bars + 8u * (2 * SA + 3 * SW);
+  auto prod_done = [&](int s) { return bars + 8u * (2 * SA + 3 * SW + s); };  // PAIRS 2: local producers done
+  auto recv_w = [&](int s) { return bars + 8u * (2 * SA + 4 * SW + s); };     // PAIRS 2: operand received
+  const uint32_t tmem_full_bar = bars + 8u * (2 * SA + 5 * SW);
   const uint32_t tmem_empty_bar = tmem_full_bar + 8;
   const uint32_t final_bar = tmem_full_bar + 16;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base_ptr + (bars - base) + 8 * (2 * SA + 3 * SW + 3));
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base_ptr + (bars - base) + 8 * (2 * SA + 5 * SW + 3));
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t cta = CG == 2 ? cluster_ctarank() : 0u;
+  const uint32_t rank = CG == 2 ? cluster_ctarank() : 0u;
+  const uint32_t cta = rank & 1u;                // half of the pair
+  const uint32_t pair = rank >> 1;               // pair within the cluster (PAIRS 2)
+  const uint32_t leader = rank & ~1u;            // the pair's MMA-issuing CTA
   const uint32_t cluster = CG == 2 ? cluster_id_x() : blockIdx.x;
   const uint32_t nclusters = CG == 2 ? num_clusters_x() : gridDim.x;
   const WaitCtl& wc = args.wc;
   const int num_tiles = args.num_m_tiles * args.num_n_tiles;
   constexpr int kTmaWarp = Cfg::kEpiWarps, kMmaWarp = Cfg::kEpiWarps + 1;
+  // does this CTA produce stage q (PAIRS 1: always)
+  auto produces = [&](uint32_t q) { return PAIRS == 1 || (q & 1u) == pair; };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < SA; ++s) {
@@ -229,8 +244,11 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
     }
     for (int s = 0; s < SW; ++s) {
       mbar_init(raw_w(s), 1);
-      mbar_init(full_w(s), Cfg::kGroupWarps * CG);  // one arrival per warp of the stage's group
-      mbar_init(empty_w(s), 1);
+      // PAIRS 1: one arrival per producer warp of the pair; PAIRS 2: one forwarded arrival per CTA
+      mbar_init(full_w(s), PAIRS == 1 ? Cfg::kGroupWarps * CG : 2);
+      mbar_init(empty_w(s), PAIRS);  // every pair's MMA frees the slot in all CTAs
+      mbar_init(prod_done(s), Cfg::kGroupWarps);
+      mbar_init(recv_w(s), 1);
     }
     mbar_init(tmem_full_bar, 1);
     mbar_init(tmem_empty_bar, Cfg::kEpiWarps * CG);
@@ -246,10 +264,12 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
   if constexpr (CG == 2) cluster_sync_all(); else __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  // Barriers the whole pair signals live in the even CTA.
-  const uint32_t leader_full_a0 = CG == 2 ? mapa_shared(full_a(0), 0) : full_a(0);
-  const uint32_t leader_full_w0 = CG == 2 ? mapa_shared(full_w(0), 0) : full_w(0);
-  const uint32_t leader_tmem_empty = CG == 2 ? mapa_shared(tmem_empty_bar, 0) : tmem_empty_bar;
+  // Barriers a whole pair signals live in the pair's even CTA.
+  const uint32_t leader_full_a0 = CG == 2 ? mapa_shared(full_a(0), leader) : full_a(0);
+  const uint32_t leader_full_w0 = CG == 2 ? mapa_shared(full_w(0), leader) : full_w(0);
+  const uint32_t leader_tmem_empty = CG == 2 ? mapa_shared(tmem_empty_bar, leader) : tmem_empty_bar;
+  const uint16_t pair_mask = static_cast<uint16_t>(3u << (2 * pair));
+  const uint16_t all_mask = static_cast<uint16_t>((1u << Cfg::kClusterCtas) - 1u);
 
   if (warp == kTmaWarp) {
     if (lane == 0) {
@@ -257,7 +277,7 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
       uint32_t q = 0, issued_mask = 0, issued_phase = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
-        const int32_t m0 = (t % args.num_m_tiles) * Cfg::kTileRows;
+        const int32_t m0 = (t % args.num_m_tiles) * (Cfg::kTileRows * PAIRS) + pair * Cfg::kTileRows;
         for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
           const uint32_t s = q % SA, ph = (q / SA) & 1u;
           if (!mbar_wait(empty_a(s), ph ^ 1u, wc)) { ok = false; break; }
@@ -277,12 +297,13 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
         for (int s = 0; s < SA; ++s)
           if (issued_mask & (1u << s)) mbar_wait_drain(full_a(s), (issued_phase >> s) & 1u);
     } else if (lane == 1) {
-      // ---------------------------------------------------------- TMA: raw W tiles (to the producers)
+      // ---------------------------------------------------------- TMA: raw W tiles this CTA produces
       uint32_t q = 0, issued_mask = 0, issued_phase = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
         const int32_t n0 = (t / args.num_m_tiles) * BN + cta * Cfg::kBRows;
         for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
+          if (!produces(q)) continue;
           const uint32_t s = q % SW, ph = (q / SW) & 1u;
           if (!mbar_wait(empty_w(s), ph ^ 1u, wc)) { ok = false; break; }
           mbar_arrive_expect_tx(raw_w(s), Cfg::kWBytes);
@@ -299,9 +320,36 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
       }
       for (int s = 0; s < SW; ++s)
         if (issued_mask & (1u << s)) mbar_wait_drain(raw_w(s), (issued_phase >> s) & 1u);
+    } else if (PAIRS == 2 && (lane == 2 || lane == 3)) {
+      // ---------------------------------------------------------- operand exchange between the pairs
+      // Lane 2, produced stages: once this CTA's producers are done, copy the half-tile to the
+      // same slot of the other pair's CTA with the same half, then report it ready to this
+      // pair's MMA.  Lane 3, received stages: arm the slot's receive barrier when the slot is
+      // free, wait for the copy, then report it ready.  Separate lanes, so neither direction
+      // waits for the other.
+      const uint32_t partner = rank ^ 2u;
+      const bool sender = lane == 2;
+      uint32_t q = 0;
+      bool ok = true;
+      for (int t = cluster; ok && t < num_tiles; t += nclusters) {
+        for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
+          if (produces(q) != sender) continue;
+          const uint32_t s = q % SW, ph = (q / SW) & 1u;
+          if (sender) {
+            if (!mbar_wait(prod_done(s), ph, wc)) { ok = false; break; }
+            bulk_copy_to_peer(mapa_shared(w_base + s * Cfg::kWBytes, partner), w_base + s * Cfg::kWBytes,
+                              Cfg::kWBytes, mapa_shared(recv_w(s), partner));
+          } else {
+            if (!mbar_wait(empty_w(s), ph ^ 1u, wc)) { ok = false; break; }
+            mbar_arrive_expect_tx(recv_w(s), Cfg::kWBytes);
+            if (!mbar_wait(recv_w(s), ph, wc)) { ok = false; break; }
+          }
+          mbar_arrive_cluster(leader_full_w0 + 8u * s);
+        }
+      }
     }
   } else if (warp == kMmaWarp) {
-    // ------------------------------------------------------------ MMA issuer (even CTA)
+    // ------------------------------------------------------------ MMA issuer (even CTA of each pair)
     if (cta == 0 && lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(Cfg::kRowsPerAcc, BN, false, B_MN);
       uint32_t q = 0, it = 0;
@@ -324,12 +372,21 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
               umma_bf16<CG>(tmem_base + acc * BN, adesc, bdesc, idesc, (kb | kk) != 0 ? 1u : 0u);
             }
           }
-          umma_commit<CG>(empty_a(sa));
-          umma_commit<CG>(empty_w(sw));
+          if constexpr (PAIRS == 1) {
+            umma_commit<CG>(empty_a(sa));
+            umma_commit<CG>(empty_w(sw));
+          } else {
+            umma_commit_pair_mask(empty_a(sa), pair_mask);
+            umma_commit_pair_mask(empty_w(sw), all_mask);
+          }
         }
-        if (ok) umma_commit<CG>(tmem_full_bar);
+        if (ok) {
+          if constexpr (PAIRS == 1) umma_commit<CG>(tmem_full_bar);
+          else umma_commit_pair_mask(tmem_full_bar, pair_mask);
+        }
       }
-      umma_commit<CG>(final_bar);
+      if constexpr (PAIRS == 1) umma_commit<CG>(final_bar);
+      else umma_commit_pair_mask(final_bar, pair_mask);
       mbar_wait_drain(final_bar, 0);
     }
   } else if (warp < Cfg::kEpiWarps) {
@@ -342,7 +399,8 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
       tc_fence_after();
 #pragma unroll 1
       for (int acc = 0; acc < NACC; ++acc) {
-        const int64_t row = (int64_t)m_blk * Cfg::kTileRows + acc * Cfg::kRowsPerAcc + cta * 128 + qd * 32 + lane;
+        const int64_t row = (int64_t)m_blk * (Cfg::kTileRows * PAIRS) + pair * Cfg::kTileRows +
+                            acc * Cfg::kRowsPerAcc + cta * 128 + qd * 32 + lane;
 #pragma unroll 1
         for (int c = 0; c < BN / 32; ++c) {
           uint32_t r[32];
@@ -361,22 +419,25 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
     // Within its group, each thread owns one row (CG 1) or half a row (CG 2) of the stage's
     // raw W tile and rewrites it in place as the Eq. 6 weight.  A row holds 64 consecutive K
     // elements of one W row, so it lies in one group (g is a multiple of 64).  Rows outside
-    // W were zero-filled by the copy and stay 0.
+    // W were zero-filled by the copy and stay 0.  The CTA's produced stages are
+    // pair, pair + PAIRS, ...; group g takes every second of them.
     constexpr int CPT = Cfg::kChunksPerThread;
     constexpr int PG = Cfg::kProdGroups;
+    constexpr int STEP = PG * PAIRS;
     const int pw = warp - (Cfg::kEpiWarps + 2);  // producer warp index
-    const int grp = pw / Cfg::kGroupWarps;       // this warp's group: stages grp, grp + PG, ...
+    const int grp = pw / Cfg::kGroupWarps;
     const int tt = threadIdx.x - 32 * (Cfg::kEpiWarps + 2) - grp * Cfg::kGroupThreads;
     const int row = tt / Cfg::kThreadsPerRow;
     const int c_begin = (tt % Cfg::kThreadsPerRow) * CPT;
     const LayerDev& L = args.L;
     const int32_t phase_t = args.sc.phase;
     const bool transform = phase_t != PHASE_TEACHER;
+    const uint32_t q0 = (PAIRS == 2 ? pair : 0u) + PAIRS * grp;
     // `cur` is the stage being produced; `ahead` runs two of this thread's stages ahead and
     // requests that stage's group inputs, so an L2 round trip is hidden behind two stages.
     OperandRowIter<CG, B_MN> cur, ahead;
     cur.init(args, cta, row, cluster, 0);
-    cur.step(args, cta, row, nclusters, grp);
+    cur.step(args, cta, row, nclusters, q0);
     ahead = cur;
     GroupRaw raw0{}, raw1{};
     int64_t j0 = -1, j1 = -1;
@@ -389,12 +450,12 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
       }
     };
     request(ahead, raw0, j0, raw1, j1);
-    ahead.step(args, cta, row, nclusters, PG);
+    ahead.step(args, cta, row, nclusters, STEP);
     request(ahead, raw1, j1, raw0, j0);
-    ahead.step(args, cta, row, nclusters, PG);
+    ahead.step(args, cta, row, nclusters, STEP);
     int64_t j_have = -1;
     ProducerConst pc{};
-    uint32_t q = grp;
+    uint32_t q = q0;
     bool ok = true;
     // One stage: consume `mine` (requested two stages ago), then refill it two stages ahead.
     auto produce = [&](GroupRaw& mine, int64_t& jm, const GroupRaw& other, int64_t jo) {
@@ -429,12 +490,15 @@ __global__ void __launch_bounds__(FusedCfg<CG>::kThreads, 1)
         fence_proxy_async_smem();
       }
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(leader_full_w0 + 8u * s);
+      if (lane == 0) {
+        if constexpr (PAIRS == 1) mbar_arrive_cluster(leader_full_w0 + 8u * s);
+        else mbar_arrive_local(prod_done(s));
+      }
       // Issued after the proxy fence, which would otherwise wait for these loads.
       request(ahead, mine, jm, other, jo);
-      ahead.step(args, cta, row, nclusters, PG);
-      q += PG;
-      cur.step(args, cta, row, nclusters, PG);
+      ahead.step(args, cta, row, nclusters, STEP);
+      q += STEP;
+      cur.step(args, cta, row, nclusters, STEP);
     };
     while (ok && cur.live(args, num_tiles)) {
       produce(raw0, j0, raw1, j1);
@@ -732,15 +796,43 @@ cudaError_t launch_persistent(Kern kern, int cg, int grid_ctas, int threads, int
   return cudaLaunchKernelExC(&cfg, reinterpret_cast<const void*>(kern), params);
 }
 
-int fused_cg_for(int64_t M) {
-  // Two-CTA tiles (512 rows) pay off once M fills them.
-  return M >= 512 ? 2 : 1;
+// Largest number of co-resident clusters of `cluster_ctas` CTAs for a kernel (cached per
+// device); a persistent grid larger than this would run a second, partial wave.
+template <typename Kern>
+int max_active_clusters(Kern kern, int cluster_ctas, int threads, int smem, int fallback) {
+  static std::mutex mu;
+  static int cache[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache[dev & 63] > 0) return cache[dev & 63];
+  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(cluster_ctas * 64);
+  cfg.blockDim = dim3(threads);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cluster_ctas;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(kern), &cfg) != cudaSuccess || n <= 0)
+    n = fallback;
+  cache[dev & 63] = n;
+  return n;
 }
 
-template <int CG, bool B_MN>
+// Tile shape by M: pairs of pairs (1024 rows per cluster tile) once M fills both pairs,
+// CTA pairs (512 rows) from 512 rows, single CTAs below.
+int fused_variant_for(int64_t M) { return M >= 1024 ? 4 : (M >= 512 ? 2 : 1); }
+
+template <int CG, bool B_MN, int PAIRS>
 cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t M, int64_t depth, void* C,
                       int64_t ncols, cudaStream_t st) {
-  using Cfg = FusedCfg<CG>;
+  using Cfg = FusedCfg<CG, PAIRS>;
   DeviceInfo& d = device_info();
   if (!d.ok) return cudaErrorInvalidDevice;
   CUtensorMap ta, tw;
@@ -756,15 +848,18 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
   args.C = static_cast<uint16_t*>(C);
   args.M = M;
   args.ncols = ncols;
-  args.num_m_tiles = static_cast<int32_t>((M + Cfg::kTileRows - 1) / Cfg::kTileRows);
+  args.num_m_tiles = static_cast<int32_t>((M + Cfg::kTileRows * PAIRS - 1) / (Cfg::kTileRows * PAIRS));
   args.num_n_tiles = static_cast<int32_t>((ncols + BN - 1) / BN);
   args.num_k_blocks = static_cast<int32_t>((depth + BK - 1) / BK);
   args.wc = make_wait_ctl(d);
+  auto kern = fused_gemm_kernel<CG, B_MN, PAIRS>;
   const int tiles = args.num_m_tiles * args.num_n_tiles;
-  const int clusters = std::min(tiles, d.sm_count / CG);
+  const int fit = max_active_clusters(kern, Cfg::kClusterCtas, Cfg::kThreads, Cfg::kSmemBytes,
+                                      d.sm_count / Cfg::kClusterCtas);
+  const int clusters = std::min(tiles, fit);
   void* params[3] = {&ta, &tw, &args};
-  return launch_persistent(fused_gemm_kernel<CG, B_MN>, CG, clusters * CG, Cfg::kThreads, Cfg::kSmemBytes, st,
-                           params);
+  return launch_persistent(kern, Cfg::kClusterCtas, clusters * Cfg::kClusterCtas, Cfg::kThreads, Cfg::kSmemBytes,
+                           st, params);
 }
 
 template <int CG>
@@ -818,13 +913,19 @@ TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count) {
 }
 
 cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st) {
-  if (fused_cg_for(M) == 2) return run_fused<2, false>(L, sc, X, M, L.K, Y, L.N, st);
-  return run_fused<1, false>(L, sc, X, M, L.K, Y, L.N, st);
+  switch (fused_variant_for(M)) {
+    case 4: return run_fused<2, false, 2>(L, sc, X, M, L.K, Y, L.N, st);
+    case 2: return run_fused<2, false, 1>(L, sc, X, M, L.K, Y, L.N, st);
+    default: return run_fused<1, false, 1>(L, sc, X, M, L.K, Y, L.N, st);
+  }
 }
 
 cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int64_t M, void* dX, cudaStream_t st) {
-  if (fused_cg_for(M) == 2) return run_fused<2, true>(L, sc, dY, M, L.N, dX, L.K, st);
-  return run_fused<1, true>(L, sc, dY, M, L.N, dX, L.K, st);
+  switch (fused_variant_for(M)) {
+    case 4: return run_fused<2, true, 2>(L, sc, dY, M, L.N, dX, L.K, st);
+    case 2: return run_fused<2, true, 1>(L, sc, dY, M, L.N, dX, L.K, st);
+    default: return run_fused<1, true, 1>(L, sc, dY, M, L.N, dX, L.K, st);
+  }
 }
 
 cudaError_t launch_tc_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M,
