@@ -289,8 +289,9 @@ def run_ours(args):
     for _ in range(args.warmup):
         step()
     barrier()
-    if C.catq_device_status() != 0:
-        raise SystemExit("device status set during warm-up")
+    status = C.catq_device_status()
+    if status != 0:
+        raise SystemExit(f"device status {C.STATUS.get(status, status)} during warm-up")
 
     E = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
     evs = [[{k: (E(), E()) for k in kinds} for _ in st] for _ in range(args.steps)]

@@ -46,6 +46,8 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint64_t kWaitTimeoutNs = 4000000000ull;
 constexpr uint64_t kDrainTimeoutNs = 200000000ull;
 
+constexpr int gcd_c(int a, int b) { return b == 0 ? a : gcd_c(b, a % b); }
+
 // PAIRS == 2 runs clusters of four CTAs: two CTA pairs compute adjacent 512-row M tiles
 // against the same produced operand tiles; each pair produces every other stage and sends
 // its transformed half-tiles to the other pair's CTAs through distributed shared memory,
@@ -73,7 +75,15 @@ struct FusedCfg {
   static constexpr int kThreadsPerRow = kGroupThreads / kBRows;  // 1 (CG 1) or 2 (CG 2)
   static constexpr int kChunksPerThread = 8 / kThreadsPerRow;    // 16-byte chunks of a 128-byte row
   static constexpr int kThreads = 32 * (kEpiWarps + 2 + kProdWarps);
-  static constexpr int kBarBytes = 8 * (2 * kStagesA + 5 * kStagesW + 3) + 16;
+  // Stage q lands on the raw-W barrier of its producer group and slot; that barrier sees one
+  // stage in every kRawPeriod, so each group waits on its own barriers strictly in phase
+  // order (one barrier per slot shared by the groups would let a group running a full phase
+  // ahead read the parity of the other group's pending phase as complete).
+  static constexpr int kStep = kProdGroups * PAIRS;  // stages between two of a group's stages
+  static constexpr int kRawPeriod = kStagesW / gcd_c(kStagesW, kStep) * kStep;
+  static constexpr int kRawBars = kProdGroups * kStagesW;
+  static_assert(kRawBars <= 32, "issued-barrier masks are 32 bits");
+  static constexpr int kBarBytes = 8 * (2 * kStagesA + kRawBars + 4 * kStagesW + 3) + 16;
   static constexpr int kSmemBytes = kStagesA * kABytes + kStagesW * kWBytes + 1024 + kBarBytes;
 };
 
@@ -214,15 +224,16 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
   const uint32_t bars = w_base + SW * Cfg::kWBytes;
   auto full_a = [&](int s) { return bars + 8u * s; };                   // A landed (pair: even CTA)
   auto empty_a = [&](int s) { return bars + 8u * (SA + s); };           // A consumed by the MMA
-  auto raw_w = [&](int s) { return bars + 8u * (2 * SA + s); };         // raw W landed (local)
-  auto full_w = [&](int s) { return bars + 8u * (2 * SA + SW + s); };   // operand ready (pair: even CTA)
-  auto empty_w = [&](int s) { return bars + 8u * (2 * SA + 2 * SW + s); };
-  auto prod_done = [&](int s) { return bars + 8u * (2 * SA + 3 * SW + s); };  // PAIRS 2: local producers done
-  auto recv_w = [&](int s) { return bars + 8u * (2 * SA + 4 * SW + s); };     // PAIRS 2: operand received
-  const uint32_t tmem_full_bar = bars + 8u * (2 * SA + 5 * SW);
+  constexpr int RB = Cfg::kRawBars;
+  auto raw_w = [&](int b) { return bars + 8u * (2 * SA + b); };          // raw W landed [group][slot] (local)
+  auto full_w = [&](int s) { return bars + 8u * (2 * SA + RB + s); };   // operand ready (pair: even CTA)
+  auto empty_w = [&](int s) { return bars + 8u * (2 * SA + RB + SW + s); };
+  auto prod_done = [&](int s) { return bars + 8u * (2 * SA + RB + 2 * SW + s); };  // PAIRS 2: local producers done
+  auto recv_w = [&](int s) { return bars + 8u * (2 * SA + RB + 3 * SW + s); };     // PAIRS 2: operand received
+  const uint32_t tmem_full_bar = bars + 8u * (2 * SA + RB + 4 * SW);
   const uint32_t tmem_empty_bar = tmem_full_bar + 8;
   const uint32_t final_bar = tmem_full_bar + 16;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base_ptr + (bars - base) + 8 * (2 * SA + 5 * SW + 3));
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base_ptr + (bars - base) + 8 * (2 * SA + RB + 4 * SW + 3));
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = CG == 2 ? cluster_ctarank() : 0u;
@@ -242,8 +253,8 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
       mbar_init(full_a(s), 1);
       mbar_init(empty_a(s), 1);
     }
+    for (int b = 0; b < RB; ++b) mbar_init(raw_w(b), 1);
     for (int s = 0; s < SW; ++s) {
-      mbar_init(raw_w(s), 1);
       // PAIRS 1: one arrival per producer warp of the pair; PAIRS 2: one forwarded arrival per CTA
       mbar_init(full_w(s), PAIRS == 1 ? Cfg::kGroupWarps * CG : 2);
       mbar_init(empty_w(s), PAIRS);  // every pair's MMA frees the slot in all CTAs
@@ -305,21 +316,23 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
         for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
           if (!produces(q)) continue;
           const uint32_t s = q % SW, ph = (q / SW) & 1u;
+          const uint32_t rb = ((q / PAIRS) % Cfg::kProdGroups) * SW + s;  // the producing group's barrier
+          const uint32_t rph = (q / Cfg::kRawPeriod) & 1u;
           if (!mbar_wait(empty_w(s), ph ^ 1u, wc)) { ok = false; break; }
-          mbar_arrive_expect_tx(raw_w(s), Cfg::kWBytes);
+          mbar_arrive_expect_tx(raw_w(rb), Cfg::kWBytes);
           const uint32_t dst = w_base + s * Cfg::kWBytes;
           if constexpr (!B_MN) {
-            tma_load_2d(dst, &tmW, raw_w(s), kb * BK, n0);
+            tma_load_2d(dst, &tmW, raw_w(rb), kb * BK, n0);
           } else {
 #pragma unroll
-            for (int b = 0; b < Cfg::kBRows / 64; ++b) tma_load_2d(dst + b * 8192, &tmW, raw_w(s), n0 + 64 * b, kb * BK);
+            for (int b = 0; b < Cfg::kBRows / 64; ++b) tma_load_2d(dst + b * 8192, &tmW, raw_w(rb), n0 + 64 * b, kb * BK);
           }
-          issued_mask |= 1u << s;
-          issued_phase = (issued_phase & ~(1u << s)) | (ph << s);
+          issued_mask |= 1u << rb;
+          issued_phase = (issued_phase & ~(1u << rb)) | (rph << rb);
         }
       }
-      for (int s = 0; s < SW; ++s)
-        if (issued_mask & (1u << s)) mbar_wait_drain(raw_w(s), (issued_phase >> s) & 1u);
+      for (int b = 0; b < RB; ++b)
+        if (issued_mask & (1u << b)) mbar_wait_drain(raw_w(b), (issued_phase >> b) & 1u);
     } else if (PAIRS == 2 && (lane == 2 || lane == 3)) {
       // ---------------------------------------------------------- operand exchange between the pairs
       // Lane 2, produced stages: once this CTA's producers are done, copy the half-tile to the
@@ -422,8 +435,7 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     // W were zero-filled by the copy and stay 0.  The CTA's produced stages are
     // pair, pair + PAIRS, ...; group g takes every second of them.
     constexpr int CPT = Cfg::kChunksPerThread;
-    constexpr int PG = Cfg::kProdGroups;
-    constexpr int STEP = PG * PAIRS;
+    constexpr int STEP = Cfg::kStep;
     const int pw = warp - (Cfg::kEpiWarps + 2);  // producer warp index
     const int grp = pw / Cfg::kGroupWarps;
     const int tt = threadIdx.x - 32 * (Cfg::kEpiWarps + 2) - grp * Cfg::kGroupThreads;
@@ -459,13 +471,13 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     bool ok = true;
     // One stage: consume `mine` (requested two stages ago), then refill it two stages ahead.
     auto produce = [&](GroupRaw& mine, int64_t& jm, const GroupRaw& other, int64_t jo) {
-      const uint32_t s = q % SW, ph = (q / SW) & 1u;
+      const uint32_t s = q % SW;
       const bool live = transform && cur.valid(args);
       if (live && cur.j != j_have) {
         pc = producer_const(group_const(mine), args.sc.s, args.sc.inv_2tanh_s, phase_t);
         j_have = cur.j;
       }
-      if (!mbar_wait(raw_w(s), ph, wc)) {
+      if (!mbar_wait(raw_w(grp * SW + s), (q / Cfg::kRawPeriod) & 1u, wc)) {
         ok = false;
         return;
       }
