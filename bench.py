@@ -37,9 +37,11 @@ CPU_SAMPLE_LINEARS = ("q_proj", "k_proj", "down_proj")  # cpu_baseline leg of ou
 CPU_SAMPLE_ROWS = 256
 REF_STEP_LINEARS = ("k_proj",)  # one step of the reference arm (runs K + W times)
 
-# DRAM traffic per launch of the dominant kernel from an ncu capture, keyed by the hash of
-# the sources it was taken at; reported only while those sources are unchanged.
-TRAFFIC = {}
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per launch, mean over the
+# seven linears of the 8B-shaped block step, from one ncu capture of the timed step; keyed
+# by the hash of the sources it was taken at and reported only while they are unchanged.
+TRAFFIC = {"sha": "950d5cf0d004725b", "workload": "c3_llama3_8b_block",
+           "fwd": 578775259, "dx": 602352749, "dw": 912416658}
 
 
 def parse():
@@ -330,9 +332,14 @@ def run_ours(args):
                    "dx": "fused_gemm_kernel (dX, MN-major Wq operand)",
                    "dw": "dw_kernel + grad_reduce_kernel (dW factor-gradient epilogue)"}[dom]
     sha = kernel_sources_sha()
-    traffic = TRAFFIC.get(dom) if TRAFFIC.get("sha") == sha else None
+    traffic = (TRAFFIC.get(dom) if TRAFFIC.get("sha") == sha and TRAFFIC.get("workload") == wl.name
+               else None)
+    esz = 2 if wl.dtype == "bf16" else 4
+    algo_bytes = sum(esz * (M * d["lin"].K + d["lin"].N * d["lin"].K + M * d["lin"].N)
+                     + 4 * (d["lin"].N * d["lin"].K // wl.g) * (9 if dom == "dw" else 6) for d in st) / len(st)
     roofline = {"bound": "tensor", "kernel": kernel_name, "achieved": achieved, "peak": peaks["bf16_sus"],
                 "unit": UNIT, "frac": achieved / peaks["bf16_sus"], "traffic": traffic,
+                "traffic_algorithmic": algo_bytes,
                 "peak_kind": f"bf16 dense sustained ({peaks['source']})",
                 "frac_of_burst": achieved / peaks["bf16"],
                 "per_kernel_ms_per_step": {k: per[k] / args.steps for k in kinds},
