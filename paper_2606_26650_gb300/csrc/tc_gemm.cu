@@ -83,7 +83,8 @@ struct FusedCfg {
   static constexpr int kRawPeriod = kStagesW / gcd_c(kStagesW, kStep) * kStep;
   static constexpr int kRawBars = kProdGroups * kStagesW;
   static_assert(kRawBars <= 32, "issued-barrier masks are 32 bits");
-  static constexpr int kBarBytes = 8 * (2 * kStagesA + kRawBars + 4 * kStagesW + 3) + 16;
+  static constexpr int kRowsPerWarp = 32 / kThreadsPerRow;     // operand rows one producer warp owns
+  static constexpr int kBarBytes = 8 * (2 * kStagesA + kRawBars + 3 * kStagesW + 3) + 16;
   static constexpr int kSmemBytes = kStagesA * kABytes + kStagesW * kWBytes + 1024 + kBarBytes;
 };
 
@@ -228,12 +229,11 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
   auto raw_w = [&](int b) { return bars + 8u * (2 * SA + b); };          // raw W landed [group][slot] (local)
   auto full_w = [&](int s) { return bars + 8u * (2 * SA + RB + s); };   // operand ready (pair: even CTA)
   auto empty_w = [&](int s) { return bars + 8u * (2 * SA + RB + SW + s); };
-  auto prod_done = [&](int s) { return bars + 8u * (2 * SA + RB + 2 * SW + s); };  // PAIRS 2: local producers done
-  auto recv_w = [&](int s) { return bars + 8u * (2 * SA + RB + 3 * SW + s); };     // PAIRS 2: operand received
-  const uint32_t tmem_full_bar = bars + 8u * (2 * SA + RB + 4 * SW);
+  auto recv_w = [&](int s) { return bars + 8u * (2 * SA + RB + 2 * SW + s); };  // PAIRS 2: received half landed
+  const uint32_t tmem_full_bar = bars + 8u * (2 * SA + RB + 3 * SW);
   const uint32_t tmem_empty_bar = tmem_full_bar + 8;
   const uint32_t final_bar = tmem_full_bar + 16;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base_ptr + (bars - base) + 8 * (2 * SA + RB + 4 * SW + 3));
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base_ptr + (bars - base) + 8 * (2 * SA + RB + 3 * SW + 3));
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = CG == 2 ? cluster_ctarank() : 0u;
@@ -255,11 +255,16 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     }
     for (int b = 0; b < RB; ++b) mbar_init(raw_w(b), 1);
     for (int s = 0; s < SW; ++s) {
-      // PAIRS 1: one arrival per producer warp of the pair; PAIRS 2: one forwarded arrival per CTA
-      mbar_init(full_w(s), PAIRS == 1 ? Cfg::kGroupWarps * CG : 2);
+      // With two pairs, slot s is always produced by pair s & 1 (the ring depth is even).
+      const bool received = PAIRS == 2 && (static_cast<uint32_t>(s) & 1u) != pair;
+      // Produced slots: one arrival per producer warp of the pair.  Received slots: one
+      // arrival from the odd CTA once its half has landed (the MMA waits on its own half).
+      mbar_init(full_w(s), received ? 1 : Cfg::kGroupWarps * CG);
       mbar_init(empty_w(s), PAIRS);  // every pair's MMA frees the slot in all CTAs
-      mbar_init(prod_done(s), Cfg::kGroupWarps);
       mbar_init(recv_w(s), 1);
+      // A receive barrier is armed for the slot's next use as soon as its current use has
+      // landed; this arms the first use.
+      if (received) mbar_arrive_expect_tx(recv_w(s), Cfg::kWBytes);
     }
     mbar_init(tmem_full_bar, 1);
     mbar_init(tmem_empty_bar, Cfg::kEpiWarps * CG);
@@ -333,33 +338,6 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
       }
       for (int b = 0; b < RB; ++b)
         if (issued_mask & (1u << b)) mbar_wait_drain(raw_w(b), (issued_phase >> b) & 1u);
-    } else if (PAIRS == 2 && (lane == 2 || lane == 3)) {
-      // ---------------------------------------------------------- operand exchange between the pairs
-      // Lane 2, produced stages: once this CTA's producers are done, copy the half-tile to the
-      // same slot of the other pair's CTA with the same half, then report it ready to this
-      // pair's MMA.  Lane 3, received stages: arm the slot's receive barrier when the slot is
-      // free, wait for the copy, then report it ready.  Separate lanes, so neither direction
-      // waits for the other.
-      const uint32_t partner = rank ^ 2u;
-      const bool sender = lane == 2;
-      uint32_t q = 0;
-      bool ok = true;
-      for (int t = cluster; ok && t < num_tiles; t += nclusters) {
-        for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
-          if (produces(q) != sender) continue;
-          const uint32_t s = q % SW, ph = (q / SW) & 1u;
-          if (sender) {
-            if (!mbar_wait(prod_done(s), ph, wc)) { ok = false; break; }
-            bulk_copy_to_peer(mapa_shared(w_base + s * Cfg::kWBytes, partner), w_base + s * Cfg::kWBytes,
-                              Cfg::kWBytes, mapa_shared(recv_w(s), partner));
-          } else {
-            if (!mbar_wait(empty_w(s), ph ^ 1u, wc)) { ok = false; break; }
-            mbar_arrive_expect_tx(recv_w(s), Cfg::kWBytes);
-            if (!mbar_wait(recv_w(s), ph, wc)) { ok = false; break; }
-          }
-          mbar_arrive_cluster(leader_full_w0 + 8u * s);
-        }
-      }
     }
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer (even CTA of each pair)
@@ -372,7 +350,13 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
         tc_fence_after();
         for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
           const uint32_t sa = q % SA, pa = (q / SA) & 1u, sw = q % SW, pw = (q / SW) & 1u;
-          if (!mbar_wait(full_a(sa), pa, wc) || !mbar_wait(full_w(sw), pw, wc)) { ok = false; break; }
+          if (!mbar_wait(full_a(sa), pa, wc)) { ok = false; break; }
+          if (PAIRS == 2 && (q & 1u) != pair) {
+            // Received stage: this CTA's half came from the other pair; arm the slot's next use.
+            if (!mbar_wait(recv_w(sw), pw, wc)) { ok = false; break; }
+            mbar_arrive_expect_tx(recv_w(sw), Cfg::kWBytes);
+          }
+          if (!mbar_wait(full_w(sw), pw, wc)) { ok = false; break; }
           tc_fence_after();
           const uint32_t aa = a_base + sa * Cfg::kABytes, ww = w_base + sw * Cfg::kWBytes;
 #pragma unroll
@@ -401,6 +385,21 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
       if constexpr (PAIRS == 1) umma_commit<CG>(final_bar);
       else umma_commit_pair_mask(final_bar, pair_mask);
       mbar_wait_drain(final_bar, 0);
+    } else if (PAIRS == 2 && cta == 1 && lane == 0) {
+      // ---------------------------------------------------------- odd CTA: received stages
+      // Once this CTA's half of a received stage has landed, arm the slot's next use and
+      // report the half to the pair's MMA.
+      uint32_t q = 0;
+      bool ok = true;
+      for (int t = cluster; ok && t < num_tiles; t += nclusters) {
+        for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
+          if ((q & 1u) == pair) continue;
+          const uint32_t s = q % SW, ph = (q / SW) & 1u;
+          if (!mbar_wait(recv_w(s), ph, wc)) { ok = false; break; }
+          mbar_arrive_expect_tx(recv_w(s), Cfg::kWBytes);
+          mbar_arrive_cluster(leader_full_w0 + 8u * s);
+        }
+      }
     }
   } else if (warp < Cfg::kEpiWarps) {
     // ------------------------------------------------------------ epilogue
@@ -438,6 +437,12 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     constexpr int STEP = Cfg::kStep;
     const int pw = warp - (Cfg::kEpiWarps + 2);  // producer warp index
     const int grp = pw / Cfg::kGroupWarps;
+    // PAIRS 2: this warp's rows of a produced half-tile go to the same slot of the CTA with
+    // the same half in the other pair.
+    const uint32_t my_rows = static_cast<uint32_t>(pw % Cfg::kGroupWarps) * Cfg::kRowsPerWarp * 128u;
+    const uint32_t peer = rank ^ 2u;
+    const uint32_t peer_w = PAIRS == 2 ? mapa_shared(w_base + my_rows, peer) : 0u;
+    const uint32_t peer_recv0 = PAIRS == 2 ? mapa_shared(recv_w(0), peer) : 0u;
     const int tt = threadIdx.x - 32 * (Cfg::kEpiWarps + 2) - grp * Cfg::kGroupThreads;
     const int row = tt / Cfg::kThreadsPerRow;
     const int c_begin = (tt % Cfg::kThreadsPerRow) * CPT;
@@ -503,8 +508,10 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
       }
       __syncwarp();
       if (lane == 0) {
-        if constexpr (PAIRS == 1) mbar_arrive_cluster(leader_full_w0 + 8u * s);
-        else mbar_arrive_local(prod_done(s));
+        if constexpr (PAIRS == 2)
+          bulk_copy_to_peer(peer_w + s * Cfg::kWBytes, w_base + my_rows + s * Cfg::kWBytes, Cfg::kRowsPerWarp * 128u,
+                            peer_recv0 + 8u * s);
+        mbar_arrive_cluster(leader_full_w0 + 8u * s);
       }
       // Issued after the proxy fence, which would otherwise wait for these loads.
       request(ahead, mine, jm, other, jo);
