@@ -131,16 +131,45 @@ __device__ __forceinline__ bool mbar_wait_drain(uint32_t bar, uint32_t parity) {
   return true;
 }
 
-__device__ __forceinline__ void store_bf16x32(uint16_t* dst, const uint32_t (&r)[32], int64_t cols_left) {
+// 32 fp32 accumulator columns of one row per lane (32 rows per warp, 32 consecutive columns
+// from `col`) stored as bf16.  A 4 x 4 transpose of 16-byte chunks inside each group of four
+// lanes (two xor-shuffle rounds) turns the lane-per-row layout into stores where four lanes
+// cover 64 contiguous bytes of one row, so each store instruction writes 8 row segments
+// instead of touching 32 rows.  ncols is a multiple of 8, so a chunk is wholly in or out.
+__device__ __forceinline__ void store_rows_bf16x32(uint16_t* C, int64_t M, int64_t ncols, int64_t row0, int64_t col,
+                                                   const uint32_t (&r)[32], int lane) {
+  uint4 v[4];
 #pragma unroll
   for (int p = 0; p < 4; ++p) {
-    if (8 * p >= cols_left) break;
-    uint4 v;
-    v.x = pack_bf16x2(__uint_as_float(r[8 * p + 0]), __uint_as_float(r[8 * p + 1]));
-    v.y = pack_bf16x2(__uint_as_float(r[8 * p + 2]), __uint_as_float(r[8 * p + 3]));
-    v.z = pack_bf16x2(__uint_as_float(r[8 * p + 4]), __uint_as_float(r[8 * p + 5]));
-    v.w = pack_bf16x2(__uint_as_float(r[8 * p + 6]), __uint_as_float(r[8 * p + 7]));
-    *reinterpret_cast<uint4*>(dst + 8 * p) = v;
+    v[p].x = pack_bf16x2(__uint_as_float(r[8 * p + 0]), __uint_as_float(r[8 * p + 1]));
+    v[p].y = pack_bf16x2(__uint_as_float(r[8 * p + 2]), __uint_as_float(r[8 * p + 3]));
+    v[p].z = pack_bf16x2(__uint_as_float(r[8 * p + 4]), __uint_as_float(r[8 * p + 5]));
+    v[p].w = pack_bf16x2(__uint_as_float(r[8 * p + 6]), __uint_as_float(r[8 * p + 7]));
+  }
+  // Round k exchanges chunk pairs (p, p | k) with lane ^ k; afterwards lane 4a + i holds
+  // chunk i of rows 4a .. 4a + 3 in v[0 .. 3].
+#pragma unroll
+  for (int k = 1; k <= 2; k <<= 1) {
+    const bool upper = (lane & k) != 0;
+#pragma unroll
+    for (int p = 0; p < 4; ++p) {
+      if (p & k) continue;
+      const uint4 send = upper ? v[p] : v[p | k];
+      uint4 got;
+      got.x = __shfl_xor_sync(0xffffffffu, send.x, k);
+      got.y = __shfl_xor_sync(0xffffffffu, send.y, k);
+      got.z = __shfl_xor_sync(0xffffffffu, send.z, k);
+      got.w = __shfl_xor_sync(0xffffffffu, send.w, k);
+      if (upper) v[p] = got;
+      else v[p | k] = got;
+    }
+  }
+  const int64_t c = col + 8 * (lane & 3);
+  if (c >= ncols) return;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int64_t row = row0 + (lane & ~3) + j;
+    if (row < M) *reinterpret_cast<uint4*>(C + row * ncols + c) = v[j];
   }
 }
 
@@ -411,15 +440,16 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
       tc_fence_after();
 #pragma unroll 1
       for (int acc = 0; acc < NACC; ++acc) {
-        const int64_t row = (int64_t)m_blk * (Cfg::kTileRows * PAIRS) + pair * Cfg::kTileRows +
-                            acc * Cfg::kRowsPerAcc + cta * 128 + qd * 32 + lane;
+        const int64_t row0 = (int64_t)m_blk * (Cfg::kTileRows * PAIRS) + pair * Cfg::kTileRows +
+                             acc * Cfg::kRowsPerAcc + cta * 128 + qd * 32;  // this warp's first row
 #pragma unroll 1
         for (int c = 0; c < BN / 32; ++c) {
+          const int64_t col = (int64_t)n_blk * BN + c * 32;
+          if (col >= args.ncols || row0 >= args.M) break;  // warp-uniform
           uint32_t r[32];
           tmem_ld32(tmem_base + (static_cast<uint32_t>(qd * 32) << 16) + acc * BN + c * 32, r);
           tmem_ld_wait();
-          const int64_t col = (int64_t)n_blk * BN + c * 32;
-          if (row < args.M && col < args.ncols) store_bf16x32(args.C + row * args.ncols + col, r, args.ncols - col);
+          store_rows_bf16x32(args.C, args.M, args.ncols, row0, col, r, lane);
         }
       }
       tc_fence_before();
