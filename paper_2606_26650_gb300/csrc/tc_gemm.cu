@@ -52,8 +52,11 @@ constexpr int gcd_c(int a, int b) { return b == 0 ? a : gcd_c(b, a % b); }
 // against the same produced operand tiles; each pair produces every other stage and sends
 // its transformed half-tiles to the other pair's CTAs through distributed shared memory,
 // which halves the per-SM transform work.
-template <int CG, int PAIRS = 1>
+// DEEP_W (two pairs only) trades an A stage for two operand slots: the operand ring's round
+// trip grows with the transform's cost (the two-tanh form doubles it), the A ring's does not.
+template <int CG, int PAIRS = 1, bool DEEP_W = false>
 struct FusedCfg {
+  static_assert(!DEEP_W || PAIRS == 2, "the deep operand ring is a four-CTA layout");
   static_assert(PAIRS == 1 || CG == 2, "pairs of pairs need CTA pairs");
   static constexpr int kClusterCtas = CG * PAIRS;
   static constexpr int kRowsPerAcc = 128 * CG;          // MMA M
@@ -61,10 +64,10 @@ struct FusedCfg {
   static constexpr int kBRows = BN / CG;                // 128-byte operand rows per CTA per stage
   static constexpr int kABytes = NACC * 128 * BK * 2;   // this CTA's A rows per stage
   static constexpr int kWBytes = kBRows * BK * 2;       // this CTA's operand rows per stage
-  static constexpr int kStagesA = CG == 1 ? 3 : 4;      // A ring: TMA -> MMA
+  static constexpr int kStagesA = (CG == 1 || DEEP_W) ? 3 : 4;  // A ring: TMA -> MMA
   // W ring: TMA -> producers (in place) -> MMA.  Even with two pairs, so every slot is always
   // produced by the same pair (and received by the other).
-  static constexpr int kStagesW = PAIRS == 2 ? 6 : (CG == 1 ? 3 : 5);
+  static constexpr int kStagesW = PAIRS == 2 ? (DEEP_W ? 8 : 6) : (CG == 1 ? 3 : 5);
   static constexpr int kEpiWarps = 4;
   // Two groups of 8 producer warps take alternate stages (of the ones this CTA produces), so
   // each group has two stage periods per operand tile and the groups' MUFU work interleaves.
@@ -239,11 +242,11 @@ struct OperandRowIter {
   }
 };
 
-template <int CG, bool B_MN, int PAIRS>
-__global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
+template <int CG, bool B_MN, int PAIRS, bool DEEP_W>
+__global__ void __launch_bounds__(FusedCfg<CG, PAIRS, DEEP_W>::kThreads, 1)
     fused_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
                       const FusedArgs args) {
-  using Cfg = FusedCfg<CG, PAIRS>;
+  using Cfg = FusedCfg<CG, PAIRS, DEEP_W>;
   constexpr int SA = Cfg::kStagesA, SW = Cfg::kStagesW;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = smem_u32(smem_raw);
@@ -286,14 +289,15 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     for (int s = 0; s < SW; ++s) {
       // With two pairs, slot s is always produced by pair s & 1 (the ring depth is even).
       const bool received = PAIRS == 2 && (static_cast<uint32_t>(s) & 1u) != pair;
-      // Produced slots: one arrival per producer warp of the pair.  Received slots: one
-      // arrival from the odd CTA once its half has landed (the MMA waits on its own half).
-      mbar_init(full_w(s), received ? 1 : Cfg::kGroupWarps * CG);
+      // Produced slots: one arrival per producer warp of the pair.  Received slots: the even
+      // CTA's half lands on full_w itself (the copies complete their bytes there), which the
+      // MMA thread arms, plus one arrival from the odd CTA once its half has landed.
+      mbar_init(full_w(s), received ? 2 : Cfg::kGroupWarps * CG);
       mbar_init(empty_w(s), PAIRS);  // every pair's MMA frees the slot in all CTAs
-      mbar_init(recv_w(s), 1);
-      // A receive barrier is armed for the slot's next use as soon as its current use has
-      // landed; this arms the first use.
-      if (received) mbar_arrive_expect_tx(recv_w(s), Cfg::kWBytes);
+      mbar_init(recv_w(s), 1);       // odd CTA: its received half landed
+      // Barriers that count received bytes are armed for a slot's next use as soon as its
+      // current use has landed; this arms the first use.
+      if (received) mbar_arrive_expect_tx(cta == 0 ? full_w(s) : recv_w(s), Cfg::kWBytes);
     }
     mbar_init(tmem_full_bar, 1);
     mbar_init(tmem_empty_bar, Cfg::kEpiWarps * CG);
@@ -379,13 +383,9 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
         tc_fence_after();
         for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
           const uint32_t sa = q % SA, pa = (q / SA) & 1u, sw = q % SW, pw = (q / SW) & 1u;
-          if (!mbar_wait(full_a(sa), pa, wc)) { ok = false; break; }
-          if (PAIRS == 2 && (q & 1u) != pair) {
-            // Received stage: this CTA's half came from the other pair; arm the slot's next use.
-            if (!mbar_wait(recv_w(sw), pw, wc)) { ok = false; break; }
-            mbar_arrive_expect_tx(recv_w(sw), Cfg::kWBytes);
-          }
-          if (!mbar_wait(full_w(sw), pw, wc)) { ok = false; break; }
+          if (!mbar_wait(full_a(sa), pa, wc) || !mbar_wait(full_w(sw), pw, wc)) { ok = false; break; }
+          // Received stage: both halves are here; arm the slot's next use.
+          if (PAIRS == 2 && (q & 1u) != pair) mbar_arrive_expect_tx(full_w(sw), Cfg::kWBytes);
           tc_fence_after();
           const uint32_t aa = a_base + sa * Cfg::kABytes, ww = w_base + sw * Cfg::kWBytes;
 #pragma unroll
@@ -472,7 +472,8 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     const uint32_t my_rows = static_cast<uint32_t>(pw % Cfg::kGroupWarps) * Cfg::kRowsPerWarp * 128u;
     const uint32_t peer = rank ^ 2u;
     const uint32_t peer_w = PAIRS == 2 ? mapa_shared(w_base + my_rows, peer) : 0u;
-    const uint32_t peer_recv0 = PAIRS == 2 ? mapa_shared(recv_w(0), peer) : 0u;
+    // the peer's barrier that counts the bytes: full_w in an even CTA, recv_w in an odd one
+    const uint32_t peer_recv0 = PAIRS == 2 ? mapa_shared(cta == 0 ? full_w(0) : recv_w(0), peer) : 0u;
     const int tt = threadIdx.x - 32 * (Cfg::kEpiWarps + 2) - grp * Cfg::kGroupThreads;
     const int row = tt / Cfg::kThreadsPerRow;
     const int c_begin = (tt % Cfg::kThreadsPerRow) * CPT;
@@ -878,10 +879,10 @@ int max_active_clusters(Kern kern, int cluster_ctas, int threads, int smem, int 
 // CTA pairs (512 rows) from 512 rows, single CTAs below.
 int fused_variant_for(int64_t M) { return M >= 1024 ? 4 : (M >= 512 ? 2 : 1); }
 
-template <int CG, bool B_MN, int PAIRS>
+template <int CG, bool B_MN, int PAIRS, bool DEEP_W = false>
 cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t M, int64_t depth, void* C,
                       int64_t ncols, cudaStream_t st) {
-  using Cfg = FusedCfg<CG, PAIRS>;
+  using Cfg = FusedCfg<CG, PAIRS, DEEP_W>;
   DeviceInfo& d = device_info();
   if (!d.ok) return cudaErrorInvalidDevice;
   CUtensorMap ta, tw;
@@ -901,7 +902,7 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
   args.num_n_tiles = static_cast<int32_t>((ncols + BN - 1) / BN);
   args.num_k_blocks = static_cast<int32_t>((depth + BK - 1) / BK);
   args.wc = make_wait_ctl(d);
-  auto kern = fused_gemm_kernel<CG, B_MN, PAIRS>;
+  auto kern = fused_gemm_kernel<CG, B_MN, PAIRS, DEEP_W>;
   const int tiles = args.num_m_tiles * args.num_n_tiles;
   const int fit = max_active_clusters(kern, Cfg::kClusterCtas, Cfg::kThreads, Cfg::kSmemBytes,
                                       d.sm_count / Cfg::kClusterCtas);
@@ -961,9 +962,17 @@ TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count) {
   return p;
 }
 
+// SOFT steps with s below this mostly take the two-tanh form of Eq. 5 (s Delta < 6 for the
+// usual Delta near 0.5), whose longer transform wants the deep operand ring.
+constexpr float kDeepRingMaxS = 12.0f;
+
+bool deep_operand_ring(const StepScalars& sc) { return sc.phase == PHASE_SOFT && sc.s < kDeepRingMaxS; }
+
 cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st) {
   switch (fused_variant_for(M)) {
-    case 4: return run_fused<2, false, 2>(L, sc, X, M, L.K, Y, L.N, st);
+    case 4:
+      if (deep_operand_ring(sc)) return run_fused<2, false, 2, true>(L, sc, X, M, L.K, Y, L.N, st);
+      return run_fused<2, false, 2>(L, sc, X, M, L.K, Y, L.N, st);
     case 2: return run_fused<2, false, 1>(L, sc, X, M, L.K, Y, L.N, st);
     default: return run_fused<1, false, 1>(L, sc, X, M, L.K, Y, L.N, st);
   }
@@ -971,7 +980,9 @@ cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int6
 
 cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int64_t M, void* dX, cudaStream_t st) {
   switch (fused_variant_for(M)) {
-    case 4: return run_fused<2, true, 2>(L, sc, dY, M, L.N, dX, L.K, st);
+    case 4:
+      if (deep_operand_ring(sc)) return run_fused<2, true, 2, true>(L, sc, dY, M, L.N, dX, L.K, st);
+      return run_fused<2, true, 2>(L, sc, dY, M, L.N, dX, L.K, st);
     case 2: return run_fused<2, true, 1>(L, sc, dY, M, L.N, dX, L.K, st);
     default: return run_fused<1, true, 1>(L, sc, dY, M, L.N, dX, L.K, st);
   }
