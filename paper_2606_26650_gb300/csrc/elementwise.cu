@@ -91,11 +91,27 @@ __device__ __forceinline__ void store_group_stats(int64_t j, int32_t g, int32_t 
 }
 
 // ---------------------------------------------------------------- Eq. 3 statistics
-// Register variant: a team of `team` lanes owns one group and keeps its R x 16-byte
-// vectors in registers (mean, then deviations, without re-reading W); each warp works on
-// two rounds of groups at once so two loads per lane are in flight.  The signed sum (mean)
-// is compensated; the all-positive deviation and magnitude sums are pairwise fp32, whose
-// relative error stays below ~10 ulp for these group sizes.
+// Register variant: a team of `team` lanes owns one group and each lane keeps kStatsVPL
+// 16-byte vectors of it in registers, so the mean and the deviations need one read of W.
+// Lane `sub` of a team takes vectors sub, sub + team, ..., so each load instruction of a
+// team reads team x 16 contiguous bytes.  A vector is summed pairwise in fp32 and added to a
+// compensated (two-sum) accumulator, the team merges the compensated sums, and the
+// all-positive deviation and magnitude sums are plain pairwise fp32 sums (relative error a
+// few ulp).  The magnitude sum is only formed for the TWN threshold rule.
+constexpr int kStatsVPL = 4;
+
+template <int V>
+__device__ __forceinline__ float pairwise_sum(const float (&x)[V]) {
+  float t[V];
+#pragma unroll
+  for (int q = 0; q < V; ++q) t[q] = x[q];
+#pragma unroll
+  for (int w = 1; w < V; w <<= 1)
+#pragma unroll
+    for (int q = 0; q + w < V; q += 2 * w) t[q] += t[q + w];
+  return t[0];
+}
+
 template <int V>
 __device__ __forceinline__ float pairwise_abs_sum(const float (&x)[V], float shift) {
   float t[V];
@@ -113,59 +129,50 @@ __device__ __forceinline__ float team_sum(float v, int team) {
   return v;
 }
 
-template <typename T, int R>
-__global__ void __launch_bounds__(kThreads) group_stats_reg_kernel(const T* __restrict__ W, int64_t G, int32_t g,
-                                                                   int32_t team, int32_t thr_init,
-                                                                   float* __restrict__ mu0,
-                                                                   float* __restrict__ alpha0,
-                                                                   float* __restrict__ delta0) {
+template <typename T, bool TWN>
+__global__ void __launch_bounds__(kThreads) group_stats_team_kernel(const T* __restrict__ W, int64_t G, int32_t g,
+                                                                    int32_t team, float* __restrict__ mu0,
+                                                                    float* __restrict__ alpha0,
+                                                                    float* __restrict__ delta0) {
   constexpr int V = Vec16<T>::n;
-  constexpr int ROUNDS = 2;
+  constexpr int VPL = kStatsVPL;
   const int lane = threadIdx.x & 31;
-  const int sub = lane % team;
+  const int sub = lane & (team - 1);
   const int per_warp = 32 / team;
   const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
   const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
   const float inv_g = 1.0f / static_cast<float>(g);
-  for (int64_t wbase = warp * per_warp * ROUNDS; wbase < G; wbase += nwarps * per_warp * ROUNDS) {
-    float v[ROUNDS][R][V];
-    int64_t jr[ROUNDS];
+  for (int64_t wbase = warp * per_warp; wbase < G; wbase += nwarps * per_warp) {
+    const int64_t j = wbase + lane / team;
+    const bool live = j < G;
+    float v[VPL][V];
 #pragma unroll
-    for (int u = 0; u < ROUNDS; ++u) {
-      jr[u] = wbase + u * per_warp + lane / team;
+    for (int r = 0; r < VPL; ++r) {
+      if (live) {
+        Vec16<T>::load(W + j * g + static_cast<int64_t>(r * team + sub) * V, v[r]);
+      } else {
 #pragma unroll
-      for (int r = 0; r < R; ++r) {
-        if (jr[u] < G) {
-          Vec16<T>::load(W + jr[u] * g + static_cast<int64_t>(sub + r * team) * V, v[u][r]);
-        } else {
-#pragma unroll
-          for (int q = 0; q < V; ++q) v[u][r][q] = 0.f;
-        }
+        for (int q = 0; q < V; ++q) v[r][q] = 0.f;
       }
     }
+    Sum2 sum{0.f, 0.f};
 #pragma unroll
-    for (int u = 0; u < ROUNDS; ++u) {
-      Sum2 sum{0.f, 0.f};
+    for (int r = 0; r < VPL; ++r) sum2_add(sum, pairwise_sum<V>(v[r]));
+    sum = sum2_team(sum, team);
+    const float mu = sum2_float(sum) * inv_g;
+    float dev = 0.f, mag = 0.f;
 #pragma unroll
-      for (int r = 0; r < R; ++r)
-#pragma unroll
-        for (int q = 0; q < V; ++q) sum2_add(sum, v[u][r][q]);
-      sum = sum2_team(sum, team);
-      const float mu = sum2_float(sum) * inv_g;
-      float dev = 0.f, mag = 0.f;
-#pragma unroll
-      for (int r = 0; r < R; ++r) {
-        dev += pairwise_abs_sum<V>(v[u][r], mu);
-        mag += pairwise_abs_sum<V>(v[u][r], 0.0f);
-      }
-      dev = team_sum(dev, team);
-      mag = team_sum(mag, team);
-      if (jr[u] < G && sub == 0) {
-        const float a0 = dev * inv_g;
-        mu0[jr[u]] = mu;
-        alpha0[jr[u]] = a0;
-        delta0[jr[u]] = (thr_init == 1 && a0 > 0.0f) ? 0.7f * (mag * inv_g) / a0 : 0.5f;
-      }
+    for (int r = 0; r < VPL; ++r) {
+      dev += pairwise_abs_sum<V>(v[r], mu);
+      if constexpr (TWN) mag += pairwise_abs_sum<V>(v[r], 0.0f);
+    }
+    dev = team_sum(dev, team);
+    if constexpr (TWN) mag = team_sum(mag, team);
+    if (live && sub == 0) {
+      const float a0 = dev * inv_g;
+      mu0[j] = mu;
+      alpha0[j] = a0;
+      delta0[j] = (TWN && a0 > 0.0f) ? 0.7f * (mag * inv_g) / a0 : 0.5f;
     }
   }
 }
@@ -305,6 +312,66 @@ __global__ void __launch_bounds__(kThreads) hard_pack_kernel(LayerDev L, uint8_t
       alpha[j] = __ldg(L.d_alpha + j) * __ldg(L.alpha0 + j);
 }
 
+// Warp-cooperative pack for power-of-two g >= 8 V: a warp takes batches of 32 x 8 16-byte
+// chunks; load c of lane l reads chunk 32 c + l, so each load instruction covers 512
+// contiguous bytes.  The at most 32 groups a batch touches get their constants from one
+// lane each (alpha = 0 groups get a threshold no value exceeds, so their codes are 0) and
+// reach the lanes that need them by shuffles.  A chunk's V elements lie in one group and give
+// 2 V code bits.
+template <typename T>
+__global__ void __launch_bounds__(kThreads) hard_pack_warp_kernel(LayerDev L, int32_t log2g,
+                                                                  uint8_t* __restrict__ codes,
+                                                                  float* __restrict__ alpha) {
+  constexpr int V = Vec16<T>::n;
+  constexpr int kLoads = 8;
+  constexpr int64_t kBatch = 32 * kLoads * V;  // elements per warp batch
+  const int64_t n = L.N * L.K;
+  const int64_t G = n >> log2g;
+  const T* W = static_cast<const T*>(L.W);
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
+  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
+  for (int64_t b0 = warp * kBatch; b0 < n; b0 += nwarps * kBatch) {
+    const int64_t j0 = b0 >> log2g;
+    const int64_t jl = j0 + lane;
+    float r = 0.0f, b = 0.0f, delta = __int_as_float(0x7f800000);  // +inf
+    if (jl < G && (jl << log2g) < b0 + kBatch) {
+      const GroupConst gc = group_const(L, jl);
+      if (gc.alpha != 0.0f) {
+        r = gc.r;
+        b = gc.b;
+        delta = gc.delta;
+      }
+      if (alpha && (jl << log2g) >= b0) alpha[jl] = gc.alpha;  // the batch holding the group's start
+    }
+    const int first = static_cast<int>(b0 - (j0 << log2g));  // offset of b0 inside group j0
+#pragma unroll
+    for (int c = 0; c < kLoads; ++c) {
+      const int off = (c * 32 + lane) * V;  // element offset inside the batch
+      const int src = (first + off) >> log2g;
+      const float rr = __shfl_sync(0xffffffffu, r, src);
+      const float bb = __shfl_sync(0xffffffffu, b, src);
+      const float dd = __shfl_sync(0xffffffffu, delta, src);
+      const int64_t e = b0 + off;
+      if (e < n) {
+        float v[V];
+        Vec16<T>::load(W + e, v);
+        uint32_t bits = 0;
+#pragma unroll
+        for (int k = 0; k < V; ++k) {
+          const float x = fmaf(v[k], rr, bb);
+          const int q = x > dd ? 1 : (x < -dd ? -1 : 0);
+          bits |= static_cast<uint32_t>(q + 1) << (2 * k);
+        }
+        if constexpr (V == 8)
+          reinterpret_cast<uint16_t*>(codes)[e / 8] = static_cast<uint16_t>(bits);
+        else
+          codes[e / 4] = static_cast<uint8_t>(bits);
+      }
+    }
+  }
+}
+
 // ---------------------------------------------------------------- Eq. 7 loss and dY
 constexpr int kLossMaxBlocks = 1216;
 
@@ -428,23 +495,22 @@ cudaError_t launch_group_stats(const LayerDev& L, int32_t w_dtype, int32_t thr_i
   const int64_t G = L.N * L.K / L.g;
   const int V = w_dtype == 1 ? 8 : 4;  // elements per 16-byte vector
   const int nvec = L.g / V;            // vectors per group
-  if (L.g % V == 0 && nvec <= 128 && (nvec & (nvec - 1)) == 0) {
-    const int team = nvec < 32 ? nvec : 32;
-    const int R = nvec / team;
-    const int grid = grid_for((G + 2 * (32 / team) - 1) / (2 * (32 / team)), kThreads / 32);
-#define CATQ_STATS_REG(TT, RR)                                                                                  \
-  group_stats_reg_kernel<TT, RR><<<grid, kThreads, 0, st>>>(static_cast<const TT*>(L.W), G, L.g, team, thr_init, \
-                                                            mu0, alpha0, delta0)
+  const int team = nvec / kStatsVPL;
+  if (L.g % V == 0 && nvec % kStatsVPL == 0 && team <= 32 && (team & (team - 1)) == 0) {
+    const int per_warp = 32 / team;
+    const int grid = grid_for((G + per_warp - 1) / per_warp, kThreads / 32);
+    const bool twn = thr_init == 1;
+#define CATQ_STATS_TEAM(TT, TWN)                                                                                  \
+  group_stats_team_kernel<TT, TWN><<<grid, kThreads, 0, st>>>(static_cast<const TT*>(L.W), G, L.g, team, mu0, \
+                                                              alpha0, delta0)
     if (w_dtype == 1) {
-      if (R == 1) CATQ_STATS_REG(__nv_bfloat16, 1);
-      else if (R == 2) CATQ_STATS_REG(__nv_bfloat16, 2);
-      else CATQ_STATS_REG(__nv_bfloat16, 4);
+      if (twn) CATQ_STATS_TEAM(__nv_bfloat16, true);
+      else CATQ_STATS_TEAM(__nv_bfloat16, false);
     } else {
-      if (R == 1) CATQ_STATS_REG(float, 1);
-      else if (R == 2) CATQ_STATS_REG(float, 2);
-      else CATQ_STATS_REG(float, 4);
+      if (twn) CATQ_STATS_TEAM(float, true);
+      else CATQ_STATS_TEAM(float, false);
     }
-#undef CATQ_STATS_REG
+#undef CATQ_STATS_TEAM
     return cudaGetLastError();
   }
   const int grid = grid_for(G, kThreads / 32);
@@ -497,7 +563,17 @@ cudaError_t launch_recon_loss(const void* Y, const void* Yr, int64_t count, int3
 
 cudaError_t launch_hard_pack(const LayerDev& L, int32_t w_dtype, uint8_t* codes, float* alpha, cudaStream_t st) {
   const int64_t n = L.N * L.K;
-  if (L.g % 64 == 0) {
+  const int V = w_dtype == 1 ? 8 : 4;
+  if (L.g % 64 == 0 && (L.g & (L.g - 1)) == 0 && L.g >= 8 * V) {
+    int log2g = 0;
+    while ((1 << log2g) < L.g) ++log2g;
+    const int64_t batches = (n + 256LL * V - 1) / (256LL * V);
+    const int grid = grid_for(batches, kThreads / 32);
+    if (w_dtype == 1)
+      hard_pack_warp_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(L, log2g, codes, alpha);
+    else
+      hard_pack_warp_kernel<float><<<grid, kThreads, 0, st>>>(L, log2g, codes, alpha);
+  } else if (L.g % 64 == 0) {
     const int grid = grid_for(n / 64, kThreads);
     if (w_dtype == 1)
       hard_pack_kernel<__nv_bfloat16, 64><<<grid, kThreads, 0, st>>>(L, codes, alpha);

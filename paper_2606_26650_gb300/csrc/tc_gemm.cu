@@ -113,8 +113,19 @@ struct FusedArgs {
   int64_t M;        // rows of A and C
   int64_t ncols;    // columns of C
   int32_t num_m_tiles, num_n_tiles, num_k_blocks;
+  int32_t group_m;  // M blocks per raster group
   WaitCtl wc;
 };
+
+// Tile t of a persistent sequence -> (M block, N block).  Tiles run in groups of group_m M
+// blocks: inside a group the M block varies fastest, then the N block.
+__device__ __forceinline__ void tile_coords(const FusedArgs& a, int t, int& m_blk, int& n_blk) {
+  const int per_group = a.group_m * a.num_n_tiles;
+  const int grp = t / per_group, r = t - grp * per_group;
+  const int gm = min(a.group_m, a.num_m_tiles - grp * a.group_m);
+  m_blk = grp * a.group_m + r % gm;
+  n_blk = r / gm;
+}
 
 struct DwArgs {
   LayerDev L;
@@ -193,7 +204,8 @@ struct OperandRowIter {
   __device__ __forceinline__ void init(const FusedArgs& a, uint32_t cta, int row, int t_, int kb_) {
     t = t_;
     kb = kb_;
-    const int n_blk = t / a.num_m_tiles;
+    int m_blk, n_blk;
+    tile_coords(a, t, m_blk, n_blk);
     const int gk = a.L.g / BK;  // k blocks per group
     if constexpr (!B_MN) {
       n = (int64_t)n_blk * BN + cta * Cfg::kBRows + row;
@@ -326,7 +338,9 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS, DEEP_W>::kThreads, 1)
       uint32_t q = 0, issued_mask = 0, issued_phase = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
-        const int32_t m0 = (t % args.num_m_tiles) * (Cfg::kTileRows * PAIRS) + pair * Cfg::kTileRows;
+        int m_blk, n_blk;
+        tile_coords(args, t, m_blk, n_blk);
+        const int32_t m0 = m_blk * (Cfg::kTileRows * PAIRS) + pair * Cfg::kTileRows;
         for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
           const uint32_t s = q % SA, ph = (q / SA) & 1u;
           if (!mbar_wait(empty_a(s), ph ^ 1u, wc)) { ok = false; break; }
@@ -350,7 +364,9 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS, DEEP_W>::kThreads, 1)
       uint32_t q = 0, issued_mask = 0, issued_phase = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
-        const int32_t n0 = (t / args.num_m_tiles) * BN + cta * Cfg::kBRows;
+        int m_blk, n_blk;
+        tile_coords(args, t, m_blk, n_blk);
+        const int32_t n0 = n_blk * BN + cta * Cfg::kBRows;
         for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
           if (!produces(q)) continue;
           const uint32_t s = q % SW, ph = (q / SW) & 1u;
@@ -435,7 +451,8 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS, DEEP_W>::kThreads, 1)
     const int qd = warp;  // TMEM lane quarter
     uint32_t it = 0;
     for (int t = cluster; t < num_tiles; t += nclusters, ++it) {
-      const int m_blk = t % args.num_m_tiles, n_blk = t / args.num_m_tiles;
+      int m_blk, n_blk;
+      tile_coords(args, t, m_blk, n_blk);
       if (!mbar_wait(tmem_full_bar, it & 1u, wc)) break;
       tc_fence_after();
 #pragma unroll 1
@@ -901,6 +918,7 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
   args.num_m_tiles = static_cast<int32_t>((M + Cfg::kTileRows * PAIRS - 1) / (Cfg::kTileRows * PAIRS));
   args.num_n_tiles = static_cast<int32_t>((ncols + BN - 1) / BN);
   args.num_k_blocks = static_cast<int32_t>((depth + BK - 1) / BK);
+  args.group_m = std::min(4, args.num_m_tiles);
   args.wc = make_wait_ctl(d);
   auto kern = fused_gemm_kernel<CG, B_MN, PAIRS, DEEP_W>;
   const int tiles = args.num_m_tiles * args.num_n_tiles;
