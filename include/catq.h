@@ -100,10 +100,18 @@ typedef struct {
   const float* d_mu;    /* [G] learnable factor d_mu    (Eq. 3), -1 < d_mu < 1 */
   const float* d_alpha; /* [G] learnable factor d_alpha (Eq. 3), > 0 */
   const float* d_delta; /* [G] learnable factor d_delta (§2.2), > 0 */
+  /* [4*G] fp32, 16-byte aligned; required for bf16 layers by the forward and by a backward
+   * that computes dX, ignored otherwise.  Each such call first writes here the four
+   * per-group constants of its schedule point that turn a weight into its Eq. 6 operand
+   * (SOFT: s/alpha, -s mu/alpha, s Delta, alpha/(2 tanh s); HARD: 1/alpha, -mu/alpha,
+   * Delta, alpha), as float4 in group-column-major order [K/g][N], then the fused GEMMs
+   * read one 16-byte vector per group and row.  Contents are overwritten by every call, so
+   * two calls on one layer must not overlap on the GPU. */
+  float* op_const;
 } catq_layer;
 
 /* ABI version of this header; bumped on any incompatible change. */
-#define CATQ_ABI_VERSION 1
+#define CATQ_ABI_VERSION 2
 int32_t catq_abi_version(void);
 
 /* Human-readable name of a status code (static storage, never NULL). */
@@ -220,6 +228,7 @@ typedef struct {
   const float* d_mu;
   const float* d_alpha;
   const float* d_delta;
+  float* op_const; /* [E, 4*G]: per expert as catq_layer.op_const */
 } catq_grouped_layer;
 
 /* Forward of every expert: Y[rows of e] = X[rows of e] Wq_e^T (Eq. 6 weight per expert). */

@@ -40,6 +40,7 @@ class catq_layer(ctypes.Structure):
         ("W", ctypes.c_void_p),
         ("mu0", ctypes.c_void_p), ("alpha0", ctypes.c_void_p), ("delta0", ctypes.c_void_p),
         ("d_mu", ctypes.c_void_p), ("d_alpha", ctypes.c_void_p), ("d_delta", ctypes.c_void_p),
+        ("op_const", ctypes.c_void_p),
     ]
 
 
@@ -49,6 +50,7 @@ class catq_grouped_layer(ctypes.Structure):
         ("w_dtype", ctypes.c_int32), ("reserved", ctypes.c_int32), ("W", ctypes.c_void_p),
         ("mu0", ctypes.c_void_p), ("alpha0", ctypes.c_void_p), ("delta0", ctypes.c_void_p),
         ("d_mu", ctypes.c_void_p), ("d_alpha", ctypes.c_void_p), ("d_delta", ctypes.c_void_p),
+        ("op_const", ctypes.c_void_p),
     ]
 
 
@@ -132,7 +134,8 @@ def _check(status: int, where: str):
 
 @dataclasses.dataclass
 class Layer:
-    """One linear layer's device state: W [N, K] and the per-group arrays ([G] fp32)."""
+    """One linear layer's device state: W [N, K], the per-group arrays ([G] fp32) and the
+    operand-constant array the fused GEMMs read ([4 G] fp32)."""
     W: object
     g: int
     mu0: object
@@ -141,10 +144,12 @@ class Layer:
     d_mu: object
     d_alpha: object
     d_delta: object
+    op_const: object = None
 
     @classmethod
     def create(cls, W, g, d_mu=None, d_alpha=None, d_delta=None):
-        """Allocates the statistics and (identity, unless given) factor tensors."""
+        """Allocates the statistics, operand-constant and (identity, unless given) factor
+        tensors."""
         import torch
         N, K = W.shape
         G = N * K // g
@@ -152,7 +157,8 @@ class Layer:
         return cls(W, g, torch.empty(G, **kw), torch.empty(G, **kw), torch.empty(G, **kw),
                    d_mu if d_mu is not None else torch.zeros(G, **kw),
                    d_alpha if d_alpha is not None else torch.ones(G, **kw),
-                   d_delta if d_delta is not None else torch.ones(G, **kw))
+                   d_delta if d_delta is not None else torch.ones(G, **kw),
+                   torch.empty(4 * G, **kw))
 
     @property
     def N(self):
@@ -169,7 +175,8 @@ class Layer:
     def struct(self) -> catq_layer:
         return catq_layer(self.N, self.K, self.g, _dtype_code(self.W), self.W.data_ptr(),
                           self.mu0.data_ptr(), self.alpha0.data_ptr(), self.delta0.data_ptr(),
-                          self.d_mu.data_ptr(), self.d_alpha.data_ptr(), self.d_delta.data_ptr())
+                          self.d_mu.data_ptr(), self.d_alpha.data_ptr(), self.d_delta.data_ptr(),
+                          self.op_const.data_ptr() if self.op_const is not None else None)
 
 
 def schedule(phase: int, s: float = 0.0) -> catq_schedule:
@@ -276,7 +283,7 @@ class GroupedLayer:
         d = self.dense
         return catq_grouped_layer(E, self.g, N, K, _dtype_code(self.W), 0, self.W.data_ptr(), d.mu0.data_ptr(),
                                   d.alpha0.data_ptr(), d.delta0.data_ptr(), d.d_mu.data_ptr(), d.d_alpha.data_ptr(),
-                                  d.d_delta.data_ptr())
+                                  d.d_delta.data_ptr(), d.op_const.data_ptr() if d.op_const is not None else None)
 
 
 def _offsets(row_offsets):

@@ -41,6 +41,13 @@ catq_status check_layer(const catq_layer* L, bool need_factors) {
   return CATQ_OK;
 }
 
+// The fused bf16 GEMMs of a SOFT or HARD step read their operand constants from op_const.
+catq_status check_op_const(const catq_layer* L, catq_schedule sc) {
+  if (L->w_dtype != CATQ_BF16 || sc.phase == CATQ_PHASE_TEACHER) return CATQ_OK;
+  if (!L->op_const) return CATQ_ERR_INVALID_ARG;
+  return aligned16(L->op_const) ? CATQ_OK : CATQ_ERR_ALIGN;
+}
+
 catq_status check_schedule(catq_schedule sc, bool need_s) {
   if (sc.phase != CATQ_PHASE_TEACHER && sc.phase != CATQ_PHASE_SOFT && sc.phase != CATQ_PHASE_HARD)
     return CATQ_ERR_INVALID_ARG;
@@ -61,6 +68,7 @@ LayerDev to_dev(const catq_layer* L) {
   d.d_mu = L->d_mu;
   d.d_alpha = L->d_alpha;
   d.d_delta = L->d_delta;
+  d.op_const = reinterpret_cast<float4*>(L->op_const);
   return d;
 }
 
@@ -180,6 +188,7 @@ catq_status catq_soft_ternary_linear_fwd(const catq_layer* layer, catq_schedule 
   if (M == 0) return CATQ_OK;
   if (!X || !Y) return CATQ_ERR_INVALID_ARG;
   if (!aligned16(X) || !aligned16(Y)) return CATQ_ERR_ALIGN;
+  if ((st = check_op_const(layer, sched)) != CATQ_OK) return st;
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   const LayerDev L = to_dev(layer);
   if (layer->w_dtype == CATQ_F32)
@@ -211,6 +220,7 @@ catq_status catq_soft_ternary_linear_bwd(const catq_layer* layer, catq_schedule 
   if (M > 0) {
     if (!X || !dY) return CATQ_ERR_INVALID_ARG;
     if (!aligned16(X) || !aligned16(dY) || (dX && !aligned16(dX))) return CATQ_ERR_ALIGN;
+    if (dX && (st = check_op_const(layer, sched)) != CATQ_OK) return st;
   }
   TcPlan plan{};
   int32_t P = 0, splits = 0;
@@ -311,6 +321,7 @@ catq_layer expert_layer(const catq_grouped_layer* G, int32_t e) {
   L.d_mu = G->d_mu ? G->d_mu + e * groups : nullptr;
   L.d_alpha = G->d_alpha ? G->d_alpha + e * groups : nullptr;
   L.d_delta = G->d_delta ? G->d_delta + e * groups : nullptr;
+  L.op_const = G->op_const ? G->op_const + 4 * e * groups : nullptr;
   return L;
 }
 

@@ -20,6 +20,7 @@ struct LayerDev {
   const float* d_mu;
   const float* d_alpha;
   const float* d_delta;
+  float4* op_const;  // [K/g][N] operand constants (operand_const_vec), written per call
 };
 
 // Eq. 3 and §2.2 for group j:
@@ -141,6 +142,24 @@ __device__ __forceinline__ uint32_t hard_pair_bf16(uint32_t w2, const ProducerCo
   const float y0 = fabsf(x0) > p.delta ? copysignf(p.C, x0) : 0.0f;  // Q(x) = sign(x) [|x| > Delta]
   const float y1 = fabsf(x1) > p.delta ? copysignf(p.C, x1) : 0.0f;
   return pack_bf16x2(y0, y1);
+}
+
+// The four per-group values a producer row needs, packed for one 16-byte load:
+//   SOFT {A, B, D, C} = {s r, s b, s Delta, alpha / (2 tanh s)}, HARD {r, b, Delta, alpha}.
+__device__ __forceinline__ float4 operand_const_vec(const GroupConst& c, float s, float inv_2tanh_s, int32_t phase) {
+  const ProducerConst p = producer_const(c, s, inv_2tanh_s, phase);
+  return phase == PHASE_HARD ? make_float4(p.r, p.b, p.delta, p.C) : make_float4(p.A, p.B, p.D, p.C);
+}
+
+// Inverse of operand_const_vec for the transform of `phase`.
+__device__ __forceinline__ ProducerConst producer_const_from(float4 v) {
+  ProducerConst p;
+  p.A = p.r = v.x;
+  p.B = p.b = v.y;
+  p.D = p.delta = v.z;
+  p.C = v.w;
+  p.one_tanh = v.z >= 6.0f;
+  return p;
 }
 
 enum : int32_t { XF_COPY = 0, XF_SOFT1 = 1, XF_SOFT2 = 2, XF_HARD = 3 };

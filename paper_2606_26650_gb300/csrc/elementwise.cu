@@ -372,6 +372,31 @@ __global__ void __launch_bounds__(kThreads) hard_pack_warp_kernel(LayerDev L, in
   }
 }
 
+// ---------------------------------------------------------------- fused-GEMM operand constants
+// operand_const_vec of every group for one schedule point, stored [K/g][N] so that a fused
+// GEMM producer warp (consecutive W rows, one group column) reads contiguous 16-byte
+// vectors.  A 32 x 32 (row x group column) tile goes through shared memory so both the
+// row-major [N][K/g] group arrays and the output are accessed coalesced.
+constexpr int kConstTile = 32;
+
+__global__ void __launch_bounds__(kConstTile * kConstTile) operand_consts_kernel(LayerDev L, StepScalars sc) {
+  __shared__ float4 tile[kConstTile][kConstTile + 1];
+  const int64_t gpr = L.groups_per_row;
+  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kConstTile;
+  for (int64_t n0 = static_cast<int64_t>(blockIdx.y) * kConstTile; n0 < L.N;
+       n0 += static_cast<int64_t>(gridDim.y) * kConstTile) {
+    {
+      const int64_t n = n0 + threadIdx.y, c = c0 + threadIdx.x;
+      if (n < L.N && c < gpr)
+        tile[threadIdx.y][threadIdx.x] = operand_const_vec(group_const(L, n * gpr + c), sc.s, sc.inv_2tanh_s, sc.phase);
+    }
+    __syncthreads();
+    const int64_t n = n0 + threadIdx.x, c = c0 + threadIdx.y;
+    if (n < L.N && c < gpr) L.op_const[c * L.N + n] = tile[threadIdx.x][threadIdx.y];
+    __syncthreads();
+  }
+}
+
 // ---------------------------------------------------------------- Eq. 7 loss and dY
 constexpr int kLossMaxBlocks = 1216;
 
@@ -592,6 +617,14 @@ cudaError_t launch_hard_pack(const LayerDev& L, int32_t w_dtype, uint8_t* codes,
     else
       hard_pack_kernel<float, 4><<<grid, kThreads, 0, st>>>(L, codes, alpha);
   }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_operand_consts(const LayerDev& L, StepScalars sc, cudaStream_t st) {
+  const int64_t row_tiles = (L.N + kConstTile - 1) / kConstTile;
+  const dim3 grid(static_cast<unsigned>((L.groups_per_row + kConstTile - 1) / kConstTile),
+                  static_cast<unsigned>(row_tiles < 65535 ? row_tiles : 65535));
+  operand_consts_kernel<<<grid, dim3(kConstTile, kConstTile), 0, st>>>(L, sc);
   return cudaGetLastError();
 }
 

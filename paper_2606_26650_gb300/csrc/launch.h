@@ -44,6 +44,9 @@ struct TcPlan {
   int32_t dw_P;       // partial-sum chunk width (columns)
 };
 TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count);
+// Writes L.op_const (operand_const_vec of every group, [K/g][N]) for schedule point sc.
+cudaError_t launch_operand_consts(const LayerDev& L, StepScalars sc, cudaStream_t st);
+
 cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st);
 cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int64_t M, void* dX, cudaStream_t st);
 cudaError_t launch_tc_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M,

@@ -191,13 +191,14 @@ __device__ __forceinline__ void store_rows_bf16x32(uint16_t* C, int64_t M, int64
 
 // Walks the pipeline stages one producer thread handles (every kProdGroups-th stage of its
 // CTA's tile sequence) and tracks which W row, K chunk and group its 128-byte operand row
-// holds.  Divisions happen once per tile; each stage step is a few integer adds.
+// holds, the group as its index into the [K/g][N] operand-constant array.  Divisions happen
+// once per tile; each stage step is a few integer adds.
 template <int CG, bool B_MN>
 struct OperandRowIter {
   using Cfg = FusedCfg<CG>;
   int t, kb;      // tile index, k block
   int64_t n, kc;  // W row, first K column of the 64-element chunk
-  int64_t j;      // group index of (n, kc)
+  int64_t ci;     // operand-constant index of (n, kc): (kc / g) * N + n
   int kin;        // forward: k blocks into the current group (kc / 64 mod g / 64)
   bool tile_ok;   // forward: n < N; dX: kc < K
 
@@ -211,13 +212,13 @@ struct OperandRowIter {
       n = (int64_t)n_blk * BN + cta * Cfg::kBRows + row;
       kc = (int64_t)kb * BK;
       tile_ok = n < a.L.N;
-      j = n * a.L.groups_per_row + kb / gk;
+      ci = (int64_t)(kb / gk) * a.L.N + n;
       kin = kb % gk;
     } else {
       n = (int64_t)kb * BK + (row & 63);
       kc = (int64_t)n_blk * BN + cta * Cfg::kBRows + 64 * (row >> 6);
       tile_ok = kc < a.L.K;
-      j = n * a.L.groups_per_row + kc / a.L.g;
+      ci = (kc / a.L.g) * a.L.N + n;
       kin = 0;
     }
   }
@@ -245,11 +246,11 @@ struct OperandRowIter {
       const int gk = a.L.g / BK;
       while (kin >= gk) {
         kin -= gk;
-        ++j;
+        ci += a.L.N;
       }
     } else {
       n += (int64_t)steps * BK;
-      j += (int64_t)steps * BK * a.L.groups_per_row;
+      ci += (int64_t)steps * BK;
     }
   }
 };
@@ -499,19 +500,20 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS, DEEP_W>::kThreads, 1)
     const bool transform = phase_t != PHASE_TEACHER;
     const uint32_t q0 = (PAIRS == 2 ? pair : 0u) + PAIRS * grp;
     // `cur` is the stage being produced; `ahead` runs two of this thread's stages ahead and
-    // requests that stage's group inputs, so an L2 round trip is hidden behind two stages.
+    // requests that stage's operand constants (one 16-byte vector, precomputed per call), so
+    // an L2 round trip is hidden behind two stages.
     OperandRowIter<CG, B_MN> cur, ahead;
     cur.init(args, cta, row, cluster, 0);
     cur.step(args, cta, row, nclusters, q0);
     ahead = cur;
-    GroupRaw raw0{}, raw1{};
+    float4 raw0{}, raw1{};
     int64_t j0 = -1, j1 = -1;
-    auto request = [&](const OperandRowIter<CG, B_MN>& it, GroupRaw& dst, int64_t& jd, const GroupRaw& other,
+    auto request = [&](const OperandRowIter<CG, B_MN>& it, float4& dst, int64_t& jd, const float4& other,
                        int64_t jo) {
       if (transform && it.live(args, num_tiles) && it.valid(args)) {
-        if (jo == it.j) dst = other;
-        else dst = group_raw(L, it.j);
-        jd = it.j;
+        if (jo == it.ci) dst = other;
+        else dst = __ldg(L.op_const + it.ci);
+        jd = it.ci;
       }
     };
     request(ahead, raw0, j0, raw1, j1);
@@ -523,12 +525,12 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS, DEEP_W>::kThreads, 1)
     uint32_t q = q0;
     bool ok = true;
     // One stage: consume `mine` (requested two stages ago), then refill it two stages ahead.
-    auto produce = [&](GroupRaw& mine, int64_t& jm, const GroupRaw& other, int64_t jo) {
+    auto produce = [&](float4& mine, int64_t& jm, const float4& other, int64_t jo) {
       const uint32_t s = q % SW;
       const bool live = transform && cur.valid(args);
-      if (live && cur.j != j_have) {
-        pc = producer_const(group_const(mine), args.sc.s, args.sc.inv_2tanh_s, phase_t);
-        j_have = cur.j;
+      if (live && cur.ci != j_have) {
+        pc = producer_const_from(mine);
+        j_have = cur.ci;
       }
       if (!mbar_wait(raw_w(grp * SW + s), (q / Cfg::kRawPeriod) & 1u, wc)) {
         ok = false;
@@ -987,6 +989,10 @@ constexpr float kDeepRingMaxS = 12.0f;
 bool deep_operand_ring(const StepScalars& sc) { return sc.phase == PHASE_SOFT && sc.s < kDeepRingMaxS; }
 
 cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st) {
+  if (sc.phase != PHASE_TEACHER) {
+    const cudaError_t e = launch_operand_consts(L, sc, st);
+    if (e != cudaSuccess) return e;
+  }
   switch (fused_variant_for(M)) {
     case 4:
       if (deep_operand_ring(sc)) return run_fused<2, false, 2, true>(L, sc, X, M, L.K, Y, L.N, st);
@@ -997,6 +1003,10 @@ cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int6
 }
 
 cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int64_t M, void* dX, cudaStream_t st) {
+  if (sc.phase != PHASE_TEACHER) {
+    const cudaError_t e = launch_operand_consts(L, sc, st);
+    if (e != cudaSuccess) return e;
+  }
   switch (fused_variant_for(M)) {
     case 4:
       if (deep_operand_ring(sc)) return run_fused<2, true, 2, true>(L, sc, dY, M, L.N, dX, L.K, st);

@@ -24,16 +24,16 @@ def test_exports_every_declared_symbol(lib):
 
 
 def test_status_strings_and_version(lib):
-    assert lib.catq_abi_version() == 1
+    assert lib.catq_abi_version() == 2
     for code, name in C.STATUS.items():
         assert lib.catq_status_string(code).decode() == name
     assert lib.catq_status_string(99).decode() == "CATQ_ERR_UNKNOWN"
 
 
-def _layer(N=64, K=256, g=128, dtype=C.BF16, W=16, stats=32):
+def _layer(N=64, K=256, g=128, dtype=C.BF16, W=16, stats=32, op_const=65536):
     """A layer struct with fake (never dereferenced) device addresses."""
     return C.catq_layer(N, K, g, dtype, W, stats, stats + 1024, stats + 2048, stats + 4096, stats + 8192,
-                        stats + 16384)
+                        stats + 16384, op_const)
 
 
 def _stats(lib, layer, thr=0):
@@ -65,6 +65,11 @@ def test_call_validation(lib):
     assert fwd(ctypes.byref(L), soft, 16, 0, C.BF16, 16, None) == 0                  # M == 0: no-op
     assert fwd(ctypes.byref(L), soft, 0, 4, C.BF16, 16, None) == 1                   # null X
     assert fwd(ctypes.byref(L), soft, 24, 4, C.BF16, 16, None) == 4                  # misaligned X
+    # a bf16 SOFT/HARD forward or dX needs the operand-constant array, 16-byte aligned
+    assert fwd(ctypes.byref(_layer(op_const=0)), soft, 16, 4, C.BF16, 16, None) == 1
+    assert fwd(ctypes.byref(_layer(op_const=65544)), soft, 16, 4, C.BF16, 16, None) == 4
+    assert lib.catq_soft_ternary_linear_bwd(ctypes.byref(_layer(op_const=0)), soft, 16, 16, 4, C.BF16, 16,
+                                            None, None, None, None, 0, None) == 1
     bwd = lib.catq_soft_ternary_linear_bwd
     assert bwd(ctypes.byref(L), soft, 16, 16, 4, C.BF16, None, 0, 32, 32, 256, 1 << 30, None) == 1
     F = _layer(dtype=C.F32)
