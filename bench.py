@@ -44,7 +44,7 @@ TRAFFIC = {"sha": "a8406f414078935b", "workload": "c3_llama3_8b_block",
            "fwd": 432493275, "dx": 459425206, "dw": 906473179}
 
 
-def parse():
+def parse(argv=None):
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=60)
@@ -54,7 +54,7 @@ def parse():
     p.add_argument("--s", type=float, default=30.0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
-    return p.parse_args()
+    return p.parse_args(argv)
 
 
 def dist_env():
@@ -107,6 +107,23 @@ def oracle_sample(wl, s, rows=CPU_SAMPLE_ROWS, linears=CPU_SAMPLE_LINEARS):
         total_t += time.perf_counter() - t0
         flops += 6.0 * rows * lin.N * lin.K
     return total_t, flops
+
+
+def max_over_ranks(ms: float, world: int, device) -> float:
+    """The slowest rank's step time, on every rank (the timing rule: max over ranks)."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(flops_per_rank_step: float, ms: float, world: int) -> float:
+    """Whole-job TFLOP/s: every rank runs the same step on its own inputs (weak scaling), so
+    the job does `world` times one rank's work in the slowest rank's time."""
+    return world * flops_per_rank_step / (ms * 1e-3) / 1e12
 
 
 def cpu_cores():
@@ -308,14 +325,9 @@ def run_ours(args):
     status = C.catq_device_status()
     if status != 0:
         raise SystemExit(f"device status {C.STATUS.get(status, status)} in the timed region")
-    ms = t_start.elapsed_time(t_end) / args.steps
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(t_start.elapsed_time(t_end) / args.steps, world, dev)
     flops_step = wl.flops_per_step
-    value = world * flops_step / (ms * 1e-3) / 1e12
+    value = job_throughput(flops_step, ms, world)
 
     # per-kernel live timing (CUDA events on the launching stream)
     per = {k: 0.0 for k in kinds}
@@ -408,13 +420,8 @@ def measure_e2e(args, C, torch, st, step, barrier, flops_step, world, dev):
         e2e_step()
     b.record()
     barrier()
-    ms = a.elapsed_time(b) / steps
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    return {"value": world * flops_step / (ms * 1e-3) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
+    ms = max_over_ranks(a.elapsed_time(b) / steps, world, dev)
+    return {"value": job_throughput(flops_step, ms, world), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": steps}
 
 
