@@ -52,11 +52,8 @@ constexpr int gcd_c(int a, int b) { return b == 0 ? a : gcd_c(b, a % b); }
 // against the same produced operand tiles; each pair produces every other stage and sends
 // its transformed half-tiles to the other pair's CTAs through distributed shared memory,
 // which halves the per-SM transform work.
-// DEEP_W (two pairs only) trades an A stage for two operand slots: the operand ring's round
-// trip grows with the transform's cost (the two-tanh form doubles it), the A ring's does not.
-template <int CG, int PAIRS = 1, bool DEEP_W = false>
+template <int CG, int PAIRS = 1>
 struct FusedCfg {
-  static_assert(!DEEP_W || PAIRS == 2, "the deep operand ring is a four-CTA layout");
   static_assert(PAIRS == 1 || CG == 2, "pairs of pairs need CTA pairs");
   static constexpr int kClusterCtas = CG * PAIRS;
   static constexpr int kRowsPerAcc = 128 * CG;          // MMA M
@@ -64,10 +61,10 @@ struct FusedCfg {
   static constexpr int kBRows = BN / CG;                // 128-byte operand rows per CTA per stage
   static constexpr int kABytes = NACC * 128 * BK * 2;   // this CTA's A rows per stage
   static constexpr int kWBytes = kBRows * BK * 2;       // this CTA's operand rows per stage
-  static constexpr int kStagesA = (CG == 1 || DEEP_W) ? 3 : 4;  // A ring: TMA -> MMA
+  static constexpr int kStagesA = CG == 1 ? 3 : 4;      // A ring: TMA -> MMA
   // W ring: TMA -> producers (in place) -> MMA.  Even with two pairs, so every slot is always
   // produced by the same pair (and received by the other).
-  static constexpr int kStagesW = PAIRS == 2 ? (DEEP_W ? 8 : 6) : (CG == 1 ? 3 : 5);
+  static constexpr int kStagesW = PAIRS == 2 ? 6 : (CG == 1 ? 3 : 5);
   static constexpr int kEpiWarps = 4;
   // Two groups of 8 producer warps take alternate stages (of the ones this CTA produces), so
   // each group has two stage periods per operand tile and the groups' MUFU work interleaves.
@@ -255,11 +252,11 @@ struct OperandRowIter {
   }
 };
 
-template <int CG, bool B_MN, int PAIRS, bool DEEP_W>
-__global__ void __launch_bounds__(FusedCfg<CG, PAIRS, DEEP_W>::kThreads, 1)
+template <int CG, bool B_MN, int PAIRS>
+__global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     fused_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
                       const FusedArgs args) {
-  using Cfg = FusedCfg<CG, PAIRS, DEEP_W>;
+  using Cfg = FusedCfg<CG, PAIRS>;
   constexpr int SA = Cfg::kStagesA, SW = Cfg::kStagesW;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = smem_u32(smem_raw);
@@ -898,10 +895,10 @@ int max_active_clusters(Kern kern, int cluster_ctas, int threads, int smem, int 
 // CTA pairs (512 rows) from 512 rows, single CTAs below.
 int fused_variant_for(int64_t M) { return M >= 1024 ? 4 : (M >= 512 ? 2 : 1); }
 
-template <int CG, bool B_MN, int PAIRS, bool DEEP_W = false>
+template <int CG, bool B_MN, int PAIRS>
 cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t M, int64_t depth, void* C,
                       int64_t ncols, cudaStream_t st) {
-  using Cfg = FusedCfg<CG, PAIRS, DEEP_W>;
+  using Cfg = FusedCfg<CG, PAIRS>;
   DeviceInfo& d = device_info();
   if (!d.ok) return cudaErrorInvalidDevice;
   CUtensorMap ta, tw;
@@ -922,7 +919,7 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
   args.num_k_blocks = static_cast<int32_t>((depth + BK - 1) / BK);
   args.group_m = std::min(4, args.num_m_tiles);
   args.wc = make_wait_ctl(d);
-  auto kern = fused_gemm_kernel<CG, B_MN, PAIRS, DEEP_W>;
+  auto kern = fused_gemm_kernel<CG, B_MN, PAIRS>;
   const int tiles = args.num_m_tiles * args.num_n_tiles;
   const int fit = max_active_clusters(kern, Cfg::kClusterCtas, Cfg::kThreads, Cfg::kSmemBytes,
                                       d.sm_count / Cfg::kClusterCtas);
@@ -973,6 +970,9 @@ TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count) {
   const int64_t tiles = ((L.N + rows - 1) / rows) * ((L.K + BN - 1) / BN);
   const int64_t clusters = std::max(1, sm_count / p.dw_cg);
   const int64_t kb_total = std::max<int64_t>(1, (M + BK - 1) / BK);
+  // Split the contraction (M) only when the tiles leave clusters idle: every split re-runs
+  // the per-element factor-gradient epilogue on its tile, which costs about as much as the
+  // tile's MMA work, so splitting a full wave buys nothing.
   int64_t splits = 1;
   if (tiles < clusters) splits = std::min<int64_t>(clusters / tiles, std::max<int64_t>(1, kb_total / 8));
   const int64_t per = (kb_total + splits - 1) / splits;
@@ -982,21 +982,13 @@ TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count) {
   return p;
 }
 
-// SOFT steps with s below this mostly take the two-tanh form of Eq. 5 (s Delta < 6 for the
-// usual Delta near 0.5), whose longer transform wants the deep operand ring.
-constexpr float kDeepRingMaxS = 12.0f;
-
-bool deep_operand_ring(const StepScalars& sc) { return sc.phase == PHASE_SOFT && sc.s < kDeepRingMaxS; }
-
 cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st) {
   if (sc.phase != PHASE_TEACHER) {
     const cudaError_t e = launch_operand_consts(L, sc, st);
     if (e != cudaSuccess) return e;
   }
   switch (fused_variant_for(M)) {
-    case 4:
-      if (deep_operand_ring(sc)) return run_fused<2, false, 2, true>(L, sc, X, M, L.K, Y, L.N, st);
-      return run_fused<2, false, 2>(L, sc, X, M, L.K, Y, L.N, st);
+    case 4: return run_fused<2, false, 2>(L, sc, X, M, L.K, Y, L.N, st);
     case 2: return run_fused<2, false, 1>(L, sc, X, M, L.K, Y, L.N, st);
     default: return run_fused<1, false, 1>(L, sc, X, M, L.K, Y, L.N, st);
   }
@@ -1008,9 +1000,7 @@ cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int6
     if (e != cudaSuccess) return e;
   }
   switch (fused_variant_for(M)) {
-    case 4:
-      if (deep_operand_ring(sc)) return run_fused<2, true, 2, true>(L, sc, dY, M, L.N, dX, L.K, st);
-      return run_fused<2, true, 2>(L, sc, dY, M, L.N, dX, L.K, st);
+    case 4: return run_fused<2, true, 2>(L, sc, dY, M, L.N, dX, L.K, st);
     case 2: return run_fused<2, true, 1>(L, sc, dY, M, L.N, dX, L.K, st);
     default: return run_fused<1, true, 1>(L, sc, dY, M, L.N, dX, L.K, st);
   }
