@@ -216,9 +216,12 @@ __device__ __forceinline__ float ternary_weight_f32(float w, const GroupConst& c
 
 // tanh(y) and 1 - tanh(y)^2 with good relative accuracy in the tails:
 // e = exp(-2|y|), tanh|y| = (1 - e)/(1 + e), sech^2 y = 4 e / (1 + e)^2.
+// FAST uses the hardware exp2 and reciprocal (__expf, __fdividef; relative error near
+// 1e-6, also in the tails) for the bf16 path; otherwise the correctly rounded library calls.
+template <bool FAST = false>
 __device__ __forceinline__ void tanh_sech2(float y, float& t, float& s2) {
-  const float e = expf(-2.0f * fabsf(y));
-  const float rcp = 1.0f / (1.0f + e);
+  const float e = FAST ? __expf(-2.0f * fabsf(y)) : expf(-2.0f * fabsf(y));
+  const float rcp = FAST ? __fdividef(1.0f, 1.0f + e) : 1.0f / (1.0f + e);
   t = copysignf((1.0f - e) * rcp, y);
   s2 = 4.0f * e * rcp * rcp;
 }
@@ -230,12 +233,13 @@ struct GradSums {
   float smu, salpha, sdelta;
 };
 
+template <bool FAST = false>
 __device__ __forceinline__ void grad_element(float G, float w, const GroupConst& c, float s, float inv_2tanh_s,
                                              int32_t phase, GradSums& acc) {
   const float x = what(w, c);
   float ta, sa, tb, sb;
-  tanh_sech2(s * (x - c.delta), ta, sa);
-  tanh_sech2(s * (x + c.delta), tb, sb);
+  tanh_sech2<FAST>(s * (x - c.delta), ta, sa);
+  tanh_sech2<FAST>(s * (x + c.delta), tb, sb);
   const float k = s * inv_2tanh_s;
   const float fp_over_k = sa + sb;
   const float T = (phase == PHASE_SOFT) ? inv_2tanh_s * (ta + tb) : hard_q(x, c.delta);

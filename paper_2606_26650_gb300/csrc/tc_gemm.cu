@@ -721,31 +721,43 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
       int64_t cur_j = -1;
       GroupConst gc{};
       GradSums acc{0.f, 0.f, 0.f};
+      // The 32 W values of a chunk are loaded one chunk ahead of the arithmetic.
+      constexpr int kChunks = (BN / 2) / 32;
+      const int64_t k0 = (int64_t)k_blk * BN + half * (BN / 2);
+      auto load_w = [&](int c, uint4 (&dst)[4]) {
+        const int64_t k = k0 + c * 32;
+        if (row_ok && k < L.K) {
+          const uint4* wp = reinterpret_cast<const uint4*>(W + n * L.K + k);
+#pragma unroll
+          for (int v = 0; v < 4; ++v) dst[v] = __ldg(wp + v);
+        }
+      };
+      uint4 wcur[4], wnext[4];
+      load_w(0, wcur);
 #pragma unroll 1
-      for (int c = 0; c < (BN / 2) / 32; ++c) {
+      for (int c = 0; c < kChunks; ++c) {
         const int col = half * (BN / 2) + c * 32;
         uint32_t rg[32];
         tmem_ld32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + buf * BN + col, rg);
+        if (c + 1 < kChunks) load_w(c + 1, wnext);
         tmem_ld_wait();
-        const int64_t k = (int64_t)k_blk * BN + col;
+        const int64_t k = k0 + c * 32;
         if (row_ok && k < L.K) {
           const int64_t j = n * L.groups_per_row + k / L.g;
           if (j != cur_j) {
             gc = group_const(L, j);
             cur_j = j;
           }
-          const uint4* wp = reinterpret_cast<const uint4*>(W + n * L.K + k);
           if (gc.alpha != 0.0f) {
 #pragma unroll
             for (int v = 0; v < 4; ++v) {
-              const uint4 wv = __ldg(wp + v);
-              const uint32_t w4[4] = {wv.x, wv.y, wv.z, wv.w};
+              const uint32_t w4[4] = {wcur[v].x, wcur[v].y, wcur[v].z, wcur[v].w};
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
-                grad_element(__uint_as_float(rg[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), gc, args.sc.s,
-                             args.sc.inv_2tanh_s, args.sc.phase, acc);
-                grad_element(__uint_as_float(rg[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), gc, args.sc.s,
-                             args.sc.inv_2tanh_s, args.sc.phase, acc);
+                grad_element<true>(__uint_as_float(rg[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), gc, args.sc.s,
+                                   args.sc.inv_2tanh_s, args.sc.phase, acc);
+                grad_element<true>(__uint_as_float(rg[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), gc, args.sc.s,
+                                   args.sc.inv_2tanh_s, args.sc.phase, acc);
               }
             }
           }
@@ -757,6 +769,8 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
             acc = GradSums{0.f, 0.f, 0.f};
           }
         }
+#pragma unroll
+        for (int v = 0; v < 4; ++v) wcur[v] = wnext[v];
       }
       tc_fence_before();
       __syncwarp();
