@@ -54,6 +54,8 @@ def parse(argv=None):
     p.add_argument("--s", type=float, default=30.0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--streams", type=int, default=2,
+                   help="CUDA streams the block's linears are spread over (independent problems)")
     return p.parse_args(argv)
 
 
@@ -167,7 +169,7 @@ def run_reference(args):
 def workload_config(wl, args):
     return {"workload": wl.name, "tokens": wl.M, "group_size": wl.g, "phase": "soft", "s": args.s,
             "linears": {lin.name: [lin.K, lin.N] for lin in wl.linears},
-            "flops_per_step": wl.flops_per_step,
+            "flops_per_step": wl.flops_per_step, "streams": getattr(args, "streams", 1),
             "l2": "inputs larger than L2 (per-step working set of weights and activations > 129 MB)"}
 
 
@@ -269,34 +271,57 @@ def run_ours(args):
         ws_bwd = max(ws_bwd, C.catq_bwd_workspace_bytes(layer, M))
         ws_loss = max(ws_loss, C.catq_recon_loss_workspace_bytes(M * lin.N))
         st.append(d)
-    wsb = C.workspace(ws_bwd, dev)
-    wsl = C.workspace(ws_loss, dev)
+    # The block's linears are independent calibration problems (one loss per linear output,
+    # Eq. 7), so they are spread over `streams` CUDA streams: one linear's kernels can start
+    # on the SMs another linear's last tile wave leaves idle.  Each stream has its own
+    # workspaces; a step forks from and joins back into the current stream.
+    nstreams = max(1, args.streams)
+    main = torch.cuda.current_stream()
+    lanes = [main] if nstreams == 1 else [torch.cuda.Stream(device=dev) for _ in range(nstreams)]
+    wsbs = [C.workspace(ws_bwd, dev) for _ in lanes]
+    wsls = [C.workspace(ws_loss, dev) for _ in lanes]
     torch.cuda.synchronize()
 
     kinds = ("fwd", "dx", "dw")
 
-    def step(ev=None):
+    def step(ev=None, serial=False):
+        """One step; `serial` runs every linear on the current stream (kernel timing)."""
+        use = [main] if serial else lanes
+        if len(use) > 1:
+            fork = torch.cuda.Event()
+            fork.record(main)
+            for s in use:
+                s.wait_event(fork)
         for i, d in enumerate(st):
-            L = d["layer"]
-            C.catq_group_stats(L, wl.thr_init)
-            if ev is not None:
-                ev[i]["fwd"][0].record()
-            C.catq_soft_ternary_linear_fwd(L, sched, d["X"], d["Y"])
-            if ev is not None:
-                ev[i]["fwd"][1].record()
-            C.catq_recon_loss(d["Y"], d["Yt"], d["loss"], d["dY"], wsl)
-            if ev is not None:
-                ev[i]["dx"][0].record()
-            C.catq_soft_ternary_linear_bwd(L, sched, d["X"], d["dY"], dX=d["dX"])
-            if ev is not None:
-                ev[i]["dx"][1].record()
-                ev[i]["dw"][0].record()
-            C.catq_soft_ternary_linear_bwd(L, sched, d["X"], d["dY"], None, *d["grads"], workspace=wsb)
-            if ev is not None:
-                ev[i]["dw"][1].record()
-            C.catq_hard_ternarize_pack(L, d["codes"], d["alpha"])
+            k = i % len(use)
+            with torch.cuda.stream(use[k]):
+                L = d["layer"]
+                C.catq_group_stats(L, wl.thr_init)
+                if ev is not None:
+                    ev[i]["fwd"][0].record()
+                C.catq_soft_ternary_linear_fwd(L, sched, d["X"], d["Y"])
+                if ev is not None:
+                    ev[i]["fwd"][1].record()
+                C.catq_recon_loss(d["Y"], d["Yt"], d["loss"], d["dY"], wsls[k])
+                if ev is not None:
+                    ev[i]["dx"][0].record()
+                C.catq_soft_ternary_linear_bwd(L, sched, d["X"], d["dY"], dX=d["dX"])
+                if ev is not None:
+                    ev[i]["dx"][1].record()
+                    ev[i]["dw"][0].record()
+                C.catq_soft_ternary_linear_bwd(L, sched, d["X"], d["dY"], None, *d["grads"], workspace=wsbs[k])
+                if ev is not None:
+                    ev[i]["dw"][1].record()
+                C.catq_hard_ternarize_pack(L, d["codes"], d["alpha"])
+        if len(use) > 1:
+            for s in use:
+                join = torch.cuda.Event()
+                join.record(s)
+                main.wait_event(join)
 
-    launches_per_step = len(st) * (1 + 1 + 2 + 1 + 2 + 1)
+    # per linear: stats; operand constants + forward; loss (partial + final); operand
+    # constants + dX; dW + gradient reduce; pack
+    launches_per_step = len(st) * (1 + 2 + 2 + 2 + 2 + 1)
 
     def barrier():
         torch.cuda.synchronize()
@@ -315,11 +340,14 @@ def run_ours(args):
     E = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
     evs = [[{k: (E(), E()) for k in kinds} for _ in st] for _ in range(args.steps)]
     t_start, t_end = E(), E()
+    # With one stream the step's own timed region also times each kernel.  With several,
+    # kernels of different linears share the GPU, so a second timed region of the same K
+    # steps on one stream times each kernel on its own for the roofline.
     with ClockSampler(local) as clk:
         barrier()
         t_start.record()
         for k in range(args.steps):
-            step(evs[k])
+            step(evs[k] if nstreams == 1 else None)
         t_end.record()
         barrier()
     status = C.catq_device_status()
@@ -328,6 +356,13 @@ def run_ours(args):
     ms = max_over_ranks(t_start.elapsed_time(t_end) / args.steps, world, dev)
     flops_step = wl.flops_per_step
     value = job_throughput(flops_step, ms, world)
+    if nstreams > 1:
+        barrier()
+        for k in range(args.steps):
+            step(evs[k], serial=True)
+        barrier()
+        if C.catq_device_status() != 0:
+            raise SystemExit("device status set in the kernel-timing region")
 
     # per-kernel live timing (CUDA events on the launching stream)
     per = {k: 0.0 for k in kinds}
@@ -355,6 +390,9 @@ def run_ours(args):
                 "peak_kind": f"bf16 dense sustained ({peaks['source']})",
                 "frac_of_burst": achieved / peaks["bf16"],
                 "per_kernel_ms_per_step": {k: per[k] / args.steps for k in kinds},
+                "kernel_timing": ("the step's timed region (one stream)" if nstreams == 1 else
+                                  f"one stream, {args.steps} steps right after the step's timed region "
+                                  f"(the step itself spreads the linears over {nstreams} streams)"),
                 "per_kernel_tflops": {k: flops_kind / (per[k] * 1e-3) / 1e12 for k in kinds}}
 
     e2e = None
