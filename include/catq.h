@@ -248,6 +248,13 @@ catq_status catq_grouped_soft_ternary_linear_bwd(const catq_grouped_layer* layer
                                                  float* g_ddelta, void* workspace, size_t ws_bytes,
                                                  catq_stream stream);
 
+/* Self-test of the device-side failure detection (no counterpart in the paper): launches
+ * one thread that waits, through the library's bounded mbarrier wait, on a barrier nothing
+ * arrives on.  After timeout_ns (1 us .. 1 s) the wait gives up, latches CATQ_ERR_TIMEOUT
+ * in the status word and the kernel returns; nothing faults and the context stays usable.
+ * Read the result with catq_device_status.  Out-of-range timeouts: CATQ_ERR_INVALID_ARG. */
+catq_status catq_selftest_wait_timeout(uint64_t timeout_ns, catq_stream stream);
+
 /* Synchronises `stream`, then returns in *out the status latched on the current device
  * since the last call (CATQ_OK if none) and clears it.  The return value reports whether
  * the query itself succeeded. */

@@ -83,6 +83,7 @@ def lib() -> ctypes.CDLL:
         "catq_recon_loss": (I32, [P, P, I64, I32, I32, P, P, P, S, P]),
         "catq_hard_ternarize_pack": (I32, [LP, P, P, P]),
         "catq_device_status": (I32, [P, ctypes.POINTER(I32)]),
+        "catq_selftest_wait_timeout": (I32, [ctypes.c_uint64, P]),
         "catq_soft_ternary_linear_bwd_noalloc": (I32, [LP, catq_schedule, P, P, I64, I32, P, P, P, P, P]),
         "catq_bwd_noalloc_max_scratch_bytes": (S, []),
         "catq_grouped_soft_ternary_linear_fwd": (I32, [ctypes.POINTER(catq_grouped_layer), catq_schedule, P, P, I32, P,
@@ -251,6 +252,10 @@ def catq_device_status(stream=None) -> int:
     out = ctypes.c_int32(0)
     _check(lib().catq_device_status(_stream(stream), ctypes.byref(out)), "catq_device_status")
     return int(out.value)
+
+
+def catq_selftest_wait_timeout(timeout_ns: int, stream=None):
+    _check(lib().catq_selftest_wait_timeout(int(timeout_ns), _stream(stream)), "catq_selftest_wait_timeout")
 
 
 def workspace(nbytes: int, device):

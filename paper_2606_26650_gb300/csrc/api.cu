@@ -383,6 +383,11 @@ catq_status catq_grouped_soft_ternary_linear_bwd(const catq_grouped_layer* G, ca
   return CATQ_OK;
 }
 
+catq_status catq_selftest_wait_timeout(uint64_t timeout_ns, catq_stream stream) {
+  if (timeout_ns < 1000 || timeout_ns > 1000000000ull) return CATQ_ERR_INVALID_ARG;
+  return cuda_status(launch_wait_probe(timeout_ns, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 catq_status catq_device_status(catq_stream stream, int32_t* out) {
   if (!out) return CATQ_ERR_INVALID_ARG;
   if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return CATQ_ERR_CUDA;

@@ -44,6 +44,9 @@ struct TcPlan {
   int32_t dw_P;       // partial-sum chunk width (columns)
 };
 TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count);
+// One-thread kernel whose bounded wait runs out after timeout_ns (self-test).
+cudaError_t launch_wait_probe(uint64_t timeout_ns, cudaStream_t st);
+
 // Writes L.op_const (operand_const_vec of every group, [K/g][N]) for schedule point sc.
 cudaError_t launch_operand_consts(const LayerDev& L, StepScalars sc, cudaStream_t st);
 

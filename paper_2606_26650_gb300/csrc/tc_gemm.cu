@@ -581,6 +581,19 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
   }
 }
 
+// ============================================================================ wait probe
+
+// Self-test of the bounded waits: one thread waits on a shared-memory barrier nothing
+// arrives on, with the caller's limit, through the same mbar_wait the GEMMs use.  When the
+// limit passes the wait latches CATQ_ERR_TIMEOUT and returns; nothing faults or hangs.
+__global__ void wait_probe_kernel(const WaitCtl wc) {
+  __shared__ __align__(8) uint64_t bar;
+  const uint32_t b = smem_u32(&bar);
+  mbar_init(b, 1);
+  fence_mbar_init_cluster();
+  mbar_wait(b, 0, wc);
+}
+
 // ============================================================================ dW kernel
 
 template <int CG>
@@ -1018,6 +1031,15 @@ cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int6
     case 2: return run_fused<2, true, 1>(L, sc, dY, M, L.N, dX, L.K, st);
     default: return run_fused<1, true, 1>(L, sc, dY, M, L.N, dX, L.K, st);
   }
+}
+
+cudaError_t launch_wait_probe(uint64_t timeout_ns, cudaStream_t st) {
+  DeviceInfo& d = device_info();
+  if (!d.ok) return cudaErrorInvalidDevice;
+  WaitCtl w = make_wait_ctl(d);
+  w.timeout_ns = timeout_ns;
+  wait_probe_kernel<<<1, 1, 0, st>>>(w);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_tc_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M,

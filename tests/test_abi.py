@@ -89,3 +89,5 @@ def test_call_validation(lib):
     pack = lib.catq_hard_ternarize_pack
     assert pack(ctypes.byref(L), None, None, None) == 1
     assert lib.catq_device_status(None, None) == 1
+    assert lib.catq_selftest_wait_timeout(10, None) == 1              # below 1 us
+    assert lib.catq_selftest_wait_timeout(2_000_000_000, None) == 1   # above 1 s
