@@ -54,6 +54,7 @@ def parse(argv=None):
     p.add_argument("--s", type=float, default=30.0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-also", action="store_true", help="skip the secondary workloads and phase")
     p.add_argument("--streams", type=int, default=2,
                    help="CUDA streams the block's linears are spread over (independent problems)")
     return p.parse_args(argv)
@@ -227,6 +228,118 @@ class ClockSampler:
 
 # ------------------------------------------------------------------ GPU arm
 
+KINDS = ("fwd", "dx", "dw")
+# Block workloads also timed (secondary lines of the JSON output): the Qwen3-14B-shaped block
+# the 60%-of-peak target also names, and the Qwen3-1.7B-shaped one.
+ALSO_WORKLOADS = ("c4_qwen3_14b_block", "c2_qwen3_1p7b_block")
+
+
+class BlockRun:
+    """Device state and one calibration step of a block workload: every linear's seeded
+    inputs, layer and teacher output, and per-stream workspaces.
+
+    The block's linears are independent calibration problems (one loss per linear output,
+    Eq. 7), so a step spreads them over `nstreams` CUDA streams: one linear's kernels can
+    start on the SMs another linear's last tile wave leaves idle.  A step forks from and
+    joins back into the current stream."""
+
+    def __init__(self, C, torch, wl, dev, rank, nstreams):
+        self.C, self.torch, self.wl = C, torch, wl
+        M = self.M = wl.M
+        bf = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+
+        def upload(a):
+            if wl.dtype == "bf16":
+                return torch.from_numpy(syn.bf16_bits(a).view(np.int16)).to(dev).view(torch.bfloat16)
+            return torch.from_numpy(a).to(dev)
+
+        Xs = {}
+        for lin in wl.linears:
+            if (lin.x, lin.K) not in Xs:
+                Xs[(lin.x, lin.K)] = upload(syn.activations(wl, lin.x, M, lin.K, seed=rank))
+        self.st = []
+        ws_bwd = ws_loss = 0
+        for lin in wl.linears:
+            G = lin.N * lin.K // wl.g
+            fac = [torch.from_numpy(f).to(dev) for f in syn.factors(G, rank, f"bench/{lin.name}", perturbed=True)]
+            layer = C.Layer.create(upload(syn.weight(wl, lin, seed=rank)), wl.g, *fac)
+            C.catq_group_stats(layer, wl.thr_init)
+            d = dict(lin=lin, layer=layer, X=Xs[(lin.x, lin.K)],
+                     Yt=torch.empty(M, lin.N, dtype=bf, device=dev), Y=torch.empty(M, lin.N, dtype=bf, device=dev),
+                     dY=torch.empty(M, lin.N, dtype=bf, device=dev), dX=torch.empty(M, lin.K, dtype=bf, device=dev),
+                     grads=[torch.empty(G, device=dev) for _ in range(3)],
+                     codes=torch.empty(lin.N * lin.K // 4, dtype=torch.uint8, device=dev),
+                     alpha=torch.empty(G, device=dev), loss=torch.empty(1, device=dev))
+            C.catq_soft_ternary_linear_fwd(layer, C.schedule(C.PHASE_TEACHER), d["X"], d["Yt"])
+            ws_bwd = max(ws_bwd, C.catq_bwd_workspace_bytes(layer, M))
+            ws_loss = max(ws_loss, C.catq_recon_loss_workspace_bytes(M * lin.N))
+            self.st.append(d)
+        self.main = torch.cuda.current_stream()
+        self.lanes = [self.main] if nstreams == 1 else [torch.cuda.Stream(device=dev) for _ in range(nstreams)]
+        self.wsbs = [C.workspace(ws_bwd, dev) for _ in self.lanes]
+        self.wsls = [C.workspace(ws_loss, dev) for _ in self.lanes]
+        torch.cuda.synchronize()
+
+    def step(self, sched, ev=None, serial=False, before=None, after=None):
+        """One step at schedule point `sched`; `serial` runs every linear on the current
+        stream (kernel timing); before(i) / after(i) run on linear i's stream around its
+        kernels (e2e copies); ev[i][kind] are (start, end) events around each GEMM call."""
+        C, torch, wl = self.C, self.torch, self.wl
+        use = [self.main] if serial else self.lanes
+        if len(use) > 1:
+            fork = torch.cuda.Event()
+            fork.record(self.main)
+            for s in use:
+                s.wait_event(fork)
+        for i, d in enumerate(self.st):
+            k = i % len(use)
+            with torch.cuda.stream(use[k]):
+                if before is not None:
+                    before(i)
+                L = d["layer"]
+                C.catq_group_stats(L, wl.thr_init)
+                if ev is not None:
+                    ev[i]["fwd"][0].record()
+                C.catq_soft_ternary_linear_fwd(L, sched, d["X"], d["Y"])
+                if ev is not None:
+                    ev[i]["fwd"][1].record()
+                C.catq_recon_loss(d["Y"], d["Yt"], d["loss"], d["dY"], self.wsls[k])
+                if ev is not None:
+                    ev[i]["dx"][0].record()
+                C.catq_soft_ternary_linear_bwd(L, sched, d["X"], d["dY"], dX=d["dX"])
+                if ev is not None:
+                    ev[i]["dx"][1].record()
+                    ev[i]["dw"][0].record()
+                C.catq_soft_ternary_linear_bwd(L, sched, d["X"], d["dY"], None, *d["grads"], workspace=self.wsbs[k])
+                if ev is not None:
+                    ev[i]["dw"][1].record()
+                C.catq_hard_ternarize_pack(L, d["codes"], d["alpha"])
+                if after is not None:
+                    after(i)
+        if len(use) > 1:
+            for s in use:
+                join = torch.cuda.Event()
+                join.record(s)
+                self.main.wait_event(join)
+
+    def ms_per_step(self, sched, steps, warmup, barrier):
+        """Mean step time over `steps` steps after `warmup`, CUDA events on this stream."""
+        torch = self.torch
+        for _ in range(warmup):
+            self.step(sched)
+        barrier()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(steps):
+            self.step(sched)
+        b.record()
+        barrier()
+        status = self.C.catq_device_status()
+        if status != 0:
+            raise SystemExit(f"device status {self.C.STATUS.get(status, status)} in a secondary timed region")
+        return a.elapsed_time(b) / steps
+
+
 def run_ours(args):
     import torch
 
@@ -241,88 +354,14 @@ def run_ours(args):
     wl = syn.WORKLOADS[args.workload]
     if wl.experts:
         raise SystemExit("MoE workloads are parity cases, not bench lines")
-    M = wl.M
-    bf = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
     sched = C.schedule(C.PHASE_SOFT, args.s)
-
-    def upload(a):
-        if wl.dtype == "bf16":
-            return torch.from_numpy(syn.bf16_bits(a).view(np.int16)).to(dev).view(torch.bfloat16)
-        return torch.from_numpy(a).to(dev)
-
-    Xs = {}
-    for lin in wl.linears:
-        if (lin.x, lin.K) not in Xs:
-            Xs[(lin.x, lin.K)] = upload(syn.activations(wl, lin.x, M, lin.K, seed=rank))
-    st = []
-    ws_bwd = ws_loss = 0
-    for lin in wl.linears:
-        G = lin.N * lin.K // wl.g
-        fac = [torch.from_numpy(f).to(dev) for f in syn.factors(G, rank, f"bench/{lin.name}", perturbed=True)]
-        layer = C.Layer.create(upload(syn.weight(wl, lin, seed=rank)), wl.g, *fac)
-        C.catq_group_stats(layer, wl.thr_init)
-        d = dict(lin=lin, layer=layer, X=Xs[(lin.x, lin.K)],
-                 Yt=torch.empty(M, lin.N, dtype=bf, device=dev), Y=torch.empty(M, lin.N, dtype=bf, device=dev),
-                 dY=torch.empty(M, lin.N, dtype=bf, device=dev), dX=torch.empty(M, lin.K, dtype=bf, device=dev),
-                 grads=[torch.empty(G, device=dev) for _ in range(3)],
-                 codes=torch.empty(lin.N * lin.K // 4, dtype=torch.uint8, device=dev),
-                 alpha=torch.empty(G, device=dev), loss=torch.empty(1, device=dev))
-        C.catq_soft_ternary_linear_fwd(layer, C.schedule(C.PHASE_TEACHER), d["X"], d["Yt"])
-        ws_bwd = max(ws_bwd, C.catq_bwd_workspace_bytes(layer, M))
-        ws_loss = max(ws_loss, C.catq_recon_loss_workspace_bytes(M * lin.N))
-        st.append(d)
-    # The block's linears are independent calibration problems (one loss per linear output,
-    # Eq. 7), so they are spread over `streams` CUDA streams: one linear's kernels can start
-    # on the SMs another linear's last tile wave leaves idle.  Each stream has its own
-    # workspaces; a step forks from and joins back into the current stream.
     nstreams = max(1, args.streams)
-    main = torch.cuda.current_stream()
-    lanes = [main] if nstreams == 1 else [torch.cuda.Stream(device=dev) for _ in range(nstreams)]
-    wsbs = [C.workspace(ws_bwd, dev) for _ in lanes]
-    wsls = [C.workspace(ws_loss, dev) for _ in lanes]
-    torch.cuda.synchronize()
-
-    kinds = ("fwd", "dx", "dw")
+    blk = BlockRun(C, torch, wl, dev, rank, nstreams)
+    st, M = blk.st, blk.M
+    kinds = KINDS
 
     def step(ev=None, serial=False, before=None, after=None):
-        """One step; `serial` runs every linear on the current stream (kernel timing).
-        before(i) / after(i) run on linear i's stream around its kernels (e2e copies)."""
-        use = [main] if serial else lanes
-        if len(use) > 1:
-            fork = torch.cuda.Event()
-            fork.record(main)
-            for s in use:
-                s.wait_event(fork)
-        for i, d in enumerate(st):
-            k = i % len(use)
-            with torch.cuda.stream(use[k]):
-                if before is not None:
-                    before(i)
-                L = d["layer"]
-                C.catq_group_stats(L, wl.thr_init)
-                if ev is not None:
-                    ev[i]["fwd"][0].record()
-                C.catq_soft_ternary_linear_fwd(L, sched, d["X"], d["Y"])
-                if ev is not None:
-                    ev[i]["fwd"][1].record()
-                C.catq_recon_loss(d["Y"], d["Yt"], d["loss"], d["dY"], wsls[k])
-                if ev is not None:
-                    ev[i]["dx"][0].record()
-                C.catq_soft_ternary_linear_bwd(L, sched, d["X"], d["dY"], dX=d["dX"])
-                if ev is not None:
-                    ev[i]["dx"][1].record()
-                    ev[i]["dw"][0].record()
-                C.catq_soft_ternary_linear_bwd(L, sched, d["X"], d["dY"], None, *d["grads"], workspace=wsbs[k])
-                if ev is not None:
-                    ev[i]["dw"][1].record()
-                C.catq_hard_ternarize_pack(L, d["codes"], d["alpha"])
-                if after is not None:
-                    after(i)
-        if len(use) > 1:
-            for s in use:
-                join = torch.cuda.Event()
-                join.record(s)
-                main.wait_event(join)
+        blk.step(sched, ev, serial, before, after)
 
     # per linear: stats; operand constants + forward; loss (partial + final); operand
     # constants + dX; dW + gradient reduce; pack
@@ -404,6 +443,30 @@ def run_ours(args):
     if not args.no_e2e:
         e2e = measure_e2e(args, C, torch, st, step, barrier, flops_step, world, dev)
 
+    # Secondary measurements (same code path, fewer steps): the HARD phase of this workload,
+    # and the other block workloads the 60%-of-peak target names or that fit the same step.
+    also = {}
+    if not args.no_also:
+        n2, w2 = max(5, args.steps // 4), 3
+
+        def entry(wl2, ms2):
+            ms2 = max_over_ranks(ms2, world, dev)
+            v2 = job_throughput(wl2.flops_per_step, ms2, world)
+            return {"value": v2, "ms_per_step": ms2, "frac_of_burst": v2 / world / peaks["bf16"], "steps": n2}
+
+        hard = blk.ms_per_step(C.schedule(C.PHASE_HARD, args.s), n2, w2, barrier)
+        also[f"{wl.name}/hard"] = dict(entry(wl, hard), phase="hard", s=args.s)
+        del blk, st, step
+        torch.cuda.empty_cache()
+        for name in ALSO_WORKLOADS:
+            if name == wl.name:
+                continue
+            wl2 = syn.WORKLOADS[name]
+            b2 = BlockRun(C, torch, wl2, dev, rank, nstreams)
+            also[f"{name}/soft"] = dict(entry(wl2, b2.ms_per_step(sched, n2, w2, barrier)), phase="soft", s=args.s)
+            del b2
+            torch.cuda.empty_cache()
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         t, fl = oracle_sample(wl, args.s)
@@ -420,6 +483,7 @@ def run_ours(args):
                                   "burst": value / world / peaks["bf16"], "source": peaks["source"]},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches_per_step * args.steps, "clocks": clk.summary(),
+            "also": also,
         }
         print(json.dumps(line), flush=True)
     if world > 1:
