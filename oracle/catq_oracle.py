@@ -219,6 +219,16 @@ def pack_codes(T):
     return out.astype(np.uint8)
 
 
+def ternary_infer(codes, alpha, N, K, g, X):
+    """Inference with the deployed form of a calibrated layer: App. B.2 keeps only the
+    ternary codes T and the group scale alpha (W ~ alpha T, Eq. 4), so Y = X (alpha T)^T
+    with T read from the 2-bit codes (``pack_codes``'s layout) and alpha [G] per group of g
+    consecutive elements of a row.  Returns Y [M, N] in fp64."""
+    T = unpack_codes(codes, N * K).astype(np.float64).reshape(N, K)
+    Wq = T * _per_elem(alpha, g).reshape(N, K)
+    return linear_fwd(X, Wq)
+
+
 def unpack_codes(codes, n):
     """Inverse of ``pack_codes`` (used only by tests)."""
     codes = np.asarray(codes, np.uint8).astype(np.int64)

@@ -404,3 +404,38 @@ def test_pack_hand_example():
 def test_pack_round_trip():
     T = np.random.default_rng(2).integers(-1, 2, 4096)
     np.testing.assert_array_equal(O.unpack_codes(O.pack_codes(T), T.size), T)
+
+
+# ---------------------------------------------------------------- deployed-form inference
+
+def _golden_infer():
+    vals = {}
+    path = os.path.join(os.path.dirname(__file__), "golden", "ternary_infer_example.txt")
+    for line in open(path):
+        if line.startswith("#") or ":" not in line:
+            continue
+        k, v = line.split(":", 1)
+        vals[k.strip()] = np.array(v.split(), dtype=np.float64)
+    return vals
+
+
+def test_ternary_infer_hand_example():
+    v = _golden_infer()
+    X = np.stack([v["x0"], v["x1"]])
+    Y = O.ternary_infer(v["bytes"].astype(np.uint8), v["alpha"], 2, 4, 2, X)
+    np.testing.assert_array_equal(Y, np.stack([v["y0"], v["y1"]]))
+
+
+def test_ternary_infer_is_the_hard_forward():
+    """Packing a layer's hard codes and inferring from them gives the HARD-phase forward."""
+    r = np.random.default_rng(11)
+    N, K, g, M = 6, 256, 128, 5
+    W = r.standard_normal((N, K)) * 0.02
+    X = r.standard_normal((M, K))
+    G = N * K // g
+    stats = O.group_stats(W, g, O.THR_HALF)
+    fac = (r.uniform(-0.1, 0.1, G), r.uniform(0.8, 1.2, G), r.uniform(0.8, 1.2, G))
+    T, alpha, _ = O.hard_codes(W, g, stats, fac)
+    Y = O.ternary_infer(O.pack_codes(T), alpha, N, K, g, X)
+    Wq = O.ternary_weight(W, g, stats, fac, O.PHASE_HARD, 30.0)[0]
+    np.testing.assert_allclose(Y, O.linear_fwd(X, Wq), rtol=1e-12, atol=1e-12)
