@@ -458,6 +458,8 @@ def run_ours(args):
         also[f"{wl.name}/hard"] = dict(entry(wl, hard), phase="hard", s=args.s)
         del blk, st, step
         torch.cuda.empty_cache()
+        also[f"{wl.name}/decode_b1"] = measure_decode(C, torch, wl, dev, peaks, rows=1)
+        also[f"{wl.name}/decode_b8"] = measure_decode(C, torch, wl, dev, peaks, rows=8)
         for name in ALSO_WORKLOADS:
             if name == wl.name:
                 continue
@@ -489,6 +491,56 @@ def run_ours(args):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20):
+    """Inference with the deployed form (catq_ternary_infer) of every linear of `blocks`
+    blocks shaped like `wl`, for `rows` token rows: one decode step reads every layer's 2-bit
+    codes and group scales once (working set far beyond L2).  The step's launches are
+    captured in a CUDA graph and replayed; value = algorithmic bytes / time."""
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(0)
+    layers, nbytes = [], 0
+    for _ in range(blocks):
+        for lin in wl.linears:
+            N, K, g = lin.N, lin.K, wl.g
+            r = torch.randint(0, 81, (N * K // 4,), generator=gen, device=dev, dtype=torch.int32)
+            codes = (r % 3 + ((r // 3) % 3) * 4 + ((r // 9) % 3) * 16 + (r // 27) * 64).to(torch.uint8)
+            alpha = torch.rand(N * K // g, generator=gen, device=dev) * 0.02 + 0.01
+            X = torch.randn(rows, K, generator=gen, device=dev).to(torch.bfloat16)
+            Y = torch.empty(rows, N, dtype=torch.bfloat16, device=dev)
+            layers.append((codes, alpha, N, K, g, X, Y))
+            nbytes += codes.numel() + alpha.numel() * 4 + X.numel() * 2 + Y.numel() * 2
+    side = torch.cuda.Stream(device=dev)
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):  # warm-up outside the capture
+        for L in layers:
+            C.catq_ternary_infer(*L)
+    torch.cuda.current_stream().wait_stream(side)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        for L in layers:
+            C.catq_ternary_infer(*L)
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(steps):
+        graph.replay()
+    b.record()
+    torch.cuda.synchronize()
+    status = C.catq_device_status()
+    if status != 0:
+        raise SystemExit(f"device status {C.STATUS.get(status, status)} in the decode timing")
+    ms = a.elapsed_time(b) / steps
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    del graph, layers
+    torch.cuda.empty_cache()
+    return {"kernel": "ternary_gemv_kernel (catq_ternary_infer)", "blocks": blocks, "token_rows": rows,
+            "launches_per_step": blocks * len(wl.linears), "bytes_per_step": nbytes, "us_per_step": ms * 1e3,
+            "value": gbs, "unit": "GB/s", "peak": peaks["hbm"], "frac_of_hbm": gbs / peaks["hbm"],
+            "steps": steps, "graph": True}
 
 
 def measure_e2e(args, C, torch, st, step, barrier, flops_step, world, dev):

@@ -248,6 +248,18 @@ catq_status catq_grouped_soft_ternary_linear_bwd(const catq_grouped_layer* layer
                                                  float* g_ddelta, void* workspace, size_t ws_bytes,
                                                  catq_stream stream);
 
+/* Inference with the deployed form of a calibrated layer (App. B.2: only the ternary codes
+ * and the group scale are kept, W ~ alpha T, Eq. 4):
+ *   Y[b, n] = sum_k X[b, k] * alpha[n * K/g + k/g] * T[n, k]
+ * with T[n, k] read from `codes` in catq_hard_ternarize_pack's layout (element e = n*K + k
+ * of row-major W stores T + 1 in bits 2(e%4)..2(e%4)+1 of byte e/4) and alpha [N*K/g] fp32
+ * (that call's alpha output).  X [B, K] and Y [B, N] are row-major bf16 (x_dtype must be
+ * CATQ_BF16), fp32 accumulation, one rounding of Y.  Meant for decode-shaped B (a few token
+ * rows); B == 0 is a no-op.  g must be a multiple of 64 and divide K.  codes and X 16-byte
+ * aligned, alpha 4-byte, Y 2-byte aligned; all device pointers owned by the caller. */
+catq_status catq_ternary_infer(const uint8_t* codes, const float* alpha, int64_t N, int64_t K, int32_t g,
+                               const void* X, int64_t B, int32_t x_dtype, void* Y, catq_stream stream);
+
 /* Self-test of the device-side failure detection (no counterpart in the paper): launches
  * one thread that waits, through the library's bounded mbarrier wait, on a barrier nothing
  * arrives on.  After timeout_ns (1 us .. 1 s) the wait gives up, latches CATQ_ERR_TIMEOUT

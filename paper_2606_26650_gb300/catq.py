@@ -84,6 +84,7 @@ def lib() -> ctypes.CDLL:
         "catq_hard_ternarize_pack": (I32, [LP, P, P, P]),
         "catq_device_status": (I32, [P, ctypes.POINTER(I32)]),
         "catq_selftest_wait_timeout": (I32, [ctypes.c_uint64, P]),
+        "catq_ternary_infer": (I32, [P, P, I64, I64, I32, P, I64, I32, P, P]),
         "catq_soft_ternary_linear_bwd_noalloc": (I32, [LP, catq_schedule, P, P, I64, I32, P, P, P, P, P]),
         "catq_bwd_noalloc_max_scratch_bytes": (S, []),
         "catq_grouped_soft_ternary_linear_fwd": (I32, [ctypes.POINTER(catq_grouped_layer), catq_schedule, P, P, I32, P,
@@ -252,6 +253,13 @@ def catq_device_status(stream=None) -> int:
     out = ctypes.c_int32(0)
     _check(lib().catq_device_status(_stream(stream), ctypes.byref(out)), "catq_device_status")
     return int(out.value)
+
+
+def catq_ternary_infer(codes, alpha, N: int, K: int, g: int, X, Y, stream=None):
+    """Y [B, N] = X [B, K] (alpha T)^T from the 2-bit codes and group scales of
+    catq_hard_ternarize_pack."""
+    _check(lib().catq_ternary_infer(_ptr(codes), _ptr(alpha), int(N), int(K), int(g), _ptr(X), X.shape[0],
+                                    _dtype_code(X), _ptr(Y), _stream(stream)), "catq_ternary_infer")
 
 
 def catq_selftest_wait_timeout(timeout_ns: int, stream=None):

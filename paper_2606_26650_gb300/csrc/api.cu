@@ -383,6 +383,20 @@ catq_status catq_grouped_soft_ternary_linear_bwd(const catq_grouped_layer* G, ca
   return CATQ_OK;
 }
 
+catq_status catq_ternary_infer(const uint8_t* codes, const float* alpha, int64_t N, int64_t K, int32_t g,
+                              const void* X, int64_t B, int32_t x_dtype, void* Y, catq_stream stream) {
+  if (!codes || !alpha) return CATQ_ERR_INVALID_ARG;
+  if (x_dtype != CATQ_BF16) return CATQ_ERR_DTYPE;
+  if (N < 1 || K < 1 || g < 64 || g % 64 != 0 || K % g != 0 || B < 0) return CATQ_ERR_SHAPE;
+  if (N * K / g >= (int64_t(1) << 31) || N >= (int64_t(1) << 31) || K >= (int64_t(1) << 31)) return CATQ_ERR_SHAPE;
+  if (B == 0) return CATQ_OK;
+  if (!X || !Y) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(codes) || !aligned16(X) || (reinterpret_cast<uintptr_t>(alpha) & 3u) != 0 ||
+      (reinterpret_cast<uintptr_t>(Y) & 1u) != 0)
+    return CATQ_ERR_ALIGN;
+  return cuda_status(launch_ternary_infer(codes, alpha, N, K, g, X, B, Y, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 catq_status catq_selftest_wait_timeout(uint64_t timeout_ns, catq_stream stream) {
   if (timeout_ns < 1000 || timeout_ns > 1000000000ull) return CATQ_ERR_INVALID_ARG;
   return cuda_status(launch_wait_probe(timeout_ns, reinterpret_cast<cudaStream_t>(stream)));

@@ -44,6 +44,10 @@ struct TcPlan {
   int32_t dw_P;       // partial-sum chunk width (columns)
 };
 TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count);
+// Y [B, N] = X [B, K] (alpha T)^T from 2-bit codes and group scales (bf16 X and Y).
+cudaError_t launch_ternary_infer(const uint8_t* codes, const float* alpha, int64_t N, int64_t K, int32_t g,
+                                 const void* X, int64_t B, void* Y, cudaStream_t st);
+
 // One-thread kernel whose bounded wait runs out after timeout_ns (self-test).
 cudaError_t launch_wait_probe(uint64_t timeout_ns, cudaStream_t st);
 

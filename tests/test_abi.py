@@ -89,5 +89,13 @@ def test_call_validation(lib):
     pack = lib.catq_hard_ternarize_pack
     assert pack(ctypes.byref(L), None, None, None) == 1
     assert lib.catq_device_status(None, None) == 1
+    infer = lib.catq_ternary_infer
+    assert infer(None, 32, 64, 256, 128, 16, 1, C.BF16, 16, None) == 1       # null codes
+    assert infer(16, 32, 64, 256, 128, 16, 1, C.F32, 16, None) == 3           # bf16 only
+    assert infer(16, 32, 64, 256, 32, 16, 1, C.BF16, 16, None) == 2           # g % 64 != 0
+    assert infer(16, 32, 64, 250, 128, 16, 1, C.BF16, 16, None) == 2          # g does not divide K
+    assert infer(16, 32, 64, 256, 128, 16, 0, C.BF16, 16, None) == 0          # B == 0: no-op
+    assert infer(24, 32, 64, 256, 128, 16, 1, C.BF16, 16, None) == 4          # misaligned codes
+    assert infer(16, 32, 64, 256, 128, 16, 1, C.BF16, None, None) == 1        # null Y
     assert lib.catq_selftest_wait_timeout(10, None) == 1              # below 1 us
     assert lib.catq_selftest_wait_timeout(2_000_000_000, None) == 1   # above 1 s

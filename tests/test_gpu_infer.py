@@ -1,0 +1,51 @@
+"""GPU parity of inference with the deployed form (codes + group scales, App. B.2): the
+codes and alpha come from catq_hard_ternarize_pack on the GPU (whose parity with the oracle
+test_gpu_parity checks), and catq_ternary_infer's Y is compared with the oracle's
+ternary_infer on the same codes, alpha and X (bf16 relative Frobenius error 2e-2)."""
+import numpy as np
+import pytest
+
+from oracle import catq_oracle as O
+from paper_2606_26650_gb300 import synthetic as syn
+from tests import gpu_util as U
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def device():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    return torch.device("cuda:0")
+
+
+@pytest.mark.parametrize("N,K,g,B", [
+    (1024, 4096, 128, 1),     # decode, one token row
+    (1024, 4096, 128, 3),
+    (520, 192, 64, 8),        # ragged N, a single full pass of 8 rows
+    (64, 512, 512, 11),       # channel-wise groups, two passes (8 + 3)
+    (4096, 14336, 128, 2),    # the Llama-3-8B-shaped down_proj
+])
+def test_ternary_infer_matches_oracle(device, N, K, g, B):
+    import torch
+
+    from paper_2606_26650_gb300 import catq as C
+    r = syn.rng(5, f"infer/{N}/{K}/{g}")
+    W = syn.round_bf16(r.standard_normal((N, K)).astype(np.float32) * 0.02)
+    X = syn.round_bf16(r.standard_normal((B, K)).astype(np.float32))
+    G = N * K // g
+    fac = syn.factors(G, 5, f"infer/{N}/{K}", perturbed=True)
+    layer = C.Layer.create(U.to_device(W, "bf16", device), g, *(torch.from_numpy(f).to(device) for f in fac))
+    C.catq_group_stats(layer)
+    codes = torch.empty(N * K // 4, dtype=torch.uint8, device=device)
+    alpha = torch.empty(G, dtype=torch.float32, device=device)
+    C.catq_hard_ternarize_pack(layer, codes, alpha)
+    Xt = U.to_device(X, "bf16", device)
+    Y = torch.empty(B, N, dtype=torch.bfloat16, device=device)
+    for _ in range(2):  # twice: the result does not depend on earlier calls
+        C.catq_ternary_infer(codes, alpha, N, K, g, Xt, Y)
+        torch.cuda.synchronize()
+        assert C.catq_device_status() == 0
+        want = O.ternary_infer(U.to_host(codes), U.to_host(alpha), N, K, g, X)
+        assert U.fro_rel(U.to_host(Y), want) <= U.TOL_BF16
