@@ -21,7 +21,7 @@ from __future__ import annotations
 import numpy as np
 
 PHASE_TEACHER, PHASE_SOFT, PHASE_HARD = 0, 1, 2
-THR_HALF, THR_TWN07 = 0, 1
+THR_HALF, THR_TWN07, THR_ABSMEAN, THR_TWN_STATIC = 0, 1, 2, 3
 
 
 def _groups(W: np.ndarray, g: int) -> np.ndarray:
@@ -38,8 +38,28 @@ def group_stats(W: np.ndarray, g: int, thr_init: int = THR_HALF):
     mu0 = mean of the group; alpha0 = mean |W - mu0|.  Delta0 = 0.5 in What units
     (§2.2 default) or, for the TWN rule of §2.2, the threshold 0.7 * mean|W| expressed
     in What units at identity factors: 0.7 * mean|W| / alpha0.
+
+    The static approximations §2.2 starts from, as base statistics for the modulation
+    (mu0 = 0, What = W / alpha):
+      THR_ABSMEAN     (BitNet b1.58 and others): alpha0 = mean |W|, Delta = alpha / 2, so
+                      Delta0 = 0.5 (alpha0 = 0: Delta0 = 0.5);
+      THR_TWN_STATIC  (TWN): Delta_W = 0.7 mean |W|, alpha0 = mean of |W_i| over
+                      |W_i| > Delta_W, Delta0 = Delta_W / alpha0 (alpha0 = 0, no element
+                      above the threshold: Delta0 = 0.5).
     """
     Wg = _groups(W, g)
+    if thr_init in (THR_ABSMEAN, THR_TWN_STATIC):
+        mean_abs = np.abs(Wg).mean(axis=1)
+        mu0 = np.zeros(Wg.shape[0])
+        if thr_init == THR_ABSMEAN:
+            return mu0, mean_abs, np.full_like(mean_abs, 0.5)
+        dW = 0.7 * mean_abs
+        above = np.abs(Wg) > dW[:, None]
+        cnt = above.sum(axis=1)
+        alpha0 = np.where(cnt > 0, (np.abs(Wg) * above).sum(axis=1) / np.maximum(cnt, 1), 0.0)
+        with np.errstate(divide="ignore", invalid="ignore"):
+            delta0 = np.where(alpha0 > 0, dW / np.where(alpha0 > 0, alpha0, 1.0), 0.5)
+        return mu0, alpha0, delta0
     mu0 = Wg.mean(axis=1)
     alpha0 = np.abs(Wg - mu0[:, None]).mean(axis=1)
     if thr_init == THR_HALF:

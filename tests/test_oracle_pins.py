@@ -439,3 +439,40 @@ def test_ternary_infer_is_the_hard_forward():
     Y = O.ternary_infer(O.pack_codes(T), alpha, N, K, g, X)
     Wq = O.ternary_weight(W, g, stats, fac, O.PHASE_HARD, 30.0)[0]
     np.testing.assert_allclose(Y, O.linear_fwd(X, Wq), rtol=1e-12, atol=1e-12)
+
+
+# ---------------------------------------------------------------- static scale/threshold rules
+
+def test_absmean_and_twn_static_closed_form():
+    """§2.2's static approximations on a hand-computed group (g = 4):
+    W = [3, -1, 0.5, -0.2]: mean|W| = 1.175.
+    absmean: alpha = 1.175, Delta = alpha / 2 (0.5 in What = W / alpha units).
+    TWN: Delta_W = 0.7 * 1.175 = 0.8225; elements above it: 3 and -1, alpha = 2,
+    Delta0 = 0.8225 / 2 = 0.41125."""
+    W = np.array([[3.0, -1.0, 0.5, -0.2]])
+    mu0, a0, d0 = O.group_stats(W, 4, O.THR_ABSMEAN)
+    np.testing.assert_allclose([mu0[0], a0[0], d0[0]], [0.0, 1.175, 0.5], rtol=0, atol=1e-15)
+    mu0, a0, d0 = O.group_stats(W, 4, O.THR_TWN_STATIC)
+    np.testing.assert_allclose([mu0[0], a0[0], d0[0]], [0.0, 2.0, 0.41125], rtol=0, atol=1e-15)
+
+
+def test_static_rules_at_identity_factors_are_the_papers_ternarizations():
+    """At identity factors the hard ternarization reproduces each rule as §2.2 states it:
+    absmean: T = sign(W) [|W| > mean|W| / 2], alpha = mean|W|;
+    TWN: T = sign(W) [|W| > 0.7 mean|W|], alpha = mean |W| over the kept elements."""
+    r = np.random.default_rng(12)
+    N, K, g = 5, 128, 64
+    W = r.standard_normal((N, K)) * 0.02
+    G = N * K // g
+    ident = (np.zeros(G), np.ones(G), np.ones(G))
+    Wg = W.reshape(G, g)
+    mean_abs = np.abs(Wg).mean(axis=1)
+    for rule, thr, alpha in (
+            (O.THR_ABSMEAN, mean_abs / 2, mean_abs),
+            (O.THR_TWN_STATIC, 0.7 * mean_abs,
+             np.array([np.abs(w[np.abs(w) > 0.7 * m]).mean() for w, m in zip(Wg, mean_abs)]))):
+        stats = O.group_stats(W, g, rule)
+        T, a, _ = O.hard_codes(W, g, stats, ident)
+        want_T = np.sign(Wg) * (np.abs(Wg) > thr[:, None])
+        np.testing.assert_array_equal(T.reshape(G, g), want_T)
+        np.testing.assert_allclose(a, alpha, rtol=1e-12)
