@@ -69,11 +69,17 @@ typedef enum {
   CATQ_PHASE_HARD = 2     /* gamma < t <= 1: T = Q(What; Delta) */
 } catq_phase;
 
-/* Initial threshold Delta0 in What units (§2.2). */
+/* Base statistics and initial threshold Delta0 (in What units) of each group (§2.2). */
 typedef enum {
-  CATQ_THR_HALF = 0,  /* Delta0 = 0.5, the paper's default (§2.2, App. B.1) */
-  CATQ_THR_TWN07 = 1  /* Delta0 = 0.7 * mean|W_group| / alpha0: TWN's 0.7 mean|W| rule (§2.2)
-                         expressed in What units, so alpha*Delta equals it at identity factors */
+  CATQ_THR_HALF = 0,  /* Eq. 3's mu0, alpha0 with Delta0 = 0.5, the paper's default (§2.2, App. B.1) */
+  CATQ_THR_TWN07 = 1, /* Eq. 3's mu0, alpha0 with Delta0 = 0.7 * mean|W_group| / alpha0: TWN's
+                         0.7 mean|W| threshold in What units (alpha*Delta equals it at identity
+                         factors) */
+  CATQ_THR_ABSMEAN = 2,    /* the absmean static rule §2.2 quotes (BitNet b1.58 and others):
+                              mu0 = 0, alpha0 = mean|W|, Delta0 = 0.5 (Delta = alpha / 2) */
+  CATQ_THR_TWN_STATIC = 3  /* TWN's static rule (§2.2): mu0 = 0, Delta_W = 0.7 mean|W|,
+                              alpha0 = mean |W_i| over |W_i| > Delta_W, Delta0 = Delta_W / alpha0
+                              (0.5 when no element is above) */
 } catq_thr_init;
 
 typedef enum { CATQ_REDUCE_MEAN = 0, CATQ_REDUCE_SUM = 1 } catq_reduction;
@@ -117,10 +123,12 @@ int32_t catq_abi_version(void);
 /* Human-readable name of a status code (static storage, never NULL). */
 const char* catq_status_string(int32_t status);
 
-/* Group statistics (Eq. 3; TWN 0.7 rule of §2.2 for CATQ_THR_TWN07):
+/* Group statistics (Eq. 3; the threshold rules of §2.2, see catq_thr_init):
  *   mu0[j] = mean of group j;  alpha0[j] = mean |W - mu0[j]| over group j;
- *   delta0[j] = 0.5, or 0.7 * mean|W| / alpha0[j] (0.5 if alpha0[j] == 0).
- * Sums run in fp64 on the device; results are stored as fp32.  Reads W once. */
+ *   delta0[j] = 0.5, or 0.7 * mean|W| / alpha0[j] (0.5 if alpha0[j] == 0);
+ * or, for the static rules, the values catq_thr_init states.  Sums are compensated fp32
+ * (two-sum; about twice fp32's precision) for the signed mean and pairwise fp32 for the
+ * all-positive ones; results are stored as fp32.  Reads W once. */
 catq_status catq_group_stats(const catq_layer* layer, int32_t thr_init, catq_stream stream);
 
 /* Materialises the Eq. 6 weight for inspection (not used inside the GEMMs, which fuse it).

@@ -18,7 +18,7 @@ HEADER = os.path.join(os.path.dirname(PKG), "include", "catq.h")
 
 F32, BF16 = 0, 1
 PHASE_TEACHER, PHASE_SOFT, PHASE_HARD = 0, 1, 2
-THR_HALF, THR_TWN07 = 0, 1
+THR_HALF, THR_TWN07, THR_ABSMEAN, THR_TWN_STATIC = 0, 1, 2, 3
 REDUCE_MEAN, REDUCE_SUM = 0, 1
 
 STATUS = {

@@ -160,7 +160,9 @@ const char* catq_status_string(int32_t s) {
 catq_status catq_group_stats(const catq_layer* layer, int32_t thr_init, catq_stream stream) {
   catq_status st = check_layer(layer, false);
   if (st != CATQ_OK) return st;
-  if (thr_init != CATQ_THR_HALF && thr_init != CATQ_THR_TWN07) return CATQ_ERR_INVALID_ARG;
+  if (thr_init != CATQ_THR_HALF && thr_init != CATQ_THR_TWN07 && thr_init != CATQ_THR_ABSMEAN &&
+      thr_init != CATQ_THR_TWN_STATIC)
+    return CATQ_ERR_INVALID_ARG;
   const LayerDev L = to_dev(layer);
   return cuda_status(launch_group_stats(L, layer->w_dtype, thr_init, layer->mu0, layer->alpha0, layer->delta0,
                                         reinterpret_cast<cudaStream_t>(stream)));

@@ -177,6 +177,78 @@ __global__ void __launch_bounds__(kThreads) group_stats_team_kernel(const T* __r
   }
 }
 
+// §2.2's static rules as base statistics for the modulation (mu0 = 0, What = W / alpha):
+//   absmean: alpha0 = mean|W|, Delta0 = 0.5 (Delta = alpha / 2);
+//   TWN:     Delta_W = 0.7 mean|W|, alpha0 = mean of |W_i| over |W_i| > Delta_W,
+//            Delta0 = Delta_W / alpha0 (0.5 when no element is above the threshold).
+constexpr int32_t kThrAbsmean = 2, kThrTwnStatic = 3;
+
+__device__ __forceinline__ void store_static_stats(int64_t j, int32_t rule, float mean_abs, float above_sum,
+                                                   float above_cnt, float* mu0, float* alpha0, float* delta0) {
+  mu0[j] = 0.0f;
+  if (rule == kThrAbsmean) {
+    alpha0[j] = mean_abs;
+    delta0[j] = 0.5f;
+    return;
+  }
+  const float a0 = above_cnt > 0.0f ? above_sum / above_cnt : 0.0f;
+  alpha0[j] = a0;
+  delta0[j] = a0 > 0.0f ? 0.7f * mean_abs / a0 : 0.5f;
+}
+
+// Register variant of the static rules (layout of group_stats_team_kernel): mean|W| from the
+// registers, then (TWN) a second pass over the same registers for the elements above
+// 0.7 mean|W|.
+template <typename T, int RULE>
+__global__ void __launch_bounds__(kThreads) group_stats_static_kernel(const T* __restrict__ W, int64_t G, int32_t g,
+                                                                      int32_t team, float* __restrict__ mu0,
+                                                                      float* __restrict__ alpha0,
+                                                                      float* __restrict__ delta0) {
+  constexpr int V = Vec16<T>::n;
+  constexpr int VPL = kStatsVPL;
+  const int lane = threadIdx.x & 31;
+  const int sub = lane & (team - 1);
+  const int per_warp = 32 / team;
+  const int64_t warp = (static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x) >> 5;
+  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
+  const float inv_g = 1.0f / static_cast<float>(g);
+  for (int64_t wbase = warp * per_warp; wbase < G; wbase += nwarps * per_warp) {
+    const int64_t j = wbase + lane / team;
+    const bool live = j < G;
+    float v[VPL][V];
+#pragma unroll
+    for (int r = 0; r < VPL; ++r) {
+      if (live) {
+        Vec16<T>::load(W + j * g + static_cast<int64_t>(r * team + sub) * V, v[r]);
+      } else {
+#pragma unroll
+        for (int q = 0; q < V; ++q) v[r][q] = 0.f;
+      }
+    }
+    float mag = 0.f;
+#pragma unroll
+    for (int r = 0; r < VPL; ++r) mag += pairwise_abs_sum<V>(v[r], 0.0f);
+    const float mean_abs = team_sum(mag, team) * inv_g;
+    float s = 0.f, cnt = 0.f;
+    if constexpr (RULE == kThrTwnStatic) {
+      const float dW = 0.7f * mean_abs;
+#pragma unroll
+      for (int r = 0; r < VPL; ++r)
+#pragma unroll
+        for (int q = 0; q < V; ++q) {
+          const float a = fabsf(v[r][q]);
+          if (a > dW) {
+            s += a;
+            cnt += 1.0f;
+          }
+        }
+      s = team_sum(s, team);
+      cnt = team_sum(cnt, team);
+    }
+    if (live && sub == 0) store_static_stats(j, RULE, mean_abs, s, cnt, mu0, alpha0, delta0);
+  }
+}
+
 // Streaming variant for any g (one warp per group, second pass re-reads the group).
 template <typename T>
 __global__ void __launch_bounds__(kThreads) group_stats_stream_kernel(const T* __restrict__ W, int64_t G, int32_t g,
@@ -210,6 +282,29 @@ __global__ void __launch_bounds__(kThreads) group_stats_stream_kernel(const T* _
     }
     dev = sum2_team(dev, 32);
     mag = sum2_team(mag, 32);
+    if (thr_init == kThrAbsmean || thr_init == kThrTwnStatic) {
+      const float mean_abs = sum2_float(mag) / static_cast<float>(g);
+      float s = 0.f, cnt = 0.f;
+      if (thr_init == kThrTwnStatic) {
+        const float dW = 0.7f * mean_abs;
+        for (int i = lane * V; i < g; i += 32 * V) {
+          float v[V];
+          Vec16<T>::load(base + i, v);
+#pragma unroll
+          for (int q = 0; q < V; ++q) {
+            const float a = fabsf(v[q]);
+            if (a > dW) {
+              s += a;
+              cnt += 1.0f;
+            }
+          }
+        }
+        s = team_sum(s, 32);
+        cnt = team_sum(cnt, 32);
+      }
+      if (lane == 0) store_static_stats(j, thr_init, mean_abs, s, cnt, mu0, alpha0, delta0);
+      continue;
+    }
     if (lane == 0) store_group_stats(j, g, thr_init, mu, dev, mag, mu0, alpha0, delta0);
   }
 }
@@ -524,6 +619,20 @@ cudaError_t launch_group_stats(const LayerDev& L, int32_t w_dtype, int32_t thr_i
   if (L.g % V == 0 && nvec % kStatsVPL == 0 && team <= 32 && (team & (team - 1)) == 0) {
     const int per_warp = 32 / team;
     const int grid = grid_for((G + per_warp - 1) / per_warp, kThreads / 32);
+    if (thr_init == kThrAbsmean || thr_init == kThrTwnStatic) {
+#define CATQ_STATS_STATIC(TT, RULE)                                                                          \
+  group_stats_static_kernel<TT, RULE><<<grid, kThreads, 0, st>>>(static_cast<const TT*>(L.W), G, L.g, team, \
+                                                                 mu0, alpha0, delta0)
+      if (w_dtype == 1) {
+        if (thr_init == kThrAbsmean) CATQ_STATS_STATIC(__nv_bfloat16, kThrAbsmean);
+        else CATQ_STATS_STATIC(__nv_bfloat16, kThrTwnStatic);
+      } else {
+        if (thr_init == kThrAbsmean) CATQ_STATS_STATIC(float, kThrAbsmean);
+        else CATQ_STATS_STATIC(float, kThrTwnStatic);
+      }
+#undef CATQ_STATS_STATIC
+      return cudaGetLastError();
+    }
     const bool twn = thr_init == 1;
 #define CATQ_STATS_TEAM(TT, TWN)                                                                                  \
   group_stats_team_kernel<TT, TWN><<<grid, kThreads, 0, st>>>(static_cast<const TT*>(L.W), G, L.g, team, mu0, \
