@@ -122,8 +122,9 @@ def _per_elem(v, g):
     return np.repeat(np.asarray(v, np.float64), g)
 
 
-def ternary_weight(W, g, stats, factors, phase, s):
-    """Eq. 6 and the reconstruction W ~ alpha T without mu (§2.2, App. B.2).
+def ternary_weight(W, g, stats, factors, phase, s, with_mu=False):
+    """Eq. 6 and the reconstruction W ~ alpha T without mu (§2.2, App. B.2), or with it,
+    W ~ alpha T + mu, when `with_mu` (the variant of the tab:mu ablation).
 
     Returns (Wq [N, K], T [N, K], What [N, K], alpha [G], Delta [G]).
     TEACHER (t = 0): T = W and Wq = W.  SOFT: T = f(What; s, Delta).  HARD: T = Q(What; Delta).
@@ -142,6 +143,8 @@ def ternary_weight(W, g, stats, factors, phase, s):
         raise ValueError("phase")
     T = np.where((alpha != 0)[:, None], T, 0.0)
     Wq = alpha[:, None] * T
+    if with_mu:
+        Wq = Wq + mu[:, None]  # a group with alpha == 0 reconstructs as mu
     return Wq.reshape(N, K), T.reshape(N, K), What.reshape(N, K), alpha, Delta
 
 
@@ -161,7 +164,7 @@ def recon_loss(Y, Y_ref, reduction: int = 0):
     return float((d * d).sum()), 2.0 * d
 
 
-def factor_grads_from_G(Gw, W, g, stats, factors, phase, s):
+def factor_grads_from_G(Gw, W, g, stats, factors, phase, s, with_mu=False):
     """Chain rule of Eq. 3 and Eq. 5/6 from G = dL/dWq [N, K] into the three factors.
 
     Wq = alpha * T(What), What = (W - mu)/alpha, mu = mu0 + d_mu*alpha0,
@@ -170,6 +173,7 @@ def factor_grads_from_G(Gw, W, g, stats, factors, phase, s):
     and the factor gradients are the group sums times alpha0, alpha0 and Delta0.
     SOFT: T = f.  HARD (reading of §2.3's stage-2 rule): T = Q(What; Delta) as in the
     forward, with f's derivatives at the given s — parity unpinned.  TEACHER: zeros.
+    With mu in the reconstruction (Wq = alpha T + mu), dWq/dmu = 1 - f'(What).
     """
     mu0, alpha0, delta0 = (np.asarray(a, np.float64) for a in stats)
     G = mu0.shape[0]
@@ -187,31 +191,32 @@ def factor_grads_from_G(Gw, W, g, stats, factors, phase, s):
     else:
         raise ValueError("phase")
     live = alpha != 0
-    g_dmu = np.where(live, -alpha0 * (Gg * dfdx).sum(axis=1), 0.0)
+    c_mu = (1.0 - dfdx) if with_mu else -dfdx
+    g_dmu = np.where(live, alpha0 * (Gg * c_mu).sum(axis=1), 0.0)
     g_dalpha = np.where(live, alpha0 * (Gg * (T - What * dfdx)).sum(axis=1), 0.0)
     g_ddelta = np.where(live, delta0 * alpha * (Gg * dfdD).sum(axis=1), 0.0)
     return g_dmu, g_dalpha, g_ddelta
 
 
-def linear_bwd(X, dY, W, g, stats, factors, phase, s):
+def linear_bwd(X, dY, W, g, stats, factors, phase, s, with_mu=False):
     """Backward of Y = X Wq^T: dX = dY Wq, G = dY^T X (= dL/dWq), then the factor
     gradients of ``factor_grads_from_G``.  Returns (dX, g_dmu, g_dalpha, g_ddelta)."""
     X = np.asarray(X, np.float64)
     dY = np.asarray(dY, np.float64)
-    Wq = ternary_weight(W, g, stats, factors, phase, s)[0]
+    Wq = ternary_weight(W, g, stats, factors, phase, s, with_mu)[0]
     dX = dY @ Wq
     Gw = dY.T @ X
-    return (dX,) + factor_grads_from_G(Gw, W, g, stats, factors, phase, s)
+    return (dX,) + factor_grads_from_G(Gw, W, g, stats, factors, phase, s, with_mu)
 
 
-def calibration_step(X, W, g, stats, factors, phase, s, reduction=0):
+def calibration_step(X, W, g, stats, factors, phase, s, reduction=0, with_mu=False):
     """One soft-ternary calibration step for one linear (Eq. 6, Eq. 7): teacher output,
     quantized output, loss, and every gradient.  Returns a dict."""
     Y_ref = linear_fwd(X, W)
-    Wq = ternary_weight(W, g, stats, factors, phase, s)[0]
+    Wq = ternary_weight(W, g, stats, factors, phase, s, with_mu)[0]
     Y = linear_fwd(X, Wq)
     loss, dY = recon_loss(Y, Y_ref, reduction)
-    dX, g_dmu, g_dalpha, g_ddelta = linear_bwd(X, dY, W, g, stats, factors, phase, s)
+    dX, g_dmu, g_dalpha, g_ddelta = linear_bwd(X, dY, W, g, stats, factors, phase, s, with_mu)
     return dict(Y_ref=Y_ref, Y=Y, loss=loss, dY=dY, dX=dX, g_dmu=g_dmu, g_dalpha=g_dalpha,
                 g_ddelta=g_ddelta, Wq=Wq)
 
@@ -239,13 +244,16 @@ def pack_codes(T):
     return out.astype(np.uint8)
 
 
-def ternary_infer(codes, alpha, N, K, g, X):
+def ternary_infer(codes, alpha, N, K, g, X, mu=None):
     """Inference with the deployed form of a calibrated layer: App. B.2 keeps only the
     ternary codes T and the group scale alpha (W ~ alpha T, Eq. 4), so Y = X (alpha T)^T
     with T read from the 2-bit codes (``pack_codes``'s layout) and alpha [G] per group of g
-    consecutive elements of a row.  Returns Y [M, N] in fp64."""
+    consecutive elements of a row.  With the group offsets mu [G] of the W ~ alpha T + mu
+    variant, Y = X (alpha T + mu)^T.  Returns Y [M, N] in fp64."""
     T = unpack_codes(codes, N * K).astype(np.float64).reshape(N, K)
     Wq = T * _per_elem(alpha, g).reshape(N, K)
+    if mu is not None:
+        Wq = Wq + _per_elem(mu, g).reshape(N, K)
     return linear_fwd(X, Wq)
 
 

@@ -476,3 +476,61 @@ def test_static_rules_at_identity_factors_are_the_papers_ternarizations():
         want_T = np.sign(Wg) * (np.abs(Wg) > thr[:, None])
         np.testing.assert_array_equal(T.reshape(G, g), want_T)
         np.testing.assert_allclose(a, alpha, rtol=1e-12)
+
+
+# ---------------------------------------------------------------- W ~ alpha T + mu variant
+
+def test_mu_reconstruction_reproduces_two_valued_groups():
+    """A group holding two values a < b is mu0 = (a + b)/2, alpha0 = (b - a)/2, What = -1 / +1
+    (Eq. 3), so at identity factors the hard ternarization with mu (tab:mu's variant) gives
+    alpha T + mu = W exactly, while without mu it gives -alpha0 / +alpha0."""
+    W = np.array([[1.0, 3.0, 3.0, 1.0, -2.0, -1.0, -1.0, -2.0]])
+    g = 4
+    stats = O.group_stats(W, g)
+    ident = (np.zeros(2), np.ones(2), np.ones(2))
+    Wq_mu = O.ternary_weight(W, g, stats, ident, O.PHASE_HARD, 30.0, with_mu=True)[0]
+    np.testing.assert_array_equal(Wq_mu, W)
+    Wq = O.ternary_weight(W, g, stats, ident, O.PHASE_HARD, 30.0)[0]
+    np.testing.assert_array_equal(Wq, [[-1, 1, 1, -1, -0.5, 0.5, 0.5, -0.5]])
+
+
+@pytest.mark.parametrize("s", [0.625, 30.0])
+def test_mu_variant_gradients_match_central_differences(s):
+    """With mu in the reconstruction the factor gradients (dWq/dmu = 1 - f') still match
+    central differences of the loss."""
+    W, X, g, stats, fac = _tiny(seed=3)
+    Y_ref = O.linear_fwd(X, W)
+
+    def loss(f):
+        Wq = O.ternary_weight(W, g, stats, f, O.PHASE_SOFT, s, with_mu=True)[0]
+        return O.recon_loss(O.linear_fwd(X, Wq), Y_ref)[0]
+
+    Wq = O.ternary_weight(W, g, stats, fac, O.PHASE_SOFT, s, with_mu=True)[0]
+    _, dY = O.recon_loss(O.linear_fwd(X, Wq), Y_ref)
+    dX, gmu, galpha, gdelta = O.linear_bwd(X, dY, W, g, stats, fac, O.PHASE_SOFT, s, with_mu=True)
+    np.testing.assert_allclose(dX, dY @ Wq)
+    h = 1e-6
+    for which, analytic in ((0, gmu), (1, galpha), (2, gdelta)):
+        fd = np.zeros_like(analytic)
+        for j in range(analytic.size):
+            fp = [a.copy() for a in fac]
+            fm = [a.copy() for a in fac]
+            fp[which][j] += h
+            fm[which][j] -= h
+            fd[j] = (loss(fp) - loss(fm)) / (2 * h)
+        np.testing.assert_allclose(analytic, fd, atol=1e-6 * np.abs(fd).max() + 1e-12)
+
+
+def test_ternary_infer_with_mu_is_the_hard_forward_with_mu():
+    r = np.random.default_rng(13)
+    N, K, g, M = 4, 128, 64, 3
+    W = r.standard_normal((N, K)) * 0.02
+    X = r.standard_normal((M, K))
+    G = N * K // g
+    stats = O.group_stats(W, g)
+    fac = (r.uniform(-0.1, 0.1, G), r.uniform(0.8, 1.2, G), r.uniform(0.8, 1.2, G))
+    T, alpha, _ = O.hard_codes(W, g, stats, fac)
+    mu = O.modulation(*stats, *fac)[0]
+    Y = O.ternary_infer(O.pack_codes(T), alpha, N, K, g, X, mu=mu)
+    Wq = O.ternary_weight(W, g, stats, fac, O.PHASE_HARD, 30.0, with_mu=True)[0]
+    np.testing.assert_allclose(Y, O.linear_fwd(X, Wq), rtol=1e-12, atol=1e-12)
