@@ -243,7 +243,7 @@ class BlockRun:
     start on the SMs another linear's last tile wave leaves idle.  A step forks from and
     joins back into the current stream."""
 
-    def __init__(self, C, torch, wl, dev, rank, nstreams):
+    def __init__(self, C, torch, wl, dev, rank, nstreams, recon=0):
         self.C, self.torch, self.wl = C, torch, wl
         M = self.M = wl.M
         bf = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
@@ -262,7 +262,7 @@ class BlockRun:
         for lin in wl.linears:
             G = lin.N * lin.K // wl.g
             fac = [torch.from_numpy(f).to(dev) for f in syn.factors(G, rank, f"bench/{lin.name}", perturbed=True)]
-            layer = C.Layer.create(upload(syn.weight(wl, lin, seed=rank)), wl.g, *fac)
+            layer = C.Layer.create(upload(syn.weight(wl, lin, seed=rank)), wl.g, *fac, recon=recon)
             C.catq_group_stats(layer, wl.thr_init)
             d = dict(lin=lin, layer=layer, X=Xs[(lin.x, lin.K)],
                      Yt=torch.empty(M, lin.N, dtype=bf, device=dev), Y=torch.empty(M, lin.N, dtype=bf, device=dev),
@@ -458,8 +458,15 @@ def run_ours(args):
         also[f"{wl.name}/hard"] = dict(entry(wl, hard), phase="hard", s=args.s)
         del blk, st, step
         torch.cuda.empty_cache()
+        # the W ~ alpha T + mu reconstruction (the tab:mu variant) on the same workload
+        bmu = BlockRun(C, torch, wl, dev, rank, nstreams, recon=C.RECON_ALPHA_T_MU)
+        also[f"{wl.name}/soft_mu"] = dict(entry(wl, bmu.ms_per_step(sched, n2, w2, barrier)), phase="soft", s=args.s,
+                                          recon="alpha_T_plus_mu")
+        del bmu
+        torch.cuda.empty_cache()
         also[f"{wl.name}/decode_b1"] = measure_decode(C, torch, wl, dev, peaks, rows=1)
         also[f"{wl.name}/decode_b8"] = measure_decode(C, torch, wl, dev, peaks, rows=8)
+        also[f"{wl.name}/decode_b1_mu"] = measure_decode(C, torch, wl, dev, peaks, rows=1, with_mu=True)
         for name in ALSO_WORKLOADS:
             if name == wl.name:
                 continue
@@ -493,11 +500,12 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20):
+def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20, with_mu=False):
     """Inference with the deployed form (catq_ternary_infer) of every linear of `blocks`
     blocks shaped like `wl`, for `rows` token rows: one decode step reads every layer's 2-bit
-    codes and group scales once (working set far beyond L2).  The step's launches are
-    captured in a CUDA graph and replayed; value = algorithmic bytes / time."""
+    codes and group scales (and group offsets, `with_mu`) once (working set far beyond L2).
+    The step's launches are captured in a CUDA graph and replayed; value = algorithmic
+    bytes / time."""
     gen = torch.Generator(device=dev)
     gen.manual_seed(0)
     layers, nbytes = [], 0
@@ -509,18 +517,20 @@ def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20):
             alpha = torch.rand(N * K // g, generator=gen, device=dev) * 0.02 + 0.01
             X = torch.randn(rows, K, generator=gen, device=dev).to(torch.bfloat16)
             Y = torch.empty(rows, N, dtype=torch.bfloat16, device=dev)
-            layers.append((codes, alpha, N, K, g, X, Y))
+            mu = (torch.rand(N * K // g, generator=gen, device=dev) - 0.5) * 0.01 if with_mu else None
+            layers.append(((codes, alpha, N, K, g, X, Y), mu))
             nbytes += codes.numel() + alpha.numel() * 4 + X.numel() * 2 + Y.numel() * 2
+            nbytes += 0 if mu is None else mu.numel() * 4
     side = torch.cuda.Stream(device=dev)
     side.wait_stream(torch.cuda.current_stream())
     with torch.cuda.stream(side):  # warm-up outside the capture
-        for L in layers:
-            C.catq_ternary_infer(*L)
+        for L, mu in layers:
+            C.catq_ternary_infer(*L, mu=mu)
     torch.cuda.current_stream().wait_stream(side)
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph):
-        for L in layers:
-            C.catq_ternary_infer(*L)
+        for L, mu in layers:
+            C.catq_ternary_infer(*L, mu=mu)
     for _ in range(3):
         graph.replay()
     torch.cuda.synchronize()
@@ -540,7 +550,7 @@ def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20):
     return {"kernel": "ternary_gemv_kernel (catq_ternary_infer)", "blocks": blocks, "token_rows": rows,
             "launches_per_step": blocks * len(wl.linears), "bytes_per_step": nbytes, "us_per_step": ms * 1e3,
             "value": gbs, "unit": "GB/s", "peak": peaks["hbm"], "frac_of_hbm": gbs / peaks["hbm"],
-            "steps": steps, "graph": True}
+            "steps": steps, "graph": True, "with_mu": with_mu}
 
 
 def measure_e2e(args, C, torch, st, step, barrier, flops_step, world, dev):

@@ -84,6 +84,15 @@ typedef enum {
 
 typedef enum { CATQ_REDUCE_MEAN = 0, CATQ_REDUCE_SUM = 1 } catq_reduction;
 
+/* Which reconstruction a layer's quantized weight uses. */
+typedef enum {
+  CATQ_RECON_ALPHA_T = 0,   /* W ~ alpha T (§2.2, App. B.2; the paper's choice): Wq = alpha T */
+  CATQ_RECON_ALPHA_T_MU = 1 /* W ~ alpha T + mu (the variant of the tab:mu ablation):
+                               Wq = alpha T + mu with mu = mu0 + d_mu alpha0 per group; the
+                               factor gradient of d_mu then follows dWq/dmu = 1 - f'(What).
+                               A group with alpha == 0 has Wq = mu. */
+} catq_recon;
+
 /* Eq. 6 schedule point.  SOFT: s = (t / gamma) * s0 > 0.  HARD: s is the sharpness of the
  * surrogate f used for the backward pass (§2.3, last stage-1 sharpness = s0).  TEACHER:
  * s is ignored. */
@@ -106,18 +115,22 @@ typedef struct {
   const float* d_mu;    /* [G] learnable factor d_mu    (Eq. 3), -1 < d_mu < 1 */
   const float* d_alpha; /* [G] learnable factor d_alpha (Eq. 3), > 0 */
   const float* d_delta; /* [G] learnable factor d_delta (§2.2), > 0 */
-  /* [4*G] fp32, 16-byte aligned; required for bf16 layers by the forward and by a backward
-   * that computes dX, ignored otherwise.  Each such call first writes here the four
-   * per-group constants of its schedule point that turn a weight into its Eq. 6 operand
-   * (SOFT: s/alpha, -s mu/alpha, s Delta, alpha/(2 tanh s); HARD: 1/alpha, -mu/alpha,
-   * Delta, alpha), as float4 in group-column-major order [K/g][N], then the fused GEMMs
-   * read one 16-byte vector per group and row.  Contents are overwritten by every call, so
-   * two calls on one layer must not overlap on the GPU. */
+  /* [4*G] fp32 ([5*G] when recon is CATQ_RECON_ALPHA_T_MU), 16-byte aligned; required for
+   * bf16 layers by the forward and by a backward that computes dX, ignored otherwise.  Each
+   * such call first writes here the four per-group constants of its schedule point that
+   * turn a weight into its Eq. 6 operand (SOFT: s/alpha, -s mu/alpha, s Delta,
+   * alpha/(2 tanh s); HARD: 1/alpha, -mu/alpha, Delta, alpha), as float4 in
+   * group-column-major order [K/g][N], then (CATQ_RECON_ALPHA_T_MU only) the G group offsets
+   * mu in the same order; the fused GEMMs read one 16-byte vector (and one mu) per group
+   * and row.  Contents are overwritten by every call, so two calls on one layer must not
+   * overlap on the GPU. */
   float* op_const;
+  int32_t recon;    /* catq_recon */
+  int32_t reserved; /* must be 0 */
 } catq_layer;
 
 /* ABI version of this header; bumped on any incompatible change. */
-#define CATQ_ABI_VERSION 2
+#define CATQ_ABI_VERSION 3
 int32_t catq_abi_version(void);
 
 /* Human-readable name of a status code (static storage, never NULL). */
@@ -209,9 +222,11 @@ catq_status catq_recon_loss(const void* Y, const void* Y_ref, int64_t count, int
  * deployment keeps only T and the group scale alpha, App. B.2):
  *   codes [N*K/4] uint8: element e of row-major W stores Q(What_e; Delta) + 1 in bits
  *         [2*(e%4), 2*(e%4)+1] of byte e/4 (values 0, 1, 2; 3 never occurs).
- *   alpha [G] fp32: d_alpha * alpha0.  Requires N*K % 4 == 0.  The encoding is this
- *   library's; the paper fixes none.                                                     */
-catq_status catq_hard_ternarize_pack(const catq_layer* layer, uint8_t* codes, float* alpha,
+ *   alpha [G] fp32, nullable: d_alpha * alpha0.
+ *   mu    [G] fp32, nullable: mu0 + d_mu * alpha0, the group offsets a layer with
+ *         CATQ_RECON_ALPHA_T_MU deploys beside alpha.
+ * Requires N*K % 4 == 0.  The encoding is this library's; the paper fixes none.          */
+catq_status catq_hard_ternarize_pack(const catq_layer* layer, uint8_t* codes, float* alpha, float* mu,
                                      catq_stream stream);
 
 /* ------------------------------------------------------------------ grouped (MoE) layers
@@ -228,7 +243,7 @@ typedef struct {
   int32_t g;       /* group size */
   int64_t N, K;    /* one expert's out_features, in_features */
   int32_t w_dtype; /* catq_dtype */
-  int32_t reserved;
+  int32_t recon;   /* catq_recon, for every expert */
   const void* W;   /* [E, N, K] */
   float* mu0;      /* [E, G] */
   float* alpha0;
@@ -236,7 +251,8 @@ typedef struct {
   const float* d_mu;
   const float* d_alpha;
   const float* d_delta;
-  float* op_const; /* [E, 4*G]: per expert as catq_layer.op_const */
+  float* op_const; /* [E, 4*G] ([E, 5*G] with CATQ_RECON_ALPHA_T_MU): per expert as
+                      catq_layer.op_const */
 } catq_grouped_layer;
 
 /* Forward of every expert: Y[rows of e] = X[rows of e] Wq_e^T (Eq. 6 weight per expert). */
@@ -258,15 +274,18 @@ catq_status catq_grouped_soft_ternary_linear_bwd(const catq_grouped_layer* layer
 
 /* Inference with the deployed form of a calibrated layer (App. B.2: only the ternary codes
  * and the group scale are kept, W ~ alpha T, Eq. 4):
- *   Y[b, n] = sum_k X[b, k] * alpha[n * K/g + k/g] * T[n, k]
+ *   Y[b, n] = sum_k X[b, k] * (alpha[n * K/g + k/g] * T[n, k] + mu[n * K/g + k/g])
  * with T[n, k] read from `codes` in catq_hard_ternarize_pack's layout (element e = n*K + k
- * of row-major W stores T + 1 in bits 2(e%4)..2(e%4)+1 of byte e/4) and alpha [N*K/g] fp32
- * (that call's alpha output).  X [B, K] and Y [B, N] are row-major bf16 (x_dtype must be
- * CATQ_BF16), fp32 accumulation, one rounding of Y.  Meant for decode-shaped B (a few token
- * rows); B == 0 is a no-op.  g must be a multiple of 64 and divide K.  codes and X 16-byte
- * aligned, alpha 4-byte, Y 2-byte aligned; all device pointers owned by the caller. */
-catq_status catq_ternary_infer(const uint8_t* codes, const float* alpha, int64_t N, int64_t K, int32_t g,
-                               const void* X, int64_t B, int32_t x_dtype, void* Y, catq_stream stream);
+ * of row-major W stores T + 1 in bits 2(e%4)..2(e%4)+1 of byte e/4), alpha [N*K/g] fp32
+ * (that call's alpha output) and mu [N*K/g] fp32 (its mu output, for a layer calibrated with
+ * CATQ_RECON_ALPHA_T_MU; NULL for the W ~ alpha T form, mu = 0).  X [B, K] and Y [B, N] are
+ * row-major bf16 (x_dtype must be CATQ_BF16), fp32 accumulation, one rounding of Y.  Meant
+ * for decode-shaped B (a few token rows); B == 0 is a no-op.  g must be a multiple of 64
+ * and divide K.  codes and X 16-byte aligned, alpha and mu 4-byte, Y 2-byte aligned; all
+ * device pointers owned by the caller. */
+catq_status catq_ternary_infer(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K,
+                               int32_t g, const void* X, int64_t B, int32_t x_dtype, void* Y,
+                               catq_stream stream);
 
 /* Self-test of the device-side failure detection (no counterpart in the paper): launches
  * one thread that waits, through the library's bounded mbarrier wait, on a barrier nothing

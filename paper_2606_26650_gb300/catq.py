@@ -20,6 +20,7 @@ F32, BF16 = 0, 1
 PHASE_TEACHER, PHASE_SOFT, PHASE_HARD = 0, 1, 2
 THR_HALF, THR_TWN07, THR_ABSMEAN, THR_TWN_STATIC = 0, 1, 2, 3
 REDUCE_MEAN, REDUCE_SUM = 0, 1
+RECON_ALPHA_T, RECON_ALPHA_T_MU = 0, 1
 
 STATUS = {
     0: "CATQ_OK", 1: "CATQ_ERR_INVALID_ARG", 2: "CATQ_ERR_SHAPE", 3: "CATQ_ERR_DTYPE",
@@ -40,14 +41,14 @@ class catq_layer(ctypes.Structure):
         ("W", ctypes.c_void_p),
         ("mu0", ctypes.c_void_p), ("alpha0", ctypes.c_void_p), ("delta0", ctypes.c_void_p),
         ("d_mu", ctypes.c_void_p), ("d_alpha", ctypes.c_void_p), ("d_delta", ctypes.c_void_p),
-        ("op_const", ctypes.c_void_p),
+        ("op_const", ctypes.c_void_p), ("recon", ctypes.c_int32), ("reserved", ctypes.c_int32),
     ]
 
 
 class catq_grouped_layer(ctypes.Structure):
     _fields_ = [
         ("E", ctypes.c_int32), ("g", ctypes.c_int32), ("N", ctypes.c_int64), ("K", ctypes.c_int64),
-        ("w_dtype", ctypes.c_int32), ("reserved", ctypes.c_int32), ("W", ctypes.c_void_p),
+        ("w_dtype", ctypes.c_int32), ("recon", ctypes.c_int32), ("W", ctypes.c_void_p),
         ("mu0", ctypes.c_void_p), ("alpha0", ctypes.c_void_p), ("delta0", ctypes.c_void_p),
         ("d_mu", ctypes.c_void_p), ("d_alpha", ctypes.c_void_p), ("d_delta", ctypes.c_void_p),
         ("op_const", ctypes.c_void_p),
@@ -81,10 +82,10 @@ def lib() -> ctypes.CDLL:
         "catq_soft_ternary_linear_bwd": (I32, [LP, catq_schedule, P, P, I64, I32, P, P, P, P, P, S, P]),
         "catq_recon_loss_workspace_bytes": (S, [I64]),
         "catq_recon_loss": (I32, [P, P, I64, I32, I32, P, P, P, S, P]),
-        "catq_hard_ternarize_pack": (I32, [LP, P, P, P]),
+        "catq_hard_ternarize_pack": (I32, [LP, P, P, P, P]),
         "catq_device_status": (I32, [P, ctypes.POINTER(I32)]),
         "catq_selftest_wait_timeout": (I32, [ctypes.c_uint64, P]),
-        "catq_ternary_infer": (I32, [P, P, I64, I64, I32, P, I64, I32, P, P]),
+        "catq_ternary_infer": (I32, [P, P, P, I64, I64, I32, P, I64, I32, P, P]),
         "catq_soft_ternary_linear_bwd_noalloc": (I32, [LP, catq_schedule, P, P, I64, I32, P, P, P, P, P]),
         "catq_bwd_noalloc_max_scratch_bytes": (S, []),
         "catq_grouped_soft_ternary_linear_fwd": (I32, [ctypes.POINTER(catq_grouped_layer), catq_schedule, P, P, I32, P,
@@ -137,7 +138,8 @@ def _check(status: int, where: str):
 @dataclasses.dataclass
 class Layer:
     """One linear layer's device state: W [N, K], the per-group arrays ([G] fp32) and the
-    operand-constant array the fused GEMMs read ([4 G] fp32)."""
+    operand-constant array the fused GEMMs read ([4 G] fp32, [5 G] with mu in the
+    reconstruction).  `recon`: RECON_ALPHA_T (W ~ alpha T) or RECON_ALPHA_T_MU."""
     W: object
     g: int
     mu0: object
@@ -147,9 +149,10 @@ class Layer:
     d_alpha: object
     d_delta: object
     op_const: object = None
+    recon: int = RECON_ALPHA_T
 
     @classmethod
-    def create(cls, W, g, d_mu=None, d_alpha=None, d_delta=None):
+    def create(cls, W, g, d_mu=None, d_alpha=None, d_delta=None, recon=RECON_ALPHA_T):
         """Allocates the statistics, operand-constant and (identity, unless given) factor
         tensors."""
         import torch
@@ -160,7 +163,7 @@ class Layer:
                    d_mu if d_mu is not None else torch.zeros(G, **kw),
                    d_alpha if d_alpha is not None else torch.ones(G, **kw),
                    d_delta if d_delta is not None else torch.ones(G, **kw),
-                   torch.empty(4 * G, **kw))
+                   torch.empty((5 if recon else 4) * G, **kw), int(recon))
 
     @property
     def N(self):
@@ -178,7 +181,7 @@ class Layer:
         return catq_layer(self.N, self.K, self.g, _dtype_code(self.W), self.W.data_ptr(),
                           self.mu0.data_ptr(), self.alpha0.data_ptr(), self.delta0.data_ptr(),
                           self.d_mu.data_ptr(), self.d_alpha.data_ptr(), self.d_delta.data_ptr(),
-                          self.op_const.data_ptr() if self.op_const is not None else None)
+                          self.op_const.data_ptr() if self.op_const is not None else None, self.recon, 0)
 
 
 def schedule(phase: int, s: float = 0.0) -> catq_schedule:
@@ -243,9 +246,9 @@ def catq_recon_loss(Y, Y_ref, loss_out, dY=None, workspace=None, reduction: int 
                                  _ptr(dY), _ptr(workspace), ws_bytes, _stream(stream)), "catq_recon_loss")
 
 
-def catq_hard_ternarize_pack(layer: Layer, codes, alpha=None, stream=None):
+def catq_hard_ternarize_pack(layer: Layer, codes, alpha=None, mu=None, stream=None):
     st = layer.struct()
-    _check(lib().catq_hard_ternarize_pack(ctypes.byref(st), _ptr(codes), _ptr(alpha), _stream(stream)),
+    _check(lib().catq_hard_ternarize_pack(ctypes.byref(st), _ptr(codes), _ptr(alpha), _ptr(mu), _stream(stream)),
            "catq_hard_ternarize_pack")
 
 
@@ -255,11 +258,11 @@ def catq_device_status(stream=None) -> int:
     return int(out.value)
 
 
-def catq_ternary_infer(codes, alpha, N: int, K: int, g: int, X, Y, stream=None):
-    """Y [B, N] = X [B, K] (alpha T)^T from the 2-bit codes and group scales of
-    catq_hard_ternarize_pack."""
-    _check(lib().catq_ternary_infer(_ptr(codes), _ptr(alpha), int(N), int(K), int(g), _ptr(X), X.shape[0],
-                                    _dtype_code(X), _ptr(Y), _stream(stream)), "catq_ternary_infer")
+def catq_ternary_infer(codes, alpha, N: int, K: int, g: int, X, Y, mu=None, stream=None):
+    """Y [B, N] = X [B, K] (alpha T + mu)^T from the 2-bit codes, group scales and (for the
+    W ~ alpha T + mu form) group offsets of catq_hard_ternarize_pack."""
+    _check(lib().catq_ternary_infer(_ptr(codes), _ptr(alpha), _ptr(mu), int(N), int(K), int(g), _ptr(X),
+                                    X.shape[0], _dtype_code(X), _ptr(Y), _stream(stream)), "catq_ternary_infer")
 
 
 def catq_selftest_wait_timeout(timeout_ns: int, stream=None):
@@ -283,9 +286,9 @@ class GroupedLayer:
     dense: Layer
 
     @classmethod
-    def create(cls, W, g, d_mu=None, d_alpha=None, d_delta=None):
+    def create(cls, W, g, d_mu=None, d_alpha=None, d_delta=None, recon=RECON_ALPHA_T):
         E, N, K = W.shape
-        return cls(W, g, Layer.create(W.reshape(E * N, K), g, d_mu, d_alpha, d_delta))
+        return cls(W, g, Layer.create(W.reshape(E * N, K), g, d_mu, d_alpha, d_delta, recon))
 
     @property
     def E(self):
@@ -294,7 +297,7 @@ class GroupedLayer:
     def struct(self) -> catq_grouped_layer:
         E, N, K = self.W.shape
         d = self.dense
-        return catq_grouped_layer(E, self.g, N, K, _dtype_code(self.W), 0, self.W.data_ptr(), d.mu0.data_ptr(),
+        return catq_grouped_layer(E, self.g, N, K, _dtype_code(self.W), d.recon, self.W.data_ptr(), d.mu0.data_ptr(),
                                   d.alpha0.data_ptr(), d.delta0.data_ptr(), d.d_mu.data_ptr(), d.d_alpha.data_ptr(),
                                   d.d_delta.data_ptr(), d.op_const.data_ptr() if d.op_const is not None else None)
 

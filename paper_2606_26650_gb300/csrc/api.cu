@@ -36,6 +36,8 @@ catq_status check_layer(const catq_layer* L, bool need_factors) {
     if (!(L->g % 64 == 0 || L->g == 4 || L->g == 8 || L->g == 16 || L->g == 32)) return CATQ_ERR_SHAPE;
   }
   if (!aligned16(L->W)) return CATQ_ERR_ALIGN;
+  if (L->recon != CATQ_RECON_ALPHA_T && L->recon != CATQ_RECON_ALPHA_T_MU) return CATQ_ERR_INVALID_ARG;
+  if (L->reserved != 0) return CATQ_ERR_INVALID_ARG;
   if (!L->mu0 || !L->alpha0 || !L->delta0) return CATQ_ERR_INVALID_ARG;
   if (need_factors && (!L->d_mu || !L->d_alpha || !L->d_delta)) return CATQ_ERR_INVALID_ARG;
   return CATQ_OK;
@@ -69,6 +71,8 @@ LayerDev to_dev(const catq_layer* L) {
   d.d_alpha = L->d_alpha;
   d.d_delta = L->d_delta;
   d.op_const = reinterpret_cast<float4*>(L->op_const);
+  d.recon = L->recon;
+  d.op_mu = (L->recon && L->op_const) ? L->op_const + 4 * (L->N * L->K / L->g) : nullptr;
   return d;
 }
 
@@ -293,13 +297,14 @@ catq_status catq_recon_loss(const void* Y, const void* Y_ref, int64_t count, int
                                        static_cast<double*>(workspace), reinterpret_cast<cudaStream_t>(stream)));
 }
 
-catq_status catq_hard_ternarize_pack(const catq_layer* layer, uint8_t* codes, float* alpha, catq_stream stream) {
+catq_status catq_hard_ternarize_pack(const catq_layer* layer, uint8_t* codes, float* alpha, float* mu,
+                                     catq_stream stream) {
   catq_status st = check_layer(layer, true);
   if (st != CATQ_OK) return st;
   if (!codes) return CATQ_ERR_INVALID_ARG;
   if ((layer->N * layer->K) % 4 != 0) return CATQ_ERR_SHAPE;
   if (layer->g % 16 == 0 && !aligned16(codes)) return CATQ_ERR_ALIGN;
-  return cuda_status(launch_hard_pack(to_dev(layer), layer->w_dtype, codes, alpha,
+  return cuda_status(launch_hard_pack(to_dev(layer), layer->w_dtype, codes, alpha, mu,
                                       reinterpret_cast<cudaStream_t>(stream)));
 }
 
@@ -323,7 +328,9 @@ catq_layer expert_layer(const catq_grouped_layer* G, int32_t e) {
   L.d_mu = G->d_mu ? G->d_mu + e * groups : nullptr;
   L.d_alpha = G->d_alpha ? G->d_alpha + e * groups : nullptr;
   L.d_delta = G->d_delta ? G->d_delta + e * groups : nullptr;
-  L.op_const = G->op_const ? G->op_const + 4 * e * groups : nullptr;
+  L.op_const = G->op_const ? G->op_const + (G->recon ? 5 : 4) * e * groups : nullptr;
+  L.recon = G->recon;
+  L.reserved = 0;
   return L;
 }
 
@@ -385,8 +392,8 @@ catq_status catq_grouped_soft_ternary_linear_bwd(const catq_grouped_layer* G, ca
   return CATQ_OK;
 }
 
-catq_status catq_ternary_infer(const uint8_t* codes, const float* alpha, int64_t N, int64_t K, int32_t g,
-                              const void* X, int64_t B, int32_t x_dtype, void* Y, catq_stream stream) {
+catq_status catq_ternary_infer(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K,
+                              int32_t g, const void* X, int64_t B, int32_t x_dtype, void* Y, catq_stream stream) {
   if (!codes || !alpha) return CATQ_ERR_INVALID_ARG;
   if (x_dtype != CATQ_BF16) return CATQ_ERR_DTYPE;
   if (N < 1 || K < 1 || g < 64 || g % 64 != 0 || K % g != 0 || B < 0) return CATQ_ERR_SHAPE;
@@ -394,9 +401,10 @@ catq_status catq_ternary_infer(const uint8_t* codes, const float* alpha, int64_t
   if (B == 0) return CATQ_OK;
   if (!X || !Y) return CATQ_ERR_INVALID_ARG;
   if (!aligned16(codes) || !aligned16(X) || (reinterpret_cast<uintptr_t>(alpha) & 3u) != 0 ||
-      (reinterpret_cast<uintptr_t>(Y) & 1u) != 0)
+      (reinterpret_cast<uintptr_t>(mu) & 3u) != 0 || (reinterpret_cast<uintptr_t>(Y) & 1u) != 0)
     return CATQ_ERR_ALIGN;
-  return cuda_status(launch_ternary_infer(codes, alpha, N, K, g, X, B, Y, reinterpret_cast<cudaStream_t>(stream)));
+  return cuda_status(
+      launch_ternary_infer(codes, alpha, mu, N, K, g, X, B, Y, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 catq_status catq_selftest_wait_timeout(uint64_t timeout_ns, catq_stream stream) {

@@ -21,6 +21,8 @@ struct LayerDev {
   const float* d_alpha;
   const float* d_delta;
   float4* op_const;  // [K/g][N] operand constants (operand_const_vec), written per call
+  float* op_mu;      // [K/g][N] group offsets mu after op_const when recon, else nullptr
+  int32_t recon;     // 0: W ~ alpha T (§2.2);  1: W ~ alpha T + mu (the tab:mu variant)
 };
 
 // Eq. 3 and §2.2 for group j:
@@ -28,7 +30,7 @@ struct LayerDev {
 //   What = (W - mu) / alpha evaluated as fma(W, r, b) with r = 1/alpha, b = -mu r.
 // alpha == 0 (degenerate group) gives r = b = 0, so What = 0 and alpha * T = 0.
 struct GroupConst {
-  float r, b, alpha, delta, alpha0, delta0;
+  float r, b, alpha, delta, alpha0, delta0, mu;
 };
 
 // The six per-group inputs, loaded separately from the arithmetic so callers can issue the
@@ -60,6 +62,7 @@ __device__ __forceinline__ GroupConst group_const(const GroupRaw& g) {
   c.delta = delta;
   c.alpha0 = g.a0;
   c.delta0 = g.D0;
+  c.mu = mu;
   return c;
 }
 
@@ -90,15 +93,19 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 //         1 to well below bf16 resolution (and symmetrically for u < 0), so
 //         alpha f = sign(u) C (1 + tanh(|u| - D)) needs one tanh instead of two.
 //   HARD: What = fma(w, r, b), threshold Delta, C = alpha.
+//   M: the group offset mu added to alpha T in the W ~ alpha T + mu reconstruction (read only
+//   by the transforms of that reconstruction).
 struct ProducerConst {
   float A, B, D, C;
   float r, b, delta;
+  float M;
   bool one_tanh;
 };
 
 __device__ __forceinline__ ProducerConst producer_const(const GroupConst& c, float s, float inv_2tanh_s,
                                                         int32_t phase) {
   ProducerConst p;
+  p.M = c.mu;
   p.A = s * c.r;
   p.B = s * c.b;
   p.D = s * c.delta;
@@ -119,15 +126,19 @@ __device__ __forceinline__ float tanh_fast(float x) {
 // Eq. 5/6 SOFT weight alpha f(What; s, Delta) for two bf16 weights, fp32 arithmetic with
 // the hardware tanh, rounded once to bf16.  ONE_TANH selects the one-tanh form (valid when
 // p.one_tanh); the choice is made once per row, outside the element loop.
-template <bool ONE_TANH>
+// MU adds the group offset (alpha f + mu, one rounding).
+template <bool ONE_TANH, bool MU = false>
 __device__ __forceinline__ uint32_t soft_pair_bf16(uint32_t w2, const ProducerConst& p) {
   const float u0 = fmaf(bf16lo_to_f32(w2), p.A, p.B);
   const float u1 = fmaf(bf16hi_to_f32(w2), p.A, p.B);
   float y0, y1;
   if constexpr (ONE_TANH) {
     const float c0 = copysignf(p.C, u0), c1 = copysignf(p.C, u1);
-    y0 = fmaf(tanh_fast(fabsf(u0) - p.D), c0, c0);
-    y1 = fmaf(tanh_fast(fabsf(u1) - p.D), c1, c1);
+    y0 = fmaf(tanh_fast(fabsf(u0) - p.D), c0, MU ? c0 + p.M : c0);
+    y1 = fmaf(tanh_fast(fabsf(u1) - p.D), c1, MU ? c1 + p.M : c1);
+  } else if constexpr (MU) {
+    y0 = fmaf(p.C, tanh_fast(u0 - p.D) + tanh_fast(u0 + p.D), p.M);
+    y1 = fmaf(p.C, tanh_fast(u1 - p.D) + tanh_fast(u1 + p.D), p.M);
   } else {
     y0 = p.C * (tanh_fast(u0 - p.D) + tanh_fast(u0 + p.D));
     y1 = p.C * (tanh_fast(u1 - p.D) + tanh_fast(u1 + p.D));
@@ -135,12 +146,17 @@ __device__ __forceinline__ uint32_t soft_pair_bf16(uint32_t w2, const ProducerCo
   return pack_bf16x2(y0, y1);
 }
 
-// Eq. 2/6 HARD weight alpha Q(What; Delta) for two bf16 weights.
+// Eq. 2/6 HARD weight alpha Q(What; Delta) (+ mu when MU) for two bf16 weights.
+template <bool MU = false>
 __device__ __forceinline__ uint32_t hard_pair_bf16(uint32_t w2, const ProducerConst& p) {
   const float x0 = fmaf(bf16lo_to_f32(w2), p.r, p.b);
   const float x1 = fmaf(bf16hi_to_f32(w2), p.r, p.b);
-  const float y0 = fabsf(x0) > p.delta ? copysignf(p.C, x0) : 0.0f;  // Q(x) = sign(x) [|x| > Delta]
-  const float y1 = fabsf(x1) > p.delta ? copysignf(p.C, x1) : 0.0f;
+  float y0 = fabsf(x0) > p.delta ? copysignf(p.C, x0) : 0.0f;  // Q(x) = sign(x) [|x| > Delta]
+  float y1 = fabsf(x1) > p.delta ? copysignf(p.C, x1) : 0.0f;
+  if constexpr (MU) {
+    y0 += p.M;
+    y1 += p.M;
+  }
   return pack_bf16x2(y0, y1);
 }
 
@@ -151,9 +167,11 @@ __device__ __forceinline__ float4 operand_const_vec(const GroupConst& c, float s
   return phase == PHASE_HARD ? make_float4(p.r, p.b, p.delta, p.C) : make_float4(p.A, p.B, p.D, p.C);
 }
 
-// Inverse of operand_const_vec for the transform of `phase`.
-__device__ __forceinline__ ProducerConst producer_const_from(float4 v) {
+// Inverse of operand_const_vec for the transform of `phase`; m is the group offset mu (0
+// when the reconstruction has none).
+__device__ __forceinline__ ProducerConst producer_const_from(float4 v, float m) {
   ProducerConst p;
+  p.M = m;
   p.A = p.r = v.x;
   p.B = p.b = v.y;
   p.D = p.delta = v.z;
@@ -162,54 +180,62 @@ __device__ __forceinline__ ProducerConst producer_const_from(float4 v) {
   return p;
 }
 
-enum : int32_t { XF_COPY = 0, XF_SOFT1 = 1, XF_SOFT2 = 2, XF_HARD = 3 };
+// Element transforms; XF_MU marks the W ~ alpha T + mu forms of SOFT1, SOFT2 and HARD.
+enum : int32_t { XF_COPY = 0, XF_SOFT1 = 1, XF_SOFT2 = 2, XF_HARD = 3, XF_MU = 4 };
 
-// Which element transform a row uses in `phase`.
-__device__ __forceinline__ int32_t transform_kind(const ProducerConst& p, int32_t phase) {
-  if (phase == PHASE_SOFT) return p.one_tanh ? XF_SOFT1 : XF_SOFT2;
-  return phase == PHASE_HARD ? XF_HARD : XF_COPY;
+// Which element transform a row uses in `phase` (`recon` as LayerDev::recon).
+__device__ __forceinline__ int32_t transform_kind(const ProducerConst& p, int32_t phase, int32_t recon) {
+  const int32_t mu = recon ? XF_MU : 0;
+  if (phase == PHASE_SOFT) return (p.one_tanh ? XF_SOFT1 : XF_SOFT2) | mu;
+  return phase == PHASE_HARD ? (XF_HARD | mu) : XF_COPY;
 }
 
 template <int KIND>
 __device__ __forceinline__ uint4 transform_chunk(uint4 v, const ProducerConst& p) {
-  if constexpr (KIND == XF_SOFT1) {
-    v.x = soft_pair_bf16<true>(v.x, p);
-    v.y = soft_pair_bf16<true>(v.y, p);
-    v.z = soft_pair_bf16<true>(v.z, p);
-    v.w = soft_pair_bf16<true>(v.w, p);
-  } else if constexpr (KIND == XF_SOFT2) {
-    v.x = soft_pair_bf16<false>(v.x, p);
-    v.y = soft_pair_bf16<false>(v.y, p);
-    v.z = soft_pair_bf16<false>(v.z, p);
-    v.w = soft_pair_bf16<false>(v.w, p);
-  } else if constexpr (KIND == XF_HARD) {
-    v.x = hard_pair_bf16(v.x, p);
-    v.y = hard_pair_bf16(v.y, p);
-    v.z = hard_pair_bf16(v.z, p);
-    v.w = hard_pair_bf16(v.w, p);
+  constexpr bool MU = (KIND & XF_MU) != 0;
+  constexpr int BASE = KIND & ~XF_MU;
+  if constexpr (BASE == XF_SOFT1) {
+    v.x = soft_pair_bf16<true, MU>(v.x, p);
+    v.y = soft_pair_bf16<true, MU>(v.y, p);
+    v.z = soft_pair_bf16<true, MU>(v.z, p);
+    v.w = soft_pair_bf16<true, MU>(v.w, p);
+  } else if constexpr (BASE == XF_SOFT2) {
+    v.x = soft_pair_bf16<false, MU>(v.x, p);
+    v.y = soft_pair_bf16<false, MU>(v.y, p);
+    v.z = soft_pair_bf16<false, MU>(v.z, p);
+    v.w = soft_pair_bf16<false, MU>(v.w, p);
+  } else if constexpr (BASE == XF_HARD) {
+    v.x = hard_pair_bf16<MU>(v.x, p);
+    v.y = hard_pair_bf16<MU>(v.y, p);
+    v.z = hard_pair_bf16<MU>(v.z, p);
+    v.w = hard_pair_bf16<MU>(v.w, p);
   }
   return v;
 }
 
 // The Eq. 6 operand for one 16-byte chunk of a row (8 bf16 weights of one group).
-__device__ __forceinline__ uint4 transform_chunk_bf16(uint4 v, const ProducerConst& p, int32_t phase) {
-  switch (transform_kind(p, phase)) {
+__device__ __forceinline__ uint4 transform_chunk_bf16(uint4 v, const ProducerConst& p, int32_t phase, int32_t recon) {
+  switch (transform_kind(p, phase, recon)) {
     case XF_SOFT1: return transform_chunk<XF_SOFT1>(v, p);
     case XF_SOFT2: return transform_chunk<XF_SOFT2>(v, p);
     case XF_HARD: return transform_chunk<XF_HARD>(v, p);
+    case XF_SOFT1 | XF_MU: return transform_chunk<XF_SOFT1 | XF_MU>(v, p);
+    case XF_SOFT2 | XF_MU: return transform_chunk<XF_SOFT2 | XF_MU>(v, p);
+    case XF_HARD | XF_MU: return transform_chunk<XF_HARD | XF_MU>(v, p);
     default: return v;
   }
 }
 
 // ---------------------------------------------------------------- fp32 path
 
-// Eq. 5/6 in fp32 with accurate tanh (CUDA-core path).
+// Eq. 5/6 in fp32 with accurate tanh (CUDA-core path); recon adds mu.
 __device__ __forceinline__ float ternary_weight_f32(float w, const GroupConst& c, float s, float inv_2tanh_s,
-                                                    int32_t phase) {
+                                                    int32_t phase, int32_t recon) {
   if (phase == PHASE_TEACHER) return w;
   const float x = what(w, c);
-  if (phase == PHASE_HARD) return c.alpha * hard_q(x, c.delta);
-  return c.alpha * inv_2tanh_s * (tanhf(s * (x - c.delta)) + tanhf(s * (x + c.delta)));
+  const float m = recon ? c.mu : 0.0f;
+  if (phase == PHASE_HARD) return fmaf(c.alpha, hard_q(x, c.delta), m);
+  return fmaf(c.alpha * inv_2tanh_s, tanhf(s * (x - c.delta)) + tanhf(s * (x + c.delta)), m);
 }
 
 // ---------------------------------------------------------------- factor-gradient element
@@ -229,13 +255,16 @@ __device__ __forceinline__ void tanh_sech2(float y, float& t, float& s2) {
 // Running per-group sums of the chain rule (Eq. 3, 5, 6):
 //   smu = sum G f'(What) / k,  salpha = sum G (T - What f'(What)),  sdelta = sum G df/dDelta / k
 // with f' = k (sech^2 a + sech^2 b), df/dDelta = k (sech^2 b - sech^2 a), k = s / (2 tanh s).
+// With mu in the reconstruction (W ~ alpha T + mu) dWq/dmu is 1 - f' instead of -f', and
+// MU accumulates smu = sum G (f' - 1) / k instead (inv_k = 1/k), so that the factor
+// gradient is -alpha0 k smu in both cases.
 struct GradSums {
   float smu, salpha, sdelta;
 };
 
-template <bool FAST = false>
+template <bool FAST = false, bool MU = false>
 __device__ __forceinline__ void grad_element(float G, float w, const GroupConst& c, float s, float inv_2tanh_s,
-                                             int32_t phase, GradSums& acc) {
+                                             int32_t phase, GradSums& acc, float inv_k = 0.0f) {
   const float x = what(w, c);
   float ta, sa, tb, sb;
   tanh_sech2<FAST>(s * (x - c.delta), ta, sa);
@@ -243,7 +272,7 @@ __device__ __forceinline__ void grad_element(float G, float w, const GroupConst&
   const float k = s * inv_2tanh_s;
   const float fp_over_k = sa + sb;
   const float T = (phase == PHASE_SOFT) ? inv_2tanh_s * (ta + tb) : hard_q(x, c.delta);
-  acc.smu = fmaf(G, fp_over_k, acc.smu);
+  acc.smu = fmaf(G, MU ? fp_over_k - inv_k : fp_over_k, acc.smu);
   acc.salpha = fmaf(G, T - x * k * fp_over_k, acc.salpha);
   acc.sdelta = fmaf(G, sb - sa, acc.sdelta);
 }

@@ -324,7 +324,7 @@ __global__ void __launch_bounds__(kThreads) modulate_bf16_kernel(LayerDev L, Ste
     const uint4 v = __ldg(reinterpret_cast<const uint4*>(W + e));
     if (Wq) {
       const ProducerConst pc = producer_const(gc, sc.s, sc.inv_2tanh_s, sc.phase);
-      *reinterpret_cast<uint4*>(Wq + e) = transform_chunk_bf16(v, pc, sc.phase);
+      *reinterpret_cast<uint4*>(Wq + e) = transform_chunk_bf16(v, pc, sc.phase, L.recon);
     }
     if (Tout) {
       const uint32_t w[4] = {v.x, v.y, v.z, v.w};
@@ -351,7 +351,7 @@ __global__ void __launch_bounds__(kThreads) modulate_f32_kernel(LayerDev L, Step
   for (int64_t e = blockIdx.x * (int64_t)kThreads + threadIdx.x; e < n; e += (int64_t)gridDim.x * kThreads) {
     const GroupConst gc = group_const(L, e / L.g);
     const float w = W[e];
-    if (Wq) Wq[e] = ternary_weight_f32(w, gc, sc.s, sc.inv_2tanh_s, sc.phase);
+    if (Wq) Wq[e] = ternary_weight_f32(w, gc, sc.s, sc.inv_2tanh_s, sc.phase, L.recon);
     if (Tout) Tout[e] = (gc.alpha != 0.0f) ? static_cast<int8_t>(hard_q(what(w, gc), gc.delta)) : int8_t(0);
   }
   if (alpha)
@@ -363,7 +363,7 @@ __global__ void __launch_bounds__(kThreads) modulate_f32_kernel(LayerDev L, Step
 // EPT consecutive elements per thread (EPT divides g, so one group), EPT/4 output bytes.
 template <typename T, int EPT>
 __global__ void __launch_bounds__(kThreads) hard_pack_kernel(LayerDev L, uint8_t* __restrict__ codes,
-                                                             float* __restrict__ alpha) {
+                                                             float* __restrict__ alpha, float* __restrict__ mu) {
   const int64_t n = L.N * L.K;
   const int64_t G = n / L.g;
   const T* W = static_cast<const T*>(L.W);
@@ -402,9 +402,12 @@ __global__ void __launch_bounds__(kThreads) hard_pack_kernel(LayerDev L, uint8_t
     else
       codes[e0 / 4] = static_cast<uint8_t>(words[0]);
   }
-  if (alpha)
-    for (int64_t j = blockIdx.x * (int64_t)kThreads + threadIdx.x; j < G; j += (int64_t)gridDim.x * kThreads)
-      alpha[j] = __ldg(L.d_alpha + j) * __ldg(L.alpha0 + j);
+  if (alpha || mu)
+    for (int64_t j = blockIdx.x * (int64_t)kThreads + threadIdx.x; j < G; j += (int64_t)gridDim.x * kThreads) {
+      const GroupConst gc = group_const(L, j);
+      if (alpha) alpha[j] = gc.alpha;
+      if (mu) mu[j] = gc.mu;
+    }
 }
 
 // Warp-cooperative pack for power-of-two g >= 8 V: a warp takes batches of 32 x 8 16-byte
@@ -416,7 +419,8 @@ __global__ void __launch_bounds__(kThreads) hard_pack_kernel(LayerDev L, uint8_t
 template <typename T>
 __global__ void __launch_bounds__(kThreads) hard_pack_warp_kernel(LayerDev L, int32_t log2g,
                                                                   uint8_t* __restrict__ codes,
-                                                                  float* __restrict__ alpha) {
+                                                                  float* __restrict__ alpha,
+                                                                  float* __restrict__ mu) {
   constexpr int V = Vec16<T>::n;
   constexpr int kLoads = 8;
   constexpr int64_t kBatch = 32 * kLoads * V;  // elements per warp batch
@@ -437,7 +441,10 @@ __global__ void __launch_bounds__(kThreads) hard_pack_warp_kernel(LayerDev L, in
         b = gc.b;
         delta = gc.delta;
       }
-      if (alpha && (jl << log2g) >= b0) alpha[jl] = gc.alpha;  // the batch holding the group's start
+      if ((jl << log2g) >= b0) {  // the batch holding the group's start
+        if (alpha) alpha[jl] = gc.alpha;
+        if (mu) mu[jl] = gc.mu;
+      }
     }
     const int first = static_cast<int>(b0 - (j0 << log2g));  // offset of b0 inside group j0
 #pragma unroll
@@ -470,24 +477,32 @@ __global__ void __launch_bounds__(kThreads) hard_pack_warp_kernel(LayerDev L, in
 // ---------------------------------------------------------------- fused-GEMM operand constants
 // operand_const_vec of every group for one schedule point, stored [K/g][N] so that a fused
 // GEMM producer warp (consecutive W rows, one group column) reads contiguous 16-byte
-// vectors.  A 32 x 32 (row x group column) tile goes through shared memory so both the
-// row-major [N][K/g] group arrays and the output are accessed coalesced.
+// vectors; with mu in the reconstruction the group offsets go to op_mu in the same order.
+// A 32 x 32 (row x group column) tile goes through shared memory so both the row-major
+// [N][K/g] group arrays and the output are accessed coalesced.
 constexpr int kConstTile = 32;
 
 __global__ void __launch_bounds__(kConstTile * kConstTile) operand_consts_kernel(LayerDev L, StepScalars sc) {
   __shared__ float4 tile[kConstTile][kConstTile + 1];
+  __shared__ float tile_mu[kConstTile][kConstTile + 1];
   const int64_t gpr = L.groups_per_row;
   const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kConstTile;
   for (int64_t n0 = static_cast<int64_t>(blockIdx.y) * kConstTile; n0 < L.N;
        n0 += static_cast<int64_t>(gridDim.y) * kConstTile) {
     {
       const int64_t n = n0 + threadIdx.y, c = c0 + threadIdx.x;
-      if (n < L.N && c < gpr)
-        tile[threadIdx.y][threadIdx.x] = operand_const_vec(group_const(L, n * gpr + c), sc.s, sc.inv_2tanh_s, sc.phase);
+      if (n < L.N && c < gpr) {
+        const GroupConst gc = group_const(L, n * gpr + c);
+        tile[threadIdx.y][threadIdx.x] = operand_const_vec(gc, sc.s, sc.inv_2tanh_s, sc.phase);
+        tile_mu[threadIdx.y][threadIdx.x] = gc.mu;
+      }
     }
     __syncthreads();
     const int64_t n = n0 + threadIdx.x, c = c0 + threadIdx.y;
-    if (n < L.N && c < gpr) L.op_const[c * L.N + n] = tile[threadIdx.x][threadIdx.y];
+    if (n < L.N && c < gpr) {
+      L.op_const[c * L.N + n] = tile[threadIdx.x][threadIdx.y];
+      if (L.recon) L.op_mu[c * L.N + n] = tile_mu[threadIdx.x][threadIdx.y];
+    }
     __syncthreads();
   }
 }
@@ -695,7 +710,8 @@ cudaError_t launch_recon_loss(const void* Y, const void* Yr, int64_t count, int3
   return cudaGetLastError();
 }
 
-cudaError_t launch_hard_pack(const LayerDev& L, int32_t w_dtype, uint8_t* codes, float* alpha, cudaStream_t st) {
+cudaError_t launch_hard_pack(const LayerDev& L, int32_t w_dtype, uint8_t* codes, float* alpha, float* mu,
+                             cudaStream_t st) {
   const int64_t n = L.N * L.K;
   const int V = w_dtype == 1 ? 8 : 4;
   if (L.g % 64 == 0 && (L.g & (L.g - 1)) == 0 && L.g >= 8 * V) {
@@ -704,27 +720,27 @@ cudaError_t launch_hard_pack(const LayerDev& L, int32_t w_dtype, uint8_t* codes,
     const int64_t batches = (n + 256LL * V - 1) / (256LL * V);
     const int grid = grid_for(batches, kThreads / 32);
     if (w_dtype == 1)
-      hard_pack_warp_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(L, log2g, codes, alpha);
+      hard_pack_warp_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(L, log2g, codes, alpha, mu);
     else
-      hard_pack_warp_kernel<float><<<grid, kThreads, 0, st>>>(L, log2g, codes, alpha);
+      hard_pack_warp_kernel<float><<<grid, kThreads, 0, st>>>(L, log2g, codes, alpha, mu);
   } else if (L.g % 64 == 0) {
     const int grid = grid_for(n / 64, kThreads);
     if (w_dtype == 1)
-      hard_pack_kernel<__nv_bfloat16, 64><<<grid, kThreads, 0, st>>>(L, codes, alpha);
+      hard_pack_kernel<__nv_bfloat16, 64><<<grid, kThreads, 0, st>>>(L, codes, alpha, mu);
     else
-      hard_pack_kernel<float, 64><<<grid, kThreads, 0, st>>>(L, codes, alpha);
+      hard_pack_kernel<float, 64><<<grid, kThreads, 0, st>>>(L, codes, alpha, mu);
   } else if (L.g % 16 == 0) {
     const int grid = grid_for(n / 16, kThreads);
     if (w_dtype == 1)
-      hard_pack_kernel<__nv_bfloat16, 16><<<grid, kThreads, 0, st>>>(L, codes, alpha);
+      hard_pack_kernel<__nv_bfloat16, 16><<<grid, kThreads, 0, st>>>(L, codes, alpha, mu);
     else
-      hard_pack_kernel<float, 16><<<grid, kThreads, 0, st>>>(L, codes, alpha);
+      hard_pack_kernel<float, 16><<<grid, kThreads, 0, st>>>(L, codes, alpha, mu);
   } else {
     const int grid = grid_for(n / 4, kThreads);
     if (w_dtype == 1)
-      hard_pack_kernel<__nv_bfloat16, 4><<<grid, kThreads, 0, st>>>(L, codes, alpha);
+      hard_pack_kernel<__nv_bfloat16, 4><<<grid, kThreads, 0, st>>>(L, codes, alpha, mu);
     else
-      hard_pack_kernel<float, 4><<<grid, kThreads, 0, st>>>(L, codes, alpha);
+      hard_pack_kernel<float, 4><<<grid, kThreads, 0, st>>>(L, codes, alpha, mu);
   }
   return cudaGetLastError();
 }

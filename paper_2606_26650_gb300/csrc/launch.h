@@ -24,7 +24,8 @@ cudaError_t launch_modulate_ternarize(const LayerDev& L, int32_t w_dtype, StepSc
 int recon_loss_blocks(int64_t count);
 cudaError_t launch_recon_loss(const void* Y, const void* Yr, int64_t count, int32_t dtype, int32_t reduction,
                               float* loss_out, void* dY, double* partials, cudaStream_t st);
-cudaError_t launch_hard_pack(const LayerDev& L, int32_t w_dtype, uint8_t* codes, float* alpha, cudaStream_t st);
+cudaError_t launch_hard_pack(const LayerDev& L, int32_t w_dtype, uint8_t* codes, float* alpha, float* mu,
+                             cudaStream_t st);
 // Sums the partial group sums of the dW epilogue ([splits][3][N][K/P]) into the factor
 // gradients and applies the per-group scales.
 cudaError_t launch_grad_reduce(const LayerDev& L, StepScalars sc, const float* partials, int32_t splits, int32_t P,
@@ -44,9 +45,10 @@ struct TcPlan {
   int32_t dw_P;       // partial-sum chunk width (columns)
 };
 TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count);
-// Y [B, N] = X [B, K] (alpha T)^T from 2-bit codes and group scales (bf16 X and Y).
-cudaError_t launch_ternary_infer(const uint8_t* codes, const float* alpha, int64_t N, int64_t K, int32_t g,
-                                 const void* X, int64_t B, void* Y, cudaStream_t st);
+// Y [B, N] = X [B, K] (alpha T + mu)^T from 2-bit codes, group scales and (nullable) group
+// offsets (bf16 X and Y).
+cudaError_t launch_ternary_infer(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K,
+                                 int32_t g, const void* X, int64_t B, void* Y, cudaStream_t st);
 
 // One-thread kernel whose bounded wait runs out after timeout_ns (self-test).
 cudaError_t launch_wait_probe(uint64_t timeout_ns, cudaStream_t st);

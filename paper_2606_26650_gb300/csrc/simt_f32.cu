@@ -29,7 +29,7 @@ __device__ __forceinline__ float w_elem(const SimtArgs& a, int64_t n, int64_t k)
   const float w = static_cast<const float*>(a.L.W)[n * a.L.K + k];
   if (a.sc.phase == PHASE_TEACHER) return w;
   const GroupConst gc = group_const(a.L, n * a.L.groups_per_row + k / a.L.g);
-  return ternary_weight_f32(w, gc, a.sc.s, a.sc.inv_2tanh_s, a.sc.phase);
+  return ternary_weight_f32(w, gc, a.sc.s, a.sc.inv_2tanh_s, a.sc.phase, a.L.recon);
 }
 
 // C[i][j] = sum_c A(i, c) B(j, c) with
@@ -135,9 +135,14 @@ __global__ void __launch_bounds__(kThr) simt_gemm_kernel(SimtArgs a) {
       GradSums e{0.f, 0.f, 0.f};
       if (row_ok && k < L.K) {
         const GroupConst gc = group_const(L, n * L.groups_per_row + k / L.g);
-        if (gc.alpha != 0.0f)
-          grad_element(acc[u][v], static_cast<const float*>(L.W)[n * L.K + k], gc, a.sc.s, a.sc.inv_2tanh_s,
-                       a.sc.phase, e);
+        if (gc.alpha != 0.0f) {
+          const float w = static_cast<const float*>(L.W)[n * L.K + k];
+          if (L.recon)
+            grad_element<false, true>(acc[u][v], w, gc, a.sc.s, a.sc.inv_2tanh_s, a.sc.phase, e,
+                                      1.0f / (a.sc.s * a.sc.inv_2tanh_s));
+          else
+            grad_element(acc[u][v], w, gc, a.sc.s, a.sc.inv_2tanh_s, a.sc.phase, e);
+        }
       }
       if (P >= 16) {  // all 16 tx share the chunk of this v; accumulate over v in the chunk
         run.smu += e.smu;

@@ -503,30 +503,38 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     cur.init(args, cta, row, cluster, 0);
     cur.step(args, cta, row, nclusters, q0);
     ahead = cur;
+    // With mu in the reconstruction the group offset comes from its own [K/g][N] plane.
     float4 raw0{}, raw1{};
+    float m0 = 0.0f, m1 = 0.0f;
     int64_t j0 = -1, j1 = -1;
-    auto request = [&](const OperandRowIter<CG, B_MN>& it, float4& dst, int64_t& jd, const float4& other,
-                       int64_t jo) {
+    const bool with_mu = L.recon != 0;
+    auto request = [&](const OperandRowIter<CG, B_MN>& it, float4& dst, float& dm, int64_t& jd, const float4& other,
+                       float om, int64_t jo) {
       if (transform && it.live(args, num_tiles) && it.valid(args)) {
-        if (jo == it.ci) dst = other;
-        else dst = __ldg(L.op_const + it.ci);
+        if (jo == it.ci) {
+          dst = other;
+          dm = om;
+        } else {
+          dst = __ldg(L.op_const + it.ci);
+          if (with_mu) dm = __ldg(L.op_mu + it.ci);
+        }
         jd = it.ci;
       }
     };
-    request(ahead, raw0, j0, raw1, j1);
+    request(ahead, raw0, m0, j0, raw1, m1, j1);
     ahead.step(args, cta, row, nclusters, STEP);
-    request(ahead, raw1, j1, raw0, j0);
+    request(ahead, raw1, m1, j1, raw0, m0, j0);
     ahead.step(args, cta, row, nclusters, STEP);
     int64_t j_have = -1;
     ProducerConst pc{};
     uint32_t q = q0;
     bool ok = true;
     // One stage: consume `mine` (requested two stages ago), then refill it two stages ahead.
-    auto produce = [&](float4& mine, int64_t& jm, const float4& other, int64_t jo) {
+    auto produce = [&](float4& mine, float& mm, int64_t& jm, const float4& other, float om, int64_t jo) {
       const uint32_t s = q % SW;
       const bool live = transform && cur.valid(args);
       if (live && cur.ci != j_have) {
-        pc = producer_const_from(mine);
+        pc = producer_const_from(mine, mm);
         j_have = cur.ci;
       }
       if (!mbar_wait(raw_w(grp * SW + s), (q / Cfg::kRawPeriod) & 1u, wc)) {
@@ -545,10 +553,13 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
           for (int i = 0; i < CPT; ++i)
             *reinterpret_cast<uint4*>(rowp + (((c_begin + i) ^ (row & 7)) * 16)) = transform_chunk<KIND>(v[i], pc);
         };
-        switch (transform_kind(pc, phase_t)) {
+        switch (transform_kind(pc, phase_t, L.recon)) {
           case XF_SOFT1: run(std::integral_constant<int, XF_SOFT1>{}); break;
           case XF_SOFT2: run(std::integral_constant<int, XF_SOFT2>{}); break;
           case XF_HARD: run(std::integral_constant<int, XF_HARD>{}); break;
+          case XF_SOFT1 | XF_MU: run(std::integral_constant<int, XF_SOFT1 | XF_MU>{}); break;
+          case XF_SOFT2 | XF_MU: run(std::integral_constant<int, XF_SOFT2 | XF_MU>{}); break;
+          case XF_HARD | XF_MU: run(std::integral_constant<int, XF_HARD | XF_MU>{}); break;
           default: break;
         }
         fence_proxy_async_smem();
@@ -561,15 +572,15 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
         mbar_arrive_cluster(leader_full_w0 + 8u * s);
       }
       // Issued after the proxy fence, which would otherwise wait for these loads.
-      request(ahead, mine, jm, other, jo);
+      request(ahead, mine, mm, jm, other, om, jo);
       ahead.step(args, cta, row, nclusters, STEP);
       q += STEP;
       cur.step(args, cta, row, nclusters, STEP);
     };
     while (ok && cur.live(args, num_tiles)) {
-      produce(raw0, j0, raw1, j1);
+      produce(raw0, m0, j0, raw1, m1, j1);
       if (!ok || !cur.live(args, num_tiles)) break;
-      produce(raw1, j1, raw0, j0);
+      produce(raw1, m1, j1, raw0, m0, j0);
     }
   }
 
@@ -721,6 +732,8 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
     const int64_t cpr = L.K / args.P;
     const int64_t plane = L.N * cpr;
     const uint16_t* W = static_cast<const uint16_t*>(L.W);
+    const float k_sc = args.sc.s * args.sc.inv_2tanh_s;
+    const float inv_k = (L.recon && k_sc > 0.0f) ? 1.0f / k_sc : 0.0f;
     uint32_t it = 0;
     for (int t = cluster; t < num_tiles; t += nclusters, ++it) {
       const int split = t / tiles_per_split, r = t % tiles_per_split;
@@ -762,17 +775,22 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
             cur_j = j;
           }
           if (gc.alpha != 0.0f) {
+            auto accumulate = [&](auto mu_tag) {
+              constexpr bool MU = decltype(mu_tag)::value;
 #pragma unroll
-            for (int v = 0; v < 4; ++v) {
-              const uint32_t w4[4] = {wcur[v].x, wcur[v].y, wcur[v].z, wcur[v].w};
+              for (int v = 0; v < 4; ++v) {
+                const uint32_t w4[4] = {wcur[v].x, wcur[v].y, wcur[v].z, wcur[v].w};
 #pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                grad_element<true>(__uint_as_float(rg[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), gc, args.sc.s,
-                                   args.sc.inv_2tanh_s, args.sc.phase, acc);
-                grad_element<true>(__uint_as_float(rg[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), gc, args.sc.s,
-                                   args.sc.inv_2tanh_s, args.sc.phase, acc);
+                for (int e = 0; e < 4; ++e) {
+                  grad_element<true, MU>(__uint_as_float(rg[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), gc, args.sc.s,
+                                         args.sc.inv_2tanh_s, args.sc.phase, acc, inv_k);
+                  grad_element<true, MU>(__uint_as_float(rg[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), gc,
+                                         args.sc.s, args.sc.inv_2tanh_s, args.sc.phase, acc, inv_k);
+                }
               }
-            }
+            };
+            if (L.recon) accumulate(std::true_type{});
+            else accumulate(std::false_type{});
           }
           if (((k + 32) % args.P) == 0 || k + 32 >= L.K) {
             const int64_t idx = n * cpr + k / args.P;

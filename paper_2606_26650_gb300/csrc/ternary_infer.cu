@@ -19,6 +19,9 @@
 // and multiplying by x 4^-i (the activation pre-scaled once per chunk by a power of two,
 // exact for activations above ~1e-30) gives T x exactly.  Pairs of elements go through the
 // packed fp32x2 add and fma.
+//
+// With the group offsets of the W ~ alpha T + mu reconstruction (MU), a row's chunk also adds
+// mu times the chunk's activation sum, which is formed once per chunk for all R rows.
 #include <cstdint>
 
 #include "launch.h"
@@ -63,9 +66,10 @@ __device__ __forceinline__ f32x2 codes_scaled(uint32_t w, int i) {
   return add2(pack2((w & (3u << (2 * i))) | 0x4B000000u, (w & (3u << (2 * (i + 1)))) | 0x4B000000u), neg_magic(i));
 }
 
-template <int R>
+template <int R, bool MU>
 __global__ void __launch_bounds__(kInferThreads) ternary_gemv_kernel(const uint8_t* __restrict__ codes,
-                                                                     const float* __restrict__ alpha, int64_t N,
+                                                                     const float* __restrict__ alpha,
+                                                                     const float* __restrict__ mu, int64_t N,
                                                                      int64_t K, int32_t g,
                                                                      const uint16_t* __restrict__ X, int64_t B,
                                                                      uint16_t* __restrict__ Y) {
@@ -83,16 +87,18 @@ __global__ void __launch_bounds__(kInferThreads) ternary_gemv_kernel(const uint8
       for (int r = 0; r < R; ++r) acc[r] = 0.0f;
       for (int64_t c = lane; c < chunks; c += 32) {
         uint4 w[R];
-        float a[R];
+        float a[R], m[R];
 #pragma unroll
         for (int r = 0; r < R; ++r) {
           const int64_t n = n0 + r < N ? n0 + r : N - 1;  // rows past N repeat the last (not stored)
           w[r] = __ldg(reinterpret_cast<const uint4*>(codes + n * (K / 4)) + c);
           a[r] = __ldg(alpha + n * gpr + (c * 64) / g);
+          if constexpr (MU) m[r] = __ldg(mu + n * gpr + (c * 64) / g);
         }
         f32x2 p[R];
 #pragma unroll
         for (int r = 0; r < R; ++r) p[r] = 0ull;
+        f32x2 xsum = 0ull;  // activation sum of the chunk (MU only)
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
           const uint4* xp = reinterpret_cast<const uint4*>(X + b * K + c * 64 + q * 16);
@@ -106,6 +112,8 @@ __global__ void __launch_bounds__(kInferThreads) ternary_gemv_kernel(const uint8
             const float s0 = __uint_as_float(static_cast<uint32_t>(127 - 2 * i) << 23);
             const float s1 = __uint_as_float(static_cast<uint32_t>(127 - 2 * (i + 1)) << 23);
             xs[e2] = pack2(__float_as_uint(bf16lo_to_f32(xw[e2]) * s0), __float_as_uint(bf16hi_to_f32(xw[e2]) * s1));
+            if constexpr (MU)
+              xsum = add2(xsum, pack2(__float_as_uint(bf16lo_to_f32(xw[e2])), __float_as_uint(bf16hi_to_f32(xw[e2]))));
           }
 #pragma unroll
           for (int r = 0; r < R; ++r) {
@@ -118,11 +126,14 @@ __global__ void __launch_bounds__(kInferThreads) ternary_gemv_kernel(const uint8
             }
           }
         }
+        float xs_lo = 0.0f, xs_hi = 0.0f;
+        if constexpr (MU) unpack2(xsum, xs_lo, xs_hi);
 #pragma unroll
         for (int r = 0; r < R; ++r) {
           float lo, hi;
           unpack2(p[r], lo, hi);
           acc[r] = fmaf(a[r], lo + hi, acc[r]);
+          if constexpr (MU) acc[r] = fmaf(m[r], xs_lo + xs_hi, acc[r]);
         }
 
       }
@@ -142,26 +153,31 @@ __global__ void __launch_bounds__(kInferThreads) ternary_gemv_kernel(const uint8
 }
 
 template <int R>
-cudaError_t launch_gemv(const uint8_t* codes, const float* alpha, int64_t N, int64_t K, int32_t g,
+cudaError_t launch_gemv(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K, int32_t g,
                         const uint16_t* X, int64_t B, uint16_t* Y, cudaStream_t st) {
   const int64_t warps = (N + R - 1) / R;
   int64_t blocks = (warps + kInferThreads / 32 - 1) / (kInferThreads / 32);
   if (blocks > 152 * 16) blocks = 152 * 16;
-  ternary_gemv_kernel<R><<<static_cast<int>(blocks), kInferThreads, 0, st>>>(codes, alpha, N, K, g, X, B, Y);
+  if (mu)
+    ternary_gemv_kernel<R, true><<<static_cast<int>(blocks), kInferThreads, 0, st>>>(codes, alpha, mu, N, K, g, X,
+                                                                                    B, Y);
+  else
+    ternary_gemv_kernel<R, false><<<static_cast<int>(blocks), kInferThreads, 0, st>>>(codes, alpha, nullptr, N, K, g,
+                                                                                     X, B, Y);
   return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_ternary_infer(const uint8_t* codes, const float* alpha, int64_t N, int64_t K, int32_t g,
-                                 const void* X, int64_t B, void* Y, cudaStream_t st) {
+cudaError_t launch_ternary_infer(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K,
+                                 int32_t g, const void* X, int64_t B, void* Y, cudaStream_t st) {
   const uint16_t* x = static_cast<const uint16_t*>(X);
   uint16_t* y = static_cast<uint16_t*>(Y);
   // Rows per warp by the layer's height: enough warps to fill the GPU, as few activation
   // reads per weight as that allows.
-  if (N >= 8192) return launch_gemv<4>(codes, alpha, N, K, g, x, B, y, st);
-  if (N >= 2048) return launch_gemv<2>(codes, alpha, N, K, g, x, B, y, st);
-  return launch_gemv<1>(codes, alpha, N, K, g, x, B, y, st);
+  if (N >= 8192) return launch_gemv<4>(codes, alpha, mu, N, K, g, x, B, y, st);
+  if (N >= 2048) return launch_gemv<2>(codes, alpha, mu, N, K, g, x, B, y, st);
+  return launch_gemv<1>(codes, alpha, mu, N, K, g, x, B, y, st);
 }
 
 }  // namespace catq

@@ -49,9 +49,9 @@ def to_host(t) -> np.ndarray:
     return t.cpu().numpy()
 
 
-def gpu_step(W, X, g, fac, thr, phase, s, dtype, device, with_dx=True):
-    """Group stats, teacher and phase forward, loss, backward and hard pack on the GPU.
-    Returns a dict of host arrays."""
+def gpu_step(W, X, g, fac, thr, phase, s, dtype, device, with_dx=True, recon=0):
+    """Group stats, teacher and phase forward, loss, backward and hard pack on the GPU
+    (`recon` 1: the W ~ alpha T + mu reconstruction).  Returns a dict of host arrays."""
     import torch
 
     from paper_2606_26650_gb300 import catq as C
@@ -59,7 +59,8 @@ def gpu_step(W, X, g, fac, thr, phase, s, dtype, device, with_dx=True):
     N = W.shape[0]
     G = N * K // g
     Wt, Xt = to_device(W, dtype, device), to_device(X, dtype, device)
-    layer = C.Layer.create(Wt, g, *(torch.from_numpy(np.asarray(f, np.float32)).to(device) for f in fac))
+    layer = C.Layer.create(Wt, g, *(torch.from_numpy(np.asarray(f, np.float32)).to(device) for f in fac),
+                           recon=recon)
     C.catq_group_stats(layer, thr)
     tdt = Wt.dtype
     Yref = torch.empty(M, N, dtype=tdt, device=device)
@@ -76,13 +77,14 @@ def gpu_step(W, X, g, fac, thr, phase, s, dtype, device, with_dx=True):
     C.catq_soft_ternary_linear_bwd(layer, C.schedule(phase, s), Xt, dY, dX, *gr, wsb)
     codes = torch.empty(N * K // 4, dtype=torch.uint8, device=device)
     alpha = torch.empty(G, dtype=torch.float32, device=device)
-    C.catq_hard_ternarize_pack(layer, codes, alpha)
+    mu = torch.empty(G, dtype=torch.float32, device=device)
+    C.catq_hard_ternarize_pack(layer, codes, alpha, mu)
     torch.cuda.synchronize()
     assert C.catq_device_status() == 0
     out = dict(mu0=to_host(layer.mu0), alpha0=to_host(layer.alpha0), delta0=to_host(layer.delta0),
                Y_ref=to_host(Yref), Y=to_host(Y), loss=float(loss.item()), dY=to_host(dY),
                g_dmu=to_host(gr[0]), g_dalpha=to_host(gr[1]), g_ddelta=to_host(gr[2]),
-               codes=to_host(codes), alpha=to_host(alpha))
+               codes=to_host(codes), alpha=to_host(alpha), mu=to_host(mu))
     if with_dx:
         out["dX"] = to_host(dX)
     return out

@@ -24,16 +24,16 @@ def test_exports_every_declared_symbol(lib):
 
 
 def test_status_strings_and_version(lib):
-    assert lib.catq_abi_version() == 2
+    assert lib.catq_abi_version() == 3
     for code, name in C.STATUS.items():
         assert lib.catq_status_string(code).decode() == name
     assert lib.catq_status_string(99).decode() == "CATQ_ERR_UNKNOWN"
 
 
-def _layer(N=64, K=256, g=128, dtype=C.BF16, W=16, stats=32, op_const=65536):
+def _layer(N=64, K=256, g=128, dtype=C.BF16, W=16, stats=32, op_const=65536, recon=C.RECON_ALPHA_T, reserved=0):
     """A layer struct with fake (never dereferenced) device addresses."""
     return C.catq_layer(N, K, g, dtype, W, stats, stats + 1024, stats + 2048, stats + 4096, stats + 8192,
-                        stats + 16384, op_const)
+                        stats + 16384, op_const, recon, reserved)
 
 
 def _stats(lib, layer, thr=0):
@@ -51,6 +51,8 @@ def test_layer_validation(lib):
     assert _stats(lib, _layer(W=24)) == 4                    # misaligned W
     assert _stats(lib, _layer(), thr=5) == 1                 # bad threshold rule
     assert _stats(lib, _layer(N=0)) == 2
+    assert _stats(lib, _layer(recon=2)) == 1                 # unknown reconstruction
+    assert _stats(lib, _layer(reserved=1)) == 1              # reserved field must be 0
 
 
 def test_call_validation(lib):
@@ -87,15 +89,16 @@ def test_call_validation(lib):
     assert loss(16, 16, 1000, C.BF16, 0, 16, None, 256, ws - 256, None) == 9
     assert loss(16, 24, 1000, C.BF16, 0, 16, None, 256, ws, None) == 4
     pack = lib.catq_hard_ternarize_pack
-    assert pack(ctypes.byref(L), None, None, None) == 1
+    assert pack(ctypes.byref(L), None, None, None, None) == 1
     assert lib.catq_device_status(None, None) == 1
     infer = lib.catq_ternary_infer
-    assert infer(None, 32, 64, 256, 128, 16, 1, C.BF16, 16, None) == 1       # null codes
-    assert infer(16, 32, 64, 256, 128, 16, 1, C.F32, 16, None) == 3           # bf16 only
-    assert infer(16, 32, 64, 256, 32, 16, 1, C.BF16, 16, None) == 2           # g % 64 != 0
-    assert infer(16, 32, 64, 250, 128, 16, 1, C.BF16, 16, None) == 2          # g does not divide K
-    assert infer(16, 32, 64, 256, 128, 16, 0, C.BF16, 16, None) == 0          # B == 0: no-op
-    assert infer(24, 32, 64, 256, 128, 16, 1, C.BF16, 16, None) == 4          # misaligned codes
-    assert infer(16, 32, 64, 256, 128, 16, 1, C.BF16, None, None) == 1        # null Y
+    assert infer(None, 32, None, 64, 256, 128, 16, 1, C.BF16, 16, None) == 1       # null codes
+    assert infer(16, 32, None, 64, 256, 128, 16, 1, C.F32, 16, None) == 3           # bf16 only
+    assert infer(16, 32, None, 64, 256, 32, 16, 1, C.BF16, 16, None) == 2           # g % 64 != 0
+    assert infer(16, 32, None, 64, 250, 128, 16, 1, C.BF16, 16, None) == 2          # g does not divide K
+    assert infer(16, 32, None, 64, 256, 128, 16, 0, C.BF16, 16, None) == 0          # B == 0: no-op
+    assert infer(24, 32, None, 64, 256, 128, 16, 1, C.BF16, 16, None) == 4          # misaligned codes
+    assert infer(16, 32, 34, 64, 256, 128, 16, 1, C.BF16, 16, None) == 4            # misaligned mu
+    assert infer(16, 32, None, 64, 256, 128, 16, 1, C.BF16, None, None) == 1        # null Y
     assert lib.catq_selftest_wait_timeout(10, None) == 1              # below 1 us
     assert lib.catq_selftest_wait_timeout(2_000_000_000, None) == 1   # above 1 s
