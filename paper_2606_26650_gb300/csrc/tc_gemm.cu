@@ -252,7 +252,9 @@ struct OperandRowIter {
   }
 };
 
-template <int CG, bool B_MN, int PAIRS>
+// MU: the layer reconstructs W ~ alpha T + mu (a separate instantiation, so the W ~ alpha T
+// kernel carries none of its work).
+template <int CG, bool B_MN, int PAIRS, bool MU>
 __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     fused_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
                       const FusedArgs args) {
@@ -507,7 +509,7 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     float4 raw0{}, raw1{};
     float m0 = 0.0f, m1 = 0.0f;
     int64_t j0 = -1, j1 = -1;
-    const bool with_mu = L.recon != 0;
+    constexpr bool with_mu = MU;
     auto request = [&](const OperandRowIter<CG, B_MN>& it, float4& dst, float& dm, int64_t& jd, const float4& other,
                        float om, int64_t jo) {
       if (transform && it.live(args, num_tiles) && it.valid(args)) {
@@ -553,13 +555,11 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
           for (int i = 0; i < CPT; ++i)
             *reinterpret_cast<uint4*>(rowp + (((c_begin + i) ^ (row & 7)) * 16)) = transform_chunk<KIND>(v[i], pc);
         };
-        switch (transform_kind(pc, phase_t, L.recon)) {
-          case XF_SOFT1: run(std::integral_constant<int, XF_SOFT1>{}); break;
-          case XF_SOFT2: run(std::integral_constant<int, XF_SOFT2>{}); break;
-          case XF_HARD: run(std::integral_constant<int, XF_HARD>{}); break;
-          case XF_SOFT1 | XF_MU: run(std::integral_constant<int, XF_SOFT1 | XF_MU>{}); break;
-          case XF_SOFT2 | XF_MU: run(std::integral_constant<int, XF_SOFT2 | XF_MU>{}); break;
-          case XF_HARD | XF_MU: run(std::integral_constant<int, XF_HARD | XF_MU>{}); break;
+        constexpr int kMu = MU ? XF_MU : 0;
+        switch (transform_kind(pc, phase_t, MU ? 1 : 0)) {
+          case XF_SOFT1 | kMu: run(std::integral_constant<int, XF_SOFT1 | kMu>{}); break;
+          case XF_SOFT2 | kMu: run(std::integral_constant<int, XF_SOFT2 | kMu>{}); break;
+          case XF_HARD | kMu: run(std::integral_constant<int, XF_HARD | kMu>{}); break;
           default: break;
         }
         fence_proxy_async_smem();
@@ -607,7 +607,7 @@ __global__ void wait_probe_kernel(const WaitCtl wc) {
 
 // ============================================================================ dW kernel
 
-template <int CG>
+template <int CG, bool MU>
 __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
     dw_kernel(const __grid_constant__ CUtensorMap tmDY, const __grid_constant__ CUtensorMap tmX, const DwArgs args) {
   using Cfg = DwCfg<CG>;
@@ -733,7 +733,7 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
     const int64_t plane = L.N * cpr;
     const uint16_t* W = static_cast<const uint16_t*>(L.W);
     const float k_sc = args.sc.s * args.sc.inv_2tanh_s;
-    const float inv_k = (L.recon && k_sc > 0.0f) ? 1.0f / k_sc : 0.0f;
+    const float inv_k = (MU && k_sc > 0.0f) ? 1.0f / k_sc : 0.0f;
     uint32_t it = 0;
     for (int t = cluster; t < num_tiles; t += nclusters, ++it) {
       const int split = t / tiles_per_split, r = t % tiles_per_split;
@@ -775,22 +775,17 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
             cur_j = j;
           }
           if (gc.alpha != 0.0f) {
-            auto accumulate = [&](auto mu_tag) {
-              constexpr bool MU = decltype(mu_tag)::value;
 #pragma unroll
-              for (int v = 0; v < 4; ++v) {
-                const uint32_t w4[4] = {wcur[v].x, wcur[v].y, wcur[v].z, wcur[v].w};
+            for (int v = 0; v < 4; ++v) {
+              const uint32_t w4[4] = {wcur[v].x, wcur[v].y, wcur[v].z, wcur[v].w};
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                  grad_element<true, MU>(__uint_as_float(rg[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), gc, args.sc.s,
-                                         args.sc.inv_2tanh_s, args.sc.phase, acc, inv_k);
-                  grad_element<true, MU>(__uint_as_float(rg[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), gc,
-                                         args.sc.s, args.sc.inv_2tanh_s, args.sc.phase, acc, inv_k);
-                }
+              for (int e = 0; e < 4; ++e) {
+                grad_element<true, MU>(__uint_as_float(rg[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), gc, args.sc.s,
+                                       args.sc.inv_2tanh_s, args.sc.phase, acc, inv_k);
+                grad_element<true, MU>(__uint_as_float(rg[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), gc, args.sc.s,
+                                       args.sc.inv_2tanh_s, args.sc.phase, acc, inv_k);
               }
-            };
-            if (L.recon) accumulate(std::true_type{});
-            else accumulate(std::false_type{});
+            }
           }
           if (((k + 32) % args.P) == 0 || k + 32 >= L.K) {
             const int64_t idx = n * cpr + k / args.P;
@@ -940,7 +935,7 @@ int max_active_clusters(Kern kern, int cluster_ctas, int threads, int smem, int 
 // CTA pairs (512 rows) from 512 rows, single CTAs below.
 int fused_variant_for(int64_t M) { return M >= 1024 ? 4 : (M >= 512 ? 2 : 1); }
 
-template <int CG, bool B_MN, int PAIRS>
+template <int CG, bool B_MN, int PAIRS, bool MU>
 cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t M, int64_t depth, void* C,
                       int64_t ncols, cudaStream_t st) {
   using Cfg = FusedCfg<CG, PAIRS>;
@@ -964,7 +959,7 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
   args.num_k_blocks = static_cast<int32_t>((depth + BK - 1) / BK);
   args.group_m = std::min(4, args.num_m_tiles);
   args.wc = make_wait_ctl(d);
-  auto kern = fused_gemm_kernel<CG, B_MN, PAIRS>;
+  auto kern = fused_gemm_kernel<CG, B_MN, PAIRS, MU>;
   const int tiles = args.num_m_tiles * args.num_n_tiles;
   const int fit = max_active_clusters(kern, Cfg::kClusterCtas, Cfg::kThreads, Cfg::kSmemBytes,
                                       d.sm_count / Cfg::kClusterCtas);
@@ -974,7 +969,7 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
                            st, params);
 }
 
-template <int CG>
+template <int CG, bool MU>
 cudaError_t run_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M, const TcPlan& plan,
                    float* part, cudaStream_t st) {
   using Cfg = DwCfg<CG>;
@@ -998,7 +993,22 @@ cudaError_t run_dw(const LayerDev& L, StepScalars sc, const void* X, const void*
   const int tiles = args.num_n_tiles * args.num_k_tiles * args.splits;
   const int clusters = std::min(tiles, d.sm_count / CG);
   void* params[3] = {&tdy, &tx, &args};
-  return launch_persistent(dw_kernel<CG>, CG, clusters * CG, Cfg::kThreads, Cfg::kSmemBytes, st, params);
+  return launch_persistent(dw_kernel<CG, MU>, CG, clusters * CG, Cfg::kThreads, Cfg::kSmemBytes, st, params);
+}
+
+// Tile shape by M, and the W ~ alpha T + mu instantiation for such layers outside TEACHER.
+template <bool B_MN>
+cudaError_t dispatch_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t M, int64_t depth, void* C,
+                           int64_t ncols, cudaStream_t st) {
+  const bool mu = L.recon != 0 && sc.phase != PHASE_TEACHER;
+  switch (fused_variant_for(M) * 2 + (mu ? 1 : 0)) {
+    case 8: return run_fused<2, B_MN, 2, false>(L, sc, A, M, depth, C, ncols, st);
+    case 9: return run_fused<2, B_MN, 2, true>(L, sc, A, M, depth, C, ncols, st);
+    case 4: return run_fused<2, B_MN, 1, false>(L, sc, A, M, depth, C, ncols, st);
+    case 5: return run_fused<2, B_MN, 1, true>(L, sc, A, M, depth, C, ncols, st);
+    case 3: return run_fused<1, B_MN, 1, true>(L, sc, A, M, depth, C, ncols, st);
+    default: return run_fused<1, B_MN, 1, false>(L, sc, A, M, depth, C, ncols, st);
+  }
 }
 
 }  // namespace
@@ -1032,11 +1042,7 @@ cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int6
     const cudaError_t e = launch_operand_consts(L, sc, st);
     if (e != cudaSuccess) return e;
   }
-  switch (fused_variant_for(M)) {
-    case 4: return run_fused<2, false, 2>(L, sc, X, M, L.K, Y, L.N, st);
-    case 2: return run_fused<2, false, 1>(L, sc, X, M, L.K, Y, L.N, st);
-    default: return run_fused<1, false, 1>(L, sc, X, M, L.K, Y, L.N, st);
-  }
+  return dispatch_fused<false>(L, sc, X, M, L.K, Y, L.N, st);
 }
 
 cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int64_t M, void* dX, cudaStream_t st) {
@@ -1044,11 +1050,7 @@ cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int6
     const cudaError_t e = launch_operand_consts(L, sc, st);
     if (e != cudaSuccess) return e;
   }
-  switch (fused_variant_for(M)) {
-    case 4: return run_fused<2, true, 2>(L, sc, dY, M, L.N, dX, L.K, st);
-    case 2: return run_fused<2, true, 1>(L, sc, dY, M, L.N, dX, L.K, st);
-    default: return run_fused<1, true, 1>(L, sc, dY, M, L.N, dX, L.K, st);
-  }
+  return dispatch_fused<true>(L, sc, dY, M, L.N, dX, L.K, st);
 }
 
 cudaError_t launch_wait_probe(uint64_t timeout_ns, cudaStream_t st) {
@@ -1062,8 +1064,12 @@ cudaError_t launch_wait_probe(uint64_t timeout_ns, cudaStream_t st) {
 
 cudaError_t launch_tc_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M,
                          const TcPlan& plan, float* partials, cudaStream_t st) {
-  if (plan.dw_cg == 2) return run_dw<2>(L, sc, X, dY, M, plan, partials, st);
-  return run_dw<1>(L, sc, X, dY, M, plan, partials, st);
+  if (L.recon) {
+    if (plan.dw_cg == 2) return run_dw<2, true>(L, sc, X, dY, M, plan, partials, st);
+    return run_dw<1, true>(L, sc, X, dY, M, plan, partials, st);
+  }
+  if (plan.dw_cg == 2) return run_dw<2, false>(L, sc, X, dY, M, plan, partials, st);
+  return run_dw<1, false>(L, sc, X, dY, M, plan, partials, st);
 }
 
 cudaError_t read_and_clear_device_status(int32_t* out) {
