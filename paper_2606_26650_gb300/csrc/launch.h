@@ -50,6 +50,11 @@ TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count);
 cudaError_t launch_ternary_infer(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K,
                                  int32_t g, const void* X, int64_t B, void* Y, cudaStream_t st);
 
+// Wait control (abort word, status word, epoch, time limit) for one launch of a kernel with
+// bounded waits; false when the device's status words are unavailable.
+struct WaitCtl;
+bool launch_wait_ctl(WaitCtl* out);
+
 // One-thread kernel whose bounded wait runs out after timeout_ns (self-test).
 cudaError_t launch_wait_probe(uint64_t timeout_ns, cudaStream_t st);
 

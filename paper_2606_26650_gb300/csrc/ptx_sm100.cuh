@@ -99,7 +99,7 @@ struct WaitCtl {
 
 __device__ __forceinline__ bool aborted(const WaitCtl& w) { return *w.abort_word == w.epoch; }
 
-__device__ __noinline__ void signal_timeout(const WaitCtl& w) {
+static __device__ __noinline__ void signal_timeout(const WaitCtl& w) {
   atomicCAS(w.status_word, 0, 6 /* CATQ_ERR_TIMEOUT */);
   *w.abort_word = w.epoch;
   __threadfence();
@@ -216,6 +216,15 @@ __device__ __forceinline__ void umma_commit_pair_mask(uint32_t bar, uint16_t cta
   asm volatile(
       "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
       "h"(cta_mask)
+      : "memory");
+}
+
+// Bulk copy of `bytes` (multiple of 16, both addresses 16-byte aligned) from global memory into
+// this CTA's shared memory; completion is signalled as transaction bytes on `bar`.
+__device__ __forceinline__ void bulk_load_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar)
       : "memory");
 }
 

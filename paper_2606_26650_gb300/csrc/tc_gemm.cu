@@ -1053,6 +1053,13 @@ cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int6
   return dispatch_fused<true>(L, sc, dY, M, L.N, dX, L.K, st);
 }
 
+bool launch_wait_ctl(WaitCtl* out) {
+  DeviceInfo& d = device_info();
+  if (!d.ok) return false;
+  *out = make_wait_ctl(d);
+  return true;
+}
+
 cudaError_t launch_wait_probe(uint64_t timeout_ns, cudaStream_t st) {
   DeviceInfo& d = device_info();
   if (!d.ok) return cudaErrorInvalidDevice;
