@@ -72,15 +72,40 @@ __host__ __device__ constexpr uint32_t pos_inv(int p) {
   return pos_i(p) == 0 ? 0x3F803F80u : (pos_i(p) == 1 ? 0x3E803E80u : 0x3D803D80u);
 }
 
-// The three shifted copies of a code word.
+// The three shifted copies of a code word, and the magic constant held in a register, so
+// that mask-and-insert is one three-input logic operation (a & mask | magic).
 struct Shifted {
   uint32_t t[3];
+  uint32_t magic;
 };
-__device__ __forceinline__ Shifted shifted(uint32_t w) { return Shifted{{w, w >> 6, w >> 12}}; }
+__device__ __forceinline__ Shifted shifted(uint32_t w, uint32_t magic) {
+  return Shifted{{w, w >> 6, w >> 12}, magic};
+}
 
 template <int P>
 __device__ __forceinline__ uint32_t code_pair(const Shifted& s) {
-  return (s.t[pos_shift(P)] & pos_mask(P)) | kMagic;
+  uint32_t d;
+  asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(d) : "r"(s.t[pos_shift(P)]), "n"(pos_mask(P)), "r"(s.magic));
+  return d;
+}
+
+// An opaque copy of the magic constant (kept in a register instead of being folded into
+// each logic operation as a second immediate).
+__device__ __forceinline__ uint32_t magic_reg() {
+  uint32_t m;
+  asm volatile("mov.b32 %0, %1;" : "=r"(m) : "n"(kMagic));
+  return m;
+}
+
+// Four 16-byte loads of read-only global data under a predicate (no branch); zeros when
+// the predicate is false.
+__device__ __forceinline__ uint4 ldg_pred(const uint4* p, bool pred) {
+  uint4 v = make_uint4(0u, 0u, 0u, 0u);
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.u32 p, %4, 0;\n @p ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%5];\n}"
+      : "+r"(v.x), "+r"(v.y), "+r"(v.z), "+r"(v.w)
+      : "r"(static_cast<uint32_t>(pred)), "l"(p));
+  return v;
 }
 
 // Activation pair (x[p], x[p + 8]) of 16 consecutive bf16 (h0 = elements 0..7, h1 = 8..15),
@@ -124,7 +149,7 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
 // the fragment reads (four lanes per row, eight rows per instruction) are free of bank
 // conflicts.
 template <int R, int VW, bool MU>
-__global__ void __launch_bounds__(kMmaWarps * 32) ternary_mma_kernel(const uint8_t* __restrict__ codes,
+__global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const uint8_t* __restrict__ codes,
                                                                      const float* __restrict__ alpha,
                                                                      const float* __restrict__ mu, int64_t N,
                                                                      int64_t K, int32_t g, int64_t KS,
@@ -152,6 +177,7 @@ __global__ void __launch_bounds__(kMmaWarps * 32) ternary_mma_kernel(const uint8
   }
   __syncthreads();
   uint32_t uses = 0;  // completed phases of both barriers, bit b for barrier b (CTA-uniform)
+  const uint32_t magic = magic_reg();
 
   // Warp 0 issues the bulk copies of slab `slab` of rows n0.. into buffer `buf`.
   auto issue = [&](int64_t n0, int64_t slab, int buf) {
@@ -216,12 +242,10 @@ __global__ void __launch_bounds__(kMmaWarps * 32) ternary_mma_kernel(const uint8
         auto load_x = [&](int32_t sc, uint4 (&xv)[2 * VW]) {
           const uint4* xp = reinterpret_cast<const uint4*>(xrow + k0 + sc * 64 * VW + 16 * VW * q);
 #pragma unroll
-          for (int i = 0; i < 2 * VW; ++i) xv[i] = tok_ok ? __ldg(xp + i) : make_uint4(0u, 0u, 0u, 0u);
+          for (int i = 0; i < 2 * VW; ++i) xv[i] = ldg_pred(xp + i, tok_ok);
         };
-        uint4 xv[2 * VW], xn[2 * VW];
-        if (lo < hi) load_x(lo, xv);
-        for (int32_t sc = lo; sc < hi; ++sc) {
-          if (sc + 1 < hi) load_x(sc + 1, xn);  // in flight during this super-chunk's MMAs
+        // one super-chunk: this thread's code words from shared memory, its activations xv
+        auto step = [&](int32_t sc, const uint4 (&xv)[2 * VW]) {
           const uint32_t woff = static_cast<uint32_t>((sc * 4 * VW + VW * q) * 4);
           uint32_t cw[R][2][VW];  // the thread's code words of rows gid and gid + 8 of each tile
 #pragma unroll
@@ -249,7 +273,7 @@ __global__ void __launch_bounds__(kMmaWarps * 32) ternary_mma_kernel(const uint8
             mma_16816(da, pos_corr(6), pos_unit(6), pos_corr(7), pos_unit(7), xb[6], xb[7]);
 #pragma unroll
             for (int r = 0; r < R; ++r) {
-              const Shifted s0 = shifted(cw[r][0][v]), s1 = shifted(cw[r][1][v]);
+              const Shifted s0 = shifted(cw[r][0][v], magic), s1 = shifted(cw[r][1][v], magic);
               word_mma<0>(d[r], s0, s1, xb);
               word_mma<1>(d[r], s0, s1, xb);
               word_mma<2>(d[r], s0, s1, xb);
@@ -281,8 +305,16 @@ __global__ void __launch_bounds__(kMmaWarps * 32) ternary_mma_kernel(const uint8
               left = sc_per_group;
             }
           }
-#pragma unroll
-          for (int i = 0; i < 2 * VW; ++i) xv[i] = xn[i];
+        };
+        // activations one super-chunk ahead, in two alternating register sets
+        uint4 xa[2 * VW], xc[2 * VW];
+        if (lo < hi) load_x(lo, xa);
+        for (int32_t sc = lo; sc < hi; sc += 2) {
+          if (sc + 1 < hi) load_x(sc + 1, xc);
+          step(sc, xa);
+          if (sc + 1 >= hi) break;
+          if (sc + 2 < hi) load_x(sc + 2, xa);
+          step(sc + 1, xc);
         }
         __syncthreads();  // every warp is done with this buffer
         if (warp == 0 && slab + 2 < nslabs) issue(n0, slab + 2, buf);
