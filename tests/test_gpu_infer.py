@@ -26,6 +26,8 @@ def device():
     (520, 192, 64, 8),        # ragged N, a single full pass of 8 rows
     (64, 512, 512, 11),       # channel-wise groups, two passes (8 + 3)
     (4096, 14336, 128, 2),    # the Llama-3-8B-shaped down_proj
+    (328, 1024, 128, 5),      # a partial 128-row block, K split over two CTAs
+    (256, 2048, 128, 19),     # two passes over 16 token rows
 ])
 def test_ternary_infer_matches_oracle(device, N, K, g, B):
     import torch
