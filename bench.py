@@ -547,7 +547,7 @@ def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20, with_m
     gbs = nbytes / (ms * 1e-3) / 1e9
     del graph, layers
     torch.cuda.empty_cache()
-    return {"kernel": "ternary_gemv_kernel (catq_ternary_infer)", "blocks": blocks, "token_rows": rows,
+    return {"kernel": "ternary_mma_kernel (catq_ternary_infer)", "blocks": blocks, "token_rows": rows,
             "launches_per_step": blocks * len(wl.linears), "bytes_per_step": nbytes, "us_per_step": ms * 1e3,
             "value": gbs, "unit": "GB/s", "peak": peaks["hbm"], "frac_of_hbm": gbs / peaks["hbm"],
             "steps": steps, "graph": True, "with_mu": with_mu}
