@@ -534,3 +534,45 @@ def test_ternary_infer_with_mu_is_the_hard_forward_with_mu():
     Y = O.ternary_infer(O.pack_codes(T), alpha, N, K, g, X, mu=mu)
     Wq = O.ternary_weight(W, g, stats, fac, O.PHASE_HARD, 30.0, with_mu=True)[0]
     np.testing.assert_allclose(Y, O.linear_fwd(X, Wq), rtol=1e-12, atol=1e-12)
+
+
+# ---------------------------------------------------------------- direct learning (Fig. fig:error)
+
+@pytest.mark.parametrize("s", [0.625, 30.0])
+def test_direct_learning_is_a_reparametrization_of_the_modulation(s):
+    """Learning alpha and a weight-space threshold Delta_W directly (the comparison of
+    Fig. fig:error), from a static rule's statistics (mu0 = 0), is the modulation with
+    d_mu = 0 under alpha = d_alpha alpha0, Delta_W = alpha d_delta Delta0: the forward is the
+    same function, and the direct parameters' gradients follow from the factor gradients by
+    the chain rule.  Checked against central differences of the direct parametrisation."""
+    W, X, g, _, fac = _tiny(seed=5)
+    stats = O.group_stats(W, g, O.THR_ABSMEAN)
+    mu0, alpha0, delta0 = stats
+    assert not mu0.any()
+    G = alpha0.size
+    zero = np.zeros(G)
+    a_d = fac[1] * alpha0                      # direct scale
+    D_d = a_d * fac[2] * delta0                # direct threshold in W units
+    Y_ref = O.linear_fwd(X, W)
+
+    def loss_direct(a, D):
+        f = (zero, a / alpha0, (D / a) / delta0)
+        return O.recon_loss(O.linear_fwd(X, O.ternary_weight(W, g, stats, f, O.PHASE_SOFT, s)[0]), Y_ref)[0]
+
+    f0 = (zero, fac[1], fac[2])
+    Wq = O.ternary_weight(W, g, stats, f0, O.PHASE_SOFT, s)[0]
+    _, dY = O.recon_loss(O.linear_fwd(X, Wq), Y_ref)
+    _, _, g_dalpha, g_ddelta = O.linear_bwd(X, dY, W, g, stats, f0, O.PHASE_SOFT, s)
+    want_a = g_dalpha / alpha0 - g_ddelta * D_d / (a_d * a_d * delta0)
+    want_D = g_ddelta / (a_d * delta0)
+    h = 1e-7
+    for which, want in ((0, want_a), (1, want_D)):
+        fd = np.zeros(G)
+        for j in range(G):
+            p = [a_d.copy(), D_d.copy()]
+            m = [a_d.copy(), D_d.copy()]
+            scale = p[which][j]
+            p[which][j] += h * scale
+            m[which][j] -= h * scale
+            fd[j] = (loss_direct(*p) - loss_direct(*m)) / (2 * h * scale)
+        np.testing.assert_allclose(want, fd, rtol=1e-4, atol=1e-6 * np.abs(fd).max())
