@@ -467,6 +467,7 @@ def run_ours(args):
         also[f"{wl.name}/decode_b1"] = measure_decode(C, torch, wl, dev, peaks, rows=1)
         also[f"{wl.name}/decode_b8"] = measure_decode(C, torch, wl, dev, peaks, rows=8)
         also[f"{wl.name}/decode_b1_mu"] = measure_decode(C, torch, wl, dev, peaks, rows=1, with_mu=True)
+        also["c5_qwen3_235b_moe/soft"] = measure_moe(C, torch, dev, peaks, world, args.s)
         for name in ALSO_WORKLOADS:
             if name == wl.name:
                 continue
@@ -551,6 +552,72 @@ def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20, with_m
             "launches_per_step": blocks * len(wl.linears), "bytes_per_step": nbytes, "us_per_step": ms * 1e3,
             "value": gbs, "unit": "GB/s", "peak": peaks["hbm"], "frac_of_hbm": gbs / peaks["hbm"],
             "steps": steps, "graph": True, "with_mu": with_mu}
+
+
+def measure_moe(C, torch, dev, peaks, world, s, steps=5, warmup=2):
+    """One calibration step of the Qwen3-235B-shaped MoE layer: gate/up/down of all 128
+    experts over 8192 tokens routed top-8 (65,536 expert-sorted rows, Zipf(1.1) loads) through
+    the grouped calls (stats once; per step forward, loss, backward, pack).  Weights and
+    activations are drawn on the device (seeded); value = sum 6 M_e N K / step time."""
+    wl = syn.WORKLOADS["c5_qwen3_235b_moe"]
+    token_of_row, off = syn.moe_routing(wl, seed=0)
+    R, E, g = int(off[-1]), wl.experts, wl.g
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(0)
+    tok = torch.from_numpy(token_of_row).to(dev)
+    xs = {"x_hidden": torch.randn(wl.tokens, 4096, generator=gen, device=dev).to(torch.bfloat16)[tok],
+          "x_ffn": torch.randn(R, 1536, generator=gen, device=dev).to(torch.bfloat16)}
+    sched, teacher = C.schedule(C.PHASE_SOFT, s), C.schedule(C.PHASE_TEACHER)
+    lins, flops = [], 0.0
+    for lin in wl.linears:
+        N, K = lin.N, lin.K
+        G = N * K // g
+        W = (torch.randn(E * N, K, generator=gen, device=dev) * wl.w_std).to(torch.bfloat16).reshape(E, N, K)
+        fac = [(torch.rand(E * G, generator=gen, device=dev) - 0.5) * 0.2,
+               0.8 + 0.4 * torch.rand(E * G, generator=gen, device=dev),
+               0.8 + 0.4 * torch.rand(E * G, generator=gen, device=dev)]
+        layer = C.GroupedLayer.create(W, g, *fac)
+        C.catq_group_stats(layer.dense, wl.thr_init)
+        X = xs[lin.x]
+        Yt = torch.empty(R, N, dtype=torch.bfloat16, device=dev)
+        C.catq_grouped_soft_ternary_linear_fwd(layer, teacher, X, off, Yt)
+        lins.append(dict(layer=layer, X=X, Yt=Yt, Y=torch.empty_like(Yt), dY=torch.empty_like(Yt),
+                         dX=torch.empty_like(X), grads=[torch.empty(E * G, device=dev) for _ in range(3)],
+                         codes=torch.empty(E * N * K // 4, dtype=torch.uint8, device=dev),
+                         alpha=torch.empty(E * G, device=dev), loss=torch.empty(1, device=dev),
+                         wsb=C.workspace(C.catq_grouped_bwd_workspace_bytes(layer, off), dev),
+                         wsl=C.workspace(C.catq_recon_loss_workspace_bytes(R * N), dev)))
+        flops += 6.0 * R * N * K
+
+    def step():
+        for d in lins:
+            C.catq_grouped_soft_ternary_linear_fwd(d["layer"], sched, d["X"], off, d["Y"])
+            C.catq_recon_loss(d["Y"], d["Yt"], d["loss"], d["dY"], d["wsl"])
+            C.catq_grouped_soft_ternary_linear_bwd(d["layer"], sched, d["X"], d["dY"], off, d["dX"], *d["grads"],
+                                                   workspace=d["wsb"])
+            C.catq_hard_ternarize_pack(d["layer"].dense, d["codes"], d["alpha"])
+
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(steps):
+        step()
+    b.record()
+    torch.cuda.synchronize()
+    status = C.catq_device_status()
+    if status != 0:
+        raise SystemExit(f"device status {C.STATUS.get(status, status)} in the MoE timing")
+    ms = max_over_ranks(a.elapsed_time(b) / steps, world, dev)
+    value = job_throughput(flops, ms, world)
+    counts = np.diff(off)
+    del lins, xs
+    torch.cuda.empty_cache()
+    return {"value": value, "ms_per_step": ms, "frac_of_burst": value / world / peaks["bf16"], "steps": steps,
+            "experts": E, "routed_rows": R, "rows_per_expert": [int(counts.min()), int(np.median(counts)),
+                                                                 int(counts.max())],
+            "path": "grouped calls: one persistent launch for every expert's forward and dX tiles, factor gradients expert by expert", "phase": "soft", "s": s}
 
 
 def measure_e2e(args, C, torch, st, step, barrier, flops_step, world, dev):

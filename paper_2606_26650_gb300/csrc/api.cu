@@ -344,10 +344,40 @@ catq_status check_grouped(const catq_grouped_layer* G, const int64_t* off) {
 
 }  // namespace
 
+// The bf16 forward or dX of every expert as one grouped tensor-core launch: every expert's
+// tiles in one persistent sweep.  *used is false when the layer does not qualify (fp32,
+// more experts than one launch takes, 2^31 rows or more), and the caller loops instead.
+catq_status grouped_tc(const catq_grouped_layer* G, catq_schedule sched, const void* A, const int64_t* off,
+                       int32_t x_dtype, void* C, bool dx, catq_stream stream, bool* used) {
+  *used = false;
+  if (G->w_dtype != CATQ_BF16 || x_dtype != CATQ_BF16 || G->E > kGroupedMaxExperts) return CATQ_OK;
+  const int64_t R = off[G->E];
+  if (R >= (int64_t(1) << 31)) return CATQ_OK;
+  const catq_layer L = expert_layer(G, 0);
+  catq_status st = check_layer(&L, sched.phase != CATQ_PHASE_TEACHER);
+  if (st != CATQ_OK) return st;
+  if ((st = check_schedule(sched, sched.phase == CATQ_PHASE_SOFT)) != CATQ_OK) return st;
+  if ((st = check_op_const(&L, sched)) != CATQ_OK) return st;
+  const int64_t groups = G->N * G->K / G->g;
+  const int64_t const_stride = (G->recon ? 5 : 4) * groups;
+  if (const_stride % 4 != 0) return CATQ_OK;
+  *used = true;
+  if (R == 0) return CATQ_OK;
+  if (!A || !C) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(A) || !aligned16(C)) return CATQ_ERR_ALIGN;
+  if ((st = check_tensor_core_device()) != CATQ_OK) return st;
+  const GroupSpec grp{G->E, off, const_stride};
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return cuda_status(dx ? launch_tc_dx_grouped(to_dev(&L), scalars(sched), A, grp, C, s)
+                        : launch_tc_fwd_grouped(to_dev(&L), scalars(sched), A, grp, C, s));
+}
+
 catq_status catq_grouped_soft_ternary_linear_fwd(const catq_grouped_layer* G, catq_schedule sched, const void* X,
                                                  const int64_t* off, int32_t x_dtype, void* Y, catq_stream stream) {
   catq_status st = check_grouped(G, off);
   if (st != CATQ_OK) return st;
+  bool used = false;
+  if ((st = grouped_tc(G, sched, X, off, x_dtype, Y, false, stream, &used)) != CATQ_OK || used) return st;
   const size_t esize = x_dtype == CATQ_BF16 ? 2 : 4;
   for (int32_t e = 0; e < G->E; ++e) {
     const catq_layer L = expert_layer(G, e);
@@ -378,13 +408,18 @@ catq_status catq_grouped_soft_ternary_linear_bwd(const catq_grouped_layer* G, ca
   if (st != CATQ_OK) return st;
   const size_t esize = x_dtype == CATQ_BF16 ? 2 : 4;
   const int64_t groups = G->N * G->K / G->g;
+  // dX of every expert in one grouped launch where the layer qualifies; the factor
+  // gradients (and dX otherwise) expert by expert
+  bool dx_done = false;
+  if (dX && (st = grouped_tc(G, sched, dY, off, x_dtype, dX, true, stream, &dx_done)) != CATQ_OK) return st;
   for (int32_t e = 0; e < G->E; ++e) {
     const catq_layer L = expert_layer(G, e);
     const int64_t m = off[e + 1] - off[e];
     st = catq_soft_ternary_linear_bwd(
         &L, sched, static_cast<const char*>(X) + off[e] * G->K * esize,
         static_cast<const char*>(dY) + off[e] * G->N * esize, m, x_dtype,
-        dX ? static_cast<char*>(dX) + off[e] * G->K * esize : nullptr, g_dmu ? g_dmu + e * groups : nullptr,
+        dX && !dx_done ? static_cast<char*>(dX) + off[e] * G->K * esize : nullptr,
+        g_dmu ? g_dmu + e * groups : nullptr,
         g_dalpha ? g_dalpha + e * groups : nullptr, g_ddelta ? g_ddelta + e * groups : nullptr, workspace, ws_bytes,
         stream);
     if (st != CATQ_OK) return st;

@@ -482,7 +482,21 @@ __global__ void __launch_bounds__(kThreads) hard_pack_warp_kernel(LayerDev L, in
 // [N][K/g] group arrays and the output are accessed coalesced.
 constexpr int kConstTile = 32;
 
-__global__ void __launch_bounds__(kConstTile * kConstTile) operand_consts_kernel(LayerDev L, StepScalars sc) {
+// blockIdx.z: expert of a stacked (grouped) layer, whose per-group arrays start z G after
+// expert 0's and whose constants start z const_stride floats after (0 for a dense layer).
+__global__ void __launch_bounds__(kConstTile * kConstTile) operand_consts_kernel(LayerDev L, StepScalars sc,
+                                                                                 int64_t const_stride) {
+  if (blockIdx.z > 0) {
+    const int64_t G = L.N * L.groups_per_row, e = blockIdx.z;
+    L.mu0 += e * G;
+    L.alpha0 += e * G;
+    L.delta0 += e * G;
+    L.d_mu += e * G;
+    L.d_alpha += e * G;
+    L.d_delta += e * G;
+    L.op_const = reinterpret_cast<float4*>(reinterpret_cast<float*>(L.op_const) + e * const_stride);
+    if (L.op_mu) L.op_mu += e * const_stride;
+  }
   __shared__ float4 tile[kConstTile][kConstTile + 1];
   __shared__ float tile_mu[kConstTile][kConstTile + 1];
   const int64_t gpr = L.groups_per_row;
@@ -749,7 +763,16 @@ cudaError_t launch_operand_consts(const LayerDev& L, StepScalars sc, cudaStream_
   const int64_t row_tiles = (L.N + kConstTile - 1) / kConstTile;
   const dim3 grid(static_cast<unsigned>((L.groups_per_row + kConstTile - 1) / kConstTile),
                   static_cast<unsigned>(row_tiles < 65535 ? row_tiles : 65535));
-  operand_consts_kernel<<<grid, dim3(kConstTile, kConstTile), 0, st>>>(L, sc);
+  operand_consts_kernel<<<grid, dim3(kConstTile, kConstTile), 0, st>>>(L, sc, 0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_operand_consts_grouped(const LayerDev& L0, StepScalars sc, int32_t E, int64_t const_stride,
+                                          cudaStream_t st) {
+  const int64_t row_tiles = (L0.N + kConstTile - 1) / kConstTile;
+  const dim3 grid(static_cast<unsigned>((L0.groups_per_row + kConstTile - 1) / kConstTile),
+                  static_cast<unsigned>(row_tiles < 65535 ? row_tiles : 65535), static_cast<unsigned>(E));
+  operand_consts_kernel<<<grid, dim3(kConstTile, kConstTile), 0, st>>>(L0, sc, const_stride);
   return cudaGetLastError();
 }
 

@@ -61,6 +61,23 @@ cudaError_t launch_wait_probe(uint64_t timeout_ns, cudaStream_t st);
 // Writes L.op_const (operand_const_vec of every group, [K/g][N]) for schedule point sc.
 cudaError_t launch_operand_consts(const LayerDev& L, StepScalars sc, cudaStream_t st);
 
+// Grouped (MoE) launches: E experts of identical shape, L0 is expert 0's layer with the
+// stacked weights [E N, K] from L0.W on; per-group arrays of expert e start e G after
+// expert 0's, its operand constants const_stride floats after; rows of A and C are
+// expert-sorted with host offsets off[0..E].
+constexpr int32_t kGroupedMaxExperts = 128;
+struct GroupSpec {
+  int32_t E;
+  const int64_t* off;
+  int64_t const_stride;
+};
+cudaError_t launch_operand_consts_grouped(const LayerDev& L0, StepScalars sc, int32_t E, int64_t const_stride,
+                                          cudaStream_t st);
+cudaError_t launch_tc_fwd_grouped(const LayerDev& L0, StepScalars sc, const void* X, const GroupSpec& grp, void* Y,
+                                  cudaStream_t st);
+cudaError_t launch_tc_dx_grouped(const LayerDev& L0, StepScalars sc, const void* dY, const GroupSpec& grp, void* dX,
+                                 cudaStream_t st);
+
 cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st);
 cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int64_t M, void* dX, cudaStream_t st);
 cudaError_t launch_tc_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M,

@@ -103,6 +103,9 @@ struct DwCfg {
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + kBarBytes;
 };
 
+// Experts of one grouped launch (stacked expert weights, expert-sorted rows).
+constexpr int kMaxGroupExperts = kGroupedMaxExperts;
+
 struct FusedArgs {
   LayerDev L;
   StepScalars sc;
@@ -112,16 +115,52 @@ struct FusedArgs {
   int32_t num_m_tiles, num_n_tiles, num_k_blocks;
   int32_t group_m;  // M blocks per raster group
   WaitCtl wc;
+  // Grouped launches (E > 0): expert e owns rows [row0[e], row0[e+1]) of A and C, W rows
+  // [e N, (e+1) N) of the stacked weights, operand constants from float e * const_stride
+  // on, and tiles [tile0[e], tile0[e+1]) (its M blocks, then N blocks).
+  int32_t E;
+  int64_t const_stride;
+  int32_t tile0[kMaxGroupExperts + 1];
+  int32_t row0[kMaxGroupExperts + 1];
 };
 
-// Tile t of a persistent sequence -> (M block, N block).  Tiles run in groups of group_m M
-// blocks: inside a group the M block varies fastest, then the N block.
-__device__ __forceinline__ void tile_coords(const FusedArgs& a, int t, int& m_blk, int& n_blk) {
-  const int per_group = a.group_m * a.num_n_tiles;
-  const int grp = t / per_group, r = t - grp * per_group;
-  const int gm = min(a.group_m, a.num_m_tiles - grp * a.group_m);
-  m_blk = grp * a.group_m + r % gm;
-  n_blk = r / gm;
+// Tile t of a persistent sequence: its M and N block, expert, first row and row limit.
+struct TileInfo {
+  int m_blk, n_blk, e;
+  int64_t row0, row_end;
+};
+
+// Dense: tiles run in groups of group_m M blocks (inside a group the M block varies fastest,
+// then the N block).  Grouped: the expert is found by binary search over its first tiles;
+// inside an expert the M block varies fastest.
+__device__ __forceinline__ TileInfo tile_info(const FusedArgs& a, int t, int rows_per_tile) {
+  TileInfo ti;
+  if (a.E == 0) {
+    const int per_group = a.group_m * a.num_n_tiles;
+    const int grp = t / per_group, r = t - grp * per_group;
+    const int gm = min(a.group_m, a.num_m_tiles - grp * a.group_m);
+    ti.m_blk = grp * a.group_m + r % gm;
+    ti.n_blk = r / gm;
+    ti.e = 0;
+    ti.row0 = (int64_t)ti.m_blk * rows_per_tile;
+    ti.row_end = a.M;
+    return ti;
+  }
+  int lo = 0, hi = a.E;  // last e with tile0[e] <= t
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (a.tile0[mid] <= t) lo = mid;
+    else hi = mid;
+  }
+  const int r0 = a.row0[lo], r1 = a.row0[lo + 1];
+  const int mt = (r1 - r0 + rows_per_tile - 1) / rows_per_tile;
+  const int local = t - a.tile0[lo];
+  ti.e = lo;
+  ti.m_blk = local % mt;
+  ti.n_blk = local / mt;
+  ti.row0 = r0 + (int64_t)ti.m_blk * rows_per_tile;
+  ti.row_end = r1;
+  return ti;
 }
 
 struct DwArgs {
@@ -190,34 +229,38 @@ __device__ __forceinline__ void store_rows_bf16x32(uint16_t* C, int64_t M, int64
 // CTA's tile sequence) and tracks which W row, K chunk and group its 128-byte operand row
 // holds, the group as its index into the [K/g][N] operand-constant array.  Divisions happen
 // once per tile; each stage step is a few integer adds.
-template <int CG, bool B_MN>
+template <int CG, bool B_MN, int PAIRS>
 struct OperandRowIter {
-  using Cfg = FusedCfg<CG>;
+  using Cfg = FusedCfg<CG, PAIRS>;
   int t, kb;      // tile index, k block
-  int64_t n, kc;  // W row, first K column of the 64-element chunk
-  int64_t ci;     // operand-constant index of (n, kc): (kc / g) * N + n
+  int64_t n, kc;  // W row (within its expert), first K column of the 64-element chunk
+  int64_t ci;     // operand-constant index of (n, kc): (kc / g) * N + n, in float4 units from
+                  // the launch's first expert's constants
+  int64_t mi;     // the same entry's index into the mu plane (floats)
   int kin;        // forward: k blocks into the current group (kc / 64 mod g / 64)
   bool tile_ok;   // forward: n < N; dX: kc < K
 
   __device__ __forceinline__ void init(const FusedArgs& a, uint32_t cta, int row, int t_, int kb_) {
     t = t_;
     kb = kb_;
-    int m_blk, n_blk;
-    tile_coords(a, t, m_blk, n_blk);
+    const TileInfo ti = tile_info(a, t, Cfg::kTileRows * PAIRS);
     const int gk = a.L.g / BK;  // k blocks per group
+    int64_t local;
     if constexpr (!B_MN) {
-      n = (int64_t)n_blk * BN + cta * Cfg::kBRows + row;
+      n = (int64_t)ti.n_blk * BN + cta * Cfg::kBRows + row;
       kc = (int64_t)kb * BK;
       tile_ok = n < a.L.N;
-      ci = (int64_t)(kb / gk) * a.L.N + n;
+      local = (int64_t)(kb / gk) * a.L.N + n;
       kin = kb % gk;
     } else {
       n = (int64_t)kb * BK + (row & 63);
-      kc = (int64_t)n_blk * BN + cta * Cfg::kBRows + 64 * (row >> 6);
+      kc = (int64_t)ti.n_blk * BN + cta * Cfg::kBRows + 64 * (row >> 6);
       tile_ok = kc < a.L.K;
-      ci = (kc / a.L.g) * a.L.N + n;
+      local = (kc / a.L.g) * a.L.N + n;
       kin = 0;
     }
+    ci = (ti.e * a.const_stride) / 4 + local;
+    mi = ti.e * a.const_stride + local;
   }
 
   __device__ __forceinline__ bool live(const FusedArgs& a, int num_tiles) const { return t < num_tiles; }
@@ -244,10 +287,12 @@ struct OperandRowIter {
       while (kin >= gk) {
         kin -= gk;
         ci += a.L.N;
+        mi += a.L.N;
       }
     } else {
       n += (int64_t)steps * BK;
       ci += (int64_t)steps * BK;
+      mi += (int64_t)steps * BK;
     }
   }
 };
@@ -338,9 +383,8 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
       uint32_t q = 0, issued_mask = 0, issued_phase = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
-        int m_blk, n_blk;
-        tile_coords(args, t, m_blk, n_blk);
-        const int32_t m0 = m_blk * (Cfg::kTileRows * PAIRS) + pair * Cfg::kTileRows;
+        const TileInfo ti = tile_info(args, t, Cfg::kTileRows * PAIRS);
+        const int32_t m0 = static_cast<int32_t>(ti.row0) + pair * Cfg::kTileRows;
         for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
           const uint32_t s = q % SA, ph = (q / SA) & 1u;
           if (!mbar_wait(empty_a(s), ph ^ 1u, wc)) { ok = false; break; }
@@ -364,9 +408,9 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
       uint32_t q = 0, issued_mask = 0, issued_phase = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
-        int m_blk, n_blk;
-        tile_coords(args, t, m_blk, n_blk);
-        const int32_t n0 = n_blk * BN + cta * Cfg::kBRows;
+        const TileInfo ti = tile_info(args, t, Cfg::kTileRows * PAIRS);
+        const int32_t n0 = ti.n_blk * BN + cta * Cfg::kBRows;
+        const int32_t wrow = static_cast<int32_t>(ti.e * args.L.N);  // the expert's first W row
         for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
           if (!produces(q)) continue;
           const uint32_t s = q % SW, ph = (q / SW) & 1u;
@@ -376,10 +420,11 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
           mbar_arrive_expect_tx(raw_w(rb), Cfg::kWBytes);
           const uint32_t dst = w_base + s * Cfg::kWBytes;
           if constexpr (!B_MN) {
-            tma_load_2d(dst, &tmW, raw_w(rb), kb * BK, n0);
+            tma_load_2d(dst, &tmW, raw_w(rb), kb * BK, wrow + n0);
           } else {
 #pragma unroll
-            for (int b = 0; b < Cfg::kBRows / 64; ++b) tma_load_2d(dst + b * 8192, &tmW, raw_w(rb), n0 + 64 * b, kb * BK);
+            for (int b = 0; b < Cfg::kBRows / 64; ++b)
+              tma_load_2d(dst + b * 8192, &tmW, raw_w(rb), n0 + 64 * b, wrow + kb * BK);
           }
           issued_mask |= 1u << rb;
           issued_phase = (issued_phase & ~(1u << rb)) | (rph << rb);
@@ -451,22 +496,21 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     const int qd = warp;  // TMEM lane quarter
     uint32_t it = 0;
     for (int t = cluster; t < num_tiles; t += nclusters, ++it) {
-      int m_blk, n_blk;
-      tile_coords(args, t, m_blk, n_blk);
+      const TileInfo ti = tile_info(args, t, Cfg::kTileRows * PAIRS);
       if (!mbar_wait(tmem_full_bar, it & 1u, wc)) break;
       tc_fence_after();
 #pragma unroll 1
       for (int acc = 0; acc < NACC; ++acc) {
-        const int64_t row0 = (int64_t)m_blk * (Cfg::kTileRows * PAIRS) + pair * Cfg::kTileRows +
-                             acc * Cfg::kRowsPerAcc + cta * 128 + qd * 32;  // this warp's first row
+        const int64_t row0 = ti.row0 + pair * Cfg::kTileRows + acc * Cfg::kRowsPerAcc + cta * 128 +
+                             qd * 32;  // this warp's first row
 #pragma unroll 1
         for (int c = 0; c < BN / 32; ++c) {
-          const int64_t col = (int64_t)n_blk * BN + c * 32;
-          if (col >= args.ncols || row0 >= args.M) break;  // warp-uniform
+          const int64_t col = (int64_t)ti.n_blk * BN + c * 32;
+          if (col >= args.ncols || row0 >= ti.row_end) break;  // warp-uniform
           uint32_t r[32];
           tmem_ld32(tmem_base + (static_cast<uint32_t>(qd * 32) << 16) + acc * BN + c * 32, r);
           tmem_ld_wait();
-          store_rows_bf16x32(args.C, args.M, args.ncols, row0, col, r, lane);
+          store_rows_bf16x32(args.C, ti.row_end, args.ncols, row0, col, r, lane);
         }
       }
       tc_fence_before();
@@ -501,7 +545,7 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     // `cur` is the stage being produced; `ahead` runs two of this thread's stages ahead and
     // requests that stage's operand constants (one 16-byte vector, precomputed per call), so
     // an L2 round trip is hidden behind two stages.
-    OperandRowIter<CG, B_MN> cur, ahead;
+    OperandRowIter<CG, B_MN, PAIRS> cur, ahead;
     cur.init(args, cta, row, cluster, 0);
     cur.step(args, cta, row, nclusters, q0);
     ahead = cur;
@@ -510,15 +554,15 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     float m0 = 0.0f, m1 = 0.0f;
     int64_t j0 = -1, j1 = -1;
     constexpr bool with_mu = MU;
-    auto request = [&](const OperandRowIter<CG, B_MN>& it, float4& dst, float& dm, int64_t& jd, const float4& other,
-                       float om, int64_t jo) {
+    auto request = [&](const OperandRowIter<CG, B_MN, PAIRS>& it, float4& dst, float& dm, int64_t& jd,
+                       const float4& other, float om, int64_t jo) {
       if (transform && it.live(args, num_tiles) && it.valid(args)) {
         if (jo == it.ci) {
           dst = other;
           dm = om;
         } else {
           dst = __ldg(L.op_const + it.ci);
-          if (with_mu) dm = __ldg(L.op_mu + it.ci);
+          if (with_mu) dm = __ldg(L.op_mu + it.mi);
         }
         jd = it.ci;
       }
@@ -935,18 +979,21 @@ int max_active_clusters(Kern kern, int cluster_ctas, int threads, int smem, int 
 // CTA pairs (512 rows) from 512 rows, single CTAs below.
 int fused_variant_for(int64_t M) { return M >= 1024 ? 4 : (M >= 512 ? 2 : 1); }
 
+// grp (nullable): a grouped launch over grp->E experts whose weights are stacked from L.W on
+// and whose rows of A and C are expert-sorted (host offsets grp->off).
 template <int CG, bool B_MN, int PAIRS, bool MU>
 cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t M, int64_t depth, void* C,
-                      int64_t ncols, cudaStream_t st) {
+                      int64_t ncols, cudaStream_t st, const GroupSpec* grp = nullptr) {
   using Cfg = FusedCfg<CG, PAIRS>;
   DeviceInfo& d = device_info();
   if (!d.ok) return cudaErrorInvalidDevice;
+  const int64_t wrows = grp ? grp->E * L.N : L.N;
   CUtensorMap ta, tw;
   if (!make_tmap(&ta, A, depth, M, BK, 128)) return cudaErrorInvalidValue;
   if constexpr (!B_MN) {
-    if (!make_tmap(&tw, L.W, L.K, L.N, BK, Cfg::kBRows)) return cudaErrorInvalidValue;
+    if (!make_tmap(&tw, L.W, L.K, wrows, BK, Cfg::kBRows)) return cudaErrorInvalidValue;
   } else {
-    if (!make_tmap(&tw, L.W, L.K, L.N, 64, BK)) return cudaErrorInvalidValue;
+    if (!make_tmap(&tw, L.W, L.K, wrows, 64, BK)) return cudaErrorInvalidValue;
   }
   FusedArgs args;
   args.L = L;
@@ -959,8 +1006,25 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
   args.num_k_blocks = static_cast<int32_t>((depth + BK - 1) / BK);
   args.group_m = std::min(4, args.num_m_tiles);
   args.wc = make_wait_ctl(d);
+  args.E = 0;
+  args.const_stride = 0;
+  int tiles = args.num_m_tiles * args.num_n_tiles;
+  if (grp) {
+    if (grp->E < 1 || grp->E > kMaxGroupExperts) return cudaErrorInvalidValue;
+    args.E = grp->E;
+    args.const_stride = grp->const_stride;
+    const int64_t rows_per_tile = Cfg::kTileRows * PAIRS;
+    int64_t t = 0;
+    for (int e = 0; e <= grp->E; ++e) {
+      args.tile0[e] = static_cast<int32_t>(t);
+      args.row0[e] = static_cast<int32_t>(grp->off[e]);
+      if (e < grp->E) t += (grp->off[e + 1] - grp->off[e] + rows_per_tile - 1) / rows_per_tile * args.num_n_tiles;
+    }
+    tiles = static_cast<int>(t);
+    args.num_m_tiles = static_cast<int32_t>(t / args.num_n_tiles);  // the kernel's tile count is M x N blocks
+    if (tiles == 0) return cudaSuccess;
+  }
   auto kern = fused_gemm_kernel<CG, B_MN, PAIRS, MU>;
-  const int tiles = args.num_m_tiles * args.num_n_tiles;
   const int fit = max_active_clusters(kern, Cfg::kClusterCtas, Cfg::kThreads, Cfg::kSmemBytes,
                                       d.sm_count / Cfg::kClusterCtas);
   const int clusters = std::min(tiles, fit);
@@ -1011,7 +1075,41 @@ cudaError_t dispatch_fused(const LayerDev& L, StepScalars sc, const void* A, int
   }
 }
 
+// Grouped: the tile shape by the mean rows per expert.
+template <bool B_MN>
+cudaError_t dispatch_fused_grouped(const LayerDev& L, StepScalars sc, const void* A, int64_t depth, void* C,
+                                   int64_t ncols, const GroupSpec& grp, cudaStream_t st) {
+  const int64_t R = grp.off[grp.E];
+  const bool mu = L.recon != 0 && sc.phase != PHASE_TEACHER;
+  switch (fused_variant_for(R / grp.E) * 2 + (mu ? 1 : 0)) {
+    case 8: return run_fused<2, B_MN, 2, false>(L, sc, A, R, depth, C, ncols, st, &grp);
+    case 9: return run_fused<2, B_MN, 2, true>(L, sc, A, R, depth, C, ncols, st, &grp);
+    case 4: return run_fused<2, B_MN, 1, false>(L, sc, A, R, depth, C, ncols, st, &grp);
+    case 5: return run_fused<2, B_MN, 1, true>(L, sc, A, R, depth, C, ncols, st, &grp);
+    case 3: return run_fused<1, B_MN, 1, true>(L, sc, A, R, depth, C, ncols, st, &grp);
+    default: return run_fused<1, B_MN, 1, false>(L, sc, A, R, depth, C, ncols, st, &grp);
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_tc_fwd_grouped(const LayerDev& L0, StepScalars sc, const void* X, const GroupSpec& grp, void* Y,
+                                  cudaStream_t st) {
+  if (sc.phase != PHASE_TEACHER) {
+    const cudaError_t e = launch_operand_consts_grouped(L0, sc, grp.E, grp.const_stride, st);
+    if (e != cudaSuccess) return e;
+  }
+  return dispatch_fused_grouped<false>(L0, sc, X, L0.K, Y, L0.N, grp, st);
+}
+
+cudaError_t launch_tc_dx_grouped(const LayerDev& L0, StepScalars sc, const void* dY, const GroupSpec& grp, void* dX,
+                                 cudaStream_t st) {
+  if (sc.phase != PHASE_TEACHER) {
+    const cudaError_t e = launch_operand_consts_grouped(L0, sc, grp.E, grp.const_stride, st);
+    if (e != cudaSuccess) return e;
+  }
+  return dispatch_fused_grouped<true>(L0, sc, dY, L0.N, dX, L0.K, grp, st);
+}
 
 bool tensor_map_encoder_available() {
   init_encoder();
