@@ -6,6 +6,7 @@
 #include <cmath>
 #include <cstdint>
 #include <mutex>
+#include <numeric>
 
 #include "catq.h"
 #include "launch.h"
@@ -344,6 +345,21 @@ catq_status check_grouped(const catq_grouped_layer* G, const int64_t* off) {
 
 }  // namespace
 
+// Whether the factor gradients of a grouped layer run as grouped launches (bf16, at most
+// kGroupedMaxExperts experts, fewer than 2^31 rows); otherwise expert by expert.
+bool grouped_dw_ok(const catq_grouped_layer* G, const int64_t* off) {
+  return G->w_dtype == CATQ_BF16 && G->E <= kGroupedMaxExperts && off[G->E] < (int64_t(1) << 31) && G->g > 0 &&
+         G->K % G->g == 0;
+}
+
+int32_t grouped_dw_P(const catq_grouped_layer* G) { return std::gcd(G->g, 128); }
+
+// Partial group sums of every expert: [E][3][N][K/P] fp32.
+size_t grouped_partials_bytes(const catq_grouped_layer* G) {
+  return static_cast<size_t>(G->E) * 3 * static_cast<size_t>(G->N) * static_cast<size_t>(G->K / grouped_dw_P(G)) *
+         sizeof(float);
+}
+
 // The bf16 forward or dX of every expert as one grouped tensor-core launch: every expert's
 // tiles in one persistent sweep.  *used is false when the layer does not qualify (fp32,
 // more experts than one launch takes, 2^31 rows or more), and the caller loops instead.
@@ -391,6 +407,7 @@ catq_status catq_grouped_soft_ternary_linear_fwd(const catq_grouped_layer* G, ca
 
 size_t catq_grouped_bwd_workspace_bytes(const catq_grouped_layer* G, const int64_t* off) {
   if (check_grouped(G, off) != CATQ_OK) return 0;
+  if (grouped_dw_ok(G, off)) return round256(grouped_partials_bytes(G));
   size_t best = 0;
   for (int32_t e = 0; e < G->E; ++e) {
     const catq_layer L = expert_layer(G, e);
@@ -412,6 +429,39 @@ catq_status catq_grouped_soft_ternary_linear_bwd(const catq_grouped_layer* G, ca
   // gradients (and dX otherwise) expert by expert
   bool dx_done = false;
   if (dX && (st = grouped_tc(G, sched, dY, off, x_dtype, dX, true, stream, &dx_done)) != CATQ_OK) return st;
+  const bool want_grads = g_dmu || g_dalpha || g_ddelta;
+  bool dw_done = !want_grads;
+  if (want_grads && x_dtype == CATQ_BF16 && grouped_dw_ok(G, off)) {
+    if (!(g_dmu && g_dalpha && g_ddelta)) return CATQ_ERR_INVALID_ARG;
+    const catq_layer L = expert_layer(G, 0);
+    if ((st = check_layer(&L, sched.phase != CATQ_PHASE_TEACHER)) != CATQ_OK) return st;
+    if ((st = check_schedule(sched, sched.phase != CATQ_PHASE_TEACHER)) != CATQ_OK) return st;
+    const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const int64_t R = off[G->E];
+    if (sched.phase == CATQ_PHASE_TEACHER || R == 0) {
+      const size_t b = static_cast<size_t>(G->E) * groups * sizeof(float);
+      if (cudaMemsetAsync(g_dmu, 0, b, s) != cudaSuccess || cudaMemsetAsync(g_dalpha, 0, b, s) != cudaSuccess ||
+          cudaMemsetAsync(g_ddelta, 0, b, s) != cudaSuccess)
+        return CATQ_ERR_CUDA;
+    } else {
+      if (!X || !dY) return CATQ_ERR_INVALID_ARG;
+      if (!aligned16(X) || !aligned16(dY)) return CATQ_ERR_ALIGN;
+      if (!workspace || ws_bytes < grouped_partials_bytes(G)) return CATQ_ERR_WORKSPACE;
+      if (!aligned256(workspace)) return CATQ_ERR_ALIGN;
+      if ((st = check_tensor_core_device()) != CATQ_OK) return st;
+      const GroupSpec grp{G->E, off, 0};
+      const LayerDev L0 = to_dev(&L);
+      const StepScalars sc = scalars(sched);
+      float* part = static_cast<float*>(workspace);
+      const int32_t P = grouped_dw_P(G);
+      if (launch_tc_dw_grouped(L0, sc, X, dY, grp, P, part, s) != cudaSuccess) return CATQ_ERR_CUDA;
+      if ((st = cuda_status(launch_grad_reduce_grouped(L0, sc, part, P, grp, g_dmu, g_dalpha, g_ddelta, s))) !=
+          CATQ_OK)
+        return st;
+    }
+    dw_done = true;
+  }
+  if (dw_done && (dx_done || !dX)) return CATQ_OK;
   for (int32_t e = 0; e < G->E; ++e) {
     const catq_layer L = expert_layer(G, e);
     const int64_t m = off[e + 1] - off[e];
@@ -419,9 +469,9 @@ catq_status catq_grouped_soft_ternary_linear_bwd(const catq_grouped_layer* G, ca
         &L, sched, static_cast<const char*>(X) + off[e] * G->K * esize,
         static_cast<const char*>(dY) + off[e] * G->N * esize, m, x_dtype,
         dX && !dx_done ? static_cast<char*>(dX) + off[e] * G->K * esize : nullptr,
-        g_dmu ? g_dmu + e * groups : nullptr,
-        g_dalpha ? g_dalpha + e * groups : nullptr, g_ddelta ? g_ddelta + e * groups : nullptr, workspace, ws_bytes,
-        stream);
+        g_dmu && !dw_done ? g_dmu + e * groups : nullptr,
+        g_dalpha && !dw_done ? g_dalpha + e * groups : nullptr,
+        g_ddelta && !dw_done ? g_ddelta + e * groups : nullptr, workspace, ws_bytes, stream);
     if (st != CATQ_OK) return st;
   }
   return CATQ_OK;

@@ -630,6 +630,45 @@ __global__ void __launch_bounds__(kThreads) grad_reduce_kernel(LayerDev L, StepS
   }
 }
 
+// Grouped: groups of all experts of a stacked layer; expert e's partials [3][N][K/P] start
+// e 3 N K/P floats in, its group arrays e G in; experts without rows get zeros.
+struct ExpertRows {
+  int32_t rows[kGroupedMaxExperts];
+};
+
+__global__ void __launch_bounds__(kThreads) grad_reduce_grouped_kernel(LayerDev L, StepScalars sc,
+                                                                       const float* __restrict__ part, int32_t P,
+                                                                       int32_t E, const ExpertRows er,
+                                                                       float* __restrict__ g_dmu,
+                                                                       float* __restrict__ g_dalpha,
+                                                                       float* __restrict__ g_ddelta) {
+  const int64_t G = L.N * L.K / L.g;
+  const int64_t cpr = L.K / P;
+  const int32_t cpg = L.g / P;
+  const int64_t plane = L.N * cpr;
+  const float k = sc.s * sc.inv_2tanh_s;
+  for (int64_t ej = blockIdx.x * (int64_t)kThreads + threadIdx.x; ej < E * G; ej += (int64_t)gridDim.x * kThreads) {
+    const int64_t e = ej / G, j = ej - e * G;
+    float s3[3] = {0.f, 0.f, 0.f};
+    bool live = false;
+    GroupConst gc{};
+    if (er.rows[e] > 0) {
+      const int64_t n = j / L.groups_per_row;
+      const int64_t c0 = (j % L.groups_per_row) * cpg;
+#pragma unroll
+      for (int q = 0; q < 3; ++q) {
+        const float* p = part + (e * 3 + q) * plane + n * cpr + c0;
+        for (int32_t c = 0; c < cpg; ++c) s3[q] += p[c];
+      }
+      gc = group_const(L, ej);
+      live = gc.alpha != 0.0f;
+    }
+    g_dmu[ej] = live ? -gc.alpha0 * k * s3[0] : 0.0f;
+    g_dalpha[ej] = live ? gc.alpha0 * s3[1] : 0.0f;
+    g_ddelta[ej] = live ? gc.delta0 * gc.alpha * k * s3[2] : 0.0f;
+  }
+}
+
 int grid_for(int64_t work, int64_t per_block) {
   int64_t b = (work + per_block - 1) / per_block;
   if (b < 1) b = 1;
@@ -773,6 +812,17 @@ cudaError_t launch_operand_consts_grouped(const LayerDev& L0, StepScalars sc, in
   const dim3 grid(static_cast<unsigned>((L0.groups_per_row + kConstTile - 1) / kConstTile),
                   static_cast<unsigned>(row_tiles < 65535 ? row_tiles : 65535), static_cast<unsigned>(E));
   operand_consts_kernel<<<grid, dim3(kConstTile, kConstTile), 0, st>>>(L0, sc, const_stride);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_grad_reduce_grouped(const LayerDev& L0, StepScalars sc, const float* partials, int32_t P,
+                                       const GroupSpec& grp, float* g_dmu, float* g_dalpha, float* g_ddelta,
+                                       cudaStream_t st) {
+  ExpertRows er{};
+  for (int32_t e = 0; e < grp.E; ++e) er.rows[e] = static_cast<int32_t>(grp.off[e + 1] - grp.off[e] > 0 ? 1 : 0);
+  const int64_t G = L0.N * L0.K / L0.g;
+  grad_reduce_grouped_kernel<<<grid_for(grp.E * G, kThreads), kThreads, 0, st>>>(L0, sc, partials, P, grp.E, er, g_dmu,
+                                                                                 g_dalpha, g_ddelta);
   return cudaGetLastError();
 }
 

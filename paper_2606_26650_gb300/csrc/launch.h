@@ -77,6 +77,13 @@ cudaError_t launch_tc_fwd_grouped(const LayerDev& L0, StepScalars sc, const void
                                   cudaStream_t st);
 cudaError_t launch_tc_dx_grouped(const LayerDev& L0, StepScalars sc, const void* dY, const GroupSpec& grp, void* dX,
                                  cudaStream_t st);
+// Partial group sums of every expert with rows, [E][3][N][K/P] (P = gcd(g, 128)).
+cudaError_t launch_tc_dw_grouped(const LayerDev& L0, StepScalars sc, const void* X, const void* dY,
+                                 const GroupSpec& grp, int32_t P, float* partials, cudaStream_t st);
+// Factor gradients [E G] from those partials; zeros for experts without rows.
+cudaError_t launch_grad_reduce_grouped(const LayerDev& L0, StepScalars sc, const float* partials, int32_t P,
+                                       const GroupSpec& grp, float* g_dmu, float* g_dalpha, float* g_ddelta,
+                                       cudaStream_t st);
 
 cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st);
 cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int64_t M, void* dX, cudaStream_t st);

@@ -166,11 +166,24 @@ __device__ __forceinline__ TileInfo tile_info(const FusedArgs& a, int t, int row
 struct DwArgs {
   LayerDev L;
   StepScalars sc;
-  float* part;      // [splits][3][N][K/P]
+  float* part;      // [splits][3][N][K/P]; grouped: [E][3][N][K/P]
   int64_t M;
   int32_t splits, P, kb_per_split, kb_total;
   int32_t num_n_tiles, num_k_tiles;
   WaitCtl wc;
+  int32_t n_experts;  // grouped: experts of this launch (0: dense)
+};
+
+// Grouped dW launch: up to kDwGroupExperts experts with rows, each with tensor maps over its
+// own rows of dY and X (so the contraction stops at the expert's last row: rows past it
+// read as zeros), its index in the stacked layer and its row count.
+constexpr int kDwGroupExperts = 64;
+template <int NE>
+struct DwMaps {
+  CUtensorMap dy[NE];
+  CUtensorMap x[NE];
+  int32_t expert[NE];
+  int32_t rows[NE];
 };
 
 // Wait that ignores the abort flag (used to drain work already issued).
@@ -651,9 +664,11 @@ __global__ void wait_probe_kernel(const WaitCtl wc) {
 
 // ============================================================================ dW kernel
 
-template <int CG, bool MU>
+// NE > 1: a grouped launch over gm's experts (tmDY, tmX unused).
+template <int CG, bool MU, int NE>
 __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
-    dw_kernel(const __grid_constant__ CUtensorMap tmDY, const __grid_constant__ CUtensorMap tmX, const DwArgs args) {
+    dw_kernel(const __grid_constant__ CUtensorMap tmDY, const __grid_constant__ CUtensorMap tmX, const DwArgs args,
+              const __grid_constant__ DwMaps<NE> gm) {
   using Cfg = DwCfg<CG>;
   constexpr int S = Cfg::kStages;
   extern __shared__ uint8_t smem_raw[];
@@ -674,7 +689,19 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
   const uint32_t nclusters = CG == 2 ? num_clusters_x() : gridDim.x;
   const WaitCtl& wc = args.wc;
   const int tiles_per_split = args.num_n_tiles * args.num_k_tiles;
-  const int num_tiles = tiles_per_split * args.splits;
+  // grouped: expert slot i owns tiles [i tiles_per_split, (i + 1) tiles_per_split)
+  const int num_tiles = tiles_per_split * (NE > 1 ? args.n_experts : args.splits);
+  // The contraction range of tile t: its split's k blocks (dense) or its expert's rows.
+  auto kb_range = [&](int t, int& kb0, int& kb1) {
+    if constexpr (NE > 1) {
+      kb0 = 0;
+      kb1 = (gm.rows[t / tiles_per_split] + BK - 1) / BK;
+    } else {
+      const int split = t / tiles_per_split;
+      kb0 = split * args.kb_per_split;
+      kb1 = min(kb0 + args.kb_per_split, args.kb_total);
+    }
+  };
   constexpr int kTma = Cfg::kEpiWarps, kMma = Cfg::kEpiWarps + 1;
 
   if (threadIdx.x == 0) {
@@ -690,7 +717,7 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
     fence_mbar_init_cluster();
   }
   if (warp == kMma) tmem_alloc<CG>(smem_u32(tmem_slot), kTmemCols);
-  if (warp == kTma && lane == 0) {
+  if (NE == 1 && warp == kTma && lane == 0) {
     prefetch_tmap(&tmDY);
     prefetch_tmap(&tmX);
   }
@@ -706,10 +733,16 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
       uint32_t stage = 0, phase = 0, issued_mask = 0, issued_phase = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
-        const int split = t / tiles_per_split, r = t % tiles_per_split;
+        const int r = t % tiles_per_split;
         const int k_blk = r % args.num_k_tiles, n_blk = r / args.num_k_tiles;
-        const int kb0 = split * args.kb_per_split;
-        const int kb1 = min(kb0 + args.kb_per_split, args.kb_total);
+        int kb0, kb1;
+        kb_range(t, kb0, kb1);
+        const void* mdy = &tmDY;
+        const void* mx = &tmX;
+        if constexpr (NE > 1) {
+          mdy = &gm.dy[t / tiles_per_split];
+          mx = &gm.x[t / tiles_per_split];
+        }
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(empty(stage), phase ^ 1u, wc)) { ok = false; break; }
           const uint32_t sa = base + stage * Cfg::kStageBytes, sb = sa + Cfg::kABytes;
@@ -719,14 +752,14 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
 #pragma unroll
           for (int b = 0; b < 2; ++b) {
             const int32_t n = n_blk * Cfg::kTileRows + cta * 128 + 64 * b;
-            if constexpr (CG == 1) tma_load_2d(sa + b * 8192, &tmDY, fb, n, m);
-            else tma_load_2d_pair(sa + b * 8192, &tmDY, fb, n, m);
+            if constexpr (CG == 1) tma_load_2d(sa + b * 8192, mdy, fb, n, m);
+            else tma_load_2d_pair(sa + b * 8192, mdy, fb, n, m);
           }
 #pragma unroll
           for (int b = 0; b < Cfg::kBCols / 64; ++b) {
             const int32_t k = k_blk * BN + cta * Cfg::kBCols + 64 * b;
-            if constexpr (CG == 1) tma_load_2d(sb + b * 8192, &tmX, fb, k, m);
-            else tma_load_2d_pair(sb + b * 8192, &tmX, fb, k, m);
+            if constexpr (CG == 1) tma_load_2d(sb + b * 8192, mx, fb, k, m);
+            else tma_load_2d_pair(sb + b * 8192, mx, fb, k, m);
           }
           issued_mask |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -744,9 +777,8 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
       uint32_t stage = 0, phase = 0, it = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters, ++it) {
-        const int split = t / tiles_per_split;
-        const int kb0 = split * args.kb_per_split;
-        const int kb1 = min(kb0 + args.kb_per_split, args.kb_total);
+        int kb0, kb1;
+        kb_range(t, kb0, kb1);
         const uint32_t buf = it & 1u;
         if (!mbar_wait(tmem_empty0 + 8u * buf, ((it >> 1) & 1u) ^ 1u, wc)) break;
         tc_fence_after();
@@ -772,22 +804,36 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
     // ------------------------------------------------------------ factor-gradient epilogue
     const int q = warp & 3;        // TMEM lane quarter
     const int half = warp >> 2;    // column half of the tile
-    const LayerDev& L = args.L;
-    const int64_t cpr = L.K / args.P;
-    const int64_t plane = L.N * cpr;
-    const uint16_t* W = static_cast<const uint16_t*>(L.W);
+    const int64_t cpr = args.L.K / args.P;
+    const int64_t plane = args.L.N * cpr;
     const float k_sc = args.sc.s * args.sc.inv_2tanh_s;
     const float inv_k = (MU && k_sc > 0.0f) ? 1.0f / k_sc : 0.0f;
     uint32_t it = 0;
     for (int t = cluster; t < num_tiles; t += nclusters, ++it) {
       const int split = t / tiles_per_split, r = t % tiles_per_split;
       const int k_blk = r % args.num_k_tiles, n_blk = r / args.num_k_tiles;
+      // the tile's layer: the dense one, or (grouped) its expert's slice of the stacked layer
+      LayerDev L = args.L;
+      int64_t slab = split;  // which [3][N][K/P] partial block the tile writes
+      if constexpr (NE > 1) {
+        const int64_t e = gm.expert[split];
+        const int64_t G = L.N * L.groups_per_row;
+        L.W = static_cast<const uint16_t*>(L.W) + e * L.N * L.K;
+        L.mu0 += e * G;
+        L.alpha0 += e * G;
+        L.delta0 += e * G;
+        L.d_mu += e * G;
+        L.d_alpha += e * G;
+        L.d_delta += e * G;
+        slab = e;
+      }
+      const uint16_t* W = static_cast<const uint16_t*>(L.W);
       const uint32_t buf = it & 1u;
       if (!mbar_wait(tmem_full0 + 8u * buf, (it >> 1) & 1u, wc)) break;
       tc_fence_after();
       const int64_t n = (int64_t)n_blk * Cfg::kTileRows + cta * 128 + q * 32 + lane;
       const bool row_ok = n < L.N;
-      float* out = args.part + (int64_t)split * 3 * plane;
+      float* out = args.part + slab * 3 * plane;
       int64_t cur_j = -1;
       GroupConst gc{};
       GradSums acc{0.f, 0.f, 0.f};
@@ -1036,6 +1082,7 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
 template <int CG, bool MU>
 cudaError_t run_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M, const TcPlan& plan,
                    float* part, cudaStream_t st) {
+  static DwMaps<1> unused_maps;  // the dense kernel's (unread) grouped-map parameter
   using Cfg = DwCfg<CG>;
   DeviceInfo& d = device_info();
   if (!d.ok) return cudaErrorInvalidDevice;
@@ -1054,10 +1101,61 @@ cudaError_t run_dw(const LayerDev& L, StepScalars sc, const void* X, const void*
   args.num_n_tiles = static_cast<int32_t>((L.N + Cfg::kTileRows - 1) / Cfg::kTileRows);
   args.num_k_tiles = static_cast<int32_t>((L.K + BN - 1) / BN);
   args.wc = make_wait_ctl(d);
+  args.n_experts = 0;
   const int tiles = args.num_n_tiles * args.num_k_tiles * args.splits;
   const int clusters = std::min(tiles, d.sm_count / CG);
-  void* params[3] = {&tdy, &tx, &args};
-  return launch_persistent(dw_kernel<CG, MU>, CG, clusters * CG, Cfg::kThreads, Cfg::kSmemBytes, st, params);
+  void* params[4] = {&tdy, &tx, &args, &unused_maps};
+  return launch_persistent(dw_kernel<CG, MU, 1>, CG, clusters * CG, Cfg::kThreads, Cfg::kSmemBytes, st, params);
+}
+
+// Grouped dW: every expert with rows, kDwGroupExperts per launch; partials [E][3][N][K/P].
+template <int CG, bool MU>
+cudaError_t run_dw_grouped(const LayerDev& L0, StepScalars sc, const void* X, const void* dY, const GroupSpec& grp,
+                           int32_t P, float* part, cudaStream_t st) {
+  using Cfg = DwCfg<CG>;
+  DeviceInfo& d = device_info();
+  if (!d.ok) return cudaErrorInvalidDevice;
+  static std::mutex mu;  // the parameter block below is reused per call
+  std::lock_guard<std::mutex> lock(mu);
+  static DwMaps<kDwGroupExperts> gm;
+  CUtensorMap unused{};
+  DwArgs args;
+  args.L = L0;
+  args.sc = sc;
+  args.part = part;
+  args.M = 0;
+  args.splits = 1;
+  args.P = P;
+  args.kb_total = 0;
+  args.kb_per_split = 0;
+  args.num_n_tiles = static_cast<int32_t>((L0.N + Cfg::kTileRows - 1) / Cfg::kTileRows);
+  args.num_k_tiles = static_cast<int32_t>((L0.K + BN - 1) / BN);
+  const uint16_t* x = static_cast<const uint16_t*>(X);
+  const uint16_t* dy = static_cast<const uint16_t*>(dY);
+  int32_t e = 0;
+  while (e < grp.E) {
+    int n = 0;
+    for (; e < grp.E && n < kDwGroupExperts; ++e) {
+      const int64_t rows = grp.off[e + 1] - grp.off[e];
+      if (rows == 0) continue;
+      if (!make_tmap(&gm.dy[n], dy + grp.off[e] * L0.N, L0.N, rows, 64, BK) ||
+          !make_tmap(&gm.x[n], x + grp.off[e] * L0.K, L0.K, rows, 64, BK))
+        return cudaErrorInvalidValue;
+      gm.expert[n] = e;
+      gm.rows[n] = static_cast<int32_t>(rows);
+      ++n;
+    }
+    if (n == 0) break;
+    args.n_experts = n;
+    args.wc = make_wait_ctl(d);
+    const int tiles = args.num_n_tiles * args.num_k_tiles * n;
+    const int clusters = std::min(tiles, d.sm_count / CG);
+    void* params[4] = {&unused, &unused, &args, &gm};
+    const cudaError_t err = launch_persistent(dw_kernel<CG, MU, kDwGroupExperts>, CG, clusters * CG, Cfg::kThreads,
+                                              Cfg::kSmemBytes, st, params);
+    if (err != cudaSuccess) return err;
+  }
+  return cudaSuccess;
 }
 
 // Tile shape by M, and the W ~ alpha T + mu instantiation for such layers outside TEACHER.
@@ -1175,6 +1273,15 @@ cudaError_t launch_tc_dw(const LayerDev& L, StepScalars sc, const void* X, const
   }
   if (plan.dw_cg == 2) return run_dw<2, false>(L, sc, X, dY, M, plan, partials, st);
   return run_dw<1, false>(L, sc, X, dY, M, plan, partials, st);
+}
+
+cudaError_t launch_tc_dw_grouped(const LayerDev& L0, StepScalars sc, const void* X, const void* dY,
+                                 const GroupSpec& grp, int32_t P, float* partials, cudaStream_t st) {
+  const bool cg2 = L0.N >= 256;
+  if (L0.recon) return cg2 ? run_dw_grouped<2, true>(L0, sc, X, dY, grp, P, partials, st)
+                           : run_dw_grouped<1, true>(L0, sc, X, dY, grp, P, partials, st);
+  return cg2 ? run_dw_grouped<2, false>(L0, sc, X, dY, grp, P, partials, st)
+             : run_dw_grouped<1, false>(L0, sc, X, dY, grp, P, partials, st);
 }
 
 cudaError_t read_and_clear_device_status(int32_t* out) {
