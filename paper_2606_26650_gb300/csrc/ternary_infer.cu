@@ -97,17 +97,6 @@ __device__ __forceinline__ uint32_t magic_reg() {
   return m;
 }
 
-// Four 16-byte loads of read-only global data under a predicate (no branch); zeros when
-// the predicate is false.
-__device__ __forceinline__ uint4 ldg_pred(const uint4* p, bool pred) {
-  uint4 v = make_uint4(0u, 0u, 0u, 0u);
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.u32 p, %4, 0;\n @p ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%5];\n}"
-      : "+r"(v.x), "+r"(v.y), "+r"(v.z), "+r"(v.w)
-      : "r"(static_cast<uint32_t>(pred)), "l"(p));
-  return v;
-}
-
 // Activation pair (x[p], x[p + 8]) of 16 consecutive bf16 (h0 = elements 0..7, h1 = 8..15),
 // scaled by 4^-i of position p.
 template <int P>
@@ -208,8 +197,9 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const ui
         issue(n0, 0, 0);
         if (nslabs > 1) issue(n0, 1, 1);
       }
-      const bool tok_ok = b0 + gid < B;
-      const uint16_t* xrow = X + (tok_ok ? b0 + gid : 0) * K;
+      // Token columns past B read token b0's activations instead: their sums are computed
+      // and never stored, so no load needs a predicate.
+      const uint16_t* xrow = X + (b0 + gid < B ? b0 + gid : b0) * K;
       float acc[R][4], d[R][4], da[4];
 #pragma unroll
       for (int r = 0; r < R; ++r)
@@ -239,20 +229,27 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const ui
         int32_t grp = (slab * sc_per_slab + lo) / sc_per_group;
         int32_t left = (grp + 1) * sc_per_group - (slab * sc_per_slab + lo);  // super-chunks to its end
         const uint32_t tile = ring_base + buf * ROWS * row_bytes;
-        auto load_x = [&](int32_t sc, uint4 (&xv)[2 * VW]) {
-          const uint4* xp = reinterpret_cast<const uint4*>(xrow + k0 + sc * 64 * VW + 16 * VW * q);
+        // per-thread bases, advanced by the super-chunk index inside the loop
+        uint32_t rowa[R][2];  // shared-memory address of the thread's words in each of its rows
 #pragma unroll
-          for (int i = 0; i < 2 * VW; ++i) xv[i] = ldg_pred(xp + i, tok_ok);
+        for (int r = 0; r < R; ++r)
+#pragma unroll
+          for (int h = 0; h < 2; ++h) rowa[r][h] = tile + (16 * r + gid + 8 * h) * row_bytes + VW * q * 4;
+        const uint4* xbase = reinterpret_cast<const uint4*>(xrow + k0 + 16 * VW * q);
+        const bool every_sc = sc_per_group == 1;  // each super-chunk is a whole group
+        auto load_x = [&](int32_t sc, uint4 (&xv)[2 * VW]) {
+          const uint4* xp = xbase + sc * (8 * VW);
+#pragma unroll
+          for (int i = 0; i < 2 * VW; ++i) xv[i] = __ldg(xp + i);
         };
         // one super-chunk: this thread's code words from shared memory, its activations xv
         auto step = [&](int32_t sc, const uint4 (&xv)[2 * VW]) {
-          const uint32_t woff = static_cast<uint32_t>((sc * 4 * VW + VW * q) * 4);
+          const uint32_t woff = static_cast<uint32_t>(sc * 16 * VW);
           uint32_t cw[R][2][VW];  // the thread's code words of rows gid and gid + 8 of each tile
 #pragma unroll
           for (int r = 0; r < R; ++r) {
-            const uint32_t a = tile + (16 * r + gid) * row_bytes + woff;
-            ld_shared_words<VW>(a, cw[r][0]);
-            ld_shared_words<VW>(a + 8 * row_bytes, cw[r][1]);
+            ld_shared_words<VW>(rowa[r][0] + woff, cw[r][0]);
+            ld_shared_words<VW>(rowa[r][1] + woff, cw[r][1]);
           }
 #pragma unroll
           for (int v = 0; v < VW; ++v) {
@@ -280,7 +277,7 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const ui
               word_mma<3>(d[r], s0, s1, xb);
             }
           }
-          if (--left == 0 || sc + 1 == hi) {  // the group, or this warp's range, ends
+          if (every_sc || --left == 0 || sc + 1 == hi) {  // the group, or this warp's range, ends
 #pragma unroll
             for (int r = 0; r < R; ++r) {
               const float a0 = __ldg(alpha + goff[r][0] + grp), a1 = __ldg(alpha + goff[r][1] + grp);
@@ -300,7 +297,9 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const ui
             }
 #pragma unroll
             for (int e = 0; e < 4; ++e) da[e] = 0.0f;
-            if (left == 0) {
+            if (every_sc) {
+              ++grp;
+            } else if (left == 0) {
               ++grp;
               left = sc_per_group;
             }
