@@ -55,7 +55,7 @@ def parse(argv=None):
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-also", action="store_true", help="skip the secondary workloads and phase")
-    p.add_argument("--streams", type=int, default=2,
+    p.add_argument("--streams", type=int, default=4,
                    help="CUDA streams the block's linears are spread over (independent problems)")
     return p.parse_args(argv)
 
