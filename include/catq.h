@@ -255,16 +255,25 @@ typedef struct {
                       catq_layer.op_const */
 } catq_grouped_layer;
 
-/* Forward of every expert: Y[rows of e] = X[rows of e] Wq_e^T (Eq. 6 weight per expert). */
+/* Forward of every expert: Y[rows of e] = X[rows of e] Wq_e^T (Eq. 6 weight per expert).
+ * bf16 layers with at most 128 experts and fewer than 2^31 rows run as one persistent
+ * launch over every expert's tiles (X, Y 16-byte aligned; op_const as for dense layers);
+ * other layers, expert by expert.  Calls on one layer must not overlap on the GPU (they
+ * rewrite op_const). */
 catq_status catq_grouped_soft_ternary_linear_fwd(const catq_grouped_layer* layer, catq_schedule sched,
                                                  const void* X, const int64_t* row_offsets,
                                                  int32_t x_dtype, void* Y, catq_stream stream);
 
-/* Workspace bytes catq_grouped_soft_ternary_linear_bwd needs (the largest expert's). */
+/* Workspace bytes catq_grouped_soft_ternary_linear_bwd needs: for bf16 layers with at most
+ * 128 experts, every expert's partial group sums at once (E * 3 * N * K/gcd(g, 128) fp32);
+ * otherwise the largest expert's catq_bwd_workspace_bytes. */
 size_t catq_grouped_bwd_workspace_bytes(const catq_grouped_layer* layer, const int64_t* row_offsets);
 
 /* Backward of every expert (see catq_soft_ternary_linear_bwd): dX [R, K] (nullable) and the
- * factor gradients [E, G] (all three or none). */
+ * factor gradients [E, G] (all three or none).  For bf16 layers with at most 128 experts,
+ * dX runs as one launch over every expert's tiles and the factor gradients as launches of
+ * up to 64 experts with rows each (each expert's contraction stops at its last row) plus
+ * one reduction; otherwise expert by expert. */
 catq_status catq_grouped_soft_ternary_linear_bwd(const catq_grouped_layer* layer, catq_schedule sched,
                                                  const void* X, const void* dY,
                                                  const int64_t* row_offsets, int32_t x_dtype,
