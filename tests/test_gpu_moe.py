@@ -101,3 +101,58 @@ def test_moe_grouped_matches_oracle(device, lin_name, phase, s):
     empty = np.nonzero(counts == 0)[0]
     for e in empty:
         assert not U.to_host(gr[0])[e * G:(e + 1) * G].any()
+
+
+@pytest.mark.parametrize("E", [128, 130])
+def test_many_small_experts(device, E):
+    """Many experts with a handful of rows each (some none): 128 experts run as grouped
+    launches (dW in two launches of 64), 130 take the expert-by-expert path; both against
+    the oracle."""
+    import torch
+
+    from paper_2606_26650_gb300 import catq as C
+    N, K, g = 256, 512, 128
+    r = syn.rng(11, f"moe/many/{E}")
+    counts = r.integers(0, 9, size=E)
+    counts[::7] = 0
+    off = np.concatenate([[0], np.cumsum(counts)]).astype(np.int64)
+    R = int(off[-1])
+    W = syn.round_bf16((r.standard_normal((E, N, K)) * 0.02).astype(np.float32))
+    X = syn.round_bf16(r.standard_normal((R, K)).astype(np.float32))
+    dY = syn.round_bf16((r.standard_normal((R, N)) * 1e-2).astype(np.float32))
+    G = N * K // g
+    fac = syn.factors(E * G, 11, f"moe/many/{E}", perturbed=True)
+    phase, s = O.PHASE_SOFT, 30.0
+    Wt = U.to_device(W.reshape(E * N, K), "bf16", device).reshape(E, N, K)
+    layer = C.GroupedLayer.create(Wt, g, *(torch.from_numpy(f).to(device) for f in fac))
+    C.catq_group_stats(layer.dense)
+    Xt, dYt = U.to_device(X, "bf16", device), U.to_device(dY, "bf16", device)
+    Y = torch.empty(R, N, dtype=torch.bfloat16, device=device)
+    C.catq_grouped_soft_ternary_linear_fwd(layer, C.schedule(phase, s), Xt, off, Y)
+    dX = torch.empty_like(Xt)
+    gr = [torch.full((E * G,), 7.0, device=device) for _ in range(3)]
+    ws = C.workspace(C.catq_grouped_bwd_workspace_bytes(layer, off), device)
+    C.catq_grouped_soft_ternary_linear_bwd(layer, C.schedule(phase, s), Xt, dYt, off, dX, *gr, ws)
+    torch.cuda.synchronize()
+    assert C.catq_device_status() == 0
+    Yh, dXh = U.to_host(Y), U.to_host(dX)
+    grh = [U.to_host(t) for t in gr]
+    Y_ref, dX_ref = np.zeros((R, N)), np.zeros((R, K))
+    g_ref = [np.zeros(E * G) for _ in range(3)]
+    for e in range(E):
+        rows = slice(int(off[e]), int(off[e + 1]))
+        st = O.group_stats(W[e], g)
+        fe = tuple(f[e * G:(e + 1) * G] for f in fac)
+        Wq = O.ternary_weight(W[e], g, st, fe, phase, s)[0]
+        Y_ref[rows] = O.linear_fwd(X[rows], Wq)
+        dxe, *ge = O.linear_bwd(X[rows], dY[rows], W[e], g, st, fe, phase, s)
+        dX_ref[rows] = dxe
+        for dst, src in zip(g_ref, ge):
+            dst[e * G:(e + 1) * G] = src
+    errs = {"Y": U.fro_rel(Yh, Y_ref), "dX": U.fro_rel(dXh, dX_ref)}
+    for name, got, want in zip(("g_dmu", "g_dalpha", "g_ddelta"), grh, g_ref):
+        errs[name] = U.fro_rel(got, want)
+    bad = {k: v for k, v in errs.items() if not v <= U.TOL_BF16}
+    assert not bad, errs
+    for e in np.nonzero(counts == 0)[0]:
+        assert not grh[0][e * G:(e + 1) * G].any() and not grh[2][e * G:(e + 1) * G].any()
