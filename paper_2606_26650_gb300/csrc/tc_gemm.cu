@@ -84,8 +84,10 @@ struct FusedCfg {
   static constexpr int kRawBars = kProdGroups * kStagesW;
   static_assert(kRawBars <= 32, "issued-barrier masks are 32 bits");
   static constexpr int kRowsPerWarp = 32 / kThreadsPerRow;     // operand rows one producer warp owns
-  static constexpr int kBarBytes = 8 * (2 * kStagesA + kRawBars + 3 * kStagesW + 3) + 16;
+  static constexpr int kBarBytes = 8 * (2 * kStagesA + kRawBars + 3 * kStagesW + 2 * NACC + 1) + 16;
   static constexpr int kSmemBytes = kStagesA * kABytes + kStagesW * kWBytes + 1024 + kBarBytes;
+  // Stages the MMA issuer holds at a tile's edges (see the issuer), bounded by both rings.
+  static constexpr int kHold = (kStagesA < kStagesW ? kStagesA : kStagesW) - 1;
 };
 
 template <int CG>
@@ -332,10 +334,12 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
   auto full_w = [&](int s) { return bars + 8u * (2 * SA + RB + s); };   // operand ready (pair: even CTA)
   auto empty_w = [&](int s) { return bars + 8u * (2 * SA + RB + SW + s); };
   auto recv_w = [&](int s) { return bars + 8u * (2 * SA + RB + 2 * SW + s); };  // PAIRS 2: received half landed
-  const uint32_t tmem_full_bar = bars + 8u * (2 * SA + RB + 3 * SW);
-  const uint32_t tmem_empty_bar = tmem_full_bar + 8;
-  const uint32_t final_bar = tmem_full_bar + 16;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base_ptr + (bars - base) + 8 * (2 * SA + RB + 3 * SW + 3));
+  // one full/empty pair per accumulator: a tile's accumulators drain and refill separately
+  const uint32_t tmem_full0 = bars + 8u * (2 * SA + RB + 3 * SW);     // [NACC]
+  const uint32_t tmem_empty0 = tmem_full0 + 8u * NACC;                // [NACC]
+  const uint32_t final_bar = tmem_empty0 + 8u * NACC;
+  uint32_t* tmem_slot =
+      reinterpret_cast<uint32_t*>(base_ptr + (bars - base) + 8 * (2 * SA + RB + 3 * SW + 2 * NACC + 1));
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = CG == 2 ? cluster_ctarank() : 0u;
@@ -369,8 +373,10 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
       // current use has landed; this arms the first use.
       if (received) mbar_arrive_expect_tx(cta == 0 ? full_w(s) : recv_w(s), Cfg::kWBytes);
     }
-    mbar_init(tmem_full_bar, 1);
-    mbar_init(tmem_empty_bar, Cfg::kEpiWarps * CG);
+    for (int a = 0; a < NACC; ++a) {
+      mbar_init(tmem_full0 + 8u * a, 1);
+      mbar_init(tmem_empty0 + 8u * a, Cfg::kEpiWarps * CG);
+    }
     mbar_init(final_bar, 1);
     fence_mbar_init_cluster();
   }
@@ -386,7 +392,7 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
   // Barriers a whole pair signals live in the pair's even CTA.
   const uint32_t leader_full_a0 = CG == 2 ? mapa_shared(full_a(0), leader) : full_a(0);
   const uint32_t leader_full_w0 = CG == 2 ? mapa_shared(full_w(0), leader) : full_w(0);
-  const uint32_t leader_tmem_empty = CG == 2 ? mapa_shared(tmem_empty_bar, leader) : tmem_empty_bar;
+  const uint32_t leader_tmem_empty0 = CG == 2 ? mapa_shared(tmem_empty0, leader) : tmem_empty0;
   const uint16_t pair_mask = static_cast<uint16_t>(3u << (2 * pair));
   const uint16_t all_mask = static_cast<uint16_t>((1u << Cfg::kClusterCtas) - 1u);
 
@@ -450,40 +456,82 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     // ------------------------------------------------------------ MMA issuer (even CTA of each pair)
     if (cta == 0 && lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(Cfg::kRowsPerAcc, BN, false, B_MN);
+      const int T = args.num_k_blocks;
+      // Accumulators drain and refill separately, so the epilogue overlaps the MMAs: a tile's
+      // last J stages run accumulator 0 first (the epilogue drains it while accumulator 1
+      // finishes), and the next tile's first J stages start accumulator 0 as soon as it is
+      // drained (accumulator 1 follows once it is).  Those stages stay held in between.
+      const int J = min(Cfg::kHold, T / 2);
       uint32_t q = 0, it = 0;
       bool ok = true;
-      for (int t = cluster; ok && t < num_tiles; t += nclusters, ++it) {
-        if (!mbar_wait(tmem_empty_bar, (it & 1u) ^ 1u, wc)) break;
+      auto stage_in = [&](uint32_t qq) -> bool {  // wait for stage qq; arm a received slot's next use
+        const uint32_t sa = qq % SA, pa = (qq / SA) & 1u, sw = qq % SW, pw = (qq / SW) & 1u;
+        if (!mbar_wait(full_a(sa), pa, wc) || !mbar_wait(full_w(sw), pw, wc)) return false;
+        if (PAIRS == 2 && (qq & 1u) != pair) mbar_arrive_expect_tx(full_w(sw), Cfg::kWBytes);
         tc_fence_after();
-        for (int kb = 0; kb < args.num_k_blocks; ++kb, ++q) {
-          const uint32_t sa = q % SA, pa = (q / SA) & 1u, sw = q % SW, pw = (q / SW) & 1u;
-          if (!mbar_wait(full_a(sa), pa, wc) || !mbar_wait(full_w(sw), pw, wc)) { ok = false; break; }
-          // Received stage: both halves are here; arm the slot's next use.
-          if (PAIRS == 2 && (q & 1u) != pair) mbar_arrive_expect_tx(full_w(sw), Cfg::kWBytes);
-          tc_fence_after();
-          const uint32_t aa = a_base + sa * Cfg::kABytes, ww = w_base + sw * Cfg::kWBytes;
+        return true;
+      };
+      auto issue = [&](uint32_t qq, int acc, bool first) {  // one accumulator's MMAs of stage qq
+        const uint32_t aa = a_base + (qq % SA) * Cfg::kABytes, ww = w_base + (qq % SW) * Cfg::kWBytes;
 #pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t bdesc = B_MN ? smem_desc_sw128(ww + kk * 2048, 8192, 1024)
-                                        : smem_desc_sw128(ww + kk * 32, 16, 1024);
-#pragma unroll
-            for (int acc = 0; acc < NACC; ++acc) {
-              const uint64_t adesc = smem_desc_sw128(aa + acc * (128 * BK * 2) + kk * 32, 16, 1024);
-              umma_bf16<CG>(tmem_base + acc * BN, adesc, bdesc, idesc, (kb | kk) != 0 ? 1u : 0u);
-            }
-          }
-          if constexpr (PAIRS == 1) {
-            umma_commit<CG>(empty_a(sa));
-            umma_commit<CG>(empty_w(sw));
-          } else {
-            umma_commit_pair_mask(empty_a(sa), pair_mask);
-            umma_commit_pair_mask(empty_w(sw), all_mask);
-          }
+        for (int kk = 0; kk < BK / 16; ++kk) {
+          const uint64_t bdesc = B_MN ? smem_desc_sw128(ww + kk * 2048, 8192, 1024)
+                                      : smem_desc_sw128(ww + kk * 32, 16, 1024);
+          const uint64_t adesc = smem_desc_sw128(aa + acc * (128 * BK * 2) + kk * 32, 16, 1024);
+          umma_bf16<CG>(tmem_base + acc * BN, adesc, bdesc, idesc, (first && kk == 0) ? 0u : 1u);
         }
-        if (ok) {
-          if constexpr (PAIRS == 1) umma_commit<CG>(tmem_full_bar);
-          else umma_commit_pair_mask(tmem_full_bar, pair_mask);
+      };
+      auto release = [&](uint32_t qq) {  // both accumulators are done with stage qq
+        if constexpr (PAIRS == 1) {
+          umma_commit<CG>(empty_a(qq % SA));
+          umma_commit<CG>(empty_w(qq % SW));
+        } else {
+          umma_commit_pair_mask(empty_a(qq % SA), pair_mask);
+          umma_commit_pair_mask(empty_w(qq % SW), all_mask);
         }
+      };
+      auto full = [&](int acc) {
+        if constexpr (PAIRS == 1) umma_commit<CG>(tmem_full0 + 8u * acc);
+        else umma_commit_pair_mask(tmem_full0 + 8u * acc, pair_mask);
+      };
+      for (int t = cluster; ok && t < num_tiles; t += nclusters, ++it) {
+        const uint32_t ep = (it & 1u) ^ 1u;  // the epilogue has drained the previous tile's accumulator
+        // head: accumulator 0 over stages 0 .. J-1
+        if (!mbar_wait(tmem_empty0, ep, wc)) break;
+        tc_fence_after();
+        for (int h = 0; ok && h < J; ++h) {
+          if (!stage_in(q + h)) { ok = false; break; }
+          issue(q + h, 0, h == 0);
+        }
+        if (!ok || !mbar_wait(tmem_empty0 + 8u * (NACC - 1), ep, wc)) break;
+        tc_fence_after();
+        for (int h = 0; h < J; ++h) {
+          issue(q + h, 1, h == 0);
+          release(q + h);
+        }
+        q += J;
+        // body: both accumulators per stage
+        for (int kb = J; kb < T - J; ++kb, ++q) {
+          if (!stage_in(q)) { ok = false; break; }
+          issue(q, 0, kb == 0);
+          issue(q, 1, kb == 0);
+          release(q);
+        }
+        if (!ok) break;
+        // tail: accumulator 0 over the last J stages, which the epilogue then drains while
+        // accumulator 1 finishes them
+        for (int h = 0; ok && h < J; ++h) {
+          if (!stage_in(q + h)) { ok = false; break; }
+          issue(q + h, 0, false);
+        }
+        if (!ok) break;
+        full(0);
+        for (int h = 0; h < J; ++h) {
+          issue(q + h, 1, false);
+          release(q + h);
+        }
+        q += J;
+        full(1);
       }
       if constexpr (PAIRS == 1) umma_commit<CG>(final_bar);
       else umma_commit_pair_mask(final_bar, pair_mask);
@@ -508,12 +556,13 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     // ------------------------------------------------------------ epilogue
     const int qd = warp;  // TMEM lane quarter
     uint32_t it = 0;
-    for (int t = cluster; t < num_tiles; t += nclusters, ++it) {
+    bool ok = true;
+    for (int t = cluster; ok && t < num_tiles; t += nclusters, ++it) {
       const TileInfo ti = tile_info(args, t, Cfg::kTileRows * PAIRS);
-      if (!mbar_wait(tmem_full_bar, it & 1u, wc)) break;
-      tc_fence_after();
 #pragma unroll 1
       for (int acc = 0; acc < NACC; ++acc) {
+        if (!mbar_wait(tmem_full0 + 8u * acc, it & 1u, wc)) { ok = false; break; }
+        tc_fence_after();
         const int64_t row0 = ti.row0 + pair * Cfg::kTileRows + acc * Cfg::kRowsPerAcc + cta * 128 +
                              qd * 32;  // this warp's first row
 #pragma unroll 1
@@ -525,10 +574,11 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
           tmem_ld_wait();
           store_rows_bf16x32(args.C, ti.row_end, args.ncols, row0, col, r, lane);
         }
+        // this accumulator is drained: the MMA may refill it
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(leader_tmem_empty0 + 8u * acc);
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(leader_tmem_empty);
     }
   } else {
     // ------------------------------------------------------------ operand producers
