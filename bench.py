@@ -601,11 +601,14 @@ def measure_moe(C, torch, dev, peaks, world, s, steps=5, warmup=2):
         step()
     torch.cuda.synchronize()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record()
-    for _ in range(steps):
-        step()
-    b.record()
-    torch.cuda.synchronize()
+    with ClockSampler(dev.index or 0) as clk:
+        a.record()
+        h0 = time.perf_counter()
+        for _ in range(steps):
+            step()
+        host_ms = (time.perf_counter() - h0) * 1e3 / steps  # issuing the calls, per step
+        b.record()
+        torch.cuda.synchronize()
     status = C.catq_device_status()
     if status != 0:
         raise SystemExit(f"device status {C.STATUS.get(status, status)} in the MoE timing")
@@ -617,7 +620,9 @@ def measure_moe(C, torch, dev, peaks, world, s, steps=5, warmup=2):
     return {"value": value, "ms_per_step": ms, "frac_of_burst": value / world / peaks["bf16"], "steps": steps,
             "experts": E, "routed_rows": R, "rows_per_expert": [int(counts.min()), int(np.median(counts)),
                                                                  int(counts.max())],
-            "path": "grouped calls: one persistent launch for every expert's forward and dX tiles, factor gradients expert by expert", "phase": "soft", "s": s}
+            "path": "grouped calls: one persistent launch for every expert's forward and dX tiles, grouped "
+                    "factor-gradient launches of up to 64 experts",
+            "phase": "soft", "s": s, "host_issue_ms_per_step": host_ms, "clocks": clk.summary()}
 
 
 def measure_e2e(args, C, torch, st, step, barrier, flops_step, world, dev):

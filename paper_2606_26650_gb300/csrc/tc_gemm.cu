@@ -25,6 +25,7 @@
 #include <cudaTypedefs.h>
 
 #include <atomic>
+#include <map>
 #include <mutex>
 #include <numeric>
 #include <type_traits>
@@ -1042,16 +1043,20 @@ cudaError_t launch_persistent(Kern kern, int cg, int grid_ctas, int threads, int
   return cudaLaunchKernelExC(&cfg, reinterpret_cast<const void*>(kern), params);
 }
 
-// Largest number of co-resident clusters of `cluster_ctas` CTAs for a kernel (cached per
-// device); a persistent grid larger than this would run a second, partial wave.
+// Largest number of co-resident clusters of `cluster_ctas` CTAs for a kernel, cached per
+// (device, kernel); a persistent grid larger than this would run a second, partial wave.
+// (The kernel variants share one function type, so the cache is keyed by the kernel's
+// address, not by the template instance.)
 template <typename Kern>
 int max_active_clusters(Kern kern, int cluster_ctas, int threads, int smem, int fallback) {
   static std::mutex mu;
-  static int cache[64] = {};
+  static std::map<std::pair<int, const void*>, int> cache;
   int dev = 0;
   cudaGetDevice(&dev);
+  const std::pair<int, const void*> key{dev, reinterpret_cast<const void*>(kern)};
   std::lock_guard<std::mutex> lock(mu);
-  if (cache[dev & 63] > 0) return cache[dev & 63];
+  const auto hit = cache.find(key);
+  if (hit != cache.end()) return hit->second;
   cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(cluster_ctas * 64);
@@ -1067,7 +1072,7 @@ int max_active_clusters(Kern kern, int cluster_ctas, int threads, int smem, int 
   int n = 0;
   if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(kern), &cfg) != cudaSuccess || n <= 0)
     n = fallback;
-  cache[dev & 63] = n;
+  cache[key] = n;
   return n;
 }
 
