@@ -36,6 +36,10 @@ DEFAULT_WORKLOAD = "c3_llama3_8b_block"
 CPU_SAMPLE_LINEARS = ("q_proj", "k_proj", "down_proj")  # cpu_baseline leg of our arm
 CPU_SAMPLE_ROWS = 256
 REF_STEP_LINEARS = ("k_proj",)  # one step of the reference arm (runs K + W times)
+# App. B.1: AdamW on the factors at learning rate 1e-3, decayed linearly to zero over 60
+# epochs of ceil(512 / 3) batches of three 2048-token samples.
+LR0 = 1e-3
+UPDATES = 60 * -(-512 // 3)
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per launch, mean over the
 # seven linears of the 8B-shaped block step, from one ncu capture of the timed step; keyed
@@ -88,7 +92,8 @@ def measured_peaks():
 
 def oracle_sample(wl, s, rows=CPU_SAMPLE_ROWS, linears=CPU_SAMPLE_LINEARS):
     """Times the fp64 oracle on a bounded sample of the workload: the named linears at
-    `rows` tokens, every hot-path row (stats, fwd, loss, dX, factor gradients, pack).
+    `rows` tokens, every hot-path row (stats, fwd, loss, dX, factor gradients, factor
+    update, pack).
     Returns (seconds, algorithmic flops)."""
     from oracle import catq_oracle as O
     total_t, flops = 0.0, 0.0
@@ -104,7 +109,8 @@ def oracle_sample(wl, s, rows=CPU_SAMPLE_ROWS, linears=CPU_SAMPLE_LINEARS):
         Wq = O.ternary_weight(W, wl.g, stats, fac, O.PHASE_SOFT, s)[0]
         Y = O.linear_fwd(X, Wq)
         _, dY = O.recon_loss(Y, Y_ref)
-        O.linear_bwd(X, dY, W, wl.g, stats, fac, O.PHASE_SOFT, s)
+        grads = O.linear_bwd(X, dY, W, wl.g, stats, fac, O.PHASE_SOFT, s)[1:]
+        fac, _ = O.factor_update(fac, grads, (np.zeros(G),) * 6, 1, LR0)
         T, _, _ = O.hard_codes(W, wl.g, stats, fac)
         O.pack_codes(T)
         total_t += time.perf_counter() - t0
@@ -138,8 +144,8 @@ def cpu_cores():
 
 def sample_text(wl, rows=CPU_SAMPLE_ROWS, linears=CPU_SAMPLE_LINEARS):
     return (f"{'+'.join(linears)} of {wl.name} at {rows} of {wl.M} tokens, fp64 numpy oracle, all hot-path rows "
-            f"(stats, fwd, loss, dX, factor grads, pack); matmuls on multi-threaded BLAS, elementwise "
-            f"single-threaded; per-layer modulation cost is paid once per sample, as in the full step")
+            f"(stats, fwd, loss, dX, factor grads, AdamW factor update, pack); matmuls on multi-threaded BLAS, "
+            f"elementwise single-threaded; per-layer modulation cost is paid once per sample, as in the full step")
 
 
 def run_reference(args):
@@ -234,6 +240,25 @@ KINDS = ("fwd", "dx", "dw")
 ALSO_WORKLOADS = ("c4_qwen3_14b_block", "c2_qwen3_1p7b_block")
 
 
+class FactorUpdate:
+    """The optimizer step closing each calibration step: AdamW on every linear's three
+    factors (moments zero at the start) at the linearly decayed learning rate of the update
+    count; the count wraps after a full calibration's updates."""
+
+    def __init__(self, C, torch, dev, group_counts):
+        self.C, self.hp, self.t, self.lr = C, C.adamw(), 0, LR0
+        # zeros copied from the host: no fill kernel among the step's launches
+        self.moments = [torch.zeros(6 * G).to(dev) for G in group_counts]
+
+    def advance(self):
+        self.t += 1
+        self.lr = self.C.catq_linear_decay_lr(LR0, (self.t - 1) % UPDATES, UPDATES)
+
+    def apply(self, i, layer, grads):
+        self.C.catq_factor_adamw_step(layer.d_mu, layer.d_alpha, layer.d_delta, *grads, self.moments[i], self.hp,
+                                      self.t, self.lr)
+
+
 class BlockRun:
     """Device state and one calibration step of a block workload: every linear's seeded
     inputs, layer and teacher output, and per-stream workspaces.
@@ -274,6 +299,7 @@ class BlockRun:
             ws_bwd = max(ws_bwd, C.catq_bwd_workspace_bytes(layer, M))
             ws_loss = max(ws_loss, C.catq_recon_loss_workspace_bytes(M * lin.N))
             self.st.append(d)
+        self.upd = FactorUpdate(C, torch, dev, [d["grads"][0].numel() for d in self.st])
         self.main = torch.cuda.current_stream()
         self.lanes = [self.main] if nstreams == 1 else [torch.cuda.Stream(device=dev) for _ in range(nstreams)]
         self.wsbs = [C.workspace(ws_bwd, dev) for _ in self.lanes]
@@ -286,6 +312,7 @@ class BlockRun:
         kernels (e2e copies); ev[i][kind] are (start, end) events around each GEMM call."""
         C, torch, wl = self.C, self.torch, self.wl
         use = [self.main] if serial else self.lanes
+        self.upd.advance()
         if len(use) > 1:
             fork = torch.cuda.Event()
             fork.record(self.main)
@@ -313,6 +340,7 @@ class BlockRun:
                 C.catq_soft_ternary_linear_bwd(L, sched, d["X"], d["dY"], None, *d["grads"], workspace=self.wsbs[k])
                 if ev is not None:
                     ev[i]["dw"][1].record()
+                self.upd.apply(i, L, d["grads"])
                 C.catq_hard_ternarize_pack(L, d["codes"], d["alpha"])
                 if after is not None:
                     after(i)
@@ -364,8 +392,8 @@ def run_ours(args):
         blk.step(sched, ev, serial, before, after)
 
     # per linear: stats; operand constants + forward; loss (partial + final); operand
-    # constants + dX; dW + gradient reduce; pack
-    launches_per_step = len(st) * (1 + 2 + 2 + 2 + 2 + 1)
+    # constants + dX; dW + gradient reduce; factor update; pack
+    launches_per_step = len(st) * (1 + 2 + 2 + 2 + 2 + 1 + 1)
 
     def barrier():
         torch.cuda.synchronize()
@@ -557,7 +585,7 @@ def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20, with_m
 def measure_moe(C, torch, dev, peaks, world, s, steps=5, warmup=2):
     """One calibration step of the Qwen3-235B-shaped MoE layer: gate/up/down of all 128
     experts over 8192 tokens routed top-8 (65,536 expert-sorted rows, Zipf(1.1) loads) through
-    the grouped calls (stats once; per step forward, loss, backward, pack).  Weights and
+    the grouped calls (stats once; per step forward, loss, backward, factor update, pack).  Weights and
     activations are drawn on the device (seeded); value = sum 6 M_e N K / step time."""
     wl = syn.WORKLOADS["c5_qwen3_235b_moe"]
     token_of_row, off = syn.moe_routing(wl, seed=0)
@@ -588,13 +616,16 @@ def measure_moe(C, torch, dev, peaks, world, s, steps=5, warmup=2):
                          wsb=C.workspace(C.catq_grouped_bwd_workspace_bytes(layer, off), dev),
                          wsl=C.workspace(C.catq_recon_loss_workspace_bytes(R * N), dev)))
         flops += 6.0 * R * N * K
+    upd = FactorUpdate(C, torch, dev, [d["grads"][0].numel() for d in lins])
 
     def step():
-        for d in lins:
+        upd.advance()
+        for i, d in enumerate(lins):
             C.catq_grouped_soft_ternary_linear_fwd(d["layer"], sched, d["X"], off, d["Y"])
             C.catq_recon_loss(d["Y"], d["Yt"], d["loss"], d["dY"], d["wsl"])
             C.catq_grouped_soft_ternary_linear_bwd(d["layer"], sched, d["X"], d["dY"], off, d["dX"], *d["grads"],
                                                    workspace=d["wsb"])
+            upd.apply(i, d["layer"].dense, d["grads"])
             C.catq_hard_ternarize_pack(d["layer"].dense, d["codes"], d["alpha"])
 
     for _ in range(warmup):

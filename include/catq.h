@@ -229,6 +229,53 @@ catq_status catq_recon_loss(const void* Y, const void* Y_ref, int64_t count, int
 catq_status catq_hard_ternarize_pack(const catq_layer* layer, uint8_t* codes, float* alpha, float* mu,
                                      catq_stream stream);
 
+/* ------------------------------------------------------------------ calibration schedule and update
+ * App. B.1 calibrates the learnable factors with AdamW for m = 60 epochs at learning rate
+ * 1e-3 decayed linearly to zero, gamma = 0.8, s0 = 30; §2.3 maps the normalised epoch t to
+ * the branch and sharpness of Eq. 6.  These calls give a calibration loop what it needs
+ * beyond the step itself. */
+
+/* Eq. 6's schedule point of calibration epoch e of m (host only, no device work):
+ * t = e / m; e == 0 is the teacher branch (t = 0); e <= floor(gamma m + 1e-9) the soft
+ * stage with s = (t / gamma) s0; later epochs the hard stage with the backward sharpness s0
+ * (the last soft value, §2.3).  Requires 0 <= e <= m, m >= 1, 0 < gamma <= 1, finite
+ * s0 > 0 and a non-null `out`; else CATQ_ERR_INVALID_ARG. */
+catq_status catq_schedule_at_epoch(int32_t e, int32_t m, double gamma, double s0, catq_schedule* out);
+
+/* Learning rate of update k (0-based) of `total` under App. B.1's linear decay to zero
+ * (host only): lr0 (1 - k / total).  Requires 0 <= k < total, finite lr0 >= 0 and a
+ * non-null `lr_out`; else CATQ_ERR_INVALID_ARG. */
+catq_status catq_linear_decay_lr(double lr0, int64_t k, int64_t total, float* lr_out);
+
+/* AdamW hyperparameters beyond the learning rate (App. B.1 names the optimizer only). */
+typedef struct {
+  float beta1;        /* first-moment decay, 0 <= beta1 < 1 (the optimizer's usual 0.9) */
+  float beta2;        /* second-moment decay, 0 <= beta2 < 1 (0.999) */
+  float eps;          /* added to sqrt(v_hat), finite and > 0 (1e-8) */
+  float weight_decay; /* decoupled decay, scaled by the learning rate, >= 0 (0: a decay of the
+                         factors towards zero would shrink alpha and Delta) */
+  float margin;       /* projection margin of §2.2's constraints, 0 <= margin < 0.5 */
+} catq_adamw;
+
+/* The update of the learnable factors after a calibration step: for each of d_mu, d_alpha,
+ * d_delta (in place, [G] fp32 device) with its gradient ([G] fp32 device, e.g. the output
+ * of catq_soft_ternary_linear_bwd), one AdamW step (Loshchilov & Hutter's decoupled weight
+ * decay, Adam's bias-corrected moments, update count t >= 1):
+ *   p <- p (1 - lr weight_decay)
+ *   m <- beta1 m + (1 - beta1) grad,  v <- beta2 v + (1 - beta2) grad^2
+ *   p <- p - (lr / (1 - beta1^t)) m / (sqrt(v) / sqrt(1 - beta2^t) + eps)
+ * then the projection of §2.2's constraints -1 < d_mu < 1, d_alpha > 0, d_delta > 0 onto
+ * [-1 + margin, 1 - margin], [margin, inf), [margin, inf) (NaN passes through unchanged).
+ * moments: [6, G] fp32 device, the optimizer state m_mu, m_alpha, m_delta, v_mu, v_alpha,
+ * v_delta, zero before the first update and updated in place.  fp32 arithmetic with
+ * IEEE division and square root.  For a stacked MoE layer pass G = E * groups per expert.
+ * G == 0 is a no-op whatever the pointers.  Pointers 4-byte aligned.  Errors: G < 0 CATQ_ERR_SHAPE; a null
+ * pointer, t < 1, a negative or non-finite lr or out-of-range hyperparameters
+ * CATQ_ERR_INVALID_ARG. */
+catq_status catq_factor_adamw_step(int64_t G, float* d_mu, float* d_alpha, float* d_delta, const float* g_dmu,
+                                   const float* g_dalpha, const float* g_ddelta, float* moments,
+                                   const catq_adamw* hp, int64_t t, float lr, catq_stream stream);
+
 /* ------------------------------------------------------------------ grouped (MoE) layers
  * A mixture-of-experts layer quantizes every expert's linear like a dense one (App. B.2:
  * experts are quantized, routers are not).  E experts of identical shape are stacked:

@@ -264,3 +264,79 @@ def unpack_codes(codes, n):
     for i in range(4):
         T[i::4] = ((codes >> (2 * i)) & 3) - 1
     return T[:n].astype(np.int8)
+
+
+# ------------------------------------------------------------------ calibration schedule and update
+# App. B.1 fixes the optimizer (AdamW), the epochs (m = 60), the learning rate of the
+# modulation factors (1e-3) with a linear decay to zero, gamma = 0.8 and s0 = 30; §2.3 maps
+# the normalised epoch t to Eq. 6's branch and sharpness.
+
+def schedule_at_epoch(e: int, m: int, gamma: float, s0: float):
+    """Eq. 6's schedule point of calibration epoch e of m: t = e / m; t = 0 is the teacher
+    branch, 0 < t <= gamma the soft stage with s = (t / gamma) s0, gamma < t <= 1 the hard
+    stage, whose backward keeps the last soft sharpness s0 (§2.3).  The comparison
+    t <= gamma is made as e <= floor(gamma m + 1e-9), so that gamma m = 48 at the paper's
+    defaults counts 48 soft epochs whatever the rounding of 0.8 * 60.
+    Returns (phase, s)."""
+    assert 0 <= e <= m and m >= 1 and 0.0 < gamma <= 1.0 and s0 > 0.0
+    if e == 0:
+        return PHASE_TEACHER, 0.0
+    if e <= int(np.floor(gamma * m + 1e-9)):
+        t = e / m
+        return PHASE_SOFT, (t / gamma) * s0
+    return PHASE_HARD, float(s0)
+
+
+def linear_decay_lr(lr0: float, k: int, total: int) -> float:
+    """Learning rate of update k (0-based) of `total` under App. B.1's linear decay to zero:
+    lr0 (1 - k / total), which reaches zero one update after the last."""
+    assert 0 <= k < total
+    return lr0 * (1.0 - k / total)
+
+
+def adamw_step(p, grad, m, v, t: int, lr: float, beta1: float = 0.9, beta2: float = 0.999,
+               eps: float = 1e-8, weight_decay: float = 0.0):
+    """One AdamW update of parameters p (Loshchilov & Hutter, "Decoupled weight decay
+    regularization": the decay acts on p directly, not through the gradient) with Adam's
+    bias-corrected moments (Kingma & Ba), update count t >= 1.  The decay is scaled by the
+    learning rate, the PyTorch convention.  In order:
+        p <- p - lr * weight_decay * p
+        m <- beta1 m + (1 - beta1) grad,   v <- beta2 v + (1 - beta2) grad^2
+        p <- p - lr * m_hat / (sqrt(v_hat) + eps),  m_hat = m / (1 - beta1^t),
+                                                      v_hat = v / (1 - beta2^t)
+    Returns (p, m, v) as new fp64 arrays."""
+    p = np.asarray(p, np.float64)
+    grad = np.asarray(grad, np.float64)
+    m = np.asarray(m, np.float64)
+    v = np.asarray(v, np.float64)
+    p = p - lr * weight_decay * p
+    m = beta1 * m + (1.0 - beta1) * grad
+    v = beta2 * v + (1.0 - beta2) * grad * grad
+    m_hat = m / (1.0 - beta1 ** t)
+    v_hat = v / (1.0 - beta2 ** t)
+    p = p - lr * m_hat / (np.sqrt(v_hat) + eps)
+    return p, m, v
+
+
+def project_factors(d_mu, d_alpha, d_delta, margin: float):
+    """§2.2's constraints -1 < d_mu < 1, d_alpha > 0, d_delta > 0, enforced as the Euclidean
+    projection onto the closed sets [-1 + margin, 1 - margin], [margin, inf), [margin, inf)
+    (the paper does not say how they are kept; NaN stays NaN)."""
+    return (np.clip(np.asarray(d_mu, np.float64), -1.0 + margin, 1.0 - margin),
+            np.clip(np.asarray(d_alpha, np.float64), margin, np.inf),
+            np.clip(np.asarray(d_delta, np.float64), margin, np.inf))
+
+
+def factor_update(factors, grads, moments, t: int, lr: float, beta1: float = 0.9, beta2: float = 0.999,
+                  eps: float = 1e-8, weight_decay: float = 0.0, margin: float = 1e-4):
+    """The update after a calibration step: AdamW on each of (d_mu, d_alpha, d_delta) with
+    its gradient, then the projection of ``project_factors``.  moments = (m_mu, m_alpha,
+    m_delta, v_mu, v_alpha, v_delta).  Returns (factors, moments) as tuples of fp64 arrays."""
+    new_p, new_m, new_v = [], [], []
+    for q in range(3):
+        p, m, v = adamw_step(factors[q], grads[q], moments[q], moments[3 + q], t, lr, beta1, beta2, eps,
+                             weight_decay)
+        new_p.append(p)
+        new_m.append(m)
+        new_v.append(v)
+    return project_factors(*new_p, margin), tuple(new_m) + tuple(new_v)

@@ -59,6 +59,11 @@ class catq_schedule(ctypes.Structure):
     _fields_ = [("phase", ctypes.c_int32), ("s", ctypes.c_float)]
 
 
+class catq_adamw(ctypes.Structure):
+    _fields_ = [("beta1", ctypes.c_float), ("beta2", ctypes.c_float), ("eps", ctypes.c_float),
+                ("weight_decay", ctypes.c_float), ("margin", ctypes.c_float)]
+
+
 _lib = None
 
 
@@ -91,6 +96,9 @@ def lib() -> ctypes.CDLL:
         "catq_grouped_soft_ternary_linear_fwd": (I32, [ctypes.POINTER(catq_grouped_layer), catq_schedule, P, P, I32, P,
                                                        P]),
         "catq_grouped_bwd_workspace_bytes": (S, [ctypes.POINTER(catq_grouped_layer), P]),
+        "catq_schedule_at_epoch": (I32, [I32, I32, ctypes.c_double, ctypes.c_double, ctypes.POINTER(catq_schedule)]),
+        "catq_linear_decay_lr": (I32, [ctypes.c_double, I64, I64, ctypes.POINTER(F)]),
+        "catq_factor_adamw_step": (I32, [I64, P, P, P, P, P, P, P, ctypes.POINTER(catq_adamw), I64, F, P]),
         "catq_grouped_soft_ternary_linear_bwd": (I32, [ctypes.POINTER(catq_grouped_layer), catq_schedule, P, P, P, I32,
                                                        P, P, P, P, P, S, P]),
     }
@@ -263,6 +271,35 @@ def catq_ternary_infer(codes, alpha, N: int, K: int, g: int, X, Y, mu=None, stre
     W ~ alpha T + mu form) group offsets of catq_hard_ternarize_pack."""
     _check(lib().catq_ternary_infer(_ptr(codes), _ptr(alpha), _ptr(mu), int(N), int(K), int(g), _ptr(X),
                                     X.shape[0], _dtype_code(X), _ptr(Y), _stream(stream)), "catq_ternary_infer")
+
+
+def catq_schedule_at_epoch(e: int, m: int = 60, gamma: float = 0.8, s0: float = 30.0) -> catq_schedule:
+    """Eq. 6's (phase, s) of calibration epoch e of m (host only)."""
+    out = catq_schedule()
+    _check(lib().catq_schedule_at_epoch(int(e), int(m), float(gamma), float(s0), ctypes.byref(out)),
+           "catq_schedule_at_epoch")
+    return out
+
+
+def catq_linear_decay_lr(lr0: float, k: int, total: int) -> float:
+    """Learning rate of update k of `total` under a linear decay to zero (host only)."""
+    out = ctypes.c_float()
+    _check(lib().catq_linear_decay_lr(float(lr0), int(k), int(total), ctypes.byref(out)), "catq_linear_decay_lr")
+    return float(out.value)
+
+
+def adamw(beta1: float = 0.9, beta2: float = 0.999, eps: float = 1e-8, weight_decay: float = 0.0,
+          margin: float = 1e-4) -> catq_adamw:
+    return catq_adamw(beta1, beta2, eps, weight_decay, margin)
+
+
+def catq_factor_adamw_step(d_mu, d_alpha, d_delta, g_dmu, g_dalpha, g_ddelta, moments, hp: catq_adamw, t: int,
+                           lr: float, stream=None):
+    """One AdamW update of the factors [G] in place from their gradients; moments [6 * G]
+    (zero before the first update) is the optimizer state."""
+    _check(lib().catq_factor_adamw_step(d_mu.numel(), _ptr(d_mu), _ptr(d_alpha), _ptr(d_delta), _ptr(g_dmu),
+                                        _ptr(g_dalpha), _ptr(g_ddelta), _ptr(moments), ctypes.byref(hp), int(t),
+                                        float(lr), _stream(stream)), "catq_factor_adamw_step")
 
 
 def catq_selftest_wait_timeout(timeout_ns: int, stream=None):

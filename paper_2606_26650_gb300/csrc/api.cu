@@ -492,6 +492,67 @@ catq_status catq_ternary_infer(const uint8_t* codes, const float* alpha, const f
       launch_ternary_infer(codes, alpha, mu, N, K, g, X, B, Y, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+catq_status catq_schedule_at_epoch(int32_t e, int32_t m, double gamma, double s0, catq_schedule* out) {
+  if (!out || m < 1 || e < 0 || e > m) return CATQ_ERR_INVALID_ARG;
+  if (!(gamma > 0.0 && gamma <= 1.0) || !(s0 > 0.0) || !std::isfinite(s0)) return CATQ_ERR_INVALID_ARG;
+  const int64_t soft_epochs = static_cast<int64_t>(std::floor(gamma * m + 1e-9));
+  if (e == 0) {
+    *out = catq_schedule{CATQ_PHASE_TEACHER, 0.0f};
+  } else if (e <= soft_epochs) {
+    const double t = static_cast<double>(e) / m;
+    *out = catq_schedule{CATQ_PHASE_SOFT, static_cast<float>(t / gamma * s0)};
+  } else {
+    *out = catq_schedule{CATQ_PHASE_HARD, static_cast<float>(s0)};
+  }
+  return CATQ_OK;
+}
+
+catq_status catq_linear_decay_lr(double lr0, int64_t k, int64_t total, float* lr_out) {
+  if (!lr_out || k < 0 || k >= total || !(lr0 >= 0.0) || !std::isfinite(lr0)) return CATQ_ERR_INVALID_ARG;
+  *lr_out = static_cast<float>(lr0 * (1.0 - static_cast<double>(k) / static_cast<double>(total)));
+  return CATQ_OK;
+}
+
+catq_status catq_factor_adamw_step(int64_t G, float* d_mu, float* d_alpha, float* d_delta, const float* g_dmu,
+                                   const float* g_dalpha, const float* g_ddelta, float* moments,
+                                   const catq_adamw* hp, int64_t t, float lr, catq_stream stream) {
+  if (G < 0) return CATQ_ERR_SHAPE;
+  if (G == 0) return CATQ_OK;
+  if (!d_mu || !d_alpha || !d_delta || !g_dmu || !g_dalpha || !g_ddelta || !moments || !hp)
+    return CATQ_ERR_INVALID_ARG;
+  if (t < 1 || !(lr >= 0.0f) || !std::isfinite(lr)) return CATQ_ERR_INVALID_ARG;
+  if (!(hp->beta1 >= 0.0f && hp->beta1 < 1.0f) || !(hp->beta2 >= 0.0f && hp->beta2 < 1.0f) ||
+      !(hp->eps > 0.0f) || !std::isfinite(hp->eps) || !(hp->weight_decay >= 0.0f) ||
+      !std::isfinite(hp->weight_decay) || !(hp->margin >= 0.0f && hp->margin < 0.5f))
+    return CATQ_ERR_INVALID_ARG;
+  const void* ptrs[7] = {d_mu, d_alpha, d_delta, g_dmu, g_dalpha, g_ddelta, moments};
+  for (const void* p : ptrs)
+    if (reinterpret_cast<uintptr_t>(p) & 3u) return CATQ_ERR_ALIGN;
+  AdamwArgs a{};
+  float* const p[3] = {d_mu, d_alpha, d_delta};
+  const float* const g[3] = {g_dmu, g_dalpha, g_ddelta};
+  for (int q = 0; q < 3; ++q) {
+    a.p[q] = p[q];
+    a.g[q] = g[q];
+    a.m[q] = moments + q * G;
+    a.v[q] = moments + (3 + q) * G;
+  }
+  const double b1 = hp->beta1, b2 = hp->beta2;
+  a.decay = static_cast<float>(1.0 - static_cast<double>(lr) * hp->weight_decay);
+  a.beta1 = hp->beta1;
+  a.one_minus_beta1 = static_cast<float>(1.0 - b1);
+  a.beta2 = hp->beta2;
+  a.one_minus_beta2 = static_cast<float>(1.0 - b2);
+  a.step = static_cast<float>(lr / (1.0 - std::pow(b1, static_cast<double>(t))));
+  a.inv_sqrt_bc2 = static_cast<float>(1.0 / std::sqrt(1.0 - std::pow(b2, static_cast<double>(t))));
+  a.eps = hp->eps;
+  a.lo[0] = -1.0f + hp->margin;
+  a.hi[0] = 1.0f - hp->margin;
+  a.lo[1] = a.lo[2] = hp->margin;
+  a.hi[1] = a.hi[2] = INFINITY;
+  return cuda_status(launch_factor_adamw(G, a, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 catq_status catq_selftest_wait_timeout(uint64_t timeout_ns, catq_stream stream) {
   if (timeout_ns < 1000 || timeout_ns > 1000000000ull) return CATQ_ERR_INVALID_ARG;
   return cuda_status(launch_wait_probe(timeout_ns, reinterpret_cast<cudaStream_t>(stream)));

@@ -1,7 +1,8 @@
 // elementwise.cu — the HBM-bound kernels of the path: group statistics (Eq. 3), the
 // materialised Eq. 6 weight (inspection only), the reconstruction loss of Eq. 7 with its
 // gradient, the final hard ternarization + 2-bit pack, and the reduction of the dW
-// epilogue's partial sums into the three factor gradients.
+// epilogue's partial sums into the three factor gradients, and the optimizer's update of
+// the factors after a step.
 #include <cuda_bf16.h>
 
 #include "launch.h"
@@ -669,6 +670,34 @@ __global__ void __launch_bounds__(kThreads) grad_reduce_grouped_kernel(LayerDev 
   }
 }
 
+// ---------------------------------------------------------------- factor update (AdamW)
+// One thread per group and factor array: decoupled decay, the two moment updates, the
+// bias-corrected step and the projection of the factor's constraint.  Comparisons keep NaN
+// as NaN (a NaN factor is not hidden at a bound).  Reads 16 B and writes 12 B per element.
+__global__ void __launch_bounds__(kThreads) factor_adamw_kernel(int64_t G, const AdamwArgs a) {
+  for (int64_t j = blockIdx.x * (int64_t)kThreads + threadIdx.x; j < 3 * G; j += (int64_t)gridDim.x * kThreads) {
+    const int q = static_cast<int>(j / G);
+    const int64_t i = j - q * G;
+    // constant indices into the parameter arrays (no local copy of the argument block)
+    float* const P = q == 0 ? a.p[0] : q == 1 ? a.p[1] : a.p[2];
+    const float* const Gr = q == 0 ? a.g[0] : q == 1 ? a.g[1] : a.g[2];
+    float* const Mo = q == 0 ? a.m[0] : q == 1 ? a.m[1] : a.m[2];
+    float* const Vo = q == 0 ? a.v[0] : q == 1 ? a.v[1] : a.v[2];
+    const float lo = q == 0 ? a.lo[0] : q == 1 ? a.lo[1] : a.lo[2];
+    const float hi = q == 0 ? a.hi[0] : q == 1 ? a.hi[1] : a.hi[2];
+    const float grad = Gr[i];
+    float p = P[i] * a.decay;
+    const float m = fmaf(a.beta1, Mo[i], a.one_minus_beta1 * grad);
+    const float v = fmaf(a.beta2, Vo[i], a.one_minus_beta2 * (grad * grad));
+    const float denom = fmaf(sqrtf(v), a.inv_sqrt_bc2, a.eps);
+    p -= a.step * (m / denom);
+    p = p < lo ? lo : (p > hi ? hi : p);
+    P[i] = p;
+    Mo[i] = m;
+    Vo[i] = v;
+  }
+}
+
 int grid_for(int64_t work, int64_t per_block) {
   int64_t b = (work + per_block - 1) / per_block;
   if (b < 1) b = 1;
@@ -831,6 +860,12 @@ cudaError_t launch_grad_reduce(const LayerDev& L, StepScalars sc, const float* p
   const int64_t G = L.N * L.K / L.g;
   grad_reduce_kernel<<<grid_for(G, kThreads), kThreads, 0, st>>>(L, sc, partials, splits, P, g_dmu, g_dalpha,
                                                                  g_ddelta);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_factor_adamw(int64_t G, const AdamwArgs& a, cudaStream_t st) {
+  if (G == 0) return cudaSuccess;
+  factor_adamw_kernel<<<grid_for(3 * G, kThreads), kThreads, 0, st>>>(G, a);
   return cudaGetLastError();
 }
 

@@ -58,6 +58,23 @@ bool launch_wait_ctl(WaitCtl* out);
 // One-thread kernel whose bounded wait runs out after timeout_ns (self-test).
 cudaError_t launch_wait_probe(uint64_t timeout_ns, cudaStream_t st);
 
+// One AdamW step on the three factor arrays p[q] with gradients g[q] and moments m[q], v[q]
+// (q = mu, alpha, delta; each [G] fp32), then the projection onto [lo[q], hi[q]].  The
+// scalars that depend only on the update count are folded on the host.
+struct AdamwArgs {
+  float* p[3];
+  const float* g[3];
+  float* m[3];
+  float* v[3];
+  float decay;        // 1 - lr weight_decay
+  float beta1, one_minus_beta1, beta2, one_minus_beta2;
+  float step;         // lr / (1 - beta1^t)
+  float inv_sqrt_bc2; // 1 / sqrt(1 - beta2^t)
+  float eps;
+  float lo[3], hi[3];
+};
+cudaError_t launch_factor_adamw(int64_t G, const AdamwArgs& a, cudaStream_t st);
+
 // Writes L.op_const (operand_const_vec of every group, [K/g][N]) for schedule point sc.
 cudaError_t launch_operand_consts(const LayerDev& L, StepScalars sc, cudaStream_t st);
 

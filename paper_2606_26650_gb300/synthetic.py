@@ -189,6 +189,19 @@ def factors(G: int, seed: int, tag: str, perturbed: bool):
             r.uniform(0.8, 1.2, G).astype(np.float32))
 
 
+def gradients(G: int, seed: int, tag: str):
+    """Stand-ins for the three factor gradients, float32 [G] each: signed normal values whose
+    scales spread log-uniformly over 1e-6 .. 1e-2, as per-group sums of a calibration
+    batch do, with a few exact zeros."""
+    r = rng(seed, tag + "/grads")
+    out = []
+    for _ in range(3):
+        v = r.standard_normal(G) * 10.0 ** r.uniform(-6, -2, G)
+        v[r.random(G) < 0.01] = 0.0
+        out.append(v.astype(np.float32))
+    return tuple(out)
+
+
 def moe_routing(wl: Workload, seed: int = 0):
     """Top-k expert assignment per token: k distinct experts drawn without replacement
     (Gumbel top-k) from p_e proportional to (e + 1)^-a.  Returns (token_of_row,

@@ -102,3 +102,54 @@ def test_call_validation(lib):
     assert infer(16, 32, None, 64, 256, 128, 16, 1, C.BF16, None, None) == 1        # null Y
     assert lib.catq_selftest_wait_timeout(10, None) == 1              # below 1 us
     assert lib.catq_selftest_wait_timeout(2_000_000_000, None) == 1   # above 1 s
+
+
+def test_schedule_and_lr_host_calls_follow_the_oracle(lib):
+    """The host-only schedule calls against the oracle: the branch exactly, s and the
+    learning rate to fp32 rounding."""
+    from oracle import catq_oracle as O
+    for m, gamma, s0 in [(60, 0.8, 30.0), (10, 1.0, 5.0), (7, 0.5, 12.0), (100, 0.57, 30.0), (1, 0.3, 2.0)]:
+        for e in range(m + 1):
+            got = C.catq_schedule_at_epoch(e, m, gamma, s0)
+            phase, s = O.schedule_at_epoch(e, m, gamma, s0)
+            assert got.phase == phase, (m, gamma, e)
+            assert got.s == pytest.approx(s, rel=1e-7, abs=0.0), (m, gamma, e)
+    for total in (1, 8, 10260):
+        for k in sorted({0, 1, total // 2, total - 1}):
+            if k < total:
+                assert C.catq_linear_decay_lr(1e-3, k, total) == pytest.approx(O.linear_decay_lr(1e-3, k, total),
+                                                                                rel=1e-7)
+
+
+def test_schedule_and_update_validation(lib):
+    out = C.catq_schedule()
+    sched = lib.catq_schedule_at_epoch
+    assert sched(1, 60, 0.8, 30.0, ctypes.byref(out)) == 0
+    assert sched(61, 60, 0.8, 30.0, ctypes.byref(out)) == 1   # e > m
+    assert sched(-1, 60, 0.8, 30.0, ctypes.byref(out)) == 1
+    assert sched(0, 0, 0.8, 30.0, ctypes.byref(out)) == 1     # m < 1
+    assert sched(1, 60, 0.0, 30.0, ctypes.byref(out)) == 1    # gamma outside (0, 1]
+    assert sched(1, 60, 1.5, 30.0, ctypes.byref(out)) == 1
+    assert sched(1, 60, 0.8, 0.0, ctypes.byref(out)) == 1     # s0 <= 0
+    assert sched(1, 60, 0.8, float("inf"), ctypes.byref(out)) == 1
+    assert sched(1, 60, 0.8, 30.0, None) == 1
+    lr = ctypes.c_float()
+    assert lib.catq_linear_decay_lr(1e-3, 5, 5, ctypes.byref(lr)) == 1  # k >= total
+    assert lib.catq_linear_decay_lr(-1.0, 0, 5, ctypes.byref(lr)) == 1
+    assert lib.catq_linear_decay_lr(float("nan"), 0, 5, ctypes.byref(lr)) == 1
+    # the update rejects bad arguments on the host (fake, never dereferenced addresses)
+    hp = C.adamw()
+    step = lib.catq_factor_adamw_step
+    ptrs = [4096 * (i + 1) for i in range(7)]
+    assert step(-1, *ptrs, ctypes.byref(hp), 1, 1e-3, None) == 2
+    assert step(0, *ptrs, ctypes.byref(hp), 1, 1e-3, None) == 0  # no work, nothing launched
+    assert step(0, *([None] * 7), None, 0, -1.0, None) == 0
+    assert step(8, *ptrs[:6], None, ctypes.byref(hp), 1, 1e-3, None) == 1
+    assert step(8, *ptrs, None, 1, 1e-3, None) == 1
+    assert step(8, *ptrs, ctypes.byref(hp), 0, 1e-3, None) == 1  # t < 1
+    assert step(8, *ptrs, ctypes.byref(hp), 1, -1e-3, None) == 1
+    assert step(8, *ptrs, ctypes.byref(hp), 1, float("nan"), None) == 1
+    for bad in (C.adamw(beta1=1.0), C.adamw(beta2=-0.1), C.adamw(eps=0.0), C.adamw(weight_decay=-1.0),
+                C.adamw(margin=0.5), C.adamw(eps=float("inf"))):
+        assert step(8, *ptrs, ctypes.byref(bad), 1, 1e-3, None) == 1
+    assert step(8, *ptrs[:6], ptrs[6] + 2, ctypes.byref(hp), 1, 1e-3, None) == 4  # misaligned moments

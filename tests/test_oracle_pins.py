@@ -576,3 +576,103 @@ def test_direct_learning_is_a_reparametrization_of_the_modulation(s):
             m[which][j] -= h * scale
             fd[j] = (loss_direct(*p) - loss_direct(*m)) / (2 * h * scale)
         np.testing.assert_allclose(want, fd, rtol=1e-4, atol=1e-6 * np.abs(fd).max())
+
+
+# ----------------------------------------------------------------- App. B.1: schedule and AdamW update
+
+def test_schedule_at_epoch_paper_defaults():
+    """App. B.1 (m = 60, gamma = 0.8, s0 = 30) with §2.3's t = e / m: 48 soft epochs whose
+    sharpness rises linearly from s0 / 48 to exactly s0, then 12 hard epochs at s0; t = 0 is
+    the teacher."""
+    m, gamma, s0 = 60, 0.8, 30.0
+    assert O.schedule_at_epoch(0, m, gamma, s0)[0] == O.PHASE_TEACHER
+    pts = [O.schedule_at_epoch(e, m, gamma, s0) for e in range(1, m + 1)]
+    phases = [p for p, _ in pts]
+    assert phases == [O.PHASE_SOFT] * 48 + [O.PHASE_HARD] * 12
+    s = np.array([v for _, v in pts[:48]])
+    np.testing.assert_allclose(s, 0.625 * np.arange(1, 49), rtol=1e-15)
+    assert s[-1] == s0
+    assert all(v == s0 for _, v in pts[48:])
+    # gamma = 1: no hard stage; gamma m not an integer: floor(gamma m) soft epochs
+    assert [O.schedule_at_epoch(e, 10, 1.0, 5.0)[0] for e in range(1, 11)] == [O.PHASE_SOFT] * 10
+    assert sum(O.schedule_at_epoch(e, 7, 0.5, 5.0)[0] == O.PHASE_SOFT for e in range(1, 8)) == 3
+    # rounding of gamma m (0.57 * 100 = 56.99999999999999 in fp64) does not drop an epoch
+    assert sum(O.schedule_at_epoch(e, 100, 0.57, 5.0)[0] == O.PHASE_SOFT for e in range(1, 101)) == 57
+
+
+def test_linear_decay_lr_closed_form():
+    """A linear decay to zero: lr0 at the first update, equal decrements lr0 / total, the
+    last update at lr0 / total, and the sum lr0 (total + 1) / 2."""
+    lr0, total = 1e-3, 171
+    lrs = np.array([O.linear_decay_lr(lr0, k, total) for k in range(total)])
+    assert lrs[0] == lr0
+    np.testing.assert_allclose(np.diff(lrs), -lr0 / total, rtol=1e-9)
+    np.testing.assert_allclose(lrs[-1], lr0 / total, rtol=1e-12)
+    np.testing.assert_allclose(lrs.sum(), lr0 * (total + 1) / 2, rtol=1e-12)
+
+
+def test_adamw_first_step_and_constant_gradient_closed_forms():
+    """From zero moments the bias correction makes m_hat = g and v_hat = g^2 exactly, so the
+    first step is p (1 - lr wd) - lr g / (|g| + eps); under a constant gradient the same
+    holds at every step (m_t = g (1 - beta1^t)), so each step moves p by lr g / (|g| + eps)."""
+    r = np.random.default_rng(3)
+    p0 = r.uniform(-1, 1, 64)
+    g = r.normal(0, 1e-3, 64)
+    z = np.zeros(64)
+    lr, wd, eps = 1e-3, 0.01, 1e-8
+    p1, m1, v1 = O.adamw_step(p0, g, z, z, 1, lr, 0.9, 0.999, eps, wd)
+    np.testing.assert_allclose(p1, p0 * (1 - lr * wd) - lr * g / (np.abs(g) + eps), rtol=1e-13, atol=1e-18)
+    np.testing.assert_allclose(m1, 0.1 * g, rtol=1e-13)
+    np.testing.assert_allclose(v1, 0.001 * g * g, rtol=1e-12)
+    p, m, v = p0, z, z
+    lrs = [1e-3 * (1 - k / 10) for k in range(10)]
+    for t, lr_t in enumerate(lrs, start=1):
+        p, m, v = O.adamw_step(p, g, m, v, t, lr_t, 0.8, 0.95, eps, 0.0)
+    np.testing.assert_allclose(p, p0 - sum(lrs) * g / (np.abs(g) + eps), rtol=1e-12, atol=1e-15)
+
+
+@pytest.mark.parametrize("betas,eps,wd", [((0.9, 0.999), 1e-8, 0.0), ((0.9, 0.999), 1e-8, 0.01),
+                                          ((0.8, 0.95), 1e-6, 0.1)])
+def test_adamw_matches_torch_adamw(betas, eps, wd):
+    """Eight updates with a decaying learning rate and changing gradients against PyTorch's
+    own AdamW (fp64 on the CPU, single-tensor path): parameters and both moments."""
+    torch = pytest.importorskip("torch")
+    r = np.random.default_rng(11)
+    p0 = r.uniform(0.5, 1.5, 257)
+    grads = [r.normal(0, 10.0 ** -r.integers(2, 6), 257) for _ in range(8)]
+    param = torch.nn.Parameter(torch.from_numpy(p0.copy()))
+    opt = torch.optim.AdamW([param], lr=1e-3, betas=betas, eps=eps, weight_decay=wd, foreach=False)
+    p, m, v = p0, np.zeros(257), np.zeros(257)
+    for k, gk in enumerate(grads):
+        lr = 1e-3 * (1 - k / 8)
+        for grp in opt.param_groups:
+            grp["lr"] = lr
+        param.grad = torch.from_numpy(gk.copy())
+        opt.step()
+        p, m, v = O.adamw_step(p, gk, m, v, k + 1, lr, betas[0], betas[1], eps, wd)
+    state = opt.state[param]
+    np.testing.assert_allclose(p, param.detach().numpy(), rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(m, state["exp_avg"].numpy(), rtol=1e-12, atol=1e-20)
+    np.testing.assert_allclose(v, state["exp_avg_sq"].numpy(), rtol=1e-12, atol=1e-30)
+
+
+def test_factor_update_projects_onto_the_constraints():
+    """§2.2's constraints after the update: values inside the sets are untouched, values
+    outside land on the nearest bound, NaN stays NaN; each factor uses its own gradient and
+    its own moments."""
+    margin = 1e-4
+    mu, al, de = O.project_factors([-1.5, -0.5, 0.99995, np.nan], [-2.0, 0.0, 0.5, 3.0], [1e-5, 2.0, -1.0, 0.2],
+                                   margin)
+    np.testing.assert_array_equal(mu[:3], [-1 + margin, -0.5, 1 - margin])
+    assert np.isnan(mu[3])
+    np.testing.assert_array_equal(al, [margin, margin, 0.5, 3.0])
+    np.testing.assert_array_equal(de, [margin, 2.0, margin, 0.2])
+    # gradients routed to their own factor: only d_alpha moves when only its gradient is set
+    f = (np.zeros(4), np.ones(4), np.ones(4))
+    gr = (np.zeros(4), np.full(4, 0.3), np.zeros(4))
+    (nm, na, nd), mom = O.factor_update(f, gr, (np.zeros(4),) * 6, 1, 1e-3)
+    np.testing.assert_array_equal(nm, 0.0)
+    np.testing.assert_array_equal(nd, 1.0)
+    np.testing.assert_allclose(na, 1.0 - 1e-3 * 0.3 / (0.3 + 1e-8), rtol=1e-14)
+    np.testing.assert_allclose(mom[1], 0.1 * 0.3, rtol=1e-14)
+    np.testing.assert_allclose(mom[4], 0.001 * 0.09, rtol=1e-13)
