@@ -12,7 +12,8 @@ G = N*K/g consecutive groups of g elements (App. B.2); every statistic and facto
 group.
 
 Pins (tests/test_oracle_pins.py) tie each function to something other than itself:
-brute force, closed forms, limits and finite differences.  One part is
+brute force, closed forms, limits and finite differences; the optimizer update also to
+PyTorch's own AdamW.  One part is
 "parity unpinned": the HARD-phase factor gradients (see ``linear_bwd``), which rest on
 this library's reading of §2.3's stage-2 rule and have no independent reference.
 """
