@@ -143,6 +143,22 @@ def _check(status: int, where: str):
         raise CatqError(status, where)
 
 
+def _buf(t, name: str, nbytes: int, where: str):
+    """The library reads and writes `nbytes` bytes at a tensor's address without seeing its
+    size or device: refuse a host tensor or one too small before the call, so that a
+    caller's mistake raises here instead of touching memory the tensor does not own.
+    None passes (the call decides whether the argument is optional)."""
+    if t is None:
+        return
+    if not t.is_cuda:
+        raise ValueError(f"{where}: {name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{where}: {name} must be contiguous")
+    have = t.numel() * t.element_size()
+    if have < nbytes:
+        raise ValueError(f"{where}: {name} holds {have} bytes, the call needs {nbytes}")
+
+
 @dataclasses.dataclass
 class Layer:
     """One linear layer's device state: W [N, K], the per-group arrays ([G] fp32) and the
@@ -186,6 +202,11 @@ class Layer:
         return self.N * self.K // self.g
 
     def struct(self) -> catq_layer:
+        G, where = self.G, "Layer"
+        _buf(self.W, "W", self.N * self.K * self.W.element_size(), where)
+        for name in ("mu0", "alpha0", "delta0", "d_mu", "d_alpha", "d_delta"):
+            _buf(getattr(self, name), name, 4 * G, where)
+        _buf(self.op_const, "op_const", 4 * (5 if self.recon else 4) * G, where)
         return catq_layer(self.N, self.K, self.g, _dtype_code(self.W), self.W.data_ptr(),
                           self.mu0.data_ptr(), self.alpha0.data_ptr(), self.delta0.data_ptr(),
                           self.d_mu.data_ptr(), self.d_alpha.data_ptr(), self.d_delta.data_ptr(),
@@ -206,12 +227,19 @@ def catq_group_stats(layer: Layer, thr_init: int = THR_HALF, stream=None):
 def catq_modulate_ternarize(layer: Layer, sched: catq_schedule, Wq_out=None, T_out=None, alpha_out=None,
                             stream=None):
     st = layer.struct()
+    w = "catq_modulate_ternarize"
+    _buf(Wq_out, "Wq_out", layer.N * layer.K * layer.W.element_size(), w)
+    _buf(T_out, "T_out", layer.N * layer.K, w)
+    _buf(alpha_out, "alpha_out", 4 * layer.G, w)
     _check(lib().catq_modulate_ternarize(ctypes.byref(st), sched, _ptr(Wq_out), _ptr(T_out), _ptr(alpha_out),
                                          _stream(stream)), "catq_modulate_ternarize")
 
 
 def catq_soft_ternary_linear_fwd(layer: Layer, sched: catq_schedule, X, Y, stream=None):
     st = layer.struct()
+    M, e, w = X.shape[0], X.element_size(), "catq_soft_ternary_linear_fwd"
+    _buf(X, "X", M * layer.K * e, w)
+    _buf(Y, "Y", M * layer.N * e, w)
     _check(lib().catq_soft_ternary_linear_fwd(ctypes.byref(st), sched, _ptr(X), X.shape[0], _dtype_code(X),
                                               _ptr(Y), _stream(stream)), "catq_soft_ternary_linear_fwd")
 
@@ -224,6 +252,8 @@ def catq_bwd_workspace_bytes(layer: Layer, M: int) -> int:
 def catq_soft_ternary_linear_bwd(layer: Layer, sched: catq_schedule, X, dY, dX=None, g_dmu=None, g_dalpha=None,
                                  g_ddelta=None, workspace=None, stream=None):
     st = layer.struct()
+    _bwd_bufs(layer, X, dY, dX, (g_dmu, g_dalpha, g_ddelta), "catq_soft_ternary_linear_bwd")
+    _buf(workspace, "workspace", 0, "catq_soft_ternary_linear_bwd")
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     _check(lib().catq_soft_ternary_linear_bwd(ctypes.byref(st), sched, _ptr(X), _ptr(dY), X.shape[0],
                                               _dtype_code(X), _ptr(dX), _ptr(g_dmu), _ptr(g_dalpha),
@@ -234,10 +264,21 @@ def catq_soft_ternary_linear_bwd(layer: Layer, sched: catq_schedule, X, dY, dX=N
 def catq_soft_ternary_linear_bwd_noalloc(layer: Layer, sched: catq_schedule, X, dY, dX=None, g_dmu=None,
                                          g_dalpha=None, g_ddelta=None, stream=None):
     st = layer.struct()
+    _bwd_bufs(layer, X, dY, dX, (g_dmu, g_dalpha, g_ddelta), "catq_soft_ternary_linear_bwd_noalloc")
     _check(lib().catq_soft_ternary_linear_bwd_noalloc(ctypes.byref(st), sched, _ptr(X), _ptr(dY), X.shape[0],
                                                       _dtype_code(X), _ptr(dX), _ptr(g_dmu), _ptr(g_dalpha),
                                                       _ptr(g_ddelta), _stream(stream)),
            "catq_soft_ternary_linear_bwd_noalloc")
+
+
+def _bwd_bufs(layer, X, dY, dX, grads, where, rows=None, groups=None):
+    M = X.shape[0] if rows is None else rows
+    e = X.element_size()
+    _buf(X, "X", M * layer.K * e, where)
+    _buf(dY, "dY", M * layer.N * e, where)
+    _buf(dX, "dX", M * layer.K * e, where)
+    for name, t in zip(("g_dmu", "g_dalpha", "g_ddelta"), grads):
+        _buf(t, name, 4 * (layer.G if groups is None else groups), where)
 
 
 def catq_bwd_noalloc_max_scratch_bytes() -> int:
@@ -249,6 +290,12 @@ def catq_recon_loss_workspace_bytes(count: int) -> int:
 
 
 def catq_recon_loss(Y, Y_ref, loss_out, dY=None, workspace=None, reduction: int = REDUCE_MEAN, stream=None):
+    w, n = "catq_recon_loss", Y.numel() * Y.element_size()
+    _buf(Y, "Y", n, w)
+    _buf(Y_ref, "Y_ref", n, w)
+    _buf(dY, "dY", n, w)
+    _buf(loss_out, "loss_out", 4, w)
+    _buf(workspace, "workspace", 0, w)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     _check(lib().catq_recon_loss(_ptr(Y), _ptr(Y_ref), Y.numel(), _dtype_code(Y), int(reduction), _ptr(loss_out),
                                  _ptr(dY), _ptr(workspace), ws_bytes, _stream(stream)), "catq_recon_loss")
@@ -256,6 +303,10 @@ def catq_recon_loss(Y, Y_ref, loss_out, dY=None, workspace=None, reduction: int 
 
 def catq_hard_ternarize_pack(layer: Layer, codes, alpha=None, mu=None, stream=None):
     st = layer.struct()
+    w = "catq_hard_ternarize_pack"
+    _buf(codes, "codes", layer.N * layer.K // 4, w)
+    _buf(alpha, "alpha", 4 * layer.G, w)
+    _buf(mu, "mu", 4 * layer.G, w)
     _check(lib().catq_hard_ternarize_pack(ctypes.byref(st), _ptr(codes), _ptr(alpha), _ptr(mu), _stream(stream)),
            "catq_hard_ternarize_pack")
 
@@ -269,6 +320,12 @@ def catq_device_status(stream=None) -> int:
 def catq_ternary_infer(codes, alpha, N: int, K: int, g: int, X, Y, mu=None, stream=None):
     """Y [B, N] = X [B, K] (alpha T + mu)^T from the 2-bit codes, group scales and (for the
     W ~ alpha T + mu form) group offsets of catq_hard_ternarize_pack."""
+    w, B, G = "catq_ternary_infer", X.shape[0], int(N) * int(K) // max(int(g), 1)
+    _buf(codes, "codes", int(N) * int(K) // 4, w)
+    _buf(alpha, "alpha", 4 * G, w)
+    _buf(mu, "mu", 4 * G, w)
+    _buf(X, "X", B * int(K) * X.element_size(), w)
+    _buf(Y, "Y", B * int(N) * X.element_size(), w)
     _check(lib().catq_ternary_infer(_ptr(codes), _ptr(alpha), _ptr(mu), int(N), int(K), int(g), _ptr(X),
                                     X.shape[0], _dtype_code(X), _ptr(Y), _stream(stream)), "catq_ternary_infer")
 
@@ -297,6 +354,11 @@ def catq_factor_adamw_step(d_mu, d_alpha, d_delta, g_dmu, g_dalpha, g_ddelta, mo
                            lr: float, stream=None):
     """One AdamW update of the factors [G] in place from their gradients; moments [6 * G]
     (zero before the first update) is the optimizer state."""
+    G, w = d_mu.numel(), "catq_factor_adamw_step"
+    for name, t in zip(("d_mu", "d_alpha", "d_delta", "g_dmu", "g_dalpha", "g_ddelta"),
+                       (d_mu, d_alpha, d_delta, g_dmu, g_dalpha, g_ddelta)):
+        _buf(t, name, 4 * G, w)
+    _buf(moments, "moments", 4 * 6 * G, w)
     _check(lib().catq_factor_adamw_step(d_mu.numel(), _ptr(d_mu), _ptr(d_alpha), _ptr(d_delta), _ptr(g_dmu),
                                         _ptr(g_dalpha), _ptr(g_ddelta), _ptr(moments), ctypes.byref(hp), int(t),
                                         float(lr), _stream(stream)), "catq_factor_adamw_step")
@@ -334,6 +396,7 @@ class GroupedLayer:
     def struct(self) -> catq_grouped_layer:
         E, N, K = self.W.shape
         d = self.dense
+        d.struct()  # checks the stacked weights and the [E * G] per-group arrays
         return catq_grouped_layer(E, self.g, N, K, _dtype_code(self.W), d.recon, self.W.data_ptr(), d.mu0.data_ptr(),
                                   d.alpha0.data_ptr(), d.delta0.data_ptr(), d.d_mu.data_ptr(), d.d_alpha.data_ptr(),
                                   d.d_delta.data_ptr(), d.op_const.data_ptr() if d.op_const is not None else None)
@@ -344,8 +407,24 @@ def _offsets(row_offsets):
     return arr
 
 
+def _grouped_bufs(layer, row_offsets, where, X=None, Y=None, dY=None, dX=None, grads=()):
+    """The library reads E + 1 row offsets and rows 0 .. R-1 of the row-indexed arrays."""
+    E, N, K = layer.W.shape
+    if len(row_offsets) != E + 1:
+        raise ValueError(f"{where}: row_offsets has {len(row_offsets)} entries, the layer's {E} experts need {E + 1}")
+    R = int(row_offsets[-1])
+    e = X.element_size() if X is not None else 2
+    _buf(X, "X", R * K * e, where)
+    _buf(Y, "Y", R * N * e, where)
+    _buf(dY, "dY", R * N * e, where)
+    _buf(dX, "dX", R * K * e, where)
+    for name, t in zip(("g_dmu", "g_dalpha", "g_ddelta"), grads):
+        _buf(t, name, 4 * E * (N * K // layer.g), where)
+
+
 def catq_grouped_soft_ternary_linear_fwd(layer: GroupedLayer, sched: catq_schedule, X, row_offsets, Y, stream=None):
     st = layer.struct()
+    _grouped_bufs(layer, row_offsets, "catq_grouped_soft_ternary_linear_fwd", X=X, Y=Y)
     off = _offsets(row_offsets)
     _check(lib().catq_grouped_soft_ternary_linear_fwd(ctypes.byref(st), sched, _ptr(X), off, _dtype_code(X), _ptr(Y),
                                                       _stream(stream)), "catq_grouped_soft_ternary_linear_fwd")
@@ -353,12 +432,16 @@ def catq_grouped_soft_ternary_linear_fwd(layer: GroupedLayer, sched: catq_schedu
 
 def catq_grouped_bwd_workspace_bytes(layer: GroupedLayer, row_offsets) -> int:
     st = layer.struct()
+    _grouped_bufs(layer, row_offsets, "catq_grouped_bwd_workspace_bytes")
     return int(lib().catq_grouped_bwd_workspace_bytes(ctypes.byref(st), _offsets(row_offsets)))
 
 
 def catq_grouped_soft_ternary_linear_bwd(layer: GroupedLayer, sched: catq_schedule, X, dY, row_offsets, dX=None,
                                          g_dmu=None, g_dalpha=None, g_ddelta=None, workspace=None, stream=None):
     st = layer.struct()
+    _grouped_bufs(layer, row_offsets, "catq_grouped_soft_ternary_linear_bwd", X=X, dY=dY, dX=dX,
+                  grads=(g_dmu, g_dalpha, g_ddelta))
+    _buf(workspace, "workspace", 0, "catq_grouped_soft_ternary_linear_bwd")
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     _check(lib().catq_grouped_soft_ternary_linear_bwd(ctypes.byref(st), sched, _ptr(X), _ptr(dY),
                                                       _offsets(row_offsets), _dtype_code(X), _ptr(dX), _ptr(g_dmu),
