@@ -52,7 +52,8 @@ typedef enum {
   CATQ_ERR_INVALID_ARG = 1, /* null pointer, bad enum, non-finite or non-positive s */
   CATQ_ERR_SHAPE = 2,       /* g does not divide K, unsupported g, M < 0, N/K < 1 */
   CATQ_ERR_DTYPE = 3,       /* unknown dtype or mixed weight/activation dtypes */
-  CATQ_ERR_ALIGN = 4,       /* buffer not 16-byte aligned (workspace: 256-byte) */
+  CATQ_ERR_ALIGN = 4,       /* buffer misaligned: 16 bytes for TMA operands, 256 for workspaces,
+                               4 for the fp32 arrays of catq_factor_adamw_step */
   CATQ_ERR_CUDA = 5,        /* a CUDA runtime call failed (launch, attribute, tensor map) */
   CATQ_ERR_TIMEOUT = 6,     /* a bounded device-side wait expired (latched) */
   CATQ_ERR_NONFINITE = 7,   /* reserved: non-finite data detected (latched) */
