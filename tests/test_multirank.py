@@ -1,4 +1,5 @@
-"""The multi-rank path of bench.py on the CPU: two `gloo` ranks.
+"""bench.py's host logic on the CPU: the multi-rank path (two `gloo` ranks) and the
+sequencing of the factor update that closes each step.
 
 Each rank runs the same step on its own seeded inputs (independent replicas, weak scaling),
 the step time is the slowest rank's, and the job's throughput is the ranks' total work over
@@ -80,3 +81,40 @@ def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
     args = bench.parse(["--impl", "reference", "--steps", "1", "--warmup", "0"])
     assert bench.run_reference(args) is None
     assert capsys.readouterr().out == ""
+
+
+def test_factor_update_sequence_of_the_bench_step():
+    """bench.py's step closes with one AdamW update per linear: the update count rises by
+    one per step, the learning rate follows the linear decay of App. B.1 through the
+    library's host call and wraps after a full calibration's updates, and every linear gets
+    its own moments of 6 G floats."""
+    from paper_2606_26650_gb300 import catq as C
+
+    calls = []
+
+    class FakeC:
+        adamw = staticmethod(C.adamw)
+        catq_linear_decay_lr = staticmethod(C.catq_linear_decay_lr)
+
+        @staticmethod
+        def catq_factor_adamw_step(*args):
+            calls.append(args)
+
+    class L:
+        d_mu, d_alpha, d_delta = "mu", "alpha", "delta"
+
+    upd = bench.FactorUpdate(FakeC, torch, torch.device("cpu"), [4, 6])
+    assert [m.numel() for m in upd.moments] == [24, 36]
+    lrs = []
+    for _ in range(3):
+        upd.advance()
+        lrs.append(upd.lr)
+        upd.apply(1, L, ["g0", "g1", "g2"])
+    assert lrs[0] == pytest.approx(bench.LR0)
+    assert lrs[1] == pytest.approx(bench.LR0 * (1 - 1 / bench.UPDATES), rel=1e-6)
+    assert [c[-2] for c in calls] == [1, 2, 3]                   # update count t
+    assert calls[0][:6] == ("mu", "alpha", "delta", "g0", "g1", "g2")
+    assert calls[0][6] is upd.moments[1]
+    upd.t = bench.UPDATES
+    upd.advance()
+    assert upd.lr == pytest.approx(bench.LR0)                     # wraps to a fresh decay
