@@ -277,8 +277,8 @@ def _bwd_bufs(layer, X, dY, dX, grads, where, rows=None, groups=None):
     _buf(X, "X", M * layer.K * e, where)
     _buf(dY, "dY", M * layer.N * e, where)
     _buf(dX, "dX", M * layer.K * e, where)
-    for name, t in zip(("g_dmu", "g_dalpha", "g_ddelta"), grads):
-        _buf(t, name, 4 * (layer.G if groups is None else groups), where)
+    for name, arr in zip(("g_dmu", "g_dalpha", "g_ddelta"), grads):
+        _buf(arr, name, 4 * (layer.G if groups is None else groups), where)
 
 
 def catq_bwd_noalloc_max_scratch_bytes() -> int:
@@ -355,9 +355,9 @@ def catq_factor_adamw_step(d_mu, d_alpha, d_delta, g_dmu, g_dalpha, g_ddelta, mo
     """One AdamW update of the factors [G] in place from their gradients; moments [6 * G]
     (zero before the first update) is the optimizer state."""
     G, w = d_mu.numel(), "catq_factor_adamw_step"
-    for name, t in zip(("d_mu", "d_alpha", "d_delta", "g_dmu", "g_dalpha", "g_ddelta"),
-                       (d_mu, d_alpha, d_delta, g_dmu, g_dalpha, g_ddelta)):
-        _buf(t, name, 4 * G, w)
+    for name, arr in zip(("d_mu", "d_alpha", "d_delta", "g_dmu", "g_dalpha", "g_ddelta"),
+                         (d_mu, d_alpha, d_delta, g_dmu, g_dalpha, g_ddelta)):
+        _buf(arr, name, 4 * G, w)
     _buf(moments, "moments", 4 * 6 * G, w)
     _check(lib().catq_factor_adamw_step(d_mu.numel(), _ptr(d_mu), _ptr(d_alpha), _ptr(d_delta), _ptr(g_dmu),
                                         _ptr(g_dalpha), _ptr(g_ddelta), _ptr(moments), ctypes.byref(hp), int(t),
@@ -418,8 +418,8 @@ def _grouped_bufs(layer, row_offsets, where, X=None, Y=None, dY=None, dX=None, g
     _buf(Y, "Y", R * N * e, where)
     _buf(dY, "dY", R * N * e, where)
     _buf(dX, "dX", R * K * e, where)
-    for name, t in zip(("g_dmu", "g_dalpha", "g_ddelta"), grads):
-        _buf(t, name, 4 * E * (N * K // layer.g), where)
+    for name, arr in zip(("g_dmu", "g_dalpha", "g_ddelta"), grads):
+        _buf(arr, name, 4 * E * (N * K // layer.g), where)
 
 
 def catq_grouped_soft_ternary_linear_fwd(layer: GroupedLayer, sched: catq_schedule, X, row_offsets, Y, stream=None):

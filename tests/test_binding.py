@@ -106,3 +106,31 @@ def test_grouped_offsets_and_rows():
         C._grouped_bufs(layer, off, "t", X=X, Y=FakeDev(9 * N - 1, 2))
     with pytest.raises(ValueError, match="g_ddelta"):
         C._grouped_bufs(layer, off, "t", X=X, grads=(FakeDev(E * G), FakeDev(E * G), FakeDev(E * G - 1)))
+
+
+def test_wrappers_pass_their_scalars_through(monkeypatch):
+    """With valid buffers the wrappers reach the library with the caller's scalars (a fake
+    library records the call)."""
+    seen = {}
+
+    class FakeLib:
+        def __getattr__(self, name):
+            def call(*args):
+                seen[name] = args
+                return 0
+            return call
+
+    monkeypatch.setattr(C, "lib", lambda: FakeLib())
+    monkeypatch.setattr(C, "_stream", lambda stream=None: None)
+    G = 10
+    C.catq_factor_adamw_step(*(FakeDev(G) for _ in range(6)), FakeDev(6 * G), C.adamw(), 7, 5e-4)
+    args = seen["catq_factor_adamw_step"]
+    assert args[0] == G and args[-3] == 7 and args[-2] == pytest.approx(5e-4)
+    L = _layer()
+    M = 12
+    X, Y = FakeDev(M * L.K, 2, shape=(M, L.K)), FakeDev(M * L.N, 2, shape=(M, L.N))
+    C.catq_soft_ternary_linear_fwd(L, C.schedule(C.PHASE_SOFT, 30.0), X, Y)
+    assert seen["catq_soft_ternary_linear_fwd"][3] == M
+    C.catq_soft_ternary_linear_bwd(L, C.schedule(C.PHASE_SOFT, 30.0), X, Y, None,
+                                   *(FakeDev(L.G) for _ in range(3)), workspace=FakeDev(256, 1))
+    assert seen["catq_soft_ternary_linear_bwd"][4] == M
