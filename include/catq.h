@@ -95,8 +95,8 @@ typedef enum {
 } catq_recon;
 
 /* Eq. 6 schedule point.  SOFT: s = (t / gamma) * s0 > 0.  HARD: s is the sharpness of the
- * surrogate f used for the backward pass (§2.3, last stage-1 sharpness = s0).  TEACHER:
- * s is ignored. */
+ * surrogate f used for the backward pass (§2.3: the last soft epoch's sharpness, see
+ * catq_schedule_at_epoch).  TEACHER: s is ignored. */
 typedef struct {
   int32_t phase; /* catq_phase */
   float s;
@@ -238,9 +238,11 @@ catq_status catq_hard_ternarize_pack(const catq_layer* layer, uint8_t* codes, fl
 
 /* Eq. 6's schedule point of calibration epoch e of m (host only, no device work):
  * t = e / m; e == 0 is the teacher branch (t = 0); e <= floor(gamma m + 1e-9) the soft
- * stage with s = (t / gamma) s0; later epochs the hard stage with the backward sharpness s0
- * (the last soft value, §2.3).  Requires 0 <= e <= m, m >= 1, 0 < gamma <= 1, finite
- * s0 > 0 and a non-null `out`; else CATQ_ERR_INVALID_ARG. */
+ * stage with s = (t / gamma) s0; later epochs the hard stage, whose backward sharpness is
+ * the last soft epoch's, (floor(gamma m) / m / gamma) s0 (§2.3 keeps the gradients of the
+ * first stage's last iteration): s0 when gamma m is an integer, as at the paper's
+ * defaults; s0 also when no epoch is soft (gamma m < 1).  Requires 0 <= e <= m, m >= 1,
+ * 0 < gamma <= 1, finite s0 > 0 and a non-null `out`; else CATQ_ERR_INVALID_ARG. */
 catq_status catq_schedule_at_epoch(int32_t e, int32_t m, double gamma, double s0, catq_schedule* out);
 
 /* Learning rate of update k (0-based) of `total` under App. B.1's linear decay to zero

@@ -275,17 +275,25 @@ def unpack_codes(codes, n):
 def schedule_at_epoch(e: int, m: int, gamma: float, s0: float):
     """Eq. 6's schedule point of calibration epoch e of m: t = e / m; t = 0 is the teacher
     branch, 0 < t <= gamma the soft stage with s = (t / gamma) s0, gamma < t <= 1 the hard
-    stage, whose backward keeps the last soft sharpness s0 (§2.3).  The comparison
-    t <= gamma is made as e <= floor(gamma m + 1e-9), so that gamma m = 48 at the paper's
-    defaults counts 48 soft epochs whatever the rounding of 0.8 * 60.
+    stage.  The comparison t <= gamma is made as e <= floor(gamma m + 1e-9), so that
+    gamma m = 48 at the paper's defaults counts 48 soft epochs whatever the rounding of
+    0.8 * 60.  The hard stage's backward keeps the sharpness of the last soft epoch (§2.3:
+    the gradients of the last iteration of the first stage), i.e. (t_last / gamma) s0 with
+    t_last = floor(gamma m) / m; that is s0 when gamma m is an integer (the paper's
+    defaults) and below s0 otherwise.  With no soft epoch at all (gamma m < 1) there is no
+    last soft sharpness, and s0 is used.
     Returns (phase, s)."""
     assert 0 <= e <= m and m >= 1 and 0.0 < gamma <= 1.0 and s0 > 0.0
     if e == 0:
         return PHASE_TEACHER, 0.0
-    if e <= int(np.floor(gamma * m + 1e-9)):
+    soft_epochs = int(np.floor(gamma * m + 1e-9))
+    if e <= soft_epochs:
         t = e / m
         return PHASE_SOFT, (t / gamma) * s0
-    return PHASE_HARD, float(s0)
+    if soft_epochs == 0:
+        return PHASE_HARD, float(s0)
+    t_last = soft_epochs / m
+    return PHASE_HARD, (t_last / gamma) * s0
 
 
 def linear_decay_lr(lr0: float, k: int, total: int) -> float:

@@ -501,8 +501,12 @@ catq_status catq_schedule_at_epoch(int32_t e, int32_t m, double gamma, double s0
   } else if (e <= soft_epochs) {
     const double t = static_cast<double>(e) / m;
     *out = catq_schedule{CATQ_PHASE_SOFT, static_cast<float>(t / gamma * s0)};
+  } else if (soft_epochs == 0) {
+    *out = catq_schedule{CATQ_PHASE_HARD, static_cast<float>(s0)};  // no soft epoch to inherit from
   } else {
-    *out = catq_schedule{CATQ_PHASE_HARD, static_cast<float>(s0)};
+    // the last soft epoch's sharpness (§2.3): s0 when gamma m is an integer
+    const double t_last = static_cast<double>(soft_epochs) / m;
+    *out = catq_schedule{CATQ_PHASE_HARD, static_cast<float>(t_last / gamma * s0)};
   }
   return CATQ_OK;
 }

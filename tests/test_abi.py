@@ -108,7 +108,8 @@ def test_schedule_and_lr_host_calls_follow_the_oracle(lib):
     """The host-only schedule calls against the oracle: the branch exactly, s and the
     learning rate to fp32 rounding."""
     from oracle import catq_oracle as O
-    for m, gamma, s0 in [(60, 0.8, 30.0), (10, 1.0, 5.0), (7, 0.5, 12.0), (100, 0.57, 30.0), (1, 0.3, 2.0)]:
+    for m, gamma, s0 in [(60, 0.8, 30.0), (10, 1.0, 5.0), (7, 0.5, 12.0), (100, 0.57, 30.0), (1, 0.3, 2.0),
+                          (10, 0.75, 30.0), (3, 0.2, 30.0)]:
         for e in range(m + 1):
             got = C.catq_schedule_at_epoch(e, m, gamma, s0)
             phase, s = O.schedule_at_epoch(e, m, gamma, s0)

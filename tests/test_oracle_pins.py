@@ -336,6 +336,39 @@ def test_bwd_uses_transposes_correctly_non_square():
     np.testing.assert_allclose(step["Y_ref"], Y_ref)
 
 
+def _golden(name):
+    vals = {}
+    with open(os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", name)) as fh:
+        for line in fh:
+            if line.startswith("#") or ":" not in line:
+                continue
+            k, v = line.split(":", 1)
+            vals[k.strip()] = np.array([float(t) for t in v.split()])
+    return vals
+
+
+def test_hard_gradients_hand_computed_golden():
+    """The HARD-phase reading (§2.3, stage 2 keeps the last soft iteration's gradients) on a
+    hand-computed group at s = 2, where f and Q differ (tests/golden/hard_grad_example.txt):
+    the alpha term must use the forward value T = Q; substituting T = f moves g_dalpha from
+    -0.472 to -0.408 and fails.  The same numbers pin d_mu and d_delta's derivatives of Eq. 5,
+    and the SOFT phase must reproduce the T = f value."""
+    gd = _golden("hard_grad_example.txt")
+    W = gd["W"].reshape(1, 4)
+    Gw = gd["G"].reshape(1, 4)
+    s = float(gd["s"][0])
+    stats = O.group_stats(W, 4)
+    fac = (np.zeros(1), np.ones(1), np.ones(1))
+    got = O.factor_grads_from_G(Gw, W, 4, stats, fac, O.PHASE_HARD, s)
+    for name, v in zip(("g_dmu", "g_dalpha", "g_ddelta"), got):
+        np.testing.assert_allclose(v, gd[name], rtol=1e-12, err_msg=name)
+    assert abs(got[1][0] - gd["g_dalpha_if_T_were_f"][0]) > 0.05
+    soft = O.factor_grads_from_G(Gw, W, 4, stats, fac, O.PHASE_SOFT, s)
+    np.testing.assert_allclose(soft[1], gd["g_dalpha_if_T_were_f"], rtol=1e-12)
+    np.testing.assert_allclose(soft[0], gd["g_dmu"], rtol=1e-12)
+    np.testing.assert_allclose(soft[2], gd["g_ddelta"], rtol=1e-12)
+
+
 def test_hard_gradients_reading_self_consistency():
     """HARD-phase factor gradients (parity unpinned: §2.3's stage-2 rule read as a
     surrogate) coincide with the SOFT ones at the same large s when no element sits
@@ -598,6 +631,20 @@ def test_schedule_at_epoch_paper_defaults():
     assert sum(O.schedule_at_epoch(e, 7, 0.5, 5.0)[0] == O.PHASE_SOFT for e in range(1, 8)) == 3
     # rounding of gamma m (0.57 * 100 = 56.99999999999999 in fp64) does not drop an epoch
     assert sum(O.schedule_at_epoch(e, 100, 0.57, 5.0)[0] == O.PHASE_SOFT for e in range(1, 101)) == 57
+
+
+def test_hard_stage_keeps_the_last_soft_sharpness():
+    """§2.3: the hard stage takes the gradients of the first stage's last iteration, so its
+    backward sharpness is the last soft epoch's.  With gamma m = 7.5 (m = 10, gamma = 0.75)
+    the soft stage ends at e = 7 with s = (0.7 / 0.75) s0 = 28 for s0 = 30, not s0; with
+    gamma m < 1 there is no soft epoch and s0 is kept."""
+    m, gamma, s0 = 10, 0.75, 30.0
+    phases = [O.schedule_at_epoch(e, m, gamma, s0) for e in range(1, m + 1)]
+    assert [p for p, _ in phases] == [O.PHASE_SOFT] * 7 + [O.PHASE_HARD] * 3
+    last_soft = phases[6][1]
+    assert last_soft == pytest.approx(28.0, rel=1e-15)
+    assert all(s == last_soft for _, s in phases[7:])
+    assert [O.schedule_at_epoch(e, 3, 0.2, s0) for e in (1, 2, 3)] == [(O.PHASE_HARD, s0)] * 3
 
 
 def test_linear_decay_lr_closed_form():
