@@ -671,20 +671,18 @@ __global__ void __launch_bounds__(kThreads) grad_reduce_grouped_kernel(LayerDev 
 }
 
 // ---------------------------------------------------------------- factor update (AdamW)
-// One thread per group and factor array: decoupled decay, the two moment updates, the
-// bias-corrected step and the projection of the factor's constraint.  Comparisons keep NaN
-// as NaN (a NaN factor is not hidden at a bound).  Reads 16 B and writes 12 B per element.
-__global__ void __launch_bounds__(kThreads) factor_adamw_kernel(int64_t G, const AdamwArgs a) {
-  for (int64_t j = blockIdx.x * (int64_t)kThreads + threadIdx.x; j < 3 * G; j += (int64_t)gridDim.x * kThreads) {
-    const int q = static_cast<int>(j / G);
-    const int64_t i = j - q * G;
-    // constant indices into the parameter arrays (no local copy of the argument block)
-    float* const P = q == 0 ? a.p[0] : q == 1 ? a.p[1] : a.p[2];
-    const float* const Gr = q == 0 ? a.g[0] : q == 1 ? a.g[1] : a.g[2];
-    float* const Mo = q == 0 ? a.m[0] : q == 1 ? a.m[1] : a.m[2];
-    float* const Vo = q == 0 ? a.v[0] : q == 1 ? a.v[1] : a.v[2];
-    const float lo = q == 0 ? a.lo[0] : q == 1 ? a.lo[1] : a.lo[2];
-    const float hi = q == 0 ? a.hi[0] : q == 1 ? a.hi[1] : a.hi[2];
+// One thread per group and factor array (blockIdx.y = the factor): decoupled decay, the two
+// moment updates, the bias-corrected step and the projection of the factor's constraint.
+// Comparisons keep NaN as NaN (a NaN factor is not hidden at a bound).  Reads 16 B and
+// writes 12 B per element.
+template <int Q>
+__device__ __forceinline__ void factor_adamw_array(int64_t G, const AdamwArgs& a) {
+  float* const P = a.p[Q];
+  const float* const Gr = a.g[Q];
+  float* const Mo = a.m[Q];
+  float* const Vo = a.v[Q];
+  const float lo = a.lo[Q], hi = a.hi[Q];
+  for (int64_t i = blockIdx.x * (int64_t)kThreads + threadIdx.x; i < G; i += (int64_t)gridDim.x * kThreads) {
     const float grad = Gr[i];
     float p = P[i] * a.decay;
     const float m = fmaf(a.beta1, Mo[i], a.one_minus_beta1 * grad);
@@ -696,6 +694,14 @@ __global__ void __launch_bounds__(kThreads) factor_adamw_kernel(int64_t G, const
     Mo[i] = m;
     Vo[i] = v;
   }
+}
+
+__global__ void __launch_bounds__(kThreads) factor_adamw_kernel(int64_t G, const AdamwArgs a) {
+  // blockIdx.y is uniform per block: each block walks one factor array, no per-element
+  // division or pointer select
+  if (blockIdx.y == 0) factor_adamw_array<0>(G, a);
+  else if (blockIdx.y == 1) factor_adamw_array<1>(G, a);
+  else factor_adamw_array<2>(G, a);
 }
 
 int grid_for(int64_t work, int64_t per_block) {
@@ -865,7 +871,7 @@ cudaError_t launch_grad_reduce(const LayerDev& L, StepScalars sc, const float* p
 
 cudaError_t launch_factor_adamw(int64_t G, const AdamwArgs& a, cudaStream_t st) {
   if (G == 0) return cudaSuccess;
-  factor_adamw_kernel<<<grid_for(3 * G, kThreads), kThreads, 0, st>>>(G, a);
+  factor_adamw_kernel<<<dim3(grid_for(G, kThreads), 3), kThreads, 0, st>>>(G, a);
   return cudaGetLastError();
 }
 

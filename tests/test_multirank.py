@@ -86,8 +86,8 @@ def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
 def test_factor_update_sequence_of_the_bench_step():
     """bench.py's step closes with one AdamW update per linear: the update count rises by
     one per step, the learning rate follows the linear decay of App. B.1 through the
-    library's host call and wraps after a full calibration's updates, and every linear gets
-    its own moments of 6 G floats."""
+    library's host call, a full calibration's updates later a fresh calibration starts (count
+    1, zero moments), and every linear gets its own moments of 6 G floats."""
     from paper_2606_26650_gb300 import catq as C
 
     calls = []
@@ -115,6 +115,9 @@ def test_factor_update_sequence_of_the_bench_step():
     assert [c[-2] for c in calls] == [1, 2, 3]                   # update count t
     assert calls[0][:6] == ("mu", "alpha", "delta", "g0", "g1", "g2")
     assert calls[0][6] is upd.moments[1]
+    upd.moments[1].fill_(0.5)
     upd.t = bench.UPDATES
     upd.advance()
-    assert upd.lr == pytest.approx(bench.LR0)                     # wraps to a fresh decay
+    assert upd.lr == pytest.approx(bench.LR0)                     # a fresh calibration starts:
+    assert upd.t == 1                                             # first update again (bias correction)
+    assert not upd.moments[1].any()                               # and zero moments
