@@ -13,7 +13,8 @@ group.
 
 Pins (tests/test_oracle_pins.py) tie each function to something other than itself:
 brute force, closed forms, limits and finite differences; the optimizer update also to
-PyTorch's own AdamW.  One part is
+PyTorch's own AdamW; the 8-bit activation quantizer to exact grids, its error bound and a
+brute-force nearest code.  One part is
 "parity unpinned": the HARD-phase factor gradients (see ``linear_bwd``), which rest on
 this library's reading of §2.3's stage-2 rule and have no independent reference.
 """
@@ -220,6 +221,41 @@ def calibration_step(X, W, g, stats, factors, phase, s, reduction=0, with_mu=Fal
     dX, g_dmu, g_dalpha, g_ddelta = linear_bwd(X, dY, W, g, stats, factors, phase, s, with_mu)
     return dict(Y_ref=Y_ref, Y=Y, loss=loss, dY=dY, dX=dX, g_dmu=g_dmu, g_dalpha=g_dalpha,
                 g_ddelta=g_ddelta, Wq=Wq)
+
+
+def act_quant_a8(X):
+    """Per-token symmetric 8-bit quantization of a linear's input, the activation side of
+    the W1.58A8 setting (§1, App. B.2; the paper does not state the quantizer, and this is
+    the reading of dynamic per-token absmax quantization):
+        scale_m = max_k |X[m, k]| / 127,   q[m, k] = clamp(round(X[m, k] / scale_m), -127, 127)
+    with round-half-to-even, and scale 0 with q = 0 for a row of zeros.  Because the scale
+    and the quotient decide integer codes, both are taken in fp32 with IEEE division (the
+    precision of the kernel); everything after them is fp64.
+    Returns (q [M, K] int64, scale [M] float32)."""
+    X32 = np.asarray(X, np.float32)
+    amax = np.abs(X32).max(axis=1)
+    scale = (amax / np.float32(127.0)).astype(np.float32)
+    safe = np.where(scale > 0, scale, np.float32(1.0)).astype(np.float32)
+    q = np.clip(np.rint(X32 / safe[:, None]), -127, 127)
+    q[scale == 0] = 0
+    return q.astype(np.int64), scale
+
+
+def a8_calibration_step(X, W, g, stats, factors, phase, s, reduction=0, with_mu=False):
+    """One calibration step of a linear whose input is quantized to 8 bits per token
+    (``act_quant_a8``): the teacher is the full-precision output X W^T (Eq. 7's F(W, X)),
+    the quantized output Y = X_q Wq^T with X_q = scale q; the rounding passes gradients
+    straight through, so dX = dY Wq, and G = dY^T X_q is the gradient of Wq.  Returns the
+    dict of ``calibration_step`` plus q, scale and X_q."""
+    q, scale = act_quant_a8(X)
+    Xq = q.astype(np.float64) * scale.astype(np.float64)[:, None]
+    Y_ref = linear_fwd(X, W)
+    Wq = ternary_weight(W, g, stats, factors, phase, s, with_mu)[0]
+    Y = linear_fwd(Xq, Wq)
+    loss, dY = recon_loss(Y, Y_ref, reduction)
+    dX, g_dmu, g_dalpha, g_ddelta = linear_bwd(Xq, dY, W, g, stats, factors, phase, s, with_mu)
+    return dict(Y_ref=Y_ref, Y=Y, loss=loss, dY=dY, dX=dX, g_dmu=g_dmu, g_dalpha=g_dalpha,
+                g_ddelta=g_ddelta, Wq=Wq, q=q, scale=scale, Xq=Xq)
 
 
 def hard_codes(W, g, stats, factors):

@@ -752,3 +752,64 @@ def test_calibration_loop_lowers_the_hard_reconstruction_error():
             t += 1
             fac, mom = O.factor_update(fac, (step["g_dmu"], step["g_dalpha"], step["g_ddelta"]), mom, t, lr)
     assert hard_loss(fac) < 0.9 * start
+
+
+# ----------------------------------------------------------------- W1.58A8: 8-bit activations
+
+def test_act_quant_a8_exact_on_its_own_grid():
+    """Rows that already lie on an 8-bit grid whose largest entry is +-127 steps come back
+    exactly: the scale is the grid step (a power of two here, so fp32 division is exact)
+    and the codes are the integers; each row has its own scale (per token)."""
+    r = np.random.default_rng(30)
+    M, K = 5, 48
+    steps = 2.0 ** r.integers(-12, -2, M)
+    ints = r.integers(-127, 128, (M, K))
+    ints[np.arange(M), r.integers(0, K, M)] = np.where(r.random(M) < 0.5, 127, -127)
+    X = ints * steps[:, None]
+    q, scale = O.act_quant_a8(X)
+    np.testing.assert_array_equal(scale, steps.astype(np.float32))
+    np.testing.assert_array_equal(q, ints)
+
+
+def test_act_quant_a8_error_bound_and_range():
+    """Round-to-nearest on a symmetric grid: every element within half a step of scale q,
+    codes in [-127, 127], the row's absmax at +-127, and a zero row giving zero codes."""
+    r = np.random.default_rng(31)
+    X = (r.standard_t(4.0, (64, 200)) * 3).astype(np.float32)
+    X[7] = 0.0
+    q, scale = O.act_quant_a8(X)
+    assert np.abs(q).max() <= 127
+    err = np.abs(X.astype(np.float64) - q * scale[:, None].astype(np.float64))
+    assert np.all(err <= 0.5 * scale[:, None] * (1 + 1e-6) + 1e-30)
+    live = np.arange(64) != 7
+    assert np.all(np.abs(q[live]).max(axis=1) == 127)
+    assert scale[7] == 0 and not q[7].any()
+
+
+def test_act_quant_a8_is_the_nearest_code_by_brute_force():
+    """Each code is the integer in [-127, 127] nearest to x / scale (all 255 candidates
+    tried; ties, if any, to the even one)."""
+    r = np.random.default_rng(32)
+    X = r.standard_normal((6, 40)).astype(np.float32)
+    q, scale = O.act_quant_a8(X)
+    cand = np.arange(-127, 128)
+    for m in range(6):
+        u = X[m].astype(np.float32) / scale[m]
+        dist = np.abs(u[:, None].astype(np.float64) - cand[None, :])
+        best = dist.min(axis=1)
+        np.testing.assert_allclose(np.abs(u - q[m]), best, atol=1e-6)
+
+
+def test_a8_step_reduces_to_the_plain_step_on_grid_inputs():
+    """When X already lies on its 8-bit grid the quantizer is the identity, so the A8 step
+    (teacher from X, forward and dW from X_q) equals the plain calibration step."""
+    W, X, g, stats, fac = _tiny(seed=33, N=8, K=16, g=8, M=6)
+    r = np.random.default_rng(33)
+    ints = r.integers(-127, 128, X.shape)
+    ints[:, 0] = 127
+    X = ints * 2.0 ** -7
+    a8 = O.a8_calibration_step(X, W, g, stats, fac, O.PHASE_SOFT, 15.0)
+    ref = O.calibration_step(X, W, g, stats, fac, O.PHASE_SOFT, 15.0)
+    for k in ("Y", "Y_ref", "dY", "dX", "g_dmu", "g_dalpha", "g_ddelta"):
+        np.testing.assert_allclose(a8[k], ref[k], rtol=1e-13, atol=1e-15, err_msg=k)
+    assert a8["loss"] == pytest.approx(ref["loss"], rel=1e-13)
