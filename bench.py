@@ -6,7 +6,9 @@ a decoder block (default: the Llama-3-8B-shaped block, 4 x 2048 tokens):
   group statistics (Eq. 3) -> fused soft-ternary forward Y = X Wq^T (Eq. 5/6, s = 30)
   -> reconstruction loss and dY against the cached teacher output (Eq. 7)
   -> dX = dY Wq -> factor gradients from dY^T X (chain rule of Eq. 3/5/6)
-  -> hard ternarization + 2-bit pack (Eq. 2/4).
+  -> AdamW update of the factors -> hard ternarization + 2-bit pack (Eq. 2/4).
+The forward and the loss run as two calls: the fused call (catq_soft_ternary_linear_fwd_loss)
+is exact but slower on this GPU (its epilogue lengthens the accumulator drain).
 The metric is the algorithmic 6 M N K flops per linear (fwd + dX + dW) per second.
 
 Prints ONE JSON line (rank 0).  `--impl reference` times the fp64 CPU oracle instead (the
@@ -459,6 +461,7 @@ def run_ours(args):
     traffic = (TRAFFIC.get(dom) if TRAFFIC.get("sha") == sha and TRAFFIC.get("workload") == wl.name
                else None)
     esz = 2 if wl.dtype == "bf16" else 4
+    # forward: X, W, Y; dX: dY, W, dX; dW: dY, X, W (plus the per-group arrays)
     algo_bytes = sum(esz * (M * d["lin"].K + d["lin"].N * d["lin"].K + M * d["lin"].N)
                      + 4 * (d["lin"].N * d["lin"].K // wl.g) * (9 if dom == "dw" else 6) for d in st) / len(st)
     # The per-kernel durations come from a region of `steps` steps on one stream (a fraction

@@ -160,6 +160,63 @@ catq_status catq_soft_ternary_linear_fwd(const catq_layer* layer, catq_schedule 
                                          const void* X, int64_t M, int32_t x_dtype, void* Y,
                                          catq_stream stream);
 
+/* Forward with the two options the plain forward lacks (Eq. 6 weight; §1 and App. B.2's
+ * weight-activation setting):
+ *   Y[m, :] = x_row_scale[m] * (X Wq^T)[m, :]   (x_row_scale NULL: scale 1)
+ * x_row_scale [M] fp32 (4-byte aligned) is the per-token scale of 8-bit activation codes
+ * in X (catq_act_quant_a8): X then holds the integer codes, exact in bf16, and the scale
+ * is applied to the fp32 accumulator before the output rounding.  y_dtype is x_dtype or
+ * CATQ_F32 (an fp32 output of a bf16 layer, e.g. a full-precision teacher output for
+ * catq_soft_ternary_linear_fwd_loss); fp32 layers need CATQ_F32.  Other arguments and
+ * errors as catq_soft_ternary_linear_fwd. */
+catq_status catq_soft_ternary_linear_fwd_ex(const catq_layer* layer, catq_schedule sched, const void* X,
+                                            int64_t M, int32_t x_dtype, const float* x_row_scale, void* Y,
+                                            int32_t y_dtype, catq_stream stream);
+
+/* Workspace bytes catq_soft_ternary_linear_fwd_loss needs for this layer and M on the
+ * current device (fp64 partial sums of the loss). */
+size_t catq_fwd_loss_workspace_bytes(const catq_layer* layer, int64_t M);
+
+/* Forward and reconstruction loss of one linear in one pass (Eq. 6 weight, Eq. 7 loss):
+ *   Y = diag(x_row_scale) X Wq^T     (the accumulator, never rounded before the loss)
+ *   loss_out[0] = sum (Y - Y_ref)^2 / (M N)  (CATQ_REDUCE_MEAN)  or the plain sum (SUM)
+ *   dY          = 2 (Y - Y_ref) / (M N)      (MEAN)              or 2 (Y - Y_ref) (SUM)
+ * The bf16 path forms Y - Y_ref in the GEMM's epilogue from the fp32 accumulator, so Y is
+ * rounded neither before the difference nor (unless requested) at all; dY is rounded once
+ * to bf16.  Y_ref [M, N] has ref_dtype: x_dtype, or CATQ_F32 for a full-precision teacher of
+ * a bf16 layer.  dY [M, N] (x_dtype) is required; Y [M, N] (x_dtype) is optional (NULL:
+ * not stored).  x_row_scale as in catq_soft_ternary_linear_fwd_ex (NULL: 1).  loss_out:
+ * device fp32 scalar.  The loss sums fp32 compensated partials per epilogue warp, then
+ * the partials in fp64, in a fixed order (deterministic for a given device and shape).
+ * fp32 layers run the CUDA-core forward (into Y, or into dY as scratch) and then the loss
+ * kernel.  M >= 1 (else CATQ_ERR_SHAPE); X, Y_ref, dY, Y 16-byte aligned; workspace
+ * >= catq_fwd_loss_workspace_bytes(layer, M), 256-byte aligned.
+ * Cost: the loss lengthens the GEMM's accumulator drain, which the next tile's MMAs wait
+ * for, so on a GB300 this call takes longer than catq_soft_ternary_linear_fwd followed by
+ * catq_recon_loss (8B-shaped gate_proj, 8192 tokens: 827 us against 571 + 121 us).  Use it
+ * where the unrounded Y - Y_ref matters; the two calls are the faster path. */
+catq_status catq_soft_ternary_linear_fwd_loss(const catq_layer* layer, catq_schedule sched, const void* X,
+                                              int64_t M, int32_t x_dtype, const float* x_row_scale,
+                                              const void* Y_ref, int32_t ref_dtype, int32_t reduction,
+                                              float* loss_out, void* dY, void* Y, void* workspace,
+                                              size_t ws_bytes, catq_stream stream);
+
+/* Per-token symmetric 8-bit quantization of activations X [M, K] (the weight-activation
+ * setting W1.58A8 of §1 and App. B.2, which leaves the activation quantizer unstated; this
+ * library reads it as dynamic per-token absmax quantization):
+ *   scale[m]    = max_k |X[m, k]| / 127                      (fp32, IEEE division)
+ *   codes[m, k] = clamp(rint(X[m, k] / scale[m]), -127, 127)  (fp32 IEEE division, ties to
+ *                 even), 0 for a row of zeros (scale 0)
+ *   X_deq[m, k] = scale[m] * codes[m, k], computed in fp32 and rounded to x_dtype (nullable)
+ * codes and X_deq have x_dtype (integers up to 127 are exact in bf16) and [M, K] layout;
+ * scale [M] fp32.  The forward uses codes with x_row_scale = scale
+ * (catq_soft_ternary_linear_fwd_ex / _fwd_loss); the backward's dW uses X_deq (the
+ * rounding is passed straight through to dX).  K * sizeof(x_dtype) must be a multiple of 16
+ * (else CATQ_ERR_SHAPE); X, codes, X_deq 16-byte aligned, scale 4-byte.  M == 0 is a
+ * no-op. */
+catq_status catq_act_quant_a8(const void* X, int64_t M, int64_t K, int32_t x_dtype, void* codes, float* scale,
+                              void* X_deq, catq_stream stream);
+
 /* Workspace bytes catq_soft_ternary_linear_bwd needs for this layer and M (partial
  * per-group sums); 0 is never returned for M > 0. */
 size_t catq_bwd_workspace_bytes(const catq_layer* layer, int64_t M);
@@ -313,6 +370,21 @@ typedef struct {
 catq_status catq_grouped_soft_ternary_linear_fwd(const catq_grouped_layer* layer, catq_schedule sched,
                                                  const void* X, const int64_t* row_offsets,
                                                  int32_t x_dtype, void* Y, catq_stream stream);
+
+/* Workspace bytes catq_grouped_soft_ternary_linear_fwd_loss needs on the current device. */
+size_t catq_grouped_fwd_loss_workspace_bytes(const catq_grouped_layer* layer, const int64_t* row_offsets);
+
+/* Forward of every expert and the reconstruction loss over all routed rows R in one pass
+ * (see catq_soft_ternary_linear_fwd_loss; count = R N): loss_out, dY [R, N] (required) and
+ * Y [R, N] (nullable) from X [R, K] and Y_ref [R, N] of x_dtype.  bf16 layers with at most
+ * 128 experts run one persistent launch over every expert's tiles with the loss in its
+ * epilogue; other layers compute Y expert by expert (into dY when Y is NULL), then the
+ * loss.  R >= 1 (else CATQ_ERR_SHAPE). */
+catq_status catq_grouped_soft_ternary_linear_fwd_loss(const catq_grouped_layer* layer, catq_schedule sched,
+                                                      const void* X, const int64_t* row_offsets, int32_t x_dtype,
+                                                      const void* Y_ref, int32_t reduction, float* loss_out,
+                                                      void* dY, void* Y, void* workspace, size_t ws_bytes,
+                                                      catq_stream stream);
 
 /* Workspace bytes catq_grouped_soft_ternary_linear_bwd needs: for bf16 layers with at most
  * 128 experts, every expert's partial group sums at once (E * 3 * N * K/gcd(g, 128) fp32);

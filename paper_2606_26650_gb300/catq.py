@@ -101,6 +101,13 @@ def lib() -> ctypes.CDLL:
         "catq_factor_adamw_step": (I32, [I64, P, P, P, P, P, P, P, ctypes.POINTER(catq_adamw), I64, F, P]),
         "catq_grouped_soft_ternary_linear_bwd": (I32, [ctypes.POINTER(catq_grouped_layer), catq_schedule, P, P, P, I32,
                                                        P, P, P, P, P, S, P]),
+        "catq_soft_ternary_linear_fwd_ex": (I32, [LP, catq_schedule, P, I64, I32, P, P, I32, P]),
+        "catq_fwd_loss_workspace_bytes": (S, [LP, I64]),
+        "catq_soft_ternary_linear_fwd_loss": (I32, [LP, catq_schedule, P, I64, I32, P, P, I32, I32, P, P, P, P, S, P]),
+        "catq_act_quant_a8": (I32, [P, I64, I64, I32, P, P, P, P]),
+        "catq_grouped_fwd_loss_workspace_bytes": (S, [ctypes.POINTER(catq_grouped_layer), P]),
+        "catq_grouped_soft_ternary_linear_fwd_loss": (I32, [ctypes.POINTER(catq_grouped_layer), catq_schedule, P, P,
+                                                            I32, P, I32, P, P, P, P, S, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -242,6 +249,54 @@ def catq_soft_ternary_linear_fwd(layer: Layer, sched: catq_schedule, X, Y, strea
     _buf(Y, "Y", M * layer.N * e, w)
     _check(lib().catq_soft_ternary_linear_fwd(ctypes.byref(st), sched, _ptr(X), X.shape[0], _dtype_code(X),
                                               _ptr(Y), _stream(stream)), "catq_soft_ternary_linear_fwd")
+
+
+def catq_soft_ternary_linear_fwd_ex(layer: Layer, sched: catq_schedule, X, Y, x_row_scale=None, stream=None):
+    """Y = diag(x_row_scale) X Wq^T; Y may be fp32 for a bf16 layer."""
+    st = layer.struct()
+    M, w = X.shape[0], "catq_soft_ternary_linear_fwd_ex"
+    _buf(X, "X", M * layer.K * X.element_size(), w)
+    _buf(Y, "Y", M * layer.N * (Y.element_size() if Y is not None else 0), w)
+    _buf(x_row_scale, "x_row_scale", 4 * M, w)
+    _check(lib().catq_soft_ternary_linear_fwd_ex(ctypes.byref(st), sched, _ptr(X), M, _dtype_code(X),
+                                                 _ptr(x_row_scale), _ptr(Y), _dtype_code(Y), _stream(stream)), w)
+
+
+def catq_fwd_loss_workspace_bytes(layer: Layer, M: int) -> int:
+    st = layer.struct()
+    return int(lib().catq_fwd_loss_workspace_bytes(ctypes.byref(st), int(M)))
+
+
+def catq_soft_ternary_linear_fwd_loss(layer: Layer, sched: catq_schedule, X, Y_ref, loss_out, dY, Y=None,
+                                      x_row_scale=None, workspace=None, reduction: int = REDUCE_MEAN, stream=None):
+    """Forward, Eq. 7 loss and dY in one pass; Y_ref may be fp32 for a bf16 layer."""
+    st = layer.struct()
+    M, e, w = X.shape[0], X.element_size(), "catq_soft_ternary_linear_fwd_loss"
+    _buf(X, "X", M * layer.K * e, w)
+    _buf(Y_ref, "Y_ref", M * layer.N * Y_ref.element_size(), w)
+    _buf(dY, "dY", M * layer.N * e, w)
+    _buf(Y, "Y", M * layer.N * e, w)
+    _buf(loss_out, "loss_out", 4, w)
+    _buf(x_row_scale, "x_row_scale", 4 * M, w)
+    _buf(workspace, "workspace", 0, w)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib().catq_soft_ternary_linear_fwd_loss(ctypes.byref(st), sched, _ptr(X), M, _dtype_code(X),
+                                                   _ptr(x_row_scale), _ptr(Y_ref), _dtype_code(Y_ref),
+                                                   int(reduction), _ptr(loss_out), _ptr(dY), _ptr(Y),
+                                                   _ptr(workspace), ws_bytes, _stream(stream)), w)
+
+
+def catq_act_quant_a8(X, codes, scale, X_deq=None, stream=None):
+    """Per-token 8-bit codes (as exact values of X's dtype), scales [M] and (optionally) the
+    dequantized activations."""
+    M, K = X.shape
+    n, w = M * K * X.element_size(), "catq_act_quant_a8"
+    _buf(X, "X", n, w)
+    _buf(codes, "codes", n, w)
+    _buf(X_deq, "X_deq", n, w)
+    _buf(scale, "scale", 4 * M, w)
+    _check(lib().catq_act_quant_a8(_ptr(X), M, K, _dtype_code(X), _ptr(codes), _ptr(scale), _ptr(X_deq),
+                                   _stream(stream)), w)
 
 
 def catq_bwd_workspace_bytes(layer: Layer, M: int) -> int:
@@ -447,3 +502,25 @@ def catq_grouped_soft_ternary_linear_bwd(layer: GroupedLayer, sched: catq_schedu
                                                       _offsets(row_offsets), _dtype_code(X), _ptr(dX), _ptr(g_dmu),
                                                       _ptr(g_dalpha), _ptr(g_ddelta), _ptr(workspace), ws_bytes,
                                                       _stream(stream)), "catq_grouped_soft_ternary_linear_bwd")
+
+
+def catq_grouped_fwd_loss_workspace_bytes(layer: GroupedLayer, row_offsets) -> int:
+    st = layer.struct()
+    _grouped_bufs(layer, row_offsets, "catq_grouped_fwd_loss_workspace_bytes")
+    return int(lib().catq_grouped_fwd_loss_workspace_bytes(ctypes.byref(st), _offsets(row_offsets)))
+
+
+def catq_grouped_soft_ternary_linear_fwd_loss(layer: GroupedLayer, sched: catq_schedule, X, row_offsets, Y_ref,
+                                              loss_out, dY, Y=None, workspace=None, reduction: int = REDUCE_MEAN,
+                                              stream=None):
+    st = layer.struct()
+    w = "catq_grouped_soft_ternary_linear_fwd_loss"
+    _grouped_bufs(layer, row_offsets, w, X=X, Y=Y, dY=dY)
+    _grouped_bufs(layer, row_offsets, w, Y=Y_ref)
+    _buf(loss_out, "loss_out", 4, w)
+    _buf(workspace, "workspace", 0, w)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib().catq_grouped_soft_ternary_linear_fwd_loss(ctypes.byref(st), sched, _ptr(X), _offsets(row_offsets),
+                                                           _dtype_code(X), _ptr(Y_ref), int(reduction),
+                                                           _ptr(loss_out), _ptr(dY), _ptr(Y), _ptr(workspace),
+                                                           ws_bytes, _stream(stream)), w)

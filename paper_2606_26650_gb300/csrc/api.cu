@@ -3,6 +3,7 @@
 // here allocates memory; every launch goes to the caller's stream.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 #include <mutex>
@@ -118,6 +119,13 @@ size_t bwd_partials_bytes(const catq_layer* L, int64_t M, TcPlan* plan_out, int3
   return 3 * static_cast<size_t>(L->N) * static_cast<size_t>(L->K / P) * sizeof(float);
 }
 
+// Fused-loss workspace: the fp64 loss partials (one per epilogue warp of the bf16 GEMM, or
+// the loss kernel's block partials on the fp32 path).
+size_t fwd_loss_ws_bytes(int64_t count) {
+  const int parts = std::max(fused_loss_max_parts(current_sm_count()), recon_loss_blocks(count < 1 ? 1 : count));
+  return round256(static_cast<size_t>(parts) * sizeof(double));
+}
+
 // Scratch of catq_soft_ternary_linear_bwd_noalloc: the dW epilogue's partial group sums.
 // Every GPU that loads the library holds this array until the process exits.
 constexpr size_t kNoAllocScratchBytes = size_t(16) << 20;
@@ -202,6 +210,96 @@ catq_status catq_soft_ternary_linear_fwd(const catq_layer* layer, catq_schedule 
     return cuda_status(launch_simt_fwd(L, scalars(sched), static_cast<const float*>(X), M, static_cast<float*>(Y), s));
   if ((st = check_tensor_core_device()) != CATQ_OK) return st;
   return cuda_status(launch_tc_fwd(L, scalars(sched), X, M, Y, s));
+}
+
+catq_status catq_soft_ternary_linear_fwd_ex(const catq_layer* layer, catq_schedule sched, const void* X, int64_t M,
+                                            int32_t x_dtype, const float* x_row_scale, void* Y, int32_t y_dtype,
+                                            catq_stream stream) {
+  catq_status st = check_layer(layer, sched.phase != CATQ_PHASE_TEACHER);
+  if (st != CATQ_OK) return st;
+  if ((st = check_schedule(sched, sched.phase == CATQ_PHASE_SOFT)) != CATQ_OK) return st;
+  if (x_dtype != layer->w_dtype) return CATQ_ERR_DTYPE;
+  if (y_dtype != x_dtype && y_dtype != CATQ_F32) return CATQ_ERR_DTYPE;
+  if (M < 0) return CATQ_ERR_SHAPE;
+  if (M == 0) return CATQ_OK;
+  if (!X || !Y) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(X) || !aligned16(Y) || (reinterpret_cast<uintptr_t>(x_row_scale) & 3u)) return CATQ_ERR_ALIGN;
+  if ((st = check_op_const(layer, sched)) != CATQ_OK) return st;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const LayerDev L = to_dev(layer);
+  if (layer->w_dtype == CATQ_F32)
+    return cuda_status(
+        launch_simt_fwd(L, scalars(sched), static_cast<const float*>(X), M, static_cast<float*>(Y), s, x_row_scale));
+  if ((st = check_tensor_core_device()) != CATQ_OK) return st;
+  EpiOpts o;
+  o.y_f32 = y_dtype == CATQ_F32;
+  o.row_scale = x_row_scale;
+  return cuda_status(launch_tc_fwd(L, scalars(sched), X, M, Y, s, &o));
+}
+
+size_t catq_fwd_loss_workspace_bytes(const catq_layer* layer, int64_t M) {
+  if (!layer || layer->N < 1) return 0;
+  if (M < 1) M = 1;
+  return fwd_loss_ws_bytes(M * layer->N);
+}
+
+catq_status catq_soft_ternary_linear_fwd_loss(const catq_layer* layer, catq_schedule sched, const void* X, int64_t M,
+                                              int32_t x_dtype, const float* x_row_scale, const void* Y_ref,
+                                              int32_t ref_dtype, int32_t reduction, float* loss_out, void* dY,
+                                              void* Y, void* workspace, size_t ws_bytes, catq_stream stream) {
+  catq_status st = check_layer(layer, sched.phase != CATQ_PHASE_TEACHER);
+  if (st != CATQ_OK) return st;
+  if ((st = check_schedule(sched, sched.phase == CATQ_PHASE_SOFT)) != CATQ_OK) return st;
+  if (x_dtype != layer->w_dtype) return CATQ_ERR_DTYPE;
+  if (ref_dtype != x_dtype && ref_dtype != CATQ_F32) return CATQ_ERR_DTYPE;
+  if (reduction != CATQ_REDUCE_MEAN && reduction != CATQ_REDUCE_SUM) return CATQ_ERR_INVALID_ARG;
+  if (M < 1) return CATQ_ERR_SHAPE;
+  if (!X || !Y_ref || !loss_out || !dY) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(X) || !aligned16(Y_ref) || !aligned16(dY) || (Y && !aligned16(Y)) ||
+      (reinterpret_cast<uintptr_t>(x_row_scale) & 3u))
+    return CATQ_ERR_ALIGN;
+  if (!workspace || ws_bytes < catq_fwd_loss_workspace_bytes(layer, M)) return CATQ_ERR_WORKSPACE;
+  if (!aligned256(workspace)) return CATQ_ERR_ALIGN;
+  if ((st = check_op_const(layer, sched)) != CATQ_OK) return st;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const LayerDev L = to_dev(layer);
+  const int64_t count = M * layer->N;
+  const double inv = reduction == CATQ_REDUCE_MEAN ? 1.0 / static_cast<double>(count) : 1.0;
+  double* part = static_cast<double*>(workspace);
+  if (layer->w_dtype == CATQ_F32) {
+    // fp32 layers: the CUDA-core forward (into Y, or into dY as scratch), then the loss kernel
+    // in place (each element of dY is read before it is written by the same thread)
+    float* Yw = static_cast<float*>(Y ? Y : dY);
+    if (launch_simt_fwd(L, scalars(sched), static_cast<const float*>(X), M, Yw, s, x_row_scale) != cudaSuccess)
+      return CATQ_ERR_CUDA;
+    return cuda_status(launch_recon_loss(Yw, Y_ref, count, CATQ_F32, reduction, loss_out, dY, part, s));
+  }
+  if ((st = check_tensor_core_device()) != CATQ_OK) return st;
+  EpiOpts o;
+  o.row_scale = x_row_scale;
+  o.yref = Y_ref;
+  o.yref_f32 = ref_dtype == CATQ_F32;
+  o.dscale = static_cast<float>(2.0 * inv);
+  o.dY = dY;
+  o.loss_part = part;
+  int nparts = 0;
+  o.n_parts = &nparts;
+  if (launch_tc_fwd(L, scalars(sched), X, M, Y, s, &o) != cudaSuccess) return CATQ_ERR_CUDA;
+  return cuda_status(launch_loss_final(part, nparts, inv, loss_out, s));
+}
+
+catq_status catq_act_quant_a8(const void* X, int64_t M, int64_t K, int32_t x_dtype, void* codes, float* scale,
+                              void* X_deq, catq_stream stream) {
+  if (x_dtype != CATQ_F32 && x_dtype != CATQ_BF16) return CATQ_ERR_DTYPE;
+  if (M < 0 || K < 1) return CATQ_ERR_SHAPE;
+  if (K % (x_dtype == CATQ_BF16 ? 8 : 4) != 0) return CATQ_ERR_SHAPE;  // 16-byte rows
+  if (M == 0) return CATQ_OK;
+  if (!X || !codes || !scale) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(X) || !aligned16(codes) || (X_deq && !aligned16(X_deq)) ||
+      (reinterpret_cast<uintptr_t>(scale) & 3u))
+    return CATQ_ERR_ALIGN;
+  return cuda_status(
+      launch_act_quant_a8(X, M, K, x_dtype, codes, scale, X_deq, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 size_t catq_bwd_workspace_bytes(const catq_layer* layer, int64_t M) {
@@ -364,7 +462,8 @@ size_t grouped_partials_bytes(const catq_grouped_layer* G) {
 // tiles in one persistent sweep.  *used is false when the layer does not qualify (fp32,
 // more experts than one launch takes, 2^31 rows or more), and the caller loops instead.
 catq_status grouped_tc(const catq_grouped_layer* G, catq_schedule sched, const void* A, const int64_t* off,
-                       int32_t x_dtype, void* C, bool dx, catq_stream stream, bool* used) {
+                       int32_t x_dtype, void* C, bool dx, catq_stream stream, bool* used,
+                       const EpiOpts* opts = nullptr) {
   *used = false;
   if (G->w_dtype != CATQ_BF16 || x_dtype != CATQ_BF16 || G->E > kGroupedMaxExperts) return CATQ_OK;
   const int64_t R = off[G->E];
@@ -379,13 +478,13 @@ catq_status grouped_tc(const catq_grouped_layer* G, catq_schedule sched, const v
   if (const_stride % 4 != 0) return CATQ_OK;
   *used = true;
   if (R == 0) return CATQ_OK;
-  if (!A || !C) return CATQ_ERR_INVALID_ARG;
-  if (!aligned16(A) || !aligned16(C)) return CATQ_ERR_ALIGN;
+  if (!A || (!C && !opts)) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(A) || (C && !aligned16(C))) return CATQ_ERR_ALIGN;
   if ((st = check_tensor_core_device()) != CATQ_OK) return st;
   const GroupSpec grp{G->E, off, const_stride};
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   return cuda_status(dx ? launch_tc_dx_grouped(to_dev(&L), scalars(sched), A, grp, C, s)
-                        : launch_tc_fwd_grouped(to_dev(&L), scalars(sched), A, grp, C, s));
+                        : launch_tc_fwd_grouped(to_dev(&L), scalars(sched), A, grp, C, s, opts));
 }
 
 catq_status catq_grouped_soft_ternary_linear_fwd(const catq_grouped_layer* G, catq_schedule sched, const void* X,
@@ -403,6 +502,46 @@ catq_status catq_grouped_soft_ternary_linear_fwd(const catq_grouped_layer* G, ca
     if (st != CATQ_OK) return st;
   }
   return CATQ_OK;
+}
+
+size_t catq_grouped_fwd_loss_workspace_bytes(const catq_grouped_layer* G, const int64_t* off) {
+  if (check_grouped(G, off) != CATQ_OK || G->N < 1) return 0;
+  return fwd_loss_ws_bytes(std::max<int64_t>(1, off[G->E] * G->N));
+}
+
+catq_status catq_grouped_soft_ternary_linear_fwd_loss(const catq_grouped_layer* G, catq_schedule sched,
+                                                      const void* X, const int64_t* off, int32_t x_dtype,
+                                                      const void* Y_ref, int32_t reduction, float* loss_out,
+                                                      void* dY, void* Y, void* workspace, size_t ws_bytes,
+                                                      catq_stream stream) {
+  catq_status st = check_grouped(G, off);
+  if (st != CATQ_OK) return st;
+  if (x_dtype != G->w_dtype) return CATQ_ERR_DTYPE;
+  if (reduction != CATQ_REDUCE_MEAN && reduction != CATQ_REDUCE_SUM) return CATQ_ERR_INVALID_ARG;
+  const int64_t R = off[G->E];
+  if (R < 1 || G->N < 1) return CATQ_ERR_SHAPE;
+  if (!X || !Y_ref || !loss_out || !dY) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(X) || !aligned16(Y_ref) || !aligned16(dY) || (Y && !aligned16(Y))) return CATQ_ERR_ALIGN;
+  if (!workspace || ws_bytes < catq_grouped_fwd_loss_workspace_bytes(G, off)) return CATQ_ERR_WORKSPACE;
+  if (!aligned256(workspace)) return CATQ_ERR_ALIGN;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int64_t count = R * G->N;
+  const double inv = reduction == CATQ_REDUCE_MEAN ? 1.0 / static_cast<double>(count) : 1.0;
+  double* part = static_cast<double*>(workspace);
+  EpiOpts o;
+  o.yref = Y_ref;
+  o.dscale = static_cast<float>(2.0 * inv);
+  o.dY = dY;
+  o.loss_part = part;
+  int nparts = 0;
+  o.n_parts = &nparts;
+  bool used = false;
+  if ((st = grouped_tc(G, sched, X, off, x_dtype, Y, false, stream, &used, &o)) != CATQ_OK) return st;
+  if (used) return cuda_status(launch_loss_final(part, nparts, inv, loss_out, s));
+  // expert by expert into Y (or into dY as scratch), then the loss over every routed row
+  void* Yw = Y ? Y : dY;
+  if ((st = catq_grouped_soft_ternary_linear_fwd(G, sched, X, off, x_dtype, Yw, stream)) != CATQ_OK) return st;
+  return cuda_status(launch_recon_loss(Yw, Y_ref, count, x_dtype, reduction, loss_out, dY, part, s));
 }
 
 size_t catq_grouped_bwd_workspace_bytes(const catq_grouped_layer* G, const int64_t* off) {

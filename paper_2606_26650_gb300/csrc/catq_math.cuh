@@ -75,6 +75,42 @@ __device__ __forceinline__ float hard_q(float x, float delta) {
   return x > delta ? 1.0f : (x < -delta ? -1.0f : 0.0f);
 }
 
+// ---------------------------------------------------------------- compensated fp32 sums
+// (used by the statistics, the loss and the fused forward + loss epilogue)
+// fp64 arithmetic is slow on this GPU, so sums use an fp32 value plus an fp32 error term
+// (Knuth's two-sum), which carries about twice fp32's precision.
+struct Sum2 {
+  float hi, lo;
+};
+
+__device__ __forceinline__ void sum2_add(Sum2& a, float x) {
+  const float s = a.hi + x;
+  const float bp = s - a.hi;
+  const float err = (a.hi - (s - bp)) + (x - bp);
+  a.hi = s;
+  a.lo += err;
+}
+
+__device__ __forceinline__ Sum2 sum2_merge(Sum2 a, Sum2 b) {
+  const float s = a.hi + b.hi;
+  const float bp = s - a.hi;
+  const float err = (a.hi - (s - bp)) + (b.hi - bp);
+  return Sum2{s, a.lo + b.lo + err};
+}
+
+// Butterfly reduction over aligned teams of `team` lanes (team a power of two <= 32).
+__device__ __forceinline__ Sum2 sum2_team(Sum2 v, int team) {
+  for (int o = team >> 1; o > 0; o >>= 1) {
+    Sum2 w;
+    w.hi = __shfl_xor_sync(0xffffffffu, v.hi, o);
+    w.lo = __shfl_xor_sync(0xffffffffu, v.lo, o);
+    v = sum2_merge(v, w);
+  }
+  return v;
+}
+
+__device__ __forceinline__ double sum2_value(Sum2 v) { return static_cast<double>(v.hi) + static_cast<double>(v.lo); }
+
 // ---------------------------------------------------------------- bf16 helpers
 
 __device__ __forceinline__ float bf16lo_to_f32(uint32_t w2) { return __uint_as_float(w2 << 16); }

@@ -43,41 +43,6 @@ struct Vec16<__nv_bfloat16> {
   }
 };
 
-// ---------------------------------------------------------------- compensated fp32 sums
-// fp64 arithmetic is slow on this GPU, so sums use an fp32 value plus an fp32 error term
-// (Knuth's two-sum), which carries about twice fp32's precision.
-struct Sum2 {
-  float hi, lo;
-};
-
-__device__ __forceinline__ void sum2_add(Sum2& a, float x) {
-  const float s = a.hi + x;
-  const float bp = s - a.hi;
-  const float err = (a.hi - (s - bp)) + (x - bp);
-  a.hi = s;
-  a.lo += err;
-}
-
-__device__ __forceinline__ Sum2 sum2_merge(Sum2 a, Sum2 b) {
-  const float s = a.hi + b.hi;
-  const float bp = s - a.hi;
-  const float err = (a.hi - (s - bp)) + (b.hi - bp);
-  return Sum2{s, a.lo + b.lo + err};
-}
-
-// Butterfly reduction over aligned teams of `team` lanes (team a power of two <= 32).
-__device__ __forceinline__ Sum2 sum2_team(Sum2 v, int team) {
-  for (int o = team >> 1; o > 0; o >>= 1) {
-    Sum2 w;
-    w.hi = __shfl_xor_sync(0xffffffffu, v.hi, o);
-    w.lo = __shfl_xor_sync(0xffffffffu, v.lo, o);
-    v = sum2_merge(v, w);
-  }
-  return v;
-}
-
-__device__ __forceinline__ double sum2_value(Sum2 v) { return static_cast<double>(v.hi) + static_cast<double>(v.lo); }
-
 // Rounded once to fp32 (all a stored fp32 statistic needs; avoids fp64 arithmetic).
 __device__ __forceinline__ float sum2_float(Sum2 v) { return v.hi + v.lo; }
 
@@ -598,6 +563,63 @@ __global__ void __launch_bounds__(kThreads) recon_loss_final_kernel(const double
   }
 }
 
+// ---------------------------------------------------------------- 8-bit activations
+// Per-token symmetric absmax quantization of one row per warp (the W1.58A8 setting): the
+// warp's max |x| gives scale = max / 127 (IEEE division); each element's code is
+// rint(x / scale) (IEEE division, ties to even), clamped to [-127, 127]; a zero row has
+// scale 0 and codes 0.  Codes are written as exact values of the input dtype (|q| <= 127
+// is exact in bf16), and `deq` (nullable) gets scale * q rounded once to that dtype.
+template <typename T>
+__device__ __forceinline__ void store_vec(T* p, const float (&v)[Vec16<T>::n]);
+template <>
+__device__ __forceinline__ void store_vec<float>(float* p, const float (&v)[4]) {
+  *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+}
+template <>
+__device__ __forceinline__ void store_vec<__nv_bfloat16>(__nv_bfloat16* p, const float (&v)[8]) {
+  uint4 q;
+  q.x = pack_bf16x2(v[0], v[1]);
+  q.y = pack_bf16x2(v[2], v[3]);
+  q.z = pack_bf16x2(v[4], v[5]);
+  q.w = pack_bf16x2(v[6], v[7]);
+  *reinterpret_cast<uint4*>(p) = q;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads) act_quant_a8_kernel(const T* __restrict__ X, int64_t M, int64_t K,
+                                                                 T* __restrict__ codes, float* __restrict__ scale,
+                                                                 T* __restrict__ deq) {
+  constexpr int V = Vec16<T>::n;
+  const int lane = threadIdx.x & 31;
+  const int64_t nvec = K / V;  // K is a multiple of V (16-byte rows)
+  for (int64_t m = (blockIdx.x * (int64_t)kThreads + threadIdx.x) >> 5; m < M;
+       m += ((int64_t)gridDim.x * kThreads) >> 5) {
+    const T* row = X + m * K;
+    float amax = 0.0f;
+    for (int64_t v = lane; v < nvec; v += 32) {
+      float x[V];
+      Vec16<T>::load(row + v * V, x);
+#pragma unroll
+      for (int q = 0; q < V; ++q) amax = fmaxf(amax, fabsf(x[q]));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+    const float s = __fdiv_rn(amax, 127.0f);
+    if (lane == 0) scale[m] = s;
+    for (int64_t v = lane; v < nvec; v += 32) {
+      float x[V], q[V], d[V];
+      Vec16<T>::load(row + v * V, x);
+#pragma unroll
+      for (int i = 0; i < V; ++i) {
+        q[i] = s > 0.0f ? fminf(fmaxf(rintf(__fdiv_rn(x[i], s)), -127.0f), 127.0f) : 0.0f;
+        d[i] = q[i] * s;
+      }
+      store_vec<T>(codes + m * K + v * V, q);
+      if (deq) store_vec<T>(deq + m * K + v * V, d);
+    }
+  }
+}
+
 // ---------------------------------------------------------------- factor-gradient reduction
 // One thread per group: sums the dW epilogue's partial sums over contraction splits and
 // over the g/P column chunks of the group in a fixed order, then applies
@@ -795,6 +817,25 @@ cudaError_t launch_recon_loss(const void* Y, const void* Yr, int64_t count, int3
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   recon_loss_final_kernel<<<1, kThreads, 0, st>>>(partials, nb, inv, loss_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_loss_final(const double* partials, int n, double out_scale, float* loss, cudaStream_t st) {
+  recon_loss_final_kernel<<<1, kThreads, 0, st>>>(partials, n, out_scale, loss);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_act_quant_a8(const void* X, int64_t M, int64_t K, int32_t dtype, void* codes, float* scale,
+                                void* deq, cudaStream_t st) {
+  const int grid = grid_for((M + kThreads / 32 - 1) / (kThreads / 32), 1);
+  if (dtype == 1)
+    act_quant_a8_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(static_cast<const __nv_bfloat16*>(X), M, K,
+                                                                   static_cast<__nv_bfloat16*>(codes), scale,
+                                                                   static_cast<__nv_bfloat16*>(deq));
+  else
+    act_quant_a8_kernel<float><<<grid, kThreads, 0, st>>>(static_cast<const float*>(X), M, K,
+                                                           static_cast<float*>(codes), scale,
+                                                           static_cast<float*>(deq));
   return cudaGetLastError();
 }
 

@@ -22,17 +22,26 @@ cudaError_t launch_group_stats(const LayerDev& L, int32_t w_dtype, int32_t thr_i
 cudaError_t launch_modulate_ternarize(const LayerDev& L, int32_t w_dtype, StepScalars sc, void* Wq, int8_t* T,
                                       float* alpha, cudaStream_t st);
 int recon_loss_blocks(int64_t count);
+// loss[0] = out_scale * (sum of n fp64 partials), in a fixed order.
+cudaError_t launch_loss_final(const double* partials, int n, double out_scale, float* loss, cudaStream_t st);
 cudaError_t launch_recon_loss(const void* Y, const void* Yr, int64_t count, int32_t dtype, int32_t reduction,
                               float* loss_out, void* dY, double* partials, cudaStream_t st);
 cudaError_t launch_hard_pack(const LayerDev& L, int32_t w_dtype, uint8_t* codes, float* alpha, float* mu,
                              cudaStream_t st);
+// Per-token symmetric 8-bit quantization of X [M, K] (dtype 1 bf16, 0 fp32): scale[m] =
+// max|X[m, :]| / 127, codes q = rint(X / scale) in [-127, 127] written as exact values of
+// the same dtype, and (nullable) the dequantized scale q rounded once to that dtype.
+cudaError_t launch_act_quant_a8(const void* X, int64_t M, int64_t K, int32_t dtype, void* codes, float* scale,
+                                void* deq, cudaStream_t st);
 // Sums the partial group sums of the dW epilogue ([splits][3][N][K/P]) into the factor
 // gradients and applies the per-group scales.
 cudaError_t launch_grad_reduce(const LayerDev& L, StepScalars sc, const float* partials, int32_t splits, int32_t P,
                                float* g_dmu, float* g_dalpha, float* g_ddelta, cudaStream_t st);
 
 // simt_f32.cu (fp32 CUDA-core path)
-cudaError_t launch_simt_fwd(const LayerDev& L, StepScalars sc, const float* X, int64_t M, float* Y, cudaStream_t st);
+// row_scale (nullable): Y row m is multiplied by row_scale[m].
+cudaError_t launch_simt_fwd(const LayerDev& L, StepScalars sc, const float* X, int64_t M, float* Y, cudaStream_t st,
+                            const float* row_scale = nullptr);
 cudaError_t launch_simt_dx(const LayerDev& L, StepScalars sc, const float* dY, int64_t M, float* dX, cudaStream_t st);
 cudaError_t launch_simt_dw(const LayerDev& L, StepScalars sc, const float* X, const float* dY, int64_t M,
                            float* partials, cudaStream_t st);
@@ -45,6 +54,17 @@ struct TcPlan {
   int32_t dw_P;       // partial-sum chunk width (columns)
 };
 TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count);
+// Epilogue options of the bf16 forward (defaults: Y stored in bf16).
+struct EpiOpts {
+  bool y_f32 = false;               // store Y in fp32
+  const float* row_scale = nullptr; // [M] per-row scale of the accumulator (8-bit activation codes)
+  const void* yref = nullptr;       // fused Eq. 7 loss against this teacher output [M, N]
+  bool yref_f32 = false;
+  float dscale = 0.0f;              // dY = dscale (Y - Y_ref)
+  void* dY = nullptr;               // bf16 [M, N]
+  double* loss_part = nullptr;      // partial sums of (Y - Y_ref)^2
+  int* n_parts = nullptr;           // out: partials written
+};
 // Y [B, N] = X [B, K] (alpha T + mu)^T from 2-bit codes, group scales and (nullable) group
 // offsets (bf16 X and Y).
 cudaError_t launch_ternary_infer(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K,
@@ -91,7 +111,7 @@ struct GroupSpec {
 cudaError_t launch_operand_consts_grouped(const LayerDev& L0, StepScalars sc, int32_t E, int64_t const_stride,
                                           cudaStream_t st);
 cudaError_t launch_tc_fwd_grouped(const LayerDev& L0, StepScalars sc, const void* X, const GroupSpec& grp, void* Y,
-                                  cudaStream_t st);
+                                  cudaStream_t st, const EpiOpts* opts = nullptr);
 cudaError_t launch_tc_dx_grouped(const LayerDev& L0, StepScalars sc, const void* dY, const GroupSpec& grp, void* dX,
                                  cudaStream_t st);
 // Partial group sums of every expert with rows, [E][3][N][K/P] (P = gcd(g, 128)).
@@ -102,7 +122,10 @@ cudaError_t launch_grad_reduce_grouped(const LayerDev& L0, StepScalars sc, const
                                        const GroupSpec& grp, float* g_dmu, float* g_dalpha, float* g_ddelta,
                                        cudaStream_t st);
 
-cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st);
+// Upper bound of EpiOpts::n_parts for any launch on a device with `sm_count` SMs.
+int fused_loss_max_parts(int sm_count);
+cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st,
+                         const EpiOpts* opts = nullptr);
 cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int64_t M, void* dX, cudaStream_t st);
 cudaError_t launch_tc_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M,
                          const TcPlan& plan, float* partials, cudaStream_t st);

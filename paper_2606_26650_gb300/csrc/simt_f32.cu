@@ -23,6 +23,7 @@ struct SimtArgs {
   float* C;        // FWD: Y [M,N]; DX: dX [M,K]; DW: partials [3][N][K/P]
   int64_t M;
   int32_t P;       // DW partial chunk width
+  const float* row_scale;  // FWD, nullable: Y row m times row_scale[m]
 };
 
 __device__ __forceinline__ float w_elem(const SimtArgs& a, int64_t n, int64_t k) {
@@ -108,7 +109,7 @@ __global__ void __launch_bounds__(kThr) simt_gemm_kernel(SimtArgs a) {
 #pragma unroll
       for (int v = 0; v < 4; ++v) {
         const int64_t i = i0 + ty + 16 * u, j = j0 + tx + 16 * v;
-        if (i < rowsI && j < colsJ) a.C[i * ldc + j] = acc[u][v];
+        if (i < rowsI && j < colsJ) a.C[i * ldc + j] = a.row_scale ? acc[u][v] * a.row_scale[i] : acc[u][v];
       }
     return;
   }
@@ -178,14 +179,15 @@ static dim3 grid2(int64_t rows, int64_t cols) {
   return dim3(static_cast<unsigned>((cols + TN - 1) / TN), static_cast<unsigned>((rows + TM - 1) / TM));
 }
 
-cudaError_t launch_simt_fwd(const LayerDev& L, StepScalars sc, const float* X, int64_t M, float* Y, cudaStream_t st) {
-  SimtArgs a{L, sc, X, nullptr, Y, M, 0};
+cudaError_t launch_simt_fwd(const LayerDev& L, StepScalars sc, const float* X, int64_t M, float* Y, cudaStream_t st,
+                            const float* row_scale) {
+  SimtArgs a{L, sc, X, nullptr, Y, M, 0, row_scale};
   simt_gemm_kernel<MODE_FWD><<<grid2(M, L.N), kThr, 0, st>>>(a);
   return cudaGetLastError();
 }
 
 cudaError_t launch_simt_dx(const LayerDev& L, StepScalars sc, const float* dY, int64_t M, float* dX, cudaStream_t st) {
-  SimtArgs a{L, sc, dY, nullptr, dX, M, 0};
+  SimtArgs a{L, sc, dY, nullptr, dX, M, 0, nullptr};
   simt_gemm_kernel<MODE_DX><<<grid2(M, L.K), kThr, 0, st>>>(a);
   return cudaGetLastError();
 }
@@ -193,7 +195,7 @@ cudaError_t launch_simt_dx(const LayerDev& L, StepScalars sc, const float* dY, i
 cudaError_t launch_simt_dw(const LayerDev& L, StepScalars sc, const float* X, const float* dY, int64_t M,
                            float* partials, cudaStream_t st) {
   const int32_t P = L.g < TN ? L.g : TN;
-  SimtArgs a{L, sc, dY, X, partials, M, P};
+  SimtArgs a{L, sc, dY, X, partials, M, P, nullptr};
   simt_gemm_kernel<MODE_DW><<<grid2(L.N, L.K), kThr, 0, st>>>(a);
   return cudaGetLastError();
 }

@@ -112,7 +112,19 @@ constexpr int kMaxGroupExperts = kGroupedMaxExperts;
 struct FusedArgs {
   LayerDev L;
   StepScalars sc;
-  uint16_t* C;      // bf16 [M, ncols]
+  void* C;          // [M, ncols], bf16 (fp32 when c_f32); nullable in the fused-loss epilogue
+  int32_t c_f32;
+  // Per-row scale of the accumulator (nullable): C row m = row_scale[m] * (A Wq^T)[m], the
+  // per-token scale of 8-bit activation codes in A.
+  const float* row_scale;
+  // Fused reconstruction loss (Eq. 7) when yref is set: the epilogue forms d = Y - Y_ref from
+  // the fp32 accumulator, writes dY = dscale d (bf16) and sums d^2 into one partial per
+  // epilogue warp, loss_part[blockIdx.x * kEpiWarps + warp].
+  const void* yref;  // [M, ncols] bf16, or fp32 when yref_f32
+  int32_t yref_f32;
+  float dscale;
+  uint16_t* dY;      // bf16 [M, ncols]
+  double* loss_part;
   int64_t M;        // rows of A and C
   int64_t ncols;    // columns of C
   int32_t num_m_tiles, num_n_tiles, num_k_blocks;
@@ -239,6 +251,81 @@ __device__ __forceinline__ void store_rows_bf16x32(uint16_t* C, int64_t M, int64
   }
 }
 
+// 16 bf16 values of one row per lane (32 rows per warp, columns from `col`, as two 16-byte
+// vectors) stored through a 2 x 2 transpose of the vectors between lane pairs (one
+// xor-shuffle round), so that two lanes store 32 contiguous bytes of one row.
+__device__ __forceinline__ void store_rows_packed16(uint16_t* C, int64_t M, int64_t ncols, int64_t row0, int64_t col,
+                                                    uint4 (&v)[2], int lane) {
+  // lane 2a + i ends with chunk i of rows 2a, 2a + 1 in v[0], v[1]
+  const bool upper = (lane & 1) != 0;
+  const uint4 send = upper ? v[0] : v[1];
+  uint4 got;
+  got.x = __shfl_xor_sync(0xffffffffu, send.x, 1);
+  got.y = __shfl_xor_sync(0xffffffffu, send.y, 1);
+  got.z = __shfl_xor_sync(0xffffffffu, send.z, 1);
+  got.w = __shfl_xor_sync(0xffffffffu, send.w, 1);
+  if (upper) v[0] = got;
+  else v[1] = got;
+  const int64_t c = col + 8 * (lane & 1);
+  if (c >= ncols) return;
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    const int64_t row = row0 + (lane & ~1) + j;
+    if (row < M) *reinterpret_cast<uint4*>(C + row * ncols + c) = v[j];
+  }
+}
+
+// 16 fp32 accumulator columns of one row per lane stored as bf16 (store_rows_packed16).
+__device__ __forceinline__ void store_rows_bf16x16(uint16_t* C, int64_t M, int64_t ncols, int64_t row0, int64_t col,
+                                                   const uint32_t (&r)[16], int lane) {
+  uint4 v[2];
+#pragma unroll
+  for (int p = 0; p < 2; ++p) {
+    v[p].x = pack_bf16x2(__uint_as_float(r[8 * p + 0]), __uint_as_float(r[8 * p + 1]));
+    v[p].y = pack_bf16x2(__uint_as_float(r[8 * p + 2]), __uint_as_float(r[8 * p + 3]));
+    v[p].z = pack_bf16x2(__uint_as_float(r[8 * p + 4]), __uint_as_float(r[8 * p + 5]));
+    v[p].w = pack_bf16x2(__uint_as_float(r[8 * p + 6]), __uint_as_float(r[8 * p + 7]));
+  }
+  store_rows_packed16(C, M, ncols, row0, col, v, lane);
+}
+
+// 32 fp32 values of one row per lane (row < M, columns from `col`) stored as fp32: eight
+// 16-byte stores per lane (used for a full-precision teacher output, off the hot path).
+__device__ __forceinline__ void store_row_f32x32(float* C, int64_t M, int64_t ncols, int64_t row, int64_t col,
+                                                 const uint32_t (&r)[32]) {
+  if (row >= M) return;
+#pragma unroll
+  for (int p = 0; p < 8; ++p)
+    if (col + 4 * p < ncols)
+      *reinterpret_cast<float4*>(C + row * ncols + col + 4 * p) =
+          make_float4(__uint_as_float(r[4 * p]), __uint_as_float(r[4 * p + 1]), __uint_as_float(r[4 * p + 2]),
+                      __uint_as_float(r[4 * p + 3]));
+}
+
+// 16 fp32 values of one row per lane (row < M, columns from `col`) stored as fp32: four
+// 16-byte stores per lane (used for a full-precision teacher output, off the hot path).
+__device__ __forceinline__ void store_row_f32x16(float* C, int64_t M, int64_t ncols, int64_t row, int64_t col,
+                                                 const uint32_t (&r)[16]) {
+  if (row >= M) return;
+#pragma unroll
+  for (int p = 0; p < 4; ++p)
+    if (col + 4 * p < ncols)
+      *reinterpret_cast<float4*>(C + row * ncols + col + 4 * p) =
+          make_float4(__uint_as_float(r[4 * p]), __uint_as_float(r[4 * p + 1]), __uint_as_float(r[4 * p + 2]),
+                      __uint_as_float(r[4 * p + 3]));
+}
+
+// The teacher output of one row's 16 columns from `col` (bf16), as two 16-byte vectors;
+// chunks outside the row's columns, and rows past the end, read as 0.
+__device__ __forceinline__ void load_yref_bf16x16(const uint16_t* Yr, int64_t ncols, int64_t row, bool row_ok,
+                                                  int64_t col, uint4 (&v)[2]) {
+#pragma unroll
+  for (int p = 0; p < 2; ++p) {
+    v[p] = make_uint4(0u, 0u, 0u, 0u);
+    if (row_ok && col + 8 * p < ncols) v[p] = __ldg(reinterpret_cast<const uint4*>(Yr + row * ncols + col + 8 * p));
+  }
+}
+
 // ============================================================================ fused kernel
 
 // Walks the pipeline stages one producer thread handles (every kProdGroups-th stage of its
@@ -314,8 +401,10 @@ struct OperandRowIter {
 };
 
 // MU: the layer reconstructs W ~ alpha T + mu (a separate instantiation, so the W ~ alpha T
-// kernel carries none of its work).
-template <int CG, bool B_MN, int PAIRS, bool MU>
+// kernel carries none of its work).  EPI: 0 stores C in bf16; 1 is the general epilogue
+// (row scale, fp32 C, fused loss), a separate instantiation so the plain forward and dX
+// keep their register allocation.
+template <int CG, bool B_MN, int PAIRS, bool MU, int EPI = 0>
 __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     fused_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
                       const FusedArgs args) {
@@ -555,31 +644,126 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
     }
   } else if (warp < Cfg::kEpiWarps) {
     // ------------------------------------------------------------ epilogue
+    // Lane l of warp qd owns accumulator row qd * 32 + l.
+    //   EPI 0:  Y in bf16, transposed through lane quads for contiguous stores.
+    //   EPI 1:  16 columns per TMEM load: the accumulator times the row's scale (when given),
+    //           stored as bf16 or fp32 when C is given, and, with a teacher output, the fused
+    //           loss: d = Y - Y_ref from the unrounded accumulator, dY = dscale d in bf16 and a
+    //           compensated sum of d^2 over every element the warp owns.  The teacher rows
+    //           of both accumulators are sent to L2 when the tile begins, and each lane keeps
+    //           two 16-column chunks of its row in flight ahead of the arithmetic.
     const int qd = warp;  // TMEM lane quarter
+    const bool fused_loss = EPI == 1 && args.yref != nullptr;
+    const uint16_t* yref16 = static_cast<const uint16_t*>(args.yref);
+    const float* yref32 = static_cast<const float*>(args.yref);
+    Sum2 lacc{0.f, 0.f};
     uint32_t it = 0;
     bool ok = true;
     for (int t = cluster; ok && t < num_tiles; t += nclusters, ++it) {
       const TileInfo ti = tile_info(args, t, Cfg::kTileRows * PAIRS);
+      const int64_t col0 = (int64_t)ti.n_blk * BN;
+      if (fused_loss) {
+        const int64_t ncols_here = args.ncols - col0 < BN ? args.ncols - col0 : (int64_t)BN;
+        const int64_t esz = args.yref_f32 ? 4 : 2;
+#pragma unroll
+        for (int acc = 0; acc < NACC; ++acc) {
+          const int64_t row = ti.row0 + pair * Cfg::kTileRows + acc * Cfg::kRowsPerAcc + cta * 128 + qd * 32 + lane;
+          if (row < ti.row_end && ncols_here > 0)
+            prefetch_l2_bulk(static_cast<const char*>(args.yref) + (row * args.ncols + col0) * esz,
+                             static_cast<uint32_t>(ncols_here * esz));
+        }
+      }
 #pragma unroll 1
       for (int acc = 0; acc < NACC; ++acc) {
-        if (!mbar_wait(tmem_full0 + 8u * acc, it & 1u, wc)) { ok = false; break; }
-        tc_fence_after();
         const int64_t row0 = ti.row0 + pair * Cfg::kTileRows + acc * Cfg::kRowsPerAcc + cta * 128 +
                              qd * 32;  // this warp's first row
+        if constexpr (EPI == 0) {
+          if (!mbar_wait(tmem_full0 + 8u * acc, it & 1u, wc)) { ok = false; break; }
+          tc_fence_after();
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
-          const int64_t col = (int64_t)ti.n_blk * BN + c * 32;
-          if (col >= args.ncols || row0 >= ti.row_end) break;  // warp-uniform
-          uint32_t r[32];
-          tmem_ld32(tmem_base + (static_cast<uint32_t>(qd * 32) << 16) + acc * BN + c * 32, r);
-          tmem_ld_wait();
-          store_rows_bf16x32(args.C, ti.row_end, args.ncols, row0, col, r, lane);
+          for (int c = 0; c < BN / 32; ++c) {
+            const int64_t col = col0 + c * 32;
+            if (col >= args.ncols || row0 >= ti.row_end) break;  // warp-uniform
+            uint32_t r[32];
+            tmem_ld32(tmem_base + (static_cast<uint32_t>(qd * 32) << 16) + acc * BN + c * 32, r);
+            tmem_ld_wait();
+            store_rows_bf16x32(static_cast<uint16_t*>(args.C), ti.row_end, args.ncols, row0, col, r, lane);
+          }
+        } else {
+          const int64_t row = row0 + lane;
+          const bool row_ok = row < ti.row_end;
+          const float rs = args.row_scale ? (row_ok ? __ldg(args.row_scale + row) : 0.0f) : 1.0f;
+          const bool ref16 = fused_loss && !args.yref_f32;
+          uint4 y0[2], y1[2];
+          if (ref16) {
+            load_yref_bf16x16(yref16, args.ncols, row, row_ok, col0, y0);
+            load_yref_bf16x16(yref16, args.ncols, row, row_ok, col0 + 16, y1);
+          }
+          if (!mbar_wait(tmem_full0 + 8u * acc, it & 1u, wc)) { ok = false; break; }
+          tc_fence_after();
+#pragma unroll 1
+          for (int c = 0; c < BN / 16; ++c) {
+            const int64_t col = col0 + c * 16;
+            if (col >= args.ncols || row0 >= ti.row_end) break;  // warp-uniform
+            uint32_t r[16];
+            tmem_ld16(tmem_base + (static_cast<uint32_t>(qd * 32) << 16) + acc * BN + c * 16, r);
+            uint4 y2[2];
+            if (ref16) load_yref_bf16x16(yref16, args.ncols, row, row_ok, col + 32, y2);
+            tmem_ld_wait();
+            if (args.row_scale) {
+#pragma unroll
+              for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * rs);
+            }
+            if (args.C) {
+              if (args.c_f32) store_row_f32x16(static_cast<float*>(args.C), ti.row_end, args.ncols, row, col, r);
+              else store_rows_bf16x16(static_cast<uint16_t*>(args.C), ti.row_end, args.ncols, row0, col, r, lane);
+            }
+            if (fused_loss) {
+              uint4 pk[2];        // dY, packed as it is formed
+              float csum = 0.0f;  // this chunk's sum of d^2 (16 terms), then one compensated add
+#pragma unroll
+              for (int q = 0; q < 2; ++q) {  // 8 columns at a time
+                const bool live = row_ok && col + 8 * q < args.ncols;  // ncols is a multiple of 8
+                float4 ra = make_float4(0.f, 0.f, 0.f, 0.f), rb = ra;  // fp32 teacher
+                if (!ref16 && live) {
+                  const float4* qv = reinterpret_cast<const float4*>(yref32 + row * args.ncols + col + 8 * q);
+                  ra = __ldg(qv);
+                  rb = __ldg(qv + 1);
+                }
+                uint32_t* out = reinterpret_cast<uint32_t*>(&pk[q]);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {  // columns 2e, 2e + 1 of the eight
+                  const uint32_t w = ref16 ? (e == 0 ? y0[q].x : e == 1 ? y0[q].y : e == 2 ? y0[q].z : y0[q].w) : 0u;
+                  const float4 rr = (e >> 1) ? rb : ra;
+                  const float t0 = ref16 ? bf16lo_to_f32(w) : ((e & 1) ? rr.z : rr.x);
+                  const float t1 = ref16 ? bf16hi_to_f32(w) : ((e & 1) ? rr.w : rr.y);
+                  const float d0 = live ? __uint_as_float(r[8 * q + 2 * e]) - t0 : 0.0f;
+                  const float d1 = live ? __uint_as_float(r[8 * q + 2 * e + 1]) - t1 : 0.0f;
+                  csum = fmaf(d0, d0, csum);
+                  csum = fmaf(d1, d1, csum);
+                  out[e] = pack_bf16x2(d0 * args.dscale, d1 * args.dscale);
+                }
+              }
+              sum2_add(lacc, csum);
+              if (args.dY) store_rows_packed16(args.dY, ti.row_end, args.ncols, row0, col, pk, lane);
+              if (ref16) {
+                y0[0] = y1[0];
+                y0[1] = y1[1];
+                y1[0] = y2[0];
+                y1[1] = y2[1];
+              }
+            }
+          }
         }
         // this accumulator is drained: the MMA may refill it
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_cluster(leader_tmem_empty0 + 8u * acc);
       }
+    }
+    if (fused_loss) {
+      lacc = sum2_team(lacc, 32);
+      if (lane == 0) args.loss_part[blockIdx.x * Cfg::kEpiWarps + qd] = sum2_value(lacc);
     }
   } else {
     // ------------------------------------------------------------ operand producers
@@ -1082,9 +1266,9 @@ int fused_variant_for(int64_t M) { return M >= 1024 ? 4 : (M >= 512 ? 2 : 1); }
 
 // grp (nullable): a grouped launch over grp->E experts whose weights are stacked from L.W on
 // and whose rows of A and C are expert-sorted (host offsets grp->off).
-template <int CG, bool B_MN, int PAIRS, bool MU>
+template <int CG, bool B_MN, int PAIRS, bool MU, int EPI = 0>
 cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t M, int64_t depth, void* C,
-                      int64_t ncols, cudaStream_t st, const GroupSpec* grp = nullptr) {
+                      int64_t ncols, cudaStream_t st, const GroupSpec* grp = nullptr, const EpiOpts* opts = nullptr) {
   using Cfg = FusedCfg<CG, PAIRS>;
   DeviceInfo& d = device_info();
   if (!d.ok) return cudaErrorInvalidDevice;
@@ -1099,7 +1283,15 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
   FusedArgs args;
   args.L = L;
   args.sc = sc;
-  args.C = static_cast<uint16_t*>(C);
+  args.C = C;
+  args.c_f32 = opts && opts->y_f32 ? 1 : 0;
+  args.row_scale = opts ? opts->row_scale : nullptr;
+  args.yref = opts ? opts->yref : nullptr;
+  args.yref_f32 = opts && opts->yref_f32 ? 1 : 0;
+  args.dscale = opts ? opts->dscale : 0.0f;
+  args.dY = opts ? static_cast<uint16_t*>(opts->dY) : nullptr;
+  args.loss_part = opts ? opts->loss_part : nullptr;
+  if (opts && opts->n_parts) *opts->n_parts = 0;
   args.M = M;
   args.ncols = ncols;
   args.num_m_tiles = static_cast<int32_t>((M + Cfg::kTileRows * PAIRS - 1) / (Cfg::kTileRows * PAIRS));
@@ -1125,10 +1317,11 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
     args.num_m_tiles = static_cast<int32_t>(t / args.num_n_tiles);  // the kernel's tile count is M x N blocks
     if (tiles == 0) return cudaSuccess;
   }
-  auto kern = fused_gemm_kernel<CG, B_MN, PAIRS, MU>;
+  auto kern = fused_gemm_kernel<CG, B_MN, PAIRS, MU, EPI>;
   const int fit = max_active_clusters(kern, Cfg::kClusterCtas, Cfg::kThreads, Cfg::kSmemBytes,
                                       d.sm_count / Cfg::kClusterCtas);
   const int clusters = std::min(tiles, fit);
+  if (opts && opts->n_parts) *opts->n_parts = clusters * Cfg::kClusterCtas * Cfg::kEpiWarps;
   void* params[3] = {&ta, &tw, &args};
   return launch_persistent(kern, Cfg::kClusterCtas, clusters * Cfg::kClusterCtas, Cfg::kThreads, Cfg::kSmemBytes,
                            st, params);
@@ -1214,46 +1407,55 @@ cudaError_t run_dw_grouped(const LayerDev& L0, StepScalars sc, const void* X, co
 }
 
 // Tile shape by M, and the W ~ alpha T + mu instantiation for such layers outside TEACHER.
+// Tile shape by rows (M, or a grouped launch's mean rows per expert) and the W ~ alpha T + mu
+// instantiation for such layers outside TEACHER; the general epilogue (EPI 1) for a forward
+// with epilogue options.
+template <bool B_MN, int EPI>
+cudaError_t dispatch_fused_epi(const LayerDev& L, StepScalars sc, const void* A, int64_t M, int64_t tile_rows,
+                               int64_t depth, void* C, int64_t ncols, cudaStream_t st, const GroupSpec* grp,
+                               const EpiOpts* opts) {
+  const bool mu = L.recon != 0 && sc.phase != PHASE_TEACHER;
+  switch (fused_variant_for(tile_rows) * 2 + (mu ? 1 : 0)) {
+    case 8: return run_fused<2, B_MN, 2, false, EPI>(L, sc, A, M, depth, C, ncols, st, grp, opts);
+    case 9: return run_fused<2, B_MN, 2, true, EPI>(L, sc, A, M, depth, C, ncols, st, grp, opts);
+    case 4: return run_fused<2, B_MN, 1, false, EPI>(L, sc, A, M, depth, C, ncols, st, grp, opts);
+    case 5: return run_fused<2, B_MN, 1, true, EPI>(L, sc, A, M, depth, C, ncols, st, grp, opts);
+    case 3: return run_fused<1, B_MN, 1, true, EPI>(L, sc, A, M, depth, C, ncols, st, grp, opts);
+    default: return run_fused<1, B_MN, 1, false, EPI>(L, sc, A, M, depth, C, ncols, st, grp, opts);
+  }
+}
+
 template <bool B_MN>
 cudaError_t dispatch_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t M, int64_t depth, void* C,
-                           int64_t ncols, cudaStream_t st) {
-  const bool mu = L.recon != 0 && sc.phase != PHASE_TEACHER;
-  switch (fused_variant_for(M) * 2 + (mu ? 1 : 0)) {
-    case 8: return run_fused<2, B_MN, 2, false>(L, sc, A, M, depth, C, ncols, st);
-    case 9: return run_fused<2, B_MN, 2, true>(L, sc, A, M, depth, C, ncols, st);
-    case 4: return run_fused<2, B_MN, 1, false>(L, sc, A, M, depth, C, ncols, st);
-    case 5: return run_fused<2, B_MN, 1, true>(L, sc, A, M, depth, C, ncols, st);
-    case 3: return run_fused<1, B_MN, 1, true>(L, sc, A, M, depth, C, ncols, st);
-    default: return run_fused<1, B_MN, 1, false>(L, sc, A, M, depth, C, ncols, st);
-  }
+                           int64_t ncols, cudaStream_t st, const EpiOpts* opts = nullptr) {
+  if constexpr (!B_MN)
+    if (opts) return dispatch_fused_epi<false, 1>(L, sc, A, M, M, depth, C, ncols, st, nullptr, opts);
+  return dispatch_fused_epi<B_MN, 0>(L, sc, A, M, M, depth, C, ncols, st, nullptr, nullptr);
 }
 
 // Grouped: the tile shape by the mean rows per expert.
 template <bool B_MN>
 cudaError_t dispatch_fused_grouped(const LayerDev& L, StepScalars sc, const void* A, int64_t depth, void* C,
-                                   int64_t ncols, const GroupSpec& grp, cudaStream_t st) {
+                                   int64_t ncols, const GroupSpec& grp, cudaStream_t st,
+                                   const EpiOpts* opts = nullptr) {
   const int64_t R = grp.off[grp.E];
-  const bool mu = L.recon != 0 && sc.phase != PHASE_TEACHER;
-  switch (fused_variant_for(R / grp.E) * 2 + (mu ? 1 : 0)) {
-    case 8: return run_fused<2, B_MN, 2, false>(L, sc, A, R, depth, C, ncols, st, &grp);
-    case 9: return run_fused<2, B_MN, 2, true>(L, sc, A, R, depth, C, ncols, st, &grp);
-    case 4: return run_fused<2, B_MN, 1, false>(L, sc, A, R, depth, C, ncols, st, &grp);
-    case 5: return run_fused<2, B_MN, 1, true>(L, sc, A, R, depth, C, ncols, st, &grp);
-    case 3: return run_fused<1, B_MN, 1, true>(L, sc, A, R, depth, C, ncols, st, &grp);
-    default: return run_fused<1, B_MN, 1, false>(L, sc, A, R, depth, C, ncols, st, &grp);
-  }
+  if constexpr (!B_MN)
+    if (opts) return dispatch_fused_epi<false, 1>(L, sc, A, R, R / grp.E, depth, C, ncols, st, &grp, opts);
+  return dispatch_fused_epi<B_MN, 0>(L, sc, A, R, R / grp.E, depth, C, ncols, st, &grp, nullptr);
 }
 
 }  // namespace
 
 cudaError_t launch_tc_fwd_grouped(const LayerDev& L0, StepScalars sc, const void* X, const GroupSpec& grp, void* Y,
-                                  cudaStream_t st) {
+                                  cudaStream_t st, const EpiOpts* opts) {
   if (sc.phase != PHASE_TEACHER) {
     const cudaError_t e = launch_operand_consts_grouped(L0, sc, grp.E, grp.const_stride, st);
     if (e != cudaSuccess) return e;
   }
-  return dispatch_fused_grouped<false>(L0, sc, X, L0.K, Y, L0.N, grp, st);
+  return dispatch_fused_grouped<false>(L0, sc, X, L0.K, Y, L0.N, grp, st, opts);
 }
+
+int fused_loss_max_parts(int sm_count) { return (sm_count > 0 ? sm_count : 1) * FusedCfg<1>::kEpiWarps; }
 
 cudaError_t launch_tc_dx_grouped(const LayerDev& L0, StepScalars sc, const void* dY, const GroupSpec& grp, void* dX,
                                  cudaStream_t st) {
@@ -1288,12 +1490,13 @@ TcPlan tc_plan_bwd(const LayerDev& L, int64_t M, int sm_count) {
   return p;
 }
 
-cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st) {
+cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int64_t M, void* Y, cudaStream_t st,
+                         const EpiOpts* opts) {
   if (sc.phase != PHASE_TEACHER) {
     const cudaError_t e = launch_operand_consts(L, sc, st);
     if (e != cudaSuccess) return e;
   }
-  return dispatch_fused<false>(L, sc, X, M, L.K, Y, L.N, st);
+  return dispatch_fused<false>(L, sc, X, M, L.K, Y, L.N, st, opts);
 }
 
 cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int64_t M, void* dX, cudaStream_t st) {

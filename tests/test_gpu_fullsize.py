@@ -1,16 +1,19 @@
 """GPU vs oracle at the workloads' full sizes (the Qwen3-1.7B-, Llama-3-8B- and Qwen3-14B-
 shaped blocks with their full calibration batches, and the Qwen3-235B-shaped MoE layer with
 all 128 experts), in the launch configuration bench.py times (four-CTA fused forward and
-dX, CTA-pair dW), on outputs the fp64 oracle computes one by one.
+dX, CTA-pair dW), on outputs the fp64 oracle computes one by one.  Samples cover every
+output tile of every kernel, and each tile is checked on its own as well as overall:
 
 * group statistics: every group;
-* Y and the teacher output: a 64 x 64 sample of rows and columns;
+* Y and the teacher output: 4 rows of every 512-row M block x 4 columns of every 256-column
+  N block, relative Frobenius error per (M block, N block) tile and overall;
 * loss and dY: as functions of the GPU's Y and teacher output (the loss over all M x N
-  elements in fp64; dY on the sampled entries);
-* dX: a 64 x 64 sample, from the GPU's dY (the backward's input) and the oracle's Eq. 6
-  weight;
-* factor gradients, hard codes and alpha: every group of 8 sampled W rows, through the
-  oracle's own G = dY^T X for those rows.
+  elements in fp64; dY on the sampled entries, per tile);
+* dX: the same rows x 4 columns of every 256-column K block, from the GPU's dY (the
+  backward's input) and the oracle's Eq. 6 weight, per (M block, K block) tile;
+* factor gradients, hard codes and alpha: every group of 2 sampled W rows of every 256-row
+  N block, through the oracle's own G = dY^T X for those rows, per (N block, K block) tile
+  of the dW kernel; codes outside the threshold band bit-exact, the band listed.
 """
 import numpy as np
 import pytest
@@ -54,10 +57,33 @@ def test_block_full_size_sampled(device, wl_name, lin_name, phase, s):
     G = N * K // g
     fac = syn.factors(G, 0, f"full/{wl_name}/{lin_name}", perturbed=True)
     got = U.gpu_step(W, X, g, fac, wl.thr_init, phase, s, "bf16", device)
-    _check_sampled(got, W, X, g, fac, wl.thr_init, phase, s, rows_sampled=8)
+    _check_sampled(got, W, X, g, fac, wl.thr_init, phase, s, name=f"full_{wl_name}_{lin_name}_phase{phase}_s{s}")
 
 
-def _check_sampled(got, W, X, g, fac, thr, phase, s, rows_sampled, count=None):
+def _block_sample(n, block, per, r):
+    """`per` sorted indices from every `block`-wide block of range(n) (all of a short one)."""
+    out = []
+    for b0 in range(0, n, block):
+        b1 = min(n, b0 + block)
+        out.append(np.sort(r.choice(np.arange(b0, b1), min(per, b1 - b0), replace=False)))
+    return np.concatenate(out)
+
+
+def _tile_errs(got, want, rows, cols, rblock, cblock):
+    """Relative Frobenius error of every (row block, column block) tile of a sampled
+    [len(rows), len(cols)] comparison; returns the worst and its tile."""
+    worst, where = 0.0, None
+    rb, cb = rows // rblock, cols // cblock
+    for a in np.unique(rb):
+        for b in np.unique(cb):
+            sel = np.ix_(rb == a, cb == b)
+            e = U.fro_rel(got[sel], want[sel])
+            if e > worst:
+                worst, where = e, (int(a), int(b))
+    return worst, where
+
+
+def _check_sampled(got, W, X, g, fac, thr, phase, s, rows_per_block=2, count=None, name=None):
     """The checks of the module docstring for one dense layer (all arrays on the host).
     `count`: the loss's element count when the rows are part of a larger batch (the loss
     itself is then checked by the caller)."""
@@ -70,15 +96,20 @@ def _check_sampled(got, W, X, g, fac, thr, phase, s, rows_sampled, count=None):
     np.testing.assert_allclose(got["delta0"], stats[2], rtol=1e-6)
 
     r = np.random.default_rng(7)
-    ms = np.sort(r.choice(M, 64, replace=False))
-    ns = np.sort(r.choice(N, 64, replace=False))
-    ks = np.sort(r.choice(K, 64, replace=False))
+    ms = _block_sample(M, 512, 4, r)
+    ns = _block_sample(N, 256, 4, r)
+    ks = _block_sample(K, 256, 4, r)
     Wq = O.ternary_weight(W, g, stats, fac, phase, s)[0]
     Xs = X[ms].astype(np.float64)
+    errs, tiles = {}, {}
+
+    def both(key, a, b, rows, cols, rblock, cblock):
+        errs[key] = U.fro_rel(a, b)
+        tiles[key] = _tile_errs(a, b, rows, cols, rblock, cblock)
 
     # forward and teacher forward on the sampled entries
-    errs = {"Y": U.fro_rel(got["Y"][np.ix_(ms, ns)], Xs @ Wq[ns].T),
-            "Y_ref": U.fro_rel(got["Y_ref"][np.ix_(ms, ns)], Xs @ W[ns].astype(np.float64).T)}
+    both("Y", got["Y"][np.ix_(ms, ns)], Xs @ Wq[ns].T, ms, ns, 512, 256)
+    both("Y_ref", got["Y_ref"][np.ix_(ms, ns)], Xs @ W[ns].astype(np.float64).T, ms, ns, 512, 256)
 
     # loss over every element and dY on the sample, from the GPU's own Y and teacher output
     d = got["Y"].astype(np.float64) - got["Y_ref"].astype(np.float64)
@@ -86,30 +117,45 @@ def _check_sampled(got, W, X, g, fac, thr, phase, s, rows_sampled, count=None):
         count = d.size
         loss = float((d * d).sum() / count)
         assert abs(got["loss"] - loss) <= 1e-5 * loss
-    errs["dY"] = U.fro_rel(got["dY"][np.ix_(ms, ns)], 2.0 * d[np.ix_(ms, ns)] / count)
+    both("dY", got["dY"][np.ix_(ms, ns)], 2.0 * d[np.ix_(ms, ns)] / count, ms, ns, 512, 256)
     del d
 
     # dX from the GPU's dY
     dY = got["dY"].astype(np.float64)
-    errs["dX"] = U.fro_rel(got["dX"][np.ix_(ms, ks)], dY[ms] @ Wq[:, ks])
+    both("dX", got["dX"][np.ix_(ms, ks)], dY[ms] @ Wq[:, ks], ms, ks, 512, 256)
 
-    # factor gradients, codes and alpha of 8 sampled rows (all their groups)
-    rows = np.sort(r.choice(N, rows_sampled, replace=False))
+    # factor gradients, codes and alpha of the sampled rows (all their groups)
+    rows = _block_sample(N, 256, rows_per_block, r)
     per_row = K // g
     sub_stats = tuple(_rows(a, rows, per_row) for a in stats)
     sub_fac = tuple(_rows(a, rows, per_row) for a in fac)
     Wsub = W[rows]
     Gsub = dY[:, rows].T @ X.astype(np.float64)
     want = O.factor_grads_from_G(Gsub, Wsub, g, sub_stats, sub_fac, phase, s)
-    for name, w in zip(("g_dmu", "g_dalpha", "g_ddelta"), want):
-        errs[name] = U.fro_rel(_rows(got[name], rows, per_row), w)
+    gcols = np.tile(np.arange(per_row) * g, rows.size).reshape(rows.size, per_row)  # first column of each group
+    for nm, w in zip(("g_dmu", "g_dalpha", "g_ddelta"), want):
+        a = _rows(got[nm], rows, per_row).reshape(rows.size, per_row)
+        b = np.asarray(w).reshape(rows.size, per_row)
+        errs[nm] = U.fro_rel(a, b)
+        # tiles of the dW kernel: 256 rows of N by 256 columns of K
+        worst, where = 0.0, None
+        for ab in np.unique(rows // 256):
+            for kb in np.unique(gcols[0] // 256):
+                sel = np.ix_(rows // 256 == ab, gcols[0] // 256 == kb)
+                e = U.fro_rel(a[sel], b[sel])
+                if e > worst:
+                    worst, where = e, (int(ab), int(kb))
+        tiles[nm] = (worst, where)
+    print(f"{name or ''} overall {errs} worst tiles {tiles} ({ms.size} x {ns.size} Y samples, "
+          f"{rows.size} W rows)")
     bad = {k: v for k, v in errs.items() if not v <= U.TOL_BF16}
     assert not bad, f"tolerance {U.TOL_BF16} exceeded: {bad} (all: {errs})"
+    bad = {k: v for k, v in tiles.items() if not v[0] <= U.TOL_BF16}
+    assert not bad, f"per-tile tolerance {U.TOL_BF16} exceeded: {bad}"
 
     T, alpha, gap = O.hard_codes(Wsub, g, sub_stats, sub_fac)
     codes = O.unpack_codes(got["codes"], N * K).reshape(N, K)[rows].reshape(-1)
-    mism = np.nonzero((codes != T) & (gap > U.NEAR_THRESHOLD))[0]
-    assert mism.size == 0, f"{mism.size} code mismatches outside the threshold band"
+    U.check_codes(codes, T, gap, name=name)
     np.testing.assert_allclose(_rows(got["alpha"], rows, per_row), alpha, rtol=2e-6)
 
 
@@ -175,4 +221,4 @@ def test_c5_moe_full_size_sampled(device):
                    g_dmu=host["g0"][gs], g_dalpha=host["g1"][gs], g_ddelta=host["g2"][gs],
                    alpha=host["alpha"][gs], codes=codes_h[e * N * K // 4:(e + 1) * N * K // 4])
         _check_sampled(got, W[e], X_tok[token_of_row[r0:r1]], g, tuple(f[gs] for f in fac), wl.thr_init, phase, s,
-                       rows_sampled=4, count=R * N)
+                       rows_per_block=1, count=R * N, name=f"full_moe_expert{e}")

@@ -40,8 +40,7 @@ def _compare(got, W, X, g, fac, thr, phase, s, dtype):
     assert not bad, f"tolerance {t} exceeded: {bad} (all: {errs})"
     T, alpha, gap = O.hard_codes(W, g, stats, fac)
     codes = O.unpack_codes(got["codes"], W.size)
-    mism = np.nonzero((codes != T) & (gap > U.NEAR_THRESHOLD))[0]
-    assert mism.size == 0, f"{mism.size} code mismatches outside the threshold band"
+    U.check_codes(codes, T, gap)
     np.testing.assert_allclose(got["alpha"], alpha, rtol=2e-6)
     return errs
 
@@ -181,8 +180,7 @@ def test_modulate_ternarize_matches_oracle(device):
         Wq_ref = O.ternary_weight(W, wl.g, stats, fac, phase, s)[0]
         assert U.fro_rel(U.to_host(Wq), Wq_ref) < 1e-2
         Tr, ar, gap = O.hard_codes(W, wl.g, stats, fac)
-        mism = np.nonzero((U.to_host(T).reshape(-1) != Tr) & (gap > U.NEAR_THRESHOLD))[0]
-        assert mism.size == 0
+        U.check_codes(U.to_host(T).reshape(-1), Tr, gap, name=f"modulate_ternarize_phase{phase}_s{s}")
         np.testing.assert_allclose(U.to_host(alpha), ar, rtol=2e-6)
 
 
