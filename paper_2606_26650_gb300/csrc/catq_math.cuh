@@ -313,4 +313,30 @@ __device__ __forceinline__ void grad_element(float G, float w, const GroupConst&
   acc.sdelta = fmaf(G, sb - sa, acc.sdelta);
 }
 
+// One-exponential form of grad_element for a group whose threshold in sharpness units is
+// D = s Delta >= kOneExpD.  For x >= 0 the term tanh(s(x + Delta)) is then within
+// 2 exp(-2 D) <= 3e-8 of 1 and its sech^2 below 4 exp(-2 D) <= 6e-8, both under fp32
+// resolution of the O(1) terms they join (symmetrically for x < 0), so with the near term
+// y = s|x| - D alone:
+//   f'/k = sech^2 y,   (df/dDelta)/k = -sign(x) sech^2 y,
+//   SOFT T = f = sign(x) (1 + tanh y) / (2 tanh s)     (the producer's one-tanh form),
+// one exponential e = exp(-2|y|) and one reciprocal per element instead of two of each.
+constexpr float kOneExpD = 9.0f;
+
+template <bool MU = false>
+__device__ __forceinline__ void grad_element_1exp(float G, float w, const GroupConst& c, float s, float D,
+                                                  float inv_2tanh_s, float k, int32_t phase, GradSums& acc,
+                                                  float inv_k = 0.0f) {
+  const float x = what(w, c);
+  const float y = fabsf(s * x) - D;
+  const float e = __expf(-2.0f * fabsf(y));
+  const float rcp = __fdividef(1.0f, 1.0f + e);
+  const float s2 = 4.0f * e * rcp * rcp;                 // sech^2 y
+  const float T = (phase == PHASE_SOFT) ? copysignf(1.0f + copysignf((1.0f - e) * rcp, y), x) * inv_2tanh_s
+                                        : hard_q(x, c.delta);
+  acc.smu = fmaf(G, MU ? s2 - inv_k : s2, acc.smu);
+  acc.salpha = fmaf(G, T - x * k * s2, acc.salpha);
+  acc.sdelta = fmaf(G, copysignf(s2, -x), acc.sdelta);
+}
+
 }  // namespace catq

@@ -289,19 +289,6 @@ __device__ __forceinline__ void store_rows_bf16x16(uint16_t* C, int64_t M, int64
   store_rows_packed16(C, M, ncols, row0, col, v, lane);
 }
 
-// 32 fp32 values of one row per lane (row < M, columns from `col`) stored as fp32: eight
-// 16-byte stores per lane (used for a full-precision teacher output, off the hot path).
-__device__ __forceinline__ void store_row_f32x32(float* C, int64_t M, int64_t ncols, int64_t row, int64_t col,
-                                                 const uint32_t (&r)[32]) {
-  if (row >= M) return;
-#pragma unroll
-  for (int p = 0; p < 8; ++p)
-    if (col + 4 * p < ncols)
-      *reinterpret_cast<float4*>(C + row * ncols + col + 4 * p) =
-          make_float4(__uint_as_float(r[4 * p]), __uint_as_float(r[4 * p + 1]), __uint_as_float(r[4 * p + 2]),
-                      __uint_as_float(r[4 * p + 3]));
-}
-
 // 16 fp32 values of one row per lane (row < M, columns from `col`) stored as fp32: four
 // 16-byte stores per lane (used for a full-precision teacher output, off the hot path).
 __device__ __forceinline__ void store_row_f32x16(float* C, int64_t M, int64_t ncols, int64_t row, int64_t col,
@@ -965,7 +952,7 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
 
   if (warp == kTma) {
     if (lane == 0) {
-      uint32_t stage = 0, phase = 0, issued_mask = 0, issued_phase = 0;
+      uint32_t stage = 0, phase = 0, issued_mask = 0, issued_phase = 0, it_tma = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
         const int r = t % tiles_per_split;
@@ -978,7 +965,13 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
           mdy = &gm.dy[t / tiles_per_split];
           mx = &gm.x[t / tiles_per_split];
         }
-        for (int kb = kb0; kb < kb1; ++kb) {
+        // Serpentine contraction: tiles of odd iterations (every other tile wave) run their M
+        // blocks backwards, so a wave starts where the previous one ended, with that part of
+        // X still in L2.  The MMA loop walks the same order.
+        const bool rev = (it_tma & 1u) != 0;
+        ++it_tma;
+        for (int j = 0; j < kb1 - kb0; ++j) {
+          const int kb = rev ? kb1 - 1 - j : kb0 + j;
           if (!mbar_wait(empty(stage), phase ^ 1u, wc)) { ok = false; break; }
           const uint32_t sa = base + stage * Cfg::kStageBytes, sb = sa + Cfg::kABytes;
           const int32_t m = kb * BK;
@@ -1017,7 +1010,9 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
         const uint32_t buf = it & 1u;
         if (!mbar_wait(tmem_empty0 + 8u * buf, ((it >> 1) & 1u) ^ 1u, wc)) break;
         tc_fence_after();
-        for (int kb = kb0; kb < kb1; ++kb) {
+        // Stages arrive in the TMA's order (forwards or, on odd iterations, backwards over M);
+        // the sum does not depend on it, and the tile's first stage clears the accumulator.
+        for (int j = 0; j < kb1 - kb0; ++j) {
           if (!mbar_wait(full(stage), phase, wc)) { ok = false; break; }
           tc_fence_after();
           const uint32_t sa = base + stage * Cfg::kStageBytes, sb = sa + Cfg::kABytes;
@@ -1025,7 +1020,7 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
           for (int kk = 0; kk < BK / 16; ++kk) {
             const uint64_t adesc = smem_desc_sw128(sa + kk * 2048, 8192, 1024);
             const uint64_t bdesc = smem_desc_sw128(sb + kk * 2048, 8192, 1024);
-            umma_bf16<CG>(tmem_base + buf * BN, adesc, bdesc, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+            umma_bf16<CG>(tmem_base + buf * BN, adesc, bdesc, idesc, (j > 0 || kk > 0) ? 1u : 0u);
           }
           umma_commit<CG>(empty(stage));
           if (++stage == S) { stage = 0; phase ^= 1u; }
@@ -1099,7 +1094,21 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
             gc = group_const(L, j);
             cur_j = j;
           }
-          if (gc.alpha != 0.0f) {
+          const float D = args.sc.s * gc.delta;
+          if (gc.alpha != 0.0f && D >= kOneExpD) {
+            // one exponential per weight (the far tanh term is 1 to fp32 resolution)
+#pragma unroll
+            for (int v = 0; v < 4; ++v) {
+              const uint32_t w4[4] = {wcur[v].x, wcur[v].y, wcur[v].z, wcur[v].w};
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                grad_element_1exp<MU>(__uint_as_float(rg[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), gc, args.sc.s, D,
+                                      args.sc.inv_2tanh_s, k_sc, args.sc.phase, acc, inv_k);
+                grad_element_1exp<MU>(__uint_as_float(rg[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), gc, args.sc.s,
+                                      D, args.sc.inv_2tanh_s, k_sc, args.sc.phase, acc, inv_k);
+              }
+            }
+          } else if (gc.alpha != 0.0f) {
 #pragma unroll
             for (int v = 0; v < 4; ++v) {
               const uint32_t w4[4] = {wcur[v].x, wcur[v].y, wcur[v].z, wcur[v].w};
