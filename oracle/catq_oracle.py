@@ -385,3 +385,49 @@ def factor_update(factors, grads, moments, t: int, lr: float, beta1: float = 0.9
         new_m.append(m)
         new_v.append(v)
     return project_factors(*new_p, margin), tuple(new_m) + tuple(new_v)
+
+
+# ------------------------------------------------------------------ direct learning and Fig. fig:error
+# §2.2 compares three ways to set a group's alpha and Delta: a static approximation (SA, the
+# absmean rule of BitNet b1.58 and others), learning alpha and Delta directly (DL, started
+# from that static rule), and the learnable modulation (LM); Fig. fig:error plots the
+# per-group weight reconstruction error each leaves.
+
+def direct_grads(d_alpha, d_delta, g_dalpha, g_ddelta):
+    """Gradients of direct learning's parameters from the modulation's factor gradients.
+    DL learns the scale alpha and the weight-space threshold Delta_W = alpha Delta of each
+    group, with mu fixed at mu0 (0 for the static rules), read here in units of the group's
+    static statistics so that the paper's learning rate means the same relative step as for
+    the modulation's factors:
+        a = alpha / alpha0 = d_alpha,   d = Delta_W / (alpha0 Delta0) = d_alpha d_delta.
+    With d_alpha = a and d_delta = d / a the chain rule gives
+        dL/da = g_dalpha - g_ddelta d_delta / d_alpha,   dL/dd = g_ddelta / d_alpha."""
+    d_alpha = np.asarray(d_alpha, np.float64)
+    d_delta = np.asarray(d_delta, np.float64)
+    g_dalpha = np.asarray(g_dalpha, np.float64)
+    g_ddelta = np.asarray(g_ddelta, np.float64)
+    return g_dalpha - g_ddelta * d_delta / d_alpha, g_ddelta / d_alpha
+
+
+def direct_update(d_alpha, d_delta, g_dalpha, g_ddelta, moments, t: int, lr: float, beta1: float = 0.9,
+                  beta2: float = 0.999, eps: float = 1e-8, weight_decay: float = 0.0, margin: float = 1e-4):
+    """One update of direct learning: AdamW (``adamw_step``) on a = d_alpha and
+    d = d_alpha d_delta with the gradients of ``direct_grads``, the constraints alpha > 0 and
+    Delta > 0 kept as a >= margin and d >= margin, then d_alpha = a and d_delta = d / a.
+    moments = (m_a, m_d, v_a, v_d).  Returns (d_alpha, d_delta, moments)."""
+    d_alpha = np.asarray(d_alpha, np.float64)
+    d_delta = np.asarray(d_delta, np.float64)
+    ga, gd = direct_grads(d_alpha, d_delta, g_dalpha, g_ddelta)
+    a, ma, va = adamw_step(d_alpha, ga, moments[0], moments[2], t, lr, beta1, beta2, eps, weight_decay)
+    d, md, vd = adamw_step(d_alpha * d_delta, gd, moments[1], moments[3], t, lr, beta1, beta2, eps, weight_decay)
+    a = np.clip(a, margin, np.inf)
+    d = np.clip(d, margin, np.inf)
+    return a, d / a, (ma, md, va, vd)
+
+
+def group_recon_error(W, g, stats, factors):
+    """Per-group weight reconstruction error of the hard ternarization (Fig. fig:error):
+    the mean over the group of (W - alpha Q(What; Delta))^2 (W ~ alpha T, no mu)."""
+    Wq = ternary_weight(W, g, stats, factors, PHASE_HARD, 1.0)[0]
+    d = (np.asarray(W, np.float64) - Wq).reshape(-1, g)
+    return (d * d).mean(axis=1)

@@ -813,3 +813,72 @@ def test_a8_step_reduces_to_the_plain_step_on_grid_inputs():
     for k in ("Y", "Y_ref", "dY", "dX", "g_dmu", "g_dalpha", "g_ddelta"):
         np.testing.assert_allclose(a8[k], ref[k], rtol=1e-13, atol=1e-15, err_msg=k)
     assert a8["loss"] == pytest.approx(ref["loss"], rel=1e-13)
+
+
+# ----------------------------------------------------------------- direct learning (Fig. fig:error)
+
+def test_direct_grads_match_central_differences_of_the_direct_parametrization():
+    """DL's gradients in (a, d) = (alpha / alpha0, Delta_W / (alpha0 Delta0)) against central
+    differences of the loss written directly in a and d (mu at mu0 = 0 for the absmean rule),
+    in the soft phase where the loss is smooth."""
+    r = np.random.default_rng(70)
+    N, K, g, M = 3, 8, 4, 5
+    W = r.standard_normal((N, K)) * 0.05
+    X = r.standard_normal((M, K))
+    stats = O.group_stats(W, g, O.THR_ABSMEAN)
+    G = N * K // g
+    a = r.uniform(0.8, 1.2, G)
+    d = r.uniform(0.3, 0.7, G)
+    s = 8.0
+    Y_ref = O.linear_fwd(X, W)
+
+    def loss(a, d):
+        fac = (np.zeros(G), a, d / a)
+        Wq = O.ternary_weight(W, g, stats, fac, O.PHASE_SOFT, s)[0]
+        return O.recon_loss(O.linear_fwd(X, Wq), Y_ref)[0]
+
+    step = O.calibration_step(X, W, g, stats, (np.zeros(G), a, d / a), O.PHASE_SOFT, s)
+    ga, gd = O.direct_grads(a, d / a, step["g_dalpha"], step["g_ddelta"])
+    h = 1e-6
+    for j in range(G):
+        e = np.zeros(G)
+        e[j] = h
+        fa = (loss(a + e, d) - loss(a - e, d)) / (2 * h)
+        fd = (loss(a, d + e) - loss(a, d - e)) / (2 * h)
+        assert ga[j] == pytest.approx(fa, rel=1e-5, abs=1e-9)
+        assert gd[j] == pytest.approx(fd, rel=1e-5, abs=1e-9)
+
+
+def test_direct_update_is_adamw_on_a_and_d():
+    """The update against PyTorch's own AdamW on parameters (a, d) fed the converted
+    gradients (fp64, several updates), then the return to (d_alpha, d_delta)."""
+    torch = pytest.importorskip("torch")
+    r = np.random.default_rng(71)
+    G = 64
+    dal = r.uniform(0.8, 1.2, G)
+    ddl = r.uniform(0.8, 1.2, G)
+    ta = torch.tensor(dal.copy(), dtype=torch.float64, requires_grad=True)
+    td = torch.tensor(dal * ddl, dtype=torch.float64, requires_grad=True)
+    opt = torch.optim.AdamW([ta, td], lr=1e-3, betas=(0.9, 0.999), eps=1e-8, weight_decay=0.01)
+    mom = (np.zeros(G),) * 4
+    for t in range(1, 6):
+        gal = r.standard_normal(G) * 1e-3
+        gdl = r.standard_normal(G) * 1e-3
+        ga, gd = O.direct_grads(dal, ddl, gal, gdl)
+        ta.grad = torch.tensor(ga)
+        td.grad = torch.tensor(gd)
+        opt.step()
+        dal, ddl, mom = O.direct_update(dal, ddl, gal, gdl, mom, t, 1e-3, weight_decay=0.01, margin=0.0)
+        np.testing.assert_allclose(dal, ta.detach().numpy(), rtol=1e-13)
+        np.testing.assert_allclose(dal * ddl, td.detach().numpy(), rtol=1e-13)
+
+
+def test_group_recon_error_closed_form():
+    """A group [v, -v, 3v, -3v] under absmean (alpha = 2|v|, Delta = |v|): Q gives 0, 0, 1, -1,
+    so the error is (v^2 + v^2 + v^2 + v^2) / 4 = v^2 (v a power of two: every value is exact,
+    and the two small elements sit exactly on the threshold, where Eq. 2 gives 0)."""
+    v = 2.0 ** -7
+    W = np.array([[v, -v, 3 * v, -3 * v]])
+    stats = O.group_stats(W, 4, O.THR_ABSMEAN)
+    fac = (np.zeros(1), np.ones(1), np.ones(1))
+    assert O.group_recon_error(W, 4, stats, fac)[0] == pytest.approx(v * v, rel=1e-12)
