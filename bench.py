@@ -17,6 +17,7 @@ only other place this file runs the oracle besides the cpu_baseline leg).
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import os
@@ -63,6 +64,8 @@ def parse(argv=None):
     p.add_argument("--no-also", action="store_true", help="skip the secondary workloads and phase")
     p.add_argument("--streams", type=int, default=4,
                    help="CUDA streams the block's linears are spread over (independent problems)")
+    p.add_argument("--linear", default=None,
+                   help="run only this linear of the block (single-kernel profiling of one layer)")
     return p.parse_args(argv)
 
 
@@ -176,7 +179,8 @@ def run_reference(args):
 
 
 def workload_config(wl, args):
-    return {"workload": wl.name, "tokens": wl.M, "group_size": wl.g, "phase": "soft", "s": args.s,
+    return {"workload": wl.name + (f"/{args.linear}" if getattr(args, "linear", None) else ""), "tokens": wl.M,
+            "group_size": wl.g, "phase": "soft", "s": args.s,
             "linears": {lin.name: [lin.K, lin.N] for lin in wl.linears},
             "flops_per_step": wl.flops_per_step, "streams": getattr(args, "streams", 1),
             "l2": "inputs larger than L2 (per-step working set of weights and activations > 129 MB)"}
@@ -389,6 +393,8 @@ def run_ours(args):
     wl = syn.WORKLOADS[args.workload]
     if wl.experts:
         raise SystemExit("MoE workloads are parity cases, not bench lines")
+    if args.linear:
+        wl = dataclasses.replace(wl, linears=(wl.linear(args.linear),))
     sched = C.schedule(C.PHASE_SOFT, args.s)
     nstreams = max(1, args.streams)
     blk = BlockRun(C, torch, wl, dev, rank, nstreams)
@@ -507,6 +513,7 @@ def run_ours(args):
         also[f"{wl.name}/decode_b8"] = measure_decode(C, torch, wl, dev, peaks, rows=8)
         also[f"{wl.name}/decode_b1_mu"] = measure_decode(C, torch, wl, dev, peaks, rows=1, with_mu=True)
         also["c5_qwen3_235b_moe/soft"] = measure_moe(C, torch, dev, peaks, world, args.s)
+        also[f"{wl.name}/fig_error_k_proj"] = measure_fig_error(C, torch, wl, dev, args.s)
         for name in ALSO_WORKLOADS:
             if name == wl.name:
                 continue
@@ -591,6 +598,69 @@ def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20, with_m
             "launches_per_step": blocks * len(wl.linears), "bytes_per_step": nbytes, "us_per_step": ms * 1e3,
             "value": gbs, "unit": "GB/s", "peak": peaks["hbm"], "frac_of_hbm": gbs / peaks["hbm"],
             "steps": steps, "graph": True, "with_mu": with_mu}
+
+
+def measure_fig_error(C, torch, wl, dev, s0, epochs=20, batches=3, rows=2048, lr0=1e-3):
+    """The synthetic analogue of Fig. fig:error (§2.2) on the block's k_proj: per-group weight
+    reconstruction error of the hard ternarization under the static absmean rule (SA), direct
+    learning started from it (DL) and the learnable modulation (LM), the learned two after
+    `epochs` x `batches` calibration steps of `rows` tokens with hard ternarization throughout
+    (the figure's setting), AdamW at lr0 decayed linearly.  Errors are per group, relative to
+    the group's mean squared weight."""
+    lin = wl.linear("k_proj")
+    N, K, g = lin.N, lin.K, wl.g
+    G = N * K // g
+
+    def up(a):
+        return torch.from_numpy(syn.bf16_bits(a).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    W = up(syn.weight(wl, lin))
+    xs = [up(syn.activations(wl, lin.x, (b + 1) * rows, K)[b * rows:]) for b in range(batches)]
+    w2 = (W.float().reshape(G, g) ** 2).mean(dim=1)
+    out = {}
+    for kind in ("SA", "DL", "LM"):
+        layer = C.Layer.create(W, g)
+        C.catq_group_stats(layer, C.THR_HALF if kind == "LM" else C.THR_ABSMEAN)
+        if kind != "SA":
+            hp = C.adamw()
+            moments = torch.zeros((6 if kind == "LM" else 4) * G, device=dev)
+            grads = [torch.empty(G, device=dev) for _ in range(3)]
+            loss = torch.empty(1, device=dev)
+            yts = []
+            for xb in xs:
+                yt = torch.empty(rows, N, dtype=torch.bfloat16, device=dev)
+                C.catq_soft_ternary_linear_fwd(layer, C.schedule(C.PHASE_TEACHER), xb, yt)
+                yts.append(yt)
+            Y, dY = torch.empty_like(yts[0]), torch.empty_like(yts[0])
+            wsl = C.workspace(C.catq_recon_loss_workspace_bytes(Y.numel()), dev)
+            wsb = C.workspace(C.catq_bwd_workspace_bytes(layer, rows), dev)
+            sched = C.schedule(C.PHASE_HARD, s0)
+            t = 0
+            for _ in range(epochs):
+                for xb, yt in zip(xs, yts):
+                    C.catq_soft_ternary_linear_fwd(layer, sched, xb, Y)
+                    C.catq_recon_loss(Y, yt, loss, dY, wsl)
+                    C.catq_soft_ternary_linear_bwd(layer, sched, xb, dY, None, *grads, workspace=wsb)
+                    lr = C.catq_linear_decay_lr(lr0, t, epochs * batches)
+                    t += 1
+                    if kind == "LM":
+                        C.catq_factor_adamw_step(layer.d_mu, layer.d_alpha, layer.d_delta, *grads, moments, hp, t, lr)
+                    else:
+                        C.catq_direct_adamw_step(layer.d_alpha, layer.d_delta, grads[1], grads[2], moments, hp, t, lr)
+        err = torch.empty(G, device=dev)
+        C.catq_group_recon_error(layer, err)
+        out[kind] = (err / w2).cpu().numpy().astype(np.float64)
+    status = C.catq_device_status()
+    if status != 0:
+        raise SystemExit(f"device status {C.STATUS.get(status, status)} in the fig:error run")
+    res = {k: {"mean": float(v.mean()), "median": float(np.median(v)), "p99": float(np.quantile(v, 0.99)),
+               "max": float(v.max())} for k, v in out.items()}
+    res["groups"] = G
+    res["groups_worse_than_SA"] = {k: int((out[k] > out["SA"]).sum()) for k in ("DL", "LM")}
+    res["setting"] = (f"k_proj {K}->{N}, g {g}, {epochs} epochs x {batches} batches of {rows} tokens, hard "
+                      f"ternarization throughout (backward at s = {s0}), AdamW lr {lr0} decayed linearly; error = "
+                      f"mean (W - Wq)^2 / mean W^2 per group")
+    return res
 
 
 def measure_moe(C, torch, dev, peaks, world, s, steps=5, warmup=2):

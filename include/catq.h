@@ -336,6 +336,29 @@ catq_status catq_factor_adamw_step(int64_t G, float* d_mu, float* d_alpha, float
                                    const float* g_dalpha, const float* g_ddelta, float* moments,
                                    const catq_adamw* hp, int64_t t, float lr, catq_stream stream);
 
+/* Direct learning (DL) of a group's scale and threshold, the alternative to the modulation
+ * that §2.2 compares (Fig. fig:error; the paper gives no formula, so this is the library's
+ * reading).  DL learns alpha and the weight-space threshold Delta_W = alpha Delta with mu
+ * fixed at mu0 (0 for the static rules it starts from, e.g. CATQ_THR_ABSMEAN), in units of
+ * the group's static statistics, so that the paper's learning rate means the same relative
+ * step as for the modulation's factors:
+ *   a = alpha / alpha0 = d_alpha,   d = Delta_W / (alpha0 Delta0) = d_alpha d_delta.
+ * From the factor gradients of catq_soft_ternary_linear_bwd (the same forward, d_mu unused):
+ *   dL/da = g_dalpha - g_ddelta d_delta / d_alpha,   dL/dd = g_ddelta / d_alpha,
+ * then one AdamW step on a and on d as in catq_factor_adamw_step, the constraints
+ * alpha > 0, Delta > 0 as a, d >= hp->margin, and d_alpha = a, d_delta = d / a (in place).
+ * moments: [4, G] fp32 device (m_a, m_d, v_a, v_d), zero before the first update.  A group
+ * with d_alpha == 0 is left unchanged.  Errors and G == 0 as catq_factor_adamw_step. */
+catq_status catq_direct_adamw_step(int64_t G, float* d_alpha, float* d_delta, const float* g_dalpha,
+                                   const float* g_ddelta, float* moments, const catq_adamw* hp, int64_t t, float lr,
+                                   catq_stream stream);
+
+/* Per-group weight reconstruction error of the hard ternarization (Fig. fig:error):
+ *   err[j] = (1/g) sum over group j of (W - Wq)^2,  Wq = alpha Q(What; Delta) (+ mu with
+ *   CATQ_RECON_ALPHA_T_MU), with the codes the pack and the HARD forward take.
+ * err: [G] fp32 device, 4-byte aligned.  fp32 sums. */
+catq_status catq_group_recon_error(const catq_layer* layer, float* err, catq_stream stream);
+
 /* ------------------------------------------------------------------ grouped (MoE) layers
  * A mixture-of-experts layer quantizes every expert's linear like a dense one (App. B.2:
  * experts are quantized, routers are not).  E experts of identical shape are stacked:

@@ -105,6 +105,8 @@ def lib() -> ctypes.CDLL:
         "catq_fwd_loss_workspace_bytes": (S, [LP, I64]),
         "catq_soft_ternary_linear_fwd_loss": (I32, [LP, catq_schedule, P, I64, I32, P, P, I32, I32, P, P, P, P, S, P]),
         "catq_act_quant_a8": (I32, [P, I64, I64, I32, P, P, P, P]),
+        "catq_direct_adamw_step": (I32, [I64, P, P, P, P, P, ctypes.POINTER(catq_adamw), I64, F, P]),
+        "catq_group_recon_error": (I32, [LP, P, P]),
         "catq_grouped_fwd_loss_workspace_bytes": (S, [ctypes.POINTER(catq_grouped_layer), P]),
         "catq_grouped_soft_ternary_linear_fwd_loss": (I32, [ctypes.POINTER(catq_grouped_layer), catq_schedule, P, P,
                                                             I32, P, I32, P, P, P, P, S, P]),
@@ -417,6 +419,24 @@ def catq_factor_adamw_step(d_mu, d_alpha, d_delta, g_dmu, g_dalpha, g_ddelta, mo
     _check(lib().catq_factor_adamw_step(d_mu.numel(), _ptr(d_mu), _ptr(d_alpha), _ptr(d_delta), _ptr(g_dmu),
                                         _ptr(g_dalpha), _ptr(g_ddelta), _ptr(moments), ctypes.byref(hp), int(t),
                                         float(lr), _stream(stream)), "catq_factor_adamw_step")
+
+
+def catq_direct_adamw_step(d_alpha, d_delta, g_dalpha, g_ddelta, moments, hp: catq_adamw, t: int, lr: float,
+                           stream=None):
+    """Direct learning's update of (d_alpha, d_delta) [G] in place; moments [4 * G]."""
+    G, w = d_alpha.numel(), "catq_direct_adamw_step"
+    for name, arr in zip(("d_alpha", "d_delta", "g_dalpha", "g_ddelta"), (d_alpha, d_delta, g_dalpha, g_ddelta)):
+        _buf(arr, name, 4 * G, w)
+    _buf(moments, "moments", 4 * 4 * G, w)
+    _check(lib().catq_direct_adamw_step(G, _ptr(d_alpha), _ptr(d_delta), _ptr(g_dalpha), _ptr(g_ddelta),
+                                        _ptr(moments), ctypes.byref(hp), int(t), float(lr), _stream(stream)), w)
+
+
+def catq_group_recon_error(layer: Layer, err, stream=None):
+    """err [G] = per-group mean of (W - Wq)^2 for the hard reconstruction."""
+    st = layer.struct()
+    _buf(err, "err", 4 * layer.G, "catq_group_recon_error")
+    _check(lib().catq_group_recon_error(ctypes.byref(st), _ptr(err), _stream(stream)), "catq_group_recon_error")
 
 
 def catq_selftest_wait_timeout(timeout_ns: int, stream=None):

@@ -696,6 +696,48 @@ catq_status catq_factor_adamw_step(int64_t G, float* d_mu, float* d_alpha, float
   return cuda_status(launch_factor_adamw(G, a, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+catq_status catq_direct_adamw_step(int64_t G, float* d_alpha, float* d_delta, const float* g_dalpha,
+                                   const float* g_ddelta, float* moments, const catq_adamw* hp, int64_t t, float lr,
+                                   catq_stream stream) {
+  if (G < 0) return CATQ_ERR_SHAPE;
+  if (G == 0) return CATQ_OK;
+  if (!d_alpha || !d_delta || !g_dalpha || !g_ddelta || !moments || !hp) return CATQ_ERR_INVALID_ARG;
+  if (t < 1 || !(lr >= 0.0f) || !std::isfinite(lr)) return CATQ_ERR_INVALID_ARG;
+  if (!(hp->beta1 >= 0.0f && hp->beta1 < 1.0f) || !(hp->beta2 >= 0.0f && hp->beta2 < 1.0f) ||
+      !(hp->eps > 0.0f) || !std::isfinite(hp->eps) || !(hp->weight_decay >= 0.0f) ||
+      !std::isfinite(hp->weight_decay) || !(hp->margin >= 0.0f && hp->margin < 0.5f))
+    return CATQ_ERR_INVALID_ARG;
+  const void* ptrs[5] = {d_alpha, d_delta, g_dalpha, g_ddelta, moments};
+  for (const void* p : ptrs)
+    if (reinterpret_cast<uintptr_t>(p) & 3u) return CATQ_ERR_ALIGN;
+  DirectArgs a{};
+  a.d_alpha = d_alpha;
+  a.d_delta = d_delta;
+  a.g_dalpha = g_dalpha;
+  a.g_ddelta = g_ddelta;
+  a.m = moments;
+  a.v = moments + 2 * G;
+  const double b1 = hp->beta1, b2 = hp->beta2;
+  a.decay = static_cast<float>(1.0 - static_cast<double>(lr) * hp->weight_decay);
+  a.beta1 = hp->beta1;
+  a.one_minus_beta1 = static_cast<float>(1.0 - b1);
+  a.beta2 = hp->beta2;
+  a.one_minus_beta2 = static_cast<float>(1.0 - b2);
+  a.step = static_cast<float>(lr / (1.0 - std::pow(b1, static_cast<double>(t))));
+  a.inv_sqrt_bc2 = static_cast<float>(1.0 / std::sqrt(1.0 - std::pow(b2, static_cast<double>(t))));
+  a.eps = hp->eps;
+  a.margin = hp->margin;
+  return cuda_status(launch_direct_adamw(G, a, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+catq_status catq_group_recon_error(const catq_layer* layer, float* err, catq_stream stream) {
+  catq_status st = check_layer(layer, true);
+  if (st != CATQ_OK) return st;
+  if (!err) return CATQ_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(err) & 3u) return CATQ_ERR_ALIGN;
+  return cuda_status(launch_group_recon_error(to_dev(layer), layer->w_dtype, err, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 catq_status catq_selftest_wait_timeout(uint64_t timeout_ns, catq_stream stream) {
   if (timeout_ns < 1000 || timeout_ns > 1000000000ull) return CATQ_ERR_INVALID_ARG;
   return cuda_status(launch_wait_probe(timeout_ns, reinterpret_cast<cudaStream_t>(stream)));

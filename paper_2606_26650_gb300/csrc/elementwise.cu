@@ -726,6 +726,64 @@ __global__ void __launch_bounds__(kThreads) factor_adamw_kernel(int64_t G, const
   else factor_adamw_array<2>(G, a);
 }
 
+// ---------------------------------------------------------------- direct learning (DL)
+// One thread per group: DL's parameters a = d_alpha and d = d_alpha d_delta (the scale and
+// the weight-space threshold in units of the group's static statistics), their gradients
+// from the factor gradients by the chain rule, one AdamW step on each, the constraints
+// a, d >= margin, and the return to d_alpha = a, d_delta = d / a.  A group with d_alpha == 0
+// (only reachable with margin 0) is left unchanged.
+__global__ void __launch_bounds__(kThreads) direct_adamw_kernel(int64_t G, const DirectArgs a) {
+  for (int64_t i = blockIdx.x * (int64_t)kThreads + threadIdx.x; i < G; i += (int64_t)gridDim.x * kThreads) {
+    const float dal = a.d_alpha[i], ddl = a.d_delta[i];
+    if (dal == 0.0f) continue;
+    const float gal = a.g_dalpha[i], gdl = a.g_ddelta[i];
+    const float ga = gal - gdl * ddl / dal;
+    const float gd = gdl / dal;
+    float p[2] = {dal, dal * ddl};
+    const float g2[2] = {ga, gd};
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      float* const Mo = a.m + q * G;
+      float* const Vo = a.v + q * G;
+      const float m = fmaf(a.beta1, Mo[i], a.one_minus_beta1 * g2[q]);
+      const float v = fmaf(a.beta2, Vo[i], a.one_minus_beta2 * (g2[q] * g2[q]));
+      const float denom = fmaf(sqrtf(v), a.inv_sqrt_bc2, a.eps);
+      float x = p[q] * a.decay;
+      x -= a.step * (m / denom);
+      p[q] = x < a.margin ? a.margin : x;
+      Mo[i] = m;
+      Vo[i] = v;
+    }
+    a.d_alpha[i] = p[0];
+    a.d_delta[i] = p[1] / p[0];
+  }
+}
+
+// ---------------------------------------------------------------- weight reconstruction error
+// One warp per group: mean over the group of (W - Wq)^2 with Wq the hard reconstruction
+// alpha Q(What; Delta) (+ mu for W ~ alpha T + mu), as the pack and the HARD forward decide
+// the codes.  fp32 sums, reduced across the warp in a fixed order.
+template <typename T>
+__global__ void __launch_bounds__(kThreads) group_recon_error_kernel(LayerDev L, float* __restrict__ err) {
+  const int lane = threadIdx.x & 31;
+  const int64_t G = L.N * L.K / L.g;
+  const T* W = static_cast<const T*>(L.W);
+  for (int64_t j = (blockIdx.x * (int64_t)kThreads + threadIdx.x) >> 5; j < G; j += ((int64_t)gridDim.x * kThreads) >> 5) {
+    const GroupConst c = group_const(L, j);
+    const float m = L.recon ? c.mu : 0.0f;
+    float acc = 0.0f;
+    for (int32_t e = lane; e < L.g; e += 32) {
+      const float w = load_scalar(W + j * L.g + e);
+      const float q = c.alpha != 0.0f ? c.alpha * hard_q(what(w, c), c.delta) : 0.0f;
+      const float d = w - (q + m);
+      acc = fmaf(d, d, acc);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) err[j] = acc / static_cast<float>(L.g);
+  }
+}
+
 int grid_for(int64_t work, int64_t per_block) {
   int64_t b = (work + per_block - 1) / per_block;
   if (b < 1) b = 1;
@@ -907,6 +965,20 @@ cudaError_t launch_grad_reduce(const LayerDev& L, StepScalars sc, const float* p
   const int64_t G = L.N * L.K / L.g;
   grad_reduce_kernel<<<grid_for(G, kThreads), kThreads, 0, st>>>(L, sc, partials, splits, P, g_dmu, g_dalpha,
                                                                  g_ddelta);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_direct_adamw(int64_t G, const DirectArgs& a, cudaStream_t st) {
+  if (G == 0) return cudaSuccess;
+  direct_adamw_kernel<<<grid_for(G, kThreads), kThreads, 0, st>>>(G, a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_group_recon_error(const LayerDev& L, int32_t w_dtype, float* err, cudaStream_t st) {
+  const int64_t G = L.N * L.K / L.g;
+  const int grid = grid_for((G + kThreads / 32 - 1) / (kThreads / 32), 1);
+  if (w_dtype == 1) group_recon_error_kernel<__nv_bfloat16><<<grid, kThreads, 0, st>>>(L, err);
+  else group_recon_error_kernel<float><<<grid, kThreads, 0, st>>>(L, err);
   return cudaGetLastError();
 }
 

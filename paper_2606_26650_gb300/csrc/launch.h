@@ -95,6 +95,22 @@ struct AdamwArgs {
 };
 cudaError_t launch_factor_adamw(int64_t G, const AdamwArgs& a, cudaStream_t st);
 
+// Direct learning's update of (d_alpha, d_delta) (see catq_direct_adamw_step): moments m[2G]
+// (a, then d) and v[2G]; the scalars as in AdamwArgs; the projection floor `margin`.
+struct DirectArgs {
+  float* d_alpha;
+  float* d_delta;
+  const float* g_dalpha;
+  const float* g_ddelta;
+  float* m;
+  float* v;
+  float decay, beta1, one_minus_beta1, beta2, one_minus_beta2, step, inv_sqrt_bc2, eps, margin;
+};
+cudaError_t launch_direct_adamw(int64_t G, const DirectArgs& a, cudaStream_t st);
+
+// err[j] = mean over group j of (W - alpha Q(What; Delta) [- mu])^2.
+cudaError_t launch_group_recon_error(const LayerDev& L, int32_t w_dtype, float* err, cudaStream_t st);
+
 // Writes L.op_const (operand_const_vec of every group, [K/g][N]) for schedule point sc.
 cudaError_t launch_operand_consts(const LayerDev& L, StepScalars sc, cudaStream_t st);
 
