@@ -547,37 +547,48 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+# Linears of a decoder block that may run in one launch (their inputs do not depend on each
+# other): q, k, v read the block's input; o reads the attention output; gate and up read the
+# post-attention input; down reads their product.
+DECODE_GROUPS = (("q_proj", "k_proj", "v_proj"), ("o_proj",), ("gate_proj", "up_proj"), ("down_proj",))
+
+
 def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20, with_mu=False):
-    """Inference with the deployed form (catq_ternary_infer) of every linear of `blocks`
-    blocks shaped like `wl`, for `rows` token rows: one decode step reads every layer's 2-bit
-    codes and group scales (and group offsets, `with_mu`) once (working set far beyond L2).
-    The step's launches are captured in a CUDA graph and replayed; value = algorithmic
-    bytes / time."""
+    """Inference with the deployed form of every linear of `blocks` blocks shaped like `wl`,
+    for `rows` token rows: one decode step reads every layer's 2-bit codes and group scales
+    (and group offsets, `with_mu`) once (working set far beyond L2).  Each block runs as four
+    launches of catq_ternary_infer_batched, one per set of linears whose inputs are
+    independent (DECODE_GROUPS), in block order, as a decode step must.  The step's launches
+    are captured in a CUDA graph and replayed; value = algorithmic bytes / time."""
     gen = torch.Generator(device=dev)
     gen.manual_seed(0)
-    layers, nbytes = [], 0
+    launches, nbytes, g = [], 0, wl.g
     for _ in range(blocks):
-        for lin in wl.linears:
-            N, K, g = lin.N, lin.K, wl.g
-            r = torch.randint(0, 81, (N * K // 4,), generator=gen, device=dev, dtype=torch.int32)
-            codes = (r % 3 + ((r // 3) % 3) * 4 + ((r // 9) % 3) * 16 + (r // 27) * 64).to(torch.uint8)
-            alpha = torch.rand(N * K // g, generator=gen, device=dev) * 0.02 + 0.01
-            X = torch.randn(rows, K, generator=gen, device=dev).to(torch.bfloat16)
-            Y = torch.empty(rows, N, dtype=torch.bfloat16, device=dev)
-            mu = (torch.rand(N * K // g, generator=gen, device=dev) - 0.5) * 0.01 if with_mu else None
-            layers.append(((codes, alpha, N, K, g, X, Y), mu))
-            nbytes += codes.numel() + alpha.numel() * 4 + X.numel() * 2 + Y.numel() * 2
-            nbytes += 0 if mu is None else mu.numel() * 4
+        for names in DECODE_GROUPS:
+            group = []
+            for name in names:
+                lin = wl.linear(name)
+                N, K = lin.N, lin.K
+                r = torch.randint(0, 81, (N * K // 4,), generator=gen, device=dev, dtype=torch.int32)
+                codes = (r % 3 + ((r // 3) % 3) * 4 + ((r // 9) % 3) * 16 + (r // 27) * 64).to(torch.uint8)
+                alpha = torch.rand(N * K // g, generator=gen, device=dev) * 0.02 + 0.01
+                X = torch.randn(rows, K, generator=gen, device=dev).to(torch.bfloat16)
+                Y = torch.empty(rows, N, dtype=torch.bfloat16, device=dev)
+                mu = (torch.rand(N * K // g, generator=gen, device=dev) - 0.5) * 0.01 if with_mu else None
+                group.append((codes, alpha, N, K, X, Y, mu))
+                nbytes += codes.numel() + alpha.numel() * 4 + X.numel() * 2 + Y.numel() * 2
+                nbytes += 0 if mu is None else mu.numel() * 4
+            launches.append(group)
     side = torch.cuda.Stream(device=dev)
     side.wait_stream(torch.cuda.current_stream())
     with torch.cuda.stream(side):  # warm-up outside the capture
-        for L, mu in layers:
-            C.catq_ternary_infer(*L, mu=mu)
+        for group in launches:
+            C.catq_ternary_infer_batched(group, g)
     torch.cuda.current_stream().wait_stream(side)
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(graph):
-        for L, mu in layers:
-            C.catq_ternary_infer(*L, mu=mu)
+        for group in launches:
+            C.catq_ternary_infer_batched(group, g)
     for _ in range(3):
         graph.replay()
     torch.cuda.synchronize()
@@ -592,10 +603,10 @@ def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20, with_m
         raise SystemExit(f"device status {C.STATUS.get(status, status)} in the decode timing")
     ms = a.elapsed_time(b) / steps
     gbs = nbytes / (ms * 1e-3) / 1e9
-    del graph, layers
+    del graph, launches
     torch.cuda.empty_cache()
-    return {"kernel": "ternary_mma_kernel (catq_ternary_infer)", "blocks": blocks, "token_rows": rows,
-            "launches_per_step": blocks * len(wl.linears), "bytes_per_step": nbytes, "us_per_step": ms * 1e3,
+    return {"kernel": "ternary_mma_kernel (catq_ternary_infer_batched)", "blocks": blocks, "token_rows": rows,
+            "launches_per_step": blocks * len(DECODE_GROUPS), "bytes_per_step": nbytes, "us_per_step": ms * 1e3,
             "value": gbs, "unit": "GB/s", "peak": peaks["hbm"], "frac_of_hbm": gbs / peaks["hbm"],
             "steps": steps, "graph": True, "with_mu": with_mu}
 

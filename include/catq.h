@@ -441,6 +441,32 @@ catq_status catq_ternary_infer(const uint8_t* codes, const float* alpha, const f
                                int32_t g, const void* X, int64_t B, int32_t x_dtype, void* Y,
                                catq_stream stream);
 
+/* One layer of catq_ternary_infer_batched (device pointers owned by the caller, layouts as in
+ * catq_ternary_infer). */
+typedef struct {
+  const uint8_t* codes; /* [N*K/4], 16-byte aligned */
+  const float* alpha;   /* [N*K/g] */
+  const float* mu;      /* [N*K/g] or NULL; NULL for every layer or for none */
+  int64_t N, K;
+  const void* X;        /* [B, K] bf16, 16-byte aligned */
+  void* Y;              /* [B, N] bf16 */
+} catq_infer_layer;
+
+/* Maximum layers of one catq_ternary_infer_batched call. */
+int32_t catq_ternary_infer_max_layers(void);
+
+/* catq_ternary_infer for several layers of group size g and B token rows in one persistent
+ * launch (this library's addition; the paper's deployment runs layers one by one).  Each
+ * layer's Y depends only on its own codes, scales and X, so the layers must be independent of
+ * each other within the call (e.g. the q, k and v projections of a block, or gate and up):
+ * no layer's X may be another's Y.  The launch walks every layer's 16-row blocks as one
+ * stream of code slabs, so the next block's codes load while the current one computes.
+ * layers: HOST array of n_layers entries, 1 <= n_layers <= catq_ternary_infer_max_layers().
+ * Errors as catq_ternary_infer for each layer; mixing layers with and without mu is
+ * CATQ_ERR_INVALID_ARG. */
+catq_status catq_ternary_infer_batched(const catq_infer_layer* layers, int32_t n_layers, int32_t g, int64_t B,
+                                       int32_t x_dtype, catq_stream stream);
+
 /* Self-test of the device-side failure detection (no counterpart in the paper): launches
  * one thread that waits, through the library's bounded mbarrier wait, on a barrier nothing
  * arrives on.  After timeout_ns (1 us .. 1 s) the wait gives up, latches CATQ_ERR_TIMEOUT

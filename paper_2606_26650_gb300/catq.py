@@ -59,6 +59,11 @@ class catq_schedule(ctypes.Structure):
     _fields_ = [("phase", ctypes.c_int32), ("s", ctypes.c_float)]
 
 
+class catq_infer_layer(ctypes.Structure):
+    _fields_ = [("codes", ctypes.c_void_p), ("alpha", ctypes.c_void_p), ("mu", ctypes.c_void_p),
+                ("N", ctypes.c_int64), ("K", ctypes.c_int64), ("X", ctypes.c_void_p), ("Y", ctypes.c_void_p)]
+
+
 class catq_adamw(ctypes.Structure):
     _fields_ = [("beta1", ctypes.c_float), ("beta2", ctypes.c_float), ("eps", ctypes.c_float),
                 ("weight_decay", ctypes.c_float), ("margin", ctypes.c_float)]
@@ -106,6 +111,8 @@ def lib() -> ctypes.CDLL:
         "catq_soft_ternary_linear_fwd_loss": (I32, [LP, catq_schedule, P, I64, I32, P, P, I32, I32, P, P, P, P, S, P]),
         "catq_act_quant_a8": (I32, [P, I64, I64, I32, P, P, P, P]),
         "catq_direct_adamw_step": (I32, [I64, P, P, P, P, P, ctypes.POINTER(catq_adamw), I64, F, P]),
+        "catq_ternary_infer_max_layers": (I32, []),
+        "catq_ternary_infer_batched": (I32, [ctypes.POINTER(catq_infer_layer), I32, I32, I64, I32, P]),
         "catq_group_recon_error": (I32, [LP, P, P]),
         "catq_grouped_fwd_loss_workspace_bytes": (S, [ctypes.POINTER(catq_grouped_layer), P]),
         "catq_grouped_soft_ternary_linear_fwd_loss": (I32, [ctypes.POINTER(catq_grouped_layer), catq_schedule, P, P,
@@ -385,6 +392,31 @@ def catq_ternary_infer(codes, alpha, N: int, K: int, g: int, X, Y, mu=None, stre
     _buf(Y, "Y", B * int(N) * X.element_size(), w)
     _check(lib().catq_ternary_infer(_ptr(codes), _ptr(alpha), _ptr(mu), int(N), int(K), int(g), _ptr(X),
                                     X.shape[0], _dtype_code(X), _ptr(Y), _stream(stream)), "catq_ternary_infer")
+
+
+def catq_ternary_infer_max_layers() -> int:
+    return int(lib().catq_ternary_infer_max_layers())
+
+
+def catq_ternary_infer_batched(layers, g: int, stream=None):
+    """Several independent layers in one launch: `layers` is a list of tuples
+    (codes, alpha, N, K, X, Y, mu) (mu may be None), all with the same token rows X.shape[0]."""
+    w = "catq_ternary_infer_batched"
+    arr = (catq_infer_layer * max(1, len(layers)))()
+    B = layers[0][4].shape[0] if layers else 0
+    for i, (codes, alpha, N, K, X, Y, mu) in enumerate(layers):
+        G = int(N) * int(K) // max(int(g), 1)
+        _buf(codes, "codes", int(N) * int(K) // 4, w)
+        _buf(alpha, "alpha", 4 * G, w)
+        _buf(mu, "mu", 4 * G, w)
+        if X.shape[0] != B:
+            raise ValueError(f"{w}: every layer needs the same token rows ({B})")
+        _buf(X, "X", B * int(K) * X.element_size(), w)
+        _buf(Y, "Y", B * int(N) * X.element_size(), w)
+        arr[i] = catq_infer_layer(codes.data_ptr(), alpha.data_ptr(), mu.data_ptr() if mu is not None else None,
+                                  int(N), int(K), X.data_ptr(), Y.data_ptr())
+    dt = _dtype_code(layers[0][4]) if layers else BF16
+    _check(lib().catq_ternary_infer_batched(arr, len(layers), int(g), int(B), dt, _stream(stream)), w)
 
 
 def catq_schedule_at_epoch(e: int, m: int = 60, gamma: float = 0.8, s0: float = 30.0) -> catq_schedule:

@@ -631,6 +631,32 @@ catq_status catq_ternary_infer(const uint8_t* codes, const float* alpha, const f
       launch_ternary_infer(codes, alpha, mu, N, K, g, X, B, Y, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+int32_t catq_ternary_infer_max_layers(void) { return ternary_infer_max_layers(); }
+
+catq_status catq_ternary_infer_batched(const catq_infer_layer* layers, int32_t n_layers, int32_t g, int64_t B,
+                                       int32_t x_dtype, catq_stream stream) {
+  if (!layers || n_layers < 1 || n_layers > ternary_infer_max_layers()) return CATQ_ERR_INVALID_ARG;
+  if (x_dtype != CATQ_BF16) return CATQ_ERR_DTYPE;
+  if (g < 64 || g % 64 != 0 || B < 0) return CATQ_ERR_SHAPE;
+  InferDesc d[64];
+  const bool with_mu = layers[0].mu != nullptr;
+  for (int32_t i = 0; i < n_layers; ++i) {
+    const catq_infer_layer& L = layers[i];
+    if (!L.codes || !L.alpha) return CATQ_ERR_INVALID_ARG;
+    if ((L.mu != nullptr) != with_mu) return CATQ_ERR_INVALID_ARG;
+    if (L.N < 1 || L.K < 1 || L.K % g != 0) return CATQ_ERR_SHAPE;
+    if (L.N * L.K / g >= (int64_t(1) << 31) || L.N >= (int64_t(1) << 31) || L.K >= (int64_t(1) << 31))
+      return CATQ_ERR_SHAPE;
+    if (B > 0 && (!L.X || !L.Y)) return CATQ_ERR_INVALID_ARG;
+    if (!aligned16(L.codes) || (B > 0 && !aligned16(L.X)) || (reinterpret_cast<uintptr_t>(L.alpha) & 3u) != 0 ||
+        (reinterpret_cast<uintptr_t>(L.mu) & 3u) != 0 || (reinterpret_cast<uintptr_t>(L.Y) & 1u) != 0)
+      return CATQ_ERR_ALIGN;
+    d[i] = InferDesc{L.codes, L.alpha, L.mu, L.N, L.K, L.X, B, L.Y};
+  }
+  if (B == 0) return CATQ_OK;
+  return cuda_status(launch_ternary_infer_batched(d, n_layers, g, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 catq_status catq_schedule_at_epoch(int32_t e, int32_t m, double gamma, double s0, catq_schedule* out) {
   if (!out || m < 1 || e < 0 || e > m) return CATQ_ERR_INVALID_ARG;
   if (!(gamma > 0.0 && gamma <= 1.0) || !(s0 > 0.0) || !std::isfinite(s0)) return CATQ_ERR_INVALID_ARG;

@@ -69,6 +69,18 @@ struct EpiOpts {
 // offsets (bf16 X and Y).
 cudaError_t launch_ternary_infer(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K,
                                  int32_t g, const void* X, int64_t B, void* Y, cudaStream_t st);
+// Several layers of one group size in one persistent launch (at most ternary_infer_max_layers()).
+struct InferDesc {
+  const uint8_t* codes;
+  const float* alpha;
+  const float* mu;
+  int64_t N, K;
+  const void* X;
+  int64_t B;
+  void* Y;
+};
+int ternary_infer_max_layers();
+cudaError_t launch_ternary_infer_batched(const InferDesc* layers, int n, int32_t g, cudaStream_t st);
 
 // Wait control (abort word, status word, epoch, time limit) for one launch of a kernel with
 // bounded waits; false when the device's status words are unavailable.

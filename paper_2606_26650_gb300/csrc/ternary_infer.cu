@@ -25,11 +25,14 @@
 // {2q, 2q+1, 2q+8, 2q+9} are two positions of its own code word (lower and upper half), and
 // its B rows are the activations of exactly those columns.
 //
-// A CTA of 8 warps owns 16 R rows.  Its codes come in by bulk copies into shared memory, all
-// at once when they fit (so the whole layer is in flight from the first cycles), else in K
-// slabs through two buffers.  The warps split K into contiguous ranges, and their partial
-// sums meet in shared memory in a fixed order (deterministic).  Token rows are taken 8 at a
-// time (the MMA's N); all arithmetic after the MMAs is fp32, with one rounding of Y.
+// A launch covers one or several layers (independent of each other).  Its work items are
+// blocks of 16 R rows of a layer; a persistent CTA of 8 warps takes every gridDim-th item and
+// streams their codes, in K slabs, through two shared-memory buffers by bulk copies, the next
+// slab (of this item or the next) on its way while the current one is computed.  The warps
+// split each slab into contiguous K ranges, and their partial sums meet in shared memory in a
+// fixed order (deterministic).  Token rows are taken 8 at a time (the MMA's N); all
+// arithmetic after the MMAs is fp32, with one rounding of Y.
+#include <algorithm>
 #include <cstdint>
 #include <type_traits>
 
@@ -131,195 +134,283 @@ __device__ __forceinline__ void drain_wait(uint32_t bar, uint32_t parity) {
     if (globaltimer_ns() - t0 > 200000000ull) return;
 }
 
-// R: 16-row tiles per CTA.  VW: code words per thread per super-chunk (a super-chunk is
+// One layer of a launch: its buffers, shape and code slabs (KS columns per slab, nslabs per
+// token block), its group count per row, and its first work item.
+struct InferLayer {
+  const uint8_t* codes;
+  const float* alpha;
+  const float* mu;
+  const uint16_t* X;
+  uint16_t* Y;
+  int64_t N, K, B;
+  int32_t gpr;     // groups per row, K / g
+  int32_t KS;      // code columns per slab (a multiple of 64 VW)
+  int32_t nslabs;  // slabs per token block
+  int32_t item0;   // first work item of this layer
+};
+
+constexpr int kMaxInferLayers = 16;
+
+struct InferArgs {
+  int32_t n_layers;
+  int32_t total_items;  // work items (16 R-row blocks) over all layers
+  int32_t g;
+  int32_t pad_;
+  InferLayer L[kMaxInferLayers];
+};
+
+// A position in a CTA's stream of code slabs: work item t (a block of 16 R rows of layer l),
+// token block b0 and slab.  Work items run t = blockIdx.x, blockIdx.x + gridDim.x, ...
+struct Cursor {
+  int32_t t, l, slab;
+  int64_t b0;
+};
+
+__device__ __forceinline__ void cursor_at(Cursor& c, int32_t t, const InferArgs& a) {
+  c.t = t;
+  c.slab = 0;
+  c.b0 = 0;
+  c.l = 0;
+  if (t >= a.total_items) return;
+  int lo = 0, hi = a.n_layers;  // last layer whose first item is <= t
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (a.L[mid].item0 <= t) lo = mid;
+    else hi = mid;
+  }
+  c.l = lo;
+}
+
+__device__ __forceinline__ void cursor_next(Cursor& c, const InferArgs& a) {
+  const InferLayer& L = a.L[c.l];
+  if (++c.slab < L.nslabs) return;
+  c.slab = 0;
+  c.b0 += 8;
+  if (c.b0 < L.B) return;
+  cursor_at(c, c.t + static_cast<int32_t>(gridDim.x), a);
+}
+
+// R: 16-row tiles per work item.  VW: code words per thread per super-chunk (a super-chunk is
 // 64 VW columns and lies in one group).  MU: add mu times each group's activation sum.
-// The CTA's codes arrive by bulk copies (one per row and K slab of KS columns) into a ring
-// of one or two slab buffers; each row's copy lands at a stride padded by 16 VW bytes, so
-// the fragment reads (four lanes per row, eight rows per instruction) are free of bank
-// conflicts.
+// A persistent CTA walks its work items (over every layer of the launch) as one stream of
+// code slabs through two shared-memory buffers: warp 0 issues the bulk copies of slab c + 2 as
+// soon as slab c has been consumed, whichever item and layer it belongs to, so the next
+// item's codes are on their way while this one finishes its slabs and its reduction.  Each
+// row's copy lands at a stride padded by 16 VW bytes, so the fragment reads (four lanes per
+// row, eight rows per instruction) are free of bank conflicts.
 template <int R, int VW, bool MU>
-__global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const uint8_t* __restrict__ codes,
-                                                                     const float* __restrict__ alpha,
-                                                                     const float* __restrict__ mu, int64_t N,
-                                                                     int64_t K, int32_t g, int64_t KS,
-                                                                     const uint16_t* __restrict__ X, int64_t B,
-                                                                     uint16_t* __restrict__ Y, const WaitCtl wc) {
+__global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const __grid_constant__ InferArgs a,
+                                                                     int32_t buf_bytes, const WaitCtl wc) {
   constexpr int ROWS = 16 * R;
   extern __shared__ __align__(128) uint8_t ring[];
   __shared__ float red[kMmaWarps][8][ROWS];
   __shared__ __align__(8) uint64_t full_bar[2];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gid = lane >> 2, q = lane & 3;
-  const uint32_t row_bytes = static_cast<uint32_t>(KS / 4 + 16 * VW);
   const uint32_t ring_base = smem_u32(ring);
   const uint32_t bar0 = smem_u32(&full_bar[0]);
-  // column and group counts fit 32 bits (K < 2^31, N K / g < 2^31)
-  const int32_t nslabs = static_cast<int32_t>((K + KS - 1) / KS);
-  const int32_t sc_per_slab = static_cast<int32_t>(KS / (64 * VW));
-  const int32_t sc_per_group = g / (64 * VW);
-  const int32_t gpr = static_cast<int32_t>(K / g);
-  const int64_t nblocks = (N + ROWS - 1) / ROWS;
+  const int32_t sc_per_group = a.g / (64 * VW);
   if (threadIdx.x == 0) {
     mbar_init(bar0, 1);
     mbar_init(bar0 + 8, 1);
     fence_mbar_init_cluster();
   }
   __syncthreads();
-  uint32_t uses = 0;  // completed phases of both barriers, bit b for barrier b (CTA-uniform)
   const uint32_t magic = magic_reg();
 
-  // Warp 0 issues the bulk copies of slab `slab` of rows n0.. into buffer `buf`.
-  auto issue = [&](int64_t n0, int64_t slab, int buf) {
-    const int64_t k0 = slab * KS;
-    const uint32_t bytes = static_cast<uint32_t>((K - k0 < KS ? K - k0 : KS) / 4);
-    const int nvalid = static_cast<int>(N - n0 < ROWS ? N - n0 : ROWS);
+  // Warp 0 issues the bulk copies of the slab at cursor c into buffer `buf`.
+  auto issue = [&](const Cursor& c, int buf) {
+    const InferLayer& L = a.L[c.l];
+    const int64_t n0 = static_cast<int64_t>(c.t - L.item0) * ROWS;
+    const int64_t k0 = static_cast<int64_t>(c.slab) * L.KS;
+    const uint32_t bytes = static_cast<uint32_t>((L.K - k0 < L.KS ? L.K - k0 : L.KS) / 4);
+    const uint32_t row_bytes = static_cast<uint32_t>(L.KS / 4 + 16 * VW);
+    const int nvalid = static_cast<int>(L.N - n0 < ROWS ? L.N - n0 : ROWS);
     const uint32_t bar = bar0 + 8u * buf;
     if (lane == 0) mbar_arrive_expect_tx(bar, bytes * nvalid);
     __syncwarp();
     for (int r = lane; r < nvalid; r += 32)
-      bulk_load_g2s(ring_base + (buf * ROWS + r) * row_bytes, codes + (n0 + r) * (K / 4) + k0 / 4, bytes, bar);
+      bulk_load_g2s(ring_base + buf * buf_bytes + r * row_bytes, L.codes + (n0 + r) * (L.K / 4) + k0 / 4, bytes,
+                    bar);
   };
 
+  // The next kernel of the stream may launch now (it waits for this one before it touches
+  // anything this one writes).  The codes, scales and offsets are weights that inference
+  // never writes, so the first slabs' copies go out before waiting for the previous kernel,
+  // whose output may be this launch's X (or whose input may alias this launch's Y).
+  grid_launch_dependents();
+  Cursor iss, con;
+  cursor_at(iss, blockIdx.x, a);
+  cursor_at(con, blockIdx.x, a);
+  uint32_t issued = 0;  // slabs issued (tracked by warp 0, which issues them)
+  if (warp == 0) {
+    for (int b = 0; b < 2 && iss.t < a.total_items; ++b) {
+      issue(iss, b);
+      cursor_next(iss, a);
+      ++issued;
+    }
+  }
+  grid_dependency_wait();
+  uint32_t qn = 0;  // slabs consumed
   bool ok = true;
-  for (int64_t rb = blockIdx.x; ok && rb < nblocks; rb += gridDim.x) {
-    const int64_t n0 = rb * ROWS;
-    int32_t goff[R][2];  // group-array offsets of this thread's two rows of each tile (rows
-                         // past N take row N - 1's, and are not stored)
+  int32_t goff[R][2];
+  const uint16_t* xrow = nullptr;
+  float acc[R][4], d[R][4], da[4];
+
+  while (ok && con.t < a.total_items) {
+    const InferLayer& L = a.L[con.l];
+    const int64_t n0 = static_cast<int64_t>(con.t - L.item0) * ROWS;
+    if (con.slab == 0) {
+      // a new token block of this item: group offsets of the thread's rows (rows past N take
+      // row N - 1's and are not stored), accumulators, and the activation row (token columns
+      // past B read token b0's activations: their sums are computed and never stored)
 #pragma unroll
-    for (int r = 0; r < R; ++r)
+      for (int r = 0; r < R; ++r)
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int64_t n = n0 + 16 * r + gid + 8 * h;
-        goff[r][h] = static_cast<int32_t>((n < N ? n : N - 1) * gpr);
-      }
-    for (int64_t b0 = 0; ok && b0 < B; b0 += 8) {
-      if (warp == 0) {
-        issue(n0, 0, 0);
-        if (nslabs > 1) issue(n0, 1, 1);
-      }
-      // Token columns past B read token b0's activations instead: their sums are computed
-      // and never stored, so no load needs a predicate.
-      const uint16_t* xrow = X + (b0 + gid < B ? b0 + gid : b0) * K;
-      float acc[R][4], d[R][4], da[4];
+        for (int h = 0; h < 2; ++h) {
+          const int64_t n = n0 + 16 * r + gid + 8 * h;
+          goff[r][h] = static_cast<int32_t>((n < L.N ? n : L.N - 1) * L.gpr);
+        }
+      xrow = L.X + (con.b0 + gid < L.B ? con.b0 + gid : con.b0) * L.K;
 #pragma unroll
       for (int r = 0; r < R; ++r)
 #pragma unroll
         for (int e = 0; e < 4; ++e) acc[r][e] = d[r][e] = 0.0f;
 #pragma unroll
       for (int e = 0; e < 4; ++e) da[e] = 0.0f;
-
-      for (int32_t slab = 0; slab < nslabs; ++slab) {
-        const int buf = slab & 1;
-        const bool landed = mbar_wait(bar0 + 8u * buf, (uses >> buf) & 1u, wc);
-        if (!__syncthreads_and(landed)) {
-          // copies into this buffer, and the next slab's into the other, may still be in flight
-          if (threadIdx.x == 0) {
-            drain_wait(bar0 + 8u * buf, (uses >> buf) & 1u);
-            if (slab + 1 < nslabs) drain_wait(bar0 + 8u * (buf ^ 1), (uses >> (buf ^ 1)) & 1u);
-          }
-          __syncthreads();
-          ok = false;
-          break;
-        }
-        uses ^= 1u << buf;
-        // this warp's contiguous range of the slab's super-chunks, and the group it starts in
-        const int32_t k0 = slab * static_cast<int32_t>(KS);
-        const int32_t n_sc = static_cast<int32_t>(((K - k0 < KS) ? K - k0 : KS) / (64 * VW));
-        const int32_t lo = n_sc * warp / kMmaWarps, hi = n_sc * (warp + 1) / kMmaWarps;
-        int32_t grp = (slab * sc_per_slab + lo) / sc_per_group;
-        int32_t left = (grp + 1) * sc_per_group - (slab * sc_per_slab + lo);  // super-chunks to its end
-        const uint32_t tile = ring_base + buf * ROWS * row_bytes;
-        // per-thread bases, advanced by the super-chunk index inside the loop
-        uint32_t rowa[R][2];  // shared-memory address of the thread's words in each of its rows
+    }
+    const int buf = qn & 1;
+    const bool landed = mbar_wait(bar0 + 8u * buf, (qn >> 1) & 1u, wc);
+    if (!__syncthreads_and(landed)) {
+      // copies into this buffer, and the next slab's into the other, may still be in flight
+      if (threadIdx.x == 0) {
+        drain_wait(bar0 + 8u * buf, (qn >> 1) & 1u);
+        if (issued > qn + 1) drain_wait(bar0 + 8u * (buf ^ 1), ((qn + 1) >> 1) & 1u);
+      }
+      __syncthreads();
+      ok = false;
+      break;
+    }
+    {
+      // this warp's contiguous range of the slab's super-chunks, and the group it starts in
+      const int32_t sc_per_slab = L.KS / (64 * VW);
+      const int32_t k0 = con.slab * L.KS;
+      const int32_t n_sc = static_cast<int32_t>(((L.K - k0 < L.KS) ? L.K - k0 : L.KS) / (64 * VW));
+      const int32_t lo = n_sc * warp / kMmaWarps, hi = n_sc * (warp + 1) / kMmaWarps;
+      int32_t grp = (con.slab * sc_per_slab + lo) / sc_per_group;
+      int32_t left = (grp + 1) * sc_per_group - (con.slab * sc_per_slab + lo);  // super-chunks to its end
+      const uint32_t row_bytes = static_cast<uint32_t>(L.KS / 4 + 16 * VW);
+      const uint32_t tile = ring_base + buf * buf_bytes;
+      uint32_t rowa[R][2];  // shared-memory address of the thread's words in each of its rows
 #pragma unroll
-        for (int r = 0; r < R; ++r)
+      for (int r = 0; r < R; ++r)
 #pragma unroll
-          for (int h = 0; h < 2; ++h) rowa[r][h] = tile + (16 * r + gid + 8 * h) * row_bytes + VW * q * 4;
-        const uint4* xbase = reinterpret_cast<const uint4*>(xrow + k0 + 16 * VW * q);
-        const bool every_sc = sc_per_group == 1;  // each super-chunk is a whole group
-        auto load_x = [&](int32_t sc, uint4 (&xv)[2 * VW]) {
-          const uint4* xp = xbase + sc * (8 * VW);
+        for (int h = 0; h < 2; ++h) rowa[r][h] = tile + (16 * r + gid + 8 * h) * row_bytes + VW * q * 4;
+      const uint4* xbase = reinterpret_cast<const uint4*>(xrow + k0 + 16 * VW * q);
+      const bool every_sc = sc_per_group == 1;  // each super-chunk is a whole group
+      const float* alpha = L.alpha;
+      const float* mu = L.mu;
+      auto load_x = [&](int32_t sc, uint4 (&xv)[2 * VW]) {
+        const uint4* xp = xbase + sc * (8 * VW);
 #pragma unroll
-          for (int i = 0; i < 2 * VW; ++i) xv[i] = __ldg(xp + i);
-        };
-        // one super-chunk: this thread's code words from shared memory, its activations xv
-        auto step = [&](int32_t sc, const uint4 (&xv)[2 * VW]) {
-          const uint32_t woff = static_cast<uint32_t>(sc * 16 * VW);
-          uint32_t cw[R][2][VW];  // the thread's code words of rows gid and gid + 8 of each tile
+        for (int i = 0; i < 2 * VW; ++i) xv[i] = __ldg(xp + i);
+      };
+      // one super-chunk: this thread's code words from shared memory, its activations xv
+      auto step = [&](int32_t sc, const uint4 (&xv)[2 * VW]) {
+        const uint32_t woff = static_cast<uint32_t>(sc * 16 * VW);
+        // The group (or this warp's range) ends with this super-chunk: its scales (and offsets)
+        // are requested before the MMAs, which then cover their latency.
+        const bool ends = every_sc || left == 1 || sc + 1 == hi;
+        float av[R][2], mv[R][2];
+        if (ends) {
 #pragma unroll
           for (int r = 0; r < R; ++r) {
-            ld_shared_words<VW>(rowa[r][0] + woff, cw[r][0]);
-            ld_shared_words<VW>(rowa[r][1] + woff, cw[r][1]);
-          }
-#pragma unroll
-          for (int v = 0; v < VW; ++v) {
-            uint32_t xb[8];
-            const uint4 h0 = xv[2 * v], h1 = xv[2 * v + 1];
-            xb[0] = act_pair<0>(h0, h1);
-            xb[1] = act_pair<1>(h0, h1);
-            xb[2] = act_pair<2>(h0, h1);
-            xb[3] = act_pair<3>(h0, h1);
-            xb[4] = act_pair<4>(h0, h1);
-            xb[5] = act_pair<5>(h0, h1);
-            xb[6] = act_pair<6>(h0, h1);
-            xb[7] = act_pair<7>(h0, h1);
-            // rows 0..7 of the constant tile: the correction sums; rows 8..15: activation sums
-            mma_16816(da, pos_corr(0), pos_unit(0), pos_corr(1), pos_unit(1), xb[0], xb[1]);
-            mma_16816(da, pos_corr(2), pos_unit(2), pos_corr(3), pos_unit(3), xb[2], xb[3]);
-            mma_16816(da, pos_corr(4), pos_unit(4), pos_corr(5), pos_unit(5), xb[4], xb[5]);
-            mma_16816(da, pos_corr(6), pos_unit(6), pos_corr(7), pos_unit(7), xb[6], xb[7]);
-#pragma unroll
-            for (int r = 0; r < R; ++r) {
-              const Shifted s0 = shifted(cw[r][0][v], magic), s1 = shifted(cw[r][1][v], magic);
-              word_mma<0>(d[r], s0, s1, xb);
-              word_mma<1>(d[r], s0, s1, xb);
-              word_mma<2>(d[r], s0, s1, xb);
-              word_mma<3>(d[r], s0, s1, xb);
+            av[r][0] = __ldg(alpha + goff[r][0] + grp);
+            av[r][1] = __ldg(alpha + goff[r][1] + grp);
+            if constexpr (MU) {
+              mv[r][0] = __ldg(mu + goff[r][0] + grp);
+              mv[r][1] = __ldg(mu + goff[r][1] + grp);
             }
           }
-          if (every_sc || --left == 0 || sc + 1 == hi) {  // the group, or this warp's range, ends
-#pragma unroll
-            for (int r = 0; r < R; ++r) {
-              const float a0 = __ldg(alpha + goff[r][0] + grp), a1 = __ldg(alpha + goff[r][1] + grp);
-              acc[r][0] = fmaf(a0, d[r][0] - da[0], acc[r][0]);
-              acc[r][1] = fmaf(a0, d[r][1] - da[1], acc[r][1]);
-              acc[r][2] = fmaf(a1, d[r][2] - da[0], acc[r][2]);
-              acc[r][3] = fmaf(a1, d[r][3] - da[1], acc[r][3]);
-              if constexpr (MU) {
-                const float m0 = __ldg(mu + goff[r][0] + grp), m1 = __ldg(mu + goff[r][1] + grp);
-                acc[r][0] = fmaf(m0, da[2], acc[r][0]);
-                acc[r][1] = fmaf(m0, da[3], acc[r][1]);
-                acc[r][2] = fmaf(m1, da[2], acc[r][2]);
-                acc[r][3] = fmaf(m1, da[3], acc[r][3]);
-              }
-#pragma unroll
-              for (int e = 0; e < 4; ++e) d[r][e] = 0.0f;
-            }
-#pragma unroll
-            for (int e = 0; e < 4; ++e) da[e] = 0.0f;
-            if (every_sc) {
-              ++grp;
-            } else if (left == 0) {
-              ++grp;
-              left = sc_per_group;
-            }
-          }
-        };
-        // activations one super-chunk ahead, in two alternating register sets
-        uint4 xa[2 * VW], xc[2 * VW];
-        if (lo < hi) load_x(lo, xa);
-        for (int32_t sc = lo; sc < hi; sc += 2) {
-          if (sc + 1 < hi) load_x(sc + 1, xc);
-          step(sc, xa);
-          if (sc + 1 >= hi) break;
-          if (sc + 2 < hi) load_x(sc + 2, xa);
-          step(sc + 1, xc);
         }
-        __syncthreads();  // every warp is done with this buffer
-        if (warp == 0 && slab + 2 < nslabs) issue(n0, slab + 2, buf);
+        uint32_t cw[R][2][VW];  // the thread's code words of rows gid and gid + 8 of each tile
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+          ld_shared_words<VW>(rowa[r][0] + woff, cw[r][0]);
+          ld_shared_words<VW>(rowa[r][1] + woff, cw[r][1]);
+        }
+#pragma unroll
+        for (int v = 0; v < VW; ++v) {
+          uint32_t xb[8];
+          const uint4 h0 = xv[2 * v], h1 = xv[2 * v + 1];
+          xb[0] = act_pair<0>(h0, h1);
+          xb[1] = act_pair<1>(h0, h1);
+          xb[2] = act_pair<2>(h0, h1);
+          xb[3] = act_pair<3>(h0, h1);
+          xb[4] = act_pair<4>(h0, h1);
+          xb[5] = act_pair<5>(h0, h1);
+          xb[6] = act_pair<6>(h0, h1);
+          xb[7] = act_pair<7>(h0, h1);
+          // rows 0..7 of the constant tile: the correction sums; rows 8..15: activation sums
+          mma_16816(da, pos_corr(0), pos_unit(0), pos_corr(1), pos_unit(1), xb[0], xb[1]);
+          mma_16816(da, pos_corr(2), pos_unit(2), pos_corr(3), pos_unit(3), xb[2], xb[3]);
+          mma_16816(da, pos_corr(4), pos_unit(4), pos_corr(5), pos_unit(5), xb[4], xb[5]);
+          mma_16816(da, pos_corr(6), pos_unit(6), pos_corr(7), pos_unit(7), xb[6], xb[7]);
+#pragma unroll
+          for (int r = 0; r < R; ++r) {
+            const Shifted s0 = shifted(cw[r][0][v], magic), s1 = shifted(cw[r][1][v], magic);
+            word_mma<0>(d[r], s0, s1, xb);
+            word_mma<1>(d[r], s0, s1, xb);
+            word_mma<2>(d[r], s0, s1, xb);
+            word_mma<3>(d[r], s0, s1, xb);
+          }
+        }
+        if (ends) {
+#pragma unroll
+          for (int r = 0; r < R; ++r) {
+            acc[r][0] = fmaf(av[r][0], d[r][0] - da[0], acc[r][0]);
+            acc[r][1] = fmaf(av[r][0], d[r][1] - da[1], acc[r][1]);
+            acc[r][2] = fmaf(av[r][1], d[r][2] - da[0], acc[r][2]);
+            acc[r][3] = fmaf(av[r][1], d[r][3] - da[1], acc[r][3]);
+            if constexpr (MU) {
+              acc[r][0] = fmaf(mv[r][0], da[2], acc[r][0]);
+              acc[r][1] = fmaf(mv[r][0], da[3], acc[r][1]);
+              acc[r][2] = fmaf(mv[r][1], da[2], acc[r][2]);
+              acc[r][3] = fmaf(mv[r][1], da[3], acc[r][3]);
+            }
+#pragma unroll
+            for (int e = 0; e < 4; ++e) d[r][e] = 0.0f;
+          }
+#pragma unroll
+          for (int e = 0; e < 4; ++e) da[e] = 0.0f;
+        }
+        if (every_sc) {
+          ++grp;
+        } else if (--left == 0) {
+          ++grp;
+          left = sc_per_group;
+        }
+      };
+      // activations one super-chunk ahead, in two alternating register sets
+      uint4 xa[2 * VW], xc[2 * VW];
+      if (lo < hi) load_x(lo, xa);
+      for (int32_t sc = lo; sc < hi; sc += 2) {
+        if (sc + 1 < hi) load_x(sc + 1, xc);
+        step(sc, xa);
+        if (sc + 1 >= hi) break;
+        if (sc + 2 < hi) load_x(sc + 2, xa);
+        step(sc + 1, xc);
       }
-      if (!ok) break;
-
+    }
+    __syncthreads();  // every warp is done with this buffer: refill it two slabs ahead
+    if (warp == 0 && iss.t < a.total_items) {
+      issue(iss, buf);
+      cursor_next(iss, a);
+      ++issued;
+    }
+    ++qn;
+    if (con.slab + 1 == L.nslabs) {
+      // the token block's last slab: its partial sums meet in shared memory, in a fixed order
       // D fragment: (row gid, tokens 2q, 2q + 1) and (row gid + 8, the same tokens)
 #pragma unroll
       for (int r = 0; r < R; ++r) {
@@ -334,53 +425,103 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const ui
         float s = 0.0f;
 #pragma unroll
         for (int w = 0; w < kMmaWarps; ++w) s += red[w][tok][row];
-        if (b0 + tok < B && n0 + row < N)
-          Y[(b0 + tok) * N + n0 + row] = static_cast<uint16_t>(pack_bf16x2(s, 0.0f) & 0xFFFFu);
+        if (con.b0 + tok < L.B && n0 + row < L.N)
+          L.Y[(con.b0 + tok) * L.N + n0 + row] = static_cast<uint16_t>(pack_bf16x2(s, 0.0f) & 0xFFFFu);
       }
       __syncthreads();
     }
+    cursor_next(con, a);
   }
 }
 
-constexpr int64_t kRingBytes = 72 * 1024;  // code bytes of one slab buffer
+// One slab buffer: two per CTA plus the reduction array fit twice in an SM's shared memory.
+constexpr int64_t kBufBytes = 46 * 1024;
+
+// Bytes of one slab buffer for KS columns: 16 R rows of codes, each padded by 16 VW bytes.
+int64_t slab_bytes(int64_t KS, int R, int VW) { return 16 * R * (KS / 4 + 16 * VW); }
+
+// Code columns per slab for K: all of K when it fits one buffer, else the fewest equal slabs
+// (multiples of 64 VW columns) that do.
+int64_t slab_cols(int64_t K, int R, int VW) {
+  const int64_t unit = 64 * VW;
+  if (slab_bytes(K, R, VW) <= kBufBytes) return K;
+  const int64_t cap = ((kBufBytes / (16 * R) - 16 * VW) * 4) / unit * unit;
+  const int64_t nslabs = (K + cap - 1) / cap;
+  return ((K + nslabs - 1) / nslabs + unit - 1) / unit * unit;
+}
 
 template <int R, int VW>
-cudaError_t launch_mma(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K, int32_t g,
-                       const uint16_t* X, int64_t B, uint16_t* Y, cudaStream_t st) {
+cudaError_t launch_mma(const InferDesc* ls, int n, int32_t g, bool with_mu, cudaStream_t st) {
   WaitCtl wc;
   if (!launch_wait_ctl(&wc)) return cudaErrorInvalidDevice;
-  const int64_t rows = 16 * R;
-  // K slab: all of K when the CTA's rows fit one buffer, else the largest multiple of
-  // 64 VW columns that does (two buffers then alternate).
-  int64_t KS = K;
-  if (rows * (K / 4 + 16 * VW) > kRingBytes) KS = ((kRingBytes / rows - 16 * VW) * 4) / (64 * VW) * (64 * VW);
-  const int64_t nslabs = (K + KS - 1) / KS;
-  const int smem = static_cast<int>((nslabs > 1 ? 2 : 1) * rows * (KS / 4 + 16 * VW));
-  int64_t blocks = (N + rows - 1) / rows;
-  if (blocks > 152 * 16) blocks = 152 * 16;
-  auto kern = mu ? ternary_mma_kernel<R, VW, true> : ternary_mma_kernel<R, VW, false>;
+  InferArgs a{};
+  a.n_layers = n;
+  a.g = g;
+  int64_t items = 0, max_buf = 0;
+  for (int i = 0; i < n; ++i) {
+    InferLayer& L = a.L[i];
+    L.codes = ls[i].codes;
+    L.alpha = ls[i].alpha;
+    L.mu = ls[i].mu;
+    L.X = static_cast<const uint16_t*>(ls[i].X);
+    L.Y = static_cast<uint16_t*>(ls[i].Y);
+    L.N = ls[i].N;
+    L.K = ls[i].K;
+    L.B = ls[i].B;
+    L.gpr = static_cast<int32_t>(ls[i].K / g);
+    const int64_t KS = slab_cols(L.K, R, VW);
+    L.KS = static_cast<int32_t>(KS);
+    L.nslabs = static_cast<int32_t>((L.K + KS - 1) / KS);
+    L.item0 = static_cast<int32_t>(items);
+    items += (L.N + 16 * R - 1) / (16 * R);
+    max_buf = std::max<int64_t>(max_buf, slab_bytes(KS, R, VW));
+  }
+  if (items == 0) return cudaSuccess;
+  if (items >= (int64_t(1) << 31)) return cudaErrorInvalidValue;
+  a.total_items = static_cast<int32_t>(items);
+  const int buf_bytes = static_cast<int>((max_buf + 127) / 128 * 128);
+  const int smem = 2 * buf_bytes;
+  int sm = 152;
+  int dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sm, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t blocks = std::min<int64_t>(items, 2 * static_cast<int64_t>(sm));
+  auto kern = with_mu ? ternary_mma_kernel<R, VW, true> : ternary_mma_kernel<R, VW, false>;
   const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  kern<<<static_cast<int>(blocks), kMmaWarps * 32, smem, st>>>(codes, alpha, mu, N, K, g, KS, X, B, Y, wc);
-  return cudaGetLastError();
+  // programmatic dependent launch: this kernel may start while the previous one in the stream
+  // finishes (see grid_dependency_wait in the kernel)
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>(blocks));
+  cfg.blockDim = dim3(kMmaWarps * 32);
+  cfg.dynamicSmemBytes = static_cast<size_t>(smem);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, a, buf_bytes, wc);
 }
 
 template <int R>
-cudaError_t launch_rows(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K, int32_t g,
-                        const uint16_t* X, int64_t B, uint16_t* Y, cudaStream_t st) {
-  if (g % 128 == 0) return launch_mma<R, 2>(codes, alpha, mu, N, K, g, X, B, Y, st);
-  return launch_mma<R, 1>(codes, alpha, mu, N, K, g, X, B, Y, st);
+cudaError_t launch_rows(const InferDesc* ls, int n, int32_t g, bool with_mu, cudaStream_t st) {
+  if (g % 128 == 0) return launch_mma<R, 2>(ls, n, g, with_mu, st);
+  return launch_mma<R, 1>(ls, n, g, with_mu, st);
 }
 
 }  // namespace
 
-cudaError_t launch_ternary_infer(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K,
-                                 int32_t g, const void* X, int64_t B, void* Y, cudaStream_t st) {
-  const uint16_t* x = static_cast<const uint16_t*>(X);
-  uint16_t* y = static_cast<uint16_t*>(Y);
-  // 16-row tiles per CTA: the fewest rows on the busiest SM (CTAs spread evenly over the
-  // SMs), then the most tiles per CTA (the correction MMAs and the activation preparation
-  // serve more rows), with the CTA's codes within one ring buffer.
+int ternary_infer_max_layers() { return kMaxInferLayers; }
+
+cudaError_t launch_ternary_infer_batched(const InferDesc* ls, int n, int32_t g, cudaStream_t st) {
+  if (n < 1 || n > kMaxInferLayers) return cudaErrorInvalidValue;
+  bool with_mu = ls[0].mu != nullptr;
+  for (int i = 1; i < n; ++i)
+    if ((ls[i].mu != nullptr) != with_mu) return cudaErrorInvalidValue;
+  // 16-row tiles per work item (1 or 2: more hold more registers than two CTAs per SM
+  // allow without spills): the fewest rows on the busiest SM (two persistent CTAs per SM),
+  // then the most tiles per item (the correction MMAs and the activation preparation serve
+  // more rows).
   int sm = 152;
   {
     int dev = 0;
@@ -388,21 +529,23 @@ cudaError_t launch_ternary_infer(const uint8_t* codes, const float* alpha, const
   }
   int best = 1;
   int64_t best_rows = -1;
-  for (int r = 1; r <= 4; ++r) {
-    if (r > 1 && 16 * r * (K / 4 + 32) > kRingBytes) break;
-    const int64_t ctas = (N + 16 * r - 1) / (16 * r);
-    const int64_t busiest = (ctas + sm - 1) / sm * 16 * r;
+  for (int r = 1; r <= 2; ++r) {
+    int64_t items = 0;
+    for (int i = 0; i < n; ++i) items += (ls[i].N + 16 * r - 1) / (16 * r);
+    const int64_t busiest = (items + 2 * sm - 1) / (2 * sm) * 16 * r;
     if (best_rows < 0 || busiest <= best_rows) {
       best = r;
       best_rows = busiest;
     }
   }
-  switch (best) {
-    case 4: return launch_rows<4>(codes, alpha, mu, N, K, g, x, B, y, st);
-    case 3: return launch_rows<3>(codes, alpha, mu, N, K, g, x, B, y, st);
-    case 2: return launch_rows<2>(codes, alpha, mu, N, K, g, x, B, y, st);
-    default: return launch_rows<1>(codes, alpha, mu, N, K, g, x, B, y, st);
-  }
+  if (best == 2) return launch_rows<2>(ls, n, g, with_mu, st);
+  return launch_rows<1>(ls, n, g, with_mu, st);
+}
+
+cudaError_t launch_ternary_infer(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K,
+                                 int32_t g, const void* X, int64_t B, void* Y, cudaStream_t st) {
+  const InferDesc d{codes, alpha, mu, N, K, X, B, Y};
+  return launch_ternary_infer_batched(&d, 1, g, st);
 }
 
 }  // namespace catq

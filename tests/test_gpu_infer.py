@@ -51,3 +51,46 @@ def test_ternary_infer_matches_oracle(device, N, K, g, B):
         assert C.catq_device_status() == 0
         want = O.ternary_infer(U.to_host(codes), U.to_host(alpha), N, K, g, X)
         assert U.fro_rel(U.to_host(Y), want) <= U.TOL_BF16
+
+
+@pytest.mark.parametrize("shapes,g,B,with_mu", [
+    # the q, k, v projections of the Llama-3-8B-shaped block, one token row
+    (((4096, 4096), (1024, 4096), (1024, 4096)), 128, 1, False),
+    # gate and up, then a down-shaped layer with K = 14336 (several slabs) in the same launch
+    (((14336, 4096), (14336, 4096), (4096, 14336)), 128, 8, False),
+    # ragged row counts, two token blocks (8 + 3), the W ~ alpha T + mu form
+    (((520, 192), (328, 1024), (64, 192)), 64, 11, True),
+])
+def test_ternary_infer_batched_matches_oracle(device, shapes, g, B, with_mu):
+    """Several independent layers in one launch: each layer's Y against the oracle on its own
+    codes, scales and X."""
+    import torch
+
+    from paper_2606_26650_gb300 import catq as C
+    layers, want = [], []
+    for i, (N, K) in enumerate(shapes):
+        r = syn.rng(6, f"infer_batched/{i}/{N}/{K}")
+        off = np.repeat(r.uniform(-0.03, 0.03, N * K // g), g).reshape(N, K) if with_mu else 0.0
+        W = syn.round_bf16((r.standard_normal((N, K)) * 0.02 + off).astype(np.float32))
+        X = syn.round_bf16(r.standard_normal((B, K)).astype(np.float32))
+        G = N * K // g
+        fac = syn.factors(G, 6, f"infer_batched/{i}", perturbed=True)
+        layer = C.Layer.create(U.to_device(W, "bf16", device), g, *(torch.from_numpy(f).to(device) for f in fac),
+                               recon=1 if with_mu else 0)
+        C.catq_group_stats(layer)
+        codes = torch.empty(N * K // 4, dtype=torch.uint8, device=device)
+        alpha = torch.empty(G, dtype=torch.float32, device=device)
+        mu = torch.empty(G, dtype=torch.float32, device=device) if with_mu else None
+        C.catq_hard_ternarize_pack(layer, codes, alpha, mu)
+        Xt = U.to_device(X, "bf16", device)
+        Y = torch.empty(B, N, dtype=torch.bfloat16, device=device)
+        layers.append((codes, alpha, N, K, Xt, Y, mu))
+        want.append((X, N, K))
+    for _ in range(2):
+        C.catq_ternary_infer_batched(layers, g)
+        torch.cuda.synchronize()
+        assert C.catq_device_status() == 0
+        for (codes, alpha, N, K, Xt, Y, mu), (X, _, _) in zip(layers, want):
+            ref = O.ternary_infer(U.to_host(codes), U.to_host(alpha), N, K, g, X,
+                                  mu=U.to_host(mu) if mu is not None else None)
+            assert U.fro_rel(U.to_host(Y), ref) <= U.TOL_BF16, (N, K)
