@@ -431,3 +431,146 @@ def group_recon_error(W, g, stats, factors):
     Wq = ternary_weight(W, g, stats, factors, PHASE_HARD, 1.0)[0]
     d = (np.asarray(W, np.float64) - Wq).reshape(-1, g)
     return (d * d).mean(axis=1)
+
+
+# ------------------------------------------------------------------ one decoder block (§2.4)
+# Eq. 7 reconstructs the output of a window of layers.  The window here is one decoder block
+# of the Llama / Qwen family (pre-norm, grouped-query causal attention with rotary position
+# embedding, SwiGLU MLP), all seven linears soft-ternary, the teacher the same block with
+# full-precision weights.  Tokens are rows t = b S + s of a [B S, H] activation.
+
+def rmsnorm(x, gamma, eps):
+    """RMSNorm of each row: y = gamma * x / sqrt(mean(x^2) + eps).  Returns (y, r) with
+    r = 1 / sqrt(mean(x^2) + eps) per row."""
+    x = np.asarray(x, np.float64)
+    r = 1.0 / np.sqrt((x * x).mean(axis=1) + eps)
+    return x * r[:, None] * np.asarray(gamma, np.float64)[None, :], r
+
+
+def rmsnorm_bwd(x, gamma, r, dy):
+    """Gradient of ``rmsnorm`` with respect to x: with u = gamma * dy,
+    dx = r u - x r^3 mean(u x)."""
+    x = np.asarray(x, np.float64)
+    u = np.asarray(dy, np.float64) * np.asarray(gamma, np.float64)[None, :]
+    return r[:, None] * u - x * (r ** 3 * (u * x).mean(axis=1))[:, None]
+
+
+def rope(x, S, n_heads, d, base, inverse=False):
+    """Rotary position embedding of each head of x [B S, n_heads d] (the half-split pairing:
+    element i and i + d/2 of a head rotate together) by the angle s base^(-2i/d) of the
+    token's position s; ``inverse`` rotates back (the gradient of the rotation)."""
+    x = np.asarray(x, np.float64)
+    T = x.shape[0]
+    pos = (np.arange(T) % S).astype(np.float64)
+    inv_freq = base ** (-2.0 * np.arange(d // 2) / d)
+    ang = pos[:, None] * inv_freq[None, :]
+    c, s_ = np.cos(ang)[:, None, :], np.sin(ang)[:, None, :]
+    if inverse:
+        s_ = -s_
+    xh = x.reshape(T, n_heads, d)
+    a, b = xh[..., : d // 2], xh[..., d // 2:]
+    return np.concatenate([a * c - b * s_, a * s_ + b * c], axis=2).reshape(T, n_heads * d)
+
+
+def attention(q, k, v, B, S, nh, nkv, d):
+    """Causal grouped-query attention: head h uses key/value head h // (nh / nkv);
+    O = softmax(Q K^T / sqrt(d), keys <= query) V per batch and head.  Returns (o [B S, nh d],
+    P [B, nh, S, S] the attention probabilities)."""
+    q = np.asarray(q, np.float64).reshape(B, S, nh, d)
+    k = np.asarray(k, np.float64).reshape(B, S, nkv, d)
+    v = np.asarray(v, np.float64).reshape(B, S, nkv, d)
+    rep = nh // nkv
+    kh = np.repeat(k, rep, axis=2)
+    vh = np.repeat(v, rep, axis=2)
+    s = np.einsum("bqhd,bkhd->bhqk", q, kh) / np.sqrt(d)
+    s = np.where(np.tril(np.ones((S, S), bool))[None, None], s, -np.inf)
+    s = s - s.max(axis=3, keepdims=True)
+    p = np.exp(s)
+    p = p / p.sum(axis=3, keepdims=True)
+    o = np.einsum("bhqk,bkhd->bqhd", p, vh)
+    return o.reshape(B * S, nh * d), p
+
+
+def attention_bwd(q, k, v, p, do, B, S, nh, nkv, d):
+    """Gradients of ``attention``: with dS = P (dP - rowsum(dP P)), dP = dO V^T,
+    dQ = dS K / sqrt(d), dK = dS^T Q / sqrt(d), dV = P^T dO, the key/value gradients summed
+    over the heads that share them."""
+    q = np.asarray(q, np.float64).reshape(B, S, nh, d)
+    k = np.asarray(k, np.float64).reshape(B, S, nkv, d)
+    v = np.asarray(v, np.float64).reshape(B, S, nkv, d)
+    do = np.asarray(do, np.float64).reshape(B, S, nh, d)
+    rep = nh // nkv
+    kh = np.repeat(k, rep, axis=2)
+    vh = np.repeat(v, rep, axis=2)
+    dp = np.einsum("bqhd,bkhd->bhqk", do, vh)
+    ds = p * (dp - (dp * p).sum(axis=3, keepdims=True))
+    dq = np.einsum("bhqk,bkhd->bqhd", ds, kh) / np.sqrt(d)
+    dkh = np.einsum("bhqk,bqhd->bkhd", ds, q) / np.sqrt(d)
+    dvh = np.einsum("bhqk,bqhd->bkhd", p, do)
+    dk = dkh.reshape(B, S, nkv, rep, d).sum(axis=3)
+    dv = dvh.reshape(B, S, nkv, rep, d).sum(axis=3)
+    return dq.reshape(B * S, nh * d), dk.reshape(B * S, nkv * d), dv.reshape(B * S, nkv * d)
+
+
+def silu(a):
+    a = np.asarray(a, np.float64)
+    return a / (1.0 + np.exp(-a))
+
+
+BLOCK_LINEARS = ("q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj")
+
+
+def block_forward(x, Wq, gamma1, gamma2, B, S, nh, nkv, d, base, eps):
+    """One decoder block with the effective weights Wq[name] ([N, K] each):
+    z1 = RMSNorm(x); q, k, v = z1 W^T; rotary q, k; a = attention; h = x + a Wo^T;
+    z2 = RMSNorm(h); m = silu(z2 Wg^T) * (z2 Wu^T); out = h + m Wd^T.  Returns (out, cache)."""
+    x = np.asarray(x, np.float64)
+    z1, r1 = rmsnorm(x, gamma1, eps)
+    q = rope(linear_fwd(z1, Wq["q_proj"]), S, nh, d, base)
+    k = rope(linear_fwd(z1, Wq["k_proj"]), S, nkv, d, base)
+    v = linear_fwd(z1, Wq["v_proj"])
+    a, p = attention(q, k, v, B, S, nh, nkv, d)
+    h = x + linear_fwd(a, Wq["o_proj"])
+    z2, r2 = rmsnorm(h, gamma2, eps)
+    gt = linear_fwd(z2, Wq["gate_proj"])
+    u = linear_fwd(z2, Wq["up_proj"])
+    m = silu(gt) * u
+    out = h + linear_fwd(m, Wq["down_proj"])
+    return out, dict(z1=z1, q=q, k=k, v=v, a=a, p=p, h=h, z2=z2, r2=r2, gt=gt, u=u, m=m)
+
+
+def block_calibration_step(x, W, g, stats, factors, gamma1, gamma2, B, S, nh, nkv, d, base, eps, phase, s,
+                           reduction=0):
+    """One calibration step of a window of one decoder block (Eq. 7 over the block output):
+    the teacher block with full-precision weights, the block with each linear's Eq. 6 weight
+    (W, stats, factors: dicts by linear name), the loss, and every linear's factor gradients
+    through the block's backward.  The block input is fixed (the window's input), so no
+    gradient flows into x.  Returns a dict: out, out_ref, loss, and g[name] = (g_dmu,
+    g_dalpha, g_ddelta)."""
+    Wq = {n: ternary_weight(W[n], g, stats[n], factors[n], phase, s)[0] for n in BLOCK_LINEARS}
+    out_ref, _ = block_forward(x, {n: np.asarray(W[n], np.float64) for n in BLOCK_LINEARS}, gamma1, gamma2, B,
+                               S, nh, nkv, d, base, eps)
+    out, c = block_forward(x, Wq, gamma1, gamma2, B, S, nh, nkv, d, base, eps)
+    loss, d_out = recon_loss(out, out_ref, reduction)
+    G = {}
+
+    def grads(name, X, dY):
+        G[name] = factor_grads_from_G(np.asarray(dY).T @ np.asarray(X), W[name], g, stats[name], factors[name],
+                                      phase, s)
+
+    grads("down_proj", c["m"], d_out)
+    dm = d_out @ Wq["down_proj"]
+    sg = 1.0 / (1.0 + np.exp(-c["gt"]))
+    d_gt = dm * c["u"] * sg * (1.0 + c["gt"] * (1.0 - sg))
+    d_u = dm * silu(c["gt"])
+    grads("gate_proj", c["z2"], d_gt)
+    grads("up_proj", c["z2"], d_u)
+    dz2 = d_gt @ Wq["gate_proj"] + d_u @ Wq["up_proj"]
+    dh = d_out + rmsnorm_bwd(c["h"], gamma2, c["r2"], dz2)
+    grads("o_proj", c["a"], dh)
+    da = dh @ Wq["o_proj"]
+    dq, dk, dv = attention_bwd(c["q"], c["k"], c["v"], c["p"], da, B, S, nh, nkv, d)
+    grads("q_proj", c["z1"], rope(dq, S, nh, d, base, inverse=True))
+    grads("k_proj", c["z1"], rope(dk, S, nkv, d, base, inverse=True))
+    grads("v_proj", c["z1"], dv)
+    return dict(out=out, out_ref=out_ref, loss=loss, g=G, cache=c)

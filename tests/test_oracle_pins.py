@@ -882,3 +882,139 @@ def test_group_recon_error_closed_form():
     stats = O.group_stats(W, 4, O.THR_ABSMEAN)
     fac = (np.zeros(1), np.ones(1), np.ones(1))
     assert O.group_recon_error(W, 4, stats, fac)[0] == pytest.approx(v * v, rel=1e-12)
+
+
+# ----------------------------------------------------------------- one decoder block (§2.4, Eq. 7)
+
+def _tiny_block(seed=80, B=2, S=5, nh=4, nkv=2, d=4, I=12, g=4):
+    r = np.random.default_rng(seed)
+    H = nh * d
+    shapes = {"q_proj": (nh * d, H), "k_proj": (nkv * d, H), "v_proj": (nkv * d, H), "o_proj": (H, nh * d),
+              "gate_proj": (I, H), "up_proj": (I, H), "down_proj": (H, I)}
+    W = {n: r.standard_normal(sh) * 0.3 for n, sh in shapes.items()}
+    stats = {n: O.group_stats(W[n], g) for n in shapes}
+    fac = {n: (r.uniform(-0.1, 0.1, W[n].size // g), r.uniform(0.8, 1.2, W[n].size // g),
+               r.uniform(0.8, 1.2, W[n].size // g)) for n in shapes}
+    x = r.standard_normal((B * S, H))
+    gamma1 = r.uniform(0.5, 1.5, H)
+    gamma2 = r.uniform(0.5, 1.5, H)
+    return dict(x=x, W=W, g=g, stats=stats, fac=fac, gamma1=gamma1, gamma2=gamma2, B=B, S=S, nh=nh, nkv=nkv,
+                d=d, base=10000.0, eps=1e-5)
+
+
+def _block_loss(blk, fac, s):
+    return O.block_calibration_step(blk["x"], blk["W"], blk["g"], blk["stats"], fac, blk["gamma1"], blk["gamma2"],
+                                    blk["B"], blk["S"], blk["nh"], blk["nkv"], blk["d"], blk["base"], blk["eps"],
+                                    O.PHASE_SOFT, s)["loss"]
+
+
+def test_block_factor_gradients_match_central_differences():
+    """The block's backward (SwiGLU, RMSNorm with the residual, attention with grouped heads,
+    rotary embedding, every linear's chain rule) against central differences of the block
+    loss, for sampled groups of every linear and all three factors, soft phase."""
+    blk = _tiny_block()
+    s = 3.0
+    step = O.block_calibration_step(blk["x"], blk["W"], blk["g"], blk["stats"], blk["fac"], blk["gamma1"],
+                                    blk["gamma2"], blk["B"], blk["S"], blk["nh"], blk["nkv"], blk["d"], blk["base"],
+                                    blk["eps"], O.PHASE_SOFT, s)
+    r = np.random.default_rng(81)
+    h = 1e-6
+    for name in O.BLOCK_LINEARS:
+        G = blk["W"][name].size // blk["g"]
+        for q in range(3):
+            for j in r.choice(G, 2, replace=False):
+                fp = {n: tuple(a.copy() for a in f) for n, f in blk["fac"].items()}
+                fm = {n: tuple(a.copy() for a in f) for n, f in blk["fac"].items()}
+                fp[name][q][j] += h
+                fm[name][q][j] -= h
+                fd = (_block_loss(blk, fp, s) - _block_loss(blk, fm, s)) / (2 * h)
+                got = step["g"][name][q][j]
+                assert got == pytest.approx(fd, rel=1e-5, abs=1e-10 * max(1.0, abs(fd))), (name, q, j)
+
+
+def test_block_teacher_reconstructs_itself():
+    """With the teacher's weights (TEACHER phase) the block output equals the teacher output
+    and the loss is zero."""
+    blk = _tiny_block(seed=82)
+    st = O.block_calibration_step(blk["x"], blk["W"], blk["g"], blk["stats"], blk["fac"], blk["gamma1"],
+                                  blk["gamma2"], blk["B"], blk["S"], blk["nh"], blk["nkv"], blk["d"], blk["base"],
+                                  blk["eps"], O.PHASE_TEACHER, 0.0)
+    np.testing.assert_array_equal(st["out"], st["out_ref"])
+    assert st["loss"] == 0.0
+
+
+def test_attention_closed_forms():
+    """Causal attention with all-zero queries gives equal weights to the keys up to each
+    query: O at position s is the mean of V over positions 0..s; a single position returns
+    its value row; the query head h reads key/value head h // (nh / nkv)."""
+    r = np.random.default_rng(83)
+    B, S, nh, nkv, d = 2, 6, 4, 2, 3
+    v = r.standard_normal((B * S, nkv * d))
+    k = r.standard_normal((B * S, nkv * d))
+    o, _ = O.attention(np.zeros((B * S, nh * d)), k, v, B, S, nh, nkv, d)
+    vb = v.reshape(B, S, nkv, d)
+    want = np.cumsum(vb, axis=1) / np.arange(1, S + 1)[None, :, None, None]
+    want = np.repeat(want, nh // nkv, axis=2).reshape(B * S, nh * d)
+    np.testing.assert_allclose(o, want, rtol=1e-13)
+    o1, _ = O.attention(r.standard_normal((B, nh * d)), k[:B], v[:B], B, 1, nh, nkv, d)
+    np.testing.assert_allclose(o1, np.repeat(v[:B].reshape(B, nkv, d), nh // nkv, axis=1).reshape(B, nh * d),
+                               rtol=1e-13)
+
+
+def test_attention_gradients_match_central_differences():
+    """attention_bwd against central differences of sum(dO * O) in q, k and v."""
+    r = np.random.default_rng(84)
+    B, S, nh, nkv, d = 1, 4, 2, 1, 4
+    q, k, v = (r.standard_normal((B * S, n * d)) for n in (nh, nkv, nkv))
+    do = r.standard_normal((B * S, nh * d))
+    _, p = O.attention(q, k, v, B, S, nh, nkv, d)
+    dq, dk, dv = O.attention_bwd(q, k, v, p, do, B, S, nh, nkv, d)
+    f = lambda q, k, v: float((O.attention(q, k, v, B, S, nh, nkv, d)[0] * do).sum())  # noqa: E731
+    h = 1e-6
+    for arr, grad, which in ((q, dq, 0), (k, dk, 1), (v, dv, 2)):
+        for idx in [(0, 0), (S - 1, arr.shape[1] - 1), (1, 2)]:
+            args_p = [q.copy(), k.copy(), v.copy()]
+            args_m = [q.copy(), k.copy(), v.copy()]
+            args_p[which][idx] += h
+            args_m[which][idx] -= h
+            fd = (f(*args_p) - f(*args_m)) / (2 * h)
+            assert grad[idx] == pytest.approx(fd, rel=1e-6, abs=1e-9)
+
+
+def test_rope_identity_norm_and_inverse():
+    """Position 0 is not rotated; every rotated pair keeps its length; the inverse rotation
+    undoes the rotation; with d = 2 the angle of position s is exactly s (base^0 = 1)."""
+    r = np.random.default_rng(85)
+    S, nh, d = 7, 3, 8
+    x = r.standard_normal((2 * S, nh * d))
+    y = O.rope(x, S, nh, d, 10000.0)
+    np.testing.assert_allclose(y[0], x[0], rtol=1e-15)
+    xh, yh = x.reshape(-1, nh, d), y.reshape(-1, nh, d)
+    nx = xh[..., : d // 2] ** 2 + xh[..., d // 2:] ** 2
+    ny = yh[..., : d // 2] ** 2 + yh[..., d // 2:] ** 2
+    np.testing.assert_allclose(ny, nx, rtol=1e-12)
+    np.testing.assert_allclose(O.rope(y, S, nh, d, 10000.0, inverse=True), x, rtol=1e-12, atol=1e-14)
+    z = np.array([[1.0, 0.0]] * 4)
+    rz = O.rope(z, 4, 1, 2, 10000.0)
+    np.testing.assert_allclose(rz, np.stack([np.cos(np.arange(4.0) % 4), np.sin(np.arange(4.0) % 4)], 1),
+                               rtol=1e-15)
+
+
+def test_rmsnorm_closed_forms():
+    """A constant row c maps to gamma * c / sqrt(c^2 + eps); without eps the norm is scale
+    invariant; its gradient matches central differences."""
+    gamma = np.array([0.5, 2.0, 1.5])
+    y, _ = O.rmsnorm(np.full((1, 3), 3.0), gamma, 1e-5)
+    np.testing.assert_allclose(y[0], gamma * 3.0 / np.sqrt(9.0 + 1e-5), rtol=1e-15)
+    x = np.random.default_rng(86).standard_normal((4, 3))
+    np.testing.assert_allclose(O.rmsnorm(7.0 * x, gamma, 0.0)[0], O.rmsnorm(x, gamma, 0.0)[0], rtol=1e-13)
+    dy = np.random.default_rng(87).standard_normal((4, 3))
+    _, rr = O.rmsnorm(x, gamma, 1e-5)
+    dx = O.rmsnorm_bwd(x, gamma, rr, dy)
+    h = 1e-6
+    for i, j in ((0, 0), (3, 2), (2, 1)):
+        xp, xm = x.copy(), x.copy()
+        xp[i, j] += h
+        xm[i, j] -= h
+        fd = ((O.rmsnorm(xp, gamma, 1e-5)[0] - O.rmsnorm(xm, gamma, 1e-5)[0]) * dy).sum() / (2 * h)
+        assert dx[i, j] == pytest.approx(fd, rel=1e-6)
