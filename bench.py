@@ -514,6 +514,8 @@ def run_ours(args):
         also[f"{wl.name}/decode_b1_mu"] = measure_decode(C, torch, wl, dev, peaks, rows=1, with_mu=True)
         also["c5_qwen3_235b_moe/soft"] = measure_moe(C, torch, dev, peaks, world, args.s)
         also[f"{wl.name}/fig_error_k_proj"] = measure_fig_error(C, torch, wl, dev, args.s)
+        if wl.name == "c3_llama3_8b_block" and not args.linear:
+            also[f"{wl.name}/block_window"] = measure_block_window(C, torch, wl, dev, peaks, world, args.s, barrier)
         for name in ALSO_WORKLOADS:
             if name == wl.name:
                 continue
@@ -545,6 +547,80 @@ def run_ours(args):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def measure_block_window(C, torch, wl, dev, peaks, world, s, barrier, steps=5, warmup=3):
+    """Eq. 7 over a window of one whole decoder block (§2.4) on the Llama-3-8B shape: 4 x 2048
+    tokens, 32 query heads and 8 key/value heads of 128, RoPE base 500000.  One step is the
+    student block forward (seven soft-ternary linears, RMSNorm, rotary embedding, causal
+    attention, SwiGLU), the loss on the block output against the cached teacher output, the
+    block backward into every linear's factor gradients, and the AdamW update of all factors.
+    Throughput counts the linears' 6 T N K and attention's 7 B h S^2 d flops; the attention
+    forward + backward is also timed alone on the same tensors."""
+    from paper_2606_26650_gb300 import block as BK
+    shape = BK.BlockShape(H=4096, n_heads=32, n_kv_heads=8, d=128, I=14336, B=4, S=2048, base=500000.0, eps=1e-5)
+    assert shape.T == wl.M
+    bf = torch.bfloat16
+
+    def upload(a):
+        return torch.from_numpy(syn.bf16_bits(a).view(np.int16)).to(dev).view(bf)
+
+    W = {lin.name: upload(syn.weight(wl, lin)) for lin in wl.linears}
+    r = syn.rng(97, "bench/block_window")
+    g1, g2 = (torch.from_numpy(r.uniform(0.5, 1.5, shape.H).astype(np.float32)).to(dev) for _ in range(2))
+    fac = {n: tuple(torch.from_numpy(f).to(dev) for f in syn.factors(W[n].numel() // wl.g, 0, f"window/{n}", True))
+           for n in W}
+    blk = BK.Block(shape, W, g1, g2, wl.g, factors=fac)
+    x = upload(syn.activations(wl, "x_hidden", shape.T, shape.H))
+    out_ref = torch.empty(shape.T, shape.H, dtype=torch.float32, device=dev)
+    blk.teacher(x, out_ref)
+    loss = torch.zeros(1, dtype=torch.float32, device=dev)
+    grads = {n: [torch.empty(W[n].numel() // wl.g, dtype=torch.float32, device=dev) for _ in range(3)] for n in W}
+    upd = FactorUpdate(C, torch, dev, [W[n].numel() // wl.g for n in BK.LINEARS])
+    sched = C.schedule(C.PHASE_SOFT, s)
+
+    def step():
+        blk.step(x, out_ref, sched, loss, grads)
+        upd.advance()
+        for i, n in enumerate(BK.LINEARS):
+            upd.apply(i, blk.layers[n], grads[n])
+
+    def timed(fn, n, w):
+        for _ in range(w):
+            fn()
+        barrier()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(n):
+            fn()
+        b.record()
+        barrier()
+        status = C.catq_device_status()
+        if status != 0:
+            raise SystemExit(f"device status {C.STATUS.get(status, status)} in the block-window timed region")
+        return a.elapsed_time(b) / n
+
+    ms = max_over_ranks(timed(step, steps, warmup), world, dev)
+    first_loss = loss.item()
+
+    def attention():
+        C.catq_attention_fwd(blk.q, blk.k, blk.v, blk.a, blk.lse, shape.B, shape.S, shape.n_heads, shape.n_kv_heads,
+                             shape.d)
+        C.catq_attention_bwd(blk.q, blk.k, blk.v, blk.a, blk.da, blk.lse, blk.delta, blk.dq, blk.dk, blk.dv, shape.B,
+                             shape.S, shape.n_heads, shape.n_kv_heads, shape.d)
+
+    attn_ms = timed(attention, steps, 2)
+    flops = shape.linear_flops() + shape.attention_flops()
+    value = job_throughput(flops, ms, world)
+    out = {"value": value, "unit": UNIT, "ms_per_step": ms, "steps": steps, "frac_of_burst": value / world / peaks["bf16"],
+           "flops_per_step": {"linears": shape.linear_flops(), "attention": shape.attention_flops()},
+           "attention_fwd_bwd_ms": attn_ms,
+           "attention_tflops": shape.attention_flops() / (attn_ms * 1e-3) / 1e12,
+           "loss_after_steps": first_loss, "phase": "soft", "s": s,
+           "shape": dataclasses.asdict(shape), "l2": "working set > L2 (no flush)"}
+    del blk, W, x, out_ref, grads, upd
+    torch.cuda.empty_cache()
+    return out
 
 
 # Linears of a decoder block that may run in one launch (their inputs do not depend on each

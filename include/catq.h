@@ -467,6 +467,86 @@ int32_t catq_ternary_infer_max_layers(void);
 catq_status catq_ternary_infer_batched(const catq_infer_layer* layers, int32_t n_layers, int32_t g, int64_t B,
                                        int32_t x_dtype, catq_stream stream);
 
+/* ------------------------------------------------------------------ decoder-block layers
+ * Eq. 7 reconstructs the output of a sliding window of layers (§2.4); with a window of one
+ * decoder block the loss reaches each linear's factors through the layers
+ * between the linears.  These calls are those layers for the Llama / Qwen block (pre-norm,
+ * causal grouped-query attention with rotary position embedding, SwiGLU MLP), forward and
+ * backward, on bf16 activations with fp32 arithmetic and an fp32 residual stream.  Tokens are
+ * rows t = b S + s of [T = B S, *]
+ * row-major activations; every activation pointer is device memory, 16-byte aligned, owned by
+ * the caller; vectors (gamma, r, lse) are fp32.  T == 0 (or n == 0) is a no-op.  Errors:
+ * negative sizes or a violated shape rule CATQ_ERR_SHAPE, a required NULL pointer
+ * CATQ_ERR_INVALID_ARG, misalignment CATQ_ERR_ALIGN, a failed launch CATQ_ERR_CUDA. */
+
+/* RMSNorm of each row, with the residual add fused in front:
+ *   h = X + residual (in fp32, never rounded; h = X when residual is NULL), stored into h_out
+ *       when it is given (the block's residual stream, kept in fp32);
+ *   r[t] = 1 / sqrt(mean_i h[t,i]^2 + eps),  Z = gamma * h * r  (bf16).
+ * X [T, H] has x_dtype (CATQ_BF16 or CATQ_F32), residual [T, H] bf16, h_out [T, H] fp32,
+ * Z [T, H] bf16; gamma [H]; r [T] (kept for the backward).  H % 8 == 0, eps >= 0. */
+catq_status catq_rmsnorm_fwd(const void* X, int32_t x_dtype, const void* residual, const float* gamma, int64_t T,
+                             int64_t H, float eps, float* h_out, void* Z, float* r, catq_stream stream);
+
+/* Backward of catq_rmsnorm_fwd at h (its input, or the stored residual sum; h_dtype
+ * CATQ_BF16 or CATQ_F32):
+ *   u = gamma * (dZ + dZ2),  dX = r u - h r^3 mean_i(u h) (+ d_residual)
+ * dZ2 (a second consumer of Z, e.g. the gate and up projections) and d_residual (the
+ * gradient reaching h around the norm) are nullable; dZ, dZ2, d_residual, dX bf16.  dX may
+ * alias dZ, dZ2 or d_residual. */
+catq_status catq_rmsnorm_bwd(const void* h, int32_t h_dtype, const float* gamma, const float* r, const void* dZ,
+                             const void* dZ2, const void* d_residual, int64_t T, int64_t H, void* dX,
+                             catq_stream stream);
+
+/* Rotary position embedding in place on X [T, n_heads d]: in every head, elements i and
+ * i + d/2 rotate together by the angle s base^(-2i/d), s = t mod S the token's position
+ * (inverse != 0: by its negative, which is the backward of the rotation).  d even, 8 <= d,
+ * S >= 1, base > 1. */
+catq_status catq_rope(void* X, int64_t T, int64_t S, int32_t n_heads, int32_t d, float base, int32_t inverse,
+                      catq_stream stream);
+
+/* SwiGLU: M = silu(gate) * up elementwise over n elements. */
+catq_status catq_swiglu_fwd(const void* gate, const void* up, int64_t n, void* M, catq_stream stream);
+
+/* Backward of catq_swiglu_fwd: d_gate = dM up sigma(gate) (1 + gate (1 - sigma(gate))),
+ * d_up = dM silu(gate). */
+catq_status catq_swiglu_bwd(const void* gate, const void* up, const void* dM, int64_t n, void* d_gate, void* d_up,
+                            catq_stream stream);
+
+/* The block output and Eq. 7's loss on it, in one pass over count elements:
+ *   out = h + branch          (h fp32, the residual stream; branch bf16, e.g. the down
+ *                              projection's output); stored into out (fp32) when given;
+ *   with out_ref (fp32, the teacher block's output; NULL computes out only):
+ *   loss_out[0] = sum (out - out_ref)^2 / count (CATQ_REDUCE_MEAN) or the plain sum (SUM),
+ *   d_out = 2 (out - out_ref) / count (MEAN) or 2 (out - out_ref) (SUM), rounded once to
+ *   bf16 (nullable).
+ * The difference is taken in fp32 before any rounding, so the residual stream's magnitude
+ * does not swamp the student-teacher difference.  count % 8 == 0.  With out_ref: loss_out
+ * (device fp32 scalar) required, workspace >= catq_recon_loss_workspace_bytes(count),
+ * 256-byte aligned (else CATQ_ERR_WORKSPACE).  Summation as in catq_recon_loss
+ * (deterministic). */
+catq_status catq_block_output_loss(const float* h, const void* branch, int64_t count, const float* out_ref,
+                                   int32_t reduction, float* loss_out, void* d_out, float* out, void* workspace,
+                                   size_t ws_bytes, catq_stream stream);
+
+/* Causal grouped-query attention: query head h uses key/value head h / (n_heads / n_kv_heads),
+ *   O = softmax(Q K^T / sqrt(d), keys s' <= s) V   for every sequence b and head h,
+ * with Q, O [B S, n_heads d], K, V [B S, n_kv_heads d], and lse [B, n_heads, S] the natural
+ * log-sum-exp of each row's scaled scores (kept for the backward).  Scores, the softmax and
+ * the accumulation run in fp32; the probabilities enter P V in bf16.  d is 64 or 128;
+ * S % 64 == 0; n_heads % n_kv_heads == 0. */
+catq_status catq_attention_fwd(const void* Q, const void* K, const void* V, int32_t B, int32_t S, int32_t n_heads,
+                               int32_t n_kv_heads, int32_t d, void* O, float* lse, catq_stream stream);
+
+/* Backward of catq_attention_fwd from dO [B S, n_heads d] and the forward's O and lse:
+ *   dS = P (dO V^T - rowsum(dO O)),  dQ = dS K / sqrt(d),
+ *   dK = sum over the heads sharing it of dS^T Q / sqrt(d),  dV = the same sum of P^T dO.
+ * delta: device fp32 scratch [B, n_heads, S].  dQ like Q, dK and dV like K; all three are
+ * overwritten (no atomics: the result does not depend on scheduling). */
+catq_status catq_attention_bwd(const void* Q, const void* K, const void* V, const void* O, const void* dO,
+                               const float* lse, int32_t B, int32_t S, int32_t n_heads, int32_t n_kv_heads,
+                               int32_t d, float* delta, void* dQ, void* dK, void* dV, catq_stream stream);
+
 /* Self-test of the device-side failure detection (no counterpart in the paper): launches
  * one thread that waits, through the library's bounded mbarrier wait, on a barrier nothing
  * arrives on.  After timeout_ns (1 us .. 1 s) the wait gives up, latches CATQ_ERR_TIMEOUT

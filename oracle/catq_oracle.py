@@ -512,9 +512,33 @@ def attention_bwd(q, k, v, p, do, B, S, nh, nkv, d):
     return dq.reshape(B * S, nh * d), dk.reshape(B * S, nkv * d), dv.reshape(B * S, nkv * d)
 
 
+def attention_logsumexp(q, k, B, S, nh, nkv, d):
+    """The softmax normaliser of ``attention``: for every sequence, head and query s, the
+    natural log of the sum over keys s' <= s of exp(q . k / sqrt(d)); [B, nh, S]."""
+    q = np.asarray(q, np.float64).reshape(B, S, nh, d)
+    k = np.repeat(np.asarray(k, np.float64).reshape(B, S, nkv, d), nh // nkv, axis=2)
+    s = np.einsum("bqhd,bkhd->bhqk", q, k) / np.sqrt(d)
+    s = np.where(np.tril(np.ones((S, S), bool))[None, None], s, -np.inf)
+    m = s.max(axis=3)
+    return m + np.log(np.exp(s - m[..., None]).sum(axis=3))
+
+
 def silu(a):
     a = np.asarray(a, np.float64)
     return a / (1.0 + np.exp(-a))
+
+
+def swiglu(gt, u):
+    """The SwiGLU MLP's gate: silu(gt) * u elementwise."""
+    return silu(gt) * np.asarray(u, np.float64)
+
+
+def swiglu_bwd(gt, u, dm):
+    """Gradients of ``swiglu`` from dm: with sigma the logistic function,
+    d_gt = dm u sigma(gt) (1 + gt (1 - sigma(gt))) and d_u = dm silu(gt)."""
+    gt, u, dm = (np.asarray(a, np.float64) for a in (gt, u, dm))
+    sg = 1.0 / (1.0 + np.exp(-gt))
+    return dm * u * sg * (1.0 + gt * (1.0 - sg)), dm * silu(gt)
 
 
 BLOCK_LINEARS = ("q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj")
@@ -534,7 +558,7 @@ def block_forward(x, Wq, gamma1, gamma2, B, S, nh, nkv, d, base, eps):
     z2, r2 = rmsnorm(h, gamma2, eps)
     gt = linear_fwd(z2, Wq["gate_proj"])
     u = linear_fwd(z2, Wq["up_proj"])
-    m = silu(gt) * u
+    m = swiglu(gt, u)
     out = h + linear_fwd(m, Wq["down_proj"])
     return out, dict(z1=z1, q=q, k=k, v=v, a=a, p=p, h=h, z2=z2, r2=r2, gt=gt, u=u, m=m)
 
@@ -560,9 +584,7 @@ def block_calibration_step(x, W, g, stats, factors, gamma1, gamma2, B, S, nh, nk
 
     grads("down_proj", c["m"], d_out)
     dm = d_out @ Wq["down_proj"]
-    sg = 1.0 / (1.0 + np.exp(-c["gt"]))
-    d_gt = dm * c["u"] * sg * (1.0 + c["gt"] * (1.0 - sg))
-    d_u = dm * silu(c["gt"])
+    d_gt, d_u = swiglu_bwd(c["gt"], c["u"], dm)
     grads("gate_proj", c["z2"], d_gt)
     grads("up_proj", c["z2"], d_u)
     dz2 = d_gt @ Wq["gate_proj"] + d_u @ Wq["up_proj"]

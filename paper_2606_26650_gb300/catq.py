@@ -115,6 +115,14 @@ def lib() -> ctypes.CDLL:
         "catq_ternary_infer_batched": (I32, [ctypes.POINTER(catq_infer_layer), I32, I32, I64, I32, P]),
         "catq_group_recon_error": (I32, [LP, P, P]),
         "catq_grouped_fwd_loss_workspace_bytes": (S, [ctypes.POINTER(catq_grouped_layer), P]),
+        "catq_rmsnorm_fwd": (I32, [P, I32, P, P, I64, I64, F, P, P, P, P]),
+        "catq_rmsnorm_bwd": (I32, [P, I32, P, P, P, P, P, I64, I64, P, P]),
+        "catq_rope": (I32, [P, I64, I64, I32, I32, F, I32, P]),
+        "catq_swiglu_fwd": (I32, [P, P, I64, P, P]),
+        "catq_swiglu_bwd": (I32, [P, P, P, I64, P, P, P]),
+        "catq_block_output_loss": (I32, [P, P, I64, P, I32, P, P, P, P, S, P]),
+        "catq_attention_fwd": (I32, [P, P, P, I32, I32, I32, I32, I32, P, P, P]),
+        "catq_attention_bwd": (I32, [P, P, P, P, P, P, I32, I32, I32, I32, I32, P, P, P, P, P]),
         "catq_grouped_soft_ternary_linear_fwd_loss": (I32, [ctypes.POINTER(catq_grouped_layer), catq_schedule, P, P,
                                                             I32, P, I32, P, P, P, P, S, P]),
     }
@@ -576,3 +584,101 @@ def catq_grouped_soft_ternary_linear_fwd_loss(layer: GroupedLayer, sched: catq_s
                                                            _dtype_code(X), _ptr(Y_ref), int(reduction),
                                                            _ptr(loss_out), _ptr(dY), _ptr(Y), _ptr(workspace),
                                                            ws_bytes, _stream(stream)), w)
+
+
+# ------------------------------------------------------------------ decoder-block layers
+# bf16 activations [T, *] (tokens t = b S + s); fp32 gamma, r, lse, delta.
+
+def _bf16_bufs(where, nbytes, **bufs):
+    import torch
+    for name, t in bufs.items():
+        if t is not None and t.dtype != torch.bfloat16:
+            raise ValueError(f"{where}: {name} must be bfloat16")
+        _buf(t, name, nbytes, where)
+
+
+def catq_rmsnorm_fwd(X, gamma, Z, r, eps, residual=None, h_out=None, stream=None):
+    """Z = gamma * h / rms(h), h = X (+ residual, in fp32, stored into h_out); r [T] = 1 / rms(h).
+    X bf16 or fp32; residual, Z bf16; h_out fp32."""
+    import torch
+    T, H = X.shape
+    w = "catq_rmsnorm_fwd"
+    _buf(X, "X", T * H * X.element_size(), w)
+    _bf16_bufs(w, 2 * T * H, residual=residual, Z=Z)
+    if h_out is not None and h_out.dtype != torch.float32:
+        raise ValueError(f"{w}: h_out must be float32")
+    _buf(h_out, "h_out", 4 * T * H, w)
+    _buf(gamma, "gamma", 4 * H, w)
+    _buf(r, "r", 4 * T, w)
+    _check(lib().catq_rmsnorm_fwd(_ptr(X), _dtype_code(X), _ptr(residual), _ptr(gamma), T, H, float(eps),
+                                  _ptr(h_out), _ptr(Z), _ptr(r), _stream(stream)), w)
+
+
+def catq_rmsnorm_bwd(h, gamma, r, dZ, dX, dZ2=None, d_residual=None, stream=None):
+    """dX of catq_rmsnorm_fwd at h (bf16 or fp32); dZ, dZ2, d_residual, dX bf16."""
+    T, H = h.shape
+    w = "catq_rmsnorm_bwd"
+    _buf(h, "h", T * H * h.element_size(), w)
+    _bf16_bufs(w, 2 * T * H, dZ=dZ, dZ2=dZ2, d_residual=d_residual, dX=dX)
+    _buf(gamma, "gamma", 4 * H, w)
+    _buf(r, "r", 4 * T, w)
+    _check(lib().catq_rmsnorm_bwd(_ptr(h), _dtype_code(h), _ptr(gamma), _ptr(r), _ptr(dZ), _ptr(dZ2),
+                                  _ptr(d_residual), T, H, _ptr(dX), _stream(stream)), w)
+
+
+def catq_rope(X, S, n_heads, d, base, inverse=False, stream=None):
+    T = X.shape[0]
+    w = "catq_rope"
+    _bf16_bufs(w, 2 * T * n_heads * d, X=X)
+    _check(lib().catq_rope(_ptr(X), T, int(S), int(n_heads), int(d), float(base), int(bool(inverse)),
+                           _stream(stream)), w)
+
+
+def catq_swiglu_fwd(gate, up, M, stream=None):
+    n = gate.numel()
+    _bf16_bufs("catq_swiglu_fwd", 2 * n, gate=gate, up=up, M=M)
+    _check(lib().catq_swiglu_fwd(_ptr(gate), _ptr(up), n, _ptr(M), _stream(stream)), "catq_swiglu_fwd")
+
+
+def catq_swiglu_bwd(gate, up, dM, d_gate, d_up, stream=None):
+    n = gate.numel()
+    _bf16_bufs("catq_swiglu_bwd", 2 * n, gate=gate, up=up, dM=dM, d_gate=d_gate, d_up=d_up)
+    _check(lib().catq_swiglu_bwd(_ptr(gate), _ptr(up), _ptr(dM), n, _ptr(d_gate), _ptr(d_up), _stream(stream)),
+           "catq_swiglu_bwd")
+
+
+def catq_block_output_loss(h, branch, out_ref=None, loss_out=None, d_out=None, out=None, workspace=None,
+                           reduction: int = REDUCE_MEAN, stream=None):
+    """out = h + branch in fp32; with out_ref, Eq. 7's loss into loss_out and d_out (bf16)."""
+    import torch
+    n, w = h.numel(), "catq_block_output_loss"
+    for name, t in (("h", h), ("out_ref", out_ref), ("out", out)):
+        if t is not None and t.dtype != torch.float32:
+            raise ValueError(f"{w}: {name} must be float32")
+        _buf(t, name, 4 * n, w)
+    _bf16_bufs(w, 2 * n, branch=branch, d_out=d_out)
+    _buf(loss_out, "loss_out", 4, w)
+    _buf(workspace, "workspace", 0, w)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib().catq_block_output_loss(_ptr(h), _ptr(branch), n, _ptr(out_ref), int(reduction), _ptr(loss_out),
+                                        _ptr(d_out), _ptr(out), _ptr(workspace), ws_bytes, _stream(stream)), w)
+
+
+def catq_attention_fwd(Q, K, V, O, lse, B, S, n_heads, n_kv_heads, d, stream=None):
+    w = "catq_attention_fwd"
+    _bf16_bufs(w, 2 * B * S * n_heads * d, Q=Q, O=O)
+    _bf16_bufs(w, 2 * B * S * n_kv_heads * d, K=K, V=V)
+    _buf(lse, "lse", 4 * B * n_heads * S, w)
+    _check(lib().catq_attention_fwd(_ptr(Q), _ptr(K), _ptr(V), int(B), int(S), int(n_heads), int(n_kv_heads),
+                                    int(d), _ptr(O), _ptr(lse), _stream(stream)), w)
+
+
+def catq_attention_bwd(Q, K, V, O, dO, lse, delta, dQ, dK, dV, B, S, n_heads, n_kv_heads, d, stream=None):
+    w = "catq_attention_bwd"
+    _bf16_bufs(w, 2 * B * S * n_heads * d, Q=Q, O=O, dO=dO, dQ=dQ)
+    _bf16_bufs(w, 2 * B * S * n_kv_heads * d, K=K, V=V, dK=dK, dV=dV)
+    _buf(lse, "lse", 4 * B * n_heads * S, w)
+    _buf(delta, "delta", 4 * B * n_heads * S, w)
+    _check(lib().catq_attention_bwd(_ptr(Q), _ptr(K), _ptr(V), _ptr(O), _ptr(dO), _ptr(lse), int(B), int(S),
+                                    int(n_heads), int(n_kv_heads), int(d), _ptr(delta), _ptr(dQ), _ptr(dK),
+                                    _ptr(dV), _stream(stream)), w)

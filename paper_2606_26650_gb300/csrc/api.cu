@@ -775,4 +775,134 @@ catq_status catq_device_status(catq_stream stream, int32_t* out) {
   return cuda_status(read_and_clear_device_status(out));
 }
 
+// ------------------------------------------------------------------ decoder-block layers
+
+namespace {
+bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
+cudaStream_t as_stream(catq_stream s) { return reinterpret_cast<cudaStream_t>(s); }
+}  // namespace
+
+catq_status catq_rmsnorm_fwd(const void* X, int32_t x_dtype, const void* residual, const float* gamma, int64_t T,
+                             int64_t H, float eps, float* h_out, void* Z, float* r, catq_stream stream) {
+  if (x_dtype != CATQ_BF16 && x_dtype != CATQ_F32) return CATQ_ERR_DTYPE;
+  if (T < 0 || H < 1 || H % 8 != 0 || T > 0x7fffffff) return CATQ_ERR_SHAPE;
+  if (!(eps >= 0.0f) || !std::isfinite(eps)) return CATQ_ERR_INVALID_ARG;
+  if (T == 0) return CATQ_OK;
+  if (!X || !gamma || !Z || !r) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(X) || !aligned16(Z) || (residual && !aligned16(residual)) || (h_out && !aligned16(h_out)) ||
+      !aligned4(gamma) || !aligned4(r))
+    return CATQ_ERR_ALIGN;
+  return cuda_status(launch_rmsnorm_fwd(X, x_dtype == CATQ_F32, residual, gamma, T, H, eps, h_out, Z, r,
+                                        as_stream(stream)));
+}
+
+catq_status catq_rmsnorm_bwd(const void* h, int32_t h_dtype, const float* gamma, const float* r, const void* dZ,
+                             const void* dZ2, const void* d_residual, int64_t T, int64_t H, void* dX,
+                             catq_stream stream) {
+  if (h_dtype != CATQ_BF16 && h_dtype != CATQ_F32) return CATQ_ERR_DTYPE;
+  if (T < 0 || H < 1 || H % 8 != 0 || T > 0x7fffffff) return CATQ_ERR_SHAPE;
+  if (T == 0) return CATQ_OK;
+  if (!h || !gamma || !r || !dZ || !dX) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(h) || !aligned16(dZ) || !aligned16(dX) || (dZ2 && !aligned16(dZ2)) ||
+      (d_residual && !aligned16(d_residual)) || !aligned4(gamma) || !aligned4(r))
+    return CATQ_ERR_ALIGN;
+  return cuda_status(launch_rmsnorm_bwd(h, h_dtype == CATQ_F32, gamma, r, dZ, dZ2, d_residual, T, H, dX,
+                                        as_stream(stream)));
+}
+
+catq_status catq_rope(void* X, int64_t T, int64_t S, int32_t n_heads, int32_t d, float base, int32_t inverse,
+                      catq_stream stream) {
+  if (T < 0 || S < 1 || n_heads < 1 || d < 8 || d % 2 != 0) return CATQ_ERR_SHAPE;
+  if (!(base > 1.0f) || !std::isfinite(base)) return CATQ_ERR_INVALID_ARG;
+  if (T == 0) return CATQ_OK;
+  if (!X) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(X)) return CATQ_ERR_ALIGN;
+  return cuda_status(launch_rope(X, T, S, n_heads, d, base, inverse, as_stream(stream)));
+}
+
+catq_status catq_swiglu_fwd(const void* gate, const void* up, int64_t n, void* M, catq_stream stream) {
+  if (n < 0) return CATQ_ERR_SHAPE;
+  if (n == 0) return CATQ_OK;
+  if (!gate || !up || !M) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(gate) || !aligned16(up) || !aligned16(M)) return CATQ_ERR_ALIGN;
+  return cuda_status(launch_swiglu(gate, up, nullptr, n, M, nullptr, nullptr, as_stream(stream)));
+}
+
+catq_status catq_swiglu_bwd(const void* gate, const void* up, const void* dM, int64_t n, void* d_gate, void* d_up,
+                            catq_stream stream) {
+  if (n < 0) return CATQ_ERR_SHAPE;
+  if (n == 0) return CATQ_OK;
+  if (!gate || !up || !dM || !d_gate || !d_up) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(gate) || !aligned16(up) || !aligned16(dM) || !aligned16(d_gate) || !aligned16(d_up))
+    return CATQ_ERR_ALIGN;
+  return cuda_status(launch_swiglu(gate, up, dM, n, nullptr, d_gate, d_up, as_stream(stream)));
+}
+
+catq_status catq_block_output_loss(const float* h, const void* branch, int64_t count, const float* out_ref,
+                                   int32_t reduction, float* loss_out, void* d_out, float* out, void* workspace,
+                                   size_t ws_bytes, catq_stream stream) {
+  if (count < 0 || count % 8 != 0) return CATQ_ERR_SHAPE;
+  if (reduction != CATQ_REDUCE_MEAN && reduction != CATQ_REDUCE_SUM) return CATQ_ERR_INVALID_ARG;
+  if (count == 0) return CATQ_OK;
+  if (!h || !branch || (out_ref && !loss_out)) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(h) || !aligned16(branch) || (out_ref && !aligned16(out_ref)) || (out && !aligned16(out)) ||
+      (d_out && !aligned16(d_out)) || (loss_out && !aligned4(loss_out)))
+    return CATQ_ERR_ALIGN;
+  if (out_ref) {
+    if (!workspace || ws_bytes < catq_recon_loss_workspace_bytes(count)) return CATQ_ERR_WORKSPACE;
+    if (!aligned256(workspace)) return CATQ_ERR_ALIGN;
+  }
+  return cuda_status(launch_block_output_loss(h, branch, out_ref, count, reduction, out, d_out, loss_out,
+                                              static_cast<double*>(workspace), as_stream(stream)));
+}
+
+namespace {
+catq_status check_attention(int32_t B, int32_t S, int32_t nh, int32_t nkv, int32_t d) {
+  if (B < 0 || B > 65535 || S < 64 || S % 64 != 0 || nh < 1 || nh > 65535 || nkv < 1 || nh % nkv != 0 ||
+      (d != 64 && d != 128))
+    return CATQ_ERR_SHAPE;
+  return CATQ_OK;
+}
+}  // namespace
+
+catq_status catq_attention_fwd(const void* Q, const void* K, const void* V, int32_t B, int32_t S, int32_t n_heads,
+                               int32_t n_kv_heads, int32_t d, void* O, float* lse, catq_stream stream) {
+  catq_status st = check_attention(B, S, n_heads, n_kv_heads, d);
+  if (st != CATQ_OK) return st;
+  if (B == 0) return CATQ_OK;
+  if (!Q || !K || !V || !O || !lse) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O) || !aligned4(lse)) return CATQ_ERR_ALIGN;
+  AttnIo io{};
+  io.q = Q;
+  io.k = K;
+  io.v = V;
+  io.out = O;
+  io.lse = lse;
+  return cuda_status(launch_attention(io, B, S, n_heads, n_kv_heads, d, false, as_stream(stream)));
+}
+
+catq_status catq_attention_bwd(const void* Q, const void* K, const void* V, const void* O, const void* dO,
+                               const float* lse, int32_t B, int32_t S, int32_t n_heads, int32_t n_kv_heads,
+                               int32_t d, float* delta, void* dQ, void* dK, void* dV, catq_stream stream) {
+  catq_status st = check_attention(B, S, n_heads, n_kv_heads, d);
+  if (st != CATQ_OK) return st;
+  if (B == 0) return CATQ_OK;
+  if (!Q || !K || !V || !O || !dO || !lse || !delta || !dQ || !dK || !dV) return CATQ_ERR_INVALID_ARG;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O) || !aligned16(dO) || !aligned16(dQ) ||
+      !aligned16(dK) || !aligned16(dV) || !aligned4(lse) || !aligned4(delta))
+    return CATQ_ERR_ALIGN;
+  AttnIo io{};
+  io.q = Q;
+  io.k = K;
+  io.v = V;
+  io.o = O;
+  io.dO = dO;
+  io.dq = dQ;
+  io.dk = dK;
+  io.dv = dV;
+  io.lse = const_cast<float*>(lse);
+  io.delta = delta;
+  return cuda_status(launch_attention(io, B, S, n_heads, n_kv_heads, d, true, as_stream(stream)));
+}
+
 }  // extern "C"

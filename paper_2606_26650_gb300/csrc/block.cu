@@ -1,0 +1,696 @@
+// block.cu — the layers around the seven soft-ternary linears of one decoder block, for the
+// block-output reconstruction step (§2.4, Eq. 7 over a window of one block): RMSNorm (with the
+// residual add fused into the forward, and the residual and second upstream gradient fused
+// into the backward), rotary position embedding, SwiGLU, an add, and causal grouped-query
+// attention (forward, and a deterministic backward in two kernels).
+//
+// Attention runs on the tensor pipe with mma.sync m16n8k16 (bf16 in, fp32 accumulate):
+// blocks of 64 queries (four warps of 16) against blocks of 64 keys staged in shared memory,
+// an online softmax in fp32 with the probabilities fed back as the A operand of P V straight
+// from the score accumulators, and operand fragments read from shared memory with ldmatrix
+// (transposed where the contraction runs along rows).  The backward recomputes the
+// probabilities from the forward's log-sum-exp: one kernel per query block accumulates dQ;
+// one per key block accumulates dK and dV over every query head that shares the key/value
+// head, so no atomics are needed and the result is deterministic.
+#include <cuda_bf16.h>
+
+#include "launch.h"
+#include "ptx_sm100.cuh"
+
+namespace catq {
+namespace {
+
+constexpr int kRowThreads = 256;
+
+__device__ __forceinline__ float bf16_at(const uint16_t* p, int64_t i) { return __uint_as_float(uint32_t(p[i]) << 16); }
+__device__ __forceinline__ uint16_t to_bf16(float v) { return static_cast<uint16_t>(pack_bf16x2(v, 0.0f) & 0xFFFFu); }
+
+__device__ __forceinline__ float block_sum(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float t = 0.0f;
+#pragma unroll
+  for (int i = 0; i < kRowThreads / 32; ++i) t += red[i];
+  return t;
+}
+
+// ---------------------------------------------------------------- RMSNorm
+__device__ __forceinline__ float load_act(const uint16_t* p, int64_t i) { return bf16_at(p, i); }
+__device__ __forceinline__ float load_act(const float* p, int64_t i) { return p[i]; }
+
+// One CTA per token row: h = x (+ residual, in fp32, stored unrounded when h_out is given),
+// r = 1 / sqrt(mean(h^2) + eps), z = gamma * h * r.
+template <typename TX>
+__global__ void __launch_bounds__(kRowThreads) rmsnorm_fwd_kernel(const TX* __restrict__ x,
+                                                                   const uint16_t* __restrict__ res,
+                                                                   const float* __restrict__ gamma, int64_t H,
+                                                                   float eps, float* __restrict__ h_out,
+                                                                   uint16_t* __restrict__ z, float* __restrict__ r) {
+  __shared__ float red[kRowThreads / 32];
+  const int64_t t = blockIdx.x;
+  float ss = 0.0f;
+  for (int64_t i = threadIdx.x; i < H; i += kRowThreads) {
+    float h = load_act(x, t * H + i);
+    if (res) h += bf16_at(res, t * H + i);
+    if (h_out) h_out[t * H + i] = h;
+    ss = fmaf(h, h, ss);
+  }
+  const float rr = rsqrtf(block_sum(ss, red) / static_cast<float>(H) + eps);
+  if (threadIdx.x == 0) r[t] = rr;
+  for (int64_t i = threadIdx.x; i < H; i += kRowThreads) {
+    float h = load_act(x, t * H + i);
+    if (res) h += bf16_at(res, t * H + i);
+    z[t * H + i] = to_bf16(gamma[i] * h * rr);
+  }
+}
+
+// dx = r u - h r^3 mean(u h) (+ dres), u = gamma (dy + dy2).
+template <typename TH>
+__global__ void __launch_bounds__(kRowThreads) rmsnorm_bwd_kernel(const TH* __restrict__ x,
+                                                                   const float* __restrict__ gamma,
+                                                                   const float* __restrict__ r,
+                                                                   const uint16_t* __restrict__ dy,
+                                                                   const uint16_t* __restrict__ dy2,
+                                                                   const uint16_t* __restrict__ dres, int64_t H,
+                                                                   uint16_t* __restrict__ dx) {
+  __shared__ float red[kRowThreads / 32];
+  const int64_t t = blockIdx.x;
+  const float rr = r[t];
+  float sux = 0.0f;
+  for (int64_t i = threadIdx.x; i < H; i += kRowThreads) {
+    const float g = bf16_at(dy, t * H + i) + (dy2 ? bf16_at(dy2, t * H + i) : 0.0f);
+    sux = fmaf(gamma[i] * g, load_act(x, t * H + i), sux);
+  }
+  const float c = block_sum(sux, red) / static_cast<float>(H) * rr * rr * rr;
+  for (int64_t i = threadIdx.x; i < H; i += kRowThreads) {
+    const float g = bf16_at(dy, t * H + i) + (dy2 ? bf16_at(dy2, t * H + i) : 0.0f);
+    float v = rr * gamma[i] * g - load_act(x, t * H + i) * c;
+    if (dres) v += bf16_at(dres, t * H + i);
+    dx[t * H + i] = to_bf16(v);
+  }
+}
+
+// ---------------------------------------------------------------- rotary embedding
+// Element pair (i, i + d/2) of every head of token t (position s = t mod S) rotated by the
+// angle s base^(-2i/d) (its negative for the inverse), in place.
+__global__ void __launch_bounds__(kRowThreads) rope_kernel(uint16_t* __restrict__ x, int64_t T, int64_t S,
+                                                            int32_t nheads, int32_t d, float log2_base,
+                                                            int32_t inverse) {
+  const int32_t half = d / 2;
+  const int64_t pairs = T * nheads * half;
+  for (int64_t e = blockIdx.x * (int64_t)kRowThreads + threadIdx.x; e < pairs; e += (int64_t)gridDim.x * kRowThreads) {
+    const int32_t i = static_cast<int32_t>(e % half);
+    const int64_t th = e / half;  // token * nheads + head
+    const int64_t t = th / nheads;
+    const float inv_freq = exp2f(-log2_base * (2.0f * i) / static_cast<float>(d));
+    float sn, cs;
+    sincosf(static_cast<float>(t % S) * inv_freq, &sn, &cs);
+    if (inverse) sn = -sn;
+    uint16_t* p = x + th * d;
+    const float a = bf16_at(p, i), b = bf16_at(p, i + half);
+    p[i] = to_bf16(a * cs - b * sn);
+    p[i + half] = to_bf16(a * sn + b * cs);
+  }
+}
+
+// ---------------------------------------------------------------- SwiGLU and add
+__device__ __forceinline__ float sigmoidf(float a) { return 1.0f / (1.0f + expf(-a)); }
+
+__global__ void __launch_bounds__(kRowThreads) swiglu_fwd_kernel(const uint16_t* __restrict__ gt,
+                                                                  const uint16_t* __restrict__ u, int64_t n,
+                                                                  uint16_t* __restrict__ m) {
+  for (int64_t e = blockIdx.x * (int64_t)kRowThreads + threadIdx.x; e < n; e += (int64_t)gridDim.x * kRowThreads) {
+    const float a = bf16_at(gt, e);
+    m[e] = to_bf16(a * sigmoidf(a) * bf16_at(u, e));
+  }
+}
+
+// d_gate = dm u sigma(a) (1 + a (1 - sigma(a))), d_up = dm a sigma(a).
+__global__ void __launch_bounds__(kRowThreads) swiglu_bwd_kernel(const uint16_t* __restrict__ gt,
+                                                                  const uint16_t* __restrict__ u,
+                                                                  const uint16_t* __restrict__ dm, int64_t n,
+                                                                  uint16_t* __restrict__ dgt,
+                                                                  uint16_t* __restrict__ du) {
+  for (int64_t e = blockIdx.x * (int64_t)kRowThreads + threadIdx.x; e < n; e += (int64_t)gridDim.x * kRowThreads) {
+    const float a = bf16_at(gt, e), s = sigmoidf(a), g = bf16_at(dm, e);
+    dgt[e] = to_bf16(g * bf16_at(u, e) * s * (1.0f + a * (1.0f - s)));
+    du[e] = to_bf16(g * a * s);
+  }
+}
+
+// Block output in fp32, out = h + branch, and (with a teacher output) Eq. 7's loss: partial
+// sums of (out - ref)^2 per CTA (compensated fp32, then fp64) and d_out = scale (out - ref)
+// rounded once to bf16.  Eight elements per thread and iteration (count % 8 == 0).
+__global__ void __launch_bounds__(kRowThreads) block_output_loss_kernel(const float* __restrict__ h,
+                                                                         const uint16_t* __restrict__ branch,
+                                                                         const float* __restrict__ ref, int64_t count,
+                                                                         float scale, float* __restrict__ out,
+                                                                         uint16_t* __restrict__ d_out,
+                                                                         double* __restrict__ partials) {
+  Sum2 acc{0.f, 0.f};
+  const int64_t nvec = count / 8;
+  for (int64_t i = blockIdx.x * (int64_t)kRowThreads + threadIdx.x; i < nvec; i += (int64_t)gridDim.x * kRowThreads) {
+    const float4 h0 = reinterpret_cast<const float4*>(h)[2 * i], h1 = reinterpret_cast<const float4*>(h)[2 * i + 1];
+    const uint4 bw = reinterpret_cast<const uint4*>(branch)[i];
+    float o[8] = {h0.x + bf16lo_to_f32(bw.x), h0.y + bf16hi_to_f32(bw.x), h0.z + bf16lo_to_f32(bw.y),
+                  h0.w + bf16hi_to_f32(bw.y), h1.x + bf16lo_to_f32(bw.z), h1.y + bf16hi_to_f32(bw.z),
+                  h1.z + bf16lo_to_f32(bw.w), h1.w + bf16hi_to_f32(bw.w)};
+    if (out) {
+      reinterpret_cast<float4*>(out)[2 * i] = make_float4(o[0], o[1], o[2], o[3]);
+      reinterpret_cast<float4*>(out)[2 * i + 1] = make_float4(o[4], o[5], o[6], o[7]);
+    }
+    if (ref) {
+      const float4 r0 = reinterpret_cast<const float4*>(ref)[2 * i], r1 = reinterpret_cast<const float4*>(ref)[2 * i + 1];
+      const float rv[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
+      Sum2 local{0.f, 0.f};
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        o[q] -= rv[q];
+        sum2_add(local, o[q] * o[q]);
+      }
+      acc = sum2_merge(acc, local);
+      if (d_out) {
+        uint4 w;
+        w.x = pack_bf16x2(o[0] * scale, o[1] * scale);
+        w.y = pack_bf16x2(o[2] * scale, o[3] * scale);
+        w.z = pack_bf16x2(o[4] * scale, o[5] * scale);
+        w.w = pack_bf16x2(o[6] * scale, o[7] * scale);
+        reinterpret_cast<uint4*>(d_out)[i] = w;
+      }
+    }
+  }
+  if (!ref) return;
+  __shared__ Sum2 red[kRowThreads / 32];
+  acc = sum2_team(acc, 32);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    Sum2 v = threadIdx.x < kRowThreads / 32 ? red[threadIdx.x] : Sum2{0.f, 0.f};
+    v = sum2_team(v, 32);
+    if (threadIdx.x == 0) partials[blockIdx.x] = sum2_value(v);
+  }
+}
+
+// ---------------------------------------------------------------- attention
+constexpr int kBlk = 64;          // queries / keys per block
+constexpr int kAttnThreads = 128; // four warps of 16 rows
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                               uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// A shared-memory tile of 64 rows x HD bf16, rows padded by 16 bytes (conflict-free ldmatrix).
+template <int HD>
+struct Tile {
+  static constexpr int kStride = HD + 8;  // elements per row
+  static constexpr int kBytes = kBlk * kStride * 2;
+};
+
+// Rows row0.. row0 + 63 of a [rows, ld] bf16 matrix, columns col0 .. col0 + HD - 1, into a tile.
+template <int HD>
+__device__ __forceinline__ void load_tile(uint16_t* tile, const uint16_t* src, int64_t row0, int64_t ld,
+                                          int64_t col0) {
+  constexpr int kChunks = kBlk * HD / 8;  // 16-byte chunks
+  for (int c = threadIdx.x; c < kChunks; c += kAttnThreads) {
+    const int r = c / (HD / 8), k = (c % (HD / 8)) * 8;
+    *reinterpret_cast<uint4*>(tile + r * Tile<HD>::kStride + k) =
+        *reinterpret_cast<const uint4*>(src + (row0 + r) * ld + col0 + k);
+  }
+}
+
+// Address of the row that this lane supplies to an ldmatrix.x4 of a 16 x 16 fragment at
+// (row0, col0) of a tile: matrix m = lane / 8 covers rows + (m & 1) 8 when `row_from_bit0`
+// (A operands and transposed B operands), else + (m >> 1) 8 (B operands stored n-major), and
+// columns + the other bit times 8.
+template <int HD>
+__device__ __forceinline__ uint32_t frag_addr(uint32_t tile, int row0, int col0, bool row_from_bit0) {
+  const int lane = threadIdx.x & 31, m = lane >> 3, r = lane & 7;
+  const int dr = row_from_bit0 ? (m & 1) * 8 : (m >> 1) * 8;
+  const int dc = row_from_bit0 ? (m >> 1) * 8 : (m & 1) * 8;
+  return tile + static_cast<uint32_t>(((row0 + dr + r) * Tile<HD>::kStride + col0 + dc) * 2);
+}
+
+// Scores of this warp's 16 rows of A (tile rows a_row0..) against the 64 rows of B (an
+// n-major tile of keys), over HD columns: acc[n-tile 0..7][4].
+template <int HD>
+__device__ __forceinline__ void scores_16x64(float (&acc)[8][4], uint32_t a_tile, int a_row0, uint32_t b_tile) {
+#pragma unroll
+  for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) acc[nt][e] = 0.0f;
+#pragma unroll
+  for (int kk = 0; kk < HD / 16; ++kk) {
+    uint32_t a0, a1, a2, a3;
+    ldsm_x4(frag_addr<HD>(a_tile, a_row0, kk * 16, true), a0, a1, a2, a3);
+#pragma unroll
+    for (int p = 0; p < 4; ++p) {
+      uint32_t b0, b1, b2, b3;
+      ldsm_x4(frag_addr<HD>(b_tile, p * 16, kk * 16, false), b0, b1, b2, b3);
+      mma_bf16_16816(acc[2 * p], a0, a1, a2, a3, b0, b1);
+      mma_bf16_16816(acc[2 * p + 1], a0, a1, a2, a3, b2, b3);
+    }
+  }
+}
+
+// acc[d-tile 0 .. HD/8)[4] += P (16 x 64, as bf16 A fragments from fp32 values p[n-tile][4])
+// times the 64 x HD tile (rows = the contraction), read transposed.
+template <int HD>
+__device__ __forceinline__ void accum_pv(float (&acc)[HD / 8][4], const float (&p)[8][4], uint32_t v_tile) {
+#pragma unroll
+  for (int ks = 0; ks < 4; ++ks) {
+    const uint32_t a0 = pack_bf16x2(p[2 * ks][0], p[2 * ks][1]);
+    const uint32_t a1 = pack_bf16x2(p[2 * ks][2], p[2 * ks][3]);
+    const uint32_t a2 = pack_bf16x2(p[2 * ks + 1][0], p[2 * ks + 1][1]);
+    const uint32_t a3 = pack_bf16x2(p[2 * ks + 1][2], p[2 * ks + 1][3]);
+#pragma unroll
+    for (int dp = 0; dp < HD / 16; ++dp) {
+      uint32_t b0, b1, b2, b3;
+      ldsm_x4_t(frag_addr<HD>(v_tile, ks * 16, dp * 16, true), b0, b1, b2, b3);
+      mma_bf16_16816(acc[2 * dp], a0, a1, a2, a3, b0, b1);
+      mma_bf16_16816(acc[2 * dp + 1], a0, a1, a2, a3, b2, b3);
+    }
+  }
+}
+
+struct AttnArgs {
+  const uint16_t *q, *k, *v, *o, *dO;
+  uint16_t *out, *dq, *dk, *dv;
+  float *lse, *delta;
+  int32_t B, S, nh, nkv;
+  float scale_log2;  // log2(e) / sqrt(d)
+  float scale;       // 1 / sqrt(d)
+};
+
+// Forward: one CTA per (query block, head, sequence).  Rows g and g + 8 of the warp's 16 are
+// the thread's (lane / 4); its columns within each 8-wide n-tile are 2 (lane % 4) + {0, 1}.
+template <int HD>
+__global__ void __launch_bounds__(kAttnThreads) attn_fwd_kernel(const AttnArgs a) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  uint16_t* Qs = reinterpret_cast<uint16_t*>(smem);
+  uint16_t* Ks = Qs + kBlk * Tile<HD>::kStride;
+  uint16_t* Vs = Ks + kBlk * Tile<HD>::kStride;
+  const int nqb = a.S / kBlk;
+  const int qb = nqb - 1 - static_cast<int>(blockIdx.x);  // the longest rows first
+  const int h = blockIdx.y, b = blockIdx.z, hk = h / (a.nh / a.nkv);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
+  const int64_t tok0 = static_cast<int64_t>(b) * a.S;
+  load_tile<HD>(Qs, a.q, tok0 + qb * kBlk, static_cast<int64_t>(a.nh) * HD, static_cast<int64_t>(h) * HD);
+  float o[HD / 8][4];
+#pragma unroll
+  for (int i = 0; i < HD / 8; ++i)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) o[i][e] = 0.0f;
+  float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.0f, 0.0f};
+  const uint32_t qa = smem_u32(Qs), ka = smem_u32(Ks), va = smem_u32(Vs);
+  for (int kb = 0; kb <= qb; ++kb) {
+    __syncthreads();
+    load_tile<HD>(Ks, a.k, tok0 + kb * kBlk, static_cast<int64_t>(a.nkv) * HD, static_cast<int64_t>(hk) * HD);
+    load_tile<HD>(Vs, a.v, tok0 + kb * kBlk, static_cast<int64_t>(a.nkv) * HD, static_cast<int64_t>(hk) * HD);
+    __syncthreads();
+    float s[8][4];
+    scores_16x64<HD>(s, qa, warp * 16, ka);
+    float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        float v = s[nt][e] * a.scale_log2;
+        if (kb == qb) {
+          const int key = nt * 8 + 2 * t4 + (e & 1), qry = warp * 16 + g + (e >> 1) * 8;
+          if (key > qry) v = -INFINITY;
+        }
+        s[nt][e] = v;
+        mx[e >> 1] = fmaxf(mx[e >> 1], v);
+      }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      mx[i] = fmaxf(mx[i], __shfl_xor_sync(0xffffffffu, mx[i], 1));
+      mx[i] = fmaxf(mx[i], __shfl_xor_sync(0xffffffffu, mx[i], 2));
+    }
+    float corr[2], ls[2] = {0.0f, 0.0f};
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const float mn = fmaxf(mrow[i], mx[i]);
+      corr[i] = mrow[i] == -INFINITY ? 0.0f : exp2f(mrow[i] - mn);
+      mrow[i] = mn;
+    }
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float p = exp2f(s[nt][e] - mrow[e >> 1]);
+        s[nt][e] = p;
+        ls[e >> 1] += p;
+      }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) lrow[i] = lrow[i] * corr[i] + ls[i];
+#pragma unroll
+    for (int dn = 0; dn < HD / 8; ++dn) {
+      o[dn][0] *= corr[0];
+      o[dn][1] *= corr[0];
+      o[dn][2] *= corr[1];
+      o[dn][3] *= corr[1];
+    }
+    accum_pv<HD>(o, s, va);
+  }
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    lrow[i] += __shfl_xor_sync(0xffffffffu, lrow[i], 1);
+    lrow[i] += __shfl_xor_sync(0xffffffffu, lrow[i], 2);
+  }
+  const float inv[2] = {1.0f / lrow[0], 1.0f / lrow[1]};
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int64_t tok = tok0 + qb * kBlk + warp * 16 + g + 8 * i;
+    uint16_t* orow = a.out + tok * a.nh * HD + static_cast<int64_t>(h) * HD;
+#pragma unroll
+    for (int dn = 0; dn < HD / 8; ++dn)
+      *reinterpret_cast<uint32_t*>(orow + dn * 8 + 2 * t4) = pack_bf16x2(o[dn][2 * i] * inv[i], o[dn][2 * i + 1] * inv[i]);
+    if (t4 == 0)  // natural log-sum-exp of the scaled scores
+      a.lse[(static_cast<int64_t>(b) * a.nh + h) * a.S + qb * kBlk + warp * 16 + g + 8 * i] =
+          (mrow[i] + log2f(lrow[i])) * 0.69314718055994531f;
+  }
+}
+
+// delta[b, h, s] = sum over the head's columns of dO * O (one warp per token and head).
+template <int HD>
+__global__ void __launch_bounds__(kRowThreads) attn_delta_kernel(const AttnArgs a) {
+  const int64_t rows = static_cast<int64_t>(a.B) * a.S * a.nh;
+  const int lane = threadIdx.x & 31;
+  for (int64_t w = (blockIdx.x * (int64_t)kRowThreads + threadIdx.x) >> 5; w < rows;
+       w += ((int64_t)gridDim.x * kRowThreads) >> 5) {
+    const int64_t tok = w / a.nh;
+    const int h = static_cast<int>(w % a.nh);
+    const uint16_t* o = a.o + tok * a.nh * HD + static_cast<int64_t>(h) * HD;
+    const uint16_t* d = a.dO + tok * a.nh * HD + static_cast<int64_t>(h) * HD;
+    float s = 0.0f;
+    for (int i = lane; i < HD; i += 32) s = fmaf(bf16_at(o, i), bf16_at(d, i), s);
+#pragma unroll
+    for (int o2 = 16; o2 > 0; o2 >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o2);
+    if (lane == 0) {
+      const int64_t b = tok / a.S, sidx = tok % a.S;
+      a.delta[(b * a.nh + h) * a.S + sidx] = s;
+    }
+  }
+}
+
+// dQ: one CTA per (query block, head, sequence), over the key blocks up to the diagonal.
+template <int HD>
+__global__ void __launch_bounds__(kAttnThreads) attn_bwd_dq_kernel(const AttnArgs a) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  uint16_t* Qs = reinterpret_cast<uint16_t*>(smem);
+  uint16_t* Ds = Qs + kBlk * Tile<HD>::kStride;  // dO
+  uint16_t* Ks = Ds + kBlk * Tile<HD>::kStride;
+  uint16_t* Vs = Ks + kBlk * Tile<HD>::kStride;
+  const int nqb = a.S / kBlk;
+  const int qb = nqb - 1 - static_cast<int>(blockIdx.x);
+  const int h = blockIdx.y, b = blockIdx.z, hk = h / (a.nh / a.nkv);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
+  const int64_t tok0 = static_cast<int64_t>(b) * a.S;
+  const int64_t ldq = static_cast<int64_t>(a.nh) * HD, ldk = static_cast<int64_t>(a.nkv) * HD;
+  load_tile<HD>(Qs, a.q, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
+  load_tile<HD>(Ds, a.dO, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
+  float lse2[2], dl[2];  // this thread's two rows: log-sum-exp in log2 units, and delta
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int64_t idx = (static_cast<int64_t>(b) * a.nh + h) * a.S + qb * kBlk + warp * 16 + g + 8 * i;
+    lse2[i] = a.lse[idx] * 1.4426950408889634f;
+    dl[i] = a.delta[idx];
+  }
+  float dq[HD / 8][4];
+#pragma unroll
+  for (int i = 0; i < HD / 8; ++i)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) dq[i][e] = 0.0f;
+  const uint32_t qa = smem_u32(Qs), da = smem_u32(Ds), ka = smem_u32(Ks), va = smem_u32(Vs);
+  for (int kb = 0; kb <= qb; ++kb) {
+    __syncthreads();
+    load_tile<HD>(Ks, a.k, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
+    load_tile<HD>(Vs, a.v, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
+    __syncthreads();
+    float s[8][4], dp[8][4];
+    scores_16x64<HD>(s, qa, warp * 16, ka);   // Q K^T
+    scores_16x64<HD>(dp, da, warp * 16, va);  // dO V^T
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        float p = exp2f(s[nt][e] * a.scale_log2 - lse2[e >> 1]);
+        if (kb == qb) {
+          const int key = nt * 8 + 2 * t4 + (e & 1), qry = warp * 16 + g + (e >> 1) * 8;
+          if (key > qry) p = 0.0f;
+        }
+        s[nt][e] = p * (dp[nt][e] - dl[e >> 1]);  // dS
+      }
+    accum_pv<HD>(dq, s, ka);  // dS K
+  }
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int64_t tok = tok0 + qb * kBlk + warp * 16 + g + 8 * i;
+    uint16_t* row = a.dq + tok * ldq + static_cast<int64_t>(h) * HD;
+#pragma unroll
+    for (int dn = 0; dn < HD / 8; ++dn)
+      *reinterpret_cast<uint32_t*>(row + dn * 8 + 2 * t4) = pack_bf16x2(dq[dn][2 * i] * a.scale, dq[dn][2 * i + 1] * a.scale);
+  }
+}
+
+// dK, dV: one CTA per (key block, key/value head, sequence), over every query head of the
+// group and the query blocks from the diagonal on, 16 queries at a time.  Scores are formed
+// transposed (keys as rows) so that P^T and dS^T feed the A operand from registers.
+template <int HD>
+__global__ void __launch_bounds__(kAttnThreads) attn_bwd_dkdv_kernel(const AttnArgs a) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  uint16_t* Ks = reinterpret_cast<uint16_t*>(smem);
+  uint16_t* Vs = Ks + kBlk * Tile<HD>::kStride;
+  uint16_t* Qs = Vs + kBlk * Tile<HD>::kStride;
+  uint16_t* Ds = Qs + kBlk * Tile<HD>::kStride;
+  float* lse_s = reinterpret_cast<float*>(Ds + kBlk * Tile<HD>::kStride);  // [64], log2 units
+  float* dl_s = lse_s + kBlk;                                             // [64]
+  const int nqb = a.S / kBlk;
+  const int kb = static_cast<int>(blockIdx.x);  // the most query blocks first
+  const int hk = blockIdx.y, b = blockIdx.z, rep = a.nh / a.nkv;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
+  const int64_t tok0 = static_cast<int64_t>(b) * a.S;
+  const int64_t ldq = static_cast<int64_t>(a.nh) * HD, ldk = static_cast<int64_t>(a.nkv) * HD;
+  load_tile<HD>(Ks, a.k, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
+  load_tile<HD>(Vs, a.v, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
+  float dk[HD / 8][4], dv[HD / 8][4];
+#pragma unroll
+  for (int i = 0; i < HD / 8; ++i)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) dk[i][e] = dv[i][e] = 0.0f;
+  const uint32_t ka = smem_u32(Ks), va = smem_u32(Vs), qa = smem_u32(Qs), da = smem_u32(Ds);
+  for (int hh = 0; hh < rep; ++hh) {
+    const int h = hk * rep + hh;
+    for (int qb = kb; qb < nqb; ++qb) {
+      __syncthreads();
+      load_tile<HD>(Qs, a.q, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
+      load_tile<HD>(Ds, a.dO, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
+      if (threadIdx.x < kBlk) {
+        const int64_t idx = (static_cast<int64_t>(b) * a.nh + h) * a.S + qb * kBlk + threadIdx.x;
+        lse_s[threadIdx.x] = a.lse[idx] * 1.4426950408889634f;
+        dl_s[threadIdx.x] = a.delta[idx];
+      }
+      __syncthreads();
+#pragma unroll 1
+      for (int qs = 0; qs < kBlk / 16; ++qs) {
+        // S^T and dP^T of the warp's 16 keys against 16 queries: two n-tiles each
+        float st[2][4], dpt[2][4];
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) st[nt][e] = dpt[nt][e] = 0.0f;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
+          ldsm_x4(frag_addr<HD>(ka, warp * 16, kk * 16, true), a0, a1, a2, a3);
+          ldsm_x4(frag_addr<HD>(qa, qs * 16, kk * 16, false), b0, b1, b2, b3);
+          mma_bf16_16816(st[0], a0, a1, a2, a3, b0, b1);
+          mma_bf16_16816(st[1], a0, a1, a2, a3, b2, b3);
+          ldsm_x4(frag_addr<HD>(va, warp * 16, kk * 16, true), a0, a1, a2, a3);
+          ldsm_x4(frag_addr<HD>(da, qs * 16, kk * 16, false), b0, b1, b2, b3);
+          mma_bf16_16816(dpt[0], a0, a1, a2, a3, b0, b1);
+          mma_bf16_16816(dpt[1], a0, a1, a2, a3, b2, b3);
+        }
+        float pt[2][4], dst[2][4];
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int qry = qs * 16 + nt * 8 + 2 * t4 + (e & 1);  // within the query block
+            const int key = warp * 16 + g + (e >> 1) * 8;          // within the key block
+            float p = exp2f(st[nt][e] * a.scale_log2 - lse_s[qry]);
+            if (qb == kb && key > qry) p = 0.0f;
+            pt[nt][e] = p;
+            dst[nt][e] = p * (dpt[nt][e] - dl_s[qry]);
+          }
+        // dV += P^T dO and dK += dS^T Q over these 16 queries (one k-step)
+        const uint32_t p0 = pack_bf16x2(pt[0][0], pt[0][1]), p1 = pack_bf16x2(pt[0][2], pt[0][3]);
+        const uint32_t p2 = pack_bf16x2(pt[1][0], pt[1][1]), p3 = pack_bf16x2(pt[1][2], pt[1][3]);
+        const uint32_t s0 = pack_bf16x2(dst[0][0], dst[0][1]), s1 = pack_bf16x2(dst[0][2], dst[0][3]);
+        const uint32_t s2 = pack_bf16x2(dst[1][0], dst[1][1]), s3 = pack_bf16x2(dst[1][2], dst[1][3]);
+#pragma unroll
+        for (int dp = 0; dp < HD / 16; ++dp) {
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_t(frag_addr<HD>(da, qs * 16, dp * 16, true), b0, b1, b2, b3);
+          mma_bf16_16816(dv[2 * dp], p0, p1, p2, p3, b0, b1);
+          mma_bf16_16816(dv[2 * dp + 1], p0, p1, p2, p3, b2, b3);
+          ldsm_x4_t(frag_addr<HD>(qa, qs * 16, dp * 16, true), b0, b1, b2, b3);
+          mma_bf16_16816(dk[2 * dp], s0, s1, s2, s3, b0, b1);
+          mma_bf16_16816(dk[2 * dp + 1], s0, s1, s2, s3, b2, b3);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int64_t tok = tok0 + kb * kBlk + warp * 16 + g + 8 * i;
+    uint16_t* krow = a.dk + tok * ldk + static_cast<int64_t>(hk) * HD;
+    uint16_t* vrow = a.dv + tok * ldk + static_cast<int64_t>(hk) * HD;
+#pragma unroll
+    for (int dn = 0; dn < HD / 8; ++dn) {
+      *reinterpret_cast<uint32_t*>(krow + dn * 8 + 2 * t4) = pack_bf16x2(dk[dn][2 * i] * a.scale, dk[dn][2 * i + 1] * a.scale);
+      *reinterpret_cast<uint32_t*>(vrow + dn * 8 + 2 * t4) = pack_bf16x2(dv[dn][2 * i], dv[dn][2 * i + 1]);
+    }
+  }
+}
+
+int elem_grid(int64_t n) {
+  int64_t b = (n + kRowThreads - 1) / kRowThreads;
+  if (b < 1) b = 1;
+  if (b > 152 * 16) b = 152 * 16;
+  return static_cast<int>(b);
+}
+
+template <int HD>
+cudaError_t attn_launch(const AttnArgs& a, bool backward, cudaStream_t st) {
+  const dim3 grid(static_cast<unsigned>(a.S / kBlk), static_cast<unsigned>(a.nh), static_cast<unsigned>(a.B));
+  if (!backward) {
+    const int smem = 3 * Tile<HD>::kBytes;
+    cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    attn_fwd_kernel<HD><<<grid, kAttnThreads, smem, st>>>(a);
+    return cudaGetLastError();
+  }
+  const int64_t rows = static_cast<int64_t>(a.B) * a.S * a.nh;
+  attn_delta_kernel<HD><<<elem_grid(rows * 32), kRowThreads, 0, st>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int smem_q = 4 * Tile<HD>::kBytes;
+  e = cudaFuncSetAttribute(attn_bwd_dq_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_q);
+  if (e != cudaSuccess) return e;
+  attn_bwd_dq_kernel<HD><<<grid, kAttnThreads, smem_q, st>>>(a);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  const int smem_k = 4 * Tile<HD>::kBytes + 2 * kBlk * static_cast<int>(sizeof(float));
+  e = cudaFuncSetAttribute(attn_bwd_dkdv_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_k);
+  if (e != cudaSuccess) return e;
+  const dim3 gk(static_cast<unsigned>(a.S / kBlk), static_cast<unsigned>(a.nkv), static_cast<unsigned>(a.B));
+  attn_bwd_dkdv_kernel<HD><<<gk, kAttnThreads, smem_k, st>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_rmsnorm_fwd(const void* x, bool x_f32, const void* res, const float* gamma, int64_t T, int64_t H,
+                               float eps, float* h_out, void* z, float* r, cudaStream_t st) {
+  if (x_f32)
+    rmsnorm_fwd_kernel<float><<<static_cast<unsigned>(T), kRowThreads, 0, st>>>(
+        static_cast<const float*>(x), static_cast<const uint16_t*>(res), gamma, H, eps, h_out,
+        static_cast<uint16_t*>(z), r);
+  else
+    rmsnorm_fwd_kernel<uint16_t><<<static_cast<unsigned>(T), kRowThreads, 0, st>>>(
+        static_cast<const uint16_t*>(x), static_cast<const uint16_t*>(res), gamma, H, eps, h_out,
+        static_cast<uint16_t*>(z), r);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rmsnorm_bwd(const void* x, bool x_f32, const float* gamma, const float* r, const void* dy,
+                               const void* dy2, const void* dres, int64_t T, int64_t H, void* dx, cudaStream_t st) {
+  const auto* dyp = static_cast<const uint16_t*>(dy);
+  const auto* dy2p = static_cast<const uint16_t*>(dy2);
+  const auto* drp = static_cast<const uint16_t*>(dres);
+  if (x_f32)
+    rmsnorm_bwd_kernel<float><<<static_cast<unsigned>(T), kRowThreads, 0, st>>>(
+        static_cast<const float*>(x), gamma, r, dyp, dy2p, drp, H, static_cast<uint16_t*>(dx));
+  else
+    rmsnorm_bwd_kernel<uint16_t><<<static_cast<unsigned>(T), kRowThreads, 0, st>>>(
+        static_cast<const uint16_t*>(x), gamma, r, dyp, dy2p, drp, H, static_cast<uint16_t*>(dx));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rope(void* x, int64_t T, int64_t S, int32_t nheads, int32_t d, float base, int32_t inverse,
+                        cudaStream_t st) {
+  rope_kernel<<<elem_grid(T * nheads * (d / 2)), kRowThreads, 0, st>>>(static_cast<uint16_t*>(x), T, S, nheads, d,
+                                                                        log2f(base), inverse);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_swiglu(const void* gt, const void* u, const void* dm, int64_t n, void* out, void* dgt, void* du,
+                          cudaStream_t st) {
+  if (!dm)
+    swiglu_fwd_kernel<<<elem_grid(n), kRowThreads, 0, st>>>(static_cast<const uint16_t*>(gt),
+                                                             static_cast<const uint16_t*>(u), n,
+                                                             static_cast<uint16_t*>(out));
+  else
+    swiglu_bwd_kernel<<<elem_grid(n), kRowThreads, 0, st>>>(
+        static_cast<const uint16_t*>(gt), static_cast<const uint16_t*>(u), static_cast<const uint16_t*>(dm), n,
+        static_cast<uint16_t*>(dgt), static_cast<uint16_t*>(du));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_block_output_loss(const float* h, const void* branch, const float* ref, int64_t count,
+                                     int32_t reduction, float* out, void* d_out, float* loss_out, double* partials,
+                                     cudaStream_t st) {
+  const int nb = ref ? recon_loss_blocks(count) : elem_grid(count / 8);
+  const double inv = reduction == 0 ? 1.0 / static_cast<double>(count) : 1.0;
+  block_output_loss_kernel<<<nb, kRowThreads, 0, st>>>(h, static_cast<const uint16_t*>(branch), ref, count,
+                                                        static_cast<float>(2.0 * inv), out,
+                                                        static_cast<uint16_t*>(d_out), partials);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || !ref) return e;
+  return launch_loss_final(partials, nb, inv, loss_out, st);
+}
+
+cudaError_t launch_attention(const AttnIo& io, int32_t B, int32_t S, int32_t nh, int32_t nkv, int32_t d, bool backward,
+                             cudaStream_t st) {
+  AttnArgs a{};
+  a.q = static_cast<const uint16_t*>(io.q);
+  a.k = static_cast<const uint16_t*>(io.k);
+  a.v = static_cast<const uint16_t*>(io.v);
+  a.o = static_cast<const uint16_t*>(io.o);
+  a.dO = static_cast<const uint16_t*>(io.dO);
+  a.out = static_cast<uint16_t*>(io.out);
+  a.dq = static_cast<uint16_t*>(io.dq);
+  a.dk = static_cast<uint16_t*>(io.dk);
+  a.dv = static_cast<uint16_t*>(io.dv);
+  a.lse = io.lse;
+  a.delta = io.delta;
+  a.B = B;
+  a.S = S;
+  a.nh = nh;
+  a.nkv = nkv;
+  a.scale = 1.0f / sqrtf(static_cast<float>(d));
+  a.scale_log2 = a.scale * 1.4426950408889634f;
+  return d == 128 ? attn_launch<128>(a, backward, st) : attn_launch<64>(a, backward, st);
+}
+
+}  // namespace catq

@@ -157,6 +157,32 @@ cudaError_t launch_tc_fwd(const LayerDev& L, StepScalars sc, const void* X, int6
 cudaError_t launch_tc_dx(const LayerDev& L, StepScalars sc, const void* dY, int64_t M, void* dX, cudaStream_t st);
 cudaError_t launch_tc_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M,
                          const TcPlan& plan, float* partials, cudaStream_t st);
+// block.cu (the layers between the linears of a decoder block; bf16 activations)
+// x (fp32 or bf16) + res (bf16, nullable) -> h_out (fp32, nullable), z (bf16), r.
+cudaError_t launch_rmsnorm_fwd(const void* x, bool x_f32, const void* res, const float* gamma, int64_t T, int64_t H,
+                               float eps, float* h_out, void* z, float* r, cudaStream_t st);
+cudaError_t launch_rmsnorm_bwd(const void* x, bool x_f32, const float* gamma, const float* r, const void* dy,
+                               const void* dy2, const void* dres, int64_t T, int64_t H, void* dx, cudaStream_t st);
+cudaError_t launch_rope(void* x, int64_t T, int64_t S, int32_t nheads, int32_t d, float base, int32_t inverse,
+                        cudaStream_t st);
+// dm == nullptr: out = silu(gt) u; else dgt, du = the backward from dm.
+cudaError_t launch_swiglu(const void* gt, const void* u, const void* dm, int64_t n, void* out, void* dgt, void* du,
+                          cudaStream_t st);
+// out = h + branch (fp32; nullable); with ref: loss_out = Eq. 7 loss, d_out (bf16, nullable);
+// partials: recon_loss_blocks(count) doubles.  count % 8 == 0.
+cudaError_t launch_block_output_loss(const float* h, const void* branch, const float* ref, int64_t count,
+                                     int32_t reduction, float* out, void* d_out, float* loss_out, double* partials,
+                                     cudaStream_t st);
+struct AttnIo {
+  const void *q, *k, *v;
+  const void *o, *dO;  // backward only
+  void* out;           // forward only
+  void *dq, *dk, *dv;  // backward only
+  float* lse;
+  float* delta;        // backward scratch
+};
+cudaError_t launch_attention(const AttnIo& io, int32_t B, int32_t S, int32_t nh, int32_t nkv, int32_t d, bool backward,
+                             cudaStream_t st);
 // Status word latched by device-side bounded waits (0 = none); read-and-clear.
 cudaError_t read_and_clear_device_status(int32_t* out);
 bool tensor_map_encoder_available();

@@ -1018,3 +1018,42 @@ def test_rmsnorm_closed_forms():
         xm[i, j] -= h
         fd = ((O.rmsnorm(xp, gamma, 1e-5)[0] - O.rmsnorm(xm, gamma, 1e-5)[0]) * dy).sum() / (2 * h)
         assert dx[i, j] == pytest.approx(fd, rel=1e-6)
+
+
+def test_attention_logsumexp_closed_form_and_softmax():
+    """With q = 0 every allowed score is 0, so query s's normaliser is log(s + 1); on random
+    inputs exp(score - lse) over the allowed keys must be ``attention``'s probabilities."""
+    B, S, nh, nkv, d = 2, 7, 4, 2, 8
+    r = np.random.default_rng(81)
+    k = r.standard_normal((B * S, nkv * d))
+    lse0 = O.attention_logsumexp(np.zeros((B * S, nh * d)), k, B, S, nh, nkv, d)
+    np.testing.assert_allclose(lse0, np.broadcast_to(np.log(np.arange(1, S + 1)), (B, nh, S)), rtol=0, atol=1e-14)
+    q = r.standard_normal((B * S, nh * d))
+    lse = O.attention_logsumexp(q, k, B, S, nh, nkv, d)
+    v = r.standard_normal((B * S, nkv * d))
+    _, p = O.attention(q, k, v, B, S, nh, nkv, d)
+    qh = q.reshape(B, S, nh, d)
+    kh = np.repeat(k.reshape(B, S, nkv, d), nh // nkv, axis=2)
+    for b, h, i, j in [(0, 0, 3, 1), (1, 3, 6, 6), (1, 2, 0, 0), (0, 1, 5, 2)]:
+        score = qh[b, i, h] @ kh[b, j, h] / np.sqrt(d)
+        assert abs(np.exp(score - lse[b, h, i]) - p[b, h, i, j]) < 1e-14
+    assert np.all(p[0, 0][np.triu_indices(S, 1)] == 0.0)
+
+
+def test_swiglu_gradients_match_central_differences():
+    r = np.random.default_rng(82)
+    gt, u, dm = (r.standard_normal((3, 5)) * 2.0 for _ in range(3))
+    d_gt, d_u = O.swiglu_bwd(gt, u, dm)
+    h = 1e-6
+    num_gt = (np.sum(dm * O.swiglu(gt + h, u)) - np.sum(dm * O.swiglu(gt - h, u))) / (2 * h)
+    num_u = (np.sum(dm * O.swiglu(gt, u + h)) - np.sum(dm * O.swiglu(gt, u - h))) / (2 * h)
+    # the elementwise map: perturbing everything at once sums the elementwise derivatives
+    assert abs(num_gt - d_gt.sum()) < 1e-7 * max(1.0, abs(num_gt))
+    assert abs(num_u - d_u.sum()) < 1e-7 * max(1.0, abs(num_u))
+    e = np.zeros_like(gt)
+    e[1, 2] = h
+    one = (np.sum(dm * O.swiglu(gt + e, u)) - np.sum(dm * O.swiglu(gt - e, u))) / (2 * h)
+    assert abs(one - d_gt[1, 2]) < 1e-7 * max(1.0, abs(one))
+    # silu(0) = 0 and silu's slope at 0 is 1/2
+    np.testing.assert_allclose(O.swiglu(np.zeros(2), np.ones(2)), 0.0, atol=0)
+    np.testing.assert_allclose(O.swiglu_bwd(np.zeros(1), np.ones(1), np.ones(1))[0], 0.5, rtol=1e-15)
