@@ -64,6 +64,10 @@ def parse(argv=None):
     p.add_argument("--no-also", action="store_true", help="skip the secondary workloads and phase")
     p.add_argument("--streams", type=int, default=4,
                    help="CUDA streams the block's linears are spread over (independent problems)")
+    p.add_argument("--only", default=None, choices=["moe", "decode_b1", "decode_b8", "block_window"],
+                   help="run one secondary measurement alone and print its result (for profiling)")
+    p.add_argument("--moe-experts", type=int, default=None,
+                   help="with --only moe: fewer experts (same shape and routing law; for profiling)")
     p.add_argument("--linear", default=None,
                    help="run only this linear of the block (single-kernel profiling of one layer)")
     return p.parse_args(argv)
@@ -750,12 +754,16 @@ def measure_fig_error(C, torch, wl, dev, s0, epochs=20, batches=3, rows=2048, lr
     return res
 
 
-def measure_moe(C, torch, dev, peaks, world, s, steps=5, warmup=2):
+def measure_moe(C, torch, dev, peaks, world, s, steps=5, warmup=2, experts=None):
     """One calibration step of the Qwen3-235B-shaped MoE layer: gate/up/down of all 128
     experts over 8192 tokens routed top-8 (65,536 expert-sorted rows, Zipf(1.1) loads) through
     the grouped calls (stats once; per step forward, loss, backward, factor update, pack).  Weights and
-    activations are drawn on the device (seeded); value = sum 6 M_e N K / step time."""
+    activations are drawn on the device (seeded); value = sum 6 M_e N K / step time.
+    `experts` (profiling only) keeps the expert shape and routing law with fewer experts and
+    proportionally fewer tokens, so that a capture holds less device memory."""
     wl = syn.WORKLOADS["c5_qwen3_235b_moe"]
+    if experts:
+        wl = dataclasses.replace(wl, experts=int(experts), tokens=wl.tokens * int(experts) // wl.experts)
     token_of_row, off = syn.moe_routing(wl, seed=0)
     R, E, g = int(off[-1]), wl.experts, wl.g
     gen = torch.Generator(device=dev)
@@ -911,9 +919,34 @@ def measure_e2e(args, C, torch, st, step, barrier, flops_step, world, dev):
             "pipeline": "inputs double-buffered: step t + 1's copies overlap step t's kernels"}
 
 
+def run_only(args):
+    """One secondary measurement alone on GPU 0 (used by the ncu commands under profiles/)."""
+    import torch
+
+    from paper_2606_26650_gb300 import catq as C
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    peaks = measured_peaks()
+    wl = syn.WORKLOADS[DEFAULT_WORKLOAD]
+
+    def barrier():
+        torch.cuda.synchronize()
+
+    if args.only == "moe":
+        r = measure_moe(C, torch, dev, peaks, 1, args.s, steps=args.steps, warmup=args.warmup,
+                        experts=args.moe_experts)
+    elif args.only.startswith("decode_b"):
+        r = measure_decode(C, torch, wl, dev, peaks, rows=int(args.only[len("decode_b"):]), steps=args.steps)
+    else:
+        r = measure_block_window(C, torch, wl, dev, peaks, 1, args.s, barrier, steps=args.steps, warmup=args.warmup)
+    print(json.dumps({"only": args.only, **r}), flush=True)
+
+
 def main():
     args = parse()
-    if args.impl == "reference":
+    if args.only:
+        run_only(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_ours(args)

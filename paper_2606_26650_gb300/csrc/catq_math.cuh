@@ -319,24 +319,68 @@ __device__ __forceinline__ void grad_element(float G, float w, const GroupConst&
 // resolution of the O(1) terms they join (symmetrically for x < 0), so with the near term
 // y = s|x| - D alone:
 //   f'/k = sech^2 y,   (df/dDelta)/k = -sign(x) sech^2 y,
-//   SOFT T = f = sign(x) (1 + tanh y) / (2 tanh s)     (the producer's one-tanh form),
-// one exponential e = exp(-2|y|) and one reciprocal per element instead of two of each.
+//   SOFT T = f = sign(x) (1 + tanh y) / (2 tanh s)     (the producer's one-tanh form).
 constexpr float kOneExpD = 9.0f;
 
-template <bool MU = false>
-__device__ __forceinline__ void grad_element_1exp(float G, float w, const GroupConst& c, float s, float D,
-                                                  float inv_2tanh_s, float k, int32_t phase, GradSums& acc,
-                                                  float inv_k = 0.0f) {
+// That near-term form through the logistic function, for the dW epilogue, which runs it on
+// every weight: with y = s|x| - D,
+//   exp(-2y) = 2^(|x| c1 + c2),   c1 = -2 s log2(e),  c2 = 2 D log2(e),
+//   p = 1 + tanh y = 2 / (1 + exp(-2y)),   sech^2 y = (1 - tanh y)(1 + tanh y) = p^2 exp(-2y),
+//   SOFT T = sign(x) p / (2 tanh s),
+// one exp2, one reciprocal and a handful of multiply-adds per element (the phase is a template
+// argument, decided once per chunk).  The exponent is capped at 126, reached only far inside
+// the threshold where sech^2 y is below fp32 resolution anyway, so exp(-2y) stays finite.
+struct OneExp {
+  float c1, c2;
+};
+
+__device__ __forceinline__ OneExp one_exp_consts(float s, float D) {
+  constexpr float kLog2e = 1.4426950408889634f;
+  return OneExp{-2.0f * kLog2e * s, 2.0f * kLog2e * D};
+}
+
+__device__ __forceinline__ float ex2_approx(float a) {
+  float r;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(a));
+  return r;
+}
+
+__device__ __forceinline__ float rcp_approx(float a) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(a));
+  return r;
+}
+
+template <bool MU, bool SOFT>
+__device__ __forceinline__ void grad_element_logistic(float G, float w, const GroupConst& c, const OneExp& oe,
+                                                      float inv_2tanh_s, float k, GradSums& acc, float inv_k) {
   const float x = what(w, c);
-  const float y = fabsf(s * x) - D;
-  const float e = __expf(-2.0f * fabsf(y));
-  const float rcp = __fdividef(1.0f, 1.0f + e);
-  const float s2 = 4.0f * e * rcp * rcp;                 // sech^2 y
-  const float T = (phase == PHASE_SOFT) ? copysignf(1.0f + copysignf((1.0f - e) * rcp, y), x) * inv_2tanh_s
-                                        : hard_q(x, c.delta);
+  const float e = ex2_approx(fminf(fmaf(fabsf(x), oe.c1, oe.c2), 126.0f));
+  const float p = rcp_approx(fmaf(e, 0.5f, 0.5f));
+  const float s2 = p * p * e;
+  const float T = SOFT ? copysignf(p * inv_2tanh_s, x) : hard_q(x, c.delta);
   acc.smu = fmaf(G, MU ? s2 - inv_k : s2, acc.smu);
-  acc.salpha = fmaf(G, T - x * k * s2, acc.salpha);
+  acc.salpha = fmaf(G, fmaf(-x * k, s2, T), acc.salpha);
   acc.sdelta = fmaf(G, copysignf(s2, -x), acc.sdelta);
+}
+
+// 32 consecutive elements of one row: fp32 accumulator values g[0..31] and the bf16 weights
+// packed two per word in w[0..3].
+template <bool MU, bool SOFT>
+__device__ __forceinline__ void grad_chunk_logistic(const uint32_t (&g)[32], const uint4 (&w)[4], const GroupConst& c,
+                                                    const OneExp& oe, float inv_2tanh_s, float k, GradSums& acc,
+                                                    float inv_k) {
+#pragma unroll
+  for (int v = 0; v < 4; ++v) {
+    const uint32_t w4[4] = {w[v].x, w[v].y, w[v].z, w[v].w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      grad_element_logistic<MU, SOFT>(__uint_as_float(g[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), c, oe, inv_2tanh_s,
+                                      k, acc, inv_k);
+      grad_element_logistic<MU, SOFT>(__uint_as_float(g[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), c, oe,
+                                      inv_2tanh_s, k, acc, inv_k);
+    }
+  }
 }
 
 }  // namespace catq

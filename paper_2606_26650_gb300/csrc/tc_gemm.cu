@@ -548,7 +548,11 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
         tc_fence_after();
         return true;
       };
+      // An accumulator whose rows all lie past the tile's last row (an expert's short last M
+      // block, or a ragged M) gets no MMAs; the epilogue stores nothing from it.
+      bool live[NACC];
       auto issue = [&](uint32_t qq, int acc, bool first) {  // one accumulator's MMAs of stage qq
+        if (!live[acc]) return;
         const uint32_t aa = a_base + (qq % SA) * Cfg::kABytes, ww = w_base + (qq % SW) * Cfg::kWBytes;
 #pragma unroll
         for (int kk = 0; kk < BK / 16; ++kk) {
@@ -572,6 +576,12 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
         else umma_commit_pair_mask(tmem_full0 + 8u * acc, pair_mask);
       };
       for (int t = cluster; ok && t < num_tiles; t += nclusters, ++it) {
+        {
+          const TileInfo ti = tile_info(args, t, Cfg::kTileRows * PAIRS);
+          const int64_t prow = ti.row0 + pair * Cfg::kTileRows;
+#pragma unroll
+          for (int acc = 0; acc < NACC; ++acc) live[acc] = prow + acc * Cfg::kRowsPerAcc < ti.row_end;
+        }
         const uint32_t ep = (it & 1u) ^ 1u;  // the epilogue has drained the previous tile's accumulator
         // head: accumulator 0 over stages 0 .. J-1
         if (!mbar_wait(tmem_empty0, ep, wc)) break;
@@ -1043,31 +1053,23 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
       const int split = t / tiles_per_split, r = t % tiles_per_split;
       const int k_blk = r % args.num_k_tiles, n_blk = r / args.num_k_tiles;
       // the tile's layer: the dense one, or (grouped) its expert's slice of the stacked layer
-      LayerDev L = args.L;
+      // (grouped: the expert's weights and per-group arrays start e N K elements and e G
+      // groups after expert 0's; its group j is group jbase + j of the stacked arrays)
+      const LayerDev& L = args.L;
       int64_t slab = split;  // which [3][N][K/P] partial block the tile writes
+      const uint16_t* W = static_cast<const uint16_t*>(L.W);
+      int64_t jbase = 0;
       if constexpr (NE > 1) {
         const int64_t e = gm.expert[split];
-        const int64_t G = L.N * L.groups_per_row;
-        L.W = static_cast<const uint16_t*>(L.W) + e * L.N * L.K;
-        L.mu0 += e * G;
-        L.alpha0 += e * G;
-        L.delta0 += e * G;
-        L.d_mu += e * G;
-        L.d_alpha += e * G;
-        L.d_delta += e * G;
+        W += e * L.N * L.K;
+        jbase = e * L.N * L.groups_per_row;
         slab = e;
       }
-      const uint16_t* W = static_cast<const uint16_t*>(L.W);
       const uint32_t buf = it & 1u;
-      if (!mbar_wait(tmem_full0 + 8u * buf, (it >> 1) & 1u, wc)) break;
-      tc_fence_after();
       const int64_t n = (int64_t)n_blk * Cfg::kTileRows + cta * 128 + q * 32 + lane;
       const bool row_ok = n < L.N;
       float* out = args.part + slab * 3 * plane;
-      int64_t cur_j = -1;
-      GroupConst gc{};
       GradSums acc{0.f, 0.f, 0.f};
-      // The 32 W values of a chunk are loaded one chunk ahead of the arithmetic.
       constexpr int kChunks = (BN / 2) / 32;
       const int64_t k0 = (int64_t)k_blk * BN + half * (BN / 2);
       auto load_w = [&](int c, uint4 (&dst)[4]) {
@@ -1078,36 +1080,43 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
           for (int v = 0; v < 4; ++v) dst[v] = __ldg(wp + v);
         }
       };
-      uint4 wcur[4], wnext[4];
+      // The first two chunks' weights and the group constants the tile starts in are requested
+      // before the wait for the accumulator, so their latency overlaps the tile's MMAs; later
+      // chunks' weights are loaded two chunks ahead of the arithmetic.
+      uint4 wcur[4], wnext[4], wnext2[4];
       load_w(0, wcur);
+      if (kChunks > 1) load_w(1, wnext);
+      int64_t cur_j = -1;
+      GroupRaw graw{};
+      if (row_ok && k0 < L.K) {
+        cur_j = n * L.groups_per_row + k0 / L.g;
+        graw = group_raw(L, jbase + cur_j);
+      }
+      if (!mbar_wait(tmem_full0 + 8u * buf, (it >> 1) & 1u, wc)) break;
+      tc_fence_after();
+      GroupConst gc = group_const(graw);
 #pragma unroll 1
       for (int c = 0; c < kChunks; ++c) {
         const int col = half * (BN / 2) + c * 32;
         uint32_t rg[32];
         tmem_ld32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + buf * BN + col, rg);
-        if (c + 1 < kChunks) load_w(c + 1, wnext);
+        if (c + 2 < kChunks) load_w(c + 2, wnext2);
         tmem_ld_wait();
         const int64_t k = k0 + c * 32;
         if (row_ok && k < L.K) {
           const int64_t j = n * L.groups_per_row + k / L.g;
           if (j != cur_j) {
-            gc = group_const(L, j);
+            gc = group_const(L, jbase + j);
             cur_j = j;
           }
           const float D = args.sc.s * gc.delta;
           if (gc.alpha != 0.0f && D >= kOneExpD) {
             // one exponential per weight (the far tanh term is 1 to fp32 resolution)
-#pragma unroll
-            for (int v = 0; v < 4; ++v) {
-              const uint32_t w4[4] = {wcur[v].x, wcur[v].y, wcur[v].z, wcur[v].w};
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                grad_element_1exp<MU>(__uint_as_float(rg[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), gc, args.sc.s, D,
-                                      args.sc.inv_2tanh_s, k_sc, args.sc.phase, acc, inv_k);
-                grad_element_1exp<MU>(__uint_as_float(rg[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), gc, args.sc.s,
-                                      D, args.sc.inv_2tanh_s, k_sc, args.sc.phase, acc, inv_k);
-              }
-            }
+            const OneExp oe = one_exp_consts(args.sc.s, D);
+            if (args.sc.phase == PHASE_SOFT)
+              grad_chunk_logistic<MU, true>(rg, wcur, gc, oe, args.sc.inv_2tanh_s, k_sc, acc, inv_k);
+            else
+              grad_chunk_logistic<MU, false>(rg, wcur, gc, oe, args.sc.inv_2tanh_s, k_sc, acc, inv_k);
           } else if (gc.alpha != 0.0f) {
 #pragma unroll
             for (int v = 0; v < 4; ++v) {
@@ -1130,7 +1139,10 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
           }
         }
 #pragma unroll
-        for (int v = 0; v < 4; ++v) wcur[v] = wnext[v];
+        for (int v = 0; v < 4; ++v) {
+          wcur[v] = wnext[v];
+          wnext[v] = wnext2[v];
+        }
       }
       tc_fence_before();
       __syncwarp();
