@@ -64,7 +64,8 @@ def parse(argv=None):
     p.add_argument("--no-also", action="store_true", help="skip the secondary workloads and phase")
     p.add_argument("--streams", type=int, default=4,
                    help="CUDA streams the block's linears are spread over (independent problems)")
-    p.add_argument("--only", default=None, choices=["moe", "decode_b1", "decode_b8", "block_window"],
+    p.add_argument("--only", default=None,
+                   choices=["moe", "decode_b1", "decode_b8", "decode_b1_staged", "block_window"],
                    help="run one secondary measurement alone and print its result (for profiling)")
     p.add_argument("--moe-experts", type=int, default=None,
                    help="with --only moe: fewer experts (same shape and routing law; for profiling)")
@@ -516,6 +517,7 @@ def run_ours(args):
         also[f"{wl.name}/decode_b1"] = measure_decode(C, torch, wl, dev, peaks, rows=1)
         also[f"{wl.name}/decode_b8"] = measure_decode(C, torch, wl, dev, peaks, rows=8)
         also[f"{wl.name}/decode_b1_mu"] = measure_decode(C, torch, wl, dev, peaks, rows=1, with_mu=True)
+        also[f"{wl.name}/decode_b1_staged"] = measure_decode(C, torch, wl, dev, peaks, rows=1, staged=True)
         also["c5_qwen3_235b_moe/soft"] = measure_moe(C, torch, dev, peaks, world, args.s)
         also[f"{wl.name}/fig_error_k_proj"] = measure_fig_error(C, torch, wl, dev, args.s)
         if wl.name == "c3_llama3_8b_block" and not args.linear:
@@ -633,13 +635,15 @@ def measure_block_window(C, torch, wl, dev, peaks, world, s, barrier, steps=5, w
 DECODE_GROUPS = (("q_proj", "k_proj", "v_proj"), ("o_proj",), ("gate_proj", "up_proj"), ("down_proj",))
 
 
-def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20, with_mu=False):
+def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20, with_mu=False, staged=False):
     """Inference with the deployed form of every linear of `blocks` blocks shaped like `wl`,
     for `rows` token rows: one decode step reads every layer's 2-bit codes and group scales
-    (and group offsets, `with_mu`) once (working set far beyond L2).  Each block runs as four
-    launches of catq_ternary_infer_batched, one per set of linears whose inputs are
-    independent (DECODE_GROUPS), in block order, as a decode step must.  The step's launches
-    are captured in a CUDA graph and replayed; value = algorithmic bytes / time."""
+    (and group offsets, `with_mu`) once (working set far beyond L2), layer sets in block order
+    (DECODE_GROUPS: q/k/v, o, gate/up, down), as a decode step must.
+    staged: the layer sets are the stages of catq_ternary_infer_staged, four blocks (28 layers,
+    16 stages) per cooperative launch; otherwise one catq_ternary_infer_batched launch per set,
+    captured in a CUDA graph and replayed.  value = algorithmic bytes / time."""
+    import ctypes
     gen = torch.Generator(device=dev)
     gen.manual_seed(0)
     launches, nbytes, g = [], 0, wl.g
@@ -659,23 +663,48 @@ def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20, with_m
                 nbytes += codes.numel() + alpha.numel() * 4 + X.numel() * 2 + Y.numel() * 2
                 nbytes += 0 if mu is None else mu.numel() * 4
             launches.append(group)
-    side = torch.cuda.Stream(device=dev)
-    side.wait_stream(torch.cuda.current_stream())
-    with torch.cuda.stream(side):  # warm-up outside the capture
-        for group in launches:
-            C.catq_ternary_infer_batched(group, g)
-    torch.cuda.current_stream().wait_stream(side)
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph):
-        for group in launches:
-            C.catq_ternary_infer_batched(group, g)
+    if staged:
+        per_call = 4  # blocks per launch: 28 layers, 16 stages
+        calls = []
+        sync = torch.zeros(C.catq_ternary_infer_sync_bytes() // 4, dtype=torch.int32, device=dev)
+        groups_per_call = per_call * len(DECODE_GROUPS)
+        for c0 in range(0, len(launches), groups_per_call):
+            layers, stages = [], []
+            for si, group in enumerate(launches[c0:c0 + groups_per_call]):
+                layers += group
+                stages += [si] * len(group)
+            arr, B = C._infer_layer_array(layers, g, "bench")
+            st = (ctypes.c_int32 * len(stages))(*stages)
+            calls.append((arr, len(layers), st, B))
+        lib, sp = C.lib(), ctypes.c_void_p(sync.data_ptr())
+
+        def run():
+            cs = C._stream()
+            for arr, n, st, B in calls:
+                C._check(lib.catq_ternary_infer_staged(arr, n, st, g, B, C.BF16, sp, cs), "bench decode")
+        n_launch = len(calls)
+    else:
+        side = torch.cuda.Stream(device=dev)
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):  # warm-up outside the capture
+            for group in launches:
+                C.catq_ternary_infer_batched(group, g)
+        torch.cuda.current_stream().wait_stream(side)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            for group in launches:
+                C.catq_ternary_infer_batched(group, g)
+
+        def run():
+            graph.replay()
+        n_launch = len(launches)
     for _ in range(3):
-        graph.replay()
+        run()
     torch.cuda.synchronize()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     a.record()
     for _ in range(steps):
-        graph.replay()
+        run()
     b.record()
     torch.cuda.synchronize()
     status = C.catq_device_status()
@@ -683,12 +712,13 @@ def measure_decode(C, torch, wl, dev, peaks, blocks=32, rows=1, steps=20, with_m
         raise SystemExit(f"device status {C.STATUS.get(status, status)} in the decode timing")
     ms = a.elapsed_time(b) / steps
     gbs = nbytes / (ms * 1e-3) / 1e9
-    del graph, launches
+    del launches, run
     torch.cuda.empty_cache()
-    return {"kernel": "ternary_mma_kernel (catq_ternary_infer_batched)", "blocks": blocks, "token_rows": rows,
-            "launches_per_step": blocks * len(DECODE_GROUPS), "bytes_per_step": nbytes, "us_per_step": ms * 1e3,
-            "value": gbs, "unit": "GB/s", "peak": peaks["hbm"], "frac_of_hbm": gbs / peaks["hbm"],
-            "steps": steps, "graph": True, "with_mu": with_mu}
+    return {"kernel": "ternary_mma_kernel (" + ("catq_ternary_infer_staged, cooperative" if staged else
+                                               "catq_ternary_infer_batched, CUDA graph") + ")",
+            "blocks": blocks, "token_rows": rows, "launches_per_step": n_launch, "bytes_per_step": nbytes,
+            "us_per_step": ms * 1e3, "value": gbs, "unit": "GB/s", "peak": peaks["hbm"],
+            "frac_of_hbm": gbs / peaks["hbm"], "steps": steps, "with_mu": with_mu}
 
 
 def measure_fig_error(C, torch, wl, dev, s0, epochs=20, batches=3, rows=2048, lr0=1e-3):
@@ -936,7 +966,8 @@ def run_only(args):
         r = measure_moe(C, torch, dev, peaks, 1, args.s, steps=args.steps, warmup=args.warmup,
                         experts=args.moe_experts)
     elif args.only.startswith("decode_b"):
-        r = measure_decode(C, torch, wl, dev, peaks, rows=int(args.only[len("decode_b"):]), steps=args.steps)
+        rows = int(args.only[len("decode_b"):].split("_")[0])
+        r = measure_decode(C, torch, wl, dev, peaks, rows=rows, steps=args.steps, staged="staged" in args.only)
     else:
         r = measure_block_window(C, torch, wl, dev, peaks, 1, args.s, barrier, steps=args.steps, warmup=args.warmup)
     print(json.dumps({"only": args.only, **r}), flush=True)

@@ -467,6 +467,28 @@ int32_t catq_ternary_infer_max_layers(void);
 catq_status catq_ternary_infer_batched(const catq_infer_layer* layers, int32_t n_layers, int32_t g, int64_t B,
                                        int32_t x_dtype, catq_stream stream);
 
+/* Maximum stages of one catq_ternary_infer_staged call, and the bytes of its sync buffer. */
+int32_t catq_ternary_infer_max_stages(void);
+size_t catq_ternary_infer_sync_bytes(void);
+
+/* The layers of a decode step in dependency order in one launch (this library's addition,
+ * like catq_ternary_infer_batched): layer i belongs to stage stage_of_layer[i] (a HOST array;
+ * 0 for the first layer, then non-decreasing in steps of 1, at most
+ * catq_ternary_infer_max_stages() stages).  Layers of one stage are independent of each
+ * other; a layer of stage s + 1 may read, as its X, the Y of a layer of an earlier stage (e.g.
+ * q/k/v -> o -> gate/up -> down of consecutive blocks).  Each layer computes exactly what
+ * catq_ternary_infer computes.  The launch is cooperative (every CTA resident at once) and
+ * the stages meet at device-wide barriers whose waits are bounded: on expiry the call latches
+ * CATQ_ERR_TIMEOUT (read with catq_device_status) and its outputs are undefined.  Copies of
+ * the next stage's codes start before its barrier, so the weight stream does not stop at a
+ * stage boundary.  sync: device memory of catq_ternary_infer_sync_bytes() bytes, 4-byte
+ * aligned, zero before the first call (e.g. cudaMemset); every call, completed or timed out,
+ * leaves it zero again.  Calls that may run at the same time (other streams) need separate
+ * sync buffers.  Errors as catq_ternary_infer_batched; a missing or malformed stage array or
+ * a NULL sync: CATQ_ERR_INVALID_ARG. */
+catq_status catq_ternary_infer_staged(const catq_infer_layer* layers, int32_t n_layers, const int32_t* stage_of_layer,
+                                      int32_t g, int64_t B, int32_t x_dtype, uint32_t* sync, catq_stream stream);
+
 /* ------------------------------------------------------------------ decoder-block layers
  * Eq. 7 reconstructs the output of a sliding window of layers (§2.4); with a window of one
  * decoder block the loss reaches each linear's factors through the layers

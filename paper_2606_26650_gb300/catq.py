@@ -113,6 +113,10 @@ def lib() -> ctypes.CDLL:
         "catq_direct_adamw_step": (I32, [I64, P, P, P, P, P, ctypes.POINTER(catq_adamw), I64, F, P]),
         "catq_ternary_infer_max_layers": (I32, []),
         "catq_ternary_infer_batched": (I32, [ctypes.POINTER(catq_infer_layer), I32, I32, I64, I32, P]),
+        "catq_ternary_infer_max_stages": (I32, []),
+        "catq_ternary_infer_sync_bytes": (S, []),
+        "catq_ternary_infer_staged": (I32, [ctypes.POINTER(catq_infer_layer), I32, ctypes.POINTER(I32), I32, I64, I32,
+                                            P, P]),
         "catq_group_recon_error": (I32, [LP, P, P]),
         "catq_grouped_fwd_loss_workspace_bytes": (S, [ctypes.POINTER(catq_grouped_layer), P]),
         "catq_rmsnorm_fwd": (I32, [P, I32, P, P, I64, I64, F, P, P, P, P]),
@@ -425,6 +429,46 @@ def catq_ternary_infer_batched(layers, g: int, stream=None):
                                   int(N), int(K), X.data_ptr(), Y.data_ptr())
     dt = _dtype_code(layers[0][4]) if layers else BF16
     _check(lib().catq_ternary_infer_batched(arr, len(layers), int(g), int(B), dt, _stream(stream)), w)
+
+
+def _infer_layer_array(layers, g, w):
+    arr = (catq_infer_layer * max(1, len(layers)))()
+    B = layers[0][4].shape[0] if layers else 0
+    for i, (codes, alpha, N, K, X, Y, mu) in enumerate(layers):
+        G = int(N) * int(K) // max(int(g), 1)
+        _buf(codes, "codes", int(N) * int(K) // 4, w)
+        _buf(alpha, "alpha", 4 * G, w)
+        _buf(mu, "mu", 4 * G, w)
+        if X.shape[0] != B:
+            raise ValueError(f"{w}: every layer needs the same token rows ({B})")
+        _buf(X, "X", B * int(K) * X.element_size(), w)
+        _buf(Y, "Y", B * int(N) * X.element_size(), w)
+        arr[i] = catq_infer_layer(codes.data_ptr(), alpha.data_ptr(), mu.data_ptr() if mu is not None else None,
+                                  int(N), int(K), X.data_ptr(), Y.data_ptr())
+    return arr, B
+
+
+def catq_ternary_infer_sync_bytes() -> int:
+    return int(lib().catq_ternary_infer_sync_bytes())
+
+
+def catq_ternary_infer_max_stages() -> int:
+    return int(lib().catq_ternary_infer_max_stages())
+
+
+def catq_ternary_infer_staged(layers, stages, g: int, sync, stream=None):
+    """Layers in dependency order in one cooperative launch: `layers` as in
+    catq_ternary_infer_batched, `stages` the stage of each layer (0, then non-decreasing in steps
+    of 1); a layer may read the Y of a layer of an earlier stage.  `sync`: a zeroed device buffer
+    of catq_ternary_infer_sync_bytes() bytes (left zeroed)."""
+    w = "catq_ternary_infer_staged"
+    arr, B = _infer_layer_array(layers, g, w)
+    _buf(sync, "sync", catq_ternary_infer_sync_bytes(), w)
+    st = (ctypes.c_int32 * max(1, len(stages)))(*[int(v) for v in stages])
+    if len(stages) != len(layers):
+        raise ValueError(f"{w}: one stage per layer")
+    dt = _dtype_code(layers[0][4]) if layers else BF16
+    _check(lib().catq_ternary_infer_staged(arr, len(layers), st, int(g), int(B), dt, _ptr(sync), _stream(stream)), w)
 
 
 def catq_schedule_at_epoch(e: int, m: int = 60, gamma: float = 0.8, s0: float = 30.0) -> catq_schedule:

@@ -633,12 +633,12 @@ catq_status catq_ternary_infer(const uint8_t* codes, const float* alpha, const f
 
 int32_t catq_ternary_infer_max_layers(void) { return ternary_infer_max_layers(); }
 
-catq_status catq_ternary_infer_batched(const catq_infer_layer* layers, int32_t n_layers, int32_t g, int64_t B,
-                                       int32_t x_dtype, catq_stream stream) {
+namespace {
+catq_status infer_descs(const catq_infer_layer* layers, int32_t n_layers, int32_t g, int64_t B, int32_t x_dtype,
+                        InferDesc* d) {
   if (!layers || n_layers < 1 || n_layers > ternary_infer_max_layers()) return CATQ_ERR_INVALID_ARG;
   if (x_dtype != CATQ_BF16) return CATQ_ERR_DTYPE;
   if (g < 64 || g % 64 != 0 || B < 0) return CATQ_ERR_SHAPE;
-  InferDesc d[64];
   const bool with_mu = layers[0].mu != nullptr;
   for (int32_t i = 0; i < n_layers; ++i) {
     const catq_infer_layer& L = layers[i];
@@ -653,8 +653,37 @@ catq_status catq_ternary_infer_batched(const catq_infer_layer* layers, int32_t n
       return CATQ_ERR_ALIGN;
     d[i] = InferDesc{L.codes, L.alpha, L.mu, L.N, L.K, L.X, B, L.Y};
   }
-  if (B == 0) return CATQ_OK;
+  return CATQ_OK;
+}
+}  // namespace
+
+catq_status catq_ternary_infer_batched(const catq_infer_layer* layers, int32_t n_layers, int32_t g, int64_t B,
+                                       int32_t x_dtype, catq_stream stream) {
+  InferDesc d[64];
+  const catq_status st = infer_descs(layers, n_layers, g, B, x_dtype, d);
+  if (st != CATQ_OK || B == 0) return st;
   return cuda_status(launch_ternary_infer_batched(d, n_layers, g, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int32_t catq_ternary_infer_max_stages(void) { return ternary_infer_max_stages(); }
+
+size_t catq_ternary_infer_sync_bytes(void) { return ternary_infer_sync_bytes(); }
+
+catq_status catq_ternary_infer_staged(const catq_infer_layer* layers, int32_t n_layers, const int32_t* stage_of_layer,
+                                      int32_t g, int64_t B, int32_t x_dtype, uint32_t* sync, catq_stream stream) {
+  InferDesc d[64];
+  catq_status st = infer_descs(layers, n_layers, g, B, x_dtype, d);
+  if (st != CATQ_OK) return st;
+  if (!stage_of_layer || !sync) return CATQ_ERR_INVALID_ARG;
+  if (stage_of_layer[0] != 0) return CATQ_ERR_INVALID_ARG;
+  for (int32_t i = 1; i < n_layers; ++i)
+    if (stage_of_layer[i] != stage_of_layer[i - 1] && stage_of_layer[i] != stage_of_layer[i - 1] + 1)
+      return CATQ_ERR_INVALID_ARG;
+  if (stage_of_layer[n_layers - 1] + 1 > ternary_infer_max_stages()) return CATQ_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(sync) & 3u) != 0) return CATQ_ERR_ALIGN;
+  if (B == 0) return CATQ_OK;
+  return cuda_status(
+      launch_ternary_infer_staged(d, n_layers, stage_of_layer, g, sync, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 catq_status catq_schedule_at_epoch(int32_t e, int32_t m, double gamma, double s0, catq_schedule* out) {

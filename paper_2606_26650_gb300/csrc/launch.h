@@ -81,6 +81,13 @@ struct InferDesc {
 };
 int ternary_infer_max_layers();
 cudaError_t launch_ternary_infer_batched(const InferDesc* layers, int n, int32_t g, cudaStream_t st);
+// A chain of layer sets in one cooperative launch: layer i belongs to stage stage_of[i]
+// (0, then non-decreasing in steps of 1); stage s + 1 may read what stage s wrote.  sync:
+// ternary_infer_sync_bytes() of device memory, zero on entry, zero again on exit.
+int ternary_infer_max_stages();
+size_t ternary_infer_sync_bytes();
+cudaError_t launch_ternary_infer_staged(const InferDesc* layers, int n, const int32_t* stage_of, int32_t g,
+                                        uint32_t* sync, cudaStream_t st);
 
 // Wait control (abort word, status word, epoch, time limit) for one launch of a kernel with
 // bounded waits; false when the device's status words are unavailable.

@@ -32,6 +32,15 @@
 // split each slab into contiguous K ranges, and their partial sums meet in shared memory in a
 // fixed order (deterministic).  Token rows are taken 8 at a time (the MMA's N); all
 // arithmetic after the MMAs is fp32, with one rounding of Y.
+//
+// A staged launch runs a chain of such layer sets in one cooperative launch (the layers of a
+// decode step in dependency order: stage s + 1 may read what stage s wrote).  The work items
+// of all stages form one stream; before its first item of a stage, a CTA arrives at the
+// barriers of the stages it is done with and waits (bounded) until every CTA has arrived at
+// the previous stage's.  The code slabs of the next items do not depend on earlier stages,
+// so their copies are issued before the wait and the HBM stream does not drain at a stage
+// boundary.  Activations of a staged launch are read through L2 (ld.global.cg), since a
+// previous stage of the same launch may have written them.
 #include <algorithm>
 #include <cstdint>
 #include <type_traits>
@@ -149,15 +158,45 @@ struct InferLayer {
   int32_t item0;   // first work item of this layer
 };
 
-constexpr int kMaxInferLayers = 16;
+constexpr int kMaxInferLayers = 32;
+constexpr int kMaxInferStages = 32;
 
 struct InferArgs {
   int32_t n_layers;
   int32_t total_items;  // work items (16 R-row blocks) over all layers
   int32_t g;
-  int32_t pad_;
+  int32_t n_stages;     // staged launches: stages; 1 otherwise
+  uint32_t* sync;       // staged launches: [kMaxInferStages] barrier counters, then the exit counter
+  int32_t stage_end[kMaxInferStages];  // first item after each stage
   InferLayer L[kMaxInferLayers];
 };
+
+// Staged launches: arrive at a stage barrier (after every thread's stores, by one thread).
+__device__ __forceinline__ void counter_arrive(uint32_t* ctr) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
+}
+
+__device__ __forceinline__ uint32_t counter_load(const uint32_t* ctr) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+  return v;
+}
+
+// Bounded wait until *ctr >= target: false on timeout (latched) or when another wait of the
+// launch has given up.
+__device__ __forceinline__ bool counter_wait(const uint32_t* ctr, uint32_t target, const WaitCtl& w) {
+  if (counter_load(ctr) >= target) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (;;) {
+    __nanosleep(128);
+    if (counter_load(ctr) >= target) return true;
+    if (aborted(w)) return false;
+    if (globaltimer_ns() - t0 > w.timeout_ns) {
+      signal_timeout(w);
+      return false;
+    }
+  }
+}
 
 // A position in a CTA's stream of code slabs: work item t (a block of 16 R rows of layer l),
 // token block b0 and slab.  Work items run t = blockIdx.x, blockIdx.x + gridDim.x, ...
@@ -198,7 +237,7 @@ __device__ __forceinline__ void cursor_next(Cursor& c, const InferArgs& a) {
 // item's codes are on their way while this one finishes its slabs and its reduction.  Each
 // row's copy lands at a stride padded by 16 VW bytes, so the fragment reads (four lanes per
 // row, eight rows per instruction) are free of bank conflicts.
-template <int R, int VW, bool MU>
+template <int R, int VW, bool MU, bool STAGED>
 __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const __grid_constant__ InferArgs a,
                                                                      int32_t buf_bytes, const WaitCtl wc) {
   constexpr int ROWS = 16 * R;
@@ -256,8 +295,39 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const __
   int32_t goff[R][2];
   const uint16_t* xrow = nullptr;
   float acc[R][4], d[R][4], da[4];
+  int32_t stage = 0, arrived = 0;  // staged: stage of the current item, barriers arrived at
 
   while (ok && con.t < a.total_items) {
+    if constexpr (STAGED) {
+      if (con.slab == 0 && con.b0 == 0) {
+        int32_t st = stage;
+        while (con.t >= a.stage_end[st]) ++st;
+        if (st > stage) {
+          // This CTA has no items left in stages before st (items run in order): its outputs
+          // there are stored.  Arrive at those stages' barriers, then wait until every CTA has
+          // arrived at stage st - 1's.
+          __syncthreads();
+          bool good = true;
+          if (threadIdx.x == 0) {
+            __threadfence();
+            for (int32_t b = arrived; b < st; ++b) counter_arrive(a.sync + b);
+            good = counter_wait(a.sync + (st - 1), gridDim.x, wc);
+          }
+          arrived = st;
+          stage = st;
+          if (!__syncthreads_and(good)) {
+            if (threadIdx.x == 0) {
+              // copies of this CTA's next slabs may be in flight
+              if (issued > qn) drain_wait(bar0 + 8u * (qn & 1u), (qn >> 1) & 1u);
+              if (issued > qn + 1) drain_wait(bar0 + 8u * ((qn + 1) & 1u), ((qn + 1) >> 1) & 1u);
+            }
+            __syncthreads();
+            ok = false;
+            break;
+          }
+        }
+      }
+    }
     const InferLayer& L = a.L[con.l];
     const int64_t n0 = static_cast<int64_t>(con.t - L.item0) * ROWS;
     if (con.slab == 0) {
@@ -313,7 +383,7 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const __
       auto load_x = [&](int32_t sc, uint4 (&xv)[2 * VW]) {
         const uint4* xp = xbase + sc * (8 * VW);
 #pragma unroll
-        for (int i = 0; i < 2 * VW; ++i) xv[i] = __ldg(xp + i);
+        for (int i = 0; i < 2 * VW; ++i) xv[i] = STAGED ? __ldcg(xp + i) : __ldg(xp + i);
       };
       // one super-chunk: this thread's code words from shared memory, its activations xv
       auto step = [&](int32_t sc, const uint4 (&xv)[2 * VW]) {
@@ -432,6 +502,21 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const __
     }
     cursor_next(con, a);
   }
+  if constexpr (STAGED) {
+    // Arrive at the barriers still owed, then leave; the last CTA to leave (every other one has
+    // passed all its waits by then) zeroes the counters for the next launch.
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      __threadfence();
+      for (int32_t b = arrived; b < a.n_stages - 1; ++b) counter_arrive(a.sync + b);
+      const uint32_t prev = atomicAdd(a.sync + kMaxInferStages, 1u);
+      if (prev == gridDim.x - 1) {
+        for (int32_t b = 0; b < a.n_stages - 1; ++b) a.sync[b] = 0u;
+        a.sync[kMaxInferStages] = 0u;
+        __threadfence();
+      }
+    }
+  }
 }
 
 // One slab buffer: two per CTA plus the reduction array fit twice in an SM's shared memory.
@@ -450,13 +535,18 @@ int64_t slab_cols(int64_t K, int R, int VW) {
   return ((K + nslabs - 1) / nslabs + unit - 1) / unit * unit;
 }
 
+// stage_of (nullable): the stage of each layer (non-decreasing from 0 in steps of 1); sync: the
+// staged launch's counters (zero on entry and on exit).
 template <int R, int VW>
-cudaError_t launch_mma(const InferDesc* ls, int n, int32_t g, bool with_mu, cudaStream_t st) {
+cudaError_t launch_mma(const InferDesc* ls, int n, int32_t g, bool with_mu, const int32_t* stage_of, uint32_t* sync,
+                       cudaStream_t st) {
   WaitCtl wc;
   if (!launch_wait_ctl(&wc)) return cudaErrorInvalidDevice;
   InferArgs a{};
   a.n_layers = n;
   a.g = g;
+  a.n_stages = stage_of ? stage_of[n - 1] + 1 : 1;
+  a.sync = sync;
   int64_t items = 0, max_buf = 0;
   for (int i = 0; i < n; ++i) {
     InferLayer& L = a.L[i];
@@ -475,53 +565,65 @@ cudaError_t launch_mma(const InferDesc* ls, int n, int32_t g, bool with_mu, cuda
     L.item0 = static_cast<int32_t>(items);
     items += (L.N + 16 * R - 1) / (16 * R);
     max_buf = std::max<int64_t>(max_buf, slab_bytes(KS, R, VW));
+    if (stage_of) a.stage_end[stage_of[i]] = static_cast<int32_t>(std::min<int64_t>(items, INT32_MAX));
   }
-  if (items == 0) return cudaSuccess;
   if (items >= (int64_t(1) << 31)) return cudaErrorInvalidValue;
+  if (items == 0) return cudaSuccess;
   a.total_items = static_cast<int32_t>(items);
+  if (!stage_of) a.stage_end[0] = a.total_items;
+  int64_t widest = 0;  // most items of one stage
+  for (int32_t s = 0, prev = 0; s < a.n_stages; prev = a.stage_end[s], ++s)
+    widest = std::max<int64_t>(widest, a.stage_end[s] - prev);
   const int buf_bytes = static_cast<int>((max_buf + 127) / 128 * 128);
   const int smem = 2 * buf_bytes;
   int sm = 152;
   int dev = 0;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sm, cudaDevAttrMultiProcessorCount, dev);
-  const int64_t blocks = std::min<int64_t>(items, 2 * static_cast<int64_t>(sm));
-  auto kern = with_mu ? ternary_mma_kernel<R, VW, true> : ternary_mma_kernel<R, VW, false>;
-  const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  const bool staged = a.n_stages > 1;
+  auto kern = staged ? (with_mu ? ternary_mma_kernel<R, VW, true, true> : ternary_mma_kernel<R, VW, false, true>)
+                     : (with_mu ? ternary_mma_kernel<R, VW, true, false> : ternary_mma_kernel<R, VW, false, false>);
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  // programmatic dependent launch: this kernel may start while the previous one in the stream
-  // finishes (see grid_dependency_wait in the kernel)
+  int64_t blocks = std::min<int64_t>(items, 2 * static_cast<int64_t>(sm));
   cudaLaunchConfig_t cfg{};
+  cudaLaunchAttribute attr[1];
+  if (staged) {
+    // every CTA must be resident at once (they wait on each other): a cooperative launch of
+    // at most the co-resident CTAs, and no more than the widest stage has items
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kMmaWarps * 32, static_cast<size_t>(smem));
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    blocks = std::min<int64_t>(widest, static_cast<int64_t>(per_sm) * sm);
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+  } else {
+    // programmatic dependent launch: this kernel may start while the previous one in the
+    // stream finishes (see grid_dependency_wait in the kernel)
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+  }
   cfg.gridDim = dim3(static_cast<unsigned>(blocks));
   cfg.blockDim = dim3(kMmaWarps * 32);
   cfg.dynamicSmemBytes = static_cast<size_t>(smem);
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, a, buf_bytes, wc);
 }
 
 template <int R>
-cudaError_t launch_rows(const InferDesc* ls, int n, int32_t g, bool with_mu, cudaStream_t st) {
-  if (g % 128 == 0) return launch_mma<R, 2>(ls, n, g, with_mu, st);
-  return launch_mma<R, 1>(ls, n, g, with_mu, st);
+cudaError_t launch_rows(const InferDesc* ls, int n, int32_t g, bool with_mu, const int32_t* stage_of, uint32_t* sync,
+                        cudaStream_t st) {
+  if (g % 128 == 0) return launch_mma<R, 2>(ls, n, g, with_mu, stage_of, sync, st);
+  return launch_mma<R, 1>(ls, n, g, with_mu, stage_of, sync, st);
 }
 
-}  // namespace
-
-int ternary_infer_max_layers() { return kMaxInferLayers; }
-
-cudaError_t launch_ternary_infer_batched(const InferDesc* ls, int n, int32_t g, cudaStream_t st) {
-  if (n < 1 || n > kMaxInferLayers) return cudaErrorInvalidValue;
-  bool with_mu = ls[0].mu != nullptr;
-  for (int i = 1; i < n; ++i)
-    if ((ls[i].mu != nullptr) != with_mu) return cudaErrorInvalidValue;
-  // 16-row tiles per work item (1 or 2: more hold more registers than two CTAs per SM
-  // allow without spills): the fewest rows on the busiest SM (two persistent CTAs per SM),
-  // then the most tiles per item (the correction MMAs and the activation preparation serve
-  // more rows).
+// 16-row tiles per work item (1 or 2: more hold more registers than two CTAs per SM allow
+// without spills): the fewest rows on the busiest SM summed over the stages (two persistent
+// CTAs per SM), then the most tiles per item (the correction MMAs and the activation
+// preparation serve more rows).
+int pick_rows(const InferDesc* ls, int n, const int32_t* stage_of) {
   int sm = 152;
   {
     int dev = 0;
@@ -530,16 +632,53 @@ cudaError_t launch_ternary_infer_batched(const InferDesc* ls, int n, int32_t g, 
   int best = 1;
   int64_t best_rows = -1;
   for (int r = 1; r <= 2; ++r) {
-    int64_t items = 0;
-    for (int i = 0; i < n; ++i) items += (ls[i].N + 16 * r - 1) / (16 * r);
-    const int64_t busiest = (items + 2 * sm - 1) / (2 * sm) * 16 * r;
+    int64_t busiest = 0, items = 0;
+    for (int i = 0; i < n; ++i) {
+      items += (ls[i].N + 16 * r - 1) / (16 * r);
+      if (i + 1 == n || (stage_of && stage_of[i + 1] != stage_of[i])) {
+        busiest += (items + 2 * sm - 1) / (2 * sm) * 16 * r;
+        items = 0;
+      }
+    }
     if (best_rows < 0 || busiest <= best_rows) {
       best = r;
       best_rows = busiest;
     }
   }
-  if (best == 2) return launch_rows<2>(ls, n, g, with_mu, st);
-  return launch_rows<1>(ls, n, g, with_mu, st);
+  return best;
+}
+
+cudaError_t launch_infer(const InferDesc* ls, int n, int32_t g, const int32_t* stage_of, uint32_t* sync,
+                         cudaStream_t st) {
+  if (n < 1 || n > kMaxInferLayers) return cudaErrorInvalidValue;
+  const bool with_mu = ls[0].mu != nullptr;
+  for (int i = 1; i < n; ++i)
+    if ((ls[i].mu != nullptr) != with_mu) return cudaErrorInvalidValue;
+  if (stage_of) {
+    if (stage_of[0] != 0 || !sync) return cudaErrorInvalidValue;
+    for (int i = 1; i < n; ++i)
+      if (stage_of[i] != stage_of[i - 1] && stage_of[i] != stage_of[i - 1] + 1) return cudaErrorInvalidValue;
+    if (stage_of[n - 1] + 1 > kMaxInferStages) return cudaErrorInvalidValue;
+  }
+  if (pick_rows(ls, n, stage_of) == 2) return launch_rows<2>(ls, n, g, with_mu, stage_of, sync, st);
+  return launch_rows<1>(ls, n, g, with_mu, stage_of, sync, st);
+}
+
+}  // namespace
+
+int ternary_infer_max_layers() { return kMaxInferLayers; }
+
+cudaError_t launch_ternary_infer_batched(const InferDesc* ls, int n, int32_t g, cudaStream_t st) {
+  return launch_infer(ls, n, g, nullptr, nullptr, st);
+}
+
+int ternary_infer_max_stages() { return kMaxInferStages; }
+size_t ternary_infer_sync_bytes() { return (kMaxInferStages + 1) * sizeof(uint32_t); }
+
+cudaError_t launch_ternary_infer_staged(const InferDesc* ls, int n, const int32_t* stage_of, int32_t g, uint32_t* sync,
+                                        cudaStream_t st) {
+  if (!stage_of) return cudaErrorInvalidValue;
+  return launch_infer(ls, n, g, stage_of, sync, st);
 }
 
 cudaError_t launch_ternary_infer(const uint8_t* codes, const float* alpha, const float* mu, int64_t N, int64_t K,
