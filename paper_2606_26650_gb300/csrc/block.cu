@@ -237,6 +237,29 @@ __device__ __forceinline__ void load_tile(uint16_t* tile, const uint16_t* src, i
   }
 }
 
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async4(uint32_t dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// load_tile through cp.async (16-byte copies that complete with the thread's next wait).
+template <int HD>
+__device__ __forceinline__ void load_tile_async(uint32_t tile, const uint16_t* src, int64_t row0, int64_t ld,
+                                                int64_t col0) {
+  constexpr int kChunks = kBlk * HD / 8;
+  for (int c = threadIdx.x; c < kChunks; c += kAttnThreads) {
+    const int r = c / (HD / 8), k = (c % (HD / 8)) * 8;
+    cp_async16(tile + static_cast<uint32_t>((r * Tile<HD>::kStride + k) * 2), src + (row0 + r) * ld + col0 + k);
+  }
+}
+
 // Address of the row that this lane supplies to an ldmatrix.x4 of a 16 x 16 fragment at
 // (row0, col0) of a tile: matrix m = lane / 8 covers rows + (m & 1) 8 when `row_from_bit0`
 // (A operands and transposed B operands), else + (m >> 1) 8 (B operands stored n-major), and
@@ -302,30 +325,44 @@ struct AttnArgs {
 
 // Forward: one CTA per (query block, head, sequence).  Rows g and g + 8 of the warp's 16 are
 // the thread's (lane / 4); its columns within each 8-wide n-tile are 2 (lane % 4) + {0, 1}.
+// Key/value blocks stream through two shared-memory buffers: block kb + 1's copies are in
+// flight while block kb is computed.
 template <int HD>
 __global__ void __launch_bounds__(kAttnThreads) attn_fwd_kernel(const AttnArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
   uint16_t* Qs = reinterpret_cast<uint16_t*>(smem);
-  uint16_t* Ks = Qs + kBlk * Tile<HD>::kStride;
-  uint16_t* Vs = Ks + kBlk * Tile<HD>::kStride;
+  const uint32_t qa = smem_u32(Qs);
+  const uint32_t kv0 = qa + Tile<HD>::kBytes;  // buffer b: K at kv0 + 2 b tile, V after it
   const int nqb = a.S / kBlk;
   const int qb = nqb - 1 - static_cast<int>(blockIdx.x);  // the longest rows first
   const int h = blockIdx.y, b = blockIdx.z, hk = h / (a.nh / a.nkv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
   const int64_t tok0 = static_cast<int64_t>(b) * a.S;
-  load_tile<HD>(Qs, a.q, tok0 + qb * kBlk, static_cast<int64_t>(a.nh) * HD, static_cast<int64_t>(h) * HD);
+  const int64_t ldq = static_cast<int64_t>(a.nh) * HD, ldk = static_cast<int64_t>(a.nkv) * HD;
+  auto load_kv = [&](int kb) {
+    const uint32_t kt = kv0 + static_cast<uint32_t>((kb & 1) * 2 * Tile<HD>::kBytes);
+    load_tile_async<HD>(kt, a.k, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
+    load_tile_async<HD>(kt + Tile<HD>::kBytes, a.v, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
+  };
+  load_tile_async<HD>(qa, a.q, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
+  load_kv(0);
+  cp_async_commit();
   float o[HD / 8][4];
 #pragma unroll
   for (int i = 0; i < HD / 8; ++i)
 #pragma unroll
     for (int e = 0; e < 4; ++e) o[i][e] = 0.0f;
   float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.0f, 0.0f};
-  const uint32_t qa = smem_u32(Qs), ka = smem_u32(Ks), va = smem_u32(Vs);
   for (int kb = 0; kb <= qb; ++kb) {
+    if (kb < qb) {
+      load_kv(kb + 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
     __syncthreads();
-    load_tile<HD>(Ks, a.k, tok0 + kb * kBlk, static_cast<int64_t>(a.nkv) * HD, static_cast<int64_t>(hk) * HD);
-    load_tile<HD>(Vs, a.v, tok0 + kb * kBlk, static_cast<int64_t>(a.nkv) * HD, static_cast<int64_t>(hk) * HD);
-    __syncthreads();
+    const uint32_t ka = kv0 + static_cast<uint32_t>((kb & 1) * 2 * Tile<HD>::kBytes), va = ka + Tile<HD>::kBytes;
     float s[8][4];
     scores_16x64<HD>(s, qa, warp * 16, ka);
     float mx[2] = {-INFINITY, -INFINITY};
@@ -371,6 +408,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_fwd_kernel(const AttnArgs a
       o[dn][3] *= corr[1];
     }
     accum_pv<HD>(o, s, va);
+    __syncthreads();  // buffer kb & 1 is refilled with block kb + 2 next
   }
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
@@ -381,7 +419,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_fwd_kernel(const AttnArgs a
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
     const int64_t tok = tok0 + qb * kBlk + warp * 16 + g + 8 * i;
-    uint16_t* orow = a.out + tok * a.nh * HD + static_cast<int64_t>(h) * HD;
+    uint16_t* orow = a.out + tok * ldq + static_cast<int64_t>(h) * HD;
 #pragma unroll
     for (int dn = 0; dn < HD / 8; ++dn)
       *reinterpret_cast<uint32_t*>(orow + dn * 8 + 2 * t4) = pack_bf16x2(o[dn][2 * i] * inv[i], o[dn][2 * i + 1] * inv[i]);
@@ -413,22 +451,28 @@ __global__ void __launch_bounds__(kRowThreads) attn_delta_kernel(const AttnArgs 
   }
 }
 
-// dQ: one CTA per (query block, head, sequence), over the key blocks up to the diagonal.
+// dQ: one CTA per (query block, head, sequence), over the key blocks up to the diagonal,
+// which stream through two buffers as in the forward.
 template <int HD>
 __global__ void __launch_bounds__(kAttnThreads) attn_bwd_dq_kernel(const AttnArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
-  uint16_t* Qs = reinterpret_cast<uint16_t*>(smem);
-  uint16_t* Ds = Qs + kBlk * Tile<HD>::kStride;  // dO
-  uint16_t* Ks = Ds + kBlk * Tile<HD>::kStride;
-  uint16_t* Vs = Ks + kBlk * Tile<HD>::kStride;
+  const uint32_t qa = smem_u32(smem), da = qa + Tile<HD>::kBytes;  // Q, dO
+  const uint32_t kv0 = da + Tile<HD>::kBytes;                       // buffer b: K, V at kv0 + 2 b tile
   const int nqb = a.S / kBlk;
   const int qb = nqb - 1 - static_cast<int>(blockIdx.x);
   const int h = blockIdx.y, b = blockIdx.z, hk = h / (a.nh / a.nkv);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
   const int64_t tok0 = static_cast<int64_t>(b) * a.S;
   const int64_t ldq = static_cast<int64_t>(a.nh) * HD, ldk = static_cast<int64_t>(a.nkv) * HD;
-  load_tile<HD>(Qs, a.q, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
-  load_tile<HD>(Ds, a.dO, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
+  auto load_kv = [&](int kb) {
+    const uint32_t kt = kv0 + static_cast<uint32_t>((kb & 1) * 2 * Tile<HD>::kBytes);
+    load_tile_async<HD>(kt, a.k, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
+    load_tile_async<HD>(kt + Tile<HD>::kBytes, a.v, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
+  };
+  load_tile_async<HD>(qa, a.q, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
+  load_tile_async<HD>(da, a.dO, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
+  load_kv(0);
+  cp_async_commit();
   float lse2[2], dl[2];  // this thread's two rows: log-sum-exp in log2 units, and delta
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
@@ -441,12 +485,16 @@ __global__ void __launch_bounds__(kAttnThreads) attn_bwd_dq_kernel(const AttnArg
   for (int i = 0; i < HD / 8; ++i)
 #pragma unroll
     for (int e = 0; e < 4; ++e) dq[i][e] = 0.0f;
-  const uint32_t qa = smem_u32(Qs), da = smem_u32(Ds), ka = smem_u32(Ks), va = smem_u32(Vs);
   for (int kb = 0; kb <= qb; ++kb) {
+    if (kb < qb) {
+      load_kv(kb + 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
     __syncthreads();
-    load_tile<HD>(Ks, a.k, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
-    load_tile<HD>(Vs, a.v, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
-    __syncthreads();
+    const uint32_t ka = kv0 + static_cast<uint32_t>((kb & 1) * 2 * Tile<HD>::kBytes), va = ka + Tile<HD>::kBytes;
     float s[8][4], dp[8][4];
     scores_16x64<HD>(s, qa, warp * 16, ka);   // Q K^T
     scores_16x64<HD>(dp, da, warp * 16, va);  // dO V^T
@@ -462,6 +510,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_bwd_dq_kernel(const AttnArg
         s[nt][e] = p * (dp[nt][e] - dl[e >> 1]);  // dS
       }
     accum_pv<HD>(dq, s, ka);  // dS K
+    __syncthreads();
   }
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
@@ -474,92 +523,106 @@ __global__ void __launch_bounds__(kAttnThreads) attn_bwd_dq_kernel(const AttnArg
 }
 
 // dK, dV: one CTA per (key block, key/value head, sequence), over every query head of the
-// group and the query blocks from the diagonal on, 16 queries at a time.  Scores are formed
-// transposed (keys as rows) so that P^T and dS^T feed the A operand from registers.
+// group and the query blocks from the diagonal on (one stream of (head, query block) pairs
+// through two buffers of Q, dO and their rows' log-sum-exp and delta), 16 queries at a time.
+// Scores are formed transposed (keys as rows) so that P^T and dS^T feed the A operand from
+// registers.
 template <int HD>
 __global__ void __launch_bounds__(kAttnThreads) attn_bwd_dkdv_kernel(const AttnArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
-  uint16_t* Ks = reinterpret_cast<uint16_t*>(smem);
-  uint16_t* Vs = Ks + kBlk * Tile<HD>::kStride;
-  uint16_t* Qs = Vs + kBlk * Tile<HD>::kStride;
-  uint16_t* Ds = Qs + kBlk * Tile<HD>::kStride;
-  float* lse_s = reinterpret_cast<float*>(Ds + kBlk * Tile<HD>::kStride);  // [64], log2 units
-  float* dl_s = lse_s + kBlk;                                             // [64]
+  const uint32_t ka = smem_u32(smem), va = ka + Tile<HD>::kBytes;
+  const uint32_t qd0 = va + Tile<HD>::kBytes;  // buffer b: Q at qd0 + 2 b tile, dO after it
+  float* const lsd0 = reinterpret_cast<float*>(smem + 6 * Tile<HD>::kBytes);  // buffer b: lse [64], delta [64]
   const int nqb = a.S / kBlk;
   const int kb = static_cast<int>(blockIdx.x);  // the most query blocks first
   const int hk = blockIdx.y, b = blockIdx.z, rep = a.nh / a.nkv;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
   const int64_t tok0 = static_cast<int64_t>(b) * a.S;
   const int64_t ldq = static_cast<int64_t>(a.nh) * HD, ldk = static_cast<int64_t>(a.nkv) * HD;
-  load_tile<HD>(Ks, a.k, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
-  load_tile<HD>(Vs, a.v, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
+  const int per_head = nqb - kb, n_it = rep * per_head;  // (head, query block) pairs
+  auto load_q = [&](int it) {
+    const int h = hk * rep + it / per_head, qb = kb + it % per_head;
+    const uint32_t qt = qd0 + static_cast<uint32_t>((it & 1) * 2 * Tile<HD>::kBytes);
+    load_tile_async<HD>(qt, a.q, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
+    load_tile_async<HD>(qt + Tile<HD>::kBytes, a.dO, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
+    if (threadIdx.x < kBlk) {
+      const int64_t idx = (static_cast<int64_t>(b) * a.nh + h) * a.S + qb * kBlk + threadIdx.x;
+      float* l = lsd0 + (it & 1) * 2 * kBlk;
+      cp_async4(smem_u32(l + threadIdx.x), a.lse + idx);
+      cp_async4(smem_u32(l + kBlk + threadIdx.x), a.delta + idx);
+    }
+  };
+  load_tile_async<HD>(ka, a.k, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
+  load_tile_async<HD>(va, a.v, tok0 + kb * kBlk, ldk, static_cast<int64_t>(hk) * HD);
+  load_q(0);
+  cp_async_commit();
   float dk[HD / 8][4], dv[HD / 8][4];
 #pragma unroll
   for (int i = 0; i < HD / 8; ++i)
 #pragma unroll
     for (int e = 0; e < 4; ++e) dk[i][e] = dv[i][e] = 0.0f;
-  const uint32_t ka = smem_u32(Ks), va = smem_u32(Vs), qa = smem_u32(Qs), da = smem_u32(Ds);
-  for (int hh = 0; hh < rep; ++hh) {
-    const int h = hk * rep + hh;
-    for (int qb = kb; qb < nqb; ++qb) {
-      __syncthreads();
-      load_tile<HD>(Qs, a.q, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
-      load_tile<HD>(Ds, a.dO, tok0 + qb * kBlk, ldq, static_cast<int64_t>(h) * HD);
-      if (threadIdx.x < kBlk) {
-        const int64_t idx = (static_cast<int64_t>(b) * a.nh + h) * a.S + qb * kBlk + threadIdx.x;
-        lse_s[threadIdx.x] = a.lse[idx] * 1.4426950408889634f;
-        dl_s[threadIdx.x] = a.delta[idx];
-      }
-      __syncthreads();
+  for (int it = 0; it < n_it; ++it) {
+    if (it + 1 < n_it) {
+      load_q(it + 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    const int qb = kb + it % per_head;
+    const uint32_t qa = qd0 + static_cast<uint32_t>((it & 1) * 2 * Tile<HD>::kBytes), da = qa + Tile<HD>::kBytes;
+    const float* lse_s = lsd0 + (it & 1) * 2 * kBlk;
+    const float* dl_s = lse_s + kBlk;
 #pragma unroll 1
-      for (int qs = 0; qs < kBlk / 16; ++qs) {
-        // S^T and dP^T of the warp's 16 keys against 16 queries: two n-tiles each
-        float st[2][4], dpt[2][4];
+    for (int qs = 0; qs < kBlk / 16; ++qs) {
+      // S^T and dP^T of the warp's 16 keys against 16 queries: two n-tiles each
+      float st[2][4], dpt[2][4];
 #pragma unroll
-        for (int nt = 0; nt < 2; ++nt)
+      for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
-          for (int e = 0; e < 4; ++e) st[nt][e] = dpt[nt][e] = 0.0f;
+        for (int e = 0; e < 4; ++e) st[nt][e] = dpt[nt][e] = 0.0f;
 #pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk) {
-          uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
-          ldsm_x4(frag_addr<HD>(ka, warp * 16, kk * 16, true), a0, a1, a2, a3);
-          ldsm_x4(frag_addr<HD>(qa, qs * 16, kk * 16, false), b0, b1, b2, b3);
-          mma_bf16_16816(st[0], a0, a1, a2, a3, b0, b1);
-          mma_bf16_16816(st[1], a0, a1, a2, a3, b2, b3);
-          ldsm_x4(frag_addr<HD>(va, warp * 16, kk * 16, true), a0, a1, a2, a3);
-          ldsm_x4(frag_addr<HD>(da, qs * 16, kk * 16, false), b0, b1, b2, b3);
-          mma_bf16_16816(dpt[0], a0, a1, a2, a3, b0, b1);
-          mma_bf16_16816(dpt[1], a0, a1, a2, a3, b2, b3);
+      for (int kk = 0; kk < HD / 16; ++kk) {
+        uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
+        ldsm_x4(frag_addr<HD>(ka, warp * 16, kk * 16, true), a0, a1, a2, a3);
+        ldsm_x4(frag_addr<HD>(qa, qs * 16, kk * 16, false), b0, b1, b2, b3);
+        mma_bf16_16816(st[0], a0, a1, a2, a3, b0, b1);
+        mma_bf16_16816(st[1], a0, a1, a2, a3, b2, b3);
+        ldsm_x4(frag_addr<HD>(va, warp * 16, kk * 16, true), a0, a1, a2, a3);
+        ldsm_x4(frag_addr<HD>(da, qs * 16, kk * 16, false), b0, b1, b2, b3);
+        mma_bf16_16816(dpt[0], a0, a1, a2, a3, b0, b1);
+        mma_bf16_16816(dpt[1], a0, a1, a2, a3, b2, b3);
+      }
+      float pt[2][4], dst[2][4];
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int qry = qs * 16 + nt * 8 + 2 * t4 + (e & 1);  // within the query block
+          const int key = warp * 16 + g + (e >> 1) * 8;          // within the key block
+          float p = exp2f((st[nt][e] * a.scale - lse_s[qry]) * 1.4426950408889634f);
+          if (qb == kb && key > qry) p = 0.0f;
+          pt[nt][e] = p;
+          dst[nt][e] = p * (dpt[nt][e] - dl_s[qry]);
         }
-        float pt[2][4], dst[2][4];
+      // dV += P^T dO and dK += dS^T Q over these 16 queries (one k-step)
+      const uint32_t p0 = pack_bf16x2(pt[0][0], pt[0][1]), p1 = pack_bf16x2(pt[0][2], pt[0][3]);
+      const uint32_t p2 = pack_bf16x2(pt[1][0], pt[1][1]), p3 = pack_bf16x2(pt[1][2], pt[1][3]);
+      const uint32_t s0 = pack_bf16x2(dst[0][0], dst[0][1]), s1 = pack_bf16x2(dst[0][2], dst[0][3]);
+      const uint32_t s2 = pack_bf16x2(dst[1][0], dst[1][1]), s3 = pack_bf16x2(dst[1][2], dst[1][3]);
 #pragma unroll
-        for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int qry = qs * 16 + nt * 8 + 2 * t4 + (e & 1);  // within the query block
-            const int key = warp * 16 + g + (e >> 1) * 8;          // within the key block
-            float p = exp2f(st[nt][e] * a.scale_log2 - lse_s[qry]);
-            if (qb == kb && key > qry) p = 0.0f;
-            pt[nt][e] = p;
-            dst[nt][e] = p * (dpt[nt][e] - dl_s[qry]);
-          }
-        // dV += P^T dO and dK += dS^T Q over these 16 queries (one k-step)
-        const uint32_t p0 = pack_bf16x2(pt[0][0], pt[0][1]), p1 = pack_bf16x2(pt[0][2], pt[0][3]);
-        const uint32_t p2 = pack_bf16x2(pt[1][0], pt[1][1]), p3 = pack_bf16x2(pt[1][2], pt[1][3]);
-        const uint32_t s0 = pack_bf16x2(dst[0][0], dst[0][1]), s1 = pack_bf16x2(dst[0][2], dst[0][3]);
-        const uint32_t s2 = pack_bf16x2(dst[1][0], dst[1][1]), s3 = pack_bf16x2(dst[1][2], dst[1][3]);
-#pragma unroll
-        for (int dp = 0; dp < HD / 16; ++dp) {
-          uint32_t b0, b1, b2, b3;
-          ldsm_x4_t(frag_addr<HD>(da, qs * 16, dp * 16, true), b0, b1, b2, b3);
-          mma_bf16_16816(dv[2 * dp], p0, p1, p2, p3, b0, b1);
-          mma_bf16_16816(dv[2 * dp + 1], p0, p1, p2, p3, b2, b3);
-          ldsm_x4_t(frag_addr<HD>(qa, qs * 16, dp * 16, true), b0, b1, b2, b3);
-          mma_bf16_16816(dk[2 * dp], s0, s1, s2, s3, b0, b1);
-          mma_bf16_16816(dk[2 * dp + 1], s0, s1, s2, s3, b2, b3);
-        }
+      for (int dp = 0; dp < HD / 16; ++dp) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4_t(frag_addr<HD>(da, qs * 16, dp * 16, true), b0, b1, b2, b3);
+        mma_bf16_16816(dv[2 * dp], p0, p1, p2, p3, b0, b1);
+        mma_bf16_16816(dv[2 * dp + 1], p0, p1, p2, p3, b2, b3);
+        ldsm_x4_t(frag_addr<HD>(qa, qs * 16, dp * 16, true), b0, b1, b2, b3);
+        mma_bf16_16816(dk[2 * dp], s0, s1, s2, s3, b0, b1);
+        mma_bf16_16816(dk[2 * dp + 1], s0, s1, s2, s3, b2, b3);
       }
     }
+    __syncthreads();  // buffer it & 1 is refilled with pair it + 2 next
   }
 #pragma unroll
   for (int i = 0; i < 2; ++i) {
@@ -585,7 +648,7 @@ template <int HD>
 cudaError_t attn_launch(const AttnArgs& a, bool backward, cudaStream_t st) {
   const dim3 grid(static_cast<unsigned>(a.S / kBlk), static_cast<unsigned>(a.nh), static_cast<unsigned>(a.B));
   if (!backward) {
-    const int smem = 3 * Tile<HD>::kBytes;
+    const int smem = 5 * Tile<HD>::kBytes;
     cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     attn_fwd_kernel<HD><<<grid, kAttnThreads, smem, st>>>(a);
@@ -595,12 +658,12 @@ cudaError_t attn_launch(const AttnArgs& a, bool backward, cudaStream_t st) {
   attn_delta_kernel<HD><<<elem_grid(rows * 32), kRowThreads, 0, st>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const int smem_q = 4 * Tile<HD>::kBytes;
+  const int smem_q = 6 * Tile<HD>::kBytes;
   e = cudaFuncSetAttribute(attn_bwd_dq_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_q);
   if (e != cudaSuccess) return e;
   attn_bwd_dq_kernel<HD><<<grid, kAttnThreads, smem_q, st>>>(a);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  const int smem_k = 4 * Tile<HD>::kBytes + 2 * kBlk * static_cast<int>(sizeof(float));
+  const int smem_k = 6 * Tile<HD>::kBytes + 4 * kBlk * static_cast<int>(sizeof(float));
   e = cudaFuncSetAttribute(attn_bwd_dkdv_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_k);
   if (e != cudaSuccess) return e;
   const dim3 gk(static_cast<unsigned>(a.S / kBlk), static_cast<unsigned>(a.nkv), static_cast<unsigned>(a.B));
