@@ -117,29 +117,111 @@ __global__ void __launch_bounds__(kRowThreads) rope_kernel(uint16_t* __restrict_
   }
 }
 
-// ---------------------------------------------------------------- SwiGLU and add
+// Rows of 8 consecutive elements of d = 16 k (half = 8 k) heads: one thread per (token, 8
+// consecutive i), its 8 angles computed once and applied to every head of the token with
+// 16-byte loads and stores.
+__global__ void __launch_bounds__(kRowThreads) rope_vec_kernel(uint16_t* __restrict__ x, int64_t T, int64_t S,
+                                                                int32_t nheads, int32_t d, float log2_base,
+                                                                int32_t inverse) {
+  const int32_t half = d / 2, groups = half / 8;
+  const int64_t items = T * groups;
+  for (int64_t e = blockIdx.x * (int64_t)kRowThreads + threadIdx.x; e < items; e += (int64_t)gridDim.x * kRowThreads) {
+    const int32_t i0 = static_cast<int32_t>(e % groups) * 8;
+    const int64_t t = e / groups;
+    const float pos = static_cast<float>(t % S);
+    float cs[8], sn[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float inv_freq = exp2f(-log2_base * (2.0f * (i0 + j)) / static_cast<float>(d));
+      sincosf(pos * inv_freq, &sn[j], &cs[j]);
+      if (inverse) sn[j] = -sn[j];
+    }
+    for (int32_t h = 0; h < nheads; ++h) {
+      uint16_t* p = x + (t * nheads + h) * d;
+      const uint4 av = *reinterpret_cast<const uint4*>(p + i0), bv = *reinterpret_cast<const uint4*>(p + i0 + half);
+      const uint32_t aw[4] = {av.x, av.y, av.z, av.w}, bw[4] = {bv.x, bv.y, bv.z, bv.w};
+      uint32_t ow[4], qw[4];
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const float a0 = bf16lo_to_f32(aw[w]), a1 = bf16hi_to_f32(aw[w]);
+        const float b0 = bf16lo_to_f32(bw[w]), b1 = bf16hi_to_f32(bw[w]);
+        const int j = 2 * w;
+        ow[w] = pack_bf16x2(a0 * cs[j] - b0 * sn[j], a1 * cs[j + 1] - b1 * sn[j + 1]);
+        qw[w] = pack_bf16x2(a0 * sn[j] + b0 * cs[j], a1 * sn[j + 1] + b1 * cs[j + 1]);
+      }
+      *reinterpret_cast<uint4*>(p + i0) = make_uint4(ow[0], ow[1], ow[2], ow[3]);
+      *reinterpret_cast<uint4*>(p + i0 + half) = make_uint4(qw[0], qw[1], qw[2], qw[3]);
+    }
+  }
+}
+
+// ---------------------------------------------------------------- SwiGLU
+// Eight elements per thread and iteration (16-byte loads and stores); block 0 takes the tail.
 __device__ __forceinline__ float sigmoidf(float a) { return 1.0f / (1.0f + expf(-a)); }
+
+__device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8]) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    f[2 * i] = bf16lo_to_f32(w[i]);
+    f[2 * i + 1] = bf16hi_to_f32(w[i]);
+  }
+}
+
+__device__ __forceinline__ uint4 pack8(const float (&f)[8]) {
+  return make_uint4(pack_bf16x2(f[0], f[1]), pack_bf16x2(f[2], f[3]), pack_bf16x2(f[4], f[5]),
+                    pack_bf16x2(f[6], f[7]));
+}
 
 __global__ void __launch_bounds__(kRowThreads) swiglu_fwd_kernel(const uint16_t* __restrict__ gt,
                                                                   const uint16_t* __restrict__ u, int64_t n,
                                                                   uint16_t* __restrict__ m) {
-  for (int64_t e = blockIdx.x * (int64_t)kRowThreads + threadIdx.x; e < n; e += (int64_t)gridDim.x * kRowThreads) {
-    const float a = bf16_at(gt, e);
-    m[e] = to_bf16(a * sigmoidf(a) * bf16_at(u, e));
+  const int64_t nvec = n / 8;
+  for (int64_t e = blockIdx.x * (int64_t)kRowThreads + threadIdx.x; e < nvec; e += (int64_t)gridDim.x * kRowThreads) {
+    float a[8], b[8], o[8];
+    unpack8(reinterpret_cast<const uint4*>(gt)[e], a);
+    unpack8(reinterpret_cast<const uint4*>(u)[e], b);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) o[i] = a[i] * sigmoidf(a[i]) * b[i];
+    reinterpret_cast<uint4*>(m)[e] = pack8(o);
   }
+  if (blockIdx.x == 0)
+    for (int64_t e = nvec * 8 + threadIdx.x; e < n; e += kRowThreads) {
+      const float a = bf16_at(gt, e);
+      m[e] = to_bf16(a * sigmoidf(a) * bf16_at(u, e));
+    }
 }
 
 // d_gate = dm u sigma(a) (1 + a (1 - sigma(a))), d_up = dm a sigma(a).
+__device__ __forceinline__ void swiglu_grad(float a, float b, float g, float& dg, float& du) {
+  const float s = sigmoidf(a);
+  dg = g * b * s * (1.0f + a * (1.0f - s));
+  du = g * a * s;
+}
+
 __global__ void __launch_bounds__(kRowThreads) swiglu_bwd_kernel(const uint16_t* __restrict__ gt,
                                                                   const uint16_t* __restrict__ u,
                                                                   const uint16_t* __restrict__ dm, int64_t n,
                                                                   uint16_t* __restrict__ dgt,
                                                                   uint16_t* __restrict__ du) {
-  for (int64_t e = blockIdx.x * (int64_t)kRowThreads + threadIdx.x; e < n; e += (int64_t)gridDim.x * kRowThreads) {
-    const float a = bf16_at(gt, e), s = sigmoidf(a), g = bf16_at(dm, e);
-    dgt[e] = to_bf16(g * bf16_at(u, e) * s * (1.0f + a * (1.0f - s)));
-    du[e] = to_bf16(g * a * s);
+  const int64_t nvec = n / 8;
+  for (int64_t e = blockIdx.x * (int64_t)kRowThreads + threadIdx.x; e < nvec; e += (int64_t)gridDim.x * kRowThreads) {
+    float a[8], b[8], g[8], dg[8], dd[8];
+    unpack8(reinterpret_cast<const uint4*>(gt)[e], a);
+    unpack8(reinterpret_cast<const uint4*>(u)[e], b);
+    unpack8(reinterpret_cast<const uint4*>(dm)[e], g);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) swiglu_grad(a[i], b[i], g[i], dg[i], dd[i]);
+    reinterpret_cast<uint4*>(dgt)[e] = pack8(dg);
+    reinterpret_cast<uint4*>(du)[e] = pack8(dd);
   }
+  if (blockIdx.x == 0)
+    for (int64_t e = nvec * 8 + threadIdx.x; e < n; e += kRowThreads) {
+      float dg, dd;
+      swiglu_grad(bf16_at(gt, e), bf16_at(u, e), bf16_at(dm, e), dg, dd);
+      dgt[e] = to_bf16(dg);
+      du[e] = to_bf16(dd);
+    }
 }
 
 // Block output in fp32, out = h + branch, and (with a teacher output) Eq. 7's loss: partial
@@ -524,7 +606,7 @@ __global__ void __launch_bounds__(kAttnThreads) attn_bwd_dq_kernel(const AttnArg
 
 // dK, dV: one CTA per (key block, key/value head, sequence), over every query head of the
 // group and the query blocks from the diagonal on (one stream of (head, query block) pairs
-// through two buffers of Q, dO and their rows' log-sum-exp and delta), 16 queries at a time.
+// through two buffers of Q, dO and their rows' log-sum-exp and delta), 32 queries at a time.
 // Scores are formed transposed (keys as rows) so that P^T and dS^T feed the A operand from
 // registers.
 template <int HD>
@@ -575,52 +657,69 @@ __global__ void __launch_bounds__(kAttnThreads) attn_bwd_dkdv_kernel(const AttnA
     const float* lse_s = lsd0 + (it & 1) * 2 * kBlk;
     const float* dl_s = lse_s + kBlk;
 #pragma unroll 1
-    for (int qs = 0; qs < kBlk / 16; ++qs) {
-      // S^T and dP^T of the warp's 16 keys against 16 queries: two n-tiles each
-      float st[2][4], dpt[2][4];
+    for (int qs = 0; qs < kBlk / 32; ++qs) {
+      // S^T and dP^T of the warp's 16 keys against 32 queries: four n-tiles each
+      float st[4][4], dpt[4][4];
 #pragma unroll
-      for (int nt = 0; nt < 2; ++nt)
+      for (int nt = 0; nt < 4; ++nt)
 #pragma unroll
         for (int e = 0; e < 4; ++e) st[nt][e] = dpt[nt][e] = 0.0f;
 #pragma unroll
       for (int kk = 0; kk < HD / 16; ++kk) {
         uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
         ldsm_x4(frag_addr<HD>(ka, warp * 16, kk * 16, true), a0, a1, a2, a3);
-        ldsm_x4(frag_addr<HD>(qa, qs * 16, kk * 16, false), b0, b1, b2, b3);
-        mma_bf16_16816(st[0], a0, a1, a2, a3, b0, b1);
-        mma_bf16_16816(st[1], a0, a1, a2, a3, b2, b3);
-        ldsm_x4(frag_addr<HD>(va, warp * 16, kk * 16, true), a0, a1, a2, a3);
-        ldsm_x4(frag_addr<HD>(da, qs * 16, kk * 16, false), b0, b1, b2, b3);
-        mma_bf16_16816(dpt[0], a0, a1, a2, a3, b0, b1);
-        mma_bf16_16816(dpt[1], a0, a1, a2, a3, b2, b3);
-      }
-      float pt[2][4], dst[2][4];
 #pragma unroll
-      for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int qry = qs * 16 + nt * 8 + 2 * t4 + (e & 1);  // within the query block
-          const int key = warp * 16 + g + (e >> 1) * 8;          // within the key block
-          float p = exp2f((st[nt][e] * a.scale - lse_s[qry]) * 1.4426950408889634f);
-          if (qb == kb && key > qry) p = 0.0f;
-          pt[nt][e] = p;
-          dst[nt][e] = p * (dpt[nt][e] - dl_s[qry]);
+        for (int hq = 0; hq < 2; ++hq) {
+          ldsm_x4(frag_addr<HD>(qa, qs * 32 + hq * 16, kk * 16, false), b0, b1, b2, b3);
+          mma_bf16_16816(st[2 * hq], a0, a1, a2, a3, b0, b1);
+          mma_bf16_16816(st[2 * hq + 1], a0, a1, a2, a3, b2, b3);
         }
-      // dV += P^T dO and dK += dS^T Q over these 16 queries (one k-step)
-      const uint32_t p0 = pack_bf16x2(pt[0][0], pt[0][1]), p1 = pack_bf16x2(pt[0][2], pt[0][3]);
-      const uint32_t p2 = pack_bf16x2(pt[1][0], pt[1][1]), p3 = pack_bf16x2(pt[1][2], pt[1][3]);
-      const uint32_t s0 = pack_bf16x2(dst[0][0], dst[0][1]), s1 = pack_bf16x2(dst[0][2], dst[0][3]);
-      const uint32_t s2 = pack_bf16x2(dst[1][0], dst[1][1]), s3 = pack_bf16x2(dst[1][2], dst[1][3]);
+        ldsm_x4(frag_addr<HD>(va, warp * 16, kk * 16, true), a0, a1, a2, a3);
 #pragma unroll
-      for (int dp = 0; dp < HD / 16; ++dp) {
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(frag_addr<HD>(da, qs * 16, dp * 16, true), b0, b1, b2, b3);
-        mma_bf16_16816(dv[2 * dp], p0, p1, p2, p3, b0, b1);
-        mma_bf16_16816(dv[2 * dp + 1], p0, p1, p2, p3, b2, b3);
-        ldsm_x4_t(frag_addr<HD>(qa, qs * 16, dp * 16, true), b0, b1, b2, b3);
-        mma_bf16_16816(dk[2 * dp], s0, s1, s2, s3, b0, b1);
-        mma_bf16_16816(dk[2 * dp + 1], s0, s1, s2, s3, b2, b3);
+        for (int hq = 0; hq < 2; ++hq) {
+          ldsm_x4(frag_addr<HD>(da, qs * 32 + hq * 16, kk * 16, false), b0, b1, b2, b3);
+          mma_bf16_16816(dpt[2 * hq], a0, a1, a2, a3, b0, b1);
+          mma_bf16_16816(dpt[2 * hq + 1], a0, a1, a2, a3, b2, b3);
+        }
       }
+      uint32_t pk[2][4], sk[2][4];  // P^T and dS^T as bf16 A fragments, one per 16 queries
+#pragma unroll
+      for (int hq = 0; hq < 2; ++hq) {
+        float pt[2][4], dst[2][4];
+#pragma unroll
+        for (int j = 0; j < 2; ++j)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int nt = 2 * hq + j;
+            const int qry = qs * 32 + nt * 8 + 2 * t4 + (e & 1);  // within the query block
+            const int key = warp * 16 + g + (e >> 1) * 8;          // within the key block
+            float p = exp2f((st[nt][e] * a.scale - lse_s[qry]) * 1.4426950408889634f);
+            if (qb == kb && key > qry) p = 0.0f;
+            pt[j][e] = p;
+            dst[j][e] = p * (dpt[nt][e] - dl_s[qry]);
+          }
+        pk[hq][0] = pack_bf16x2(pt[0][0], pt[0][1]);
+        pk[hq][1] = pack_bf16x2(pt[0][2], pt[0][3]);
+        pk[hq][2] = pack_bf16x2(pt[1][0], pt[1][1]);
+        pk[hq][3] = pack_bf16x2(pt[1][2], pt[1][3]);
+        sk[hq][0] = pack_bf16x2(dst[0][0], dst[0][1]);
+        sk[hq][1] = pack_bf16x2(dst[0][2], dst[0][3]);
+        sk[hq][2] = pack_bf16x2(dst[1][0], dst[1][1]);
+        sk[hq][3] = pack_bf16x2(dst[1][2], dst[1][3]);
+      }
+      // dV += P^T dO and dK += dS^T Q over these 32 queries (two k-steps)
+#pragma unroll
+      for (int hq = 0; hq < 2; ++hq)
+#pragma unroll
+        for (int dp = 0; dp < HD / 16; ++dp) {
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_t(frag_addr<HD>(da, qs * 32 + hq * 16, dp * 16, true), b0, b1, b2, b3);
+          mma_bf16_16816(dv[2 * dp], pk[hq][0], pk[hq][1], pk[hq][2], pk[hq][3], b0, b1);
+          mma_bf16_16816(dv[2 * dp + 1], pk[hq][0], pk[hq][1], pk[hq][2], pk[hq][3], b2, b3);
+          ldsm_x4_t(frag_addr<HD>(qa, qs * 32 + hq * 16, dp * 16, true), b0, b1, b2, b3);
+          mma_bf16_16816(dk[2 * dp], sk[hq][0], sk[hq][1], sk[hq][2], sk[hq][3], b0, b1);
+          mma_bf16_16816(dk[2 * dp + 1], sk[hq][0], sk[hq][1], sk[hq][2], sk[hq][3], b2, b3);
+        }
     }
     __syncthreads();  // buffer it & 1 is refilled with pair it + 2 next
   }
@@ -702,19 +801,23 @@ cudaError_t launch_rmsnorm_bwd(const void* x, bool x_f32, const float* gamma, co
 
 cudaError_t launch_rope(void* x, int64_t T, int64_t S, int32_t nheads, int32_t d, float base, int32_t inverse,
                         cudaStream_t st) {
-  rope_kernel<<<elem_grid(T * nheads * (d / 2)), kRowThreads, 0, st>>>(static_cast<uint16_t*>(x), T, S, nheads, d,
-                                                                        log2f(base), inverse);
+  if (d % 16 == 0)
+    rope_vec_kernel<<<elem_grid(T * (d / 16)), kRowThreads, 0, st>>>(static_cast<uint16_t*>(x), T, S, nheads, d,
+                                                                      log2f(base), inverse);
+  else
+    rope_kernel<<<elem_grid(T * nheads * (d / 2)), kRowThreads, 0, st>>>(static_cast<uint16_t*>(x), T, S, nheads, d,
+                                                                          log2f(base), inverse);
   return cudaGetLastError();
 }
 
 cudaError_t launch_swiglu(const void* gt, const void* u, const void* dm, int64_t n, void* out, void* dgt, void* du,
                           cudaStream_t st) {
   if (!dm)
-    swiglu_fwd_kernel<<<elem_grid(n), kRowThreads, 0, st>>>(static_cast<const uint16_t*>(gt),
+    swiglu_fwd_kernel<<<elem_grid((n + 7) / 8), kRowThreads, 0, st>>>(static_cast<const uint16_t*>(gt),
                                                              static_cast<const uint16_t*>(u), n,
                                                              static_cast<uint16_t*>(out));
   else
-    swiglu_bwd_kernel<<<elem_grid(n), kRowThreads, 0, st>>>(
+    swiglu_bwd_kernel<<<elem_grid((n + 7) / 8), kRowThreads, 0, st>>>(
         static_cast<const uint16_t*>(gt), static_cast<const uint16_t*>(u), static_cast<const uint16_t*>(dm), n,
         static_cast<uint16_t*>(dgt), static_cast<uint16_t*>(du));
   return cudaGetLastError();

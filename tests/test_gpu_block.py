@@ -91,7 +91,7 @@ def test_rmsnorm_bwd_two_consumers_and_residual(device, h_dtype):
     assert U.fro_rel(_f32(dX), O.rmsnorm_bwd(h, gamma, r_ref.astype(np.float32), dz)) <= U.TOL_BF16
 
 
-@pytest.mark.parametrize("S,nh,d,base", [(2048, 8, 128, 500000.0), (5, 3, 64, 10000.0)])
+@pytest.mark.parametrize("S,nh,d,base", [(2048, 8, 128, 500000.0), (5, 3, 64, 10000.0), (7, 2, 24, 10000.0)])
 def test_rope_and_inverse(device, S, nh, d, base):
     from paper_2606_26650_gb300 import catq as C
     T = 2 * S
