@@ -129,6 +129,7 @@ struct FusedArgs {
   int64_t ncols;    // columns of C
   int32_t num_m_tiles, num_n_tiles, num_k_blocks;
   int32_t group_m;  // M blocks per raster group
+  int32_t a_keep;   // a raster group's A rows fit L2 comfortably: keep them (evict_last), stream W
   WaitCtl wc;
   // Grouped launches (E > 0): expert e owns rows [row0[e], row0[e+1]) of A and C, W rows
   // [e N, (e+1) N) of the stacked weights, operand constants from float e * const_stride
@@ -476,6 +477,9 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
   if (warp == kTmaWarp) {
     if (lane == 0) {
       // ---------------------------------------------------------- TMA: A tiles (to the MMA)
+      // A raster group's A rows are read by every tile wave of the group: kept in L2 ahead of
+      // the streamed W tiles when they fit comfortably (args.a_keep).
+      const uint64_t pol_a = args.a_keep ? l2_policy_evict_last() : l2_policy_evict_normal();
       uint32_t q = 0, issued_mask = 0, issued_phase = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
@@ -489,8 +493,8 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
 #pragma unroll
           for (int acc = 0; acc < NACC; ++acc) {
             const int32_t row = m0 + acc * Cfg::kRowsPerAcc + cta * 128;
-            if constexpr (CG == 1) tma_load_2d(dst + acc * (128 * BK * 2), &tmA, fb, kb * BK, row);
-            else tma_load_2d_pair(dst + acc * (128 * BK * 2), &tmA, fb, kb * BK, row);
+            if constexpr (CG == 1) tma_load_2d_hint(dst + acc * (128 * BK * 2), &tmA, fb, kb * BK, row, pol_a);
+            else tma_load_2d_pair_hint(dst + acc * (128 * BK * 2), &tmA, fb, kb * BK, row, pol_a);
           }
           issued_mask |= 1u << s;
           issued_phase = (issued_phase & ~(1u << s)) | (ph << s);
@@ -501,6 +505,8 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
           if (issued_mask & (1u << s)) mbar_wait_drain(full_a(s), (issued_phase >> s) & 1u);
     } else if (lane == 1) {
       // ---------------------------------------------------------- TMA: raw W tiles this CTA produces
+      // (a W tile serves the raster group's M blocks at about the same time, then is done)
+      const uint64_t pol_w = args.a_keep ? l2_policy_evict_first() : l2_policy_evict_normal();
       uint32_t q = 0, issued_mask = 0, issued_phase = 0;
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
@@ -516,11 +522,11 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
           mbar_arrive_expect_tx(raw_w(rb), Cfg::kWBytes);
           const uint32_t dst = w_base + s * Cfg::kWBytes;
           if constexpr (!B_MN) {
-            tma_load_2d(dst, &tmW, raw_w(rb), kb * BK, wrow + n0);
+            tma_load_2d_hint(dst, &tmW, raw_w(rb), kb * BK, wrow + n0, pol_w);
           } else {
 #pragma unroll
             for (int b = 0; b < Cfg::kBRows / 64; ++b)
-              tma_load_2d(dst + b * 8192, &tmW, raw_w(rb), n0 + 64 * b, wrow + kb * BK);
+              tma_load_2d_hint(dst + b * 8192, &tmW, raw_w(rb), n0 + 64 * b, wrow + kb * BK, pol_w);
           }
           issued_mask |= 1u << rb;
           issued_phase = (issued_phase & ~(1u << rb)) | (rph << rb);
@@ -550,7 +556,7 @@ __global__ void __launch_bounds__(FusedCfg<CG, PAIRS>::kThreads, 1)
       };
       // An accumulator whose rows all lie past the tile's last row (an expert's short last M
       // block, or a ragged M) gets no MMAs; the epilogue stores nothing from it.
-      bool live[NACC];
+      bool live[NACC] = {};
       auto issue = [&](uint32_t qq, int acc, bool first) {  // one accumulator's MMAs of stage qq
         if (!live[acc]) return;
         const uint32_t aa = a_base + (qq % SA) * Cfg::kABytes, ww = w_base + (qq % SW) * Cfg::kWBytes;
@@ -963,6 +969,7 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
   if (warp == kTma) {
     if (lane == 0) {
       uint32_t stage = 0, phase = 0, issued_mask = 0, issued_phase = 0, it_tma = 0;
+      const uint64_t pol_keep = l2_policy_evict_last();
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
         const int r = t % tiles_per_split;
@@ -987,6 +994,9 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
           const int32_t m = kb * BK;
           if (cta == 0) mbar_arrive_expect_tx(full(stage), Cfg::kStageBytes * CG);
           const uint32_t fb = leader_full0 + 8u * stage;
+          // X is read by every tile wave, so it is kept in L2 ahead of the W the epilogue
+          // streams (dY keeps the normal policy: its column blocks serve every k block of their
+          // n rows within one wave).
 #pragma unroll
           for (int b = 0; b < 2; ++b) {
             const int32_t n = n_blk * Cfg::kTileRows + cta * 128 + 64 * b;
@@ -996,8 +1006,8 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
 #pragma unroll
           for (int b = 0; b < Cfg::kBCols / 64; ++b) {
             const int32_t k = k_blk * BN + cta * Cfg::kBCols + 64 * b;
-            if constexpr (CG == 1) tma_load_2d(sb + b * 8192, mx, fb, k, m);
-            else tma_load_2d_pair(sb + b * 8192, mx, fb, k, m);
+            if constexpr (CG == 1) tma_load_2d_hint(sb + b * 8192, mx, fb, k, m, pol_keep);
+            else tma_load_2d_pair_hint(sb + b * 8192, mx, fb, k, m, pol_keep);
           }
           issued_mask |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -1048,6 +1058,7 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
     const int64_t plane = args.L.N * cpr;
     const float k_sc = args.sc.s * args.sc.inv_2tanh_s;
     const float inv_k = (MU && k_sc > 0.0f) ? 1.0f / k_sc : 0.0f;
+    const uint64_t pol_w = l2_policy_evict_first();
     uint32_t it = 0;
     for (int t = cluster; t < num_tiles; t += nclusters, ++it) {
       const int split = t / tiles_per_split, r = t % tiles_per_split;
@@ -1072,12 +1083,12 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
       GradSums acc{0.f, 0.f, 0.f};
       constexpr int kChunks = (BN / 2) / 32;
       const int64_t k0 = (int64_t)k_blk * BN + half * (BN / 2);
-      auto load_w = [&](int c, uint4 (&dst)[4]) {
+      auto load_w = [&](int c, uint4 (&dst)[4]) {  // W is read once per launch: streamed through L2
         const int64_t k = k0 + c * 32;
         if (row_ok && k < L.K) {
           const uint4* wp = reinterpret_cast<const uint4*>(W + n * L.K + k);
 #pragma unroll
-          for (int v = 0; v < 4; ++v) dst[v] = __ldg(wp + v);
+          for (int v = 0; v < 4; ++v) dst[v] = ldg_hint(wp + v, pol_w);
         }
       };
       // The first two chunks' weights and the group constants the tile starts in are requested
@@ -1319,6 +1330,12 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
   args.num_n_tiles = static_cast<int32_t>((ncols + BN - 1) / BN);
   args.num_k_blocks = static_cast<int32_t>((depth + BK - 1) / BK);
   args.group_m = std::min(4, args.num_m_tiles);
+  {
+    // A rows of one raster group: kept in L2 when they take at most a third of it (dense
+    // launches; grouped ones stream every expert's W once and reuse little A)
+    const int64_t group_rows = static_cast<int64_t>(args.group_m) * Cfg::kTileRows * PAIRS;
+    args.a_keep = (!grp && std::min<int64_t>(group_rows, M) * depth * 2 <= (int64_t(40) << 20)) ? 1 : 0;
+  }
   args.wc = make_wait_ctl(d);
   args.E = 0;
   args.const_stride = 0;
