@@ -45,10 +45,11 @@ LR0 = 1e-3
 UPDATES = 60 * -(-512 // 3)
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per launch, mean over the
-# seven linears of the 8B-shaped block step, from one ncu capture of the timed step; keyed
-# by the hash of the sources it was taken at and reported only while they are unchanged.
-TRAFFIC = {"sha": "3ae0826043f5be2e", "workload": "c3_llama3_8b_block",
-           "fwd": 415440823, "dx": 438257774, "dw": 921276343}
+# seven linears of the 8B-shaped block step, each captured alone (bench.py --linear NAME, the
+# SOFT forward, dX and dW launches of the warm-up step; profiles/traffic_c3_linears.md); keyed
+# by the hash of the kernel sources it was taken at and reported only while they are unchanged.
+TRAFFIC = {"sha": "f9fca6678c1bda23", "workload": "c3_llama3_8b_block",
+           "fwd": 383949641, "dx": 410839845, "dw": 474656951}
 
 
 def parse(argv=None):

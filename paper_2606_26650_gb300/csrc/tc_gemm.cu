@@ -188,7 +188,22 @@ struct DwArgs {
   int32_t num_n_tiles, num_k_tiles;
   WaitCtl wc;
   int32_t n_experts;  // grouped: experts of this launch (0: dense)
+  int32_t x_keep;     // X (the contraction's K side) fits L2 comfortably: keep it (evict_last)
+  int32_t k_group;    // raster: k blocks per group (see dw_tile)
 };
+
+// Tile r of a split (or expert) of the dW launch: its n block and k block.  Tiles run in groups
+// of k_group k blocks; inside a group the k block varies fastest, then the n block.  A wave of
+// C clusters then covers about C / k_group n blocks x k_group k blocks, so it reads
+// (C / k_group + k_group) column slices of dY and X (M x 256 each) instead of all of X's, which
+// k-fastest order over the whole K reads every wave.
+__device__ __forceinline__ void dw_tile(const DwArgs& a, int r, int& n_blk, int& k_blk) {
+  const int per_group = a.k_group * a.num_n_tiles;
+  const int gi = r / per_group, rr = r - gi * per_group;
+  const int kw = min(a.k_group, a.num_k_tiles - gi * a.k_group);
+  n_blk = rr / kw;
+  k_blk = gi * a.k_group + rr % kw;
+}
 
 // Grouped dW launch: up to kDwGroupExperts experts with rows, each with tensor maps over its
 // own rows of dY and X (so the contraction stops at the expert's last row: rows past it
@@ -969,11 +984,12 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
   if (warp == kTma) {
     if (lane == 0) {
       uint32_t stage = 0, phase = 0, issued_mask = 0, issued_phase = 0, it_tma = 0;
-      const uint64_t pol_keep = l2_policy_evict_last();
+      const uint64_t pol_keep = args.x_keep ? l2_policy_evict_last() : l2_policy_evict_normal();
       bool ok = true;
       for (int t = cluster; ok && t < num_tiles; t += nclusters) {
         const int r = t % tiles_per_split;
-        const int k_blk = r % args.num_k_tiles, n_blk = r / args.num_k_tiles;
+        int k_blk, n_blk;
+        dw_tile(args, r, n_blk, k_blk);
         int kb0, kb1;
         kb_range(t, kb0, kb1);
         const void* mdy = &tmDY;
@@ -995,8 +1011,8 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
           if (cta == 0) mbar_arrive_expect_tx(full(stage), Cfg::kStageBytes * CG);
           const uint32_t fb = leader_full0 + 8u * stage;
           // X is read by every tile wave, so it is kept in L2 ahead of the W the epilogue
-          // streams (dY keeps the normal policy: its column blocks serve every k block of their
-          // n rows within one wave).
+          // streams when it fits (args.x_keep); dY keeps the normal policy: its column blocks
+          // serve every k block of their n rows within one wave.
 #pragma unroll
           for (int b = 0; b < 2; ++b) {
             const int32_t n = n_blk * Cfg::kTileRows + cta * 128 + 64 * b;
@@ -1062,7 +1078,8 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
     uint32_t it = 0;
     for (int t = cluster; t < num_tiles; t += nclusters, ++it) {
       const int split = t / tiles_per_split, r = t % tiles_per_split;
-      const int k_blk = r % args.num_k_tiles, n_blk = r / args.num_k_tiles;
+      int k_blk, n_blk;
+      dw_tile(args, r, n_blk, k_blk);
       // the tile's layer: the dense one, or (grouped) its expert's slice of the stacked layer
       // (grouped: the expert's weights and per-group arrays start e N K elements and e G
       // groups after expert 0's; its group j is group jbase + j of the stacked arrays)
@@ -1365,6 +1382,14 @@ cudaError_t run_fused(const LayerDev& L, StepScalars sc, const void* A, int64_t 
                            st, params);
 }
 
+// k blocks per raster group of the dW launch: about the square root of the clusters, so that
+// a wave's tiles span as many n blocks as k blocks.
+int dw_k_group(int num_k_tiles, int clusters) {
+  int kg = 1;
+  while ((kg + 1) * (kg + 1) <= clusters) ++kg;
+  return std::max(1, std::min(kg, num_k_tiles));
+}
+
 template <int CG, bool MU>
 cudaError_t run_dw(const LayerDev& L, StepScalars sc, const void* X, const void* dY, int64_t M, const TcPlan& plan,
                    float* part, cudaStream_t st) {
@@ -1388,6 +1413,12 @@ cudaError_t run_dw(const LayerDev& L, StepScalars sc, const void* X, const void*
   args.num_k_tiles = static_cast<int32_t>((L.K + BN - 1) / BN);
   args.wc = make_wait_ctl(d);
   args.n_experts = 0;
+  // every tile wave reads all of X: kept in L2 when it takes at most about 60 % of it (a
+  // larger X under evict_last thrashes the cache it cannot fit)
+  args.x_keep = M * L.K * 2 <= (int64_t(80) << 20) ? 1 : 0;
+  // X kept in L2: every wave may read all of it (k fastest over the whole K, each dY slice
+  // then read by one wave); otherwise waves about as wide in n as in k
+  args.k_group = args.x_keep ? args.num_k_tiles : dw_k_group(args.num_k_tiles, d.sm_count / CG);
   const int tiles = args.num_n_tiles * args.num_k_tiles * args.splits;
   const int clusters = std::min(tiles, d.sm_count / CG);
   void* params[4] = {&tdy, &tx, &args, &unused_maps};
@@ -1416,6 +1447,8 @@ cudaError_t run_dw_grouped(const LayerDev& L0, StepScalars sc, const void* X, co
   args.kb_per_split = 0;
   args.num_n_tiles = static_cast<int32_t>((L0.N + Cfg::kTileRows - 1) / Cfg::kTileRows);
   args.num_k_tiles = static_cast<int32_t>((L0.K + BN - 1) / BN);
+  args.x_keep = 0;  // an expert's rows are few: its X is read by few waves
+  args.k_group = dw_k_group(args.num_k_tiles, d.sm_count / CG);
   const uint16_t* x = static_cast<const uint16_t*>(X);
   const uint16_t* dy = static_cast<const uint16_t*>(dY);
   int32_t e = 0;
