@@ -285,3 +285,80 @@ def test_block_teacher_phase_has_zero_loss(device):
     assert got["loss"] == 0.0
     assert np.array_equal(got["out"], got["out_ref"])
     assert all(np.all(t == 0.0) for n in got["g"] for t in got["g"][n])
+
+
+def test_block_calibration_loop_matches_oracle(device):
+    """The block window's calibration loop (§8(f) row 1): epochs of block steps under the
+    epoch schedule of Eq. 6 (SOFT epochs of rising sharpness, then HARD), each followed by
+    AdamW on every linear's three factors at the linearly decayed learning rate, on the GPU
+    and in the oracle from the same seeded block.  Per-step losses within 2e-2 and each
+    linear's factor movement (end minus start) within 2e-2 relative Frobenius error, the bar of
+    the gradients the loop integrates; the loss falls on both sides."""
+    import torch
+
+    from paper_2606_26650_gb300 import block as BK
+    from paper_2606_26650_gb300 import catq as C
+    shape = BK.BlockShape(**dict(SMALL, S=64))
+    g, batches, m, gamma, s0, lr0 = 128, 2, 6, 4 / 6, 30.0, 1e-3
+    W, _, g1, g2, _ = _block_case(shape, g, 3)
+    r = syn.rng(98, "block_loop")
+    xs = [syn.round_bf16(r.standard_t(4.0, (shape.T, shape.H)).astype(np.float32)) for _ in range(batches)]
+    G = {n: W[n].size // g for n in W}
+    names = list(BK.LINEARS)
+    # oracle loop
+    stats = {n: O.group_stats(W[n], g) for n in names}
+    fac = {n: (np.zeros(G[n]), np.ones(G[n]), np.ones(G[n])) for n in names}
+    mom = {n: (np.zeros(G[n]),) * 6 for n in names}
+    losses_o, t = [], 0
+    for e in range(1, m + 1):
+        phase, s = O.schedule_at_epoch(e, m, gamma, s0)
+        for x in xs:
+            step = O.block_calibration_step(x, W, g, stats, fac, g1, g2, shape.B, shape.S, shape.n_heads,
+                                            shape.n_kv_heads, shape.d, shape.base, shape.eps, phase, s)
+            losses_o.append(step["loss"])
+            lr = O.linear_decay_lr(lr0, t, m * batches)
+            t += 1
+            for n in names:
+                fac[n], mom[n] = O.factor_update(fac[n], step["g"][n], mom[n], t, lr)
+    # GPU loop
+    Wd = {n: U.to_device(w, "bf16", device) for n, w in W.items()}
+    blk = BK.Block(shape, Wd, torch.from_numpy(g1).to(device), torch.from_numpy(g2).to(device), g)
+    xds = [U.to_device(x, "bf16", device) for x in xs]
+    refs = []
+    for xd in xds:
+        o = torch.empty(shape.T, shape.H, dtype=torch.float32, device=device)
+        blk.teacher(xd, o)
+        refs.append(o)
+    grads = {n: [torch.empty(G[n], dtype=torch.float32, device=device) for _ in range(3)] for n in names}
+    moments = {n: torch.zeros(6 * G[n], dtype=torch.float32, device=device) for n in names}
+    hp = C.adamw()
+    loss = torch.zeros(1, dtype=torch.float32, device=device)
+    losses_g = torch.zeros(m * batches, dtype=torch.float32, device=device)
+    t = 0
+    for e in range(1, m + 1):
+        sched = C.catq_schedule_at_epoch(e, m, gamma, s0)
+        for xd, ref in zip(xds, refs):
+            blk.step(xd, ref, sched, loss, grads)
+            losses_g[t].copy_(loss[0])
+            lr = C.catq_linear_decay_lr(lr0, t, m * batches)
+            t += 1
+            for n in names:
+                L = blk.layers[n]
+                C.catq_factor_adamw_step(L.d_mu, L.d_alpha, L.d_delta, *grads[n], moments[n], hp, t, lr)
+    torch.cuda.synchronize()
+    assert C.catq_device_status() == 0
+    lg, lo = U.to_host(losses_g).astype(np.float64), np.array(losses_o)
+    rel = np.abs(lg - lo) / np.abs(lo)
+    moves = {}
+    for n in names:
+        L = blk.layers[n]
+        start = (np.zeros(G[n]), np.ones(G[n]), np.ones(G[n]))
+        got = tuple(U.to_host(f).astype(np.float64) for f in (L.d_mu, L.d_alpha, L.d_delta))
+        for name, a, b, s0_ in zip(("d_mu", "d_alpha", "d_delta"), got, fac[n], start):
+            moves[f"{n}.{name}"] = U.fro_rel(a - s0_, b - s0_)
+    print(f"block loop: worst step loss error {rel.max():.3e}, worst factor movement error "
+          f"{max(moves.values()):.3e}, loss {lo[0]:.4e} -> {lo[-1]:.4e}")
+    assert rel.max() <= U.TOL_BF16, rel
+    bad = {k: v for k, v in moves.items() if not v <= U.TOL_BF16}
+    assert not bad, bad
+    assert lo[-1] < lo[0] and lg[-1] < lg[0]
