@@ -544,14 +544,24 @@ def swiglu_bwd(gt, u, dm):
 BLOCK_LINEARS = ("q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj")
 
 
-def block_forward(x, Wq, gamma1, gamma2, B, S, nh, nkv, d, base, eps):
+def _head_norm(x, gamma, d, eps):
+    """RMSNorm of every head (rows of d elements) of x [T, heads d]; returns (y, r per head)."""
+    y, r = rmsnorm(np.asarray(x, np.float64).reshape(-1, d), gamma, eps)
+    return y.reshape(np.shape(x)), r
+
+
+def block_forward(x, Wq, gamma1, gamma2, B, S, nh, nkv, d, base, eps, q_norm=None, k_norm=None):
     """One decoder block with the effective weights Wq[name] ([N, K] each):
-    z1 = RMSNorm(x); q, k, v = z1 W^T; rotary q, k; a = attention; h = x + a Wo^T;
+    z1 = RMSNorm(x); q, k, v = z1 W^T; (Qwen3: RMSNorm of every query and key head with the
+    weights q_norm, k_norm [d]); rotary q, k; a = attention; h = x + a Wo^T;
     z2 = RMSNorm(h); m = silu(z2 Wg^T) * (z2 Wu^T); out = h + m Wd^T.  Returns (out, cache)."""
     x = np.asarray(x, np.float64)
     z1, r1 = rmsnorm(x, gamma1, eps)
-    q = rope(linear_fwd(z1, Wq["q_proj"]), S, nh, d, base)
-    k = rope(linear_fwd(z1, Wq["k_proj"]), S, nkv, d, base)
+    qp, kp = linear_fwd(z1, Wq["q_proj"]), linear_fwd(z1, Wq["k_proj"])
+    qn, rq = _head_norm(qp, q_norm, d, eps) if q_norm is not None else (qp, None)
+    kn, rk = _head_norm(kp, k_norm, d, eps) if k_norm is not None else (kp, None)
+    q = rope(qn, S, nh, d, base)
+    k = rope(kn, S, nkv, d, base)
     v = linear_fwd(z1, Wq["v_proj"])
     a, p = attention(q, k, v, B, S, nh, nkv, d)
     h = x + linear_fwd(a, Wq["o_proj"])
@@ -560,11 +570,12 @@ def block_forward(x, Wq, gamma1, gamma2, B, S, nh, nkv, d, base, eps):
     u = linear_fwd(z2, Wq["up_proj"])
     m = swiglu(gt, u)
     out = h + linear_fwd(m, Wq["down_proj"])
-    return out, dict(z1=z1, q=q, k=k, v=v, a=a, p=p, h=h, z2=z2, r2=r2, gt=gt, u=u, m=m)
+    return out, dict(z1=z1, qp=qp, kp=kp, rq=rq, rk=rk, q=q, k=k, v=v, a=a, p=p, h=h, z2=z2, r2=r2, gt=gt, u=u,
+                     m=m)
 
 
 def block_calibration_step(x, W, g, stats, factors, gamma1, gamma2, B, S, nh, nkv, d, base, eps, phase, s,
-                           reduction=0):
+                           reduction=0, q_norm=None, k_norm=None):
     """One calibration step of a window of one decoder block (Eq. 7 over the block output):
     the teacher block with full-precision weights, the block with each linear's Eq. 6 weight
     (W, stats, factors: dicts by linear name), the loss, and every linear's factor gradients
@@ -573,8 +584,8 @@ def block_calibration_step(x, W, g, stats, factors, gamma1, gamma2, B, S, nh, nk
     g_dalpha, g_ddelta)."""
     Wq = {n: ternary_weight(W[n], g, stats[n], factors[n], phase, s)[0] for n in BLOCK_LINEARS}
     out_ref, _ = block_forward(x, {n: np.asarray(W[n], np.float64) for n in BLOCK_LINEARS}, gamma1, gamma2, B,
-                               S, nh, nkv, d, base, eps)
-    out, c = block_forward(x, Wq, gamma1, gamma2, B, S, nh, nkv, d, base, eps)
+                               S, nh, nkv, d, base, eps, q_norm, k_norm)
+    out, c = block_forward(x, Wq, gamma1, gamma2, B, S, nh, nkv, d, base, eps, q_norm, k_norm)
     loss, d_out = recon_loss(out, out_ref, reduction)
     G = {}
 
@@ -592,7 +603,12 @@ def block_calibration_step(x, W, g, stats, factors, gamma1, gamma2, B, S, nh, nk
     grads("o_proj", c["a"], dh)
     da = dh @ Wq["o_proj"]
     dq, dk, dv = attention_bwd(c["q"], c["k"], c["v"], c["p"], da, B, S, nh, nkv, d)
-    grads("q_proj", c["z1"], rope(dq, S, nh, d, base, inverse=True))
-    grads("k_proj", c["z1"], rope(dk, S, nkv, d, base, inverse=True))
+    dq, dk = rope(dq, S, nh, d, base, inverse=True), rope(dk, S, nkv, d, base, inverse=True)
+    if q_norm is not None:
+        dq = rmsnorm_bwd(c["qp"].reshape(-1, d), q_norm, c["rq"], dq.reshape(-1, d)).reshape(dq.shape)
+    if k_norm is not None:
+        dk = rmsnorm_bwd(c["kp"].reshape(-1, d), k_norm, c["rk"], dk.reshape(-1, d)).reshape(dk.shape)
+    grads("q_proj", c["z1"], dq)
+    grads("k_proj", c["z1"], dk)
     grads("v_proj", c["z1"], dv)
     return dict(out=out, out_ref=out_ref, loss=loss, g=G, cache=c)

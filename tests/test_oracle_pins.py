@@ -898,25 +898,28 @@ def _tiny_block(seed=80, B=2, S=5, nh=4, nkv=2, d=4, I=12, g=4):
     x = r.standard_normal((B * S, H))
     gamma1 = r.uniform(0.5, 1.5, H)
     gamma2 = r.uniform(0.5, 1.5, H)
+    qk = dict(q_norm=r.uniform(0.5, 1.5, d), k_norm=r.uniform(0.5, 1.5, d))
     return dict(x=x, W=W, g=g, stats=stats, fac=fac, gamma1=gamma1, gamma2=gamma2, B=B, S=S, nh=nh, nkv=nkv,
-                d=d, base=10000.0, eps=1e-5)
+                d=d, base=10000.0, eps=1e-5, qk=qk)
 
 
-def _block_loss(blk, fac, s):
+def _block_loss(blk, fac, s, qk_norm=False):
     return O.block_calibration_step(blk["x"], blk["W"], blk["g"], blk["stats"], fac, blk["gamma1"], blk["gamma2"],
                                     blk["B"], blk["S"], blk["nh"], blk["nkv"], blk["d"], blk["base"], blk["eps"],
-                                    O.PHASE_SOFT, s)["loss"]
+                                    O.PHASE_SOFT, s, **(blk["qk"] if qk_norm else {}))["loss"]
 
 
-def test_block_factor_gradients_match_central_differences():
+@pytest.mark.parametrize("qk_norm", [False, True])
+def test_block_factor_gradients_match_central_differences(qk_norm):
     """The block's backward (SwiGLU, RMSNorm with the residual, attention with grouped heads,
-    rotary embedding, every linear's chain rule) against central differences of the block
-    loss, for sampled groups of every linear and all three factors, soft phase."""
+    rotary embedding, every linear's chain rule; with qk_norm the per-head query/key RMSNorm of
+    the Qwen3 block) against central differences of the block loss, for sampled groups of
+    every linear and all three factors, soft phase."""
     blk = _tiny_block()
     s = 3.0
     step = O.block_calibration_step(blk["x"], blk["W"], blk["g"], blk["stats"], blk["fac"], blk["gamma1"],
                                     blk["gamma2"], blk["B"], blk["S"], blk["nh"], blk["nkv"], blk["d"], blk["base"],
-                                    blk["eps"], O.PHASE_SOFT, s)
+                                    blk["eps"], O.PHASE_SOFT, s, **(blk["qk"] if qk_norm else {}))
     r = np.random.default_rng(81)
     h = 1e-6
     for name in O.BLOCK_LINEARS:
@@ -927,7 +930,7 @@ def test_block_factor_gradients_match_central_differences():
                 fm = {n: tuple(a.copy() for a in f) for n, f in blk["fac"].items()}
                 fp[name][q][j] += h
                 fm[name][q][j] -= h
-                fd = (_block_loss(blk, fp, s) - _block_loss(blk, fm, s)) / (2 * h)
+                fd = (_block_loss(blk, fp, s, qk_norm) - _block_loss(blk, fm, s, qk_norm)) / (2 * h)
                 got = step["g"][name][q][j]
                 assert got == pytest.approx(fd, rel=1e-5, abs=1e-10 * max(1.0, abs(fd))), (name, q, j)
 
@@ -1057,3 +1060,19 @@ def test_swiglu_gradients_match_central_differences():
     # silu(0) = 0 and silu's slope at 0 is 1/2
     np.testing.assert_allclose(O.swiglu(np.zeros(2), np.ones(2)), 0.0, atol=0)
     np.testing.assert_allclose(O.swiglu_bwd(np.zeros(1), np.ones(1), np.ones(1))[0], 0.5, rtol=1e-15)
+
+
+def test_block_head_norm_is_rmsnorm_per_head_and_changes_the_block():
+    """The Qwen3 query/key norm normalises each head on its own: scaling one head's q_proj rows
+    leaves the block output unchanged (RMSNorm is scale-invariant per row up to eps), while the
+    block without the norm changes."""
+    blk = _tiny_block(seed=84)
+    W2 = {n: w.copy() for n, w in blk["W"].items()}
+    W2["q_proj"][: blk["d"]] *= 7.0  # head 0's rows
+    args = (blk["gamma1"], blk["gamma2"], blk["B"], blk["S"], blk["nh"], blk["nkv"], blk["d"], blk["base"], 0.0)
+    o1, _ = O.block_forward(blk["x"], blk["W"], *args, **blk["qk"])
+    o2, _ = O.block_forward(blk["x"], W2, *args, **blk["qk"])
+    np.testing.assert_allclose(o1, o2, rtol=1e-12, atol=1e-12)
+    p1, _ = O.block_forward(blk["x"], blk["W"], *args)
+    p2, _ = O.block_forward(blk["x"], W2, *args)
+    assert np.abs(p1 - p2).max() > 1e-3
