@@ -521,7 +521,7 @@ def run_ours(args):
         also[f"{wl.name}/decode_b1_staged"] = measure_decode(C, torch, wl, dev, peaks, rows=1, staged=True)
         also["c5_qwen3_235b_moe/soft"] = measure_moe(C, torch, dev, peaks, world, args.s)
         also[f"{wl.name}/fig_error_k_proj"] = measure_fig_error(C, torch, wl, dev, args.s)
-        if wl.name == "c3_llama3_8b_block" and not args.linear:
+        if wl.name in BLOCK_WINDOW_SHAPES and not args.linear:
             also[f"{wl.name}/block_window"] = measure_block_window(C, torch, wl, dev, peaks, world, args.s, barrier)
         for name in ALSO_WORKLOADS:
             if name == wl.name:
@@ -531,6 +531,8 @@ def run_ours(args):
             also[f"{name}/soft"] = dict(entry(wl2, b2.ms_per_step(sched, n2, w2, barrier)), phase="soft", s=args.s)
             del b2
             torch.cuda.empty_cache()
+            if name in BLOCK_WINDOW_SHAPES and not args.linear:
+                also[f"{name}/block_window"] = measure_block_window(C, torch, wl2, dev, peaks, world, args.s, barrier)
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -556,16 +558,28 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+# Decoder blocks of the block-window lines: (hidden, query heads, key/value heads, head dim,
+# MLP width, sequences, tokens per sequence, RoPE base, per-head query/key norm).  The Llama-3-8B
+# block has no query/key norm; the Qwen3 blocks normalise every query and key head.
+BLOCK_WINDOW_SHAPES = {
+    "c3_llama3_8b_block": (4096, 32, 8, 128, 14336, 4, 2048, 500000.0, False),
+    "c4_qwen3_14b_block": (5120, 40, 8, 128, 17408, 2, 2048, 1000000.0, True),
+    "c2_qwen3_1p7b_block": (2048, 16, 8, 128, 6144, 4, 2048, 1000000.0, True),
+}
+
+
 def measure_block_window(C, torch, wl, dev, peaks, world, s, barrier, steps=5, warmup=3):
-    """Eq. 7 over a window of one whole decoder block (§2.4) on the Llama-3-8B shape: 4 x 2048
-    tokens, 32 query heads and 8 key/value heads of 128, RoPE base 500000.  One step is the
-    student block forward (seven soft-ternary linears, RMSNorm, rotary embedding, causal
-    attention, SwiGLU), the loss on the block output against the cached teacher output, the
-    block backward into every linear's factor gradients, and the AdamW update of all factors.
-    Throughput counts the linears' 6 T N K and attention's 7 B h S^2 d flops; the attention
-    forward + backward is also timed alone on the same tensors."""
+    """Eq. 7 over a window of one whole decoder block (§2.4) of the workload's shape (e.g. the
+    Llama-3-8B block: 4 x 2048 tokens, 32 query heads and 8 key/value heads of 128, RoPE base
+    500000).  One step is the student block forward (seven soft-ternary linears, RMSNorm,
+    rotary embedding, causal attention, SwiGLU; the Qwen3 blocks' query/key head norms), the
+    loss on the block output against the cached teacher output, the block backward into every
+    linear's factor gradients, and the AdamW update of all factors.  Throughput counts the
+    linears' 6 T N K and attention's 7 B h S^2 d flops; the attention forward + backward is also
+    timed alone on the same tensors."""
     from paper_2606_26650_gb300 import block as BK
-    shape = BK.BlockShape(H=4096, n_heads=32, n_kv_heads=8, d=128, I=14336, B=4, S=2048, base=500000.0, eps=1e-5)
+    H, nh, nkv, d, I, B, S, base, qk_norm = BLOCK_WINDOW_SHAPES[wl.name]
+    shape = BK.BlockShape(H=H, n_heads=nh, n_kv_heads=nkv, d=d, I=I, B=B, S=S, base=base, eps=1e-5)
     assert shape.T == wl.M
     bf = torch.bfloat16
 
@@ -577,7 +591,10 @@ def measure_block_window(C, torch, wl, dev, peaks, world, s, barrier, steps=5, w
     g1, g2 = (torch.from_numpy(r.uniform(0.5, 1.5, shape.H).astype(np.float32)).to(dev) for _ in range(2))
     fac = {n: tuple(torch.from_numpy(f).to(dev) for f in syn.factors(W[n].numel() // wl.g, 0, f"window/{n}", True))
            for n in W}
-    blk = BK.Block(shape, W, g1, g2, wl.g, factors=fac)
+    norms = {}
+    if qk_norm:
+        norms = {k: torch.from_numpy(r.uniform(0.5, 1.5, d).astype(np.float32)).to(dev) for k in ("q_norm", "k_norm")}
+    blk = BK.Block(shape, W, g1, g2, wl.g, factors=fac, **norms)
     x = upload(syn.activations(wl, "x_hidden", shape.T, shape.H))
     out_ref = torch.empty(shape.T, shape.H, dtype=torch.float32, device=dev)
     blk.teacher(x, out_ref)
@@ -623,7 +640,7 @@ def measure_block_window(C, torch, wl, dev, peaks, world, s, barrier, steps=5, w
            "flops_per_step": {"linears": shape.linear_flops(), "attention": shape.attention_flops()},
            "attention_fwd_bwd_ms": attn_ms,
            "attention_tflops": shape.attention_flops() / (attn_ms * 1e-3) / 1e12,
-           "loss_after_steps": first_loss, "phase": "soft", "s": s,
+           "loss_after_steps": first_loss, "phase": "soft", "s": s, "qk_norm": qk_norm,
            "shape": dataclasses.asdict(shape), "l2": "working set > L2 (no flush)"}
     del blk, W, x, out_ref, grads, upd
     torch.cuda.empty_cache()
@@ -970,7 +987,8 @@ def run_only(args):
         rows = int(args.only[len("decode_b"):].split("_")[0])
         r = measure_decode(C, torch, wl, dev, peaks, rows=rows, steps=args.steps, staged="staged" in args.only)
     else:
-        r = measure_block_window(C, torch, wl, dev, peaks, 1, args.s, barrier, steps=args.steps, warmup=args.warmup)
+        bw = syn.WORKLOADS[args.workload] if args.workload in BLOCK_WINDOW_SHAPES else wl
+        r = measure_block_window(C, torch, bw, dev, peaks, 1, args.s, barrier, steps=args.steps, warmup=args.warmup)
     print(json.dumps({"only": args.only, **r}), flush=True)
 
 

@@ -4,8 +4,8 @@ are soft-ternary (Eq. 6 weight at the schedule's point), the block-output loss, 
 linear's factor gradients through the block's backward.
 
 Llama-family block (pre-norm, causal grouped-query attention with rotary position embedding,
-SwiGLU MLP); tokens are rows t = b S + s of [B S, H] activations.  The linears' inputs and
-outputs are bf16; the residual stream (h = x + attention branch, out = h + MLP branch) stays in
+SwiGLU MLP; with q_norm / k_norm the Qwen3 block, which normalises every query and key head);
+tokens are rows t = b S + s of [B S, H] activations.  The linears' inputs and outputs are bf16; the residual stream (h = x + attention branch, out = h + MLP branch) stays in
 fp32 and the loss is taken on the fp32 block output, so that the difference between student
 and teacher is not lost to the rounding of a value the size of the residual.  The block input
 x (bf16 or fp32) is the window's input and receives no gradient.  Every step here is a call
@@ -56,9 +56,12 @@ class BlockShape:
 class Block:
     """Device state and buffers of one block.  W: dict of bf16 [N, K] CUDA tensors by linear
     name; gamma1, gamma2: fp32 [H] norm weights; g: group size; factors: optional dict of
-    (d_mu, d_alpha, d_delta) fp32 tensors by name (identity otherwise)."""
+    (d_mu, d_alpha, d_delta) fp32 tensors by name (identity otherwise); q_norm, k_norm:
+    optional fp32 [d] weights of the Qwen3 block's RMSNorm of every query and key head (applied
+    to the projections' outputs before the rotary embedding)."""
 
-    def __init__(self, shape: BlockShape, W, gamma1, gamma2, g, factors=None, thr_init=C.THR_HALF, stream=None):
+    def __init__(self, shape: BlockShape, W, gamma1, gamma2, g, factors=None, thr_init=C.THR_HALF, stream=None,
+                 q_norm=None, k_norm=None):
         import torch
         self.shape, self.g, self.stream = shape, g, stream
         dev = W["q_proj"].device
@@ -72,6 +75,9 @@ class Block:
             self.layers[name] = C.Layer.create(W[name], g, *(f if f is not None else (None, None, None)))
             C.catq_group_stats(self.layers[name], thr_init, stream=stream)
         self.gamma1, self.gamma2 = gamma1, gamma2
+        if (q_norm is None) != (k_norm is None):
+            raise ValueError("q_norm and k_norm come together")
+        self.q_norm, self.k_norm = q_norm, k_norm
         T, H, I = shape.T, shape.H, shape.I
         qd, kvd = shape.n_heads * shape.d, shape.n_kv_heads * shape.d
         bf = dict(dtype=torch.bfloat16, device=dev)
@@ -91,6 +97,9 @@ class Block:
         self.dz2a, self.dz2b, self.dh = e(T, H, **bf), e(T, H, **bf), e(T, H, **bf)
         self.da, self.dq, self.dk, self.dv = e(T, qd, **bf), e(T, qd, **bf), e(T, kvd, **bf), e(T, kvd, **bf)
         self.delta = e(shape.B * shape.n_heads * shape.S, **f32)
+        if q_norm is not None:  # the projections' outputs before the head norm, and its RMS factors
+            self.qp, self.kp = e(T, qd, **bf), e(T, kvd, **bf)
+            self.rq, self.rk = e(T * shape.n_heads, **f32), e(T * shape.n_kv_heads, **f32)
         ws = max(C.catq_bwd_workspace_bytes(L, T) for L in self.layers.values())
         self.bwd_ws = C.workspace(ws, dev)
         self.loss_ws = C.workspace(C.catq_recon_loss_workspace_bytes(T * H), dev)
@@ -102,8 +111,14 @@ class Block:
         with out_ref, Eq. 7's loss into loss[0] and its gradient into the backward's d_out."""
         sh, st, L = self.shape, self.stream, self.layers
         C.catq_rmsnorm_fwd(x, self.gamma1, self.z1, self.r1, sh.eps, stream=st)
-        C.catq_soft_ternary_linear_fwd(L["q_proj"], sched, self.z1, self.q, stream=st)
-        C.catq_soft_ternary_linear_fwd(L["k_proj"], sched, self.z1, self.k, stream=st)
+        if self.q_norm is None:
+            C.catq_soft_ternary_linear_fwd(L["q_proj"], sched, self.z1, self.q, stream=st)
+            C.catq_soft_ternary_linear_fwd(L["k_proj"], sched, self.z1, self.k, stream=st)
+        else:
+            C.catq_soft_ternary_linear_fwd(L["q_proj"], sched, self.z1, self.qp, stream=st)
+            C.catq_soft_ternary_linear_fwd(L["k_proj"], sched, self.z1, self.kp, stream=st)
+            C.catq_rmsnorm_fwd(self.qp.view(-1, sh.d), self.q_norm, self.q.view(-1, sh.d), self.rq, sh.eps, stream=st)
+            C.catq_rmsnorm_fwd(self.kp.view(-1, sh.d), self.k_norm, self.k.view(-1, sh.d), self.rk, sh.eps, stream=st)
         C.catq_soft_ternary_linear_fwd(L["v_proj"], sched, self.z1, self.v, stream=st)
         C.catq_rope(self.q, sh.S, sh.n_heads, sh.d, sh.base, stream=st)
         C.catq_rope(self.k, sh.S, sh.n_kv_heads, sh.d, sh.base, stream=st)
@@ -140,6 +155,11 @@ class Block:
                              sh.B, sh.S, sh.n_heads, sh.n_kv_heads, sh.d, stream=st)
         C.catq_rope(self.dq, sh.S, sh.n_heads, sh.d, sh.base, inverse=True, stream=st)
         C.catq_rope(self.dk, sh.S, sh.n_kv_heads, sh.d, sh.base, inverse=True, stream=st)
+        if self.q_norm is not None:  # through the head norm, in place
+            C.catq_rmsnorm_bwd(self.qp.view(-1, sh.d), self.q_norm, self.rq, self.dq.view(-1, sh.d),
+                               self.dq.view(-1, sh.d), stream=st)
+            C.catq_rmsnorm_bwd(self.kp.view(-1, sh.d), self.k_norm, self.rk, self.dk.view(-1, sh.d),
+                               self.dk.view(-1, sh.d), stream=st)
         self._bwd("q_proj", sched, self.z1, self.dq, None, grads)
         self._bwd("k_proj", sched, self.z1, self.dk, None, grads)
         self._bwd("v_proj", sched, self.z1, self.dv, None, grads)

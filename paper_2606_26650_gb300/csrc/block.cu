@@ -14,6 +14,8 @@
 // head, so no atomics are needed and the result is deterministic.
 #include <cuda_bf16.h>
 
+#include <algorithm>
+
 #include "launch.h"
 #include "ptx_sm100.cuh"
 
@@ -72,11 +74,9 @@ __global__ void __launch_bounds__(kRowThreads) rmsnorm_fwd_kernel(const TX* __re
 template <typename TH>
 __global__ void __launch_bounds__(kRowThreads) rmsnorm_bwd_kernel(const TH* __restrict__ x,
                                                                    const float* __restrict__ gamma,
-                                                                   const float* __restrict__ r,
-                                                                   const uint16_t* __restrict__ dy,
-                                                                   const uint16_t* __restrict__ dy2,
-                                                                   const uint16_t* __restrict__ dres, int64_t H,
-                                                                   uint16_t* __restrict__ dx) {
+                                                                   const float* __restrict__ r, const uint16_t* dy,
+                                                                   const uint16_t* dy2, const uint16_t* dres,
+                                                                   int64_t H, uint16_t* dx) {  // dx may alias
   __shared__ float red[kRowThreads / 32];
   const int64_t t = blockIdx.x;
   const float rr = r[t];
@@ -91,6 +91,68 @@ __global__ void __launch_bounds__(kRowThreads) rmsnorm_bwd_kernel(const TH* __re
     float v = rr * gamma[i] * g - load_act(x, t * H + i) * c;
     if (dres) v += bf16_at(dres, t * H + i);
     dx[t * H + i] = to_bf16(v);
+  }
+}
+
+// Rows of at most 1024 elements (e.g. one attention head, the Qwen3 query/key norm): one warp
+// per row, the same arithmetic as the kernels above.
+constexpr int kRowWarps = kRowThreads / 32;
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+template <typename TX>
+__global__ void __launch_bounds__(kRowThreads) rmsnorm_fwd_warp_kernel(const TX* __restrict__ x,
+                                                                        const uint16_t* __restrict__ res,
+                                                                        const float* __restrict__ gamma, int64_t T,
+                                                                        int64_t H, float eps,
+                                                                        float* __restrict__ h_out,
+                                                                        uint16_t* __restrict__ z,
+                                                                        float* __restrict__ r) {
+  const int lane = threadIdx.x & 31;
+  for (int64_t t = (blockIdx.x * (int64_t)kRowWarps) + (threadIdx.x >> 5); t < T; t += (int64_t)gridDim.x * kRowWarps) {
+    float ss = 0.0f;
+    for (int64_t i = lane; i < H; i += 32) {
+      float h = load_act(x, t * H + i);
+      if (res) h += bf16_at(res, t * H + i);
+      if (h_out) h_out[t * H + i] = h;
+      ss = fmaf(h, h, ss);
+    }
+    const float rr = rsqrtf(warp_sum(ss) / static_cast<float>(H) + eps);
+    if (lane == 0) r[t] = rr;
+    for (int64_t i = lane; i < H; i += 32) {
+      float h = load_act(x, t * H + i);
+      if (res) h += bf16_at(res, t * H + i);
+      z[t * H + i] = to_bf16(gamma[i] * h * rr);
+    }
+  }
+}
+
+template <typename TH>
+__global__ void __launch_bounds__(kRowThreads) rmsnorm_bwd_warp_kernel(const TH* __restrict__ x,
+                                                                        const float* __restrict__ gamma,
+                                                                        const float* __restrict__ r,
+                                                                        const uint16_t* dy, const uint16_t* dy2,
+                                                                        const uint16_t* dres, int64_t T, int64_t H,
+                                                                        uint16_t* dx) {  // dx may alias
+  const int lane = threadIdx.x & 31;
+  for (int64_t t = (blockIdx.x * (int64_t)kRowWarps) + (threadIdx.x >> 5); t < T; t += (int64_t)gridDim.x * kRowWarps) {
+    const float rr = r[t];
+    float sux = 0.0f;
+    for (int64_t i = lane; i < H; i += 32) {
+      const float g = bf16_at(dy, t * H + i) + (dy2 ? bf16_at(dy2, t * H + i) : 0.0f);
+      sux = fmaf(gamma[i] * g, load_act(x, t * H + i), sux);
+    }
+    const float c = warp_sum(sux) / static_cast<float>(H) * rr * rr * rr;
+    for (int64_t i = lane; i < H; i += 32) {
+      const float g = bf16_at(dy, t * H + i) + (dy2 ? bf16_at(dy2, t * H + i) : 0.0f);
+      float v = rr * gamma[i] * g - load_act(x, t * H + i) * c;
+      if (dres) v += bf16_at(dres, t * H + i);
+      dx[t * H + i] = to_bf16(v);
+    }
   }
 }
 
@@ -774,14 +836,24 @@ cudaError_t attn_launch(const AttnArgs& a, bool backward, cudaStream_t st) {
 
 cudaError_t launch_rmsnorm_fwd(const void* x, bool x_f32, const void* res, const float* gamma, int64_t T, int64_t H,
                                float eps, float* h_out, void* z, float* r, cudaStream_t st) {
+  const auto* rp = static_cast<const uint16_t*>(res);
+  auto* zp = static_cast<uint16_t*>(z);
+  if (H <= 1024) {
+    const unsigned grid = static_cast<unsigned>(std::min<int64_t>((T + kRowWarps - 1) / kRowWarps, 152 * 16));
+    if (x_f32)
+      rmsnorm_fwd_warp_kernel<float><<<grid, kRowThreads, 0, st>>>(static_cast<const float*>(x), rp, gamma, T, H, eps,
+                                                                   h_out, zp, r);
+    else
+      rmsnorm_fwd_warp_kernel<uint16_t><<<grid, kRowThreads, 0, st>>>(static_cast<const uint16_t*>(x), rp, gamma, T, H,
+                                                                      eps, h_out, zp, r);
+    return cudaGetLastError();
+  }
   if (x_f32)
-    rmsnorm_fwd_kernel<float><<<static_cast<unsigned>(T), kRowThreads, 0, st>>>(
-        static_cast<const float*>(x), static_cast<const uint16_t*>(res), gamma, H, eps, h_out,
-        static_cast<uint16_t*>(z), r);
+    rmsnorm_fwd_kernel<float><<<static_cast<unsigned>(T), kRowThreads, 0, st>>>(static_cast<const float*>(x), rp, gamma,
+                                                                                H, eps, h_out, zp, r);
   else
-    rmsnorm_fwd_kernel<uint16_t><<<static_cast<unsigned>(T), kRowThreads, 0, st>>>(
-        static_cast<const uint16_t*>(x), static_cast<const uint16_t*>(res), gamma, H, eps, h_out,
-        static_cast<uint16_t*>(z), r);
+    rmsnorm_fwd_kernel<uint16_t><<<static_cast<unsigned>(T), kRowThreads, 0, st>>>(static_cast<const uint16_t*>(x), rp,
+                                                                                   gamma, H, eps, h_out, zp, r);
   return cudaGetLastError();
 }
 
@@ -790,12 +862,23 @@ cudaError_t launch_rmsnorm_bwd(const void* x, bool x_f32, const float* gamma, co
   const auto* dyp = static_cast<const uint16_t*>(dy);
   const auto* dy2p = static_cast<const uint16_t*>(dy2);
   const auto* drp = static_cast<const uint16_t*>(dres);
+  auto* dxp = static_cast<uint16_t*>(dx);
+  if (H <= 1024) {
+    const unsigned grid = static_cast<unsigned>(std::min<int64_t>((T + kRowWarps - 1) / kRowWarps, 152 * 16));
+    if (x_f32)
+      rmsnorm_bwd_warp_kernel<float><<<grid, kRowThreads, 0, st>>>(static_cast<const float*>(x), gamma, r, dyp, dy2p,
+                                                                   drp, T, H, dxp);
+    else
+      rmsnorm_bwd_warp_kernel<uint16_t><<<grid, kRowThreads, 0, st>>>(static_cast<const uint16_t*>(x), gamma, r, dyp,
+                                                                      dy2p, drp, T, H, dxp);
+    return cudaGetLastError();
+  }
   if (x_f32)
-    rmsnorm_bwd_kernel<float><<<static_cast<unsigned>(T), kRowThreads, 0, st>>>(
-        static_cast<const float*>(x), gamma, r, dyp, dy2p, drp, H, static_cast<uint16_t*>(dx));
+    rmsnorm_bwd_kernel<float><<<static_cast<unsigned>(T), kRowThreads, 0, st>>>(static_cast<const float*>(x), gamma, r,
+                                                                                dyp, dy2p, drp, H, dxp);
   else
-    rmsnorm_bwd_kernel<uint16_t><<<static_cast<unsigned>(T), kRowThreads, 0, st>>>(
-        static_cast<const uint16_t*>(x), gamma, r, dyp, dy2p, drp, H, static_cast<uint16_t*>(dx));
+    rmsnorm_bwd_kernel<uint16_t><<<static_cast<unsigned>(T), kRowThreads, 0, st>>>(static_cast<const uint16_t*>(x),
+                                                                                   gamma, r, dyp, dy2p, drp, H, dxp);
   return cudaGetLastError();
 }
 

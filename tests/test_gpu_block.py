@@ -39,7 +39,8 @@ def _f32(t):
 
 # ---------------------------------------------------------------- the layers one by one
 
-@pytest.mark.parametrize("T,H,x_dtype", [(300, 512, "bf16"), (7, 4096, "f32"), (1, 136, "bf16")])
+@pytest.mark.parametrize("T,H,x_dtype", [(300, 512, "bf16"), (7, 4096, "f32"), (1, 136, "bf16"), (1999, 128, "bf16"),
+                                         (5, 1032, "f32")])
 def test_rmsnorm_fwd_with_residual(device, T, H, x_dtype):
     import torch
 
@@ -66,13 +67,14 @@ def test_rmsnorm_fwd_with_residual(device, T, H, x_dtype):
     assert U.fro_rel(_f32(Z), z0) <= U.TOL_BF16
 
 
-@pytest.mark.parametrize("h_dtype", ["f32", "bf16"])
-def test_rmsnorm_bwd_two_consumers_and_residual(device, h_dtype):
+@pytest.mark.parametrize("h_dtype,H", [("f32", 1024), ("bf16", 1024), ("f32", 2048), ("bf16", 128)])
+def test_rmsnorm_bwd_two_consumers_and_residual(device, h_dtype, H):
+    """Rows up to 1024 take the warp-per-row kernel, longer ones the CTA-per-row kernel."""
     import torch
 
     from paper_2606_26650_gb300 import catq as C
-    T, H = 257, 1024
-    r = syn.rng(91, f"rms_bwd/{h_dtype}")
+    T = 257
+    r = syn.rng(91, f"rms_bwd/{h_dtype}/{H}")
     h = r.standard_normal((T, H)).astype(np.float32)
     if h_dtype == "bf16":
         h = syn.round_bf16(h)
@@ -232,14 +234,16 @@ def _block_case(shape, g, seed, x_dtype="bf16"):
     return W, x, g1, g2, fac
 
 
-def _gpu_block(shape, W, x, g1, g2, fac, g, phase, s, device, x_dtype="bf16"):
+def _gpu_block(shape, W, x, g1, g2, fac, g, phase, s, device, x_dtype="bf16", qk=None):
     import torch
 
     from paper_2606_26650_gb300 import block as BK
     from paper_2606_26650_gb300 import catq as C
     Wd = {n: U.to_device(w, "bf16", device) for n, w in W.items()}
     facd = {n: tuple(torch.from_numpy(f.copy()).to(device) for f in fac[n]) for n in W}
-    blk = BK.Block(shape, Wd, torch.from_numpy(g1).to(device), torch.from_numpy(g2).to(device), g, factors=facd)
+    norms = {k: torch.from_numpy(v).to(device) for k, v in qk.items()} if qk else {}
+    blk = BK.Block(shape, Wd, torch.from_numpy(g1).to(device), torch.from_numpy(g2).to(device), g, factors=facd,
+                   **norms)
     xd = U.to_device(x, x_dtype, device)
     out_ref = torch.empty(shape.T, shape.H, dtype=torch.float32, device=device)
     blk.teacher(xd, out_ref)
@@ -253,17 +257,27 @@ def _gpu_block(shape, W, x, g1, g2, fac, g, phase, s, device, x_dtype="bf16"):
                 g={n: tuple(_f32(t) for t in grads[n]) for n in W})
 
 
-@pytest.mark.parametrize("phase,s,x_dtype", [(O.PHASE_SOFT, 30.0, "bf16"), (O.PHASE_SOFT, 0.625, "bf16"),
-                                             (O.PHASE_HARD, 30.0, "bf16"), (O.PHASE_SOFT, 30.0, "f32")])
-def test_block_step_matches_oracle(device, phase, s, x_dtype):
+@pytest.mark.parametrize("phase,s,x_dtype,qk_norm", [(O.PHASE_SOFT, 30.0, "bf16", False),
+                                                     (O.PHASE_SOFT, 0.625, "bf16", False),
+                                                     (O.PHASE_HARD, 30.0, "bf16", False),
+                                                     (O.PHASE_SOFT, 30.0, "f32", False),
+                                                     (O.PHASE_SOFT, 30.0, "bf16", True),
+                                                     (O.PHASE_HARD, 30.0, "bf16", True)])
+def test_block_step_matches_oracle(device, phase, s, x_dtype, qk_norm):
+    """qk_norm: the Qwen3 block (per-head query/key RMSNorm, RoPE base 1e6)."""
     from paper_2606_26650_gb300 import block as BK
-    shape = BK.BlockShape(**SMALL)
+    shape = BK.BlockShape(**dict(SMALL, base=1e6 if qk_norm else SMALL["base"]))
     g = 128
     W, x, g1, g2, fac = _block_case(shape, g, 1, x_dtype)
-    got = _gpu_block(shape, W, x, g1, g2, fac, g, phase, s, device, x_dtype)
+    qk = None
+    if qk_norm:
+        rq = syn.rng(99, "block/qk")
+        qk = {"q_norm": rq.uniform(0.5, 1.5, shape.d).astype(np.float32),
+              "k_norm": rq.uniform(0.5, 1.5, shape.d).astype(np.float32)}
+    got = _gpu_block(shape, W, x, g1, g2, fac, g, phase, s, device, x_dtype, qk=qk)
     stats = {n: O.group_stats(W[n], g) for n in W}
     ref = O.block_calibration_step(x, W, g, stats, fac, g1, g2, shape.B, shape.S, shape.n_heads, shape.n_kv_heads,
-                                   shape.d, shape.base, shape.eps, phase, s)
+                                   shape.d, shape.base, shape.eps, phase, s, **(qk or {}))
     errs = {"out_ref": U.fro_rel(got["out_ref"], ref["out_ref"]), "out": U.fro_rel(got["out"], ref["out"]),
             "out-out_ref": U.fro_rel(got["out"] - got["out_ref"], ref["out"] - ref["out_ref"]),
             "loss": abs(got["loss"] - ref["loss"]) / ref["loss"]}
