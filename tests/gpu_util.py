@@ -117,9 +117,11 @@ def gpu_step(W, X, g, fac, thr, phase, s, dtype, device, with_dx=True, recon=0, 
 
 
 def listing_dir():
-    """Where the near-threshold listings go: the run's output folder (not committed)."""
+    """Where the near-threshold listings go: $CATQ_LISTING_DIR, else near_threshold/ under the
+    system's temporary directory (never inside the repository)."""
     import os
-    d = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "gpurun_out", "near_threshold")
+    import tempfile
+    d = os.environ.get("CATQ_LISTING_DIR") or os.path.join(tempfile.gettempdir(), "catq_near_threshold")
     os.makedirs(d, exist_ok=True)
     return d
 
