@@ -117,8 +117,8 @@ def gpu_step(W, X, g, fac, thr, phase, s, dtype, device, with_dx=True, recon=0, 
 
 
 def listing_dir():
-    """Where the near-threshold listings go: $CATQ_LISTING_DIR, else near_threshold/ under the
-    system's temporary directory (never inside the repository)."""
+    """Where the near-threshold listings go: $CATQ_LISTING_DIR, else catq_near_threshold/ under
+    the system's temporary directory (never inside the repository)."""
     import os
     import tempfile
     d = os.environ.get("CATQ_LISTING_DIR") or os.path.join(tempfile.gettempdir(), "catq_near_threshold")
