@@ -1,17 +1,19 @@
 // block.cu — the layers around the seven soft-ternary linears of one decoder block, for the
 // block-output reconstruction step (§2.4, Eq. 7 over a window of one block): RMSNorm (with the
 // residual add fused into the forward, and the residual and second upstream gradient fused
-// into the backward), rotary position embedding, SwiGLU, an add, and causal grouped-query
-// attention (forward, and a deterministic backward in two kernels).
+// into the backward; one CTA per long row, one warp per short row such as an attention head),
+// rotary position embedding, SwiGLU, the fp32 block output with the loss on it, and causal
+// grouped-query attention (forward, and a deterministic backward in two kernels).
 //
 // Attention runs on the tensor pipe with mma.sync m16n8k16 (bf16 in, fp32 accumulate):
-// blocks of 64 queries (four warps of 16) against blocks of 64 keys staged in shared memory,
-// an online softmax in fp32 with the probabilities fed back as the A operand of P V straight
-// from the score accumulators, and operand fragments read from shared memory with ldmatrix
-// (transposed where the contraction runs along rows).  The backward recomputes the
-// probabilities from the forward's log-sum-exp: one kernel per query block accumulates dQ;
-// one per key block accumulates dK and dV over every query head that shares the key/value
-// head, so no atomics are needed and the result is deterministic.
+// blocks of 64 queries (four warps of 16) against blocks of 64 keys, which stream through two
+// shared-memory buffers by cp.async; an online softmax in fp32 with the probabilities fed back
+// as the A operand of P V straight from the score accumulators, and operand fragments read
+// from shared memory with ldmatrix (transposed where the contraction runs along rows).  The
+// backward recomputes the probabilities from the forward's log-sum-exp: one kernel per query
+// block accumulates dQ; one per key block accumulates dK and dV (32 queries per step) over
+// every query head that shares the key/value head, so no atomics are needed and the result is
+// deterministic.
 #include <cuda_bf16.h>
 
 #include <algorithm>
