@@ -802,13 +802,15 @@ def measure_fig_error(C, torch, wl, dev, s0, epochs=20, batches=3, rows=2048, lr
     return res
 
 
-def measure_moe(C, torch, dev, peaks, world, s, steps=5, warmup=2, experts=None):
+def measure_moe(C, torch, dev, peaks, world, s, steps=5, warmup=2, experts=None, nstreams=3):
     """One calibration step of the Qwen3-235B-shaped MoE layer: gate/up/down of all 128
     experts over 8192 tokens routed top-8 (65,536 expert-sorted rows, Zipf(1.1) loads) through
     the grouped calls (stats once; per step forward, loss, backward, factor update, pack).  Weights and
     activations are drawn on the device (seeded); value = sum 6 M_e N K / step time.
-    `experts` (profiling only) keeps the expert shape and routing law with fewer experts and
-    proportionally fewer tokens, so that a capture holds less device memory."""
+    The three linears are independent calibration problems (one loss per linear output), so a
+    step spreads them over `nstreams` CUDA streams, forking from and joining back into the
+    current stream.  `experts` (profiling only) keeps the expert shape and routing law with
+    fewer experts and proportionally fewer tokens, so that a capture holds less device memory."""
     wl = syn.WORKLOADS["c5_qwen3_235b_moe"]
     if experts:
         wl = dataclasses.replace(wl, experts=int(experts), tokens=wl.tokens * int(experts) // wl.experts)
@@ -841,16 +843,29 @@ def measure_moe(C, torch, dev, peaks, world, s, steps=5, warmup=2, experts=None)
                          wsl=C.workspace(C.catq_recon_loss_workspace_bytes(R * N), dev)))
         flops += 6.0 * R * N * K
     upd = FactorUpdate(C, torch, dev, [d["grads"][0].numel() for d in lins])
+    main = torch.cuda.current_stream()
+    lanes = [main] if nstreams <= 1 else [torch.cuda.Stream(device=dev) for _ in range(nstreams)]
 
     def step():
         upd.advance()
+        if len(lanes) > 1:
+            fork = torch.cuda.Event()
+            fork.record(main)
+            for ln in lanes:
+                ln.wait_event(fork)
         for i, d in enumerate(lins):
-            C.catq_grouped_soft_ternary_linear_fwd(d["layer"], sched, d["X"], off, d["Y"])
-            C.catq_recon_loss(d["Y"], d["Yt"], d["loss"], d["dY"], d["wsl"])
-            C.catq_grouped_soft_ternary_linear_bwd(d["layer"], sched, d["X"], d["dY"], off, d["dX"], *d["grads"],
-                                                   workspace=d["wsb"])
-            upd.apply(i, d["layer"].dense, d["grads"])
-            C.catq_hard_ternarize_pack(d["layer"].dense, d["codes"], d["alpha"])
+            with torch.cuda.stream(lanes[i % len(lanes)]):
+                C.catq_grouped_soft_ternary_linear_fwd(d["layer"], sched, d["X"], off, d["Y"])
+                C.catq_recon_loss(d["Y"], d["Yt"], d["loss"], d["dY"], d["wsl"])
+                C.catq_grouped_soft_ternary_linear_bwd(d["layer"], sched, d["X"], d["dY"], off, d["dX"], *d["grads"],
+                                                       workspace=d["wsb"])
+                upd.apply(i, d["layer"].dense, d["grads"])
+                C.catq_hard_ternarize_pack(d["layer"].dense, d["codes"], d["alpha"])
+        if len(lanes) > 1:
+            for ln in lanes:
+                join = torch.cuda.Event()
+                join.record(ln)
+                main.wait_event(join)
 
     for _ in range(warmup):
         step()
@@ -877,6 +892,7 @@ def measure_moe(C, torch, dev, peaks, world, s, steps=5, warmup=2, experts=None)
                                                                  int(counts.max())],
             "path": "grouped calls: one persistent launch for every expert's forward and dX tiles, grouped "
                     "factor-gradient launches of up to 64 experts",
+            "streams": len(lanes),
             "phase": "soft", "s": s, "host_issue_ms_per_step": host_ms, "clocks": clk.summary()}
 
 
@@ -982,7 +998,7 @@ def run_only(args):
 
     if args.only == "moe":
         r = measure_moe(C, torch, dev, peaks, 1, args.s, steps=args.steps, warmup=args.warmup,
-                        experts=args.moe_experts)
+                        experts=args.moe_experts, nstreams=args.streams)
     elif args.only.startswith("decode_b"):
         rows = int(args.only[len("decode_b"):].split("_")[0])
         r = measure_decode(C, torch, wl, dev, peaks, rows=rows, steps=args.steps, staged="staged" in args.only)
