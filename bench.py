@@ -522,7 +522,8 @@ def run_ours(args):
         also["c5_qwen3_235b_moe/soft"] = measure_moe(C, torch, dev, peaks, world, args.s)
         also[f"{wl.name}/fig_error_k_proj"] = measure_fig_error(C, torch, wl, dev, args.s)
         if wl.name in BLOCK_WINDOW_SHAPES and not args.linear:
-            also[f"{wl.name}/block_window"] = measure_block_window(C, torch, wl, dev, peaks, world, args.s, barrier)
+            also[f"{wl.name}/block_window"] = measure_block_window(C, torch, wl, dev, peaks, world, args.s, barrier,
+                                                                   streams=nstreams)
         for name in ALSO_WORKLOADS:
             if name == wl.name:
                 continue
@@ -532,7 +533,8 @@ def run_ours(args):
             del b2
             torch.cuda.empty_cache()
             if name in BLOCK_WINDOW_SHAPES and not args.linear:
-                also[f"{name}/block_window"] = measure_block_window(C, torch, wl2, dev, peaks, world, args.s, barrier)
+                also[f"{name}/block_window"] = measure_block_window(C, torch, wl2, dev, peaks, world, args.s, barrier,
+                                                                    streams=nstreams)
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -568,7 +570,7 @@ BLOCK_WINDOW_SHAPES = {
 }
 
 
-def measure_block_window(C, torch, wl, dev, peaks, world, s, barrier, steps=5, warmup=3):
+def measure_block_window(C, torch, wl, dev, peaks, world, s, barrier, steps=5, warmup=3, streams=4):
     """Eq. 7 over a window of one whole decoder block (§2.4) of the workload's shape (e.g. the
     Llama-3-8B block: 4 x 2048 tokens, 32 query heads and 8 key/value heads of 128, RoPE base
     500000).  One step is the student block forward (seven soft-ternary linears, RMSNorm,
@@ -576,7 +578,8 @@ def measure_block_window(C, torch, wl, dev, peaks, world, s, barrier, steps=5, w
     loss on the block output against the cached teacher output, the block backward into every
     linear's factor gradients, and the AdamW update of all factors.  Throughput counts the
     linears' 6 T N K and attention's 7 B h S^2 d flops; the attention forward + backward is also
-    timed alone on the same tensors."""
+    timed alone on the same tensors.  `streams`: the block's main stream and streams - 1 side
+    streams for its independent calls."""
     from paper_2606_26650_gb300 import block as BK
     H, nh, nkv, d, I, B, S, base, qk_norm = BLOCK_WINDOW_SHAPES[wl.name]
     shape = BK.BlockShape(H=H, n_heads=nh, n_kv_heads=nkv, d=d, I=I, B=B, S=S, base=base, eps=1e-5)
@@ -594,7 +597,7 @@ def measure_block_window(C, torch, wl, dev, peaks, world, s, barrier, steps=5, w
     norms = {}
     if qk_norm:
         norms = {k: torch.from_numpy(r.uniform(0.5, 1.5, d).astype(np.float32)).to(dev) for k in ("q_norm", "k_norm")}
-    blk = BK.Block(shape, W, g1, g2, wl.g, factors=fac, **norms)
+    blk = BK.Block(shape, W, g1, g2, wl.g, factors=fac, side_streams=max(0, streams - 1), **norms)
     x = upload(syn.activations(wl, "x_hidden", shape.T, shape.H))
     out_ref = torch.empty(shape.T, shape.H, dtype=torch.float32, device=dev)
     blk.teacher(x, out_ref)
@@ -640,7 +643,7 @@ def measure_block_window(C, torch, wl, dev, peaks, world, s, barrier, steps=5, w
            "flops_per_step": {"linears": shape.linear_flops(), "attention": shape.attention_flops()},
            "attention_fwd_bwd_ms": attn_ms,
            "attention_tflops": shape.attention_flops() / (attn_ms * 1e-3) / 1e12,
-           "loss_after_steps": first_loss, "phase": "soft", "s": s, "qk_norm": qk_norm,
+           "loss_after_steps": first_loss, "phase": "soft", "s": s, "qk_norm": qk_norm, "streams": 1 + len(blk.sides),
            "shape": dataclasses.asdict(shape), "l2": "working set > L2 (no flush)"}
     del blk, W, x, out_ref, grads, upd
     torch.cuda.empty_cache()
@@ -1004,7 +1007,8 @@ def run_only(args):
         r = measure_decode(C, torch, wl, dev, peaks, rows=rows, steps=args.steps, staged="staged" in args.only)
     else:
         bw = syn.WORKLOADS[args.workload] if args.workload in BLOCK_WINDOW_SHAPES else wl
-        r = measure_block_window(C, torch, bw, dev, peaks, 1, args.s, barrier, steps=args.steps, warmup=args.warmup)
+        r = measure_block_window(C, torch, bw, dev, peaks, 1, args.s, barrier, steps=args.steps, warmup=args.warmup,
+                                 streams=args.streams)
     print(json.dumps({"only": args.only, **r}), flush=True)
 
 

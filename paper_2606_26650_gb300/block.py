@@ -10,7 +10,15 @@ fp32 and the loss is taken on the fp32 block output, so that the difference betw
 and teacher is not lost to the rounding of a value the size of the residual.  The block input
 x (bf16 or fp32) is the window's input and receives no gradient.  Every step here is a call
 into libcatq (the linears, RMSNorm, rotary embedding, attention, SwiGLU, the block output and
-its loss); this module only holds the buffers and orders the calls on one stream.
+its loss); this module only holds the buffers and orders the calls.
+
+Calls that do not depend on each other run on side streams, joined by events: the q, k and v
+projections (with their head norms and rotary embeddings) and the gate and up projections and
+their dX contractions on a companion stream beside the main one, and every linear's
+factor-gradient contraction (dW), which the backward's chain (dX, the layers between the
+linears, attention) never waits for, in turn on the other side streams, each with its own dW
+workspace.  A call of `forward` or `step` starts after the work already issued on the main
+stream and ends with every side stream joined back into it.
 """
 from __future__ import annotations
 
@@ -61,9 +69,10 @@ class Block:
     to the projections' outputs before the rotary embedding)."""
 
     def __init__(self, shape: BlockShape, W, gamma1, gamma2, g, factors=None, thr_init=C.THR_HALF, stream=None,
-                 q_norm=None, k_norm=None):
+                 q_norm=None, k_norm=None, side_streams=3):
         import torch
         self.shape, self.g, self.stream = shape, g, stream
+        self.torch = torch
         dev = W["q_proj"].device
         self.device = dev
         for name, (n, k) in shape.linear_shapes().items():
@@ -101,33 +110,78 @@ class Block:
             self.qp, self.kp = e(T, qd, **bf), e(T, kvd, **bf)
             self.rq, self.rk = e(T * shape.n_heads, **f32), e(T * shape.n_kv_heads, **f32)
         ws = max(C.catq_bwd_workspace_bytes(L, T) for L in self.layers.values())
-        self.bwd_ws = C.workspace(ws, dev)
+        # side streams (independent calls) and one dW workspace per side stream
+        self.sides = [torch.cuda.Stream(device=dev) for _ in range(max(0, int(side_streams)))]
+        self.bwd_ws = [C.workspace(ws, dev) for _ in range(1 + len(self.sides))]
         self.loss_ws = C.workspace(C.catq_recon_loss_workspace_bytes(T * H), dev)
+        self._next_side = 0
+
+    # ---------------------------------------------------------------- streams
+    def _main(self):
+        return self.stream if self.stream is not None else self.torch.cuda.current_stream(self.device)
+
+    def _after(self, src, dst):
+        """dst waits for the work issued so far on src."""
+        if dst is not src:
+            ev = self.torch.cuda.Event()
+            ev.record(src)
+            dst.wait_event(ev)
+
+    def _side(self, i):
+        """Side stream i (the main stream when the block has none)."""
+        return self.sides[i % len(self.sides)] if self.sides else self._main()
+
+    def _dw_lane(self, i):
+        """The i-th dW stream and its workspace: the side streams after the companion (side 0),
+        or side 0 itself when it is the only one, or the main stream."""
+        lanes = list(range(1, len(self.sides))) or list(range(len(self.sides)))
+        if not lanes:
+            return self._main(), self.bwd_ws[0]
+        j = lanes[i % len(lanes)]
+        return self.sides[j], self.bwd_ws[1 + j]
+
+    def _join(self):
+        main = self._main()
+        for sd in self.sides:
+            self._after(sd, main)
 
     # ---------------------------------------------------------------- forward
     def forward(self, x, sched, out=None, out_ref=None, loss=None, reduction=C.REDUCE_MEAN):
         """The block at schedule point sched (PHASE_TEACHER: full-precision weights), filling
         the forward cache the backward reads.  out: fp32 [T, H] block output (nullable);
         with out_ref, Eq. 7's loss into loss[0] and its gradient into the backward's d_out."""
-        sh, st, L = self.shape, self.stream, self.layers
+        self._forward(x, sched, out, out_ref, loss, reduction)
+        self._join()
+
+    def _forward(self, x, sched, out, out_ref, loss, reduction):
+        sh, L = self.shape, self.layers
+        st = self._main()
+        sq, sk, sv = st, self._side(0), self._side(1)
         C.catq_rmsnorm_fwd(x, self.gamma1, self.z1, self.r1, sh.eps, stream=st)
-        if self.q_norm is None:
-            C.catq_soft_ternary_linear_fwd(L["q_proj"], sched, self.z1, self.q, stream=st)
-            C.catq_soft_ternary_linear_fwd(L["k_proj"], sched, self.z1, self.k, stream=st)
-        else:
-            C.catq_soft_ternary_linear_fwd(L["q_proj"], sched, self.z1, self.qp, stream=st)
-            C.catq_soft_ternary_linear_fwd(L["k_proj"], sched, self.z1, self.kp, stream=st)
-            C.catq_rmsnorm_fwd(self.qp.view(-1, sh.d), self.q_norm, self.q.view(-1, sh.d), self.rq, sh.eps, stream=st)
-            C.catq_rmsnorm_fwd(self.kp.view(-1, sh.d), self.k_norm, self.k.view(-1, sh.d), self.rk, sh.eps, stream=st)
-        C.catq_soft_ternary_linear_fwd(L["v_proj"], sched, self.z1, self.v, stream=st)
-        C.catq_rope(self.q, sh.S, sh.n_heads, sh.d, sh.base, stream=st)
-        C.catq_rope(self.k, sh.S, sh.n_kv_heads, sh.d, sh.base, stream=st)
+        self._after(st, sk)
+        self._after(st, sv)
+        # q, k, v: each projection, head norm and rotary embedding on its own stream
+        for name, y, yp, norm, r, nh, s_ in (("q_proj", self.q, "qp", self.q_norm, "rq", sh.n_heads, sq),
+                                              ("k_proj", self.k, "kp", self.k_norm, "rk", sh.n_kv_heads, sk)):
+            if norm is None:
+                C.catq_soft_ternary_linear_fwd(L[name], sched, self.z1, y, stream=s_)
+            else:
+                pre = getattr(self, yp)
+                C.catq_soft_ternary_linear_fwd(L[name], sched, self.z1, pre, stream=s_)
+                C.catq_rmsnorm_fwd(pre.view(-1, sh.d), norm, y.view(-1, sh.d), getattr(self, r), sh.eps, stream=s_)
+            C.catq_rope(y, sh.S, nh, sh.d, sh.base, stream=s_)
+        C.catq_soft_ternary_linear_fwd(L["v_proj"], sched, self.z1, self.v, stream=sv)
+        self._after(sk, st)
+        self._after(sv, st)
         C.catq_attention_fwd(self.q, self.k, self.v, self.a, self.lse, sh.B, sh.S, sh.n_heads, sh.n_kv_heads, sh.d,
                              stream=st)
         C.catq_soft_ternary_linear_fwd(L["o_proj"], sched, self.a, self.ao, stream=st)
         C.catq_rmsnorm_fwd(x, self.gamma2, self.z2, self.r2, sh.eps, residual=self.ao, h_out=self.h, stream=st)
+        su = self._side(0)
+        self._after(st, su)
         C.catq_soft_ternary_linear_fwd(L["gate_proj"], sched, self.z2, self.gt, stream=st)
-        C.catq_soft_ternary_linear_fwd(L["up_proj"], sched, self.z2, self.u, stream=st)
+        C.catq_soft_ternary_linear_fwd(L["up_proj"], sched, self.z2, self.u, stream=su)
+        self._after(su, st)
         C.catq_swiglu_fwd(self.gt, self.u, self.m, stream=st)
         C.catq_soft_ternary_linear_fwd(L["down_proj"], sched, self.m, self.dn, stream=st)
         C.catq_block_output_loss(self.h, self.dn, out_ref, loss, self.d_out if out_ref is not None else None, out,
@@ -142,30 +196,46 @@ class Block:
         """Forward at sched, loss[0] = Eq. 7's loss of the block output against out_ref (fp32),
         and grads[name] = (g_dmu, g_dalpha, g_ddelta) ([G] fp32 each, overwritten) of every
         linear.  out: fp32 [T, H] for the student output (not stored when None)."""
-        sh, st, L = self.shape, self.stream, self.layers
-        self.forward(x, sched, out=out, out_ref=out_ref, loss=loss, reduction=reduction)
-        self._bwd("down_proj", sched, self.m, self.d_out, self.dm, grads)
+        sh, L = self.shape, self.layers
+        st = self._main()
+        self._next_side = 0
+        self._forward(x, sched, out, out_ref, loss, reduction)
+        self._dw("down_proj", sched, self.m, self.d_out, grads)
+        self._dx("down_proj", sched, self.m, self.d_out, self.dm, st)
         C.catq_swiglu_bwd(self.gt, self.u, self.dm, self.dgt, self.du, stream=st)
-        self._bwd("gate_proj", sched, self.z2, self.dgt, self.dz2a, grads)
-        self._bwd("up_proj", sched, self.z2, self.du, self.dz2b, grads)
+        self._dw("gate_proj", sched, self.z2, self.dgt, grads)
+        self._dw("up_proj", sched, self.z2, self.du, grads)
+        su = self._side(0)
+        self._after(st, su)
+        self._dx("gate_proj", sched, self.z2, self.dgt, self.dz2a, st)
+        self._dx("up_proj", sched, self.z2, self.du, self.dz2b, su)
+        self._after(su, st)
         C.catq_rmsnorm_bwd(self.h, self.gamma2, self.r2, self.dz2a, self.dh, dZ2=self.dz2b, d_residual=self.d_out,
                            stream=st)
-        self._bwd("o_proj", sched, self.a, self.dh, self.da, grads)
+        self._dw("o_proj", sched, self.a, self.dh, grads)
+        self._dx("o_proj", sched, self.a, self.dh, self.da, st)
         C.catq_attention_bwd(self.q, self.k, self.v, self.a, self.da, self.lse, self.delta, self.dq, self.dk, self.dv,
                              sh.B, sh.S, sh.n_heads, sh.n_kv_heads, sh.d, stream=st)
-        C.catq_rope(self.dq, sh.S, sh.n_heads, sh.d, sh.base, inverse=True, stream=st)
-        C.catq_rope(self.dk, sh.S, sh.n_kv_heads, sh.d, sh.base, inverse=True, stream=st)
-        if self.q_norm is not None:  # through the head norm, in place
-            C.catq_rmsnorm_bwd(self.qp.view(-1, sh.d), self.q_norm, self.rq, self.dq.view(-1, sh.d),
-                               self.dq.view(-1, sh.d), stream=st)
-            C.catq_rmsnorm_bwd(self.kp.view(-1, sh.d), self.k_norm, self.rk, self.dk.view(-1, sh.d),
-                               self.dk.view(-1, sh.d), stream=st)
-        self._bwd("q_proj", sched, self.z1, self.dq, None, grads)
-        self._bwd("k_proj", sched, self.z1, self.dk, None, grads)
-        self._bwd("v_proj", sched, self.z1, self.dv, None, grads)
+        self._dw("v_proj", sched, self.z1, self.dv, grads)
+        for name, dy, pre, norm, r, nh in (("k_proj", self.dk, "kp", self.k_norm, "rk", sh.n_kv_heads),
+                                           ("q_proj", self.dq, "qp", self.q_norm, "rq", sh.n_heads)):
+            C.catq_rope(dy, sh.S, nh, sh.d, sh.base, inverse=True, stream=st)
+            if norm is not None:  # through the head norm, in place
+                C.catq_rmsnorm_bwd(getattr(self, pre).view(-1, sh.d), norm, getattr(self, r), dy.view(-1, sh.d),
+                                   dy.view(-1, sh.d), stream=st)
+            self._dw(name, sched, self.z1, dy, grads)
+        self._join()
         return out
 
-    def _bwd(self, name, sched, X, dY, dX, grads):
+    def _dx(self, name, sched, X, dY, dX, stream):
+        C.catq_soft_ternary_linear_bwd(self.layers[name], sched, X, dY, dX, stream=stream)
+
+    def _dw(self, name, sched, X, dY, grads):
+        """Linear `name`'s factor gradients on the next dW stream (in turn), after the work
+        issued so far on the main stream, with that stream's workspace."""
         g = grads[name]
-        C.catq_soft_ternary_linear_bwd(self.layers[name], sched, X, dY, dX, g[0], g[1], g[2], workspace=self.bwd_ws,
-                                       stream=self.stream)
+        sd, ws = self._dw_lane(self._next_side)
+        self._next_side += 1
+        self._after(self._main(), sd)
+        C.catq_soft_ternary_linear_bwd(self.layers[name], sched, X, dY, None, g[0], g[1], g[2], workspace=ws,
+                                       stream=sd)
