@@ -328,8 +328,9 @@ constexpr float kOneExpD = 9.0f;
 //   p = 1 + tanh y = 2 / (1 + exp(-2y)),   sech^2 y = (1 - tanh y)(1 + tanh y) = p^2 exp(-2y),
 //   SOFT T = sign(x) p / (2 tanh s),
 // one exp2, one reciprocal and a handful of multiply-adds per element (the phase is a template
-// argument, decided once per chunk).  The exponent is capped at 126, reached only far inside
-// the threshold where sech^2 y is below fp32 resolution anyway, so exp(-2y) stays finite.
+// argument, decided once per chunk).  Where a group's exponent can pass 126 it is capped there,
+// which happens only far inside the threshold where sech^2 y is below fp32 resolution anyway,
+// so exp(-2y) stays finite.
 struct OneExp {
   float c1, c2;
 };
@@ -351,34 +352,73 @@ __device__ __forceinline__ float rcp_approx(float a) {
   return r;
 }
 
-template <bool MU, bool SOFT>
-__device__ __forceinline__ void grad_element_logistic(float G, float w, const GroupConst& c, const OneExp& oe,
-                                                      float inv_2tanh_s, float k, GradSums& acc, float inv_k) {
+// Running sums of the logistic form, with the per-element work cut to what varies per weight:
+//   smu   = sum G s2   (MU: sum G (s2 - 1/k)),
+//   st    = sum G sign(x) p   (SOFT; HARD: sum G Q(x)),
+//   sxs   = sum G x s2,
+//   sdelta = -sum G sign(x) s2,
+// from which salpha = (1/(2 tanh s)) st - k sxs (SOFT; HARD: st - k sxs) once per partial.
+struct LogiSums {
+  float smu, st, sxs, sdelta;
+};
+
+__device__ __forceinline__ GradSums grad_sums(const LogiSums& l, bool soft, float inv_2tanh_s, float k) {
+  return GradSums{l.smu, fmaf(-k, l.sxs, soft ? inv_2tanh_s * l.st : l.st), l.sdelta};
+}
+
+// grad_element's two-exponential form into the same sums (T without its 1/(2 tanh s) factor
+// in the SOFT phase), for groups whose threshold in sharpness units is below kOneExpD.
+template <bool MU>
+__device__ __forceinline__ void grad_element_sums(float G, float w, const GroupConst& c, float s, int32_t phase,
+                                                  LogiSums& acc, float inv_k) {
   const float x = what(w, c);
-  const float e = ex2_approx(fminf(fmaf(fabsf(x), oe.c1, oe.c2), 126.0f));
+  float ta, sa, tb, sb;
+  tanh_sech2<true>(s * (x - c.delta), ta, sa);
+  tanh_sech2<true>(s * (x + c.delta), tb, sb);
+  const float a = G * (sa + sb);
+  acc.smu += MU ? fmaf(-G, inv_k, a) : a;
+  acc.sxs = fmaf(x, a, acc.sxs);
+  acc.st = fmaf(G, phase == PHASE_SOFT ? ta + tb : hard_q(x, c.delta), acc.st);
+  acc.sdelta = fmaf(G, sb - sa, acc.sdelta);
+}
+
+// a times the sign of -x: a's sign bit flipped unless x's is set (one logic operation; x = +0
+// counts as positive, as copysign(1, -x) does).
+__device__ __forceinline__ float times_sign_of_neg(float a, float x) {
+  return __int_as_float(__float_as_int(a) ^ (~__float_as_int(x) & 0x80000000));
+}
+
+// CLAMP caps the exponent at 126; a group needs it only when its largest exponent, c2 (at
+// x = 0), is above that.
+template <bool MU, bool SOFT, bool CLAMP>
+__device__ __forceinline__ void grad_element_logistic(float G, float w, const GroupConst& c, const OneExp& oe,
+                                                      LogiSums& acc, float inv_k) {
+  const float x = what(w, c);
+  float y = fmaf(fabsf(x), oe.c1, oe.c2);
+  if constexpr (CLAMP) y = fminf(y, 126.0f);
+  const float e = ex2_approx(y);
   const float p = rcp_approx(fmaf(e, 0.5f, 0.5f));
-  const float s2 = p * p * e;
-  const float T = SOFT ? copysignf(p * inv_2tanh_s, x) : hard_q(x, c.delta);
-  acc.smu = fmaf(G, MU ? s2 - inv_k : s2, acc.smu);
-  acc.salpha = fmaf(G, fmaf(-x * k, s2, T), acc.salpha);
-  acc.sdelta = fmaf(G, copysignf(s2, -x), acc.sdelta);
+  const float a = G * (p * p * e);
+  acc.smu += MU ? fmaf(-G, inv_k, a) : a;
+  acc.sxs = fmaf(x, a, acc.sxs);
+  acc.st = fmaf(G, SOFT ? copysignf(p, x) : hard_q(x, c.delta), acc.st);
+  acc.sdelta += times_sign_of_neg(a, x);
 }
 
 // 32 consecutive elements of one row: fp32 accumulator values g[0..31] and the bf16 weights
 // packed two per word in w[0..3].
-template <bool MU, bool SOFT>
+template <bool MU, bool SOFT, bool CLAMP>
 __device__ __forceinline__ void grad_chunk_logistic(const uint32_t (&g)[32], const uint4 (&w)[4], const GroupConst& c,
-                                                    const OneExp& oe, float inv_2tanh_s, float k, GradSums& acc,
-                                                    float inv_k) {
+                                                    const OneExp& oe, LogiSums& acc, float inv_k) {
 #pragma unroll
   for (int v = 0; v < 4; ++v) {
     const uint32_t w4[4] = {w[v].x, w[v].y, w[v].z, w[v].w};
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
-      grad_element_logistic<MU, SOFT>(__uint_as_float(g[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), c, oe, inv_2tanh_s,
-                                      k, acc, inv_k);
-      grad_element_logistic<MU, SOFT>(__uint_as_float(g[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), c, oe,
-                                      inv_2tanh_s, k, acc, inv_k);
+      grad_element_logistic<MU, SOFT, CLAMP>(__uint_as_float(g[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), c, oe, acc,
+                                             inv_k);
+      grad_element_logistic<MU, SOFT, CLAMP>(__uint_as_float(g[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), c, oe,
+                                             acc, inv_k);
     }
   }
 }

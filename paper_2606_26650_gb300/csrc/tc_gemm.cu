@@ -1097,7 +1097,8 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
       const int64_t n = (int64_t)n_blk * Cfg::kTileRows + cta * 128 + q * 32 + lane;
       const bool row_ok = n < L.N;
       float* out = args.part + slab * 3 * plane;
-      GradSums acc{0.f, 0.f, 0.f};
+      LogiSums lacc{0.f, 0.f, 0.f, 0.f};
+      const bool soft = args.sc.phase == PHASE_SOFT;
       constexpr int kChunks = (BN / 2) / 32;
       const int64_t k0 = (int64_t)k_blk * BN + half * (BN / 2);
       auto load_w = [&](int c, uint4 (&dst)[4]) {  // W is read once per launch: streamed through L2
@@ -1141,29 +1142,33 @@ __global__ void __launch_bounds__(DwCfg<CG>::kThreads, 1)
           if (gc.alpha != 0.0f && D >= kOneExpD) {
             // one exponential per weight (the far tanh term is 1 to fp32 resolution)
             const OneExp oe = one_exp_consts(args.sc.s, D);
-            if (args.sc.phase == PHASE_SOFT)
-              grad_chunk_logistic<MU, true>(rg, wcur, gc, oe, args.sc.inv_2tanh_s, k_sc, acc, inv_k);
-            else
-              grad_chunk_logistic<MU, false>(rg, wcur, gc, oe, args.sc.inv_2tanh_s, k_sc, acc, inv_k);
+            if (oe.c2 <= 126.0f) {
+              if (soft) grad_chunk_logistic<MU, true, false>(rg, wcur, gc, oe, lacc, inv_k);
+              else grad_chunk_logistic<MU, false, false>(rg, wcur, gc, oe, lacc, inv_k);
+            } else {
+              if (soft) grad_chunk_logistic<MU, true, true>(rg, wcur, gc, oe, lacc, inv_k);
+              else grad_chunk_logistic<MU, false, true>(rg, wcur, gc, oe, lacc, inv_k);
+            }
           } else if (gc.alpha != 0.0f) {
 #pragma unroll
             for (int v = 0; v < 4; ++v) {
               const uint32_t w4[4] = {wcur[v].x, wcur[v].y, wcur[v].z, wcur[v].w};
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
-                grad_element<true, MU>(__uint_as_float(rg[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), gc, args.sc.s,
-                                       args.sc.inv_2tanh_s, args.sc.phase, acc, inv_k);
-                grad_element<true, MU>(__uint_as_float(rg[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), gc, args.sc.s,
-                                       args.sc.inv_2tanh_s, args.sc.phase, acc, inv_k);
+                grad_element_sums<MU>(__uint_as_float(rg[8 * v + 2 * e]), bf16lo_to_f32(w4[e]), gc, args.sc.s,
+                                      args.sc.phase, lacc, inv_k);
+                grad_element_sums<MU>(__uint_as_float(rg[8 * v + 2 * e + 1]), bf16hi_to_f32(w4[e]), gc, args.sc.s,
+                                      args.sc.phase, lacc, inv_k);
               }
             }
           }
           if (((k + 32) % args.P) == 0 || k + 32 >= L.K) {
+            const GradSums acc = grad_sums(lacc, soft, args.sc.inv_2tanh_s, k_sc);
             const int64_t idx = n * cpr + k / args.P;
             out[idx] = acc.smu;
             out[plane + idx] = acc.salpha;
             out[2 * plane + idx] = acc.sdelta;
-            acc = GradSums{0.f, 0.f, 0.f};
+            lacc = LogiSums{0.f, 0.f, 0.f, 0.f};
           }
         }
 #pragma unroll
