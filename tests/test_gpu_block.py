@@ -234,7 +234,7 @@ def _block_case(shape, g, seed, x_dtype="bf16"):
     return W, x, g1, g2, fac
 
 
-def _gpu_block(shape, W, x, g1, g2, fac, g, phase, s, device, x_dtype="bf16", qk=None):
+def _gpu_block(shape, W, x, g1, g2, fac, g, phase, s, device, x_dtype="bf16", qk=None, side_streams=3):
     import torch
 
     from paper_2606_26650_gb300 import block as BK
@@ -243,7 +243,7 @@ def _gpu_block(shape, W, x, g1, g2, fac, g, phase, s, device, x_dtype="bf16", qk
     facd = {n: tuple(torch.from_numpy(f.copy()).to(device) for f in fac[n]) for n in W}
     norms = {k: torch.from_numpy(v).to(device) for k, v in qk.items()} if qk else {}
     blk = BK.Block(shape, Wd, torch.from_numpy(g1).to(device), torch.from_numpy(g2).to(device), g, factors=facd,
-                   **norms)
+                   side_streams=side_streams, **norms)
     xd = U.to_device(x, x_dtype, device)
     out_ref = torch.empty(shape.T, shape.H, dtype=torch.float32, device=device)
     blk.teacher(xd, out_ref)
@@ -287,6 +287,29 @@ def test_block_step_matches_oracle(device, phase, s, x_dtype, qk_norm):
     print("block step errors:", {k: f"{v:.2e}" for k, v in errs.items()})
     bad = {k: v for k, v in errs.items() if not v <= U.TOL_BF16}
     assert not bad, f"tolerance {U.TOL_BF16} exceeded: {bad}"
+
+
+@pytest.mark.parametrize("qk_norm", [False, True])
+def test_block_step_same_on_any_number_of_streams(device, qk_norm):
+    """Every kernel of the step is deterministic, and the side streams only change which calls
+    overlap: the step on the main stream alone, on one side stream and on three gives the same
+    bits (the events order every read after its write)."""
+    from paper_2606_26650_gb300 import block as BK
+    shape = BK.BlockShape(**dict(SMALL, base=1e6 if qk_norm else SMALL["base"]))
+    W, x, g1, g2, fac = _block_case(shape, 128, 3)
+    qk = None
+    if qk_norm:
+        rq = syn.rng(99, "block/qk")
+        qk = {"q_norm": rq.uniform(0.5, 1.5, shape.d).astype(np.float32),
+              "k_norm": rq.uniform(0.5, 1.5, shape.d).astype(np.float32)}
+    runs = [_gpu_block(shape, W, x, g1, g2, fac, 128, O.PHASE_SOFT, 30.0, device, qk=qk, side_streams=n)
+            for n in (0, 1, 3)]
+    for r in runs[1:]:
+        assert np.array_equal(r["out"], runs[0]["out"])
+        assert r["loss"] == runs[0]["loss"]
+        for n in W:
+            for a, b in zip(r["g"][n], runs[0]["g"][n]):
+                assert np.array_equal(a, b), n
 
 
 def test_block_teacher_phase_has_zero_loss(device):
