@@ -232,11 +232,13 @@ __device__ __forceinline__ void cursor_next(Cursor& c, const InferArgs& a) {
 // R: 16-row tiles per work item.  VW: code words per thread per super-chunk (a super-chunk is
 // 64 VW columns and lies in one group).  MU: add mu times each group's activation sum.
 // A persistent CTA walks its work items (over every layer of the launch) as one stream of
-// code slabs through two shared-memory buffers: warp 0 issues the bulk copies of slab c + 2 as
-// soon as slab c has been consumed, whichever item and layer it belongs to, so the next
-// item's codes are on their way while this one finishes its slabs and its reduction.  Each
-// row's copy lands at a stride padded by 16 VW bytes, so the fragment reads (four lanes per
-// row, eight rows per instruction) are free of bank conflicts.
+// code slabs through two shared-memory buffers: once every warp has passed slab c + 1's
+// barrier (so slab c is consumed), warp 0 issues the bulk copies of slab c + 2 into slab c's
+// buffer, whichever item and layer it belongs to, so the next item's codes are on their way
+// while this one finishes its slabs and its reduction.  Each row's copy lands at a stride
+// padded by 16 VW bytes, so the fragment reads (four lanes per row, eight rows per
+// instruction) are free of bank conflicts.  Two CTA barriers per slab or item: the slab's
+// landing (which also frees the slab before it) and the partial sums' hand-over.
 template <int R, int VW, bool MU, bool STAGED>
 __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const __grid_constant__ InferArgs a,
                                                                      int32_t buf_bytes, const WaitCtl wc) {
@@ -361,6 +363,13 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const __
       ok = false;
       break;
     }
+    // Every warp is past this slab's barrier, so it is done with the slab before: that buffer
+    // takes the slab after this one (the first two went out at the start).
+    if (warp == 0 && issued < qn + 2 && iss.t < a.total_items) {
+      issue(iss, buf ^ 1);
+      cursor_next(iss, a);
+      ++issued;
+    }
     {
       // this warp's contiguous range of the slab's super-chunks, and the group it starts in
       const int32_t sc_per_slab = L.KS / (64 * VW);
@@ -472,12 +481,6 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const __
         step(sc + 1, xc);
       }
     }
-    __syncthreads();  // every warp is done with this buffer: refill it two slabs ahead
-    if (warp == 0 && iss.t < a.total_items) {
-      issue(iss, buf);
-      cursor_next(iss, a);
-      ++issued;
-    }
     ++qn;
     if (con.slab + 1 == L.nslabs) {
       // the token block's last slab: its partial sums meet in shared memory, in a fixed order
@@ -498,7 +501,8 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 2) ternary_mma_kernel(const __
         if (con.b0 + tok < L.B && n0 + row < L.N)
           L.Y[(con.b0 + tok) * L.N + n0 + row] = static_cast<uint16_t>(pack_bf16x2(s, 0.0f) & 0xFFFFu);
       }
-      __syncthreads();
+      // red is written again only after the next slab's barrier, which every thread reaches
+      // after this loop
     }
     cursor_next(con, a);
   }
