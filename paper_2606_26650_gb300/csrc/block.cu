@@ -941,6 +941,9 @@ cudaError_t launch_attention(const AttnIo& io, int32_t B, int32_t S, int32_t nh,
   a.nkv = nkv;
   a.scale = 1.0f / sqrtf(static_cast<float>(d));
   a.scale_log2 = a.scale * 1.4426950408889634f;
+  // the forward of 128-wide heads over whole 128-token tiles runs on tcgen05 (attn_tc.cu)
+  if (!backward && attention_fwd_tc_supported(S, d))
+    return launch_attention_fwd_tc(io.q, io.k, io.v, io.out, io.lse, B, S, nh, nkv, st);
   return d == 128 ? attn_launch<128>(a, backward, st) : attn_launch<64>(a, backward, st);
 }
 

@@ -190,6 +190,10 @@ struct AttnIo {
 };
 cudaError_t launch_attention(const AttnIo& io, int32_t B, int32_t S, int32_t nh, int32_t nkv, int32_t d, bool backward,
                              cudaStream_t st);
+// The forward on the tcgen05 tensor cores (attn_tc.cu): head dimension 128, S a multiple of 128.
+bool attention_fwd_tc_supported(int32_t S, int32_t d);
+cudaError_t launch_attention_fwd_tc(const void* q, const void* k, const void* v, void* out, float* lse, int32_t B,
+                                    int32_t S, int32_t nh, int32_t nkv, cudaStream_t st);
 // Status word latched by device-side bounded waits (0 = none); read-and-clear.
 cudaError_t read_and_clear_device_status(int32_t* out);
 bool tensor_map_encoder_available();

@@ -157,7 +157,9 @@ def test_block_output_loss(device, reduction):
 
 # ---------------------------------------------------------------- attention
 
-ATTN_SHAPES = [(2, 128, 4, 2, 128), (1, 192, 4, 1, 64), (1, 64, 2, 2, 128), (3, 256, 8, 8, 64)]
+# d = 128 with S a multiple of 128 takes the tcgen05 forward; the others the mma.sync one
+ATTN_SHAPES = [(2, 128, 4, 2, 128), (1, 192, 4, 1, 64), (1, 64, 2, 2, 128), (3, 256, 8, 8, 64), (2, 512, 8, 2, 128),
+               (1, 384, 4, 4, 128)]
 
 
 def _attn_inputs(B, S, nh, nkv, d, tag):
