@@ -281,6 +281,367 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   }
 }
 
+// ---------------------------------------------------------------- backward
+// With P = exp(scale S - lse) recomputed from the forward's log-sum-exp, dP = dO V^T and
+// dS = P * (dP - delta) (delta = rowsum(dO * O), from attn_delta_kernel):
+//   dQ = scale dS K,  dK = scale dS^T Q,  dV = P^T dO,
+// in two kernels, so that every accumulator has one owner and no atomics are needed.
+
+struct TcBwdArgs {
+  uint16_t *dq, *dk, *dv;
+  const float* lse;    // natural log-sum-exp per (sequence, head, row)
+  const float* delta;  // rowsum(dO * O) per (sequence, head, row)
+  int32_t S, nh, nkv;
+  float scale_log2;
+  float scale;
+  WaitCtl wc;
+};
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+          taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+      "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
+// Q/K-major SS products of the backward: D (+)= A B^T over d = 128 (A, B: 128 rows x 128
+// columns, two 64-column boxes each).
+__device__ __forceinline__ void mma_kmajor(uint32_t d_tmem, uint32_t a_smem, uint32_t b_smem, uint32_t idesc) {
+#pragma unroll
+  for (int kk = 0; kk < kHd / 16; ++kk) {
+    const uint32_t off = (kk >> 2) * kBox + (kk & 3) * 32;
+    umma_bf16<1>(d_tmem, smem_desc_sw128(a_smem + off, 16, 1024), smem_desc_sw128(b_smem + off, 16, 1024), idesc,
+                 kk > 0 ? 1u : 0u);
+  }
+}
+
+// TS products: D (+)= A[tmem] B[smem] over 128 (A: 128 x 128 bf16 in TMEM, B: the 128-row
+// tile read as K x N with N contiguous).
+__device__ __forceinline__ void mma_ts_tile(uint32_t d_tmem, uint32_t a_tmem, uint32_t b_smem, uint32_t idesc,
+                                            bool accumulate) {
+#pragma unroll
+  for (int kk = 0; kk < 8; ++kk)
+    umma_ts(d_tmem, a_tmem + 8u * kk, smem_desc_sw128(b_smem + kk * 2048, kBox, 1024), idesc,
+            (accumulate || kk > 0) ? 1u : 0u);
+}
+
+// dQ: one CTA per (128-query tile, head, sequence), over the key tiles up to the diagonal.
+// TMEM: S [0, 128), dP [128, 256), dQ [256, 384); dS (bf16) goes over S's first 64 columns.
+constexpr uint32_t kDqOffQ = 0, kDqOffDo = kTile, kDqOffK = 2 * kTile, kDqOffV = 4 * kTile, kDqOffBar = 6 * kTile;
+constexpr uint32_t kDqSmem = kDqOffBar + 128 + 1024;
+
+__global__ void __launch_bounds__(kThreadsTc, 1)
+    attn_tc_dq_kernel(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmdo,
+                      const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
+                      const TcBwdArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (base - raw) + kDqOffBar + 96);
+  const uint32_t bar = base + kDqOffBar;
+  const uint32_t qd_full = bar, kv_full0 = bar + 8, kv_empty0 = bar + 24, s_full = bar + 40, ds_full = bar + 48,
+                 q_done = bar + 56, final_bar = bar + 64;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nqt = a.S / kTq;
+  const int qt = nqt - 1 - static_cast<int>(blockIdx.x);
+  const int h = blockIdx.y, b = blockIdx.z, hk = h / (a.nh / a.nkv);
+  const int ntiles = qt + 1;
+  const int32_t row0 = b * a.S;
+  constexpr uint32_t kColS = 0, kColP = 128, kColQ = 256;
+
+  if (threadIdx.x == 0) {
+    mbar_init(qd_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(kv_full0 + 8u * i, 1);
+      mbar_init(kv_empty0 + 8u * i, 1);
+    }
+    mbar_init(s_full, 1);
+    mbar_init(ds_full, kTq);
+    mbar_init(q_done, 1);
+    mbar_init(final_bar, 1);
+    fence_mbar_init_cluster();
+  }
+  if (warp == kMmaWarp) tmem_alloc<1>(smem_u32(tmem_slot), kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  bool ok = true;
+
+  if (warp == kTmaWarp) {
+    if (lane == 0) {
+      mbar_arrive_expect_tx(qd_full, 2 * kTile);
+      for (int hf = 0; hf < 2; ++hf) {
+        tma_load_2d(base + kDqOffQ + hf * kBox, &tmq, qd_full, h * kHd + 64 * hf, row0 + qt * kTq);
+        tma_load_2d(base + kDqOffDo + hf * kBox, &tmdo, qd_full, h * kHd + 64 * hf, row0 + qt * kTq);
+      }
+      int issued = 0;
+      for (int j = 0; j < ntiles; ++j) {
+        const int st = j & 1;
+        if (j >= 2 && !mbar_wait(kv_empty0 + 8u * st, ((j >> 1) & 1) ^ 1, a.wc)) { ok = false; break; }
+        mbar_arrive_expect_tx(kv_full0 + 8u * st, 2 * kTile);
+        for (int hf = 0; hf < 2; ++hf) {
+          tma_load_2d(base + kDqOffK + st * kTile + hf * kBox, &tmk, kv_full0 + 8u * st, hk * kHd + 64 * hf,
+                      row0 + j * kTk);
+          tma_load_2d(base + kDqOffV + st * kTile + hf * kBox, &tmv, kv_full0 + 8u * st, hk * kHd + 64 * hf,
+                      row0 + j * kTk);
+        }
+        issued = j + 1;
+      }
+      drain(qd_full, 0);
+      for (int j = issued - 2 < 0 ? 0 : issued - 2; j < issued; ++j) drain(kv_full0 + 8u * (j & 1), (j >> 1) & 1);
+    }
+  } else if (warp == kMmaWarp) {
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = idesc_bf16_f32(kTq, kTk, false, false);
+      constexpr uint32_t idesc_q = idesc_bf16_f32(kTq, kHd, false, true);
+      if (!mbar_wait(qd_full, 0, a.wc)) ok = false;
+      for (int j = 0; ok && j < ntiles; ++j) {
+        const uint32_t kt = base + kDqOffK + (j & 1) * kTile, vt = base + kDqOffV + (j & 1) * kTile;
+        if (!mbar_wait(kv_full0 + 8u * (j & 1), (j >> 1) & 1, a.wc)) { ok = false; break; }
+        tc_fence_after();
+        mma_kmajor(tmem + kColS, base + kDqOffQ, kt, idesc_s);   // S = Q K^T
+        mma_kmajor(tmem + kColP, base + kDqOffDo, vt, idesc_s);  // dP = dO V^T
+        umma_commit<1>(s_full);
+        if (!mbar_wait(ds_full, j & 1, a.wc)) { ok = false; break; }
+        tc_fence_after();
+        mma_ts_tile(tmem + kColQ, tmem + kColS, kt, idesc_q, j > 0);  // dQ += dS K
+        umma_commit<1>(kv_empty0 + 8u * (j & 1));
+        umma_commit<1>(q_done);
+      }
+      umma_commit<1>(final_bar);
+      drain(final_bar, 0);
+    }
+  } else {
+    const int r = warp * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+    const int64_t ridx = (static_cast<int64_t>(b) * a.nh + h) * a.S + qt * kTq + r;
+    const float lse2 = a.lse[ridx] * kLog2e, dl = a.delta[ridx];
+    for (int j = 0; ok && j < ntiles; ++j) {
+      if (!mbar_wait(s_full, j & 1, a.wc)) { ok = false; break; }
+      tc_fence_after();
+      const bool diag = j == qt;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t sv[32], pv[32], ds[16];
+        tmem_ld32(tmem + lane_off + kColS + 32u * c, sv);
+        tmem_ld32(tmem + lane_off + kColP + 32u * c, pv);
+        tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+          float p0 = fast_exp2(fmaf(__uint_as_float(sv[i]), a.scale_log2, -lse2));
+          float p1 = fast_exp2(fmaf(__uint_as_float(sv[i + 1]), a.scale_log2, -lse2));
+          if (diag && 32 * c + i > r) p0 = 0.0f;
+          if (diag && 32 * c + i + 1 > r) p1 = 0.0f;
+          ds[i / 2] = pack2(p0 * (__uint_as_float(pv[i]) - dl), p1 * (__uint_as_float(pv[i + 1]) - dl));
+        }
+        tmem_st16(tmem + lane_off + kColS + 16u * c, ds);
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive_local(ds_full);
+    }
+    if (ok && mbar_wait(q_done, (ntiles - 1) & 1, a.wc)) {
+      tc_fence_after();
+      const int64_t tok = static_cast<int64_t>(row0) + qt * kTq + r;
+      uint16_t* drow = a.dq + tok * (static_cast<int64_t>(a.nh) * kHd) + static_cast<int64_t>(h) * kHd;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t o[32];
+        tmem_ld32(tmem + lane_off + kColQ + 32u * c, o);
+        tmem_ld_wait();
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          uint4 w;
+          w.x = pack2(__uint_as_float(o[8 * v + 0]) * a.scale, __uint_as_float(o[8 * v + 1]) * a.scale);
+          w.y = pack2(__uint_as_float(o[8 * v + 2]) * a.scale, __uint_as_float(o[8 * v + 3]) * a.scale);
+          w.z = pack2(__uint_as_float(o[8 * v + 4]) * a.scale, __uint_as_float(o[8 * v + 5]) * a.scale);
+          w.w = pack2(__uint_as_float(o[8 * v + 6]) * a.scale, __uint_as_float(o[8 * v + 7]) * a.scale);
+          *reinterpret_cast<uint4*>(drow + 32 * c + 8 * v) = w;
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc<1>(tmem, kTmemCols);
+  }
+}
+
+// dK, dV: one CTA per (128-key tile, key/value head, sequence), over every query head of the
+// group and the query tiles from the diagonal on, with the scores formed transposed (keys as
+// TMEM lanes), so P^T and dS^T are the A operands of dV and dK straight from TMEM.
+// TMEM: S^T [0, 128), dP^T [128, 256), dV [256, 384), dK [384, 512); P^T and dS^T (bf16)
+// over the first 64 columns of S^T and dP^T.  A stage holds the query tile, its dO tile
+// and their rows' log-sum-exp and delta.
+constexpr uint32_t kKvOffK = 0, kKvOffV = kTile, kKvOffStage = 2 * kTile;
+constexpr uint32_t kStageLse = 2 * kTile, kStageDelta = 2 * kTile + 512, kStageBytes = 2 * kTile + 1024;
+constexpr uint32_t kKvOffBar = kKvOffStage + 2 * kStageBytes;
+constexpr uint32_t kKvSmem = kKvOffBar + 128 + 1024;
+
+__global__ void __launch_bounds__(kThreadsTc, 1)
+    attn_tc_dkdv_kernel(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmdo,
+                        const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
+                        const TcBwdArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + kKvOffBar + 96);
+  const uint32_t bar = base + kKvOffBar;
+  const uint32_t kv_full = bar, st_full0 = bar + 8, st_empty0 = bar + 24, s_full = bar + 40, pd_full = bar + 48,
+                 kv_done = bar + 56, final_bar = bar + 64;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nqt = a.S / kTq;
+  const int kt = static_cast<int>(blockIdx.x);  // key tile; the first ones have the most query tiles
+  const int hk = blockIdx.y, b = blockIdx.z;
+  const int rep = a.nh / a.nkv;
+  const int per_head = nqt - kt;  // query tiles kt..nqt-1
+  const int nsteps = rep * per_head;
+  const int32_t row0 = b * a.S;
+  constexpr uint32_t kColS = 0, kColP = 128, kColV = 256, kColK = 384;
+
+  if (threadIdx.x == 0) {
+    mbar_init(kv_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(st_full0 + 8u * i, 1);
+      mbar_init(st_empty0 + 8u * i, 1);
+    }
+    mbar_init(s_full, 1);
+    mbar_init(pd_full, kTq);
+    mbar_init(kv_done, 1);
+    mbar_init(final_bar, 1);
+    fence_mbar_init_cluster();
+  }
+  if (warp == kMmaWarp) tmem_alloc<1>(smem_u32(tmem_slot), kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  bool ok = true;
+  auto step_head = [&](int t) { return hk * rep + t / per_head; };
+  auto step_tile = [&](int t) { return kt + t % per_head; };
+
+  if (warp == kTmaWarp) {
+    if (lane == 0) {
+      mbar_arrive_expect_tx(kv_full, 2 * kTile);
+      for (int hf = 0; hf < 2; ++hf) {
+        tma_load_2d(base + kKvOffK + hf * kBox, &tmk, kv_full, hk * kHd + 64 * hf, row0 + kt * kTk);
+        tma_load_2d(base + kKvOffV + hf * kBox, &tmv, kv_full, hk * kHd + 64 * hf, row0 + kt * kTk);
+      }
+      int issued = 0;
+      for (int t = 0; t < nsteps; ++t) {
+        const int st = t & 1, h = step_head(t), i = step_tile(t);
+        if (t >= 2 && !mbar_wait(st_empty0 + 8u * st, ((t >> 1) & 1) ^ 1, a.wc)) { ok = false; break; }
+        const uint32_t sb = base + kKvOffStage + st * kStageBytes;
+        mbar_arrive_expect_tx(st_full0 + 8u * st, kStageBytes);
+        for (int hf = 0; hf < 2; ++hf) {
+          tma_load_2d(sb + hf * kBox, &tmq, st_full0 + 8u * st, h * kHd + 64 * hf, row0 + i * kTq);
+          tma_load_2d(sb + kTile + hf * kBox, &tmdo, st_full0 + 8u * st, h * kHd + 64 * hf, row0 + i * kTq);
+        }
+        const int64_t ridx = (static_cast<int64_t>(b) * a.nh + h) * a.S + i * kTq;
+        bulk_load_g2s(sb + kStageLse, a.lse + ridx, kTq * 4, st_full0 + 8u * st);
+        bulk_load_g2s(sb + kStageDelta, a.delta + ridx, kTq * 4, st_full0 + 8u * st);
+        issued = t + 1;
+      }
+      drain(kv_full, 0);
+      for (int t = issued - 2 < 0 ? 0 : issued - 2; t < issued; ++t) drain(st_full0 + 8u * (t & 1), (t >> 1) & 1);
+    }
+  } else if (warp == kMmaWarp) {
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = idesc_bf16_f32(kTk, kTq, false, false);
+      constexpr uint32_t idesc_g = idesc_bf16_f32(kTk, kHd, false, true);
+      if (!mbar_wait(kv_full, 0, a.wc)) ok = false;
+      for (int t = 0; ok && t < nsteps; ++t) {
+        const uint32_t sb = base + kKvOffStage + (t & 1) * kStageBytes;
+        if (!mbar_wait(st_full0 + 8u * (t & 1), (t >> 1) & 1, a.wc)) { ok = false; break; }
+        tc_fence_after();
+        mma_kmajor(tmem + kColS, base + kKvOffK, sb, idesc_s);          // S^T = K Q^T
+        mma_kmajor(tmem + kColP, base + kKvOffV, sb + kTile, idesc_s);  // dP^T = V dO^T
+        umma_commit<1>(s_full);
+        if (!mbar_wait(pd_full, t & 1, a.wc)) { ok = false; break; }
+        tc_fence_after();
+        mma_ts_tile(tmem + kColV, tmem + kColS, sb + kTile, idesc_g, t > 0);  // dV += P^T dO
+        mma_ts_tile(tmem + kColK, tmem + kColP, sb, idesc_g, t > 0);          // dK += dS^T Q
+        umma_commit<1>(st_empty0 + 8u * (t & 1));
+        umma_commit<1>(kv_done);
+      }
+      umma_commit<1>(final_bar);
+      drain(final_bar, 0);
+    }
+  } else {
+    const int rk = warp * 32 + lane;  // key row of the tile (TMEM lane)
+    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+    for (int t = 0; ok && t < nsteps; ++t) {
+      if (!mbar_wait(s_full, t & 1, a.wc)) { ok = false; break; }
+      tc_fence_after();
+      const float* lse = reinterpret_cast<const float*>(gbase + kKvOffStage + (t & 1) * kStageBytes + kStageLse);
+      const float* dlt = reinterpret_cast<const float*>(gbase + kKvOffStage + (t & 1) * kStageBytes + kStageDelta);
+      const bool diag = step_tile(t) == kt;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t sv[32], pv[32], pp[16], ds[16];
+        tmem_ld32(tmem + lane_off + kColS + 32u * c, sv);
+        tmem_ld32(tmem + lane_off + kColP + 32u * c, pv);
+        tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+          const int q = 32 * c + i;
+          float p0 = fast_exp2(fmaf(__uint_as_float(sv[i]), a.scale_log2, -lse[q] * kLog2e));
+          float p1 = fast_exp2(fmaf(__uint_as_float(sv[i + 1]), a.scale_log2, -lse[q + 1] * kLog2e));
+          if (diag && q < rk) p0 = 0.0f;
+          if (diag && q + 1 < rk) p1 = 0.0f;
+          pp[i / 2] = pack2(p0, p1);
+          ds[i / 2] = pack2(p0 * (__uint_as_float(pv[i]) - dlt[q]), p1 * (__uint_as_float(pv[i + 1]) - dlt[q + 1]));
+        }
+        tmem_st16(tmem + lane_off + kColS + 16u * c, pp);
+        tmem_st16(tmem + lane_off + kColP + 16u * c, ds);
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive_local(pd_full);
+    }
+    if (ok && mbar_wait(kv_done, (nsteps - 1) & 1, a.wc)) {
+      tc_fence_after();
+      const int64_t tok = static_cast<int64_t>(row0) + kt * kTk + rk;
+      const int64_t off = tok * (static_cast<int64_t>(a.nkv) * kHd) + static_cast<int64_t>(hk) * kHd;
+#pragma unroll
+      for (int g2 = 0; g2 < 2; ++g2) {
+        uint16_t* drow = (g2 == 0 ? a.dk : a.dv) + off;
+        const uint32_t col = g2 == 0 ? kColK : kColV;
+        const float f = g2 == 0 ? a.scale : 1.0f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          uint32_t o[32];
+          tmem_ld32(tmem + lane_off + col + 32u * c, o);
+          tmem_ld_wait();
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            uint4 w;
+            w.x = pack2(__uint_as_float(o[8 * v + 0]) * f, __uint_as_float(o[8 * v + 1]) * f);
+            w.y = pack2(__uint_as_float(o[8 * v + 2]) * f, __uint_as_float(o[8 * v + 3]) * f);
+            w.z = pack2(__uint_as_float(o[8 * v + 4]) * f, __uint_as_float(o[8 * v + 5]) * f);
+            w.w = pack2(__uint_as_float(o[8 * v + 6]) * f, __uint_as_float(o[8 * v + 7]) * f);
+            *reinterpret_cast<uint4*>(drow + 32 * c + 8 * v) = w;
+          }
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc<1>(tmem, kTmemCols);
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
 std::once_flag g_enc_once;
 
@@ -330,6 +691,41 @@ cudaError_t launch_attention_fwd_tc(const void* q, const void* k, const void* v,
   cudaError_t e = cudaFuncSetAttribute(attn_tc_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
   if (e != cudaSuccess) return e;
   attn_tc_fwd_kernel<<<dim3(S / kTq, nh, B), kThreadsTc, kSmem, st>>>(tq, tk, tv, a);
+  return cudaGetLastError();
+}
+
+
+cudaError_t launch_attention_bwd_tc(const void* q, const void* k, const void* v, const void* dO, const float* lse,
+                                    const float* delta, void* dq, void* dk, void* dv, int32_t B, int32_t S, int32_t nh,
+                                    int32_t nkv, cudaStream_t st) {
+  if (!attention_fwd_tc_supported(S, kHd) || B < 1 || nh < 1 || nkv < 1 || nh % nkv != 0)
+    return cudaErrorInvalidValue;
+  CUtensorMap tq, tdo, tk, tv;
+  const uint64_t rows = static_cast<uint64_t>(B) * S;
+  if (!tmap_rows(&tq, q, static_cast<uint64_t>(nh) * kHd, rows) ||
+      !tmap_rows(&tdo, dO, static_cast<uint64_t>(nh) * kHd, rows) ||
+      !tmap_rows(&tk, k, static_cast<uint64_t>(nkv) * kHd, rows) ||
+      !tmap_rows(&tv, v, static_cast<uint64_t>(nkv) * kHd, rows))
+    return cudaErrorInvalidValue;
+  TcBwdArgs a{};
+  a.dq = static_cast<uint16_t*>(dq);
+  a.dk = static_cast<uint16_t*>(dk);
+  a.dv = static_cast<uint16_t*>(dv);
+  a.lse = lse;
+  a.delta = delta;
+  a.S = S;
+  a.nh = nh;
+  a.nkv = nkv;
+  a.scale = 1.0f / sqrtf(static_cast<float>(kHd));
+  a.scale_log2 = a.scale * kLog2e;
+  if (!launch_wait_ctl(&a.wc)) return cudaErrorInvalidDevice;
+  cudaError_t e = cudaFuncSetAttribute(attn_tc_dq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDqSmem);
+  if (e != cudaSuccess) return e;
+  attn_tc_dq_kernel<<<dim3(S / kTq, nh, B), kThreadsTc, kDqSmem, st>>>(tq, tdo, tk, tv, a);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(attn_tc_dkdv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kKvSmem);
+  if (e != cudaSuccess) return e;
+  attn_tc_dkdv_kernel<<<dim3(S / kTk, nkv, B), kThreadsTc, kKvSmem, st>>>(tq, tdo, tk, tv, a);
   return cudaGetLastError();
 }
 

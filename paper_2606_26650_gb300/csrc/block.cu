@@ -821,6 +821,9 @@ cudaError_t attn_launch(const AttnArgs& a, bool backward, cudaStream_t st) {
   attn_delta_kernel<HD><<<elem_grid(rows * 32), kRowThreads, 0, st>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  // 128-wide heads over whole 128-token tiles: dQ and dK/dV on tcgen05 (attn_tc.cu)
+  if (attention_fwd_tc_supported(a.S, HD))
+    return launch_attention_bwd_tc(a.q, a.k, a.v, a.dO, a.lse, a.delta, a.dq, a.dk, a.dv, a.B, a.S, a.nh, a.nkv, st);
   const int smem_q = 6 * Tile<HD>::kBytes;
   e = cudaFuncSetAttribute(attn_bwd_dq_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_q);
   if (e != cudaSuccess) return e;

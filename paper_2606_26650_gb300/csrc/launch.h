@@ -194,6 +194,10 @@ cudaError_t launch_attention(const AttnIo& io, int32_t B, int32_t S, int32_t nh,
 bool attention_fwd_tc_supported(int32_t S, int32_t d);
 cudaError_t launch_attention_fwd_tc(const void* q, const void* k, const void* v, void* out, float* lse, int32_t B,
                                     int32_t S, int32_t nh, int32_t nkv, cudaStream_t st);
+// dQ, dK, dV on tcgen05 from the forward's log-sum-exp and delta = rowsum(dO * O).
+cudaError_t launch_attention_bwd_tc(const void* q, const void* k, const void* v, const void* dO, const float* lse,
+                                    const float* delta, void* dq, void* dk, void* dv, int32_t B, int32_t S, int32_t nh,
+                                    int32_t nkv, cudaStream_t st);
 // Status word latched by device-side bounded waits (0 = none); read-and-clear.
 cudaError_t read_and_clear_device_status(int32_t* out);
 bool tensor_map_encoder_available();
