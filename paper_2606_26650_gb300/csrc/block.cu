@@ -5,8 +5,9 @@
 // rotary position embedding, SwiGLU, the fp32 block output with the loss on it, and causal
 // grouped-query attention (forward, and a deterministic backward in two kernels).
 //
-// Attention runs on the tensor pipe with mma.sync m16n8k16 (bf16 in, fp32 accumulate):
-// blocks of 64 queries (four warps of 16) against blocks of 64 keys, which stream through two
+// Attention with 128-wide heads over whole 128-token tiles runs on tcgen05 (attn_tc.cu); the
+// kernels here serve the other shapes (d = 64, or S a multiple of 64 only) on the tensor pipe
+// with mma.sync m16n8k16 (bf16 in, fp32 accumulate): blocks of 64 queries (four warps of 16) against blocks of 64 keys, which stream through two
 // shared-memory buffers by cp.async; an online softmax in fp32 with the probabilities fed back
 // as the A operand of P V straight from the score accumulators, and operand fragments read
 // from shared memory with ldmatrix (transposed where the contraction runs along rows).  The
