@@ -202,17 +202,26 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
 #pragma unroll
       for (int c = 0; c < 4; ++c) tmem_ld32(sbuf + 32u * c, sr[c]);
       tmem_ld_wait();
-      float mx = -INFINITY;
-      const bool diag = j == qt;
+      if (j == qt) {  // the diagonal tile: keys after the row's query do not count
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (32 * c + i > r) sr[c][i] = __float_as_uint(-INFINITY);
+      }
+      // the row maximum of the raw scores (scale > 0), in eight independent chains
+      float mv[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) mv[i] = -INFINITY;
 #pragma unroll
       for (int c = 0; c < 4; ++c)
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          float x = __uint_as_float(sr[c][i]) * a.scale_log2;
-          if (diag && 32 * c + i > r) x = -INFINITY;
-          sr[c][i] = __float_as_uint(x);
-          mx = fmaxf(mx, x);
-        }
+        for (int i = 0; i < 32; ++i) mv[i & 7] = fmaxf(mv[i & 7], __uint_as_float(sr[c][i]));
+#pragma unroll
+      for (int w = 4; w > 0; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) mv[i] = fmaxf(mv[i], mv[i + w]);
+      const float mx = mv[0] * a.scale_log2;
       if (mx > m + kLazy) {
         if (m != -INFINITY) {
           // raise the maximum: O's row (after the previous P V) and l scale by 2^(m - mx)
@@ -234,15 +243,23 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
         m = mx;
       }
       uint32_t pk[2][32];
+      float ls[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) ls[i] = 0.0f;
 #pragma unroll
       for (int c = 0; c < 4; ++c)
 #pragma unroll
         for (int i = 0; i < 32; i += 2) {
-          const float p0 = fast_exp2(__uint_as_float(sr[c][i]) - m);
-          const float p1 = fast_exp2(__uint_as_float(sr[c][i + 1]) - m);
-          l += p0 + p1;
+          const float p0 = fast_exp2(fmaf(__uint_as_float(sr[c][i]), a.scale_log2, -m));
+          const float p1 = fast_exp2(fmaf(__uint_as_float(sr[c][i + 1]), a.scale_log2, -m));
+          ls[(i >> 1) & 7] += p0 + p1;
           pk[c >> 1][(c & 1) * 16 + i / 2] = pack2(p0, p1);
         }
+#pragma unroll
+      for (int w = 4; w > 0; w >>= 1)
+#pragma unroll
+        for (int i = 0; i < w; ++i) ls[i] += ls[i + w];
+      l += ls[0];
       // P_j (bf16, keys 2t and 2t + 1 in column t) over the first 64 columns of S_j
       tmem_st32(sbuf, pk[0]);
       tmem_st32(sbuf + 32u, pk[1]);
@@ -426,20 +443,28 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
       tc_fence_after();
       const bool diag = j == qt;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        uint32_t sv[32], pv[32], ds[16];
-        tmem_ld32(tmem + lane_off + kColS + 32u * c, sv);
-        tmem_ld32(tmem + lane_off + kColP + 32u * c, pv);
+      for (int c2 = 0; c2 < 4; c2 += 2) {  // two 32-column chunks per TMEM wait
+        uint32_t sv[2][32], pv[2][32];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          tmem_ld32(tmem + lane_off + kColS + 32u * (c2 + u), sv[u]);
+          tmem_ld32(tmem + lane_off + kColP + 32u * (c2 + u), pv[u]);
+        }
         tmem_ld_wait();
 #pragma unroll
-        for (int i = 0; i < 32; i += 2) {
-          float p0 = fast_exp2(fmaf(__uint_as_float(sv[i]), a.scale_log2, -lse2));
-          float p1 = fast_exp2(fmaf(__uint_as_float(sv[i + 1]), a.scale_log2, -lse2));
-          if (diag && 32 * c + i > r) p0 = 0.0f;
-          if (diag && 32 * c + i + 1 > r) p1 = 0.0f;
-          ds[i / 2] = pack2(p0 * (__uint_as_float(pv[i]) - dl), p1 * (__uint_as_float(pv[i + 1]) - dl));
+        for (int u = 0; u < 2; ++u) {
+          const int c = c2 + u;
+          uint32_t ds[16];
+#pragma unroll
+          for (int i = 0; i < 32; i += 2) {
+            float p0 = fast_exp2(fmaf(__uint_as_float(sv[u][i]), a.scale_log2, -lse2));
+            float p1 = fast_exp2(fmaf(__uint_as_float(sv[u][i + 1]), a.scale_log2, -lse2));
+            if (diag && 32 * c + i > r) p0 = 0.0f;
+            if (diag && 32 * c + i + 1 > r) p1 = 0.0f;
+            ds[i / 2] = pack2(p0 * (__uint_as_float(pv[u][i]) - dl), p1 * (__uint_as_float(pv[u][i + 1]) - dl));
+          }
+          tmem_st16(tmem + lane_off + kColS + 16u * c, ds);
         }
-        tmem_st16(tmem + lane_off + kColS + 16u * c, ds);
       }
       tmem_st_wait();
       tc_fence_before();
@@ -585,23 +610,32 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
       const float* dlt = reinterpret_cast<const float*>(gbase + kKvOffStage + (t & 1) * kStageBytes + kStageDelta);
       const bool diag = step_tile(t) == kt;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        uint32_t sv[32], pv[32], pp[16], ds[16];
-        tmem_ld32(tmem + lane_off + kColS + 32u * c, sv);
-        tmem_ld32(tmem + lane_off + kColP + 32u * c, pv);
+      for (int c2 = 0; c2 < 4; c2 += 2) {  // two 32-column chunks per TMEM wait
+        uint32_t sv[2][32], pv[2][32];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          tmem_ld32(tmem + lane_off + kColS + 32u * (c2 + u), sv[u]);
+          tmem_ld32(tmem + lane_off + kColP + 32u * (c2 + u), pv[u]);
+        }
         tmem_ld_wait();
 #pragma unroll
-        for (int i = 0; i < 32; i += 2) {
-          const int q = 32 * c + i;
-          float p0 = fast_exp2(fmaf(__uint_as_float(sv[i]), a.scale_log2, -lse[q] * kLog2e));
-          float p1 = fast_exp2(fmaf(__uint_as_float(sv[i + 1]), a.scale_log2, -lse[q + 1] * kLog2e));
-          if (diag && q < rk) p0 = 0.0f;
-          if (diag && q + 1 < rk) p1 = 0.0f;
-          pp[i / 2] = pack2(p0, p1);
-          ds[i / 2] = pack2(p0 * (__uint_as_float(pv[i]) - dlt[q]), p1 * (__uint_as_float(pv[i + 1]) - dlt[q + 1]));
+        for (int u = 0; u < 2; ++u) {
+          const int c = c2 + u;
+          uint32_t pp[16], ds[16];
+#pragma unroll
+          for (int i = 0; i < 32; i += 2) {
+            const int q = 32 * c + i;
+            float p0 = fast_exp2(fmaf(__uint_as_float(sv[u][i]), a.scale_log2, -lse[q] * kLog2e));
+            float p1 = fast_exp2(fmaf(__uint_as_float(sv[u][i + 1]), a.scale_log2, -lse[q + 1] * kLog2e));
+            if (diag && q < rk) p0 = 0.0f;
+            if (diag && q + 1 < rk) p1 = 0.0f;
+            pp[i / 2] = pack2(p0, p1);
+            ds[i / 2] =
+                pack2(p0 * (__uint_as_float(pv[u][i]) - dlt[q]), p1 * (__uint_as_float(pv[u][i + 1]) - dlt[q + 1]));
+          }
+          tmem_st16(tmem + lane_off + kColS + 16u * c, pp);
+          tmem_st16(tmem + lane_off + kColP + 16u * c, ds);
         }
-        tmem_st16(tmem + lane_off + kColS + 16u * c, pp);
-        tmem_st16(tmem + lane_off + kColP + 16u * c, ds);
       }
       tmem_st_wait();
       tc_fence_before();
