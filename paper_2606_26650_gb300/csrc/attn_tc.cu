@@ -1,8 +1,10 @@
-// attn_tc.cu — causal grouped-query attention forward on the tcgen05 tensor cores (head
-// dimension 128), for the block window's attention (softmax(Q K^T / sqrt(d)) V per head over the
-// keys up to the query's position; the row's natural log-sum-exp is kept for the backward).
+// attn_tc.cu — causal grouped-query attention on the tcgen05 tensor cores (head dimension 128,
+// sequences in whole 128-token tiles), for the block window's attention: the forward
+// (softmax(Q K^T / sqrt(d)) V per head over the keys up to the query's position, and the row's
+// natural log-sum-exp for the backward), and the backward in two kernels (dQ per query tile;
+// dK and dV per key tile over the query heads sharing it), without atomics.
 //
-// One CTA per (128-query tile, head, sequence), longest rows first.  Warp roles:
+// Forward: one CTA per (128-query tile, head, sequence), longest rows first.  Warp roles:
 //   warps 0-3  softmax and epilogue: thread = query row = TMEM lane (warp w owns lanes 32w..);
 //   warp 4     TMA: the Q tile once, then key/value tiles of 128 through two stages;
 //   warp 5     tcgen05: S_j = Q K_j^T into one of two TMEM score buffers, then
