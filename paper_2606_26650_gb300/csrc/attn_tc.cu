@@ -269,7 +269,10 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
       tc_fence_before();
       mbar_arrive_local(p_full);
     }
-    if (ok && mbar_wait(o_bar, (ntiles - 1) & 1, a.wc)) {
+    // every MMA of the tile loop has completed: final_bar has a single phase, while o_bar's
+    // parity can still show a phase two behind the last P V here (S_{j+1} is committed before
+    // P V_j, so the last score barrier only vouches for P V up to two tiles back)
+    if (ok && mbar_wait(final_bar, 0, a.wc)) {
       tc_fence_after();
       const float inv = 1.0f / l;
       const int64_t tok = static_cast<int64_t>(row0) + qt * kTq + r;
