@@ -330,7 +330,7 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16
       : "memory");
 }
 
-// Q/K-major SS products of the backward: D (+)= A B^T over d = 128 (A, B: 128 rows x 128
+// K-major SS products of the backward: D (+)= A B^T over d = 128 (A, B: 128 rows x 128
 // columns, two 64-column boxes each).
 __device__ __forceinline__ void mma_kmajor(uint32_t d_tmem, uint32_t a_smem, uint32_t b_smem, uint32_t idesc) {
 #pragma unroll
@@ -366,7 +366,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (base - raw) + kDqOffBar + 96);
   const uint32_t bar = base + kDqOffBar;
   const uint32_t qd_full = bar, kv_full0 = bar + 8, kv_empty0 = bar + 24, s_full = bar + 40, ds_full = bar + 48,
-                 q_done = bar + 56, final_bar = bar + 64;
+                 final_bar = bar + 64;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nqt = a.S / kTq;
   const int qt = nqt - 1 - static_cast<int>(blockIdx.x);
@@ -383,7 +383,6 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
     }
     mbar_init(s_full, 1);
     mbar_init(ds_full, kTq);
-    mbar_init(q_done, 1);
     mbar_init(final_bar, 1);
     fence_mbar_init_cluster();
   }
@@ -433,7 +432,6 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
         tc_fence_after();
         mma_ts_tile(tmem + kColQ, tmem + kColS, kt, idesc_q, j > 0);  // dQ += dS K
         umma_commit<1>(kv_empty0 + 8u * (j & 1));
-        umma_commit<1>(q_done);
       }
       umma_commit<1>(final_bar);
       drain(final_bar, 0);
@@ -475,7 +473,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
       tc_fence_before();
       mbar_arrive_local(ds_full);
     }
-    if (ok && mbar_wait(q_done, (ntiles - 1) & 1, a.wc)) {
+    if (ok && mbar_wait(final_bar, 0, a.wc)) {  // every MMA has completed (one phase)
       tc_fence_after();
       const int64_t tok = static_cast<int64_t>(row0) + qt * kTq + r;
       uint16_t* drow = a.dq + tok * (static_cast<int64_t>(a.nh) * kHd) + static_cast<int64_t>(h) * kHd;
@@ -526,7 +524,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + kKvOffBar + 96);
   const uint32_t bar = base + kKvOffBar;
   const uint32_t kv_full = bar, st_full0 = bar + 8, st_empty0 = bar + 24, s_full = bar + 40, pd_full = bar + 48,
-                 kv_done = bar + 56, final_bar = bar + 64;
+                 final_bar = bar + 64;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nqt = a.S / kTq;
   const int kt = static_cast<int>(blockIdx.x);  // key tile; the first ones have the most query tiles
@@ -545,7 +543,6 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
     }
     mbar_init(s_full, 1);
     mbar_init(pd_full, kTq);
-    mbar_init(kv_done, 1);
     mbar_init(final_bar, 1);
     fence_mbar_init_cluster();
   }
@@ -600,7 +597,6 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
         mma_ts_tile(tmem + kColV, tmem + kColS, sb + kTile, idesc_g, t > 0);  // dV += P^T dO
         mma_ts_tile(tmem + kColK, tmem + kColP, sb, idesc_g, t > 0);          // dK += dS^T Q
         umma_commit<1>(st_empty0 + 8u * (t & 1));
-        umma_commit<1>(kv_done);
       }
       umma_commit<1>(final_bar);
       drain(final_bar, 0);
@@ -646,7 +642,7 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
       tc_fence_before();
       mbar_arrive_local(pd_full);
     }
-    if (ok && mbar_wait(kv_done, (nsteps - 1) & 1, a.wc)) {
+    if (ok && mbar_wait(final_bar, 0, a.wc)) {  // every MMA has completed (one phase)
       tc_fence_after();
       const int64_t tok = static_cast<int64_t>(row0) + kt * kTk + rk;
       const int64_t off = tok * (static_cast<int64_t>(a.nkv) * kHd) + static_cast<int64_t>(hk) * kHd;
