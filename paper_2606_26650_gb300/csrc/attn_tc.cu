@@ -4,9 +4,11 @@
 // natural log-sum-exp for the backward), and the backward in two kernels (dQ per query tile;
 // dK and dV per key tile over the query heads sharing it), without atomics.
 //
-// Forward: one CTA per (128-query tile, head, sequence), longest rows first.  Warp roles:
+// Forward: a persistent CTA per SM takes every gridDim-th (128-query tile, head, sequence) work
+// item, longest rows first; the output accumulator has two TMEM buffers, so one item's
+// epilogue overlaps the next item's first products.  Warp roles:
 //   warps 0-3  softmax and epilogue: thread = query row = TMEM lane (warp w owns lanes 32w..);
-//   warp 4     TMA: the Q tile once, then key/value tiles of 128 through two stages;
+//   warp 4     TMA: each item's Q tile, then its key/value tiles of 128 through two stages;
 //   warp 5     tcgen05: S_j = Q K_j^T into one of two TMEM score buffers, then
 //              O += P_j V_j with P_j read from TMEM (the softmax stores it, bf16, over S_j).
 // S_{j+1} is issued before the MMA warp waits for P_j, so the next tile's scores are computed
@@ -17,6 +19,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 #include <mutex>
@@ -36,13 +39,13 @@ constexpr uint32_t kBox = 128 * 128;                 // one 64-column box of 128
 constexpr uint32_t kTile = 2 * kBox;                 // 128 rows x 128 columns, bytes
 constexpr uint32_t kOffQ = 0, kOffK = kTile, kOffV = 3 * kTile, kOffBar = 5 * kTile;
 constexpr uint32_t kSmem = kOffBar + 128 + 1024;     // + barriers, 1 KB alignment slack
-constexpr uint32_t kColS0 = 0, kColO = 256, kTmemCols = 512;
+constexpr uint32_t kColS0 = 0, kColO = 256, kTmemCols = 512;  // S0, S1; O0, O1 (one per item parity)
 constexpr float kLazy = 8.0f;                        // rescale only past this rise (log2 units)
 
 struct TcAttnArgs {
   uint16_t* out;
   float* lse;
-  int32_t S, nh, nkv;
+  int32_t B, S, nh, nkv;
   float scale_log2;
   WaitCtl wc;
 };
@@ -95,23 +98,33 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (base - raw) + kOffBar + 96);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (base - raw) + kOffBar + 120);
   const uint32_t bar = base + kOffBar;
-  const uint32_t q_full = bar, kv_full0 = bar + 8, kv_empty0 = bar + 24, s_full0 = bar + 40, p_full = bar + 56,
-                 o_bar = bar + 64, final_bar = bar + 72;
+  // per item: q_full, q_empty; per tile: kv_full[2], kv_empty[2], s_full[2], p_full, o_bar;
+  // per item and output buffer: item_done[2], o_free[2]; final_bar once
+  const uint32_t q_full = bar, q_empty = bar + 8, kv_full0 = bar + 16, kv_empty0 = bar + 32, s_full0 = bar + 48,
+                 p_full = bar + 64, o_bar = bar + 72, item_done0 = bar + 80, o_free0 = bar + 96,
+                 final_bar = bar + 112;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nqt = a.S / kTq;
-  const int qt = nqt - 1 - static_cast<int>(blockIdx.x);  // the longest rows first
-  const int h = blockIdx.y, b = blockIdx.z, hk = h / (a.nh / a.nkv);
-  const int ntiles = qt + 1;  // key tiles 0..qt (the last one on the diagonal)
-  const int32_t row0 = b * a.S;
+  const int n_items = nqt * a.nh * a.B;
+  // item -> (query tile, head, sequence), the longest rows first
+  auto item_of = [&](int it, int& qt, int& h, int& b) {
+    qt = nqt - 1 - it / (a.nh * a.B);
+    const int rem = it % (a.nh * a.B);
+    h = rem % a.nh;
+    b = rem / a.nh;
+  };
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
+    mbar_init(q_empty, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(kv_full0 + 8u * i, 1);
       mbar_init(kv_empty0 + 8u * i, 1);
       mbar_init(s_full0 + 8u * i, 1);
+      mbar_init(item_done0 + 8u * i, 1);
+      mbar_init(o_free0 + 8u * i, kTq);
     }
     mbar_init(p_full, kTq);
     mbar_init(o_bar, 1);
@@ -130,157 +143,184 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
       prefetch_tmap(&tmq);
       prefetch_tmap(&tmk);
       prefetch_tmap(&tmv);
-      mbar_arrive_expect_tx(q_full, kTile);
-      for (int hf = 0; hf < 2; ++hf)
-        tma_load_2d(base + kOffQ + hf * kBox, &tmq, q_full, h * kHd + 64 * hf, row0 + qt * kTq);
-      int issued = 0;
-      for (int j = 0; j < ntiles; ++j) {
-        const int st = j & 1;
-        if (j >= 2 && !mbar_wait(kv_empty0 + 8u * st, ((j >> 1) & 1) ^ 1, a.wc)) { ok = false; break; }
-        mbar_arrive_expect_tx(kv_full0 + 8u * st, 2 * kTile);
-        for (int hf = 0; hf < 2; ++hf) {
-          tma_load_2d(base + kOffK + st * kTile + hf * kBox, &tmk, kv_full0 + 8u * st, hk * kHd + 64 * hf,
-                      row0 + j * kTk);
-          tma_load_2d(base + kOffV + st * kTile + hf * kBox, &tmv, kv_full0 + 8u * st, hk * kHd + 64 * hf,
-                      row0 + j * kTk);
+      int g = 0, li = 0, q_loads = 0;
+      for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x, ++li) {
+        int qt, h, b;
+        item_of(it, qt, h, b);
+        const int hk = h / (a.nh / a.nkv);
+        const int32_t row0 = b * a.S;
+        // the Q buffer is free once every score product of the previous item has completed
+        if (li > 0 && !mbar_wait(q_empty, (li - 1) & 1, a.wc)) { ok = false; break; }
+        ++q_loads;
+        mbar_arrive_expect_tx(q_full, kTile);
+        for (int hf = 0; hf < 2; ++hf)
+          tma_load_2d(base + kOffQ + hf * kBox, &tmq, q_full, h * kHd + 64 * hf, row0 + qt * kTq);
+        for (int j = 0; j <= qt; ++j, ++g) {
+          const int st = g & 1;
+          if (g >= 2 && !mbar_wait(kv_empty0 + 8u * st, ((g >> 1) & 1) ^ 1, a.wc)) { ok = false; break; }
+          mbar_arrive_expect_tx(kv_full0 + 8u * st, 2 * kTile);
+          for (int hf = 0; hf < 2; ++hf) {
+            tma_load_2d(base + kOffK + st * kTile + hf * kBox, &tmk, kv_full0 + 8u * st, hk * kHd + 64 * hf,
+                        row0 + j * kTk);
+            tma_load_2d(base + kOffV + st * kTile + hf * kBox, &tmv, kv_full0 + 8u * st, hk * kHd + 64 * hf,
+                        row0 + j * kTk);
+          }
         }
-        issued = j + 1;
       }
-      // copies still in flight (the last two tiles' and Q's) must land before the CTA exits
-      drain(q_full, 0);
-      for (int j = issued - 2 < 0 ? 0 : issued - 2; j < issued; ++j) drain(kv_full0 + 8u * (j & 1), (j >> 1) & 1);
+      // copies still in flight (the last item's Q, the last two tiles) land before the CTA exits
+      if (q_loads > 0) drain(q_full, (q_loads - 1) & 1);
+      for (int t = g - 2 < 0 ? 0 : g - 2; t < g; ++t) drain(kv_full0 + 8u * (t & 1), (t >> 1) & 1);
     }
   } else if (warp == kMmaWarp) {
     if (lane == 0) {
       constexpr uint32_t idesc_s = idesc_bf16_f32(kTq, kTk, false, false);  // Q, K both K-major
       constexpr uint32_t idesc_o = idesc_bf16_f32(kTq, kHd, false, true);   // V MN-major
-      auto issue_s = [&](int j) {  // S_j = Q K_j^T into score buffer j & 1
-        const uint32_t kt = base + kOffK + (j & 1) * kTile;
+      // S_t = Q K^T of global tile t into score buffer t & 1; after an item's last one, the Q
+      // buffer is released
+      auto issue_s = [&](int t, bool last) -> bool {
+        if (!mbar_wait(kv_full0 + 8u * (t & 1), (t >> 1) & 1, a.wc)) return false;
+        tc_fence_after();
+        const uint32_t kt = base + kOffK + (t & 1) * kTile;
 #pragma unroll
         for (int kk = 0; kk < kHd / 16; ++kk) {
           const uint32_t off = (kk >> 2) * kBox + (kk & 3) * 32;
-          umma_bf16<1>(tmem + kColS0 + 128u * (j & 1), smem_desc_sw128(base + kOffQ + off, 16, 1024),
+          umma_bf16<1>(tmem + kColS0 + 128u * (t & 1), smem_desc_sw128(base + kOffQ + off, 16, 1024),
                        smem_desc_sw128(kt + off, 16, 1024), idesc_s, kk > 0 ? 1u : 0u);
         }
-        umma_commit<1>(s_full0 + 8u * (j & 1));
+        umma_commit<1>(s_full0 + 8u * (t & 1));
+        if (last) umma_commit<1>(q_empty);
+        return true;
       };
-      if (!mbar_wait(q_full, 0, a.wc)) ok = false;
-      if (ok && !mbar_wait(kv_full0, 0, a.wc)) ok = false;
-      if (ok) {
-        tc_fence_after();
-        issue_s(0);
-      }
-      for (int j = 0; ok && j < ntiles; ++j) {
-        if (j + 1 < ntiles) {
-          if (!mbar_wait(kv_full0 + 8u * ((j + 1) & 1), ((j + 1) >> 1) & 1, a.wc)) { ok = false; break; }
+      int g = 0, li = 0;
+      for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x, ++li) {
+        int qt, h, b;
+        item_of(it, qt, h, b);
+        const int n = qt + 1;
+        const uint32_t ocol = tmem + kColO + 128u * (li & 1);
+        if (!mbar_wait(q_full, li & 1, a.wc) || !issue_s(g, n == 1)) { ok = false; break; }
+        for (int j = 0; ok && j < n; ++j) {
+          const int t = g + j;
+          if (j + 1 < n && !issue_s(t + 1, j + 2 == n)) { ok = false; break; }
+          if (!mbar_wait(p_full, t & 1, a.wc)) { ok = false; break; }
+          // the item's output buffer is free once the epilogue two items back has read it
+          if (j == 0 && li >= 2 && !mbar_wait(o_free0 + 8u * (li & 1), ((li >> 1) & 1) ^ 1, a.wc)) {
+            ok = false;
+            break;
+          }
           tc_fence_after();
-          issue_s(j + 1);
-        }
-        if (!mbar_wait(p_full, j & 1, a.wc)) { ok = false; break; }
-        tc_fence_after();
-        const uint32_t vt = base + kOffV + (j & 1) * kTile;
-        const uint32_t pcol = tmem + kColS0 + 128u * (j & 1);
+          const uint32_t vt = base + kOffV + (t & 1) * kTile;
+          const uint32_t pcol = tmem + kColS0 + 128u * (t & 1);
 #pragma unroll
-        for (int kk = 0; kk < kTk / 16; ++kk)
-          umma_ts(tmem + kColO, pcol + 8u * kk, smem_desc_sw128(vt + kk * 2048, kBox, 1024), idesc_o,
-                  (j > 0 || kk > 0) ? 1u : 0u);
-        umma_commit<1>(o_bar);
-        umma_commit<1>(kv_empty0 + 8u * (j & 1));
+          for (int kk = 0; kk < kTk / 16; ++kk)
+            umma_ts(ocol, pcol + 8u * kk, smem_desc_sw128(vt + kk * 2048, kBox, 1024), idesc_o,
+                    (j > 0 || kk > 0) ? 1u : 0u);
+          umma_commit<1>(o_bar);
+          umma_commit<1>(kv_empty0 + 8u * (t & 1));
+        }
+        if (!ok) break;
+        umma_commit<1>(item_done0 + 8u * (li & 1));
+        g += n;
       }
       // every MMA has completed before TMEM is released
       umma_commit<1>(final_bar);
       drain(final_bar, 0);
     }
   } else {
-    // softmax: this thread's query row r of the tile (TMEM lane r)
+    // softmax and epilogue: this thread's query row r of each item's tile (TMEM lane r)
     const int r = warp * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
-    float m = -INFINITY, l = 0.0f;
-    for (int j = 0; ok && j < ntiles; ++j) {
-      const uint32_t sbuf = tmem + lane_off + kColS0 + 128u * (j & 1);
-      if (!mbar_wait(s_full0 + 8u * (j & 1), (j >> 1) & 1, a.wc)) { ok = false; break; }
-      tc_fence_after();
-      uint32_t sr[4][32];
+    int g = 0, li = 0;
+    for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x, ++li) {
+      int qt, h, b;
+      item_of(it, qt, h, b);
+      const int n = qt + 1;
+      const uint32_t orow = tmem + lane_off + kColO + 128u * (li & 1);
+      float m = -INFINITY, l = 0.0f;
+      for (int j = 0; ok && j < n; ++j) {
+        const int t = g + j;
+        const uint32_t sbuf = tmem + lane_off + kColS0 + 128u * (t & 1);
+        if (!mbar_wait(s_full0 + 8u * (t & 1), (t >> 1) & 1, a.wc)) { ok = false; break; }
+        tc_fence_after();
+        uint32_t sr[4][32];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(sbuf + 32u * c, sr[c]);
-      tmem_ld_wait();
-      if (j == qt) {  // the diagonal tile: keys after the row's query do not count
+        for (int c = 0; c < 4; ++c) tmem_ld32(sbuf + 32u * c, sr[c]);
+        tmem_ld_wait();
+        if (j == qt) {  // the diagonal tile: keys after the row's query do not count
+#pragma unroll
+          for (int c = 0; c < 4; ++c)
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (32 * c + i > r) sr[c][i] = __float_as_uint(-INFINITY);
+        }
+        // the row maximum of the raw scores (scale > 0), in eight independent chains
+        float mv[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) mv[i] = -INFINITY;
 #pragma unroll
         for (int c = 0; c < 4; ++c)
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (32 * c + i > r) sr[c][i] = __float_as_uint(-INFINITY);
-      }
-      // the row maximum of the raw scores (scale > 0), in eight independent chains
-      float mv[8];
+          for (int i = 0; i < 32; ++i) mv[i & 7] = fmaxf(mv[i & 7], __uint_as_float(sr[c][i]));
 #pragma unroll
-      for (int i = 0; i < 8; ++i) mv[i] = -INFINITY;
+        for (int w = 4; w > 0; w >>= 1)
 #pragma unroll
-      for (int c = 0; c < 4; ++c)
+          for (int i = 0; i < w; ++i) mv[i] = fmaxf(mv[i], mv[i + w]);
+        const float mx = mv[0] * a.scale_log2;
+        if (mx > m + kLazy) {
+          if (m != -INFINITY) {
+            // raise the maximum: O's row (after the previous P V) and l scale by 2^(m - mx)
+            const float f = fast_exp2(m - mx);
+            l *= f;
+            if (!mbar_wait(o_bar, (t - 1) & 1, a.wc)) { ok = false; break; }
+            tc_fence_after();
 #pragma unroll
-        for (int i = 0; i < 32; ++i) mv[i & 7] = fmaxf(mv[i & 7], __uint_as_float(sr[c][i]));
+            for (int c = 0; c < 4; ++c) {
+              uint32_t o[32];
+              tmem_ld32(orow + 32u * c, o);
+              tmem_ld_wait();
 #pragma unroll
-      for (int w = 4; w > 0; w >>= 1)
-#pragma unroll
-        for (int i = 0; i < w; ++i) mv[i] = fmaxf(mv[i], mv[i + w]);
-      const float mx = mv[0] * a.scale_log2;
-      if (mx > m + kLazy) {
-        if (m != -INFINITY) {
-          // raise the maximum: O's row (after the previous P V) and l scale by 2^(m - mx)
-          const float f = fast_exp2(m - mx);
-          l *= f;
-          if (!mbar_wait(o_bar, (j - 1) & 1, a.wc)) { ok = false; break; }
-          tc_fence_after();
-          const uint32_t orow = tmem + lane_off + kColO;
-#pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            uint32_t o[32];
-            tmem_ld32(orow + 32u * c, o);
-            tmem_ld_wait();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
-            tmem_st32(orow + 32u * c, o);
+              for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
+              tmem_st32(orow + 32u * c, o);
+            }
           }
+          m = mx;
         }
-        m = mx;
+        uint32_t pk[2][32];
+        float ls[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) ls[i] = 0.0f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int i = 0; i < 32; i += 2) {
+            const float p0 = fast_exp2(fmaf(__uint_as_float(sr[c][i]), a.scale_log2, -m));
+            const float p1 = fast_exp2(fmaf(__uint_as_float(sr[c][i + 1]), a.scale_log2, -m));
+            ls[(i >> 1) & 7] += p0 + p1;
+            pk[c >> 1][(c & 1) * 16 + i / 2] = pack2(p0, p1);
+          }
+#pragma unroll
+        for (int w = 4; w > 0; w >>= 1)
+#pragma unroll
+          for (int i = 0; i < w; ++i) ls[i] += ls[i + w];
+        l += ls[0];
+        // P_t (bf16, keys 2u and 2u + 1 in column u) over the first 64 columns of S_t
+        tmem_st32(sbuf, pk[0]);
+        tmem_st32(sbuf + 32u, pk[1]);
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive_local(p_full);
       }
-      uint32_t pk[2][32];
-      float ls[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) ls[i] = 0.0f;
-#pragma unroll
-      for (int c = 0; c < 4; ++c)
-#pragma unroll
-        for (int i = 0; i < 32; i += 2) {
-          const float p0 = fast_exp2(fmaf(__uint_as_float(sr[c][i]), a.scale_log2, -m));
-          const float p1 = fast_exp2(fmaf(__uint_as_float(sr[c][i + 1]), a.scale_log2, -m));
-          ls[(i >> 1) & 7] += p0 + p1;
-          pk[c >> 1][(c & 1) * 16 + i / 2] = pack2(p0, p1);
-        }
-#pragma unroll
-      for (int w = 4; w > 0; w >>= 1)
-#pragma unroll
-        for (int i = 0; i < w; ++i) ls[i] += ls[i + w];
-      l += ls[0];
-      // P_j (bf16, keys 2t and 2t + 1 in column t) over the first 64 columns of S_j
-      tmem_st32(sbuf, pk[0]);
-      tmem_st32(sbuf + 32u, pk[1]);
-      tmem_st_wait();
-      tc_fence_before();
-      mbar_arrive_local(p_full);
-    }
-    // every MMA of the tile loop has completed: final_bar has a single phase, while o_bar's
-    // parity can still show a phase two behind the last P V here (S_{j+1} is committed before
-    // P V_j, so the last score barrier only vouches for P V up to two tiles back)
-    if (ok && mbar_wait(final_bar, 0, a.wc)) {
+      if (!ok) break;
+      // the item's output: every P V of the item has completed (item_done, one phase per use
+      // of the buffer); then the buffer goes back to the MMA warp for the item after next
+      if (!mbar_wait(item_done0 + 8u * (li & 1), (li >> 1) & 1, a.wc)) { ok = false; break; }
       tc_fence_after();
       const float inv = 1.0f / l;
-      const int64_t tok = static_cast<int64_t>(row0) + qt * kTq + r;
-      uint16_t* orow = a.out + tok * (static_cast<int64_t>(a.nh) * kHd) + static_cast<int64_t>(h) * kHd;
+      const int64_t tok = static_cast<int64_t>(b) * a.S + qt * kTq + r;
+      uint16_t* dst = a.out + tok * (static_cast<int64_t>(a.nh) * kHd) + static_cast<int64_t>(h) * kHd;
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         uint32_t o[32];
-        tmem_ld32(tmem + lane_off + kColO + 32u * c, o);
+        tmem_ld32(orow + 32u * c, o);
         tmem_ld_wait();
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
@@ -289,10 +329,13 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
           w.y = pack2(__uint_as_float(o[8 * v + 2]) * inv, __uint_as_float(o[8 * v + 3]) * inv);
           w.z = pack2(__uint_as_float(o[8 * v + 4]) * inv, __uint_as_float(o[8 * v + 5]) * inv);
           w.w = pack2(__uint_as_float(o[8 * v + 6]) * inv, __uint_as_float(o[8 * v + 7]) * inv);
-          *reinterpret_cast<uint4*>(orow + 32 * c + 8 * v) = w;
+          *reinterpret_cast<uint4*>(dst + 32 * c + 8 * v) = w;
         }
       }
       a.lse[(static_cast<int64_t>(b) * a.nh + h) * a.S + qt * kTq + r] = (m + log2f(l)) * 0.69314718055994531f;
+      tc_fence_before();
+      mbar_arrive_local(o_free0 + 8u * (li & 1));
+      g += n;
     }
   }
   tc_fence_before();
@@ -718,6 +761,7 @@ cudaError_t launch_attention_fwd_tc(const void* q, const void* k, const void* v,
   TcAttnArgs a{};
   a.out = static_cast<uint16_t*>(out);
   a.lse = lse;
+  a.B = B;
   a.S = S;
   a.nh = nh;
   a.nkv = nkv;
@@ -725,7 +769,12 @@ cudaError_t launch_attention_fwd_tc(const void* q, const void* k, const void* v,
   if (!launch_wait_ctl(&a.wc)) return cudaErrorInvalidDevice;
   cudaError_t e = cudaFuncSetAttribute(attn_tc_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
   if (e != cudaSuccess) return e;
-  attn_tc_fwd_kernel<<<dim3(S / kTq, nh, B), kThreadsTc, kSmem, st>>>(tq, tk, tv, a);
+  int sm = 152, dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sm, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t items = static_cast<int64_t>(S / kTq) * nh * B;
+  // persistent: one CTA per SM (shared memory and the 512 TMEM columns allow no second), each
+  // taking every gridDim-th work item
+  attn_tc_fwd_kernel<<<static_cast<unsigned>(std::min<int64_t>(items, sm)), kThreadsTc, kSmem, st>>>(tq, tk, tv, a);
   return cudaGetLastError();
 }
 
