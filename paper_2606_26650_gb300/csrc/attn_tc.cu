@@ -356,7 +356,7 @@ struct TcBwdArgs {
   uint16_t *dq, *dk, *dv;
   const float* lse;    // natural log-sum-exp per (sequence, head, row)
   const float* delta;  // rowsum(dO * O) per (sequence, head, row)
-  int32_t S, nh, nkv;
+  int32_t B, S, nh, nkv;
   float scale_log2;
   float scale;
   WaitCtl wc;
@@ -394,8 +394,10 @@ __device__ __forceinline__ void mma_ts_tile(uint32_t d_tmem, uint32_t a_tmem, ui
             (accumulate || kk > 0) ? 1u : 0u);
 }
 
-// dQ: one CTA per (128-query tile, head, sequence), over the key tiles up to the diagonal.
-// TMEM: S [0, 128), dP [128, 256), dQ [256, 384); dS (bf16) goes over S's first 64 columns.
+// dQ: persistent CTAs over (128-query tile, head, sequence) items (the forward's order), each
+// over the key tiles up to the diagonal.  TMEM: S [0, 128), dP [128, 256), dQ in two buffers
+// [256, 512) (one per item parity, so an item's epilogue overlaps the next item's products);
+// dS (bf16) goes over S's first 64 columns.
 constexpr uint32_t kDqOffQ = 0, kDqOffDo = kTile, kDqOffK = 2 * kTile, kDqOffV = 4 * kTile, kDqOffBar = 6 * kTile;
 constexpr uint32_t kDqSmem = kDqOffBar + 128 + 1024;
 
@@ -406,23 +408,29 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (base - raw) + kDqOffBar + 96);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem_raw + (base - raw) + kDqOffBar + 120);
   const uint32_t bar = base + kDqOffBar;
-  const uint32_t qd_full = bar, kv_full0 = bar + 8, kv_empty0 = bar + 24, s_full = bar + 40, ds_full = bar + 48,
-                 final_bar = bar + 64;
+  const uint32_t qd_full = bar, qd_empty = bar + 8, kv_full0 = bar + 16, kv_empty0 = bar + 32, s_full = bar + 48,
+                 ds_full = bar + 56, item_done0 = bar + 64, dq_free0 = bar + 80, final_bar = bar + 96;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nqt = a.S / kTq;
-  const int qt = nqt - 1 - static_cast<int>(blockIdx.x);
-  const int h = blockIdx.y, b = blockIdx.z, hk = h / (a.nh / a.nkv);
-  const int ntiles = qt + 1;
-  const int32_t row0 = b * a.S;
+  const int n_items = nqt * a.nh * a.B;
+  auto item_of = [&](int it, int& qt, int& h, int& b) {
+    qt = nqt - 1 - it / (a.nh * a.B);
+    const int rem = it % (a.nh * a.B);
+    h = rem % a.nh;
+    b = rem / a.nh;
+  };
   constexpr uint32_t kColS = 0, kColP = 128, kColQ = 256;
 
   if (threadIdx.x == 0) {
     mbar_init(qd_full, 1);
+    mbar_init(qd_empty, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(kv_full0 + 8u * i, 1);
       mbar_init(kv_empty0 + 8u * i, 1);
+      mbar_init(item_done0 + 8u * i, 1);
+      mbar_init(dq_free0 + 8u * i, kTq);
     }
     mbar_init(s_full, 1);
     mbar_init(ds_full, kTq);
@@ -438,43 +446,68 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
 
   if (warp == kTmaWarp) {
     if (lane == 0) {
-      mbar_arrive_expect_tx(qd_full, 2 * kTile);
-      for (int hf = 0; hf < 2; ++hf) {
-        tma_load_2d(base + kDqOffQ + hf * kBox, &tmq, qd_full, h * kHd + 64 * hf, row0 + qt * kTq);
-        tma_load_2d(base + kDqOffDo + hf * kBox, &tmdo, qd_full, h * kHd + 64 * hf, row0 + qt * kTq);
-      }
-      int issued = 0;
-      for (int j = 0; j < ntiles; ++j) {
-        const int st = j & 1;
-        if (j >= 2 && !mbar_wait(kv_empty0 + 8u * st, ((j >> 1) & 1) ^ 1, a.wc)) { ok = false; break; }
-        mbar_arrive_expect_tx(kv_full0 + 8u * st, 2 * kTile);
+      int g = 0, li = 0, qd_loads = 0;
+      for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x, ++li) {
+        int qt, h, b;
+        item_of(it, qt, h, b);
+        const int hk = h / (a.nh / a.nkv);
+        const int32_t row0 = b * a.S;
+        // Q and dO are free once the previous item's S and dP products have completed
+        if (li > 0 && !mbar_wait(qd_empty, (li - 1) & 1, a.wc)) { ok = false; break; }
+        ++qd_loads;
+        mbar_arrive_expect_tx(qd_full, 2 * kTile);
         for (int hf = 0; hf < 2; ++hf) {
-          tma_load_2d(base + kDqOffK + st * kTile + hf * kBox, &tmk, kv_full0 + 8u * st, hk * kHd + 64 * hf,
-                      row0 + j * kTk);
-          tma_load_2d(base + kDqOffV + st * kTile + hf * kBox, &tmv, kv_full0 + 8u * st, hk * kHd + 64 * hf,
-                      row0 + j * kTk);
+          tma_load_2d(base + kDqOffQ + hf * kBox, &tmq, qd_full, h * kHd + 64 * hf, row0 + qt * kTq);
+          tma_load_2d(base + kDqOffDo + hf * kBox, &tmdo, qd_full, h * kHd + 64 * hf, row0 + qt * kTq);
         }
-        issued = j + 1;
+        for (int j = 0; j <= qt; ++j, ++g) {
+          const int st = g & 1;
+          if (g >= 2 && !mbar_wait(kv_empty0 + 8u * st, ((g >> 1) & 1) ^ 1, a.wc)) { ok = false; break; }
+          mbar_arrive_expect_tx(kv_full0 + 8u * st, 2 * kTile);
+          for (int hf = 0; hf < 2; ++hf) {
+            tma_load_2d(base + kDqOffK + st * kTile + hf * kBox, &tmk, kv_full0 + 8u * st, hk * kHd + 64 * hf,
+                        row0 + j * kTk);
+            tma_load_2d(base + kDqOffV + st * kTile + hf * kBox, &tmv, kv_full0 + 8u * st, hk * kHd + 64 * hf,
+                        row0 + j * kTk);
+          }
+        }
       }
-      drain(qd_full, 0);
-      for (int j = issued - 2 < 0 ? 0 : issued - 2; j < issued; ++j) drain(kv_full0 + 8u * (j & 1), (j >> 1) & 1);
+      if (qd_loads > 0) drain(qd_full, (qd_loads - 1) & 1);
+      for (int t = g - 2 < 0 ? 0 : g - 2; t < g; ++t) drain(kv_full0 + 8u * (t & 1), (t >> 1) & 1);
     }
   } else if (warp == kMmaWarp) {
     if (lane == 0) {
       constexpr uint32_t idesc_s = idesc_bf16_f32(kTq, kTk, false, false);
       constexpr uint32_t idesc_q = idesc_bf16_f32(kTq, kHd, false, true);
-      if (!mbar_wait(qd_full, 0, a.wc)) ok = false;
-      for (int j = 0; ok && j < ntiles; ++j) {
-        const uint32_t kt = base + kDqOffK + (j & 1) * kTile, vt = base + kDqOffV + (j & 1) * kTile;
-        if (!mbar_wait(kv_full0 + 8u * (j & 1), (j >> 1) & 1, a.wc)) { ok = false; break; }
-        tc_fence_after();
-        mma_kmajor(tmem + kColS, base + kDqOffQ, kt, idesc_s);   // S = Q K^T
-        mma_kmajor(tmem + kColP, base + kDqOffDo, vt, idesc_s);  // dP = dO V^T
-        umma_commit<1>(s_full);
-        if (!mbar_wait(ds_full, j & 1, a.wc)) { ok = false; break; }
-        tc_fence_after();
-        mma_ts_tile(tmem + kColQ, tmem + kColS, kt, idesc_q, j > 0);  // dQ += dS K
-        umma_commit<1>(kv_empty0 + 8u * (j & 1));
+      int g = 0, li = 0;
+      for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x, ++li) {
+        int qt, h, b;
+        item_of(it, qt, h, b);
+        const int n = qt + 1;
+        const uint32_t qcol = tmem + kColQ + 128u * (li & 1);
+        if (!mbar_wait(qd_full, li & 1, a.wc)) { ok = false; break; }
+        for (int j = 0; ok && j < n; ++j) {
+          const int t = g + j;
+          const uint32_t kt = base + kDqOffK + (t & 1) * kTile, vt = base + kDqOffV + (t & 1) * kTile;
+          if (!mbar_wait(kv_full0 + 8u * (t & 1), (t >> 1) & 1, a.wc)) { ok = false; break; }
+          tc_fence_after();
+          mma_kmajor(tmem + kColS, base + kDqOffQ, kt, idesc_s);   // S = Q K^T
+          mma_kmajor(tmem + kColP, base + kDqOffDo, vt, idesc_s);  // dP = dO V^T
+          umma_commit<1>(s_full);
+          if (j + 1 == n) umma_commit<1>(qd_empty);
+          if (!mbar_wait(ds_full, t & 1, a.wc)) { ok = false; break; }
+          // the item's dQ buffer is free once the epilogue two items back has read it
+          if (j == 0 && li >= 2 && !mbar_wait(dq_free0 + 8u * (li & 1), ((li >> 1) & 1) ^ 1, a.wc)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          mma_ts_tile(qcol, tmem + kColS, kt, idesc_q, j > 0);  // dQ += dS K
+          umma_commit<1>(kv_empty0 + 8u * (t & 1));
+        }
+        if (!ok) break;
+        umma_commit<1>(item_done0 + 8u * (li & 1));
+        g += n;
       }
       umma_commit<1>(final_bar);
       drain(final_bar, 0);
@@ -482,48 +515,57 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
   } else {
     const int r = warp * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
-    const int64_t ridx = (static_cast<int64_t>(b) * a.nh + h) * a.S + qt * kTq + r;
-    const float lse2 = a.lse[ridx] * kLog2e, dl = a.delta[ridx];
-    for (int j = 0; ok && j < ntiles; ++j) {
-      if (!mbar_wait(s_full, j & 1, a.wc)) { ok = false; break; }
-      tc_fence_after();
-      const bool diag = j == qt;
+    int g = 0, li = 0;
+    for (int it = blockIdx.x; ok && it < n_items; it += gridDim.x, ++li) {
+      int qt, h, b;
+      item_of(it, qt, h, b);
+      const int n = qt + 1;
+      const int64_t ridx = (static_cast<int64_t>(b) * a.nh + h) * a.S + qt * kTq + r;
+      const float lse2 = a.lse[ridx] * kLog2e, dl = a.delta[ridx];
+      for (int j = 0; ok && j < n; ++j) {
+        const int t = g + j;
+        if (!mbar_wait(s_full, t & 1, a.wc)) { ok = false; break; }
+        tc_fence_after();
+        const bool diag = j == qt;
 #pragma unroll
-      for (int c2 = 0; c2 < 4; c2 += 2) {  // two 32-column chunks per TMEM wait
-        uint32_t sv[2][32], pv[2][32];
+        for (int c2 = 0; c2 < 4; c2 += 2) {  // two 32-column chunks per TMEM wait
+          uint32_t sv[2][32], pv[2][32];
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          tmem_ld32(tmem + lane_off + kColS + 32u * (c2 + u), sv[u]);
-          tmem_ld32(tmem + lane_off + kColP + 32u * (c2 + u), pv[u]);
-        }
-        tmem_ld_wait();
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const int c = c2 + u;
-          uint32_t ds[16];
-#pragma unroll
-          for (int i = 0; i < 32; i += 2) {
-            float p0 = fast_exp2(fmaf(__uint_as_float(sv[u][i]), a.scale_log2, -lse2));
-            float p1 = fast_exp2(fmaf(__uint_as_float(sv[u][i + 1]), a.scale_log2, -lse2));
-            if (diag && 32 * c + i > r) p0 = 0.0f;
-            if (diag && 32 * c + i + 1 > r) p1 = 0.0f;
-            ds[i / 2] = pack2(p0 * (__uint_as_float(pv[u][i]) - dl), p1 * (__uint_as_float(pv[u][i + 1]) - dl));
+          for (int u = 0; u < 2; ++u) {
+            tmem_ld32(tmem + lane_off + kColS + 32u * (c2 + u), sv[u]);
+            tmem_ld32(tmem + lane_off + kColP + 32u * (c2 + u), pv[u]);
           }
-          tmem_st16(tmem + lane_off + kColS + 16u * c, ds);
+          tmem_ld_wait();
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int c = c2 + u;
+            uint32_t ds[16];
+#pragma unroll
+            for (int i = 0; i < 32; i += 2) {
+              float p0 = fast_exp2(fmaf(__uint_as_float(sv[u][i]), a.scale_log2, -lse2));
+              float p1 = fast_exp2(fmaf(__uint_as_float(sv[u][i + 1]), a.scale_log2, -lse2));
+              if (diag && 32 * c + i > r) p0 = 0.0f;
+              if (diag && 32 * c + i + 1 > r) p1 = 0.0f;
+              ds[i / 2] = pack2(p0 * (__uint_as_float(pv[u][i]) - dl), p1 * (__uint_as_float(pv[u][i + 1]) - dl));
+            }
+            tmem_st16(tmem + lane_off + kColS + 16u * c, ds);
+          }
         }
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive_local(ds_full);
       }
-      tmem_st_wait();
-      tc_fence_before();
-      mbar_arrive_local(ds_full);
-    }
-    if (ok && mbar_wait(final_bar, 0, a.wc)) {  // every MMA has completed (one phase)
+      if (!ok) break;
+      // every dQ product of the item has completed (item_done, one phase per use of the buffer)
+      if (!mbar_wait(item_done0 + 8u * (li & 1), (li >> 1) & 1, a.wc)) { ok = false; break; }
       tc_fence_after();
-      const int64_t tok = static_cast<int64_t>(row0) + qt * kTq + r;
+      const int64_t tok = static_cast<int64_t>(b) * a.S + qt * kTq + r;
       uint16_t* drow = a.dq + tok * (static_cast<int64_t>(a.nh) * kHd) + static_cast<int64_t>(h) * kHd;
+      const uint32_t qrow = tmem + lane_off + kColQ + 128u * (li & 1);
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         uint32_t o[32];
-        tmem_ld32(tmem + lane_off + kColQ + 32u * c, o);
+        tmem_ld32(qrow + 32u * c, o);
         tmem_ld_wait();
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
@@ -535,6 +577,9 @@ __global__ void __launch_bounds__(kThreadsTc, 1)
           *reinterpret_cast<uint4*>(drow + 32 * c + 8 * v) = w;
         }
       }
+      tc_fence_before();
+      mbar_arrive_local(dq_free0 + 8u * (li & 1));
+      g += n;
     }
   }
   tc_fence_before();
@@ -797,6 +842,7 @@ cudaError_t launch_attention_bwd_tc(const void* q, const void* k, const void* v,
   a.dv = static_cast<uint16_t*>(dv);
   a.lse = lse;
   a.delta = delta;
+  a.B = B;
   a.S = S;
   a.nh = nh;
   a.nkv = nkv;
@@ -805,7 +851,11 @@ cudaError_t launch_attention_bwd_tc(const void* q, const void* k, const void* v,
   if (!launch_wait_ctl(&a.wc)) return cudaErrorInvalidDevice;
   cudaError_t e = cudaFuncSetAttribute(attn_tc_dq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDqSmem);
   if (e != cudaSuccess) return e;
-  attn_tc_dq_kernel<<<dim3(S / kTq, nh, B), kThreadsTc, kDqSmem, st>>>(tq, tdo, tk, tv, a);
+  int sm = 152, dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sm, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t items = static_cast<int64_t>(S / kTq) * nh * B;
+  attn_tc_dq_kernel<<<static_cast<unsigned>(std::min<int64_t>(items, sm)), kThreadsTc, kDqSmem, st>>>(tq, tdo, tk, tv,
+                                                                                                        a);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   e = cudaFuncSetAttribute(attn_tc_dkdv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kKvSmem);
   if (e != cudaSuccess) return e;
