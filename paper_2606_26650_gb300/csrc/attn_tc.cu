@@ -1,8 +1,9 @@
 // attn_tc.cu — causal grouped-query attention on the tcgen05 tensor cores (head dimension 128,
 // sequences in whole 128-token tiles), for the block window's attention: the forward
 // (softmax(Q K^T / sqrt(d)) V per head over the keys up to the query's position, and the row's
-// natural log-sum-exp for the backward), and the backward in two kernels (dQ per query tile;
-// dK and dV per key tile over the query heads sharing it), without atomics.
+// natural log-sum-exp for the backward), and the backward in two kernels (dQ per query tile,
+// persistent over the forward's work items; dK and dV per key tile over the query heads
+// sharing it), without atomics.
 //
 // Forward: a persistent CTA per SM takes every gridDim-th (128-query tile, head, sequence) work
 // item, longest rows first; the output accumulator has two TMEM buffers, so one item's
