@@ -551,12 +551,17 @@ catq_status catq_block_output_loss(const float* h, const void* branch, int64_t c
                                    int32_t reduction, float* loss_out, void* d_out, float* out, void* workspace,
                                    size_t ws_bytes, catq_stream stream);
 
-/* Causal grouped-query attention: query head h uses key/value head h / (n_heads / n_kv_heads),
+/* Causal grouped-query attention of the decoder block that forms the reconstruction window
+ * of Eq. 7 (§2.4): query head h uses key/value head h / (n_heads / n_kv_heads),
  *   O = softmax(Q K^T / sqrt(d), keys s' <= s) V   for every sequence b and head h,
- * with Q, O [B S, n_heads d], K, V [B S, n_kv_heads d], and lse [B, n_heads, S] the natural
- * log-sum-exp of each row's scaled scores (kept for the backward).  Scores, the softmax and
- * the accumulation run in fp32; the probabilities enter P V in bf16.  d is 64 or 128;
- * S % 64 == 0; n_heads % n_kv_heads == 0. */
+ * with Q, O [B S, n_heads d], K, V [B S, n_kv_heads d] (bf16, device, row-major, caller-owned),
+ * and lse [B, n_heads, S] (device fp32) the natural log-sum-exp of each row's scaled scores
+ * (kept for the backward).  Scores, the softmax and the accumulation run in fp32; the
+ * probabilities enter P V in bf16.  d is 64 or 128; S % 64 == 0; 0 <= B <= 65535;
+ * n_heads % n_kv_heads == 0 (else CATQ_ERR_SHAPE).  Null pointers: CATQ_ERR_INVALID_ARG;
+ * Q, K, V, O not 16-byte or lse not 4-byte aligned: CATQ_ERR_ALIGN.  d = 128 with
+ * S % 128 == 0 runs on the tcgen05 tensor cores, other shapes on the mma.sync path; the two
+ * agree up to rounding. */
 catq_status catq_attention_fwd(const void* Q, const void* K, const void* V, int32_t B, int32_t S, int32_t n_heads,
                                int32_t n_kv_heads, int32_t d, void* O, float* lse, catq_stream stream);
 
@@ -564,7 +569,8 @@ catq_status catq_attention_fwd(const void* Q, const void* K, const void* V, int3
  *   dS = P (dO V^T - rowsum(dO O)),  dQ = dS K / sqrt(d),
  *   dK = sum over the heads sharing it of dS^T Q / sqrt(d),  dV = the same sum of P^T dO.
  * delta: device fp32 scratch [B, n_heads, S].  dQ like Q, dK and dV like K; all three are
- * overwritten (no atomics: the result does not depend on scheduling). */
+ * overwritten (no atomics: the result does not depend on scheduling).  Shapes, errors and
+ * the choice of kernels as for catq_attention_fwd. */
 catq_status catq_attention_bwd(const void* Q, const void* K, const void* V, const void* O, const void* dO,
                                const float* lse, int32_t B, int32_t S, int32_t n_heads, int32_t n_kv_heads,
                                int32_t d, float* delta, void* dQ, void* dK, void* dV, catq_stream stream);
