@@ -154,3 +154,74 @@ def test_schedule_and_update_validation(lib):
                 C.adamw(margin=0.5), C.adamw(eps=float("inf"))):
         assert step(8, *ptrs, ctypes.byref(bad), 1, 1e-3, None) == 1
     assert step(8, *ptrs[:6], ptrs[6] + 2, ctypes.byref(hp), 1, 1e-3, None) == 4  # misaligned moments
+
+
+def test_block_call_validation(lib):
+    """The decoder-block calls reject bad shapes, dtypes, scalars, null and misaligned
+    pointers and short workspaces on the host, and treat empty inputs as no-ops, before any
+    launch (fake device addresses, never dereferenced)."""
+    inf, nan = float("inf"), float("nan")
+    att = lib.catq_attention_fwd
+    assert att(16, 16, 16, 1, 100, 8, 2, 128, 16, 16, None) == 2    # S % 64 != 0
+    assert att(16, 16, 16, 1, 32, 8, 2, 128, 16, 16, None) == 2     # S < 64
+    assert att(16, 16, 16, 1, 128, 8, 2, 96, 16, 16, None) == 2     # d not 64 or 128
+    assert att(16, 16, 16, 1, 128, 6, 4, 128, 16, 16, None) == 2    # heads do not share evenly
+    assert att(16, 16, 16, -1, 128, 8, 2, 128, 16, 16, None) == 2
+    assert att(16, 16, 16, 70000, 128, 8, 2, 128, 16, 16, None) == 2
+    assert att(None, None, None, 0, 128, 8, 2, 128, None, None, None) == 0  # B == 0: no-op
+    assert att(None, 16, 16, 1, 128, 8, 2, 128, 16, 16, None) == 1  # null Q
+    assert att(16, 16, 16, 1, 128, 8, 2, 128, 16, None, None) == 1  # null lse
+    assert att(24, 16, 16, 1, 128, 8, 2, 128, 16, 16, None) == 4    # misaligned Q
+    assert att(16, 16, 16, 1, 128, 8, 2, 128, 16, 18, None) == 4    # misaligned lse
+    bwd = lib.catq_attention_bwd
+    args = [16, 16, 16, 16, 16, 16, 1, 128, 8, 2, 128, 16, 16, 16, 16, None]
+    assert bwd(*args[:10], 96, *args[11:]) == 2
+    assert bwd(*args[:6], 0, *args[7:]) == 0                         # B == 0: no-op
+    assert bwd(*args[:11], None, *args[12:]) == 1                    # null delta
+    assert bwd(*args[:14], 40, None) == 4                            # misaligned dV
+    assert bwd(*args[:11], 18, *args[12:]) == 4                      # misaligned delta
+
+    rf = lib.catq_rmsnorm_fwd
+    assert rf(16, 7, None, 16, 4, 64, 1e-5, None, 16, 16, None) == 3      # unknown dtype
+    assert rf(16, C.BF16, None, 16, 4, 12, 1e-5, None, 16, 16, None) == 2  # H % 8 != 0
+    assert rf(16, C.BF16, None, 16, -1, 64, 1e-5, None, 16, 16, None) == 2
+    assert rf(16, C.BF16, None, 16, 4, 64, -1.0, None, 16, 16, None) == 1  # eps < 0
+    assert rf(16, C.BF16, None, 16, 4, 64, nan, None, 16, 16, None) == 1
+    assert rf(None, C.BF16, None, None, 0, 64, 1e-5, None, None, None, None) == 0  # T == 0
+    assert rf(16, C.BF16, None, 16, 4, 64, 1e-5, None, None, 16, None) == 1  # null Z
+    assert rf(16, C.BF16, 24, 16, 4, 64, 1e-5, None, 16, 16, None) == 4     # misaligned residual
+    assert rf(16, C.BF16, None, 18, 4, 64, 1e-5, None, 16, 16, None) == 4   # misaligned gamma
+    rb = lib.catq_rmsnorm_bwd
+    assert rb(16, 5, 16, 16, 16, None, None, 4, 64, 16, None) == 3
+    assert rb(16, C.F32, 16, 16, 16, None, None, 4, 0, 16, None) == 2      # H < 1
+    assert rb(None, C.F32, None, None, None, None, None, 0, 64, None, None) == 0
+    assert rb(16, C.F32, 16, 16, 16, None, None, 4, 64, None, None) == 1   # null dX
+    assert rb(16, C.F32, 16, 16, 16, 24, None, 4, 64, 16, None) == 4       # misaligned dZ2
+
+    rope = lib.catq_rope
+    assert rope(16, 4, 4, 2, 7, 1e4, 0, None) == 2         # odd d
+    assert rope(16, 4, 0, 2, 128, 1e4, 0, None) == 2       # S < 1
+    assert rope(16, 4, 4, 2, 128, 1.0, 0, None) == 1       # base must exceed 1
+    assert rope(16, 4, 4, 2, 128, inf, 0, None) == 1
+    assert rope(None, 0, 4, 2, 128, 1e4, 0, None) == 0     # T == 0
+    assert rope(None, 4, 4, 2, 128, 1e4, 0, None) == 1
+    assert rope(24, 4, 4, 2, 128, 1e4, 0, None) == 4
+
+    sf, sb = lib.catq_swiglu_fwd, lib.catq_swiglu_bwd
+    assert sf(16, 16, -1, 16, None) == 2
+    assert sf(None, None, 0, None, None) == 0
+    assert sf(16, 16, 64, None, None) == 1
+    assert sf(16, 24, 64, 16, None) == 4
+    assert sb(16, 16, 16, 64, 16, None, None) == 1          # null d_up
+    assert sb(16, 16, 24, 64, 16, 16, None) == 4            # misaligned dM
+
+    bl = lib.catq_block_output_loss
+    need = lib.catq_recon_loss_workspace_bytes(64)
+    assert bl(16, 16, 12, 16, 0, 16, None, None, 256, need, None) == 2      # count % 8 != 0
+    assert bl(16, 16, 64, 16, 3, 16, None, None, 256, need, None) == 1      # unknown reduction
+    assert bl(None, None, 0, None, 0, None, None, None, None, 0, None) == 0  # count == 0
+    assert bl(16, 16, 64, 16, 0, None, None, None, 256, need, None) == 1    # out_ref without loss_out
+    assert bl(16, 24, 64, 16, 0, 16, None, None, 256, need, None) == 4      # misaligned branch
+    assert bl(16, 16, 64, 16, 0, 16, None, None, 256, need - 8, None) == 9  # short workspace
+    assert bl(16, 16, 64, 16, 0, 16, None, None, None, need, None) == 9     # no workspace
+    assert bl(16, 16, 64, 16, 0, 16, None, None, 128, need, None) == 4      # workspace not 256-aligned
