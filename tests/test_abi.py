@@ -225,3 +225,146 @@ def test_block_call_validation(lib):
     assert bl(16, 16, 64, 16, 0, 16, None, None, 256, need - 8, None) == 9  # short workspace
     assert bl(16, 16, 64, 16, 0, 16, None, None, None, need, None) == 9     # no workspace
     assert bl(16, 16, 64, 16, 0, 16, None, None, 128, need, None) == 4      # workspace not 256-aligned
+
+
+def _grouped(E=4, N=64, K=256, g=128, dtype=C.BF16, W=16, stats=32, op_const=65536, recon=C.RECON_ALPHA_T):
+    """A stacked (MoE) layer struct with fake (never dereferenced) device addresses."""
+    return C.catq_grouped_layer(E, g, N, K, dtype, recon, W, stats, stats + 1024, stats + 2048, stats + 4096,
+                                stats + 8192, stats + 16384, op_const)
+
+
+def _offsets(*rows):
+    return (ctypes.c_int64 * len(rows))(*rows)
+
+
+def test_linear_variant_call_validation(lib):
+    """fwd_ex, fwd_loss, modulate_ternarize, act_quant_a8, the allocation-free backward and the
+    per-group reconstruction error: host-side rejections and no-ops (fake device addresses)."""
+    L, soft = _layer(), C.schedule(C.PHASE_SOFT, 30.0)
+    ex = lib.catq_soft_ternary_linear_fwd_ex
+    assert ex(ctypes.byref(L), soft, 16, 4, C.BF16, None, 16, 7, None) == 3     # Y dtype neither X's nor fp32
+    assert ex(ctypes.byref(L), soft, 16, 0, C.BF16, None, 16, C.F32, None) == 0  # M == 0
+    assert ex(ctypes.byref(L), soft, 16, 4, C.BF16, 18, 16, C.F32, None) == 4    # misaligned row scales
+    assert ex(ctypes.byref(L), soft, 16, 4, C.BF16, None, None, C.F32, None) == 1
+    fl = lib.catq_soft_ternary_linear_fwd_loss
+    ok = [ctypes.byref(L), soft, 16, 4, C.BF16, None, 16, C.BF16, 0, 16, 16, None, 256, 1 << 20, None]
+    assert fl(*ok[:7], 5, *ok[8:]) == 3                       # reference dtype
+    assert fl(*ok[:8], 2, *ok[9:]) == 1                       # unknown reduction
+    assert fl(*ok[:3], 0, *ok[4:]) == 2                       # M < 1
+    assert fl(*ok[:10], None, *ok[11:]) == 1                  # null dY
+    assert fl(*ok[:11], 24, *ok[12:]) == 4                    # misaligned Y
+    assert fl(*ok[:12], None, *ok[13:]) == 9                  # no workspace
+    mt = lib.catq_modulate_ternarize
+    assert mt(ctypes.byref(_layer(stats=32)), C.schedule(C.PHASE_SOFT, -1.0), 16, None, None, None) == 1
+    assert mt(ctypes.byref(L), soft, 24, None, None, None) == 4                 # misaligned Wq
+    assert mt(ctypes.byref(L), soft, None, 40, None, None) == 4                 # misaligned codes
+    assert mt(ctypes.byref(L), soft, None, None, None, None) == 0               # nothing asked for
+    aq = lib.catq_act_quant_a8
+    assert aq(16, 4, 256, 5, 16, 16, None, None) == 3
+    assert aq(16, 4, 0, C.BF16, 16, 16, None, None) == 2      # K < 1
+    assert aq(16, 4, 12, C.BF16, 16, 16, None, None) == 2     # bf16 rows of 16 bytes
+    assert aq(16, 4, 6, C.F32, 16, 16, None, None) == 2       # fp32 rows of 16 bytes
+    assert aq(None, 0, 256, C.BF16, None, None, None, None) == 0
+    assert aq(16, 4, 256, C.BF16, 16, None, None, None) == 1  # null scales
+    assert aq(16, 4, 256, C.BF16, 16, 18, None, None) == 4    # misaligned scales
+    assert aq(16, 4, 256, C.BF16, 16, 16, 24, None) == 4      # misaligned dequantized copy
+    na = lib.catq_soft_ternary_linear_bwd_noalloc
+    assert lib.catq_bwd_noalloc_max_scratch_bytes() == 16 << 20
+    assert na(ctypes.byref(_layer(W=0)), soft, 16, 16, 4, C.BF16, None, 32, 32, 32, None) == 1
+    big = _layer(N=16384, K=16384, dtype=C.F32)                # 50 MB of partial sums
+    assert na(ctypes.byref(big), soft, 16, 16, 4, C.F32, None, 32, 32, 32, None) == 9
+    re = lib.catq_group_recon_error
+    assert re(ctypes.byref(L), None, None) == 1
+    assert re(ctypes.byref(L), 18, None) == 4
+    assert re(ctypes.byref(_layer(dtype=9)), 16, None) == 3
+
+
+def test_grouped_call_validation(lib):
+    """The stacked-expert calls: offsets start at 0 and never decrease, dtype and workspace
+    rules, empty routing as a no-op, and the grouped partial-sum size."""
+    G, soft = _grouped(), C.schedule(C.PHASE_SOFT, 30.0)
+    off = _offsets(0, 5, 5, 40, 64)
+    fwd = lib.catq_grouped_soft_ternary_linear_fwd
+    assert fwd(None, soft, 16, off, C.BF16, 16, None) == 1
+    assert fwd(ctypes.byref(_grouped(E=0)), soft, 16, off, C.BF16, 16, None) == 1
+    assert fwd(ctypes.byref(G), soft, 16, _offsets(1, 5, 5, 40, 64), C.BF16, 16, None) == 2  # off[0] != 0
+    assert fwd(ctypes.byref(G), soft, 16, _offsets(0, 5, 4, 40, 64), C.BF16, 16, None) == 2  # decreasing
+    assert fwd(ctypes.byref(G), soft, 16, _offsets(0, 0, 0, 0, 0), C.BF16, 16, None) == 0    # nothing routed
+    assert fwd(ctypes.byref(G), soft, None, off, C.BF16, 16, None) == 1
+    assert fwd(ctypes.byref(G), soft, 24, off, C.BF16, 16, None) == 4
+    assert fwd(ctypes.byref(_grouped(op_const=0)), soft, 16, off, C.BF16, 16, None) == 1  # operand constants
+    fl = lib.catq_grouped_soft_ternary_linear_fwd_loss
+    ok = [ctypes.byref(G), soft, 16, off, C.BF16, 16, 0, 16, 16, None, 256, 1 << 20, None]
+    assert fl(*ok[:4], C.F32, *ok[5:]) == 3
+    assert fl(*ok[:6], 2, *ok[7:]) == 1
+    assert fl(ok[0], soft, 16, _offsets(0, 0, 0, 0, 0), *ok[4:]) == 2   # loss over no rows
+    assert fl(*ok[:8], None, *ok[9:]) == 1                               # null dY
+    assert fl(*ok[:9], 24, *ok[10:]) == 4                                # misaligned Y
+    assert fl(*ok[:10], None, *ok[11:]) == 9
+    assert lib.catq_grouped_fwd_loss_workspace_bytes(ctypes.byref(G), _offsets(2, 5, 5, 40, 64)) == 0
+    need = lib.catq_grouped_bwd_workspace_bytes(ctypes.byref(G), off)
+    assert need == 4 * 3 * 64 * (256 // 128) * 4                         # [E][3][N][K/128] fp32
+    assert lib.catq_grouped_bwd_workspace_bytes(None, off) == 0
+    bwd = lib.catq_grouped_soft_ternary_linear_bwd
+    ok = [ctypes.byref(G), soft, 16, 16, off, C.BF16, None, 32, 32, 32, 256, need, None]
+    assert bwd(*ok[:8], None, *ok[9:]) == 1                              # all three gradients or none
+    assert bwd(*ok[:2], None, *ok[3:]) == 1                              # null X
+    assert bwd(*ok[:3], 24, *ok[4:]) == 4                                # misaligned dY
+    assert bwd(*ok[:10], None, *ok[11:]) == 9
+    assert bwd(*ok[:11], need - 4, None) == 9
+    assert bwd(*ok[:10], 128, *ok[11:]) == 4                             # workspace not 256-aligned
+
+
+def test_batched_and_staged_inference_validation(lib):
+    """Layer lists of the batched and staged decode calls: limits, shared g and mu presence,
+    the stage map, and the synchronisation words."""
+    n_max, s_max = lib.catq_ternary_infer_max_layers(), lib.catq_ternary_infer_max_stages()
+    assert 1 <= n_max <= 64 and s_max >= 1
+    assert lib.catq_ternary_infer_sync_bytes() == 4 * (s_max + 1)
+
+    def layers(n=2, mu=None, K=256, X=16, codes=16):
+        arr = (C.catq_infer_layer * n)()
+        for i in range(n):
+            arr[i] = C.catq_infer_layer(codes, 32, mu, 64, K, X, 64)
+        return arr
+    bt = lib.catq_ternary_infer_batched
+    assert bt(None, 2, 128, 1, C.BF16, None) == 1
+    assert bt(layers(), 0, 128, 1, C.BF16, None) == 1
+    assert bt(layers(n_max + 1), n_max + 1, 128, 1, C.BF16, None) == 1   # more layers than one launch takes
+    assert bt(layers(), 2, 128, 1, C.F32, None) == 3
+    assert bt(layers(), 2, 96, 1, C.BF16, None) == 2                     # g % 64 != 0
+    assert bt(layers(K=320), 2, 128, 1, C.BF16, None) == 2               # g does not divide K
+    mixed = layers()
+    mixed[1].mu = 64
+    assert bt(mixed, 2, 128, 1, C.BF16, None) == 1                       # mu on some layers only
+    assert bt(layers(X=None), 2, 128, 1, C.BF16, None) == 1
+    assert bt(layers(X=None), 2, 128, 0, C.BF16, None) == 0              # B == 0: inputs not needed
+    assert bt(layers(codes=24), 2, 128, 1, C.BF16, None) == 4
+    st = lib.catq_ternary_infer_staged
+    stages = lambda *s: (ctypes.c_int32 * len(s))(*s)
+    assert st(layers(3), 3, None, 128, 1, C.BF16, 64, None) == 1
+    assert st(layers(3), 3, stages(0, 0, 1), 128, 1, C.BF16, None, None) == 1   # no sync words
+    assert st(layers(3), 3, stages(1, 1, 2), 128, 1, C.BF16, 64, None) == 1    # first stage not 0
+    assert st(layers(3), 3, stages(0, 2, 2), 128, 1, C.BF16, 64, None) == 1    # a stage skipped
+    assert st(layers(3), 3, stages(0, 1, 0), 128, 1, C.BF16, 64, None) == 1    # stages go back
+    assert st(layers(3), 3, stages(0, 0, 1), 128, 1, C.BF16, 66, None) == 4    # misaligned sync words
+    assert st(layers(3), 3, stages(0, 0, 1), 128, 0, C.BF16, 64, None) == 0    # B == 0
+    # stages rise by at most one per layer from 0, so every accepted stage map fits the limit
+    assert s_max >= n_max
+
+
+def test_direct_update_validation(lib):
+    """DL's own AdamW step: shape, hyper-parameter and alignment rules."""
+    du = lib.catq_direct_adamw_step
+    hp = C.adamw()
+    args = [8, 16, 16, 16, 16, 16, ctypes.byref(hp), 1, 1e-3, None]
+    assert du(-1, *args[1:]) == 2
+    assert du(0, None, None, None, None, None, None, 1, 1e-3, None) == 0
+    assert du(*args[:6], None, *args[7:]) == 1                 # no hyper-parameters
+    assert du(*args[:7], 0, *args[8:]) == 1                    # t starts at 1
+    assert du(*args[:8], float("nan"), None) == 1
+    assert du(*args[:8], -1e-3, None) == 1
+    for bad in (C.adamw(beta1=1.0), C.adamw(beta2=-0.1), C.adamw(eps=0.0), C.adamw(weight_decay=-1.0),
+                C.adamw(margin=0.5)):
+        assert du(*args[:6], ctypes.byref(bad), *args[7:]) == 1
+    assert du(8, 16, 16, 16, 18, 16, ctypes.byref(hp), 1, 1e-3, None) == 4
